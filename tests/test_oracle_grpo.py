@@ -1,0 +1,144 @@
+"""Pins of the oracle's GRPO signals, aggregation, routing and reductions: scipy's Gaussian
+log-density, numpy's std, central finite differences of Eq. grpo_loss, closed forms of
+Eq. alpha / Eq. s_base_corr, and the routing values printed in the paper."""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+from scipy import stats
+
+import synth
+from oracle import grpo
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def test_logprob_is_the_isotropic_gaussian_density():
+    rng = np.random.Generator(np.random.PCG64(0))
+    D = 37
+    z, zn, v = rng.standard_normal((3, D))
+    t0, t1, sig = 0.8, 0.7375, 0.31
+    mu = z + v * (t1 - t0)
+    ref = stats.norm.logpdf(zn, loc=mu, scale=sig).sum()
+    assert grpo.step_logprob(zn, z, v, t0, t1, sig) == pytest.approx(ref, rel=1e-13)
+
+
+def test_advantages_match_numpy_and_clamp_bound():
+    r = np.array([0.3, -1.2, 2.5, 0.0, 0.7])
+    A = grpo.advantages(r)
+    np.testing.assert_allclose(A, (r - r.mean()) / (np.std(r, ddof=1) + 1e-8), rtol=1e-14)
+    # unbiased std bounds |A| by (G-1)/sqrt(G); with one outlier it is attained
+    G = 8
+    r = np.zeros(G); r[0] = 1.0
+    assert abs(grpo.advantages(r)[0]) == pytest.approx((G - 1) / math.sqrt(G), rel=1e-7)
+    assert np.all(grpo.advantages(np.array([1.0, 100.0, 2.0]), adv_clip=0.5) <= 0.5)
+    np.testing.assert_array_equal(grpo.advantages(np.full(4, 3.0)), 0.0)
+
+
+def _signals_case(seed, D=6, W=3, G=3, rho_shift=None, eps=0.1):
+    rng = np.random.Generator(np.random.PCG64(seed))
+    t = synth.time_grid(W, shift=3.0)
+    sig = synth.sigma_schedule(t, 0.7)
+    z = rng.standard_normal((G, W + 1, D))
+    v = rng.standard_normal((G, W, D))
+    lp = np.array([[grpo.step_logprob(z[i, j + 1], z[i, j], v[i, j], t[j], t[j + 1], sig[j])
+                    for j in range(W)] for i in range(G)])
+    shift = rng.uniform(-3 * eps, 3 * eps, size=(G, W)) if rho_shift is None else rho_shift
+    A = np.array([1.3, -0.7, 0.4])[:G]
+    return v, z, t, sig, lp + shift, A
+
+
+@pytest.mark.parametrize("seed", [1, 2, 3])
+def test_signals_are_the_gradient_of_the_window_loss(seed):
+    """s_ij equals the central difference of scale * sum_j L_ij (Eq. grpo_loss) in v_ij."""
+    eps, scale = 0.1, 0.37
+    v, z, t, sig, lpo, A = _signals_case(seed, eps=eps)
+    s, _, ratio, clipped = grpo.step_signals(v, z, t, sig, lpo, A, eps, scale)
+    h = 1e-6
+    G, W, D = v.shape
+    for i in range(G):
+        for j in range(W):
+            if abs(abs(ratio[i, j] - 1.0) - eps) < 1e-4:
+                continue   # at the kink the loss is not differentiable
+            for k in range(D):
+                vp = v[i].copy(); vp[j, k] += h
+                vm = v[i].copy(); vm[j, k] -= h
+                fd = (grpo.window_loss(vp, z[i], t, sig, lpo[i], A[i], eps, scale)
+                      - grpo.window_loss(vm, z[i], t, sig, lpo[i], A[i], eps, scale)) / (2 * h)
+                assert fd == pytest.approx(s[i, j, k], rel=1e-6, abs=1e-9)
+    assert clipped.any() and not clipped.all()
+
+
+def test_clip_follows_the_max_of_the_surrogate():
+    """Zero gradient exactly when the clipped branch is strictly larger: (A>0, rho>1+eps)
+    or (A<0, rho<1-eps); the other two out-of-range cases keep their gradient."""
+    eps = 0.1
+    W, G = 1, 2
+    v, z, t, sig, lp, _ = _signals_case(4, W=W, G=G, rho_shift=np.zeros((G, W)), eps=eps)
+    for A, log_rho, expect_clipped in [(1.0, 0.2, 1), (1.0, -0.2, 0), (-1.0, -0.2, 1),
+                                        (-1.0, 0.2, 0), (1.0, 0.05, 0), (-1.0, -0.05, 0)]:
+        lpo = lp - log_rho
+        s, _, ratio, clipped = grpo.step_signals(v, z, t, sig, lpo, np.array([A, A]), eps, 1.0)
+        np.testing.assert_allclose(ratio, math.exp(log_rho), rtol=1e-12)
+        assert clipped[0, 0] == expect_clipped, (A, log_rho)
+        assert (np.abs(s[0]).sum() == 0) == bool(expect_clipped)
+
+
+def test_zero_advantage_and_unit_ratio():
+    v, z, t, sig, lp, _ = _signals_case(5, rho_shift=np.zeros((3, 3)))
+    s, _, ratio, clipped = grpo.step_signals(v, z, t, sig, lp, np.zeros(3), 0.1, 1.0)
+    np.testing.assert_array_equal(s, 0.0)
+    np.testing.assert_allclose(ratio, 1.0, rtol=1e-12)
+    assert not clipped.any()
+
+
+def test_alpha_closed_forms():
+    t = synth.time_grid(16, 1.0)[4:8]
+    np.testing.assert_allclose(grpo.alpha_weights(t), np.arange(4) / 3, atol=1e-15)
+    ts = synth.time_grid(16, 3.0)[4:8]
+    al = grpo.alpha_weights(ts)
+    assert al[0] == 0.0 and al[-1] == 1.0
+    assert np.all(np.diff(al) > 0)
+    # shifted grid: alpha is the affine coordinate of t, not j/(W-1)
+    assert abs(al[1] - 1 / 3) > 1e-3
+    np.testing.assert_allclose(ts[0] + al * (ts[-1] - ts[0]), ts, atol=1e-15)
+
+
+def test_aggregation_partition_of_unity_and_endpoints():
+    rng = np.random.Generator(np.random.PCG64(8))
+    s = rng.standard_normal((3, 4, 10))
+    t = synth.time_grid(16, 3.0)[8:12]
+    cot = grpo.aggregate(s, t)
+    np.testing.assert_allclose(cot[:3] + cot[3:], s.sum(1), atol=1e-14)
+    al = grpo.alpha_weights(t)
+    np.testing.assert_allclose(cot[3:], np.einsum("j,gjd->gd", al, s), atol=1e-14)
+    # s_0 only in the base row, s_{W-1} only in the correction row
+    e = np.zeros_like(s); e[:, 0] = s[:, 0]
+    np.testing.assert_array_equal(grpo.aggregate(e, t)[3:], 0.0)
+    e = np.zeros_like(s); e[:, 3] = s[:, 3]
+    np.testing.assert_array_equal(grpo.aggregate(e, t)[:3], 0.0)
+    # W = 2: the cotangents are s_0 and s_1 themselves (JAGG is exact)
+    np.testing.assert_array_equal(grpo.aggregate(s[:, :2], t[:2]), np.concatenate([s[:, 0], s[:, 1]]))
+
+
+def test_routing_reproduces_the_papers_table():
+    with open(os.path.join(GOLDEN, "routing_table.json")) as f:
+        g = json.load(f)
+    for model, row in g["calibration"].items():
+        route, frac = grpo.route_calibrate(row["cos"], g["tau"])
+        assert route.tolist() == row["route"], model
+        assert frac == pytest.approx(row["derived_frac"])
+    for case in g["schedule"]:
+        assert grpo.route_schedule(case["n_windows"], case["jagg_frac"]).tolist() == case["route"]
+
+
+def test_grad_stats_against_numpy():
+    rng = np.random.Generator(np.random.PCG64(2))
+    a, b = rng.standard_normal((2, 1000))
+    ab, aa, bb, cos, rho = grpo.grad_stats(a, b)
+    assert ab == pytest.approx(np.dot(a, b)) and aa == pytest.approx(np.dot(a, a))
+    assert cos == pytest.approx(np.dot(a, b) / np.linalg.norm(a) / np.linalg.norm(b))
+    assert rho == pytest.approx(np.linalg.norm(a) / np.linalg.norm(b))
+    assert grpo.grad_stats(a, 2 * a)[3] == pytest.approx(1.0)
