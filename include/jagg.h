@@ -1,0 +1,199 @@
+/*
+ * jagg.h -- C ABI of the JAGG backward library for GB300 (sm_103a).
+ *
+ * JAGG (Jacobian-Aggregated Group Gradient, arxiv 2607.17572) replaces the W per-step
+ * DiT backward passes of one window of W sampling steps of diffusion GRPO with one
+ * joint vector-Jacobian product at the two window endpoints (Sec. 3.3, Algorithm 1).
+ * This library is that update-stage hot path on one GPU:
+ *
+ *   dit_forward_save   Phase 1: v = DiT(z, t, txt), keeping what Phase 4 needs
+ *   grpo_step_signals  Phase 2: s_j = dL_j/dv_j through Eq. logprob and Eq. grpo_loss
+ *   jagg_aggregate     Phase 3: Eq. alpha and Eq. s_base_corr
+ *   jagg_route         jagg_frac routing (Sec. 3.3 and the gradient-quality appendix)
+ *   dit_joint_vjp      Phase 4: grad += sum_rows J(z_row, t_row)^T cot_row
+ *   grad_reduce        gradient accumulation and the cosine / norm-ratio reductions
+ *
+ * Conventions shared by every entry point:
+ *   - Memory is owned by the caller.  Pointers documented "device" must be device
+ *     memory of the current CUDA device; "host" pointers are ordinary host memory.
+ *     Device buffers must be 16-byte aligned and contiguous, row-major.
+ *   - Calls are asynchronous on `stream` unless stated otherwise; results are valid
+ *     once the stream has reached them.
+ *   - The return value is a status: JAGG_OK (0) or a negative JAGG_ERR_* code.  Argument
+ *     errors are detected on the host before anything is launched; jagg_last_error()
+ *     returns a description of the most recent error of the calling thread.
+ *   - No entry point allocates device memory except jagg_model_create (a small table).
+ *     Scratch space is a caller-provided workspace sized by the *_workspace_bytes calls.
+ *   - Waits inside kernels are bounded; a wait that gives up sets a device status bit
+ *     (read with jagg_device_status) instead of hanging or trapping.
+ *
+ * bf16 is IEEE bfloat16 stored as uint16; f32/f64 are IEEE float/double.
+ */
+#ifndef JAGG_H_
+#define JAGG_H_
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ----------------------------------------------------------------- status codes */
+#define JAGG_OK 0
+#define JAGG_ERR_ARG (-1)          /* invalid pointer, size, alignment or config     */
+#define JAGG_ERR_UNSUPPORTED (-2)  /* valid request this build does not implement     */
+#define JAGG_ERR_CUDA (-3)         /* a CUDA runtime/driver call failed               */
+#define JAGG_ERR_TIMEOUT (-4)      /* a bounded device wait gave up                   */
+#define JAGG_ERR_WORKSPACE (-5)    /* workspace or saved arena smaller than required  */
+
+#define JAGG_DTYPE_F32 0
+#define JAGG_DTYPE_BF16 1
+
+#define JAGG_ARCH_DIT 0    /* single-stream adaLN DiT blocks                           */
+#define JAGG_ARCH_MMDIT 1  /* double-stream MMDiT blocks followed by Flux-style single  */
+
+/* Device status bits (jagg_device_status). */
+#define JAGG_DEV_STATUS_TIMEOUT 1u
+#define JAGG_DEV_STATUS_BADARG 2u
+
+/* Text of the most recent error of the calling thread ("" if none). */
+const char* jagg_last_error(void);
+
+/* Reads the device status word (synchronises the device); clears it when `clear` != 0. */
+int jagg_device_status(unsigned* status_out, int clear);
+
+/* ------------------------------------------------------------------ backbone
+ * The velocity network v_theta(z, t, txt).  The paper trains Flux and Qwen-Image
+ * (Sec. 4) without describing them; the library implements the pinned DiT / MMDiT of
+ * the project's design notes: patch embedding, text projection, sinusoidal t-embedding
+ * MLP, adaLN-modulated blocks with tanh-GELU MLPs and joint [txt; img] softmax
+ * attention (per-head RMSNorm and 2D RoPE in the MMDiT), and a modulated final layer.
+ */
+typedef struct jagg_config {
+  int32_t arch;          /* JAGG_ARCH_DIT or JAGG_ARCH_MMDIT                          */
+  int32_t dtype;         /* storage/compute type of weights and activations           */
+  int32_t hidden;        /* d (multiple of 64)                                        */
+  int32_t heads;         /* d / heads = head dim: 16 (f32 only), 64 or 128             */
+  int32_t mlp;           /* MLP width (multiple of 64)                                */
+  int32_t depth;         /* DiT blocks (DIT) or Flux-style single blocks (MMDIT)      */
+  int32_t depth_double;  /* double-stream blocks (MMDIT), 0 for DIT                   */
+  int32_t in_channels;   /* latent channels C                                         */
+  int32_t latent_h;      /* latent height H (multiple of patch)                       */
+  int32_t latent_w;      /* latent width W (multiple of patch)                        */
+  int32_t patch;         /* patch size p                                              */
+  int32_t txt_len;       /* text tokens per sequence                                  */
+  int32_t txt_dim;       /* text embedding width (multiple of 8)                      */
+  int32_t freq_dim;      /* sinusoidal t-embedding width (256)                        */
+} jagg_config;
+
+typedef struct jagg_model* jagg_model_t;
+
+/* Number of scalar parameters, and of parameter tensors, of a configuration. */
+int64_t jagg_param_count(const jagg_config* cfg);
+int jagg_param_tensor_count(const jagg_config* cfg);
+
+/* Describes parameter tensor `index` (0 <= index < jagg_param_tensor_count): its name
+ * (e.g. "blocks.3.qkv.w", NUL-terminated into name[name_cap]), its element offset in
+ * the flat parameter buffer and its shape (rows x cols; cols = 1 for vectors).  Matrices
+ * are stored [out, in] row-major.  The same offsets index the fp32 gradient buffer. */
+int jagg_param_info(const jagg_config* cfg, int index, char* name, size_t name_cap,
+                    int64_t* offset, int64_t* rows, int64_t* cols);
+
+/* Creates a model over caller-owned device weights (jagg_param_count elements of
+ * cfg->dtype laid out as jagg_param_info describes).  The weights must stay valid and
+ * unchanged while the model is used.  Synchronous; allocates a small host table. */
+int jagg_model_create(const jagg_config* cfg, const void* weights, jagg_model_t* model_out);
+int jagg_model_destroy(jagg_model_t model);
+
+/* Bytes of the saved-activation arena for a forward over B sequences, and of the
+ * workspace that dit_forward_save / dit_joint_vjp need for B sequences. */
+int64_t jagg_saved_bytes(jagg_model_t model, int B);
+int64_t jagg_workspace_bytes(jagg_model_t model, int B);
+
+/* Phase 1 (Sec. 3.3, Algorithm 1): v_out = DiT(z, t, txt) for B sequences.
+ *   z      device [B, C, H, W] cfg dtype       network input latents
+ *   t      device [B] f32                      network-input times
+ *   txt    device [B, txt_len, txt_dim] dtype  text embeddings
+ *   v_out  device [B, C, H, W] cfg dtype       predicted velocities
+ *   saved  device arena of >= jagg_saved_bytes(B) bytes, or NULL for a forward that
+ *          keeps nothing (the middle steps of a window run this way)
+ *   ws     device workspace of >= jagg_workspace_bytes(B) bytes                        */
+int dit_forward_save(jagg_model_t model, const void* z, const float* t, const void* txt,
+                     int B, void* v_out, void* saved, size_t saved_bytes, void* ws,
+                     size_t ws_bytes, cudaStream_t stream);
+
+/* Phase 4 (Sec. 3.3 "Joint backward", Algorithm 1): grad += sum_b J(z_b, t_b)^T cot_b,
+ * the parameter VJP of every row of a saved forward, in one pass.  For a JAGG window the
+ * rows are [z_0 of each sample; z_{W-1} of each sample] and cot = [s_base; s_corr]
+ * (Eq. s_base_corr); for the exact per-step path they are the W*G step inputs and cot
+ * holds each s_j.  No gradient flows to z or txt (they are fixed samples, Phase 2).
+ *   saved  the arena of a dit_forward_save over the same B rows
+ *   cot    device [B, C, H, W] f32 cotangents (rounded to cfg dtype inside)
+ *   grad   device f32 [jagg_param_count], accumulated (+=), same layout as the weights */
+int dit_joint_vjp(jagg_model_t model, const void* saved, size_t saved_bytes, int B,
+                  const float* cot, float* grad, void* ws, size_t ws_bytes,
+                  cudaStream_t stream);
+
+/* ------------------------------------------------------------------ GRPO signals
+ * Phase 2 (Sec. 3.3): for sample i and step j of a window,
+ *   r_ij   = z_{i,j+1} - z_{i,j} - v_ij (t_{j+1} - t_j)
+ *   logp   = -||r_ij||^2 / (2 sigma_j^2) - D log(sqrt(2 pi) sigma_j)        (Eq. logprob)
+ *   rho    = exp(logp - logp_old_ij)
+ *   A_i    = clamp((r_i - mean) / (std + adv_eps), +-adv_clip), unbiased std (Eq. advantage)
+ *   s_ij   = scale * d max(-A rho, -A clip(rho, 1-eps, 1+eps)) / d v_ij          (Eq. grpo_loss)
+ *          = scale * (-A_i) rho r_ij (t_{j+1}-t_j) / sigma_j^2, or 0 when the clipped branch
+ *            is strictly larger (A>0 and rho>1+eps, or A<0 and rho<1-eps).
+ * The squared norms are accumulated in f64 and logp / rho are f64.
+ *   v_hat     device [G, W, D] (v_dtype)   model outputs of the window's steps
+ *   z         device [G, W+1, D] f32       trajectory states z_0 .. z_W of the window
+ *   t         device [W+1] f64             network-input times t_0 .. t_W
+ *   sigma     device [W] f64               per-step noise scale
+ *   logp_old  device [G, W] f64            rollout log-probs
+ *   rewards   device [G] f32
+ *   s_out     device [G, W, D] f32 or NULL
+ *   cot_out   device [2G, D] f32 or NULL: if given, the aggregated JAGG cotangents
+ *             (jagg_aggregate over t_0..t_{W-1}) are written in the same pass; needs W >= 2
+ *   logp_new, ratio device [G, W] f64; clipped device [G, W] u8; adv_out device [G] f64
+ *   ws        device workspace of >= jagg_signals_workspace_bytes(G, W, D) bytes       */
+int64_t jagg_signals_workspace_bytes(int G, int W, int64_t D);
+int grpo_step_signals(const void* v_hat, int v_dtype, const float* z, const double* t,
+                      const double* sigma, const double* logp_old, const float* rewards,
+                      int G, int W, int64_t D, double clip_eps, double adv_clip,
+                      double adv_eps, double scale, float* s_out, float* cot_out,
+                      double* logp_new, double* ratio, uint8_t* clipped, double* adv_out,
+                      void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* Phase 3 (Eq. alpha, Eq. s_base_corr): alpha_j = (t_0 - t_j) / (t_0 - t_{W-1}),
+ *   cot[i]     = sum_j (1 - alpha_j) s[i, j]   (s_base, endpoint j = 0)
+ *   cot[G + i] = sum_j alpha_j s[i, j]         (s_corr, endpoint j = W-1)
+ *   s      device [G, W, D] f32;  t_window device [W] f64 network-input times
+ *   cot    device [2G, D] f32.  Requires W >= 2 and t_0 != t_{W-1} (checked on device:
+ *   a zero denominator sets JAGG_DEV_STATUS_BADARG and writes zeros).                */
+int jagg_aggregate(const float* s, const double* t_window, int G, int W, int64_t D,
+                   float* cot, cudaStream_t stream);
+
+/* jagg_frac routing (Sec. 3.3 "High-noise vs. low-noise scheduling"; rule of the
+ * gradient-quality appendix).  Host-only, synchronous.
+ *   cos == NULL: schedule mode, route[w] = (w < floor(jagg_frac * n_windows + 1e-9)).
+ *   cos != NULL: calibration mode, route[w] = (cos[w] >= tau) and *derived_frac (if not
+ *   NULL) = longest qualifying prefix / n_windows.  jagg_frac is ignored.
+ *   route  host [n_windows] u8: 1 = JAGG window, 0 = exact per-step window.           */
+int jagg_route(int n_windows, double jagg_frac, const double* cos, double tau,
+               uint8_t* route, double* derived_frac);
+
+/* Gradient reductions (gradient-quality appendix: cos(g_JAGG, g_exact) and
+ * rho = ||g_JAGG|| / ||g_exact||; accumulation of window gradients).
+ *   acc != NULL: acc[k] += alpha * a[k]
+ *   out3 != NULL: out3 = { <a,b>, <a,a>, <b,b> } in f64 (b may be NULL: then <a,a> thrice)
+ *   a, b, acc device f32 [P]; out3 device f64 [3]
+ *   ws device workspace of >= jagg_grad_reduce_workspace_bytes(P) bytes (when out3)   */
+int64_t jagg_grad_reduce_workspace_bytes(int64_t P);
+int grad_reduce(const float* a, const float* b, int64_t P, float alpha, float* acc,
+                double* out3, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* JAGG_H_ */

@@ -1,0 +1,68 @@
+/*
+ * jagg_testing.h -- entry points that expose single kernels of the library to its tests.
+ *
+ * They are not part of the JAGG path; they let the tests check the dense-product and
+ * attention kernels in isolation against a plain reference before the whole backbone is
+ * compared with the oracle.  Same conventions as jagg.h (caller-owned device memory,
+ * asynchronous on `stream`, status return).
+ */
+#ifndef JAGG_TESTING_H_
+#define JAGG_TESTING_H_
+
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* D[m, n] = sum_k A[m, k] B[n, k] with the library's epilogues:
+ *   epi 0 store:  C = D (+ bias[n])
+ *   epi 1 gelu:   C = u = D + bias, C2 = gelu_tanh(u)
+ *   epi 2 gate:   C = y = D + bias, C2 = aux + gate[(m / rows_per_seq) * gate_stride + n] * y
+ *   epi 3 dgelu:  C = D * gelu_tanh'(aux)
+ *   epi 4 accum:  C += D (f32 C; split_k > 0 forces the number of K splits)
+ * A is K-major (A[m*lda + k]) or MN-major (A[k*lda + m]); B is K-major (B[n*ldb + k]) or
+ * MN-major (B[k*ldb + n]).  a_dtype/b_dtype/c_dtype/bias_dtype are JAGG_DTYPE_*; C2 and aux
+ * follow c_dtype for gelu/dgelu and are f32 for gate.  force_simt selects the SIMT kernel
+ * instead of the tcgen05 one (bf16 operands only take the tensor-core path). */
+typedef struct jagg_gemm_desc {
+  int32_t M, N, K;
+  const void* A;
+  int64_t lda;
+  int32_t a_mn, a_dtype;
+  const void* B;
+  int64_t ldb;
+  int32_t b_mn, b_dtype;
+  int32_t epi;
+  const void* bias;
+  int32_t bias_dtype;
+  void* C;
+  int64_t ldc;
+  int32_t c_dtype;
+  void* C2;
+  int64_t ldc2;
+  const void* aux;
+  int64_t ld_aux;
+  const float* gate;
+  int64_t gate_stride;
+  int32_t rows_per_seq;
+  int32_t split_k;
+  int32_t force_simt;
+} jagg_gemm_desc;
+
+int jagg_test_gemm(const jagg_gemm_desc* desc, cudaStream_t stream);
+
+/* Joint softmax attention over qkv [B*N, 3*heads*dh] (q, k, v at column offsets 0, d, 2d;
+ * dtype JAGG_DTYPE_*): o [B*N, d], lse [B, heads, N] f32.  The backward takes dO [B*N, d]
+ * and writes dqkv [B*N, 3d] using scratch of jagg_test_attention_scratch_bytes bytes. */
+int jagg_test_attention_fwd(const void* qkv, int B, int N, int heads, int dh, int dtype, void* o, float* lse,
+                            cudaStream_t stream);
+int64_t jagg_test_attention_scratch_bytes(int B, int N, int heads, int dh);
+int jagg_test_attention_bwd(const void* qkv, const void* o, const float* lse, const void* dO, int B, int N,
+                            int heads, int dh, int dtype, void* dqkv, void* scratch, cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* JAGG_TESTING_H_ */

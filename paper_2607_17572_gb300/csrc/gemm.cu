@@ -1,0 +1,623 @@
+// Dense products of the backbone on sm_103a.
+//
+// bf16 x bf16 -> f32: a persistent, warp-specialised tcgen05 kernel.  One CTA per SM;
+// warp 0 issues TMA loads of 128-byte-swizzled tiles into a multi-stage shared-memory
+// ring, warp 1 (one elected thread) issues tcgen05.mma into a double-buffered TMEM
+// accumulator, warps 2-5 drain TMEM with tcgen05.ld and run the fused epilogue while
+// the next tile's MMAs proceed.  Both operands may be K-major or MN-major, so the
+// forward (X W^T), input-gradient (dY W) and weight-gradient (dY^T X) products all read
+// their operands in place, without transposes.
+//
+// f32 operands (the fp32 configuration and the per-sequence modulation / t-embedding
+// products with B rows): a tiled SIMT kernel with the same epilogue.
+#include <cuda.h>
+#include <mutex>
+
+#include "gemm.cuh"
+#include "ptx.cuh"
+
+namespace jagg {
+
+int unit_status_gemm(unsigned* v, int clear) { return read_unit_status(v, clear); }
+
+// ------------------------------------------------------------------ epilogue
+struct EpiParams {
+  int M, N, epi;
+  const void* bias;
+  int bias_bf16;
+  void* C;
+  int64_t ldc;
+  int c_bf16;
+  void* C2;
+  int64_t ldc2;
+  const void* aux;
+  int64_t ld_aux;
+  const float* gate;
+  int64_t gate_stride;
+  int rows_per_seq;
+  int remap_rows, remap_offset;
+  int64_t remap_stride;
+  int vec_ok;  // 8-wide vector accesses are aligned
+};
+
+__device__ __forceinline__ float ldv(const void* p, int64_t i, int is_bf16) {
+  return is_bf16 ? __bfloat162float(static_cast<const bf16*>(p)[i]) : static_cast<const float*>(p)[i];
+}
+__device__ __forceinline__ void stv(void* p, int64_t i, int is_bf16, float v) {
+  if (is_bf16)
+    static_cast<bf16*>(p)[i] = __float2bfloat16_rn(v);
+  else
+    static_cast<float*>(p)[i] = v;
+}
+
+__device__ __forceinline__ int64_t epi_crow(const EpiParams& e, int m) {
+  return e.remap_rows ? (int64_t)(m / e.remap_rows) * e.remap_stride + e.remap_offset + m % e.remap_rows
+                      : (int64_t)m;
+}
+
+// One element (m < M, n < N).
+__device__ __forceinline__ void epi_apply1(const EpiParams& e, int m, int n, float acc) {
+  const int64_t cr = epi_crow(e, m);
+  switch (e.epi) {
+    case EPI_STORE: {
+      float v = acc + (e.bias ? ldv(e.bias, n, e.bias_bf16) : 0.f);
+      stv(e.C, cr * e.ldc + n, e.c_bf16, v);
+    } break;
+    case EPI_GELU: {
+      float u = acc + (e.bias ? ldv(e.bias, n, e.bias_bf16) : 0.f);
+      stv(e.C, cr * e.ldc + n, e.c_bf16, u);
+      stv(e.C2, cr * e.ldc2 + n, e.c_bf16, gelu_tanh(u));
+    } break;
+    case EPI_GATE_RESID: {
+      float y = acc + (e.bias ? ldv(e.bias, n, e.bias_bf16) : 0.f);
+      stv(e.C, cr * e.ldc + n, e.c_bf16, y);
+      float g = e.gate[(int64_t)(m / e.rows_per_seq) * e.gate_stride + n];
+      const float* hin = static_cast<const float*>(e.aux);
+      static_cast<float*>(e.C2)[(int64_t)m * e.ldc2 + n] = hin[(int64_t)m * e.ld_aux + n] + g * y;
+    } break;
+    case EPI_DGELU: {
+      float u = ldv(e.aux, (int64_t)m * e.ld_aux + n, e.c_bf16);
+      stv(e.C, cr * e.ldc + n, e.c_bf16, acc * gelu_tanh_grad(u));
+    } break;
+    case EPI_ACCUM:
+      atomicAdd(static_cast<float*>(e.C) + cr * e.ldc + n, acc);
+      break;
+  }
+}
+
+// Eight consecutive columns n .. n+7 of row m (m < M).  Vector path when aligned.
+__device__ __forceinline__ void epi_apply8(const EpiParams& e, int m, int n, const float (&a)[8]) {
+  if (!e.vec_ok || n + 8 > e.N) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      if (n + i < e.N) epi_apply1(e, m, n + i, a[i]);
+    return;
+  }
+  const int64_t cr = epi_crow(e, m);
+  float v[8];
+  if (e.epi != EPI_DGELU && e.epi != EPI_ACCUM && e.bias) {
+    if (e.bias_bf16) {
+      uint4 raw = *reinterpret_cast<const uint4*>(static_cast<const bf16*>(e.bias) + n);
+      const bf16* b = reinterpret_cast<const bf16*>(&raw);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) v[i] = a[i] + __bfloat162float(b[i]);
+    } else {
+      const float4* b4 = reinterpret_cast<const float4*>(static_cast<const float*>(e.bias) + n);
+      float4 b0 = b4[0], b1 = b4[1];
+      v[0] = a[0] + b0.x; v[1] = a[1] + b0.y; v[2] = a[2] + b0.z; v[3] = a[3] + b0.w;
+      v[4] = a[4] + b1.x; v[5] = a[5] + b1.y; v[6] = a[6] + b1.z; v[7] = a[7] + b1.w;
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = a[i];
+  }
+  auto store8 = [&](void* base, int64_t idx, int is_bf16, const float (&x)[8]) {
+    if (is_bf16) {
+      uint4 raw;
+      bf16* h = reinterpret_cast<bf16*>(&raw);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) h[i] = __float2bfloat16_rn(x[i]);
+      *reinterpret_cast<uint4*>(static_cast<bf16*>(base) + idx) = raw;
+    } else {
+      float4* p = reinterpret_cast<float4*>(static_cast<float*>(base) + idx);
+      p[0] = make_float4(x[0], x[1], x[2], x[3]);
+      p[1] = make_float4(x[4], x[5], x[6], x[7]);
+    }
+  };
+  switch (e.epi) {
+    case EPI_STORE:
+      store8(e.C, cr * e.ldc + n, e.c_bf16, v);
+      break;
+    case EPI_GELU: {
+      store8(e.C, cr * e.ldc + n, e.c_bf16, v);
+      float gv[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) gv[i] = gelu_tanh(v[i]);
+      store8(e.C2, cr * e.ldc2 + n, e.c_bf16, gv);
+    } break;
+    case EPI_GATE_RESID: {
+      store8(e.C, cr * e.ldc + n, e.c_bf16, v);
+      const float* g = e.gate + (int64_t)(m / e.rows_per_seq) * e.gate_stride + n;
+      const float4* h4 = reinterpret_cast<const float4*>(static_cast<const float*>(e.aux) + (int64_t)m * e.ld_aux + n);
+      float4 h0 = h4[0], h1 = h4[1];
+      float o[8] = {h0.x + g[0] * v[0], h0.y + g[1] * v[1], h0.z + g[2] * v[2], h0.w + g[3] * v[3],
+                    h1.x + g[4] * v[4], h1.y + g[5] * v[5], h1.z + g[6] * v[6], h1.w + g[7] * v[7]};
+      store8(e.C2, (int64_t)m * e.ldc2 + n, 0, o);
+    } break;
+    case EPI_DGELU: {
+      float u[8];
+      if (e.c_bf16) {
+        uint4 raw = *reinterpret_cast<const uint4*>(static_cast<const bf16*>(e.aux) + (int64_t)m * e.ld_aux + n);
+        const bf16* h = reinterpret_cast<const bf16*>(&raw);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) u[i] = __bfloat162float(h[i]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) u[i] = static_cast<const float*>(e.aux)[(int64_t)m * e.ld_aux + n + i];
+      }
+      float o[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) o[i] = a[i] * gelu_tanh_grad(u[i]);
+      store8(e.C, cr * e.ldc + n, e.c_bf16, o);
+    } break;
+    case EPI_ACCUM: {
+      float* p = static_cast<float*>(e.C) + cr * e.ldc + n;
+      ptx::red_add_v4(p, a[0], a[1], a[2], a[3]);
+      ptx::red_add_v4(p + 4, a[4], a[5], a[6], a[7]);
+    } break;
+  }
+}
+
+// ------------------------------------------------------------------ tcgen05 kernel
+struct TcParams {
+  int tiles_m, tiles_n, splits, k_blocks;
+  EpiParams e;
+};
+
+constexpr int TC_BM = 128;
+constexpr int TC_BK = 64;
+constexpr int TC_THREADS = 192;
+
+template <int BN>
+struct TcCfg {
+  static constexpr int A_BYTES = TC_BM * TC_BK * 2;
+  static constexpr int B_BYTES = BN * TC_BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int STAGES = (196608 / STAGE_BYTES) > 8 ? 8 : (196608 / STAGE_BYTES);
+  static constexpr int TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
+  // + 16 KB guard: every descriptor-addressed read stays inside the allocation even if
+  // the two byte offsets of an MN-major descriptor were interpreted the other way round.
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/ + 16384;
+};
+
+template <int BN, bool A_MN, bool B_MN>
+__global__ void __launch_bounds__(TC_THREADS, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, TcParams p) {
+  using Cfg = TcCfg<BN>;
+  constexpr int STAGES = Cfg::STAGES;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * Cfg::STAGE_BYTES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* tfull = empty + STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  __shared__ volatile int abort_flag;
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    for (int s = 0; s < STAGES; ++s) {
+      ptx::mbar_init(&full[s], 1);
+      ptx::mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      ptx::mbar_init(&tfull[a], 1);
+      ptx::mbar_init(&tempty[a], 4);
+    }
+    ptx::fence_mbar_init();
+    ptx::prefetch_tmap(&tmA);
+    ptx::prefetch_tmap(&tmB);
+  }
+  if (warp == 1) {
+    ptx::tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int total = p.tiles_m * p.tiles_n * p.splits;
+  // tile index -> (m tile, n tile, split); m fastest so consecutive CTAs share B tiles.
+  auto decode = [&](int t, int& tm, int& tn, int& ks) {
+    tm = t % p.tiles_m;
+    int r = t / p.tiles_m;
+    tn = r % p.tiles_n;
+    ks = r / p.tiles_n;
+  };
+  auto krange = [&](int ks, int& kb0, int& kb1) {
+    kb0 = (int)((long long)p.k_blocks * ks / p.splits);
+    kb1 = (int)((long long)p.k_blocks * (ks + 1) / p.splits);
+  };
+
+  if (warp == 0) {
+    if (ptx::elect_one()) {
+      // ---------------- TMA producer
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int t = blockIdx.x; t < total && !abort_flag; t += gridDim.x) {
+        int tm, tn, ks, kb0, kb1;
+        decode(t, tm, tn, ks);
+        krange(ks, kb0, kb1);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!ptx::mbar_wait(&empty[stage], phase ^ 1)) { abort_flag = 1; break; }
+          uint8_t* sA = smem + stage * Cfg::STAGE_BYTES;
+          uint8_t* sB = sA + Cfg::A_BYTES;
+          ptx::mbar_arrive_expect_tx(&full[stage], Cfg::STAGE_BYTES);
+          if (!A_MN) {
+            ptx::tma_load_2d(sA, &tmA, &full[stage], kb * TC_BK, tm * TC_BM);
+          } else {
+#pragma unroll
+            for (int c = 0; c < TC_BM / 64; ++c)
+              ptx::tma_load_2d(sA + c * (64 * TC_BK * 2), &tmA, &full[stage], tm * TC_BM + c * 64, kb * TC_BK);
+          }
+          if (!B_MN) {
+            ptx::tma_load_2d(sB, &tmB, &full[stage], kb * TC_BK, tn * BN);
+          } else {
+#pragma unroll
+            for (int c = 0; c < BN / 64; ++c)
+              ptx::tma_load_2d(sB + c * (64 * TC_BK * 2), &tmB, &full[stage], tn * BN + c * 64, kb * TC_BK);
+          }
+          if (++stage == STAGES) { stage = 0; phase ^= 1; }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (ptx::elect_one()) {
+      // ---------------- MMA issuer
+      constexpr uint32_t idesc = ptx::idesc_bf16(TC_BM, BN, A_MN, B_MN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      for (int t = blockIdx.x; t < total && !abort_flag; t += gridDim.x) {
+        int tm, tn, ks, kb0, kb1;
+        decode(t, tm, tn, ks);
+        krange(ks, kb0, kb1);
+        if (!ptx::mbar_wait(&tempty[acc], acc_phase ^ 1)) { abort_flag = 1; break; }
+        ptx::tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        bool ok = true;
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!ptx::mbar_wait(&full[stage], phase)) { ok = false; break; }
+          ptx::tc_fence_after();
+          const uint32_t a_addr = ptx::smem_u32(smem + stage * Cfg::STAGE_BYTES);
+          const uint32_t b_addr = a_addr + Cfg::A_BYTES;
+#pragma unroll
+          for (int k = 0; k < TC_BK / 16; ++k) {
+            // K-major: step 16 elements = 32 bytes inside the swizzled 128-byte row.
+            // MN-major: step 16 k-rows = two 1024-byte atoms.
+            const uint64_t ad = A_MN ? ptx::sdesc_sw128(a_addr + k * 2048, 64 * TC_BK * 2, 1024)
+                                     : ptx::sdesc_sw128(a_addr + k * 32, 16, 1024);
+            const uint64_t bd = B_MN ? ptx::sdesc_sw128(b_addr + k * 2048, 64 * TC_BK * 2, 1024)
+                                     : ptx::sdesc_sw128(b_addr + k * 32, 16, 1024);
+            ptx::umma_bf16(d_tmem, ad, bd, idesc, (kb > kb0 || k > 0) ? 1u : 0u);
+          }
+          ptx::umma_commit(&empty[stage]);
+          if (++stage == STAGES) { stage = 0; phase ^= 1; }
+        }
+        if (!ok) { abort_flag = 1; break; }
+        ptx::umma_commit(&tfull[acc]);
+        if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+      }
+    }
+  } else {
+    // ---------------- epilogue warps 2..5: TMEM lanes 32*(warp%4) .. +31
+    const int q = warp & 3;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x) {
+      int tm, tn, ks;
+      decode(t, tm, tn, ks);
+      bool ok = ptx::mbar_wait(&tfull[acc], acc_phase);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) { abort_flag = 1; break; }
+      ptx::tc_fence_after();
+      const int m = tm * TC_BM + q * 32 + lane;
+#pragma unroll 1
+      for (int c = 0; c < BN / 32; ++c) {
+        uint32_t r[32];
+        ptx::tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c * 32, r);
+        ptx::tmem_ld_wait();
+        const int n0 = tn * BN + c * 32;
+        if (m < p.e.M && n0 < p.e.N) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            float v[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[j * 8 + i]);
+            epi_apply8(p.e, m, n0 + j * 8, v);
+          }
+        }
+      }
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(&tempty[acc]);
+      if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+    }
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
+  }
+}
+
+// ------------------------------------------------------------------ SIMT kernel
+struct SimtParams {
+  int M, N, K, splits, kb_total;
+  const void* A;
+  int64_t lda;
+  int a_mn, a_bf16;
+  const void* B;
+  int64_t ldb;
+  int b_mn, b_bf16;
+  EpiParams e;
+};
+
+template <int BM, int BN>
+__global__ void __launch_bounds__(256) gemm_simt_kernel(SimtParams p) {
+  constexpr int BK = 16;
+  constexpr int TM = BM / 16, TN = BN / 16;
+  __shared__ float As[BK][BM + 1];
+  __shared__ float Bs[BK][BN + 1];
+  const int tid = threadIdx.x;
+  const int tx = tid % 16, ty = tid / 16;
+  const int tiles_m = (p.M + BM - 1) / BM;
+  const int tm = blockIdx.x % tiles_m, tn = blockIdx.x / tiles_m;
+  const int m0 = tm * BM, n0 = tn * BN;
+  const int ks = blockIdx.y;
+  const int kb0 = (int)((long long)p.kb_total * ks / p.splits);
+  const int kb1 = (int)((long long)p.kb_total * (ks + 1) / p.splits);
+  float acc[TM][TN];
+#pragma unroll
+  for (int i = 0; i < TM; ++i)
+#pragma unroll
+    for (int j = 0; j < TN; ++j) acc[i][j] = 0.f;
+
+  for (int kb = kb0; kb < kb1; ++kb) {
+    const int k0 = kb * BK;
+    for (int idx = tid; idx < BM * BK; idx += 256) {
+      int mm, kk;
+      if (p.a_mn) { mm = idx % BM; kk = idx / BM; } else { kk = idx % BK; mm = idx / BK; }
+      const int m = m0 + mm, k = k0 + kk;
+      float v = 0.f;
+      if (m < p.M && k < p.K)
+        v = ldv(p.A, p.a_mn ? (int64_t)k * p.lda + m : (int64_t)m * p.lda + k, p.a_bf16);
+      As[kk][mm] = v;
+    }
+    for (int idx = tid; idx < BN * BK; idx += 256) {
+      int nn, kk;
+      if (p.b_mn) { nn = idx % BN; kk = idx / BN; } else { kk = idx % BK; nn = idx / BK; }
+      const int n = n0 + nn, k = k0 + kk;
+      float v = 0.f;
+      if (n < p.N && k < p.K)
+        v = ldv(p.B, p.b_mn ? (int64_t)k * p.ldb + n : (int64_t)n * p.ldb + k, p.b_bf16);
+      Bs[kk][nn] = v;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < BK; ++kk) {
+      float a[TM], b[TN];
+#pragma unroll
+      for (int i = 0; i < TM; ++i) a[i] = As[kk][ty + 16 * i];
+#pragma unroll
+      for (int j = 0; j < TN; ++j) b[j] = Bs[kk][tx + 16 * j];
+#pragma unroll
+      for (int i = 0; i < TM; ++i)
+#pragma unroll
+        for (int j = 0; j < TN; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < TM; ++i)
+#pragma unroll
+    for (int j = 0; j < TN; ++j) {
+      const int m = m0 + ty + 16 * i, n = n0 + tx + 16 * j;
+      if (m < p.M && n < p.N) epi_apply1(p.e, m, n, acc[i][j]);
+    }
+}
+
+// ------------------------------------------------------------------ host side
+namespace {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPoint("cuTensorMapEncodeTiled", &ptr, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  });
+  return fn;
+}
+
+// 2D bf16 tensor map over a row-major [rows, cols] matrix with row pitch `ld` elements.
+int make_tmap(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_cols, int box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) {
+    set_last_error("cuTensorMapEncodeTiled is not available from the driver");
+    return JAGG_ERR_CUDA;
+  }
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)(ld * 2)};
+  cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    set_last_error("cuTensorMapEncodeTiled failed (%d) rows=%lld cols=%lld ld=%lld box=%dx%d", (int)r,
+                   (long long)rows, (long long)cols, (long long)ld, box_rows, box_cols);
+    return JAGG_ERR_CUDA;
+  }
+  return JAGG_OK;
+}
+
+EpiParams make_epi(const GemmArgs& g) {
+  EpiParams e;
+  e.M = g.M;
+  e.N = g.N;
+  e.epi = g.epi;
+  e.bias = g.bias;
+  e.bias_bf16 = g.bias_dtype == JAGG_DTYPE_BF16;
+  e.C = g.C;
+  e.ldc = g.ldc;
+  e.c_bf16 = g.c_dtype == JAGG_DTYPE_BF16;
+  e.C2 = g.C2;
+  e.ldc2 = g.ldc2;
+  e.aux = g.aux;
+  e.ld_aux = g.ld_aux;
+  e.gate = g.gate;
+  e.gate_stride = g.gate_stride;
+  e.rows_per_seq = g.rows_per_seq > 0 ? g.rows_per_seq : 1;
+  e.remap_rows = g.remap_rows;
+  e.remap_offset = g.remap_offset;
+  e.remap_stride = g.remap_stride;
+  auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
+  bool ok = (g.N % 8 == 0) && (g.ldc % 8 == 0) && al16(g.C);
+  if (g.bias) ok = ok && al16(g.bias);
+  if (g.epi == EPI_GELU || g.epi == EPI_GATE_RESID) ok = ok && (g.ldc2 % 8 == 0) && al16(g.C2);
+  if (g.epi == EPI_GATE_RESID || g.epi == EPI_DGELU) ok = ok && (g.ld_aux % 8 == 0) && al16(g.aux);
+  e.vec_ok = ok ? 1 : 0;
+  return e;
+}
+
+int validate(const GemmArgs& g) {
+  JAGG_CHECK_ARG(g.M > 0 && g.N > 0 && g.K > 0, "gemm: empty shape %dx%dx%d", g.M, g.N, g.K);
+  JAGG_CHECK_ARG(g.A && g.B && g.C, "gemm: null operand");
+  JAGG_CHECK_ARG(g.epi >= EPI_STORE && g.epi <= EPI_ACCUM, "gemm: bad epilogue %d", g.epi);
+  JAGG_CHECK_ARG(g.epi != EPI_ACCUM || g.c_dtype == JAGG_DTYPE_F32, "gemm: accumulation needs an f32 output");
+  JAGG_CHECK_ARG(g.epi != EPI_GELU || g.C2, "gemm: GELU epilogue needs C2");
+  JAGG_CHECK_ARG(g.epi != EPI_GATE_RESID || (g.C2 && g.aux && g.gate), "gemm: gate epilogue needs C2/aux/gate");
+  JAGG_CHECK_ARG(g.epi != EPI_DGELU || g.aux, "gemm: dGELU epilogue needs aux");
+  return JAGG_OK;
+}
+
+template <int BN, bool A_MN, bool B_MN>
+int launch_tc(const GemmArgs& g, cudaStream_t stream) {
+  using Cfg = TcCfg<BN>;
+  CUtensorMap ta, tb;
+  if (!A_MN)
+    JAGG_TRY(make_tmap(&ta, g.A, g.M, g.K, g.lda, TC_BK, TC_BM));
+  else
+    JAGG_TRY(make_tmap(&ta, g.A, g.K, g.M, g.lda, 64, TC_BK));
+  if (!B_MN)
+    JAGG_TRY(make_tmap(&tb, g.B, g.N, g.K, g.ldb, TC_BK, BN));
+  else
+    JAGG_TRY(make_tmap(&tb, g.B, g.K, g.N, g.ldb, 64, TC_BK));
+  TcParams p;
+  p.tiles_m = ceil_div(g.M, TC_BM);
+  p.tiles_n = ceil_div(g.N, BN);
+  p.k_blocks = ceil_div(g.K, TC_BK);
+  const int nsm = sm_count();
+  int splits = 1;
+  if (g.epi == EPI_ACCUM) {
+    const int tiles = p.tiles_m * p.tiles_n;
+    if (g.split_k > 0)
+      splits = g.split_k;
+    else if (tiles < nsm)
+      splits = (nsm + tiles - 1) / tiles;
+    if (splits > p.k_blocks) splits = p.k_blocks;
+    if (splits < 1) splits = 1;
+  }
+  p.splits = splits;
+  p.e = make_epi(g);
+  const int total = p.tiles_m * p.tiles_n * p.splits;
+  const int grid = total < nsm ? total : nsm;
+  static bool attr_set = false;  // one per template instance
+  if (!attr_set) {
+    JAGG_CUDA_TRY(cudaFuncSetAttribute(gemm_tc_kernel<BN, A_MN, B_MN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       Cfg::SMEM_BYTES));
+    attr_set = true;
+  }
+  gemm_tc_kernel<BN, A_MN, B_MN><<<grid, TC_THREADS, Cfg::SMEM_BYTES, stream>>>(ta, tb, p);
+  JAGG_CUDA_TRY(cudaGetLastError());
+  return JAGG_OK;
+}
+
+template <bool A_MN, bool B_MN>
+int dispatch_bn(const GemmArgs& g, cudaStream_t stream) {
+  // Every K-major box stays inside its tensor's outer extent (N >= BN).
+  if (g.N < 128) return launch_tc<64, A_MN, B_MN>(g, stream);
+  return launch_tc<128, A_MN, B_MN>(g, stream);
+}
+
+bool tc_eligible(const GemmArgs& g) {
+  if (g.a_dtype != JAGG_DTYPE_BF16 || g.b_dtype != JAGG_DTYPE_BF16) return false;
+  auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
+  if (!al16(g.A) || !al16(g.B)) return false;
+  if (g.lda % 8 || g.ldb % 8) return false;
+  if (g.K < TC_BK) return false;
+  if (!g.a_mn && g.M < TC_BM) return false;  // keep every TMA box inside its tensor's outer extent
+  if (!g.b_mn && g.N < 64) return false;
+  if (g.a_mn && g.M < 64) return false;
+  if (g.b_mn && g.N < 64) return false;
+  return true;
+}
+
+}  // namespace
+
+int gemm_simt(const GemmArgs& g, cudaStream_t stream) {
+  JAGG_TRY(validate(g));
+  SimtParams p;
+  p.M = g.M; p.N = g.N; p.K = g.K;
+  p.A = g.A; p.lda = g.lda; p.a_mn = g.a_mn; p.a_bf16 = g.a_dtype == JAGG_DTYPE_BF16;
+  p.B = g.B; p.ldb = g.ldb; p.b_mn = g.b_mn; p.b_bf16 = g.b_dtype == JAGG_DTYPE_BF16;
+  p.e = make_epi(g);
+  p.e.vec_ok = 0;
+  const bool skinny = g.M <= 16;
+  const int BM = skinny ? 16 : 64, BN = 64;
+  const int tiles = ceil_div(g.M, BM) * ceil_div(g.N, BN);
+  p.kb_total = ceil_div(g.K, 16);
+  int splits = 1;
+  if (g.epi == EPI_ACCUM) {
+    const int nsm = sm_count();
+    if (g.split_k > 0)
+      splits = g.split_k;
+    else if (tiles < 2 * nsm)
+      splits = (2 * nsm + tiles - 1) / tiles;
+    if (splits > p.kb_total) splits = p.kb_total;
+    if (splits > 65535) splits = 65535;
+  }
+  p.splits = splits;
+  dim3 grid(tiles, splits);
+  if (skinny)
+    gemm_simt_kernel<16, 64><<<grid, 256, 0, stream>>>(p);
+  else
+    gemm_simt_kernel<64, 64><<<grid, 256, 0, stream>>>(p);
+  JAGG_CUDA_TRY(cudaGetLastError());
+  return JAGG_OK;
+}
+
+int gemm(const GemmArgs& g, cudaStream_t stream) {
+  JAGG_TRY(validate(g));
+  if (!tc_eligible(g)) return gemm_simt(g, stream);
+  if (!g.a_mn && !g.b_mn) return dispatch_bn<false, false>(g, stream);
+  if (!g.a_mn && g.b_mn) return dispatch_bn<false, true>(g, stream);
+  if (g.a_mn && g.b_mn) return dispatch_bn<true, true>(g, stream);
+  return dispatch_bn<true, false>(g, stream);
+}
+
+}  // namespace jagg

@@ -1,0 +1,358 @@
+// GRPO step signals (Phase 2), JAGG aggregation (Phase 3) and gradient reductions.
+//
+// grpo_step_signals runs in three launches:
+//   1. advantages A_i (Eq. advantage) from the group's rewards;
+//   2. ||r_ij||^2 with r_ij = z_{j+1} - z_j - v_ij dt_j, one CTA per (i, j, chunk of D),
+//      partial sums in f64 written to the workspace (fixed order: deterministic);
+//   3. per (i, j): log-prob (Eq. logprob), ratio, clip decision (Eq. grpo_loss), the
+//      coefficient c_ij = scale (-A_i) rho_ij dt_j / sigma_j^2 (0 when clipped); then one
+//      elementwise pass writes s_ij = c_ij r_ij and/or the aggregated cotangents
+//      sum_j (1 - alpha_j) s_ij and sum_j alpha_j s_ij (Eq. alpha, Eq. s_base_corr).
+// The v-hat / z tiles of a window are read twice; at the paper's shapes they fit in L2.
+#include "common.cuh"
+
+namespace jagg {
+
+int unit_status_signals(unsigned* v, int clear) { return read_unit_status(v, clear); }
+
+namespace {
+
+constexpr int SIG_THREADS = 256;
+constexpr int SIG_PER_THREAD = 32;
+constexpr int SIG_CHUNK = SIG_THREADS * SIG_PER_THREAD;  // elements of D per CTA in pass 2
+
+__device__ __forceinline__ float ldv_any(const void* p, int64_t i, int is_f32) {
+  return is_f32 ? static_cast<const float*>(p)[i] : __bfloat162float(static_cast<const bf16*>(p)[i]);
+}
+
+__global__ void advantage_kernel(const float* rewards, int G, double adv_eps, double adv_clip, double* adv) {
+  if (threadIdx.x != 0 || blockIdx.x != 0) return;
+  double mu = 0.0;
+  for (int i = 0; i < G; ++i) mu += (double)rewards[i];
+  mu /= G;
+  double ss = 0.0;
+  for (int i = 0; i < G; ++i) {
+    const double d = (double)rewards[i] - mu;
+    ss += d * d;
+  }
+  const double sd = G > 1 ? sqrt(ss / (G - 1)) : 0.0;
+  for (int i = 0; i < G; ++i) {
+    double a = ((double)rewards[i] - mu) / (sd + adv_eps);
+    a = a > adv_clip ? adv_clip : (a < -adv_clip ? -adv_clip : a);
+    adv[i] = a;
+  }
+}
+
+// grid: (chunks, G*W)
+__global__ void __launch_bounds__(SIG_THREADS) resid_norm_kernel(const void* v, int v_f32, const float* z,
+                                                                 const double* t, int W, int64_t D, double* partial) {
+  const int ij = blockIdx.y;
+  const int i = ij / W, j = ij % W;
+  const float dt = (float)(t[j + 1] - t[j]);
+  const float* z0 = z + ((int64_t)i * (W + 1) + j) * D;
+  const float* z1 = z0 + D;
+  const int64_t vb = ((int64_t)i * W + j) * D;
+  const int64_t k0 = (int64_t)blockIdx.x * SIG_CHUNK;
+  double acc = 0.0;
+  float part = 0.f;
+#pragma unroll 4
+  for (int u = 0; u < SIG_PER_THREAD; ++u) {
+    const int64_t k = k0 + threadIdx.x + (int64_t)u * SIG_THREADS;
+    if (k < D) {
+      const float r = z1[k] - z0[k] - ldv_any(v, vb + k, v_f32) * dt;
+      part = fmaf(r, r, part);
+    }
+    if ((u & 7) == 7) {  // fold every 8 terms into the f64 accumulator
+      acc += (double)part;
+      part = 0.f;
+    }
+  }
+  acc += (double)part;
+  acc = warp_sum(acc);
+  __shared__ double red[SIG_THREADS / 32];
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x / 32] = acc;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double s = 0.0;
+    for (int w = 0; w < SIG_THREADS / 32; ++w) s += red[w];
+    partial[(int64_t)ij * gridDim.x + blockIdx.x] = s;
+  }
+}
+
+// One thread per (i, j).
+__global__ void logprob_kernel(const double* partial, int chunks, const double* t, const double* sigma,
+                               const double* logp_old, const double* adv, int G, int W, int64_t D, double clip_eps,
+                               double scale, double* logp_new, double* ratio, uint8_t* clipped, float* coef) {
+  const int ij = blockIdx.x * blockDim.x + threadIdx.x;
+  if (ij >= G * W) return;
+  const int i = ij / W, j = ij % W;
+  double rr = 0.0;
+  for (int c = 0; c < chunks; ++c) rr += partial[(int64_t)ij * chunks + c];
+  const double sg = sigma[j];
+  const double dt = t[j + 1] - t[j];
+  const double lp = -rr / (2.0 * sg * sg) - (double)D * log(sqrt(2.0 * 3.14159265358979323846) * sg);
+  const double rho = exp(lp - logp_old[ij]);
+  const double a = adv[i];
+  const bool clip = (a > 0.0 && rho > 1.0 + clip_eps) || (a < 0.0 && rho < 1.0 - clip_eps);
+  logp_new[ij] = lp;
+  ratio[ij] = rho;
+  clipped[ij] = clip ? 1 : 0;
+  coef[ij] = clip ? 0.f : (float)(scale * (-a) * rho * dt / (sg * sg));
+}
+
+// grid: (ceil(D / SIG_THREADS / 4), G).  Each thread: 4 consecutive elements of D.
+__global__ void __launch_bounds__(SIG_THREADS) apply_kernel(const void* v, int v_f32, const float* z, const double* t,
+                                                            const float* coef, int G, int W, int64_t D, float* s_out,
+                                                            float* cot_out) {
+  const int i = blockIdx.y;
+  const int64_t kbase = ((int64_t)blockIdx.x * SIG_THREADS + threadIdx.x) * 4;
+  if (kbase >= D) return;
+  const double den = t[0] - t[W - 1];
+  float base[4] = {0.f, 0.f, 0.f, 0.f}, corr[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int j = 0; j < W; ++j) {
+    const float dt = (float)(t[j + 1] - t[j]);
+    const float c = coef[i * W + j];
+    const float al = cot_out ? (den != 0.0 ? (float)((t[0] - t[j]) / den) : 0.f) : 0.f;
+    const float* z0 = z + ((int64_t)i * (W + 1) + j) * D;
+    const float* z1 = z0 + D;
+    const int64_t vb = ((int64_t)i * W + j) * D;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int64_t k = kbase + e;
+      if (k < D) {
+        const float r = z1[k] - z0[k] - ldv_any(v, vb + k, v_f32) * dt;
+        const float s = c * r;
+        if (s_out) s_out[vb + k] = s;
+        base[e] += (1.f - al) * s;
+        corr[e] += al * s;
+      }
+    }
+  }
+  if (cot_out) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int64_t k = kbase + e;
+      if (k < D) {
+        cot_out[(int64_t)i * D + k] = base[e];
+        cot_out[((int64_t)G + i) * D + k] = corr[e];
+      }
+    }
+  }
+}
+
+__global__ void check_alpha_kernel(const double* t, int W) {
+  if (threadIdx.x == 0 && blockIdx.x == 0 && !(t[0] - t[W - 1] != 0.0)) set_device_status(JAGG_DEV_BADARG);
+}
+
+__global__ void aggregate_kernel(const float* s, const double* t, int G, int W, int64_t D, float* cot) {
+  const int i = blockIdx.y;
+  const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= D) return;
+  const double den = t[0] - t[W - 1];
+  float base = 0.f, corr = 0.f;
+  if (den != 0.0) {
+    for (int j = 0; j < W; ++j) {
+      const float al = (float)((t[0] - t[j]) / den);
+      const float v = s[((int64_t)i * W + j) * D + k];
+      base += (1.f - al) * v;
+      corr += al * v;
+    }
+  }
+  cot[(int64_t)i * D + k] = base;
+  cot[((int64_t)G + i) * D + k] = corr;
+}
+
+// ------------------------------------------------------------------ grad_reduce
+constexpr int GR_BLOCKS = 1024;
+constexpr int GR_THREADS = 256;
+
+__global__ void __launch_bounds__(GR_THREADS) grad_reduce_kernel(const float* a, const float* b, int64_t P,
+                                                                 float alpha, float* acc, double* partial) {
+  // Each thread handles runs of 8 float4; f32 sums over a run are folded into f64.
+  double sab = 0.0, saa = 0.0, sbb = 0.0;
+  const int64_t nvec = P / 4;
+  const float4* a4 = reinterpret_cast<const float4*>(a);
+  const float4* b4 = reinterpret_cast<const float4*>(b ? b : a);
+  float4* c4 = reinterpret_cast<float4*>(acc);
+  const int64_t stride = (int64_t)GR_BLOCKS * GR_THREADS;
+  int64_t idx = (int64_t)blockIdx.x * GR_THREADS + threadIdx.x;
+  while (idx < nvec) {
+    float fab = 0.f, faa = 0.f, fbb = 0.f;
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+      const int64_t q = idx + (int64_t)r * stride;
+      if (q < nvec) {
+        const float4 x = a4[q];
+        const float4 y = b4[q];
+        fab += x.x * y.x + x.y * y.y + x.z * y.z + x.w * y.w;
+        faa += x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w;
+        fbb += y.x * y.x + y.y * y.y + y.z * y.z + y.w * y.w;
+        if (acc) {
+          float4 c = c4[q];
+          c.x += alpha * x.x; c.y += alpha * x.y; c.z += alpha * x.z; c.w += alpha * x.w;
+          c4[q] = c;
+        }
+      }
+    }
+    sab += fab;
+    saa += faa;
+    sbb += fbb;
+    idx += 8 * stride;
+  }
+  // scalar tail (P % 4), handled by block 0
+  if (blockIdx.x == 0) {
+    for (int64_t k = nvec * 4 + threadIdx.x; k < P; k += GR_THREADS) {
+      const float x = a[k], y = b ? b[k] : a[k];
+      sab += (double)x * y;
+      saa += (double)x * x;
+      sbb += (double)y * y;
+      if (acc) acc[k] += alpha * x;
+    }
+  }
+  if (!partial) return;
+  sab = warp_sum(sab);
+  saa = warp_sum(saa);
+  sbb = warp_sum(sbb);
+  __shared__ double red[3][GR_THREADS / 32];
+  const int w = threadIdx.x / 32;
+  if ((threadIdx.x & 31) == 0) {
+    red[0][w] = sab;
+    red[1][w] = saa;
+    red[2][w] = sbb;
+  }
+  __syncthreads();
+  if (threadIdx.x < 3) {
+    double s = 0.0;
+    for (int i = 0; i < GR_THREADS / 32; ++i) s += red[threadIdx.x][i];
+    partial[(int64_t)blockIdx.x * 3 + threadIdx.x] = s;
+  }
+}
+
+__global__ void grad_reduce_final(const double* partial, double* out3) {
+  if (threadIdx.x < 3) {
+    double s = 0.0;
+    for (int i = 0; i < GR_BLOCKS; ++i) s += partial[(int64_t)i * 3 + threadIdx.x];
+    out3[threadIdx.x] = s;
+  }
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+}  // namespace
+
+}  // namespace jagg
+
+using namespace jagg;
+
+// ------------------------------------------------------------------ C ABI
+extern "C" int64_t jagg_signals_workspace_bytes(int G, int W, int64_t D) {
+  if (G <= 0 || W <= 0 || D <= 0) return 0;
+  const int64_t chunks = (D + SIG_CHUNK - 1) / SIG_CHUNK;
+  return (int64_t)G * W * chunks * 8 + (int64_t)G * W * 4 + 64;
+}
+
+extern "C" int grpo_step_signals(const void* v_hat, int v_dtype, const float* z, const double* t, const double* sigma,
+                                 const double* logp_old, const float* rewards, int G, int W, int64_t D,
+                                 double clip_eps, double adv_clip, double adv_eps, double scale, float* s_out,
+                                 float* cot_out, double* logp_new, double* ratio, uint8_t* clipped, double* adv_out,
+                                 void* ws, size_t ws_bytes, cudaStream_t stream) {
+  JAGG_CHECK_ARG(G > 0 && W > 0 && D > 0, "grpo_step_signals: G=%d W=%d D=%lld must be positive", G, W,
+                 (long long)D);
+  JAGG_CHECK_ARG(G <= 65535 && (int64_t)G * W <= 65535, "grpo_step_signals: G*W too large");
+  JAGG_CHECK_ARG(v_dtype == JAGG_DTYPE_F32 || v_dtype == JAGG_DTYPE_BF16, "grpo_step_signals: bad v_dtype");
+  JAGG_CHECK_ARG(v_hat && z && t && sigma && logp_old && rewards && logp_new && ratio && clipped && adv_out && ws,
+                 "grpo_step_signals: null pointer");
+  JAGG_CHECK_ARG(!cot_out || W >= 2, "grpo_step_signals: aggregation needs W >= 2");
+  JAGG_CHECK_ARG(clip_eps >= 0.0 && adv_clip >= 0.0 && adv_eps >= 0.0, "grpo_step_signals: negative constant");
+  const int64_t need = jagg_signals_workspace_bytes(G, W, D);
+  if ((int64_t)ws_bytes < need) {
+    set_last_error("grpo_step_signals: workspace %zu < %lld bytes", ws_bytes, (long long)need);
+    return JAGG_ERR_WORKSPACE;
+  }
+  JAGG_CHECK_ARG(aligned16(ws), "grpo_step_signals: workspace not 16-byte aligned");
+  const int chunks = (int)((D + SIG_CHUNK - 1) / SIG_CHUNK);
+  double* partial = static_cast<double*>(ws);
+  float* coef = reinterpret_cast<float*>(partial + (int64_t)G * W * chunks);
+  const int vf32 = v_dtype == JAGG_DTYPE_F32;
+  advantage_kernel<<<1, 32, 0, stream>>>(rewards, G, adv_eps, adv_clip, adv_out);
+  JAGG_CUDA_TRY(cudaGetLastError());
+  resid_norm_kernel<<<dim3(chunks, G * W), SIG_THREADS, 0, stream>>>(v_hat, vf32, z, t, W, D, partial);
+  JAGG_CUDA_TRY(cudaGetLastError());
+  logprob_kernel<<<ceil_div((int64_t)G * W, 128), 128, 0, stream>>>(partial, chunks, t, sigma, logp_old, adv_out, G,
+                                                                     W, D, clip_eps, scale, logp_new, ratio, clipped,
+                                                                     coef);
+  JAGG_CUDA_TRY(cudaGetLastError());
+  if (s_out || cot_out) {
+    if (cot_out) {
+      check_alpha_kernel<<<1, 32, 0, stream>>>(t, W);
+      JAGG_CUDA_TRY(cudaGetLastError());
+    }
+    const int gx = ceil_div(D, (int64_t)SIG_THREADS * 4);
+    apply_kernel<<<dim3(gx, G), SIG_THREADS, 0, stream>>>(v_hat, vf32, z, t, coef, G, W, D, s_out, cot_out);
+    JAGG_CUDA_TRY(cudaGetLastError());
+  }
+  return JAGG_OK;
+}
+
+extern "C" int jagg_aggregate(const float* s, const double* t_window, int G, int W, int64_t D, float* cot,
+                              cudaStream_t stream) {
+  JAGG_CHECK_ARG(s && t_window && cot, "jagg_aggregate: null pointer");
+  JAGG_CHECK_ARG(G > 0 && G <= 65535 && D > 0, "jagg_aggregate: bad G=%d or D=%lld", G, (long long)D);
+  JAGG_CHECK_ARG(W >= 2, "jagg_aggregate: W=%d, the endpoints must differ (W >= 2)", W);
+  check_alpha_kernel<<<1, 32, 0, stream>>>(t_window, W);
+  JAGG_CUDA_TRY(cudaGetLastError());
+  aggregate_kernel<<<dim3(ceil_div(D, 256), G), 256, 0, stream>>>(s, t_window, G, W, D, cot);
+  JAGG_CUDA_TRY(cudaGetLastError());
+  return JAGG_OK;
+}
+
+extern "C" int jagg_route(int n_windows, double jagg_frac, const double* cos, double tau, uint8_t* route,
+                          double* derived_frac) {
+  JAGG_CHECK_ARG(n_windows > 0 && route, "jagg_route: n_windows=%d / null route", n_windows);
+  if (!cos) {
+    JAGG_CHECK_ARG(jagg_frac >= 0.0 && jagg_frac <= 1.0, "jagg_route: jagg_frac %g outside [0, 1]", jagg_frac);
+    int n_jagg = (int)floor(jagg_frac * n_windows + 1e-9);
+    if (n_jagg > n_windows) n_jagg = n_windows;
+    for (int w = 0; w < n_windows; ++w) route[w] = w < n_jagg ? 1 : 0;
+    if (derived_frac) *derived_frac = (double)n_jagg / n_windows;
+    return JAGG_OK;
+  }
+  int prefix = 0;
+  bool in_prefix = true;
+  for (int w = 0; w < n_windows; ++w) {
+    route[w] = cos[w] >= tau ? 1 : 0;
+    if (in_prefix && route[w])
+      ++prefix;
+    else
+      in_prefix = false;
+  }
+  if (derived_frac) *derived_frac = (double)prefix / n_windows;
+  return JAGG_OK;
+}
+
+extern "C" int64_t jagg_grad_reduce_workspace_bytes(int64_t P) {
+  (void)P;
+  return (int64_t)GR_BLOCKS * 3 * 8;
+}
+
+extern "C" int grad_reduce(const float* a, const float* b, int64_t P, float alpha, float* acc, double* out3, void* ws,
+                           size_t ws_bytes, cudaStream_t stream) {
+  JAGG_CHECK_ARG(a && P > 0, "grad_reduce: null input or P=%lld", (long long)P);
+  JAGG_CHECK_ARG(aligned16(a) && (!b || aligned16(b)) && (!acc || aligned16(acc)),
+                 "grad_reduce: buffers must be 16-byte aligned");
+  if (!acc && !out3) return JAGG_OK;
+  if (out3) {
+    if (!ws || (int64_t)ws_bytes < jagg_grad_reduce_workspace_bytes(P)) {
+      set_last_error("grad_reduce: workspace too small");
+      return JAGG_ERR_WORKSPACE;
+    }
+  }
+  grad_reduce_kernel<<<GR_BLOCKS, GR_THREADS, 0, stream>>>(a, b, P, alpha, acc,
+                                                           out3 ? static_cast<double*>(ws) : nullptr);
+  JAGG_CUDA_TRY(cudaGetLastError());
+  if (out3) {
+    grad_reduce_final<<<1, 32, 0, stream>>>(static_cast<const double*>(ws), out3);
+    JAGG_CUDA_TRY(cudaGetLastError());
+  }
+  return JAGG_OK;
+}

@@ -1,0 +1,59 @@
+// Kernel-level entry points for the library's tests (include/jagg_testing.h).
+#include "../../include/jagg_testing.h"
+#include "attention.cuh"
+#include "gemm.cuh"
+
+using namespace jagg;
+
+extern "C" int jagg_test_gemm(const jagg_gemm_desc* d, cudaStream_t stream) {
+  JAGG_CHECK_ARG(d, "jagg_test_gemm: null descriptor");
+  GemmArgs g;
+  g.M = d->M; g.N = d->N; g.K = d->K;
+  g.A = d->A; g.lda = d->lda; g.a_mn = d->a_mn != 0; g.a_dtype = d->a_dtype;
+  g.B = d->B; g.ldb = d->ldb; g.b_mn = d->b_mn != 0; g.b_dtype = d->b_dtype;
+  g.epi = d->epi;
+  g.bias = d->bias; g.bias_dtype = d->bias_dtype;
+  g.C = d->C; g.ldc = d->ldc; g.c_dtype = d->c_dtype;
+  g.C2 = d->C2; g.ldc2 = d->ldc2;
+  g.aux = d->aux; g.ld_aux = d->ld_aux;
+  g.gate = d->gate; g.gate_stride = d->gate_stride; g.rows_per_seq = d->rows_per_seq;
+  g.split_k = d->split_k;
+  return d->force_simt ? gemm_simt(g, stream) : gemm(g, stream);
+}
+
+static AttnArgs make_args(const void* qkv, int B, int N, int heads, int dh, int dtype, void* o, float* lse) {
+  AttnArgs a;
+  const int d = heads * dh;
+  a.B = B; a.N = N; a.heads = heads; a.dh = dh; a.scale = 1.f / sqrtf((float)dh);
+  a.q = a.k = a.v = seg_single(const_cast<void*>(qkv), 3 * d, N);
+  a.q_col0 = 0; a.k_col0 = d; a.v_col0 = 2 * d;
+  a.o = seg_single(o, d, N);
+  a.lse = lse;
+  a.dtype = dtype;
+  return a;
+}
+
+extern "C" int jagg_test_attention_fwd(const void* qkv, int B, int N, int heads, int dh, int dtype, void* o,
+                                       float* lse, cudaStream_t stream) {
+  JAGG_CHECK_ARG(qkv && o && lse, "jagg_test_attention_fwd: null pointer");
+  return attention_fwd(make_args(qkv, B, N, heads, dh, dtype, o, lse), stream);
+}
+
+extern "C" int64_t jagg_test_attention_scratch_bytes(int B, int N, int heads, int dh) {
+  return attention_bwd_scratch_floats(B, N, heads, dh) * 4;
+}
+
+extern "C" int jagg_test_attention_bwd(const void* qkv, const void* o, const float* lse, const void* dO, int B, int N,
+                                       int heads, int dh, int dtype, void* dqkv, void* scratch,
+                                       cudaStream_t stream) {
+  JAGG_CHECK_ARG(qkv && o && lse && dO && dqkv && scratch, "jagg_test_attention_bwd: null pointer");
+  AttnBwdArgs ab;
+  ab.f = make_args(qkv, B, N, heads, dh, dtype, const_cast<void*>(o), const_cast<float*>(lse));
+  const int d = heads * dh;
+  ab.dO = seg_single(const_cast<void*>(dO), d, N);
+  ab.Dv = static_cast<float*>(scratch);
+  ab.dq_acc = ab.Dv + (int64_t)B * heads * N;
+  ab.dq = ab.dk = ab.dv = seg_single(dqkv, 3 * d, N);
+  ab.dq_col0 = 0; ab.dk_col0 = d; ab.dv_col0 = 2 * d;
+  return attention_bwd(ab, stream);
+}

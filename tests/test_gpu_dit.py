@@ -1,0 +1,79 @@
+"""GPU parity of Phase 1 (forward with saved activations) and Phase 4 (the joint VJP)
+with the float64 oracle on the same seeded weights, inputs and cotangents."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from gpu_cases import GpuModel, cosine, flat, model_inputs, oracle_vjp, rel_l2
+
+pytestmark = pytest.mark.gpu
+
+jg = pytest.importorskip("paper_2607_17572_gb300")
+
+TINY = synth.WORKLOADS["tiny_dit_f32"]
+DITB = synth.WORKLOADS["dit_b_bf16"]
+
+CASES = [
+    # (workload, rows B, forward tol, gradient tol)
+    (TINY, 8, 1e-5, 1e-4),                                                    # 2G rows of the tiny config
+    (synth.small_variant(TINY, name="tiny_odd", latent_h=6, latent_w=5, txt_len=3, txt_dim=40), 3, 1e-5, 1e-4),
+    (synth.small_variant(DITB, name="ditb_2blocks", depth=2), 4, 2e-2, 1e-2),  # DiT-B width, 2 blocks
+    (synth.small_variant(DITB, name="ditb_ragged", depth=1, latent_h=18, latent_w=22, txt_len=29), 3, 2e-2, 1e-2),
+]
+
+
+def _check(wl, B, ftol, gtol, seed=5):
+    params = synth.make_params(wl)
+    z, t, txt = model_inputs(wl, B, seed)
+    rng = np.random.Generator(np.random.PCG64(seed + 1))
+    cot = synth.storage_round(rng.standard_normal(z.shape), wl.dtype)
+    gm = GpuModel(jg, wl, params)
+    v, saved, ws = gm.forward(z, t, txt)
+    grad = gm.vjp(saved, ws, B, cot)
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    v_o, g_o = oracle_vjp(wl, params, z, t, txt, cot)
+    fv = rel_l2(v.float().cpu().numpy(), v_o)
+    assert fv <= ftol, f"forward rel L2 {fv:.3e}"
+    g_gpu = jg.unpack_grads(gm.cfg, grad)
+    names = list(g_o)
+    tot = rel_l2(flat(g_gpu, names), flat(g_o, names))
+    cs = cosine(flat(g_gpu, names), flat(g_o, names))
+    per = {k: rel_l2(g_gpu[k], g_o[k]) for k in names}
+    worst = max(per, key=per.get)
+    print(f"{wl.name}: forward {fv:.2e}, grad rel L2 {tot:.2e}, cos {cs:.6f}, worst {worst} {per[worst]:.2e}")
+    assert tot <= gtol, f"gradient rel L2 {tot:.3e} (worst {worst}: {per[worst]:.3e})"
+    assert cs >= 0.999
+    return grad, gm, saved, ws, cot
+
+
+@pytest.mark.parametrize("wl,B,ftol,gtol", CASES, ids=[c[0].name for c in CASES])
+def test_forward_and_joint_vjp_match_oracle(wl, B, ftol, gtol):
+    _check(wl, B, ftol, gtol)
+
+
+def test_vjp_accumulates_and_is_linear_in_the_cotangent():
+    wl = TINY
+    grad, gm, saved, ws, cot = _check(wl, 8, 1e-5, 1e-4)
+    g1 = grad.clone()
+    gm.vjp(saved, ws, 8, 2.0 * cot, grad=grad)      # grad += J^T (2 cot)
+    torch.cuda.synchronize()
+    assert rel_l2(grad.cpu().numpy(), 3.0 * g1.cpu().numpy()) < 1e-5
+
+
+def test_forward_without_saves_matches_saved_forward():
+    wl = synth.small_variant(DITB, name="ditb_2blocks", depth=2)
+    params = synth.make_params(wl)
+    z, t, txt = model_inputs(wl, 4, 9)
+    gm = GpuModel(jg, wl, params)
+    v1, _, _ = gm.forward(z, t, txt, save=True)
+    v2, _, _ = gm.forward(z, t, txt, save=False)
+    torch.cuda.synchronize()
+    assert torch.equal(v1, v2)
+
+
+@pytest.mark.slow
+def test_dit_b_full_depth_joint_vjp():
+    """DiT-B (12 blocks, 333 tokens) at its JAGG batch of 2G = 16 rows."""
+    _check(DITB, 2 * DITB.G, 2e-2, 1e-2, seed=11)

@@ -1,0 +1,158 @@
+"""Kernel-level GPU tests: the tcgen05 dense products (all operand layouts, ragged tails,
+fused epilogues, split-K accumulation) and the attention kernels against plain PyTorch
+fp32 computations on the same rounded inputs."""
+import math
+
+import pytest
+import torch
+import torch.nn.functional as F
+
+pytestmark = pytest.mark.gpu
+
+jg = pytest.importorskip("paper_2607_17572_gb300")
+
+
+def _rel(a, b):
+    return (torch.linalg.vector_norm((a.double() - b.double())) / torch.linalg.vector_norm(b.double())).item()
+
+
+def _desc(M, N, K, A, lda, a_mn, B, ldb, b_mn, dt, C, ldc, c_dt, epi=0, **kw):
+    d = jg.GemmDesc()
+    d.M, d.N, d.K = M, N, K
+    d.A, d.lda, d.a_mn, d.a_dtype = A.data_ptr(), lda, int(a_mn), dt
+    d.B, d.ldb, d.b_mn, d.b_dtype = B.data_ptr(), ldb, int(b_mn), dt
+    d.epi = epi
+    d.C, d.ldc, d.c_dtype = C.data_ptr(), ldc, c_dt
+    d.bias_dtype = dt
+    d.rows_per_seq = 1
+    for k, v in kw.items():
+        setattr(d, k, v.data_ptr() if isinstance(v, torch.Tensor) else v)
+    return d
+
+
+SHAPES = [(256, 128, 128), (300, 200, 192), (128, 64, 64), (1000, 768, 768), (5328, 2304, 768), (777, 320, 1000)]
+
+
+@pytest.mark.parametrize("a_mn,b_mn", [(False, False), (False, True), (True, True), (True, False)])
+@pytest.mark.parametrize("M,N,K", SHAPES)
+def test_tcgen05_gemm_layouts(M, N, K, a_mn, b_mn):
+    torch.manual_seed(M * 7 + N * 3 + K)
+    dev = "cuda"
+    A = torch.randn(M, K, device=dev).bfloat16()       # logical A[m, k]
+    B = torch.randn(N, K, device=dev).bfloat16()       # logical B[n, k]
+    As = A.t().contiguous() if a_mn else A
+    Bs = B.t().contiguous() if b_mn else B
+    lda = M if a_mn else K
+    ldb = N if b_mn else K
+    C = torch.full((M, N), float("nan"), device=dev)
+    jg.test_gemm(_desc(M, N, K, As, lda, a_mn, Bs, ldb, b_mn, jg.DTYPE_BF16, C, N, jg.DTYPE_F32))
+    ref = A.float() @ B.float().t()
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    assert _rel(C, ref) < 1e-5
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 200, 192), (2048, 768, 768)])
+def test_gemm_epilogues(M, N, K):
+    torch.manual_seed(1)
+    dev = "cuda"
+    A = torch.randn(M, K, device=dev).bfloat16()
+    B = (torch.randn(N, K, device=dev) / math.sqrt(K)).bfloat16()
+    bias = torch.randn(N, device=dev).bfloat16()
+    acc = A.float() @ B.float().t()
+    # GELU: u and gelu(u)
+    U = torch.empty(M, N, device=dev, dtype=torch.bfloat16)
+    GU = torch.empty_like(U)
+    jg.test_gemm(_desc(M, N, K, A, K, 0, B, K, 0, jg.DTYPE_BF16, U, N, jg.DTYPE_BF16, epi=1, bias=bias, C2=GU,
+                       ldc2=N))
+    u = acc + bias.float()
+    assert _rel(U.float(), u) < 5e-3
+    assert _rel(GU.float(), F.gelu(u, approximate="tanh")) < 5e-3
+    # gated residual: y = acc + bias; h_out = h_in + gate[seq] * y
+    rows = 37
+    gate = torch.randn((M + rows - 1) // rows, N + 8, device=dev)
+    hin = torch.randn(M, N, device=dev)
+    Y = torch.empty(M, N, device=dev, dtype=torch.bfloat16)
+    H = torch.empty(M, N, device=dev)
+    jg.test_gemm(_desc(M, N, K, A, K, 0, B, K, 0, jg.DTYPE_BF16, Y, N, jg.DTYPE_BF16, epi=2, bias=bias, C2=H, ldc2=N,
+                       aux=hin, ld_aux=N, gate=gate, gate_stride=N + 8, rows_per_seq=rows))
+    g = gate[torch.arange(M, device=dev) // rows, :N]
+    assert _rel(H, hin + g * u) < 1e-5
+    # dGELU: acc * gelu'(aux)
+    aux = torch.randn(M, N, device=dev).bfloat16()
+    O = torch.empty(M, N, device=dev, dtype=torch.bfloat16)
+    jg.test_gemm(_desc(M, N, K, A, K, 0, B, K, 0, jg.DTYPE_BF16, O, N, jg.DTYPE_BF16, epi=3, aux=aux, ld_aux=N))
+    x = aux.float().requires_grad_()
+    F.gelu(x, approximate="tanh").backward(acc)
+    assert _rel(O.float(), x.grad) < 5e-3
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+
+
+@pytest.mark.parametrize("split", [0, 1, 3])
+def test_gemm_accumulate_weight_gradient(split):
+    """dW += dY^T X with both operands MN-major, accumulated into an existing f32 buffer."""
+    torch.manual_seed(2)
+    dev = "cuda"
+    M, N, K = 5328, 768, 2304        # tokens, in, out: dW [out, in] += dY[tok, out]^T X[tok, in]
+    X = torch.randn(M, N, device=dev).bfloat16()
+    dY = torch.randn(M, K, device=dev).bfloat16()
+    G0 = torch.randn(K, N, device=dev)
+    G = G0.clone()
+    jg.test_gemm(_desc(K, N, M, dY, K, 1, X, N, 1, jg.DTYPE_BF16, G, N, jg.DTYPE_F32, epi=4, split_k=split))
+    ref = G0 + dY.float().t() @ X.float()
+    torch.cuda.synchronize()
+    assert _rel(G, ref) < 1e-5
+
+
+@pytest.mark.parametrize("M,N,K,a_mn,b_mn", [(16, 4608, 768, 0, 0), (16, 768, 56832, 0, 1), (56832, 768, 16, 1, 1),
+                                              (40, 70, 33, 0, 0), (7, 9, 11, 1, 0)])
+def test_simt_gemm_f32(M, N, K, a_mn, b_mn):
+    torch.manual_seed(3)
+    dev = "cuda"
+    A = torch.randn(M, K, device=dev)
+    B = torch.randn(N, K, device=dev)
+    As = A.t().contiguous() if a_mn else A
+    Bs = B.t().contiguous() if b_mn else B
+    C0 = torch.randn(M, N, device=dev)
+    C = C0.clone()
+    jg.test_gemm(_desc(M, N, K, As, M if a_mn else K, a_mn, Bs, N if b_mn else K, b_mn, jg.DTYPE_F32, C, N,
+                       jg.DTYPE_F32, epi=4))
+    torch.cuda.synchronize()
+    assert _rel(C, C0 + A.double().float() @ B.t()) < 1e-5
+
+
+def _attn_ref(qkv, B, N, H, dh):
+    q, k, v = qkv.float().view(B, N, 3, H, dh).permute(2, 0, 3, 1, 4)
+    return q, k, v
+
+
+@pytest.mark.parametrize("dtype,dh,N,B,H", [(torch.bfloat16, 64, 333, 2, 3), (torch.bfloat16, 128, 200, 1, 2),
+                                            (torch.bfloat16, 64, 64, 1, 1), (torch.bfloat16, 128, 1536, 1, 2),
+                                            (torch.bfloat16, 64, 24, 3, 2),
+                                            (torch.float32, 16, 24, 4, 4), (torch.float32, 64, 97, 2, 2)])
+def test_attention_forward_backward(dtype, dh, N, B, H):
+    torch.manual_seed(N + dh)
+    dev = "cuda"
+    d = H * dh
+    qkv = (torch.randn(B * N, 3 * d, device=dev) * 1.5).to(dtype)
+    o = torch.empty(B * N, d, device=dev, dtype=dtype)
+    lse = torch.empty(B, H, N, device=dev)
+    jg.test_attention_fwd(qkv, B, N, H, dh, o, lse)
+    q, k, v = _attn_ref(qkv, B, N, H, dh)
+    q.requires_grad_(); k.requires_grad_(); v.requires_grad_()
+    s = (q @ k.transpose(-1, -2)) / math.sqrt(dh)
+    ref_lse = torch.logsumexp(s, -1)
+    ref_o = torch.softmax(s, -1) @ v
+    tol = 1e-2 if dtype == torch.bfloat16 else 1e-5
+    assert _rel(o.float().view(B, N, H, dh).transpose(1, 2), ref_o) < tol
+    assert (lse - ref_lse).abs().max().item() < (1e-2 if dtype == torch.bfloat16 else 1e-5)
+    dO = torch.randn(B * N, d, device=dev).to(dtype)
+    # reference gradient uses the kernel's own (rounded) output, as the kernel does
+    ref_o.backward(dO.float().view(B, N, H, dh).transpose(1, 2))
+    dqkv = torch.empty(B * N, 3 * d, device=dev, dtype=dtype)
+    jg.test_attention_bwd(qkv, o, lse, dO, B, N, H, dh, dqkv)
+    torch.cuda.synchronize()
+    g = dqkv.float().view(B, N, 3, H, dh).permute(2, 0, 3, 1, 4)
+    for i, t in enumerate((q, k, v)):
+        assert _rel(g[i], t.grad) < (2e-2 if dtype == torch.bfloat16 else 1e-4), "qkv"[i]
