@@ -1,0 +1,517 @@
+#!/usr/bin/env python3
+"""Throughput of the JAGG backward path on GB300.
+
+One step = the whole update-stage backward of one GRPO group on the DiT-B workload
+(12 single-stream blocks, d = 768, 256 image + 77 text tokens; G = 8 samples, T = 16
+sampling steps, windows of W = 4, jagg_frac = 1): for every window, the step signals with
+the fused t-weighted aggregation (Phases 2-3) and one joint VJP over the 2G endpoint rows
+accumulating the fp32 parameter gradient (Phase 4), then the gradient's squared norm.
+The forward passes of Phase 1 (endpoints saved, middle steps without saves) run before
+the timed region: their saved activations are inputs resident in HBM.  The metric is
+trajectory-steps of gradient per second: G * T (sample, step) pairs per step.
+
+The same step on the exact per-step path (jagg_frac = 0: each window's VJP over all W*G
+step inputs with their own s_j) is timed too, and `e2e` times the update stage through
+the public API from pinned host buffers (Phase 1 forwards included).  `--impl reference`
+times the float64 CPU oracle instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "JAGG backward trajectory-steps/s on 1 GB300; tensor-pipe % of BF16 peak"
+UNIT = "trajectory-steps/s"
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["jagg", "reference"], default="jagg")
+    p.add_argument("--workload", default="dit_b_bf16")
+    p.add_argument("--no-graph", action="store_true", help="launch eagerly instead of replaying a CUDA graph")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--quick", action="store_true", help="skip the full-W, e2e and CPU legs")
+    return p.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return d.get("bf16_tflops", 1914.6), d.get("bf16_tflops_sustained", 1710.6), d.get("hbm_gbs", 6771.1), "measured"
+    return 1900.0, 1700.0, 6800.0, "fallback"
+
+
+# ----------------------------------------------------------------------------- distributed
+def dist_setup():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    return ws, rank
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, ws: int) -> float:
+    if ws == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi samples (every 200 ms) of SM clock and throttle reasons during a region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.f,
+                                         stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        self.f.flush()
+        self.f.seek(0)
+        rows = [r.split(",") for r in self.f.read().strip().splitlines() if r.strip()]
+        os.unlink(self.f.name)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        sm = [float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        for r in rows:
+            for k, name in enumerate(names):
+                if len(r) > 5 + k and r[5 + k].strip().lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(rows)}
+
+
+# ----------------------------------------------------------------------------- workload
+class Bench:
+    def __init__(self, wl, dev):
+        import paper_2607_17572_gb300 as jg
+        self.jg = jg
+        self.wl = wl
+        self.dev = dev
+        self.cfg = jg.Config.from_workload(wl)
+        self.tdt = self.cfg.torch_dtype
+        params = synth.make_params(wl)
+        self.weights = jg.pack_params(self.cfg, params, dev)
+        del params
+        self.model = jg.Model(self.cfg, self.weights)
+        self.P = jg.param_count(self.cfg)
+        G, T, W = wl.G, wl.T, wl.W
+        self.nw = T // W
+        self.D = wl.D
+        self.shape = (wl.in_channels, wl.latent_h, wl.latent_w)
+        self.draws = synth.draw_group(wl)
+        self.t = synth.time_grid(T, wl.shift)
+        self.sig = synth.sigma_schedule(self.t, wl.eta)
+        self.scale = 1.0 / (G * T)
+        f64 = dict(dtype=torch.float64, device=dev)
+        self.t_dev = torch.tensor(self.t, **f64)
+        self.sig_dev = torch.tensor(self.sig, **f64)
+        self.rewards = torch.tensor(self.draws.rewards, dtype=torch.float32, device=dev)
+        self.txt1 = torch.tensor(self.draws.txt, dtype=self.tdt, device=dev)
+        maxB = W * G
+        self.ws = jg.alloc_bytes(self.model.workspace_bytes(maxB), dev)
+        self.sws = jg.alloc_bytes(jg.signals_workspace_bytes(G, W, self.D), dev)
+        self.gws = jg.alloc_bytes(jg.grad_reduce_workspace_bytes(self.P), dev)
+        self.grad = torch.zeros(self.P, dtype=torch.float32, device=dev)
+        self.out3 = torch.zeros(3, **f64)
+        self.sig_out = dict(logp_new=torch.empty(G, W, **f64), ratio=torch.empty(G, W, **f64),
+                            clipped=torch.empty(G, W, dtype=torch.uint8, device=dev), adv_out=torch.empty(G, **f64))
+        self.cot = torch.empty(2 * G, self.D, dtype=torch.float32, device=dev)
+        self.s = torch.empty(G, W, self.D, dtype=torch.float32, device=dev)
+
+    # rows of a window's forward: JAGG = [z_0 of each sample; z_{W-1} of each sample],
+    # exact = (sample, step) pairs in sample-major order, matching s [G, W, D]
+    def rows(self, z_win, w, jagg):
+        G, W = self.wl.G, self.wl.W
+        tw = self.t[w * W:(w + 1) * W]
+        if jagg:
+            z = torch.cat([z_win[:, 0], z_win[:, W - 1]], 0)
+            t = np.concatenate([np.full(G, tw[0]), np.full(G, tw[W - 1])])
+        else:
+            z = z_win.reshape(G * W, *self.shape)
+            t = np.tile(tw, G)
+        return z.to(self.tdt).contiguous(), torch.tensor(t, dtype=torch.float32, device=self.dev)
+
+    def txt_rows(self, B):
+        return self.txt1.unsqueeze(0).expand(B, -1, -1).contiguous()
+
+    def rollout(self):
+        """Synthetic trajectories from the model itself (theta_old = theta): Euler-Maruyama
+        steps z_{j+1} = z_j + v dt + sigma xi, old log-probs = rollout log-probs + delta."""
+        jg, wl, dev = self.jg, self.wl, self.dev
+        G, T, W = wl.G, wl.T, wl.W
+        z = torch.zeros(G, T + 1, self.D, dtype=torch.float32, device=dev)
+        z[:, 0] = torch.tensor(self.draws.z0.reshape(-1), dtype=torch.float32, device=dev)
+        xi = torch.tensor(self.draws.xi.reshape(G, T, -1), dtype=torch.float32, device=dev)
+        v_all = torch.empty(G, T, self.D, dtype=self.tdt, device=dev)
+        txt = self.txt_rows(G)
+        v = torch.empty(G, *self.shape, dtype=self.tdt, device=dev)
+        for j in range(T):
+            zin = z[:, j].reshape(G, *self.shape).to(self.tdt).contiguous()
+            tin = torch.full((G,), float(self.t[j]), dtype=torch.float32, device=dev)
+            jg.dit_forward_save(self.model, zin, tin, txt, v, ws=self.ws)
+            v_all[:, j] = v.reshape(G, -1)
+            z[:, j + 1] = z[:, j] + v.reshape(G, -1).float() * float(self.t[j + 1] - self.t[j]) + float(self.sig[j]) * xi[:, j]
+        self.z = z
+        self.v_all = v_all
+        self.v_win = [self.v_all[:, w * W:(w + 1) * W].contiguous() for w in range(self.nw)]
+        self.z_win = [self.z[:, w * W:w * W + W + 1].contiguous() for w in range(self.nw)]
+        # old log-probs: the rollout's log-probs (from the library's own log-prob) + delta
+        self.logp_old = torch.zeros(G, T, dtype=torch.float64, device=dev)
+        zero = torch.zeros(G, W, dtype=torch.float64, device=dev)
+        for w in range(self.nw):
+            self.signals(w, zero, cot=False)
+            self.logp_old[:, w * W:(w + 1) * W] = self.sig_out["logp_new"]
+        self.logp_old += torch.tensor(self.draws.delta, dtype=torch.float64, device=dev)
+        self.lpo_win = [self.logp_old[:, w * W:(w + 1) * W].contiguous() for w in range(self.nw)]
+        torch.cuda.synchronize()
+
+    def signals(self, w, logp_old, cot=True, s=False):
+        W = self.wl.W
+        self.jg.grpo_step_signals(self.v_win[w], self.z_win[w],
+                                  self.t_dev[w * W:w * W + W + 1], self.sig_dev[w * W:(w + 1) * W], logp_old, self.rewards,
+                                  self.wl.clip_eps, self.wl.adv_clip, self.wl.adv_eps, self.scale, ws=self.sws,
+                                  cot_out=self.cot if cot else None, s_out=self.s if s else None, **self.sig_out)
+
+    def forward_saves(self, jagg):
+        """Phase 1 endpoints (JAGG) or every step (exact) of each window, with saves."""
+        wl = self.wl
+        B = 2 * wl.G if jagg else wl.W * wl.G
+        arenas = []
+        for w in range(self.nw):
+            z_win = self.z[:, w * wl.W:(w + 1) * wl.W].reshape(wl.G, wl.W, *self.shape)
+            zr, tr = self.rows(z_win, w, jagg)
+            saved = self.jg.alloc_bytes(self.model.saved_bytes(B), self.dev)
+            v = torch.empty_like(zr)
+            self.jg.dit_forward_save(self.model, zr, tr, self.txt_rows(B), v, saved=saved, ws=self.ws)
+            arenas.append(saved)
+        torch.cuda.synchronize()
+        return arenas, B
+
+    def step(self, arenas, B, jagg, routes):
+        """Phases 2-4 over every window, then the gradient's squared norm."""
+        jg = self.jg
+        for w in range(self.nw):
+            if jagg and routes[w]:
+                self.signals(w, self.lpo_win[w], cot=True)
+                jg.dit_joint_vjp(self.model, arenas[w], B, self.cot, self.grad, self.ws)
+            else:
+                self.signals(w, self.lpo_win[w], cot=False, s=True)
+                jg.dit_joint_vjp(self.model, arenas[w], B, self.s, self.grad, self.ws)
+        jg.grad_reduce(self.grad, None, out3=self.out3, ws=self.gws)
+
+
+def time_steps(fn, steps, warmup, ws, use_graph):
+    """W warm-up calls, then K calls timed with CUDA events on the launching stream."""
+    stream = torch.cuda.current_stream()
+    graph = None
+    if use_graph:
+        side = torch.cuda.Stream()
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            fn()
+        stream.wait_stream(side)
+        torch.cuda.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            fn()
+        run = graph.replay
+    else:
+        run = fn
+    for _ in range(warmup):
+        run()
+    torch.cuda.synchronize()
+    barrier(ws)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        run()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier(ws)
+    return e0.elapsed_time(e1) / steps, graph
+
+
+# ----------------------------------------------------------------------------- oracle legs
+def oracle_window_sample(wl, G_sample):
+    """One JAGG window of the workload on the float64 oracle for G_sample samples:
+    the endpoint forwards with their caches, the step signals of the window (on synthetic
+    v-hat), the t-weighted aggregation and the joint VJP.  Returns (seconds, traj-steps)."""
+    from oracle import dit, grpo
+    params = synth.make_params(wl)
+    model = dit.Backbone(wl, params)
+    rng = np.random.Generator(np.random.PCG64(5))
+    W = wl.W
+    shape = (wl.in_channels, wl.latent_h, wl.latent_w)
+    t = synth.time_grid(wl.T, wl.shift)[:W + 1]
+    sig = synth.sigma_schedule(t, wl.eta)
+    z = synth.storage_round(rng.standard_normal((G_sample, W + 1) + shape), wl.dtype)
+    v = synth.storage_round(rng.standard_normal((G_sample, W) + shape), wl.dtype)
+    lpo = np.zeros((G_sample, W))
+    txt = np.broadcast_to(synth.draw_group(wl).txt, (2 * G_sample, wl.txt_len, wl.txt_dim))
+    t0 = time.perf_counter()
+    s, _, _, _ = grpo.step_signals(v.reshape(G_sample, W, -1), z.reshape(G_sample, W + 1, -1), t, sig, lpo,
+                                   grpo.advantages(rng.standard_normal(G_sample)), wl.clip_eps, 1.0 / (wl.G * wl.T))
+    cot = grpo.aggregate(s, t[:W]).reshape((2 * G_sample,) + shape)
+    zr = np.concatenate([z[:, 0], z[:, W - 1]])
+    tr = np.concatenate([np.full(G_sample, t[0]), np.full(G_sample, t[W - 1])])
+    _, cache = model.forward(zr, tr, txt)
+    model.vjp(cache, cot)
+    return time.perf_counter() - t0, G_sample * W
+
+
+def threads_used():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads") for i in threadpool_info() if i.get("internal_api") in ("openblas", "mkl", "blis")]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    return os.cpu_count() or 1
+
+
+def run_reference(args, ws, rank):
+    if rank != 0:
+        return
+    wl = synth.WORKLOADS[args.workload]
+    G_sample = 2
+    for _ in range(args.warmup):
+        oracle_window_sample(wl, G_sample)
+    tot, units = 0.0, 0
+    for _ in range(args.steps):
+        sec, u = oracle_window_sample(wl, G_sample)
+        tot += sec
+        units += u
+    value = units / tot
+    sample = (f"one JAGG window (W={wl.W}) of {wl.name} for {G_sample} of the G={wl.G} samples per step: "
+              f"endpoint forwards with caches, step signals, aggregation, joint VJP over {2 * G_sample} rows")
+    cores = threads_used()
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * tot / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": wl.name},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------- main leg
+def run_gpu(args, ws, rank):
+    import paper_2607_17572_gb300 as jg
+    dev = torch.device("cuda", torch.cuda.current_device())
+    wl = synth.WORKLOADS[args.workload]
+    b = Bench(wl, dev)
+    b.rollout()
+    routes, _ = jg.jagg_route(b.nw, wl.jagg_frac)
+    arenas, B = b.forward_saves(jagg=True)
+    use_graph = not args.no_graph
+    units = wl.G * wl.T
+
+    # ---- JAGG path: timed region
+    n0 = jg.launch_count()
+    b.step(arenas, B, True, routes)
+    torch.cuda.synchronize()
+    launches_per_step = jg.launch_count() - n0
+    assert jg.device_status() == 0, "device status set during the JAGG step"
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        ms, graph = time_steps(lambda: b.step(arenas, B, True, routes), args.steps, args.warmup, ws, use_graph)
+    clocks = clk.summary()
+    ms = max_over_ranks(ms, ws)
+    value = ws * units / (ms / 1000.0)
+
+    # ---- per-family device time of the same step (events around each launch, eager)
+    jg.profile_enable(True)
+    for _ in range(args.steps):
+        b.step(arenas, B, True, routes)
+    prof = jg.profile_read()
+    jg.profile_enable(False)
+    burst, sustained, hbm, src = peaks()
+    fam = {k: v for k, v in prof.items() if v["launches"]}
+    gt = fam.get("gemm_tcgen05", {"launches": 0, "ms": 0.0, "flops": 0.0})
+    achieved = gt["flops"] / (gt["ms"] / 1000.0) / 1e12 if gt["ms"] > 0 else 0.0
+    roofline = {"bound": "tensor", "achieved": achieved, "peak": sustained, "unit": "TFLOP/s",
+                "frac": achieved / sustained, "traffic": None,
+                "kernel": "gemm_tcgen05 (all dense products of the joint VJP)",
+                "peak_source": f"bf16_tflops_sustained of {src} peaks",
+                "launches_per_step": gt["launches"] / args.steps,
+                "flops_per_launch": gt["flops"] / max(gt["launches"], 1),
+                "ms_per_launch": gt["ms"] / max(gt["launches"], 1)}
+    step_flops = sum(v["flops"] for k, v in fam.items() if k != "gemm_simt") / args.steps
+    families = {k: {"launches_per_step": v["launches"] / args.steps, "ms_per_step": v["ms"] / args.steps,
+                    "tflops": (v["flops"] / (v["ms"] / 1000.0) / 1e12) if v["ms"] > 0 else None}
+                for k, v in fam.items()}
+    del graph
+
+    out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+           "config": {"workload": (f"{wl.name}: DiT {wl.depth} blocks d={wl.hidden} h={wl.heads} mlp={wl.mlp}, "
+                                   f"{wl.n_img} img + {wl.txt_len} txt tokens, G={wl.G}, T={wl.T}, W={wl.W}, "
+                                   f"jagg_frac={wl.jagg_frac}"),
+                      "rows_per_vjp": B, "windows": b.nw, "cuda_graph": use_graph,
+                      "l2": "inputs larger than L2 (saved activations %.1f GB per step)" % (
+                          sum(a.numel() for a in arenas) / 1e9),
+                      "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU"},
+           "roofline": roofline, "algorithmic_tflops_per_step": step_flops / 1e12,
+           "step_tflops_per_s": step_flops / (ms / 1000.0) / 1e12, "families": families,
+           "gpu_launches": launches_per_step * args.steps, "clocks": clocks}
+    del arenas
+    torch.cuda.empty_cache()
+
+    if not args.quick:
+        # ---- exact per-step path (jagg_frac = 0)
+        arenas_f, Bf = b.forward_saves(jagg=False)
+        b.grad.zero_()
+        ms_f, graph = time_steps(lambda: b.step(arenas_f, Bf, False, [0] * b.nw), args.steps, args.warmup, ws,
+                                 use_graph)
+        ms_f = max_over_ranks(ms_f, ws)
+        out["full_w"] = {"value": ws * units / (ms_f / 1000.0), "unit": UNIT, "ms_per_step": ms_f,
+                         "rows_per_vjp": Bf}
+        out["jagg_speedup_vs_full_w"] = ms_f / ms
+        out["ideal_speedup"] = wl.W / 2
+        del graph, arenas_f
+        torch.cuda.empty_cache()
+        if not args.no_e2e:
+            out["e2e"] = run_e2e(b, args, ws, routes)
+        if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+            G_sample = 2
+            sec, u = oracle_window_sample(wl, G_sample)
+            out["cpu_baseline"] = {"value": u / sec, "unit": UNIT, "cores": threads_used(), "kind": "oracle",
+                                   "sample": (f"one JAGG window (W={wl.W}) of {wl.name} for {G_sample} samples: "
+                                              f"endpoint forwards with caches, step signals, aggregation, joint "
+                                              f"VJP over {2 * G_sample} rows; {sec:.1f} s")}
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+
+
+def run_e2e(b, args, ws, routes):
+    """The update stage through the public API from pinned host buffers: per step, copy the
+    group's trajectory, old log-probs and rewards to the device, run every window's Phase 1
+    forwards (endpoints saved, middle steps without saves) and Phases 2-4, and copy the
+    new log-probs and the gradient norm back."""
+    jg, wl, dev = b.jg, b.wl, b.dev
+    G, W = wl.G, wl.W
+    h_z = b.z.cpu().pin_memory()
+    h_lpo = b.logp_old.cpu().pin_memory()
+    h_rw = b.rewards.cpu().pin_memory()
+    h_lpn = torch.empty(G, wl.T, dtype=torch.float64).pin_memory()
+    h_out3 = torch.empty(3, dtype=torch.float64).pin_memory()
+    B = 2 * G
+    arenas = [jg.alloc_bytes(b.model.saved_bytes(B), dev) for _ in range(b.nw)]
+    v_mid = torch.empty(G * (W - 2), *b.shape, dtype=b.tdt, device=dev)
+    v_end = torch.empty(B, *b.shape, dtype=b.tdt, device=dev)
+    txt_mid, txt_end = b.txt_rows(G * (W - 2)), b.txt_rows(B)
+
+    def step():
+        b.z.copy_(h_z, non_blocking=True)
+        b.logp_old.copy_(h_lpo, non_blocking=True)
+        b.rewards.copy_(h_rw, non_blocking=True)
+        for w in range(b.nw):
+            b.z_win[w].copy_(b.z[:, w * W:w * W + W + 1])
+            b.lpo_win[w].copy_(b.logp_old[:, w * W:(w + 1) * W])
+            z_win = b.z[:, w * W:(w + 1) * W].reshape(G, W, *b.shape)
+            zr, tr = b.rows(z_win, w, True)
+            jg.dit_forward_save(b.model, zr, tr, txt_end, v_end, saved=arenas[w], ws=b.ws)
+            zm = z_win[:, 1:W - 1].reshape(G * (W - 2), *b.shape).to(b.tdt).contiguous()
+            tm = torch.tensor(np.tile(b.t[w * W + 1:w * W + W - 1], G), dtype=torch.float32, device=dev)
+            jg.dit_forward_save(b.model, zm, tm, txt_mid, v_mid, ws=b.ws)
+            vw = b.v_win[w]
+            vw[:, 0].copy_(v_end[:G].reshape(G, -1))
+            vw[:, W - 1].copy_(v_end[G:].reshape(G, -1))
+            vw[:, 1:W - 1].copy_(v_mid.reshape(G, W - 2, -1))
+            b.signals(w, b.lpo_win[w], cot=True)
+            h_lpn[:, w * W:(w + 1) * W].copy_(b.sig_out["logp_new"], non_blocking=True)
+            jg.dit_joint_vjp(b.model, arenas[w], B, b.cot, b.grad, b.ws)
+        jg.grad_reduce(b.grad, None, out3=b.out3, ws=b.gws)
+        h_out3.copy_(b.out3, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+
+    steps = max(2, args.steps // 2)
+    for _ in range(max(1, args.warmup // 2)):
+        step()
+    barrier(ws)
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        step()
+    sec = max_over_ranks((time.perf_counter() - t0) / steps, ws)
+    h2d = h_z.numel() * 4 + h_lpo.numel() * 8 + h_rw.numel() * 4
+    d2h = h_lpn.numel() * 8 + h_out3.numel() * 8
+    return {"value": ws * wl.G * wl.T / sec, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "ms_per_step": 1000 * sec, "steps": steps,
+            "includes": "Phase 1 forwards (2G rows saved + (W-2)G rows unsaved per window), signals, joint VJP"}
+
+
+def main():
+    args = parse()
+    ws, rank = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, ws, rank)
+    else:
+        run_gpu(args, ws, rank)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

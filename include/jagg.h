@@ -64,6 +64,25 @@ const char* jagg_last_error(void);
 /* Reads the device status word (synchronises the device); clears it when `clear` != 0. */
 int jagg_device_status(unsigned* status_out, int clear);
 
+/* Number of kernels the library has launched in this process (host-side counter). */
+int64_t jagg_launch_count(void);
+
+/* Kernel timing by family.  jagg_profile_enable(1) clears earlier records and starts
+ * bracketing every dense-product and attention launch with CUDA events on its stream
+ * (this adds two event records per launch); jagg_profile_enable(0) stops.
+ * jagg_profile_read synchronises the device and fills up to `cap` entries, one per
+ * family: launches, summed device milliseconds, summed algorithmic FLOPs (2 per
+ * multiply-add of the products the operation defines) and algorithmic bytes. */
+typedef struct jagg_profile_stat {
+  char family[32];
+  int64_t launches;
+  double ms;
+  double flops;
+  double bytes;
+} jagg_profile_stat;
+int jagg_profile_enable(int on);
+int jagg_profile_read(jagg_profile_stat* out, int cap, int* n_out);
+
 /* ------------------------------------------------------------------ backbone
  * The velocity network v_theta(z, t, txt).  The paper trains Flux and Qwen-Image
  * (Sec. 4) without describing them; the library implements the pinned DiT / MMDiT of

@@ -60,6 +60,11 @@ class GemmDesc(ctypes.Structure):
                 ("force_simt", ctypes.c_int32)]
 
 
+class ProfileStat(ctypes.Structure):
+    _fields_ = [("family", ctypes.c_char * 32), ("launches", ctypes.c_int64), ("ms", ctypes.c_double),
+                ("flops", ctypes.c_double), ("bytes", ctypes.c_double)]
+
+
 _lib = None
 _P = ctypes.c_void_p
 _I = ctypes.c_int
@@ -70,6 +75,9 @@ _D = ctypes.c_double
 _SIGNATURES = {
     "jagg_last_error": (ctypes.c_char_p, []),
     "jagg_device_status": (_I, [ctypes.POINTER(ctypes.c_uint), _I]),
+    "jagg_launch_count": (_I64, []),
+    "jagg_profile_enable": (_I, [_I]),
+    "jagg_profile_read": (_I, [ctypes.POINTER(ProfileStat), _I, ctypes.POINTER(_I)]),
     "jagg_param_count": (_I64, [ctypes.POINTER(Config)]),
     "jagg_param_tensor_count": (_I, [ctypes.POINTER(Config)]),
     "jagg_param_info": (_I, [ctypes.POINTER(Config), _I, ctypes.c_char_p, _SZ, ctypes.POINTER(_I64),
@@ -277,6 +285,23 @@ def grad_reduce(a, b=None, alpha: float = 1.0, acc=None, out3=None, ws=None, str
     _need_cuda(a, b, acc, out3, ws)
     _check(lib().grad_reduce(_ptr(a), _ptr(b), a.numel(), float(alpha), _ptr(acc), _ptr(out3), _ptr(ws),
                              0 if ws is None else ws.numel(), _stream(stream)), "grad_reduce")
+
+
+def launch_count() -> int:
+    return lib().jagg_launch_count()
+
+
+def profile_enable(on: bool):
+    _check(lib().jagg_profile_enable(1 if on else 0), "jagg_profile_enable")
+
+
+def profile_read() -> dict:
+    """{family: {"launches", "ms", "flops", "bytes"}} (synchronises the device)."""
+    arr = (ProfileStat * 16)()
+    n = _I()
+    _check(lib().jagg_profile_read(arr, 16, ctypes.byref(n)), "jagg_profile_read")
+    return {arr[i].family.decode(): dict(launches=arr[i].launches, ms=arr[i].ms, flops=arr[i].flops,
+                                         bytes=arr[i].bytes) for i in range(n.value)}
 
 
 def device_status(clear: bool = True) -> int:

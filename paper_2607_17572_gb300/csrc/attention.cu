@@ -478,8 +478,12 @@ int fwd_tc(const AttnArgs& a, cudaStream_t s) {
     set = true;
   }
   dim3 grid(ceil_div(a.N, TILE), a.B * a.heads);
+  const int tok = prof_start(s);
   fa_fwd_kernel<D><<<grid, 128, smem, s>>>(a);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
+  // QK^T and PV: 2 N^2 d multiply-adds per (sequence, head)
+  prof_stop(tok, s, PROF_ATTN_FWD, 4.0 * a.B * a.heads * (double)a.N * a.N * D,
+            2.0 * a.B * (double)a.N * a.heads * D * 4);
   return JAGG_OK;
 }
 template <int D>
@@ -491,8 +495,13 @@ int bwd_tc(const AttnBwdArgs& a, cudaStream_t s) {
     set = true;
   }
   dim3 grid(ceil_div(a.f.N, TILE), a.f.B * a.f.heads);
+  const int tok = prof_start(s);
   fa_bwd_kernel<D><<<grid, 128, smem, s>>>(a);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
+  // dV = P^T dO, dP = dO V^T, dQ = dS K, dK = dS^T Q: 4 N^2 d multiply-adds per (sequence,
+  // head); the recomputation of S is not counted
+  prof_stop(tok, s, PROF_ATTN_BWD, 8.0 * a.f.B * a.f.heads * (double)a.f.N * a.f.N * D,
+            2.0 * a.f.B * (double)a.f.N * a.f.heads * D * 7);
   return JAGG_OK;
 }
 
@@ -500,14 +509,14 @@ template <int D>
 int fwd_simt(const AttnArgs& a, cudaStream_t s) {
   dim3 grid(ceil_div(a.N, 64), a.B * a.heads);
   attn_fwd_simt<D><<<grid, 64, 0, s>>>(a);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 template <int D>
 int bwd_simt(const AttnBwdArgs& a, cudaStream_t s) {
   dim3 grid(ceil_div(a.f.N, 64), a.f.B * a.f.heads);
   attn_bwd_simt<D><<<grid, 64, 0, s>>>(a);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 
@@ -539,7 +548,7 @@ int attention_bwd(const AttnBwdArgs& a, cudaStream_t s) {
   JAGG_CUDA_TRY(cudaMemsetAsync(a.dq_acc, 0, sizeof(float) * (size_t)f.B * f.N * f.heads * f.dh, s));
   const int64_t warps = (int64_t)f.B * f.N * f.heads;
   rowdot_kernel<<<(int)((warps * 32 + 255) / 256), 256, 0, s>>>(a);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   int st = JAGG_ERR_UNSUPPORTED;
   if (f.dtype == JAGG_DTYPE_BF16 && f.dh == 64)
     st = bwd_tc<64>(a, s);
@@ -559,7 +568,7 @@ int attention_bwd(const AttnBwdArgs& a, cudaStream_t s) {
   }
   const int64_t total = (int64_t)f.B * f.N * f.heads * f.dh;
   dq_store_kernel<<<(int)std::min<int64_t>((total + 255) / 256, 1 << 20), 256, 0, s>>>(a);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 

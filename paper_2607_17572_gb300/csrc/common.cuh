@@ -99,7 +99,23 @@ void set_last_error(const char* fmt, ...);
 int cuda_status(cudaError_t e, const char* where);
 int sm_count();
 
+// ------------------------------------------------------------------ launch accounting
+// Every kernel launch of the library is counted (jagg_launch_count).  While profiling is
+// enabled (jagg_profile_enable), the dense-product and attention launches are also
+// bracketed by CUDA events on their stream and attributed to a kernel family with their
+// algorithmic FLOPs and bytes.
+void count_launch();
+enum ProfFamily : int { PROF_GEMM_TC = 0, PROF_GEMM_SIMT, PROF_ATTN_FWD, PROF_ATTN_BWD, PROF_FAMILIES };
+int prof_start(cudaStream_t s);  // returns a token, or -1 when profiling is off
+void prof_stop(int token, cudaStream_t s, int family, double flops, double bytes);
+
 }  // namespace jagg
+
+#define JAGG_LAUNCHED()                                                         \
+  do {                                                                          \
+    JAGG_CUDA_TRY(cudaGetLastError());                                          \
+    ::jagg::count_launch();                                                     \
+  } while (0)
 
 #define JAGG_CUDA_TRY(expr)                                                     \
   do {                                                                          \

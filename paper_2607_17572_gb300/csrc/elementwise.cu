@@ -440,40 +440,40 @@ int launch_patchify(const void* z, int in_f32, void* xp, int out_f32, int dtype,
   (void)dtype;
   const int64_t n = (int64_t)B * C * H * W;
   patchify_kernel<<<grid_for(n, 256), 256, 0, s>>>(z, in_f32, xp, out_f32, B, C, H, W, p);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 int launch_unpatchify(const void* xp, void* z, int dtype, int B, int C, int H, int W, int p, cudaStream_t s) {
   const int64_t n = (int64_t)B * C * H * W;
   unpatchify_kernel<<<grid_for(n, 256), 256, 0, s>>>(xp, z, dtype == JAGG_DTYPE_F32, B, C, H, W, p);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 int launch_timestep_embedding(const float* t, float* phi, int B, int dim, cudaStream_t s) {
   temb_kernel<<<grid_for((int64_t)B * dim / 2, 256), 256, 0, s>>>(t, phi, B, dim);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 int launch_silu(const float* in, float* out, int64_t n, cudaStream_t s) {
   silu_kernel<<<grid_for(n, 256), 256, 0, s>>>(in, out, n);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 int launch_mul_silu_grad(float* g, const float* x, int64_t n, cudaStream_t s) {
   mul_silu_grad_kernel<<<grid_for(n, 256), 256, 0, s>>>(g, x, n);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 int launch_add_pos_embed(float* h, int B, int rows_per_seq, int row0, int gh, int gw, int d, cudaStream_t s) {
   pos_embed_kernel<<<grid_for((int64_t)B * gh * gw * d, 256), 256, 0, s>>>(h, B, rows_per_seq, row0, gh, gw, d);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 int launch_ln_mod_fwd(const LnModFwd& a, cudaStream_t s) {
   JAGG_CHECK_ARG(a.d % 4 == 0 && a.d <= 128 * LN_MAXV, "ln_mod: hidden %d unsupported", a.d);
   const int warps = 8;
   ln_mod_fwd_kernel<<<ceil_div(a.M, warps), warps * 32, 0, s>>>(a);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 int launch_ln_gate_bwd(const LnGateBwd& a, cudaStream_t s) {
@@ -482,21 +482,21 @@ int launch_ln_gate_bwd(const LnGateBwd& a, cudaStream_t s) {
   const int seqs = a.M / a.rows_per_seq;
   const int chunks = ceil_div(a.rows_per_seq, LNB_ROWS);
   ln_gate_bwd_kernel<<<seqs * chunks, LNB_THREADS, 0, s>>>(a);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 int launch_colsum(const void* X, int x_f32, int dtype, int rows, int cols, int64_t ld, float* db, cudaStream_t s) {
   (void)dtype;
   dim3 grid(ceil_div(cols, 256), ceil_div(rows, CS_ROWS));
   colsum_kernel<<<grid, 256, 0, s>>>(X, x_f32, rows, cols, ld, db);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 int launch_gather_rows(const float* in, int64_t ld_in, int seg, int seg_off, int64_t seg_stride, void* out,
                        int dtype, int rows, int cols, cudaStream_t s) {
   gather_rows_kernel<<<grid_for((int64_t)rows * cols, 256), 256, 0, s>>>(in, ld_in, seg, seg_off, seg_stride, out,
                                                                          dtype == JAGG_DTYPE_F32, rows, cols);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 int launch_copy_rows(const void* in, int64_t ld_in, int in_seg, int in_seg_off, int64_t in_seg_stride, void* out,
@@ -511,7 +511,7 @@ int launch_copy_rows(const void* in, int64_t ld_in, int in_seg, int in_seg_off, 
     copy_rows_kernel<uint16_t><<<g, 256, 0, s>>>(static_cast<const uint16_t*>(in), ld_in, in_seg, in_seg_off,
                                                 in_seg_stride, static_cast<uint16_t*>(out), ld_out, out_seg,
                                                 out_seg_off, out_seg_stride, rows, cols);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 int launch_attn_rowdot(const void* dO, const void* O, int64_t ld, float* Dv, int B, int N, int heads, int dh,
@@ -519,20 +519,20 @@ int launch_attn_rowdot(const void* dO, const void* O, int64_t ld, float* Dv, int
   const int64_t warps = (int64_t)B * N * heads;
   attn_rowdot_kernel<<<grid_for(warps * 32, 256), 256, 0, s>>>(dO, O, ld, Dv, B, N, heads, dh,
                                                               dtype == JAGG_DTYPE_F32);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 int launch_qk_norm_rope_fwd(const QkNormRope& a, cudaStream_t s) {
   JAGG_CHECK_ARG(a.d / a.heads <= 128, "qk_norm: head dim too large");
   const int64_t warps = (int64_t)a.M * a.heads;
   qk_norm_rope_fwd_kernel<<<grid_for(warps * 32, 256), 256, 0, s>>>(a);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 int launch_qk_norm_rope_bwd(const QkNormRopeBwd& a, cudaStream_t s) {
   const int64_t warps = (int64_t)a.f.M * a.f.heads;
   qk_norm_rope_bwd_kernel<<<grid_for(warps * 32, 256), 256, 0, s>>>(a);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 

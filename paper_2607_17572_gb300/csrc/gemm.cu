@@ -552,8 +552,11 @@ int launch_tc(const GemmArgs& g, cudaStream_t stream) {
                                        Cfg::SMEM_BYTES));
     attr_set = true;
   }
+  const int tok = prof_start(stream);
   gemm_tc_kernel<BN, A_MN, B_MN><<<grid, TC_THREADS, Cfg::SMEM_BYTES, stream>>>(ta, tb, p);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
+  prof_stop(tok, stream, PROF_GEMM_TC, 2.0 * g.M * g.N * g.K,
+            2.0 * ((double)g.M * g.K + (double)g.N * g.K) + (double)g.M * g.N * (g.c_dtype == JAGG_DTYPE_F32 ? 4 : 2));
   return JAGG_OK;
 }
 
@@ -603,11 +606,13 @@ int gemm_simt(const GemmArgs& g, cudaStream_t stream) {
   }
   p.splits = splits;
   dim3 grid(tiles, splits);
+  const int tok = prof_start(stream);
   if (skinny)
     gemm_simt_kernel<16, 64><<<grid, 256, 0, stream>>>(p);
   else
     gemm_simt_kernel<64, 64><<<grid, 256, 0, stream>>>(p);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
+  prof_stop(tok, stream, PROF_GEMM_SIMT, 2.0 * g.M * g.N * g.K, 0.0);
   return JAGG_OK;
 }
 

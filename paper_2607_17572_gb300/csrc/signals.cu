@@ -275,21 +275,21 @@ extern "C" int grpo_step_signals(const void* v_hat, int v_dtype, const float* z,
   float* coef = reinterpret_cast<float*>(partial + (int64_t)G * W * chunks);
   const int vf32 = v_dtype == JAGG_DTYPE_F32;
   advantage_kernel<<<1, 32, 0, stream>>>(rewards, G, adv_eps, adv_clip, adv_out);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   resid_norm_kernel<<<dim3(chunks, G * W), SIG_THREADS, 0, stream>>>(v_hat, vf32, z, t, W, D, partial);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   logprob_kernel<<<ceil_div((int64_t)G * W, 128), 128, 0, stream>>>(partial, chunks, t, sigma, logp_old, adv_out, G,
                                                                      W, D, clip_eps, scale, logp_new, ratio, clipped,
                                                                      coef);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   if (s_out || cot_out) {
     if (cot_out) {
       check_alpha_kernel<<<1, 32, 0, stream>>>(t, W);
-      JAGG_CUDA_TRY(cudaGetLastError());
+      JAGG_LAUNCHED();
     }
     const int gx = ceil_div(D, (int64_t)SIG_THREADS * 4);
     apply_kernel<<<dim3(gx, G), SIG_THREADS, 0, stream>>>(v_hat, vf32, z, t, coef, G, W, D, s_out, cot_out);
-    JAGG_CUDA_TRY(cudaGetLastError());
+    JAGG_LAUNCHED();
   }
   return JAGG_OK;
 }
@@ -300,9 +300,9 @@ extern "C" int jagg_aggregate(const float* s, const double* t_window, int G, int
   JAGG_CHECK_ARG(G > 0 && G <= 65535 && D > 0, "jagg_aggregate: bad G=%d or D=%lld", G, (long long)D);
   JAGG_CHECK_ARG(W >= 2, "jagg_aggregate: W=%d, the endpoints must differ (W >= 2)", W);
   check_alpha_kernel<<<1, 32, 0, stream>>>(t_window, W);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   aggregate_kernel<<<dim3(ceil_div(D, 256), G), 256, 0, stream>>>(s, t_window, G, W, D, cot);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   return JAGG_OK;
 }
 
@@ -349,10 +349,10 @@ extern "C" int grad_reduce(const float* a, const float* b, int64_t P, float alph
   }
   grad_reduce_kernel<<<GR_BLOCKS, GR_THREADS, 0, stream>>>(a, b, P, alpha, acc,
                                                            out3 ? static_cast<double*>(ws) : nullptr);
-  JAGG_CUDA_TRY(cudaGetLastError());
+  JAGG_LAUNCHED();
   if (out3) {
     grad_reduce_final<<<1, 32, 0, stream>>>(static_cast<const double*>(ws), out3);
-    JAGG_CUDA_TRY(cudaGetLastError());
+    JAGG_LAUNCHED();
   }
   return JAGG_OK;
 }
