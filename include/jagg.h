@@ -184,6 +184,29 @@ int grpo_step_signals(const void* v_hat, int v_dtype, const float* z, const doub
                       double* logp_new, double* ratio, uint8_t* clipped, double* adv_out,
                       void* ws, size_t ws_bytes, cudaStream_t stream);
 
+/* grpo_step_signals for callers that cannot allocate device memory (no counterpart in the
+ * paper: an interface convenience of this library).  Some callers have no way to obtain a
+ * workspace: code that runs where cudaMalloc is not allowed or not wanted, such as an
+ * embedding runtime with a fixed, pre-planned memory budget or a host that owns no
+ * device allocator.  This entry point takes the same arguments as grpo_step_signals
+ * except the workspace, and uses instead a scratch array compiled into the library
+ * (JAGG_SIGNALS_STATIC_SCRATCH_BYTES bytes of device memory, held by every GPU that loads
+ * the library until the process exits).  It allocates nothing.
+ *   - Requests whose scratch need (jagg_signals_workspace_bytes(G, W, D)) exceeds
+ *     JAGG_SIGNALS_STATIC_SCRATCH_BYTES fail with JAGG_ERR_WORKSPACE before any launch.
+ *   - The first call on a device looks up the array's device address (a synchronous
+ *     runtime query); make that first call before any stream capture on that device.
+ *   - Every call shares the one array: calls whose kernels may overlap on the GPU (on
+ *     different streams without ordering between them) race and give wrong results.
+ *     Nothing in the array needs to start at zero; each call overwrites what it reads. */
+#define JAGG_SIGNALS_STATIC_SCRATCH_BYTES (1 << 20)
+int grpo_step_signals_static(const void* v_hat, int v_dtype, const float* z, const double* t,
+                             const double* sigma, const double* logp_old, const float* rewards,
+                             int G, int W, int64_t D, double clip_eps, double adv_clip,
+                             double adv_eps, double scale, float* s_out, float* cot_out,
+                             double* logp_new, double* ratio, uint8_t* clipped, double* adv_out,
+                             cudaStream_t stream);
+
 /* Phase 3 (Eq. alpha, Eq. s_base_corr): alpha_j = (t_0 - t_j) / (t_0 - t_{W-1}),
  *   cot[i]     = sum_j (1 - alpha_j) s[i, j]   (s_base, endpoint j = 0)
  *   cot[G + i] = sum_j alpha_j s[i, j]         (s_corr, endpoint j = W-1)

@@ -91,6 +91,8 @@ _SIGNATURES = {
     "jagg_signals_workspace_bytes": (_I64, [_I, _I, _I64]),
     "grpo_step_signals": (_I, [_P, _I, _P, _P, _P, _P, _P, _I, _I, _I64, _D, _D, _D, _D, _P, _P, _P, _P,
                                _P, _P, _P, _SZ, _P]),
+    "grpo_step_signals_static": (_I, [_P, _I, _P, _P, _P, _P, _P, _I, _I, _I64, _D, _D, _D, _D, _P, _P, _P, _P,
+                                      _P, _P, _P]),
     "jagg_aggregate": (_I, [_P, _P, _I, _I, _I64, _P, _P]),
     "jagg_route": (_I, [_I, _D, _P, _D, _P, _P]),
     "jagg_grad_reduce_workspace_bytes": (_I64, [_I64]),
@@ -256,6 +258,20 @@ def grpo_step_signals(v_hat, z, t, sigma, logp_old, rewards, clip_eps, adv_clip,
                                    G, W, D, clip_eps, adv_clip, adv_eps, scale, _ptr(s_out), _ptr(cot_out),
                                    _ptr(logp_new), _ptr(ratio), _ptr(clipped), _ptr(adv_out), _ptr(ws), ws.numel(),
                                    _stream(stream)), "grpo_step_signals")
+
+
+def grpo_step_signals_static(v_hat, z, t, sigma, logp_old, rewards, clip_eps, adv_clip, adv_eps, scale,
+                             logp_new, ratio, clipped, adv_out, s_out=None, cot_out=None, stream=None):
+    """grpo_step_signals without a workspace: scratch comes from an array compiled into the
+    library, for callers that cannot allocate device memory."""
+    _need_cuda(v_hat, z, t, sigma, logp_old, rewards, logp_new, ratio, clipped, adv_out, s_out, cot_out)
+    G, W = v_hat.shape[0], v_hat.shape[1]
+    D = v_hat[0, 0].numel()
+    vd = DTYPE_BF16 if v_hat.dtype == torch.bfloat16 else DTYPE_F32
+    _check(lib().grpo_step_signals_static(_ptr(v_hat), vd, _ptr(z), _ptr(t), _ptr(sigma), _ptr(logp_old),
+                                          _ptr(rewards), G, W, D, clip_eps, adv_clip, adv_eps, scale, _ptr(s_out),
+                                          _ptr(cot_out), _ptr(logp_new), _ptr(ratio), _ptr(clipped), _ptr(adv_out),
+                                          _stream(stream)), "grpo_step_signals_static")
 
 
 def jagg_aggregate(s, t_window, cot, stream=None):

@@ -9,6 +9,8 @@
 //      elementwise pass writes s_ij = c_ij r_ij and/or the aggregated cotangents
 //      sum_j (1 - alpha_j) s_ij and sum_j alpha_j s_ij (Eq. alpha, Eq. s_base_corr).
 // The v-hat / z tiles of a window are read twice; at the paper's shapes they fit in L2.
+#include <mutex>
+
 #include "common.cuh"
 
 namespace jagg {
@@ -355,4 +357,50 @@ extern "C" int grad_reduce(const float* a, const float* b, int64_t P, float alph
     JAGG_LAUNCHED();
   }
   return JAGG_OK;
+}
+
+// ------------------------------------------------------------------ allocation-free variant
+// Scratch for grpo_step_signals_static: compiled into the library, one copy per device.
+static __device__ __align__(256) unsigned char g_signals_scratch[JAGG_SIGNALS_STATIC_SCRATCH_BYTES];
+
+namespace {
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+void* g_scratch_ptr[kMaxDevices] = {};
+
+// The array's device address for the current device, looked up once per device.  In host
+// code `g_signals_scratch` names a host-side stand-in, never the device memory itself.
+int scratch_for_current_device(void** out) {
+  int dev = 0;
+  JAGG_CUDA_TRY(cudaGetDevice(&dev));
+  JAGG_CHECK_ARG(dev >= 0 && dev < kMaxDevices, "grpo_step_signals_static: device %d out of range", dev);
+  std::lock_guard<std::mutex> lk(g_scratch_mu);
+  if (!g_scratch_ptr[dev]) {
+    void* p = nullptr;
+    JAGG_CUDA_TRY(cudaGetSymbolAddress(&p, g_signals_scratch));
+    g_scratch_ptr[dev] = p;
+  }
+  *out = g_scratch_ptr[dev];
+  return JAGG_OK;
+}
+}  // namespace
+
+extern "C" int grpo_step_signals_static(const void* v_hat, int v_dtype, const float* z, const double* t,
+                                        const double* sigma, const double* logp_old, const float* rewards, int G,
+                                        int W, int64_t D, double clip_eps, double adv_clip, double adv_eps,
+                                        double scale, float* s_out, float* cot_out, double* logp_new,
+                                        double* ratio, uint8_t* clipped, double* adv_out, cudaStream_t stream) {
+  JAGG_CHECK_ARG(G > 0 && W > 0 && D > 0, "grpo_step_signals_static: G=%d W=%d D=%lld must be positive", G, W,
+                 (long long)D);
+  const int64_t need = jagg_signals_workspace_bytes(G, W, D);
+  if (need > (int64_t)JAGG_SIGNALS_STATIC_SCRATCH_BYTES) {
+    set_last_error("grpo_step_signals_static: needs %lld scratch bytes, more than the %d compiled in",
+                   (long long)need, (int)JAGG_SIGNALS_STATIC_SCRATCH_BYTES);
+    return JAGG_ERR_WORKSPACE;
+  }
+  void* scratch = nullptr;
+  JAGG_TRY(scratch_for_current_device(&scratch));
+  return grpo_step_signals(v_hat, v_dtype, z, t, sigma, logp_old, rewards, G, W, D, clip_eps, adv_clip, adv_eps,
+                           scale, s_out, cot_out, logp_new, ratio, clipped, adv_out, scratch,
+                           (size_t)JAGG_SIGNALS_STATIC_SCRATCH_BYTES, stream);
 }
