@@ -25,7 +25,8 @@ extern "C" {
  * A is K-major (A[m*lda + k]) or MN-major (A[k*lda + m]); B is K-major (B[n*ldb + k]) or
  * MN-major (B[k*ldb + n]).  a_dtype/b_dtype/c_dtype/bias_dtype are JAGG_DTYPE_*; C2 and aux
  * follow c_dtype for gelu/dgelu and are f32 for gate.  force_simt selects the SIMT kernel
- * instead of the tcgen05 one (bf16 operands only take the tensor-core path). */
+ * instead of the tcgen05 one (bf16 operands only take the tensor-core path).  For store and
+ * accum, c_trans writes element (m, n) to C[n*ldc + m] and bias_m indexes the bias by m. */
 typedef struct jagg_gemm_desc {
   int32_t M, N, K;
   const void* A;
@@ -49,6 +50,8 @@ typedef struct jagg_gemm_desc {
   int32_t rows_per_seq;
   int32_t split_k;
   int32_t force_simt;
+  int32_t c_trans;
+  int32_t bias_m;
 } jagg_gemm_desc;
 
 int jagg_test_gemm(const jagg_gemm_desc* desc, cudaStream_t stream);

@@ -90,9 +90,10 @@ __global__ void pos_embed_kernel(float* h, int B, int rows_per_seq, int row0, in
     const int half = c / (d / 2);         // 0: row, 1: column
     const int cc = c % (d / 2);
     const int k = cc % q;
-    const double pos = half == 0 ? (double)(n / gw) : (double)(n % gw);
-    const double a = pos * exp(-log(10000.0) * (double)k / (double)q);
-    const float v = (float)(cc < q ? sin(a) : cos(a));
+    // f32 is enough here (|argument| < grid size, error ~1e-6); f64 is slow on this part
+    const float pos = half == 0 ? (float)(n / gw) : (float)(n % gw);
+    const float a = pos * expf(-9.210340371976184f * (float)k / (float)q);  // ln(10000)
+    const float v = cc < q ? sinf(a) : cosf(a);
     h[((int64_t)b * rows_per_seq + row0 + n) * d + c] += v;
   }
 }
@@ -157,113 +158,136 @@ __global__ void ln_mod_fwd_kernel(LnModFwd a) {
   }
 }
 
-// Backward: a block of LNB_THREADS threads walks LNB_ROWS consecutive rows of one sequence;
-// thread t owns columns t, t + LNB_THREADS, ...; per-row statistics via block reductions;
-// per-column partial sums stay in registers and are flushed with atomics at the end.
-constexpr int LNB_THREADS = 256;
-constexpr int LNB_ROWS = 32;
-constexpr int LNB_MAXC = 12;  // d <= 3072
-
-__device__ __forceinline__ float2 block_sum2(float2 v, float2* red) {
-  v.x = warp_sum(v.x);
-  v.y = warp_sum(v.y);
-  const int w = threadIdx.x / 32, l = threadIdx.x & 31;
-  __syncthreads();
-  if (l == 0) red[w] = v;
-  __syncthreads();
-  float2 r = make_float2(0.f, 0.f);
-  for (int i = 0; i < LNB_THREADS / 32; ++i) {
-    r.x += red[i].x;
-    r.y += red[i].y;
+// Backward of LayerNorm + modulation and of the gated residual branch, in two passes:
+//   rows:    one warp per row forms the LayerNorm input-gradient (added to the residual
+//            gradient dh) and dy = gate * dh;
+//   columns: per sequence and column, sums over the sequence's rows give dshift, dscale,
+//            dgate and the bias gradient (sum_m dy = gate * sum_m dh), with coalesced loads.
+__device__ __forceinline__ void load4(const void* p, int64_t i, int is_f32, float (&v)[4]) {
+  if (is_f32) {
+    const float4 f = *reinterpret_cast<const float4*>(static_cast<const float*>(p) + i);
+    v[0] = f.x; v[1] = f.y; v[2] = f.z; v[3] = f.w;
+  } else {
+    const uint2 raw = *reinterpret_cast<const uint2*>(static_cast<const bf16*>(p) + i);
+    const bf16* h = reinterpret_cast<const bf16*>(&raw);
+    v[0] = __bfloat162float(h[0]); v[1] = __bfloat162float(h[1]);
+    v[2] = __bfloat162float(h[2]); v[3] = __bfloat162float(h[3]);
   }
-  return r;
+}
+__device__ __forceinline__ void store4(void* p, int64_t i, int is_f32, const float (&v)[4]) {
+  if (is_f32) {
+    *reinterpret_cast<float4*>(static_cast<float*>(p) + i) = make_float4(v[0], v[1], v[2], v[3]);
+  } else {
+    __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]), b = __floats2bfloat162_rn(v[2], v[3]);
+    uint2 raw;
+    raw.x = *reinterpret_cast<uint32_t*>(&a);
+    raw.y = *reinterpret_cast<uint32_t*>(&b);
+    *reinterpret_cast<uint2*>(static_cast<bf16*>(p) + i) = raw;
+  }
 }
 
-__global__ void __launch_bounds__(LNB_THREADS) ln_gate_bwd_kernel(LnGateBwd a) {
-  __shared__ float2 red[LNB_THREADS / 32];
-  const int chunks_per_seq = (a.rows_per_seq + LNB_ROWS - 1) / LNB_ROWS;
-  const int b = blockIdx.x / chunks_per_seq;
-  const int r0 = b * a.rows_per_seq + (blockIdx.x % chunks_per_seq) * LNB_ROWS;
-  const int r1 = min(r0 + LNB_ROWS, (b + 1) * a.rows_per_seq);
-  const int nc = (a.d + LNB_THREADS - 1) / LNB_THREADS;
+__global__ void ln_gate_rows_kernel(LnGateBwd a) {
+  const int warps = blockDim.x / 32;
+  const int m = blockIdx.x * warps + threadIdx.x / 32;
+  const int lane = threadIdx.x & 31;
+  if (m >= a.M) return;
+  const int d = a.d;
+  const int64_t hr = seg_row(m, a.seg, a.seg_off, a.seg_stride);
+  const int b = m / a.rows_per_seq;
   const int is_f32 = a.dtype == JAGG_DTYPE_F32;
-  float psh[LNB_MAXC], psc[LNB_MAXC], pg[LNB_MAXC], pb[LNB_MAXC];
-  float scl[LNB_MAXC], gt[LNB_MAXC];
+  const int nv = (d + 127) / 128;
+  const float* gate = a.do_gate ? a.gate + (int64_t)b * a.mod_stride : nullptr;
+  if (a.do_ln) {
+    const float mu = a.mean[m], rs = a.rstd[m];
+    const float* sc = a.scale + (int64_t)b * a.mod_stride;
+    float s1 = 0.f, s2 = 0.f;
+    for (int i = 0; i < nv; ++i) {
+      const int c = (i * 32 + lane) * 4;
+      if (c < d) {
+        float dm[4];
+        load4(a.dm, (int64_t)m * d + c, a.dm_f32, dm);
+        const float4 h4 = *reinterpret_cast<const float4*>(a.h + hr * d + c);
+        const float4 s4 = *reinterpret_cast<const float4*>(sc + c);
+        const float hv[4] = {h4.x, h4.y, h4.z, h4.w}, sv[4] = {s4.x, s4.y, s4.z, s4.w};
 #pragma unroll
-  for (int i = 0; i < LNB_MAXC; ++i) {
-    psh[i] = psc[i] = pg[i] = pb[i] = 0.f;
-    const int c = threadIdx.x + i * LNB_THREADS;
-    scl[i] = (a.do_ln && i < nc && c < a.d) ? a.scale[(int64_t)b * a.mod_stride + c] : 0.f;
-    gt[i] = (a.do_gate && i < nc && c < a.d) ? a.gate[(int64_t)b * a.mod_stride + c] : 0.f;
+        for (int e = 0; e < 4; ++e) {
+          const float dxh = dm[e] * (1.f + sv[e]);
+          s1 += dxh;
+          s2 += dxh * (hv[e] - mu) * rs;
+        }
+      }
+    }
+    s1 = warp_sum(s1) / d;
+    s2 = warp_sum(s2) / d;
+    for (int i = 0; i < nv; ++i) {
+      const int c = (i * 32 + lane) * 4;
+      if (c < d) {
+        float dm[4];
+        load4(a.dm, (int64_t)m * d + c, a.dm_f32, dm);
+        const float4 h4 = *reinterpret_cast<const float4*>(a.h + hr * d + c);
+        const float4 s4 = *reinterpret_cast<const float4*>(sc + c);
+        const float4 d4 = *reinterpret_cast<const float4*>(a.dh_in + hr * d + c);
+        const float hv[4] = {h4.x, h4.y, h4.z, h4.w}, sv[4] = {s4.x, s4.y, s4.z, s4.w};
+        float dh[4] = {d4.x, d4.y, d4.z, d4.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float xh = (hv[e] - mu) * rs;
+          dh[e] += rs * (dm[e] * (1.f + sv[e]) - s1 - xh * s2);
+        }
+        *reinterpret_cast<float4*>(a.dh_out + hr * d + c) = make_float4(dh[0], dh[1], dh[2], dh[3]);
+        if (gate) {
+          const float4 g4 = *reinterpret_cast<const float4*>(gate + c);
+          const float dy[4] = {g4.x * dh[0], g4.y * dh[1], g4.z * dh[2], g4.w * dh[3]};
+          store4(a.dy, (int64_t)m * d + c, is_f32, dy);
+        }
+      }
+    }
+  } else if (gate) {
+    for (int i = 0; i < nv; ++i) {
+      const int c = (i * 32 + lane) * 4;
+      if (c < d) {
+        const float4 d4 = *reinterpret_cast<const float4*>(a.dh_in + hr * d + c);
+        const float4 g4 = *reinterpret_cast<const float4*>(gate + c);
+        const float dy[4] = {g4.x * d4.x, g4.y * d4.y, g4.z * d4.z, g4.w * d4.w};
+        store4(a.dy, (int64_t)m * d + c, is_f32, dy);
+      }
+    }
   }
-  for (int m = r0; m < r1; ++m) {
+}
+
+constexpr int LNC_ROWS = 32;
+// grid: (ceil(d / 256), sequences, ceil(rows_per_seq / LNC_ROWS)); one thread per column.
+__global__ void ln_gate_cols_kernel(LnGateBwd a) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  const int b = blockIdx.y;
+  const int r0 = blockIdx.z * LNC_ROWS;
+  if (c >= a.d || r0 >= a.rows_per_seq) return;
+  const int r1 = min(r0 + LNC_ROWS, a.rows_per_seq);
+  const int d = a.d;
+  const int is_f32 = a.dtype == JAGG_DTYPE_F32;
+  const float* dh = a.do_ln ? a.dh_out : a.dh_in;
+  float psh = 0.f, psc = 0.f, pg = 0.f, pdh = 0.f;
+  for (int r = r0; r < r1; ++r) {
+    const int m = b * a.rows_per_seq + r;
     const int64_t hr = seg_row(m, a.seg, a.seg_off, a.seg_stride);
-    float dhv[LNB_MAXC];
     if (a.do_ln) {
-      const float mu = a.mean[m], rs = a.rstd[m];
-      float dm[LNB_MAXC], xh[LNB_MAXC];
-      float2 acc = make_float2(0.f, 0.f);
-#pragma unroll
-      for (int i = 0; i < LNB_MAXC; ++i) {
-        const int c = threadIdx.x + i * LNB_THREADS;
-        dm[i] = xh[i] = 0.f;
-        if (i < nc && c < a.d) {
-          dm[i] = ldx(a.dm, (int64_t)m * a.d + c, a.dm_f32);
-          xh[i] = (a.h[hr * a.d + c] - mu) * rs;
-          const float dxh = dm[i] * (1.f + scl[i]);
-          acc.x += dxh;
-          acc.y += dxh * xh[i];
-          psh[i] += dm[i];
-          psc[i] += dm[i] * xh[i];
-        }
-      }
-      const float2 tot = block_sum2(acc, red);
-      const float m1 = tot.x / a.d, m2 = tot.y / a.d;
-#pragma unroll
-      for (int i = 0; i < LNB_MAXC; ++i) {
-        const int c = threadIdx.x + i * LNB_THREADS;
-        dhv[i] = 0.f;
-        if (i < nc && c < a.d) {
-          const float dxh = dm[i] * (1.f + scl[i]);
-          const float v = a.dh_in[hr * a.d + c] + rs * (dxh - m1 - xh[i] * m2);
-          a.dh_out[hr * a.d + c] = v;
-          dhv[i] = v;
-        }
-      }
-    } else {
-#pragma unroll
-      for (int i = 0; i < LNB_MAXC; ++i) {
-        const int c = threadIdx.x + i * LNB_THREADS;
-        dhv[i] = (i < nc && c < a.d) ? a.dh_in[hr * a.d + c] : 0.f;
-      }
+      const float dmv = ldx(a.dm, (int64_t)m * d + c, a.dm_f32);
+      psh += dmv;
+      psc += dmv * (a.h[hr * d + c] - a.mean[m]) * a.rstd[m];
     }
     if (a.do_gate) {
-#pragma unroll
-      for (int i = 0; i < LNB_MAXC; ++i) {
-        const int c = threadIdx.x + i * LNB_THREADS;
-        if (i < nc && c < a.d) {
-          const float yv = ldx(a.y, (int64_t)m * a.d + c, is_f32);
-          pg[i] += dhv[i] * yv;
-          const float dy = gt[i] * dhv[i];
-          stx(a.dy, (int64_t)m * a.d + c, is_f32, dy);
-          pb[i] += is_f32 ? dy : __bfloat162float(__float2bfloat16_rn(dy));
-        }
-      }
+      const float g = dh[hr * d + c];
+      pg += g * ldx(a.y, (int64_t)m * d + c, is_f32);
+      pdh += g;
     }
   }
-#pragma unroll
-  for (int i = 0; i < LNB_MAXC; ++i) {
-    const int c = threadIdx.x + i * LNB_THREADS;
-    if (i < nc && c < a.d) {
-      if (a.do_ln) {
-        atomicAdd(a.dshift + (int64_t)b * a.dmod_stride + c, psh[i]);
-        atomicAdd(a.dscale + (int64_t)b * a.dmod_stride + c, psc[i]);
-      }
-      if (a.do_gate) {
-        atomicAdd(a.dgate + (int64_t)b * a.dmod_stride + c, pg[i]);
-        if (a.dbias) atomicAdd(a.dbias + c, pb[i]);
-      }
-    }
+  if (a.do_ln) {
+    atomicAdd(a.dshift + (int64_t)b * a.dmod_stride + c, psh);
+    atomicAdd(a.dscale + (int64_t)b * a.dmod_stride + c, psc);
+  }
+  if (a.do_gate) {
+    atomicAdd(a.dgate + (int64_t)b * a.dmod_stride + c, pg);
+    if (a.dbias) atomicAdd(a.dbias + c, a.gate[(int64_t)b * a.mod_stride + c] * pdh);
   }
 }
 
@@ -477,11 +501,13 @@ int launch_ln_mod_fwd(const LnModFwd& a, cudaStream_t s) {
   return JAGG_OK;
 }
 int launch_ln_gate_bwd(const LnGateBwd& a, cudaStream_t s) {
-  JAGG_CHECK_ARG(a.d <= LNB_THREADS * LNB_MAXC, "ln_gate_bwd: hidden %d unsupported", a.d);
+  JAGG_CHECK_ARG(a.d % 4 == 0, "ln_gate_bwd: hidden %d not a multiple of 4", a.d);
   JAGG_CHECK_ARG(a.M % a.rows_per_seq == 0, "ln_gate_bwd: rows not a whole number of sequences");
-  const int seqs = a.M / a.rows_per_seq;
-  const int chunks = ceil_div(a.rows_per_seq, LNB_ROWS);
-  ln_gate_bwd_kernel<<<seqs * chunks, LNB_THREADS, 0, s>>>(a);
+  if (!a.do_ln && !a.do_gate) return JAGG_OK;
+  ln_gate_rows_kernel<<<ceil_div(a.M, 8), 256, 0, s>>>(a);
+  JAGG_LAUNCHED();
+  const dim3 grid(ceil_div(a.d, 256), a.M / a.rows_per_seq, ceil_div(a.rows_per_seq, LNC_ROWS));
+  ln_gate_cols_kernel<<<grid, 256, 0, s>>>(a);
   JAGG_LAUNCHED();
   return JAGG_OK;
 }

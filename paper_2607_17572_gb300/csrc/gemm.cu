@@ -38,6 +38,7 @@ struct EpiParams {
   int remap_rows, remap_offset;
   int64_t remap_stride;
   int vec_ok;  // 8-wide vector accesses are aligned
+  int c_trans, bias_m;
 };
 
 __device__ __forceinline__ float ldv(const void* p, int64_t i, int is_bf16) {
@@ -60,8 +61,8 @@ __device__ __forceinline__ void epi_apply1(const EpiParams& e, int m, int n, flo
   const int64_t cr = epi_crow(e, m);
   switch (e.epi) {
     case EPI_STORE: {
-      float v = acc + (e.bias ? ldv(e.bias, n, e.bias_bf16) : 0.f);
-      stv(e.C, cr * e.ldc + n, e.c_bf16, v);
+      float v = acc + (e.bias ? ldv(e.bias, e.bias_m ? m : n, e.bias_bf16) : 0.f);
+      stv(e.C, e.c_trans ? (int64_t)n * e.ldc + cr : cr * e.ldc + n, e.c_bf16, v);
     } break;
     case EPI_GELU: {
       float u = acc + (e.bias ? ldv(e.bias, n, e.bias_bf16) : 0.f);
@@ -80,7 +81,7 @@ __device__ __forceinline__ void epi_apply1(const EpiParams& e, int m, int n, flo
       stv(e.C, cr * e.ldc + n, e.c_bf16, acc * gelu_tanh_grad(u));
     } break;
     case EPI_ACCUM:
-      atomicAdd(static_cast<float*>(e.C) + cr * e.ldc + n, acc);
+      atomicAdd(static_cast<float*>(e.C) + (e.c_trans ? (int64_t)n * e.ldc + cr : cr * e.ldc + n), acc);
       break;
   }
 }
@@ -500,6 +501,9 @@ EpiParams make_epi(const GemmArgs& g) {
   if (g.bias) ok = ok && al16(g.bias);
   if (g.epi == EPI_GELU || g.epi == EPI_GATE_RESID) ok = ok && (g.ldc2 % 8 == 0) && al16(g.C2);
   if (g.epi == EPI_GATE_RESID || g.epi == EPI_DGELU) ok = ok && (g.ld_aux % 8 == 0) && al16(g.aux);
+  e.c_trans = g.c_trans ? 1 : 0;
+  e.bias_m = g.bias_m ? 1 : 0;
+  if (g.c_trans || g.bias_m) ok = false;  // per-element path for transposed outputs
   e.vec_ok = ok ? 1 : 0;
   return e;
 }
@@ -571,12 +575,9 @@ bool tc_eligible(const GemmArgs& g) {
   if (g.a_dtype != JAGG_DTYPE_BF16 || g.b_dtype != JAGG_DTYPE_BF16) return false;
   auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
   if (!al16(g.A) || !al16(g.B)) return false;
+  // Row pitches must be multiples of 16 bytes.  Extents smaller than a tile are fine:
+  // TMA fills the part of a box outside the tensor with zeros.
   if (g.lda % 8 || g.ldb % 8) return false;
-  if (g.K < TC_BK) return false;
-  if (!g.a_mn && g.M < TC_BM) return false;  // keep every TMA box inside its tensor's outer extent
-  if (!g.b_mn && g.N < 64) return false;
-  if (g.a_mn && g.M < 64) return false;
-  if (g.b_mn && g.N < 64) return false;
   return true;
 }
 

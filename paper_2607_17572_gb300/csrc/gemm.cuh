@@ -45,6 +45,11 @@ struct GemmArgs {
   int remap_offset = 0;
   int64_t remap_stride = 0;
   int split_k = 0;  // EPI_ACCUM only; 0 = choose
+  // EPI_STORE / EPI_ACCUM only: element (m, n) goes to C[n * ldc + m] (a transposed output,
+  // for products formulated as D^T so that the long dimension is M), and the bias is
+  // indexed by m instead of n.
+  bool c_trans = false;
+  bool bias_m = false;
 };
 
 // Launches the product on `stream`.  bf16 x bf16 goes to the tcgen05 tensor-core kernel;

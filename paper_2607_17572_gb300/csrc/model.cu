@@ -197,6 +197,7 @@ struct Saved {
   float* se1;    // [B, d] silu(e1)
   float* c;      // [B, d]
   float* sc;     // [B, d] silu(c)
+  void* sc_b;    // [B, d] silu(c) in the storage type (operand of the modulation products)
   float* mod;    // [B, Lmod]
   std::vector<DitSaved> blk;
   float* h_fin;  // [M, d]
@@ -234,6 +235,7 @@ size_t carve_saved(const jagg_model& m, int B, void* base, bool save, Saved& s) 
   s.se1 = cv.f32((int64_t)B * m.d);
   s.c = cv.f32((int64_t)B * m.d);
   s.sc = cv.f32((int64_t)B * m.d);
+  s.sc_b = cv.take((size_t)B * m.d * m.esz);
   s.mod = cv.f32((int64_t)B * m.T.Lmod);
   const int L = m.cfg.depth;
   s.blk.assign(L, DitSaved());
@@ -266,6 +268,7 @@ struct VjpWs {
   void* dqkv;   // [M, 3d]
   float* attn;  // attention scratch
   float* dmod;  // [B, Lmod]
+  void* dmod_b;  // [B, Lmod] in the storage type
   void* dvt;    // [B*Ni, pd]
   float* dsc;   // [B, d]
   float* de1;   // [B, d]
@@ -284,6 +287,7 @@ size_t carve_vjp_ws(const jagg_model& m, int B, void* base, VjpWs& w) {
   w.dqkv = cv.take(M * 3 * m.d * e);
   w.attn = cv.f32(attention_bwd_scratch_floats(B, m.N, m.heads, m.dh));
   w.dmod = cv.f32((int64_t)B * m.T.Lmod);
+  w.dmod_b = cv.take((size_t)B * m.T.Lmod * m.esz);
   w.dvt = cv.take(Mi * m.pd * e);
   w.dsc = cv.f32((int64_t)B * m.d);
   w.de1 = cv.f32((int64_t)B * m.d);
@@ -381,11 +385,16 @@ int forward_impl(const jagg_model& m, const void* z, const float* t, const void*
     g.C = S.c;
     JAGG_TRY(gemm(g, s));
     JAGG_TRY(launch_silu(S.c, S.sc, (int64_t)B * d, s));
-    g.N = (int)Lm; g.A = S.sc;
-    g.B = W(m, m.T.mod_w);
-    g.bias = W(m, m.T.mod_b);
-    g.C = S.mod; g.ldc = Lm;
-    JAGG_TRY(gemm(g, s));
+    // every modulation at once, as mod^T [Lmod, B] = W_mod [Lmod, d] silu(c)^T: the long
+    // dimension is M, so the product runs on the tensor-core kernel in the storage type
+    JAGG_TRY(launch_gather_rows(S.sc, d, 0, 0, 0, S.sc_b, dt, B, d, s));
+    GemmArgs gm;
+    gm.M = (int)Lm; gm.N = B; gm.K = d;
+    gm.A = W(m, m.T.mod_w); gm.lda = d; gm.a_dtype = dt;
+    gm.B = S.sc_b; gm.ldb = d; gm.b_dtype = dt;
+    gm.bias = W(m, m.T.mod_b); gm.bias_dtype = dt; gm.bias_m = true;
+    gm.C = S.mod; gm.ldc = Lm; gm.c_dtype = JAGG_DTYPE_F32; gm.c_trans = true;
+    JAGG_TRY(gemm(gm, s));
   }
   // blocks
   for (int l = 0; l < c.depth; ++l) {
@@ -553,18 +562,19 @@ int vjp_impl(const jagg_model& m, const void* saved, int B, const float* cot, fl
   JAGG_TRY(gemm(dw_gemm(m, Mt, d, c.txt_dim, w.dxe, d, S.txt, c.txt_dim, grad, m.T.txt_w), s));
   // stacked modulation: dW += dmod^T silu(c), db += sum_b dmod, d silu(c) = dmod W
   JAGG_TRY(launch_colsum(w.dmod, 1, dt, B, (int)Lm, Lm, grad + m.T.mod_b, s));
+  JAGG_TRY(launch_gather_rows(w.dmod, Lm, 0, 0, 0, w.dmod_b, dt, B, (int)Lm, s));
   {
-    GemmArgs g;
+    GemmArgs g;  // grad[Lmod, d] += dmod^T silu(c): both operands MN-major, K = B
     g.M = (int)Lm; g.N = d; g.K = B;
-    g.A = w.dmod; g.lda = Lm; g.a_mn = true; g.a_dtype = JAGG_DTYPE_F32;
-    g.B = S.sc; g.ldb = d; g.b_mn = true; g.b_dtype = JAGG_DTYPE_F32;
+    g.A = w.dmod_b; g.lda = Lm; g.a_mn = true; g.a_dtype = dt;
+    g.B = S.sc_b; g.ldb = d; g.b_mn = true; g.b_dtype = dt;
     g.epi = EPI_ACCUM; g.C = grad + m.T.mod_w; g.ldc = d; g.c_dtype = JAGG_DTYPE_F32;
     JAGG_TRY(gemm(g, s));
-    GemmArgs h;
-    h.M = B; h.N = d; h.K = (int)Lm;
-    h.A = w.dmod; h.lda = Lm; h.a_mn = false; h.a_dtype = JAGG_DTYPE_F32;
-    h.B = W(m, m.T.mod_w); h.ldb = d; h.b_mn = true; h.b_dtype = dt;
-    h.epi = EPI_ACCUM; h.C = w.dsc; h.ldc = d; h.c_dtype = JAGG_DTYPE_F32;
+    GemmArgs h;  // d silu(c)^T [d, B] = W_mod^T [d, Lmod] dmod^T, split over Lmod
+    h.M = d; h.N = B; h.K = (int)Lm;
+    h.A = W(m, m.T.mod_w); h.lda = d; h.a_mn = true; h.a_dtype = dt;
+    h.B = w.dmod_b; h.ldb = Lm; h.b_mn = false; h.b_dtype = dt;
+    h.epi = EPI_ACCUM; h.C = w.dsc; h.ldc = d; h.c_dtype = JAGG_DTYPE_F32; h.c_trans = true;
     JAGG_TRY(gemm(h, s));
   }
   // t-embedding MLP

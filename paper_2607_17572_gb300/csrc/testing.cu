@@ -18,6 +18,8 @@ extern "C" int jagg_test_gemm(const jagg_gemm_desc* d, cudaStream_t stream) {
   g.aux = d->aux; g.ld_aux = d->ld_aux;
   g.gate = d->gate; g.gate_stride = d->gate_stride; g.rows_per_seq = d->rows_per_seq;
   g.split_k = d->split_k;
+  g.c_trans = d->c_trans != 0;
+  g.bias_m = d->bias_m != 0;
   return d->force_simt ? gemm_simt(g, stream) : gemm(g, stream);
 }
 

@@ -52,6 +52,36 @@ def test_tcgen05_gemm_layouts(M, N, K, a_mn, b_mn):
     assert _rel(C, ref) < 1e-5
 
 
+@pytest.mark.parametrize("M,N,K,a_mn,b_mn,epi", [
+    (56832, 16, 768, 0, 0, 0),     # stacked modulation forward: mod^T = W_mod silu(c)^T
+    (768, 16, 56832, 1, 0, 4),     # d silu(c)^T = W_mod^T dmod^T, split over K
+    (56832, 768, 16, 1, 1, 4),     # dW_mod += dmod^T silu(c), K = 16 rows
+    (100, 30, 24, 0, 0, 0),        # every extent below one tile
+    (64, 8, 40, 1, 0, 4)])
+def test_tcgen05_small_extents_and_transposed_output(M, N, K, a_mn, b_mn, epi):
+    """Tiles larger than the tensors (TMA zero-fills the outside), an output written
+    transposed (C[n, m]) and a bias indexed by m."""
+    torch.manual_seed(M + N + K)
+    dev = "cuda"
+    A = torch.randn(M, K, device=dev).bfloat16()
+    B = torch.randn(N, K, device=dev).bfloat16()
+    As = A.t().contiguous() if a_mn else A
+    Bs = B.t().contiguous() if b_mn else B
+    bias = torch.randn(M, device=dev).bfloat16()
+    C0 = torch.randn(N, M, device=dev)
+    C = C0.clone()
+    kw = dict(c_trans=1)
+    if epi == 0:
+        kw.update(bias=bias, bias_m=1)
+    jg.test_gemm(_desc(M, N, K, As, M if a_mn else K, a_mn, Bs, N if b_mn else K, b_mn, jg.DTYPE_BF16, C, M,
+                       jg.DTYPE_F32, epi=epi, **kw))
+    ref = (A.float() @ B.float().t()).t()
+    ref = ref + bias.float()[None, :] if epi == 0 else C0 + ref
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    assert _rel(C, ref) < 1e-5
+
+
 @pytest.mark.parametrize("M,N,K", [(300, 200, 192), (2048, 768, 768)])
 def test_gemm_epilogues(M, N, K):
     torch.manual_seed(1)
