@@ -4,16 +4,17 @@
 One step = the whole update-stage backward of one GRPO group on the DiT-B workload
 (12 single-stream blocks, d = 768, 256 image + 77 text tokens; G = 8 samples, T = 16
 sampling steps, windows of W = 4, jagg_frac = 1): for every window, the step signals with
-the fused t-weighted aggregation (Phases 2-3) and one joint VJP over the 2G endpoint rows
-accumulating the fp32 parameter gradient (Phase 4), then the gradient's squared norm.
-The forward passes of Phase 1 (endpoints saved, middle steps without saves) run before
-the timed region: their saved activations are inputs resident in HBM.  The metric is
-trajectory-steps of gradient per second: G * T (sample, step) pairs per step.
+the fused t-weighted aggregation (Phases 2-3); then one joint VJP over the 2G endpoint rows
+of every window of the group at once, accumulating the fp32 parameter gradient (Phase 4;
+the window gradients add, so this equals one joint VJP per window); then the gradient's
+squared norm.  The forward passes of Phase 1 (endpoints saved, middle steps without
+saves) run before the timed region: their saved activations are inputs resident in HBM.
+The metric is trajectory-steps of gradient per second: G * T (sample, step) pairs per step.
 
-The same step on the exact per-step path (jagg_frac = 0: each window's VJP over all W*G
-step inputs with their own s_j) is timed too, and `e2e` times the update stage through
-the public API from pinned host buffers (Phase 1 forwards included).  `--impl reference`
-times the float64 CPU oracle instead.
+Also timed: the same step with one joint VJP per window (Algorithm 1 as written), the
+exact per-step path (jagg_frac = 0: the VJP over all W*G step inputs of every window with
+their own s_j), and `e2e`, the update stage through the public API from pinned host
+buffers (Phase 1 forwards included).  `--impl reference` times the float64 CPU oracle.
 """
 from __future__ import annotations
 
@@ -166,16 +167,14 @@ class Bench:
         self.sig_dev = torch.tensor(self.sig, **f64)
         self.rewards = torch.tensor(self.draws.rewards, dtype=torch.float32, device=dev)
         self.txt1 = torch.tensor(self.draws.txt, dtype=self.tdt, device=dev)
-        maxB = W * G
-        self.ws = jg.alloc_bytes(self.model.workspace_bytes(maxB), dev)
+        self.ws = jg.alloc_bytes(self.model.workspace_bytes(self.nw * W * G), dev)
         self.sws = jg.alloc_bytes(jg.signals_workspace_bytes(G, W, self.D), dev)
         self.gws = jg.alloc_bytes(jg.grad_reduce_workspace_bytes(self.P), dev)
         self.grad = torch.zeros(self.P, dtype=torch.float32, device=dev)
         self.out3 = torch.zeros(3, **f64)
         self.sig_out = dict(logp_new=torch.empty(G, W, **f64), ratio=torch.empty(G, W, **f64),
                             clipped=torch.empty(G, W, dtype=torch.uint8, device=dev), adv_out=torch.empty(G, **f64))
-        self.cot = torch.empty(2 * G, self.D, dtype=torch.float32, device=dev)
-        self.s = torch.empty(G, W, self.D, dtype=torch.float32, device=dev)
+        self.cot_all = torch.empty(self.nw * W * G, self.D, dtype=torch.float32, device=dev)
 
     # rows of a window's forward: JAGG = [z_0 of each sample; z_{W-1} of each sample],
     # exact = (sample, step) pairs in sample-major order, matching s [G, W, D]
@@ -218,44 +217,64 @@ class Bench:
         self.logp_old = torch.zeros(G, T, dtype=torch.float64, device=dev)
         zero = torch.zeros(G, W, dtype=torch.float64, device=dev)
         for w in range(self.nw):
-            self.signals(w, zero, cot=False)
+            self.signals(w, zero)
             self.logp_old[:, w * W:(w + 1) * W] = self.sig_out["logp_new"]
         self.logp_old += torch.tensor(self.draws.delta, dtype=torch.float64, device=dev)
         self.lpo_win = [self.logp_old[:, w * W:(w + 1) * W].contiguous() for w in range(self.nw)]
         torch.cuda.synchronize()
 
-    def signals(self, w, logp_old, cot=True, s=False):
+    def signals(self, w, logp_old, cot_out=None, s_out=None):
         W = self.wl.W
-        self.jg.grpo_step_signals(self.v_win[w], self.z_win[w],
-                                  self.t_dev[w * W:w * W + W + 1], self.sig_dev[w * W:(w + 1) * W], logp_old, self.rewards,
-                                  self.wl.clip_eps, self.wl.adv_clip, self.wl.adv_eps, self.scale, ws=self.sws,
-                                  cot_out=self.cot if cot else None, s_out=self.s if s else None, **self.sig_out)
+        self.jg.grpo_step_signals(self.v_win[w], self.z_win[w], self.t_dev[w * W:w * W + W + 1],
+                                  self.sig_dev[w * W:(w + 1) * W], logp_old, self.rewards, self.wl.clip_eps,
+                                  self.wl.adv_clip, self.wl.adv_eps, self.scale, ws=self.sws, cot_out=cot_out,
+                                  s_out=s_out, **self.sig_out)
 
-    def forward_saves(self, jagg):
-        """Phase 1 endpoints (JAGG) or every step (exact) of each window, with saves."""
+    def plan(self, routes):
+        """Rows of the group's Phase 4: (window, is_jagg, first_row, rows) per window --
+        the 2G endpoint rows of a JAGG window, the W*G step rows of an exact window."""
+        G, W = self.wl.G, self.wl.W
+        out, r = [], 0
+        for w in range(self.nw):
+            n = 2 * G if routes[w] else W * G
+            out.append((w, bool(routes[w]), r, n))
+            r += n
+        return out, r
+
+    def forward_saves(self, routes, batched):
+        """Phase 1 with saves for the rows of the plan.  batched: one arena holding every
+        window's rows (one joint VJP per group); otherwise one arena per window."""
         wl = self.wl
-        B = 2 * wl.G if jagg else wl.W * wl.G
+        G, W = wl.G, wl.W
+        plan, _ = self.plan(routes)
+        rows = [self.rows(self.z[:, w * W:(w + 1) * W].reshape(G, W, *self.shape), w, jagg)
+                for (w, jagg, _, _) in plan]
+        if batched:
+            groups = [(torch.cat([r[0] for r in rows]), torch.cat([r[1] for r in rows]), plan)]
+        else:
+            groups = [(rows[i][0], rows[i][1], [plan[i]]) for i in range(len(plan))]
         arenas = []
-        for w in range(self.nw):
-            z_win = self.z[:, w * wl.W:(w + 1) * wl.W].reshape(wl.G, wl.W, *self.shape)
-            zr, tr = self.rows(z_win, w, jagg)
+        for z, t, pl in groups:
+            B = z.shape[0]
             saved = self.jg.alloc_bytes(self.model.saved_bytes(B), self.dev)
-            v = torch.empty_like(zr)
-            self.jg.dit_forward_save(self.model, zr, tr, self.txt_rows(B), v, saved=saved, ws=self.ws)
-            arenas.append(saved)
+            v = torch.empty_like(z)
+            self.jg.dit_forward_save(self.model, z, t, self.txt_rows(B), v, saved=saved, ws=self.ws)
+            arenas.append((saved, B, pl))
         torch.cuda.synchronize()
-        return arenas, B
+        return arenas
 
-    def step(self, arenas, B, jagg, routes):
-        """Phases 2-4 over every window, then the gradient's squared norm."""
-        jg = self.jg
-        for w in range(self.nw):
-            if jagg and routes[w]:
-                self.signals(w, self.lpo_win[w], cot=True)
-                jg.dit_joint_vjp(self.model, arenas[w], B, self.cot, self.grad, self.ws)
-            else:
-                self.signals(w, self.lpo_win[w], cot=False, s=True)
-                jg.dit_joint_vjp(self.model, arenas[w], B, self.s, self.grad, self.ws)
+    def step(self, arenas):
+        """Phases 2-4 for every window of the group, then the gradient's squared norm."""
+        jg, G, W, D = self.jg, self.wl.G, self.wl.W, self.D
+        for saved, B, pl in arenas:
+            row0 = pl[0][2]
+            for (w, jagg, r, n) in pl:
+                dst = self.cot_all[r:r + n]
+                if jagg:
+                    self.signals(w, self.lpo_win[w], cot_out=dst)
+                else:
+                    self.signals(w, self.lpo_win[w], s_out=dst.view(G, W, D))
+            jg.dit_joint_vjp(self.model, saved, B, self.cot_all[row0:row0 + B], self.grad, self.ws)
         jg.grad_reduce(self.grad, None, out3=self.out3, ws=self.gws)
 
 
@@ -363,26 +382,28 @@ def run_gpu(args, ws, rank):
     b = Bench(wl, dev)
     b.rollout()
     routes, _ = jg.jagg_route(b.nw, wl.jagg_frac)
-    arenas, B = b.forward_saves(jagg=True)
+    arenas = b.forward_saves(routes, batched=True)
+    B = arenas[0][1]
     use_graph = not args.no_graph
     units = wl.G * wl.T
 
-    # ---- JAGG path: timed region
+    # ---- JAGG path, one joint VJP over every window's endpoint rows: timed region
     n0 = jg.launch_count()
-    b.step(arenas, B, True, routes)
+    b.step(arenas)
     torch.cuda.synchronize()
     launches_per_step = jg.launch_count() - n0
     assert jg.device_status() == 0, "device status set during the JAGG step"
     with ClockSampler(torch.cuda.current_device()) as clk:
-        ms, graph = time_steps(lambda: b.step(arenas, B, True, routes), args.steps, args.warmup, ws, use_graph)
+        ms, graph = time_steps(lambda: b.step(arenas), args.steps, args.warmup, ws, use_graph)
     clocks = clk.summary()
     ms = max_over_ranks(ms, ws)
     value = ws * units / (ms / 1000.0)
+    del graph
 
     # ---- per-family device time of the same step (events around each launch, eager)
     jg.profile_enable(True)
     for _ in range(args.steps):
-        b.step(arenas, B, True, routes)
+        b.step(arenas)
     prof = jg.profile_read()
     jg.profile_enable(False)
     burst, sustained, hbm, src = peaks()
@@ -400,7 +421,6 @@ def run_gpu(args, ws, rank):
     families = {k: {"launches_per_step": v["launches"] / args.steps, "ms_per_step": v["ms"] / args.steps,
                     "tflops": (v["flops"] / (v["ms"] / 1000.0) / 1e12) if v["ms"] > 0 else None}
                 for k, v in fam.items()}
-    del graph
 
     out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
@@ -409,8 +429,9 @@ def run_gpu(args, ws, rank):
                                    f"{wl.n_img} img + {wl.txt_len} txt tokens, G={wl.G}, T={wl.T}, W={wl.W}, "
                                    f"jagg_frac={wl.jagg_frac}"),
                       "rows_per_vjp": B, "windows": b.nw, "cuda_graph": use_graph,
+                      "vjp_batching": f"one joint VJP per group over all {b.nw} windows' endpoint rows",
                       "l2": "inputs larger than L2 (saved activations %.1f GB per step)" % (
-                          sum(a.numel() for a in arenas) / 1e9),
+                          sum(a[0].numel() for a in arenas) / 1e9),
                       "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU"},
            "roofline": roofline, "algorithmic_tflops_per_step": step_flops / 1e12,
            "step_tflops_per_s": step_flops / (ms / 1000.0) / 1e12, "families": families,
@@ -419,14 +440,20 @@ def run_gpu(args, ws, rank):
     torch.cuda.empty_cache()
 
     if not args.quick:
-        # ---- exact per-step path (jagg_frac = 0)
-        arenas_f, Bf = b.forward_saves(jagg=False)
+        # ---- the same JAGG step with one joint VJP per window (Algorithm 1 as written)
+        arenas_w = b.forward_saves(routes, batched=False)
+        ms_w, graph = time_steps(lambda: b.step(arenas_w), args.steps, args.warmup, ws, use_graph)
+        ms_w = max_over_ranks(ms_w, ws)
+        out["per_window_vjp"] = {"value": ws * units / (ms_w / 1000.0), "unit": UNIT, "ms_per_step": ms_w,
+                                 "rows_per_vjp": arenas_w[0][1], "vjps_per_step": len(arenas_w)}
+        del graph, arenas_w
+        # ---- exact per-step path (jagg_frac = 0), batched like the headline
+        arenas_f = b.forward_saves([0] * b.nw, batched=True)
         b.grad.zero_()
-        ms_f, graph = time_steps(lambda: b.step(arenas_f, Bf, False, [0] * b.nw), args.steps, args.warmup, ws,
-                                 use_graph)
+        ms_f, graph = time_steps(lambda: b.step(arenas_f), args.steps, args.warmup, ws, use_graph)
         ms_f = max_over_ranks(ms_f, ws)
         out["full_w"] = {"value": ws * units / (ms_f / 1000.0), "unit": UNIT, "ms_per_step": ms_f,
-                         "rows_per_vjp": Bf}
+                         "rows_per_vjp": arenas_f[0][1]}
         out["jagg_speedup_vs_full_w"] = ms_f / ms
         out["ideal_speedup"] = wl.W / 2
         del graph, arenas_f
@@ -456,32 +483,47 @@ def run_e2e(b, args, ws, routes):
     h_rw = b.rewards.cpu().pin_memory()
     h_lpn = torch.empty(G, wl.T, dtype=torch.float64).pin_memory()
     h_out3 = torch.empty(3, dtype=torch.float64).pin_memory()
-    B = 2 * G
-    arenas = [jg.alloc_bytes(b.model.saved_bytes(B), dev) for _ in range(b.nw)]
-    v_mid = torch.empty(G * (W - 2), *b.shape, dtype=b.tdt, device=dev)
+    nw = b.nw
+    B = nw * 2 * G                       # every window's two endpoints, saved
+    Bm = nw * (W - 2) * G                # every window's middle steps, not saved
+    saved = jg.alloc_bytes(b.model.saved_bytes(B), dev)
     v_end = torch.empty(B, *b.shape, dtype=b.tdt, device=dev)
-    txt_mid, txt_end = b.txt_rows(G * (W - 2)), b.txt_rows(B)
+    v_mid = torch.empty(max(Bm, 1), *b.shape, dtype=b.tdt, device=dev)
+    txt_mid, txt_end = b.txt_rows(max(Bm, 1)), b.txt_rows(B)
+    t_end = torch.tensor(np.concatenate([np.repeat([b.t[w * W], b.t[w * W + W - 1]], G) for w in range(nw)]),
+                         dtype=torch.float32, device=dev)
+    t_mid = torch.tensor(np.concatenate([np.tile(b.t[w * W + 1:w * W + W - 1], G) for w in range(nw)]),
+                         dtype=torch.float32, device=dev)
+    z_end = torch.empty(B, *b.shape, dtype=b.tdt, device=dev)
+    z_mid = torch.empty(max(Bm, 1), *b.shape, dtype=b.tdt, device=dev)
 
     def step():
         b.z.copy_(h_z, non_blocking=True)
         b.logp_old.copy_(h_lpo, non_blocking=True)
         b.rewards.copy_(h_rw, non_blocking=True)
-        for w in range(b.nw):
+        for w in range(nw):
+            zw = b.z[:, w * W:(w + 1) * W].reshape(G, W, *b.shape)
+            z_end[w * 2 * G:w * 2 * G + G].copy_(zw[:, 0])
+            z_end[w * 2 * G + G:(w + 1) * 2 * G].copy_(zw[:, W - 1])
+            if W > 2:
+                z_mid[w * (W - 2) * G:(w + 1) * (W - 2) * G].copy_(zw[:, 1:W - 1].reshape(-1, *b.shape))
+        # Phase 1: endpoints of every window with saves, middle steps without
+        jg.dit_forward_save(b.model, z_end, t_end, txt_end, v_end, saved=saved, ws=b.ws)
+        if W > 2:
+            jg.dit_forward_save(b.model, z_mid[:Bm], t_mid, txt_mid[:Bm], v_mid[:Bm], ws=b.ws)
+        for w in range(nw):
             b.z_win[w].copy_(b.z[:, w * W:w * W + W + 1])
             b.lpo_win[w].copy_(b.logp_old[:, w * W:(w + 1) * W])
-            z_win = b.z[:, w * W:(w + 1) * W].reshape(G, W, *b.shape)
-            zr, tr = b.rows(z_win, w, True)
-            jg.dit_forward_save(b.model, zr, tr, txt_end, v_end, saved=arenas[w], ws=b.ws)
-            zm = z_win[:, 1:W - 1].reshape(G * (W - 2), *b.shape).to(b.tdt).contiguous()
-            tm = torch.tensor(np.tile(b.t[w * W + 1:w * W + W - 1], G), dtype=torch.float32, device=dev)
-            jg.dit_forward_save(b.model, zm, tm, txt_mid, v_mid, ws=b.ws)
             vw = b.v_win[w]
-            vw[:, 0].copy_(v_end[:G].reshape(G, -1))
-            vw[:, W - 1].copy_(v_end[G:].reshape(G, -1))
-            vw[:, 1:W - 1].copy_(v_mid.reshape(G, W - 2, -1))
-            b.signals(w, b.lpo_win[w], cot=True)
+            vw[:, 0].copy_(v_end[w * 2 * G:w * 2 * G + G].reshape(G, -1))
+            vw[:, W - 1].copy_(v_end[w * 2 * G + G:(w + 1) * 2 * G].reshape(G, -1))
+            if W > 2:
+                vw[:, 1:W - 1].copy_(v_mid[w * (W - 2) * G:(w + 1) * (W - 2) * G].reshape(G, W - 2, -1))
+            # Phases 2-3
+            b.signals(w, b.lpo_win[w], cot_out=b.cot_all[w * 2 * G:(w + 1) * 2 * G])
             h_lpn[:, w * W:(w + 1) * W].copy_(b.sig_out["logp_new"], non_blocking=True)
-            jg.dit_joint_vjp(b.model, arenas[w], B, b.cot, b.grad, b.ws)
+        # Phase 4 for the whole group
+        jg.dit_joint_vjp(b.model, saved, B, b.cot_all[:B], b.grad, b.ws)
         jg.grad_reduce(b.grad, None, out3=b.out3, ws=b.gws)
         h_out3.copy_(b.out3, non_blocking=True)
         torch.cuda.current_stream().synchronize()
@@ -498,7 +540,7 @@ def run_e2e(b, args, ws, routes):
     d2h = h_lpn.numel() * 8 + h_out3.numel() * 8
     return {"value": ws * wl.G * wl.T / sec, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "ms_per_step": 1000 * sec, "steps": steps,
-            "includes": "Phase 1 forwards (2G rows saved + (W-2)G rows unsaved per window), signals, joint VJP"}
+            "includes": "Phase 1 forwards (2G rows saved + (W-2)G rows unsaved per window), signals, one joint VJP"}
 
 
 def main():

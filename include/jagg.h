@@ -82,6 +82,15 @@ typedef struct jagg_profile_stat {
 } jagg_profile_stat;
 int jagg_profile_enable(int on);
 int jagg_profile_read(jagg_profile_stat* out, int cap, int* n_out);
+/* The recorded launches one by one, in launch order (up to `cap`): family, the product's
+ * M, N, K (0 for attention), device milliseconds and algorithmic FLOPs.  Synchronises. */
+typedef struct jagg_profile_launch {
+  char family[32];
+  int32_t m, n, k;
+  double ms;
+  double flops;
+} jagg_profile_launch;
+int jagg_profile_launches(jagg_profile_launch* out, int cap, int* n_out);
 
 /* ------------------------------------------------------------------ backbone
  * The velocity network v_theta(z, t, txt).  The paper trains Flux and Qwen-Image

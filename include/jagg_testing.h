@@ -18,9 +18,9 @@ extern "C" {
 
 /* D[m, n] = sum_k A[m, k] B[n, k] with the library's epilogues:
  *   epi 0 store:  C = D (+ bias[n])
- *   epi 1 gelu:   C = u = D + bias, C2 = gelu_tanh(u)
+ *   epi 1 gelu:   u = D + bias, C = gelu_tanh'(u), C2 = gelu_tanh(u)
  *   epi 2 gate:   C = y = D + bias, C2 = aux + gate[(m / rows_per_seq) * gate_stride + n] * y
- *   epi 3 dgelu:  C = D * gelu_tanh'(aux)
+ *   epi 3 mul:    C = D * aux
  *   epi 4 accum:  C += D (f32 C; split_k > 0 forces the number of K splits)
  * A is K-major (A[m*lda + k]) or MN-major (A[k*lda + m]); B is K-major (B[n*ldb + k]) or
  * MN-major (B[k*ldb + n]).  a_dtype/b_dtype/c_dtype/bias_dtype are JAGG_DTYPE_*; C2 and aux

@@ -65,6 +65,11 @@ class ProfileStat(ctypes.Structure):
                 ("flops", ctypes.c_double), ("bytes", ctypes.c_double)]
 
 
+class ProfileLaunch(ctypes.Structure):
+    _fields_ = [("family", ctypes.c_char * 32), ("m", ctypes.c_int32), ("n", ctypes.c_int32),
+                ("k", ctypes.c_int32), ("ms", ctypes.c_double), ("flops", ctypes.c_double)]
+
+
 _lib = None
 _P = ctypes.c_void_p
 _I = ctypes.c_int
@@ -78,6 +83,7 @@ _SIGNATURES = {
     "jagg_launch_count": (_I64, []),
     "jagg_profile_enable": (_I, [_I]),
     "jagg_profile_read": (_I, [ctypes.POINTER(ProfileStat), _I, ctypes.POINTER(_I)]),
+    "jagg_profile_launches": (_I, [ctypes.POINTER(ProfileLaunch), _I, ctypes.POINTER(_I)]),
     "jagg_param_count": (_I64, [ctypes.POINTER(Config)]),
     "jagg_param_tensor_count": (_I, [ctypes.POINTER(Config)]),
     "jagg_param_info": (_I, [ctypes.POINTER(Config), _I, ctypes.c_char_p, _SZ, ctypes.POINTER(_I64),
@@ -318,6 +324,14 @@ def profile_read() -> dict:
     _check(lib().jagg_profile_read(arr, 16, ctypes.byref(n)), "jagg_profile_read")
     return {arr[i].family.decode(): dict(launches=arr[i].launches, ms=arr[i].ms, flops=arr[i].flops,
                                          bytes=arr[i].bytes) for i in range(n.value)}
+
+
+def profile_launches(cap: int = 200000) -> list:
+    """Recorded launches in order: (family, m, n, k, ms, flops)."""
+    arr = (ProfileLaunch * cap)()
+    n = _I()
+    _check(lib().jagg_profile_launches(arr, cap, ctypes.byref(n)), "jagg_profile_launches")
+    return [(arr[i].family.decode(), arr[i].m, arr[i].n, arr[i].k, arr[i].ms, arr[i].flops) for i in range(n.value)]
 
 
 def device_status(clear: bool = True) -> int:

@@ -86,6 +86,13 @@ __device__ __forceinline__ float gelu_tanh_grad(float u) {
   float th = tanhf(c * (u + a * u * u * u));
   return 0.5f * (1.f + th) + 0.5f * u * (1.f - th * th) * c * (1.f + 3.f * a * u * u);
 }
+// gelu(u) and gelu'(u) sharing one tanh.
+__device__ __forceinline__ void gelu_tanh_both(float u, float& g, float& dg) {
+  const float c = 0.7978845608028654f, a = 0.044715f;
+  const float th = tanhf(c * (u + a * u * u * u));
+  g = 0.5f * u * (1.f + th);
+  dg = 0.5f * (1.f + th) + 0.5f * u * (1.f - th * th) * c * (1.f + 3.f * a * u * u);
+}
 __device__ __forceinline__ float silu_f(float x) { return x / (1.f + expf(-x)); }
 __device__ __forceinline__ float silu_grad_f(float x) {
   float s = 1.f / (1.f + expf(-x));
@@ -107,7 +114,7 @@ int sm_count();
 void count_launch();
 enum ProfFamily : int { PROF_GEMM_TC = 0, PROF_GEMM_SIMT, PROF_ATTN_FWD, PROF_ATTN_BWD, PROF_FAMILIES };
 int prof_start(cudaStream_t s);  // returns a token, or -1 when profiling is off
-void prof_stop(int token, cudaStream_t s, int family, double flops, double bytes);
+void prof_stop(int token, cudaStream_t s, int family, double flops, double bytes, int m = 0, int n = 0, int k = 0);
 
 }  // namespace jagg
 

@@ -65,9 +65,10 @@ __device__ __forceinline__ void epi_apply1(const EpiParams& e, int m, int n, flo
       stv(e.C, e.c_trans ? (int64_t)n * e.ldc + cr : cr * e.ldc + n, e.c_bf16, v);
     } break;
     case EPI_GELU: {
-      float u = acc + (e.bias ? ldv(e.bias, n, e.bias_bf16) : 0.f);
-      stv(e.C, cr * e.ldc + n, e.c_bf16, u);
-      stv(e.C2, cr * e.ldc2 + n, e.c_bf16, gelu_tanh(u));
+      float g, dg;
+      gelu_tanh_both(acc + (e.bias ? ldv(e.bias, n, e.bias_bf16) : 0.f), g, dg);
+      stv(e.C, cr * e.ldc + n, e.c_bf16, dg);
+      stv(e.C2, cr * e.ldc2 + n, e.c_bf16, g);
     } break;
     case EPI_GATE_RESID: {
       float y = acc + (e.bias ? ldv(e.bias, n, e.bias_bf16) : 0.f);
@@ -76,10 +77,9 @@ __device__ __forceinline__ void epi_apply1(const EpiParams& e, int m, int n, flo
       const float* hin = static_cast<const float*>(e.aux);
       static_cast<float*>(e.C2)[(int64_t)m * e.ldc2 + n] = hin[(int64_t)m * e.ld_aux + n] + g * y;
     } break;
-    case EPI_DGELU: {
-      float u = ldv(e.aux, (int64_t)m * e.ld_aux + n, e.c_bf16);
-      stv(e.C, cr * e.ldc + n, e.c_bf16, acc * gelu_tanh_grad(u));
-    } break;
+    case EPI_MUL_AUX:
+      stv(e.C, cr * e.ldc + n, e.c_bf16, acc * ldv(e.aux, (int64_t)m * e.ld_aux + n, e.c_bf16));
+      break;
     case EPI_ACCUM:
       atomicAdd(static_cast<float*>(e.C) + (e.c_trans ? (int64_t)n * e.ldc + cr : cr * e.ldc + n), acc);
       break;
@@ -96,7 +96,7 @@ __device__ __forceinline__ void epi_apply8(const EpiParams& e, int m, int n, con
   }
   const int64_t cr = epi_crow(e, m);
   float v[8];
-  if (e.epi != EPI_DGELU && e.epi != EPI_ACCUM && e.bias) {
+  if (e.epi != EPI_MUL_AUX && e.epi != EPI_ACCUM && e.bias) {
     if (e.bias_bf16) {
       uint4 raw = *reinterpret_cast<const uint4*>(static_cast<const bf16*>(e.bias) + n);
       const bf16* b = reinterpret_cast<const bf16*>(&raw);
@@ -130,10 +130,10 @@ __device__ __forceinline__ void epi_apply8(const EpiParams& e, int m, int n, con
       store8(e.C, cr * e.ldc + n, e.c_bf16, v);
       break;
     case EPI_GELU: {
-      store8(e.C, cr * e.ldc + n, e.c_bf16, v);
-      float gv[8];
+      float gv[8], dv[8];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) gv[i] = gelu_tanh(v[i]);
+      for (int i = 0; i < 8; ++i) gelu_tanh_both(v[i], gv[i], dv[i]);
+      store8(e.C, cr * e.ldc + n, e.c_bf16, dv);
       store8(e.C2, cr * e.ldc2 + n, e.c_bf16, gv);
     } break;
     case EPI_GATE_RESID: {
@@ -145,7 +145,7 @@ __device__ __forceinline__ void epi_apply8(const EpiParams& e, int m, int n, con
                     h1.x + g[4] * v[4], h1.y + g[5] * v[5], h1.z + g[6] * v[6], h1.w + g[7] * v[7]};
       store8(e.C2, (int64_t)m * e.ldc2 + n, 0, o);
     } break;
-    case EPI_DGELU: {
+    case EPI_MUL_AUX: {
       float u[8];
       if (e.c_bf16) {
         uint4 raw = *reinterpret_cast<const uint4*>(static_cast<const bf16*>(e.aux) + (int64_t)m * e.ld_aux + n);
@@ -158,7 +158,7 @@ __device__ __forceinline__ void epi_apply8(const EpiParams& e, int m, int n, con
       }
       float o[8];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) o[i] = a[i] * gelu_tanh_grad(u[i]);
+      for (int i = 0; i < 8; ++i) o[i] = a[i] * u[i];
       store8(e.C, cr * e.ldc + n, e.c_bf16, o);
     } break;
     case EPI_ACCUM: {
@@ -500,7 +500,7 @@ EpiParams make_epi(const GemmArgs& g) {
   bool ok = (g.N % 8 == 0) && (g.ldc % 8 == 0) && al16(g.C);
   if (g.bias) ok = ok && al16(g.bias);
   if (g.epi == EPI_GELU || g.epi == EPI_GATE_RESID) ok = ok && (g.ldc2 % 8 == 0) && al16(g.C2);
-  if (g.epi == EPI_GATE_RESID || g.epi == EPI_DGELU) ok = ok && (g.ld_aux % 8 == 0) && al16(g.aux);
+  if (g.epi == EPI_GATE_RESID || g.epi == EPI_MUL_AUX) ok = ok && (g.ld_aux % 8 == 0) && al16(g.aux);
   e.c_trans = g.c_trans ? 1 : 0;
   e.bias_m = g.bias_m ? 1 : 0;
   if (g.c_trans || g.bias_m) ok = false;  // per-element path for transposed outputs
@@ -515,7 +515,7 @@ int validate(const GemmArgs& g) {
   JAGG_CHECK_ARG(g.epi != EPI_ACCUM || g.c_dtype == JAGG_DTYPE_F32, "gemm: accumulation needs an f32 output");
   JAGG_CHECK_ARG(g.epi != EPI_GELU || g.C2, "gemm: GELU epilogue needs C2");
   JAGG_CHECK_ARG(g.epi != EPI_GATE_RESID || (g.C2 && g.aux && g.gate), "gemm: gate epilogue needs C2/aux/gate");
-  JAGG_CHECK_ARG(g.epi != EPI_DGELU || g.aux, "gemm: dGELU epilogue needs aux");
+  JAGG_CHECK_ARG(g.epi != EPI_MUL_AUX || g.aux, "gemm: multiply epilogue needs aux");
   return JAGG_OK;
 }
 
@@ -560,7 +560,8 @@ int launch_tc(const GemmArgs& g, cudaStream_t stream) {
   gemm_tc_kernel<BN, A_MN, B_MN><<<grid, TC_THREADS, Cfg::SMEM_BYTES, stream>>>(ta, tb, p);
   JAGG_LAUNCHED();
   prof_stop(tok, stream, PROF_GEMM_TC, 2.0 * g.M * g.N * g.K,
-            2.0 * ((double)g.M * g.K + (double)g.N * g.K) + (double)g.M * g.N * (g.c_dtype == JAGG_DTYPE_F32 ? 4 : 2));
+            2.0 * ((double)g.M * g.K + (double)g.N * g.K) + (double)g.M * g.N * (g.c_dtype == JAGG_DTYPE_F32 ? 4 : 2),
+            g.M, g.N, g.K);
   return JAGG_OK;
 }
 
@@ -613,7 +614,7 @@ int gemm_simt(const GemmArgs& g, cudaStream_t stream) {
   else
     gemm_simt_kernel<64, 64><<<grid, 256, 0, stream>>>(p);
   JAGG_LAUNCHED();
-  prof_stop(tok, stream, PROF_GEMM_SIMT, 2.0 * g.M * g.N * g.K, 0.0);
+  prof_stop(tok, stream, PROF_GEMM_SIMT, 2.0 * g.M * g.N * g.K, 0.0, g.M, g.N, g.K);
   return JAGG_OK;
 }
 

@@ -182,7 +182,7 @@ struct DitSaved {
   void* y1;      // [M, d] proj output (before the gate)
   float* h_mid;  // [M, d]
   void* m;       // [M, d] LN2 + modulation
-  void* u;       // [M, dm] fc1 output (GELU input)
+  void* gp;      // [M, dm] GELU'(u) at the fc1 output u (all the backward needs of u)
   void* gu;      // [M, dm] GELU(u)
   void* y2;      // [M, d] fc2 output (before the gate)
   float* st1;    // [2, M] mean, rstd of LN1
@@ -193,6 +193,8 @@ struct Saved {
   void* xp;      // [B*Ni, pd]
   void* txt;     // [B*Nt, txt_dim]
   float* phi;    // [B, freq]
+  void* phi_b;   // [B, freq] storage type
+  void* se1_b;   // [B, d] silu(e1), storage type
   float* e1;     // [B, d]
   float* se1;    // [B, d] silu(e1)
   float* c;      // [B, d]
@@ -216,7 +218,7 @@ void carve_block(Carver& cv, const jagg_model& m, int B, DitSaved& s) {
   s.y1 = cv.take(M * m.d * e);
   s.h_mid = cv.f32(M * m.d);
   s.m = cv.take(M * m.d * e);
-  s.u = cv.take(M * m.dm * e);
+  s.gp = cv.take(M * m.dm * e);
   s.gu = cv.take(M * m.dm * e);
   s.y2 = cv.take(M * m.d * e);
   s.st1 = cv.f32(2 * M);
@@ -231,6 +233,8 @@ size_t carve_saved(const jagg_model& m, int B, void* base, bool save, Saved& s) 
   s.xp = cv.take(Mi * m.pd * m.esz);
   s.txt = cv.take(Mt * m.cfg.txt_dim * m.esz);
   s.phi = cv.f32((int64_t)B * m.cfg.freq_dim);
+  s.phi_b = cv.take((size_t)B * m.cfg.freq_dim * m.esz);
+  s.se1_b = cv.take((size_t)B * m.d * m.esz);
   s.e1 = cv.f32((int64_t)B * m.d);
   s.se1 = cv.f32((int64_t)B * m.d);
   s.c = cv.f32((int64_t)B * m.d);
@@ -272,6 +276,7 @@ struct VjpWs {
   void* dvt;    // [B*Ni, pd]
   float* dsc;   // [B, d]
   float* de1;   // [B, d]
+  void* dc_b;   // [B, d] storage-type copy of dc, then of de1
   void* dxe;    // [max(Mi, Mt), d] embedding-input gradients in storage type
 };
 
@@ -291,6 +296,7 @@ size_t carve_vjp_ws(const jagg_model& m, int B, void* base, VjpWs& w) {
   w.dvt = cv.take(Mi * m.pd * e);
   w.dsc = cv.f32((int64_t)B * m.d);
   w.de1 = cv.f32((int64_t)B * m.d);
+  w.dc_b = cv.take((size_t)B * m.d * m.esz);
   w.dxe = cv.take((Mi > Mt ? Mi : Mt) * m.d * e);
   return align256(cv.off);
 }
@@ -338,6 +344,40 @@ GemmArgs dw_gemm(const jagg_model& m, int M, int N, int K, const void* dY, int64
   return g;
 }
 
+// Products over the B per-sequence rows (t-embedding MLP, stacked modulation), in the
+// transposed form whose M is a feature dimension:
+//   rows_gemm: C[B, out] (f32) = X[B, in] W[out, in]^T + b   as  C^T = W X^T
+//   rows_dw:   grad[out, in] += dY[B, out]^T X[B, in]        (K = B)
+//   rows_dx:   dX[B, in] += dY[B, out] W[out, in]             as  dX^T = W^T dY^T
+// X / dY are in the storage type; dX accumulates in f32 (split over out).
+GemmArgs rows_gemm(const jagg_model& m, int out, int in, int B, const void* X, int64_t w_off, int64_t b_off,
+                   float* C) {
+  GemmArgs g;
+  g.M = out; g.N = B; g.K = in;
+  g.A = W(m, w_off); g.lda = in; g.a_dtype = m.cfg.dtype;
+  g.B = X; g.ldb = in; g.b_dtype = m.cfg.dtype;
+  g.bias = W(m, b_off); g.bias_dtype = m.cfg.dtype; g.bias_m = true;
+  g.C = C; g.ldc = out; g.c_dtype = JAGG_DTYPE_F32; g.c_trans = true;
+  return g;
+}
+GemmArgs rows_dw(const jagg_model& m, int out, int in, int B, const void* dY, const void* X, float* grad,
+                 int64_t w_off) {
+  GemmArgs g;
+  g.M = out; g.N = in; g.K = B;
+  g.A = dY; g.lda = out; g.a_mn = true; g.a_dtype = m.cfg.dtype;
+  g.B = X; g.ldb = in; g.b_mn = true; g.b_dtype = m.cfg.dtype;
+  g.epi = EPI_ACCUM; g.C = grad + w_off; g.ldc = in; g.c_dtype = JAGG_DTYPE_F32;
+  return g;
+}
+GemmArgs rows_dx(const jagg_model& m, int out, int in, int B, const void* dY, int64_t w_off, float* dX) {
+  GemmArgs g;
+  g.M = in; g.N = B; g.K = out;
+  g.A = W(m, w_off); g.lda = in; g.a_mn = true; g.a_dtype = m.cfg.dtype;
+  g.B = dY; g.ldb = out; g.b_mn = false; g.b_dtype = m.cfg.dtype;
+  g.epi = EPI_ACCUM; g.C = dX; g.ldc = in; g.c_dtype = JAGG_DTYPE_F32; g.c_trans = true;
+  return g;
+}
+
 int forward_impl(const jagg_model& m, const void* z, const float* t, const void* txt, int B, void* v_out,
                  void* saved, void* ws, cudaStream_t s) {
   const jagg_config& c = m.cfg;
@@ -370,32 +410,16 @@ int forward_impl(const jagg_model& m, const void* z, const float* t, const void*
   JAGG_TRY(launch_add_pos_embed(hstart, B, N, Nt, m.gh, m.gw, d, s));
   // t-embedding MLP and every block's modulation (per-sequence rows, f32 activations)
   JAGG_TRY(launch_timestep_embedding(t, S.phi, B, c.freq_dim, s));
-  {
-    GemmArgs g;
-    g.M = B; g.N = d; g.K = c.freq_dim;
-    g.A = S.phi; g.lda = c.freq_dim; g.a_dtype = JAGG_DTYPE_F32;
-    g.B = W(m, m.T.t_w1); g.ldb = c.freq_dim; g.b_dtype = dt;
-    g.bias = W(m, m.T.t_b1); g.bias_dtype = dt;
-    g.C = S.e1; g.ldc = d; g.c_dtype = JAGG_DTYPE_F32;
-    JAGG_TRY(gemm(g, s));
-    JAGG_TRY(launch_silu(S.e1, S.se1, (int64_t)B * d, s));
-    g.K = d; g.A = S.se1; g.lda = d;
-    g.B = W(m, m.T.t_w2); g.ldb = d;
-    g.bias = W(m, m.T.t_b2);
-    g.C = S.c;
-    JAGG_TRY(gemm(g, s));
-    JAGG_TRY(launch_silu(S.c, S.sc, (int64_t)B * d, s));
-    // every modulation at once, as mod^T [Lmod, B] = W_mod [Lmod, d] silu(c)^T: the long
-    // dimension is M, so the product runs on the tensor-core kernel in the storage type
-    JAGG_TRY(launch_gather_rows(S.sc, d, 0, 0, 0, S.sc_b, dt, B, d, s));
-    GemmArgs gm;
-    gm.M = (int)Lm; gm.N = B; gm.K = d;
-    gm.A = W(m, m.T.mod_w); gm.lda = d; gm.a_dtype = dt;
-    gm.B = S.sc_b; gm.ldb = d; gm.b_dtype = dt;
-    gm.bias = W(m, m.T.mod_b); gm.bias_dtype = dt; gm.bias_m = true;
-    gm.C = S.mod; gm.ldc = Lm; gm.c_dtype = JAGG_DTYPE_F32; gm.c_trans = true;
-    JAGG_TRY(gemm(gm, s));
-  }
+  // t-embedding MLP and every block's modulation at once (stacked weights): products
+  // with B per-sequence rows, each run as Y^T = W X^T so that the long dimension is M
+  JAGG_TRY(launch_gather_rows(S.phi, c.freq_dim, 0, 0, 0, S.phi_b, dt, B, c.freq_dim, s));
+  JAGG_TRY(gemm(rows_gemm(m, d, c.freq_dim, B, S.phi_b, m.T.t_w1, m.T.t_b1, S.e1), s));
+  JAGG_TRY(launch_silu(S.e1, S.se1, (int64_t)B * d, s));
+  JAGG_TRY(launch_gather_rows(S.se1, d, 0, 0, 0, S.se1_b, dt, B, d, s));
+  JAGG_TRY(gemm(rows_gemm(m, d, d, B, S.se1_b, m.T.t_w2, m.T.t_b2, S.c), s));
+  JAGG_TRY(launch_silu(S.c, S.sc, (int64_t)B * d, s));
+  JAGG_TRY(launch_gather_rows(S.sc, d, 0, 0, 0, S.sc_b, dt, B, d, s));
+  JAGG_TRY(gemm(rows_gemm(m, (int)Lm, d, B, S.sc_b, m.T.mod_w, m.T.mod_b, S.mod), s));
   // blocks
   for (int l = 0; l < c.depth; ++l) {
     const DitBlockW& bw = m.T.blocks[l];
@@ -423,7 +447,7 @@ int forward_impl(const jagg_model& m, const void* z, const float* t, const void*
     LnModFwd ln2{k.h_mid, 0, 0, 0, M, d, N, mod + 3 * d, mod + 4 * d, Lm, k.m, dt, k.st2, k.st2 + M};
     JAGG_TRY(launch_ln_mod_fwd(ln2, s));
     g = fwd_gemm(m, M, m.dm, d, k.m, d, bw.fc1_w, bw.fc1_b);
-    g.epi = EPI_GELU; g.C = k.u; g.ldc = m.dm; g.C2 = k.gu; g.ldc2 = m.dm;
+    g.epi = EPI_GELU; g.C = k.gp; g.ldc = m.dm; g.C2 = k.gu; g.ldc2 = m.dm;
     JAGG_TRY(gemm(g, s));
     g = fwd_gemm(m, M, d, m.dm, k.gu, m.dm, bw.fc2_w, bw.fc2_b);
     g.epi = EPI_GATE_RESID; g.C = k.y2; g.ldc = d;
@@ -456,6 +480,7 @@ int vjp_impl(const jagg_model& m, const void* saved, int B, const float* cot, fl
   JAGG_CUDA_TRY(cudaMemsetAsync(w.dmod, 0, sizeof(float) * (size_t)B * Lm, s));
   JAGG_CUDA_TRY(cudaMemsetAsync(w.dh, 0, sizeof(float) * (size_t)M * d, s));
   JAGG_CUDA_TRY(cudaMemsetAsync(w.dsc, 0, sizeof(float) * (size_t)B * d, s));
+  JAGG_CUDA_TRY(cudaMemsetAsync(w.de1, 0, sizeof(float) * (size_t)B * d, s));
 
   // final layer
   JAGG_TRY(launch_patchify(cot, 1, w.dvt, dt == JAGG_DTYPE_F32, dt, B, c.in_channels, c.latent_h, c.latent_w,
@@ -496,7 +521,7 @@ int vjp_impl(const jagg_model& m, const void* saved, int B, const float* cot, fl
     JAGG_TRY(gemm(dw_gemm(m, M, d, dmw, w.dy, d, k.gu, dmw, grad, bw.fc2_w), s));
     {
       GemmArgs g = dx_gemm(m, M, d, dmw, w.dy, d, bw.fc2_w);
-      g.epi = EPI_DGELU; g.C = w.du; g.ldc = dmw; g.aux = k.u; g.ld_aux = dmw;
+      g.epi = EPI_MUL_AUX; g.C = w.du; g.ldc = dmw; g.aux = k.gp; g.ld_aux = dmw;
       JAGG_TRY(gemm(g, s));
     }
     JAGG_TRY(launch_colsum(w.du, dt == JAGG_DTYPE_F32, dt, M, dmw, dmw, grad + bw.fc1_b, s));
@@ -563,47 +588,18 @@ int vjp_impl(const jagg_model& m, const void* saved, int B, const float* cot, fl
   // stacked modulation: dW += dmod^T silu(c), db += sum_b dmod, d silu(c) = dmod W
   JAGG_TRY(launch_colsum(w.dmod, 1, dt, B, (int)Lm, Lm, grad + m.T.mod_b, s));
   JAGG_TRY(launch_gather_rows(w.dmod, Lm, 0, 0, 0, w.dmod_b, dt, B, (int)Lm, s));
-  {
-    GemmArgs g;  // grad[Lmod, d] += dmod^T silu(c): both operands MN-major, K = B
-    g.M = (int)Lm; g.N = d; g.K = B;
-    g.A = w.dmod_b; g.lda = Lm; g.a_mn = true; g.a_dtype = dt;
-    g.B = S.sc_b; g.ldb = d; g.b_mn = true; g.b_dtype = dt;
-    g.epi = EPI_ACCUM; g.C = grad + m.T.mod_w; g.ldc = d; g.c_dtype = JAGG_DTYPE_F32;
-    JAGG_TRY(gemm(g, s));
-    GemmArgs h;  // d silu(c)^T [d, B] = W_mod^T [d, Lmod] dmod^T, split over Lmod
-    h.M = d; h.N = B; h.K = (int)Lm;
-    h.A = W(m, m.T.mod_w); h.lda = d; h.a_mn = true; h.a_dtype = dt;
-    h.B = w.dmod_b; h.ldb = Lm; h.b_mn = false; h.b_dtype = dt;
-    h.epi = EPI_ACCUM; h.C = w.dsc; h.ldc = d; h.c_dtype = JAGG_DTYPE_F32; h.c_trans = true;
-    JAGG_TRY(gemm(h, s));
-  }
+  JAGG_TRY(gemm(rows_dw(m, (int)Lm, d, B, w.dmod_b, S.sc_b, grad, m.T.mod_w), s));
+  JAGG_TRY(gemm(rows_dx(m, (int)Lm, d, B, w.dmod_b, m.T.mod_w, w.dsc), s));  // d silu(c)
   // t-embedding MLP
   JAGG_TRY(launch_mul_silu_grad(w.dsc, S.c, (int64_t)B * d, s));  // dc
   JAGG_TRY(launch_colsum(w.dsc, 1, dt, B, d, d, grad + m.T.t_b2, s));
-  {
-    GemmArgs g;
-    g.M = d; g.N = d; g.K = B;
-    g.A = w.dsc; g.lda = d; g.a_mn = true; g.a_dtype = JAGG_DTYPE_F32;
-    g.B = S.se1; g.ldb = d; g.b_mn = true; g.b_dtype = JAGG_DTYPE_F32;
-    g.epi = EPI_ACCUM; g.C = grad + m.T.t_w2; g.ldc = d; g.c_dtype = JAGG_DTYPE_F32;
-    JAGG_TRY(gemm(g, s));
-    GemmArgs h;
-    h.M = B; h.N = d; h.K = d;
-    h.A = w.dsc; h.lda = d; h.a_dtype = JAGG_DTYPE_F32;
-    h.B = W(m, m.T.t_w2); h.ldb = d; h.b_mn = true; h.b_dtype = dt;
-    h.C = w.de1; h.ldc = d; h.c_dtype = JAGG_DTYPE_F32;
-    JAGG_TRY(gemm(h, s));
-  }
+  JAGG_TRY(launch_gather_rows(w.dsc, d, 0, 0, 0, w.dc_b, dt, B, d, s));
+  JAGG_TRY(gemm(rows_dw(m, d, d, B, w.dc_b, S.se1_b, grad, m.T.t_w2), s));
+  JAGG_TRY(gemm(rows_dx(m, d, d, B, w.dc_b, m.T.t_w2, w.de1), s));  // d silu(e1)
   JAGG_TRY(launch_mul_silu_grad(w.de1, S.e1, (int64_t)B * d, s));
   JAGG_TRY(launch_colsum(w.de1, 1, dt, B, d, d, grad + m.T.t_b1, s));
-  {
-    GemmArgs g;
-    g.M = d; g.N = c.freq_dim; g.K = B;
-    g.A = w.de1; g.lda = d; g.a_mn = true; g.a_dtype = JAGG_DTYPE_F32;
-    g.B = S.phi; g.ldb = c.freq_dim; g.b_mn = true; g.b_dtype = JAGG_DTYPE_F32;
-    g.epi = EPI_ACCUM; g.C = grad + m.T.t_w1; g.ldc = c.freq_dim; g.c_dtype = JAGG_DTYPE_F32;
-    JAGG_TRY(gemm(g, s));
-  }
+  JAGG_TRY(launch_gather_rows(w.de1, d, 0, 0, 0, w.dc_b, dt, B, d, s));
+  JAGG_TRY(gemm(rows_dw(m, d, c.freq_dim, B, w.dc_b, S.phi_b, grad, m.T.t_w1), s));
   return JAGG_OK;
 }
 

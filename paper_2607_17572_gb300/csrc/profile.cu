@@ -17,6 +17,7 @@ struct Rec {
   cudaEvent_t a = nullptr, b = nullptr;
   int family = -1;
   double flops = 0, bytes = 0;
+  int m = 0, n = 0, k = 0;
 };
 std::vector<Rec> g_recs;
 std::vector<cudaEvent_t> g_pool;
@@ -50,7 +51,7 @@ int prof_start(cudaStream_t s) {
   return (int)g_recs.size() - 1;
 }
 
-void prof_stop(int token, cudaStream_t s, int family, double flops, double bytes) {
+void prof_stop(int token, cudaStream_t s, int family, double flops, double bytes, int m, int n, int k) {
   if (token < 0) return;
   std::lock_guard<std::mutex> lk(g_mu);
   if (token >= (int)g_recs.size()) return;
@@ -59,6 +60,9 @@ void prof_stop(int token, cudaStream_t s, int family, double flops, double bytes
   r.family = family;
   r.flops = flops;
   r.bytes = bytes;
+  r.m = m;
+  r.n = n;
+  r.k = k;
 }
 
 }  // namespace jagg
@@ -96,6 +100,29 @@ extern "C" int jagg_profile_read(jagg_profile_stat* out, int cap, int* n_out) {
   }
   int n = 0;
   for (int f = 0; f < PROF_FAMILIES && n < cap; ++f) out[n++] = acc[f];
+  *n_out = n;
+  return JAGG_OK;
+}
+
+extern "C" int jagg_profile_launches(jagg_profile_launch* out, int cap, int* n_out) {
+  JAGG_CHECK_ARG(out && n_out && cap >= 0, "jagg_profile_launches: null output");
+  JAGG_CUDA_TRY(cudaDeviceSynchronize());
+  std::lock_guard<std::mutex> lk(g_mu);
+  int n = 0;
+  for (const Rec& r : g_recs) {
+    if (n >= cap) break;
+    if (r.family < 0 || r.family >= PROF_FAMILIES) continue;
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, r.a, r.b) != cudaSuccess) continue;
+    jagg_profile_launch& o = out[n++];
+    std::memset(&o, 0, sizeof(o));
+    std::strncpy(o.family, kFamilyNames[r.family], sizeof(o.family) - 1);
+    o.m = r.m;
+    o.n = r.n;
+    o.k = r.k;
+    o.ms = ms;
+    o.flops = r.flops;
+  }
   *n_out = n;
   return JAGG_OK;
 }
