@@ -83,12 +83,14 @@ typedef struct jagg_profile_stat {
 int jagg_profile_enable(int on);
 int jagg_profile_read(jagg_profile_stat* out, int cap, int* n_out);
 /* The recorded launches one by one, in launch order (up to `cap`): family, the product's
- * M, N, K (0 for attention), device milliseconds and algorithmic FLOPs.  Synchronises. */
+ * M, N, K (0 for other families), device milliseconds, algorithmic FLOPs and bytes.
+ * Synchronises. */
 typedef struct jagg_profile_launch {
   char family[32];
   int32_t m, n, k;
   double ms;
   double flops;
+  double bytes;
 } jagg_profile_launch;
 int jagg_profile_launches(jagg_profile_launch* out, int cap, int* n_out);
 

@@ -67,7 +67,8 @@ class ProfileStat(ctypes.Structure):
 
 class ProfileLaunch(ctypes.Structure):
     _fields_ = [("family", ctypes.c_char * 32), ("m", ctypes.c_int32), ("n", ctypes.c_int32),
-                ("k", ctypes.c_int32), ("ms", ctypes.c_double), ("flops", ctypes.c_double)]
+                ("k", ctypes.c_int32), ("ms", ctypes.c_double), ("flops", ctypes.c_double),
+                ("bytes", ctypes.c_double)]
 
 
 _lib = None
@@ -327,11 +328,12 @@ def profile_read() -> dict:
 
 
 def profile_launches(cap: int = 200000) -> list:
-    """Recorded launches in order: (family, m, n, k, ms, flops)."""
+    """Recorded launches in order: (family, m, n, k, ms, flops, bytes)."""
     arr = (ProfileLaunch * cap)()
     n = _I()
     _check(lib().jagg_profile_launches(arr, cap, ctypes.byref(n)), "jagg_profile_launches")
-    return [(arr[i].family.decode(), arr[i].m, arr[i].n, arr[i].k, arr[i].ms, arr[i].flops) for i in range(n.value)]
+    return [(arr[i].family.decode(), arr[i].m, arr[i].n, arr[i].k, arr[i].ms, arr[i].flops, arr[i].bytes)
+            for i in range(n.value)]
 
 
 def device_status(clear: bool = True) -> int:

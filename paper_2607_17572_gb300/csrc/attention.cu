@@ -61,8 +61,20 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src, bool vali
 __device__ __forceinline__ void cp_async_wait_all() {
   asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
 }
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
 
 constexpr int TILE = 64;
+
+// Shared memory of the backward kernel: K, V, NBUF x (Q, dO), dS^T, NBUF x (lse, rowsum).
+template <int D>
+struct BwdCfg {
+  static constexpr int NBUF = D <= 64 ? 2 : 1;
+  static constexpr int SMEM = (2 + 2 * NBUF) * TILE * (D + 8) * 2 + TILE * (TILE + 8) * 2 + 2 * NBUF * TILE * 4;
+};
 
 // Copies rows n0 .. n0+63 (zero beyond N) of one head's D columns into smem with pitch D+8.
 template <int D>
@@ -206,13 +218,17 @@ __global__ void __launch_bounds__(128) fa_bwd_kernel(AttnBwdArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
   constexpr int P = D + 8;
   constexpr int PS = TILE + 8;
+  // Query-side tiles (Q, dO, lse, rowsum) are double-buffered for head dim 64: the next
+  // tile's cp.async copies overlap the current tile's products.  (At 128 the second buffer
+  // would halve the CTAs per SM.)
+  constexpr int NBUF = BwdCfg<D>::NBUF;
   bf16* sK = reinterpret_cast<bf16*>(smem);
   bf16* sV = sK + TILE * P;
-  bf16* sQ = sV + TILE * P;
-  bf16* sdO = sQ + TILE * P;
-  bf16* sdS = sdO + TILE * P;  // [key][query], pitch PS
-  float* sL = reinterpret_cast<float*>(sdS + TILE * PS);  // lse * log2e (+inf beyond N)
-  float* sDv = sL + TILE;
+  bf16* sQ0 = sV + TILE * P;            // NBUF tiles of Q
+  bf16* sdO0 = sQ0 + NBUF * TILE * P;   // NBUF tiles of dO
+  bf16* sdS = sdO0 + NBUF * TILE * P;   // [key][query], pitch PS
+  float* sL0 = reinterpret_cast<float*>(sdS + TILE * PS);  // NBUF x (lse * log2e, +inf beyond N)
+  float* sDv0 = sL0 + NBUF * TILE;
   const AttnArgs& f = a.f;
   const int N = f.N;
   const int kt = blockIdx.x, bh = blockIdx.y;
@@ -221,10 +237,21 @@ __global__ void __launch_bounds__(128) fa_bwd_kernel(AttnBwdArgs a) {
   const int g = lane >> 2, tig = lane & 3;
   const float sl2 = f.scale * kLog2e;
 
+  auto fetch_queries = [&](int qt) {
+    const int buf = qt % NBUF;
+    load_tile<D>(sQ0 + buf * TILE * P, f.q, b, qt * TILE, N, f.q_col0 + (int64_t)h * D);
+    load_tile<D>(sdO0 + buf * TILE * P, a.dO, b, qt * TILE, N, (int64_t)h * D);
+    cp_async_commit();
+    for (int i = threadIdx.x; i < TILE; i += blockDim.x) {
+      const int q = qt * TILE + i;
+      sL0[buf * TILE + i] = q < N ? f.lse[(int64_t)bh * N + q] * kLog2e : INFINITY;
+      sDv0[buf * TILE + i] = q < N ? a.Dv[(int64_t)bh * N + q] : 0.f;
+    }
+  };
+
   load_tile<D>(sK, f.k, b, kt * TILE, N, f.k_col0 + (int64_t)h * D);
   load_tile<D>(sV, f.v, b, kt * TILE, N, f.v_col0 + (int64_t)h * D);
-  cp_async_wait_all();
-  __syncthreads();
+  cp_async_commit();
 
   float dk[D / 8][4], dv[D / 8][4];
 #pragma unroll
@@ -233,17 +260,23 @@ __global__ void __launch_bounds__(128) fa_bwd_kernel(AttnBwdArgs a) {
     dv[i][0] = dv[i][1] = dv[i][2] = dv[i][3] = 0.f;
   }
   const int nqt = (N + TILE - 1) / TILE;
+  if (NBUF == 2) fetch_queries(0);
   for (int qt = 0; qt < nqt; ++qt) {
-    __syncthreads();
-    load_tile<D>(sQ, f.q, b, qt * TILE, N, f.q_col0 + (int64_t)h * D);
-    load_tile<D>(sdO, a.dO, b, qt * TILE, N, (int64_t)h * D);
-    for (int i = threadIdx.x; i < TILE; i += blockDim.x) {
-      const int q = qt * TILE + i;
-      sL[i] = q < N ? f.lse[(int64_t)bh * N + q] * kLog2e : INFINITY;
-      sDv[i] = q < N ? a.Dv[(int64_t)bh * N + q] : 0.f;
+    __syncthreads();  // every warp is done with the buffer about to be refilled
+    if (NBUF == 1) {
+      fetch_queries(qt);
+      cp_async_wait<0>();
+    } else if (qt + 1 < nqt) {
+      fetch_queries(qt + 1);
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
     }
-    cp_async_wait_all();
     __syncthreads();
+    const bf16* sQ = sQ0 + (qt % NBUF) * TILE * P;
+    const bf16* sdO = sdO0 + (qt % NBUF) * TILE * P;
+    const float* sL = sL0 + (qt % NBUF) * TILE;
+    const float* sDv = sDv0 + (qt % NBUF) * TILE;
 
     // S^T = K_w Q^T and dP^T = V_w dO^T: 16 keys x 64 queries per warp
     float st[8][4], dpt[8][4];
@@ -328,19 +361,25 @@ __global__ void __launch_bounds__(128) fa_bwd_kernel(AttnBwdArgs a) {
           mma16816(dq[2 * dp + 1], sa, kb[2], kb[3]);
         }
       }
+      // Lanes tig and tig^1 swap halves so that each issues one 16-byte reduction: even
+      // lanes add row q0, columns 2tig..2tig+3; odd lanes add row q1, columns 2tig-2..2tig+1.
+      // (dq_acc is 16-byte aligned and its row pitch a multiple of 4 floats: checked on launch.)
+      const bool even = (tig & 1) == 0;
+      const int64_t ld = (int64_t)f.heads * D;
 #pragma unroll
       for (int dt = 0; dt < 8; ++dt) {
-        const int col = h * D + dc * 64 + dt * 8 + 2 * tig;
-        const int64_t ld = (int64_t)f.heads * D;
-        if (q0 < N) {
-          float* p = a.dq_acc + ((int64_t)b * N + q0) * ld + col;
-          atomicAdd(p, dq[dt][0] * f.scale);
-          atomicAdd(p + 1, dq[dt][1] * f.scale);
-        }
-        if (q1 < N) {
-          float* p = a.dq_acc + ((int64_t)b * N + q1) * ld + col;
-          atomicAdd(p, dq[dt][2] * f.scale);
-          atomicAdd(p + 1, dq[dt][3] * f.scale);
+        const float s0 = even ? dq[dt][2] : dq[dt][0];
+        const float s1 = even ? dq[dt][3] : dq[dt][1];
+        const float r0 = __shfl_xor_sync(0xffffffffu, s0, 1);
+        const float r1 = __shfl_xor_sync(0xffffffffu, s1, 1);
+        const int qrow = even ? q0 : q1;
+        const int col = h * D + dc * 64 + dt * 8 + 2 * (even ? tig : tig - 1);
+        if (qrow < N) {
+          float* p = a.dq_acc + ((int64_t)b * N + qrow) * ld + col;
+          if (even)
+            ptx::red_add_v4(p, dq[dt][0] * f.scale, dq[dt][1] * f.scale, r0 * f.scale, r1 * f.scale);
+          else
+            ptx::red_add_v4(p, r0 * f.scale, r1 * f.scale, dq[dt][2] * f.scale, dq[dt][3] * f.scale);
         }
       }
     }
@@ -438,34 +477,70 @@ __global__ void attn_bwd_simt(AttnBwdArgs a) {
   }
 }
 
-// Dv[b, h, n] = sum_c dO[n, h*D + c] * O[n, h*D + c]; one warp per (row, head).
-__global__ void rowdot_kernel(AttnBwdArgs a) {
+// Before the backward: Dv[b, h, n] = sum_c dO[n, h*D + c] O[n, h*D + c] and dq_acc = 0.
+// One thread per (row, 8 columns); the D/8 threads of a head are adjacent lanes and
+// combine their partial dots with shuffles.
+__global__ void rowdot_zero_kernel(AttnBwdArgs a) {
   const AttnArgs& f = a.f;
-  const int64_t w = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  const int N = f.N, D = f.dh;
-  if (w >= (int64_t)f.B * N * f.heads) return;
-  const int h = (int)(w % f.heads);
-  const int64_t row = w / f.heads;
-  const int b = (int)(row / N), n = (int)(row % N);
-  const int f32 = f.dtype == JAGG_DTYPE_F32;
-  const int64_t go = a.dO.off(b, n, N, (int64_t)h * D), oo = f.o.off(b, n, N, (int64_t)h * D);
+  const int d = f.heads * f.dh;
+  const int cpr = d / 8;  // 8-column chunks per row
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  const int row = idx / cpr, ch = idx % cpr;
+  const bool live = row < f.B * f.N;
+  const int b = live ? row / f.N : 0, n = live ? row % f.N : 0;
+  const int col = ch * 8;
   float s = 0.f;
-  for (int c = lane; c < D; c += 32) s += ldx(a.dO.base(n), go + c, f32) * ldx(f.o.base(n), oo + c, f32);
-  s = warp_sum(s);
-  if (lane == 0) a.Dv[((int64_t)b * f.heads + h) * N + n] = s;
+  if (live) {
+    const int64_t go = a.dO.off(b, n, f.N, col), oo = f.o.off(b, n, f.N, col);
+    if (f.dtype == JAGG_DTYPE_F32) {
+      const float4* g4 = reinterpret_cast<const float4*>(static_cast<const float*>(a.dO.base(n)) + go);
+      const float4* o4 = reinterpret_cast<const float4*>(static_cast<const float*>(f.o.base(n)) + oo);
+#pragma unroll
+      for (int k = 0; k < 2; ++k) {
+        const float4 x = g4[k], y = o4[k];
+        s += x.x * y.x + x.y * y.y + x.z * y.z + x.w * y.w;
+      }
+    } else {
+      const uint4 gr = *reinterpret_cast<const uint4*>(static_cast<const bf16*>(a.dO.base(n)) + go);
+      const uint4 orr = *reinterpret_cast<const uint4*>(static_cast<const bf16*>(f.o.base(n)) + oo);
+      const bf16* gh = reinterpret_cast<const bf16*>(&gr);
+      const bf16* oh = reinterpret_cast<const bf16*>(&orr);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) s += __bfloat162float(gh[k]) * __bfloat162float(oh[k]);
+    }
+    float4* z = reinterpret_cast<float4*>(a.dq_acc + (int64_t)row * d + col);
+    z[0] = make_float4(0.f, 0.f, 0.f, 0.f);
+    z[1] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  const int per_head = f.dh / 8;  // a power of two <= 32
+  for (int o = per_head / 2; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  if (live && ch % per_head == 0) a.Dv[((int64_t)b * f.heads + ch / per_head) * f.N + n] = s;
 }
 
-// dq (dtype) <- dq_acc (f32).
+// dq (storage type, segment rows) <- dq_acc (f32); one thread per (row, 8 columns).
 __global__ void dq_store_kernel(AttnBwdArgs a) {
   const AttnArgs& f = a.f;
-  const int64_t ld = (int64_t)f.heads * f.dh;
-  const int64_t total = (int64_t)f.B * f.N * ld;
-  const int f32 = f.dtype == JAGG_DTYPE_F32;
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t row = i / ld, c = i % ld;
-    const int b = (int)(row / f.N), n = (int)(row % f.N);
-    stx(a.dq.base(n), a.dq.off(b, n, f.N, a.dq_col0 + c), f32, a.dq_acc[i]);
+  const int d = f.heads * f.dh;
+  const int cpr = d / 8;
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  const int row = idx / cpr, col = (idx % cpr) * 8;
+  if (row >= f.B * f.N) return;
+  const int b = row / f.N, n = row % f.N;
+  const float4* src = reinterpret_cast<const float4*>(a.dq_acc + (int64_t)row * d + col);
+  const float4 x = src[0], y = src[1];
+  const int64_t o = a.dq.off(b, n, f.N, a.dq_col0 + col);
+  if (f.dtype == JAGG_DTYPE_F32) {
+    float4* dst = reinterpret_cast<float4*>(static_cast<float*>(a.dq.base(n)) + o);
+    dst[0] = x;
+    dst[1] = y;
+  } else {
+    uint4 raw;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&raw);
+    h[0] = __floats2bfloat162_rn(x.x, x.y);
+    h[1] = __floats2bfloat162_rn(x.z, x.w);
+    h[2] = __floats2bfloat162_rn(y.x, y.y);
+    h[3] = __floats2bfloat162_rn(y.z, y.w);
+    *reinterpret_cast<uint4*>(static_cast<bf16*>(a.dq.base(n)) + o) = raw;
   }
 }
 
@@ -488,7 +563,7 @@ int fwd_tc(const AttnArgs& a, cudaStream_t s) {
 }
 template <int D>
 int bwd_tc(const AttnBwdArgs& a, cudaStream_t s) {
-  const int smem = 4 * TILE * (D + 8) * 2 + TILE * (TILE + 8) * 2 + 2 * TILE * 4;
+  const int smem = BwdCfg<D>::SMEM;
   static bool set = false;
   if (!set) {
     JAGG_CUDA_TRY(cudaFuncSetAttribute(fa_bwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
@@ -522,8 +597,15 @@ int bwd_simt(const AttnBwdArgs& a, cudaStream_t s) {
 
 }  // namespace
 
+static int64_t dv_floats_padded(int B, int N, int heads) { return ((int64_t)B * heads * N + 63) / 64 * 64; }
+
 int64_t attention_bwd_scratch_floats(int B, int N, int heads, int dh) {
-  return (int64_t)B * heads * N + (int64_t)B * N * heads * dh;
+  return dv_floats_padded(B, N, heads) + (int64_t)B * N * heads * dh;
+}
+
+void attention_bwd_scratch(float* scratch, int B, int N, int heads, float** Dv, float** dq_acc) {
+  *Dv = scratch;
+  *dq_acc = scratch + dv_floats_padded(B, N, heads);
 }
 
 int attention_fwd(const AttnArgs& a, cudaStream_t s) {
@@ -545,10 +627,15 @@ int attention_fwd(const AttnArgs& a, cudaStream_t s) {
 int attention_bwd(const AttnBwdArgs& a, cudaStream_t s) {
   const AttnArgs& f = a.f;
   JAGG_CHECK_ARG(f.B > 0 && f.N > 0 && f.heads > 0, "attention: empty shape");
-  JAGG_CUDA_TRY(cudaMemsetAsync(a.dq_acc, 0, sizeof(float) * (size_t)f.B * f.N * f.heads * f.dh, s));
-  const int64_t warps = (int64_t)f.B * f.N * f.heads;
-  rowdot_kernel<<<(int)((warps * 32 + 255) / 256), 256, 0, s>>>(a);
+  JAGG_CHECK_ARG((reinterpret_cast<uintptr_t>(a.dq_acc) & 15) == 0 && (f.heads * f.dh) % 4 == 0,
+                 "attention: dq accumulator must be 16-byte aligned with a row pitch of 4k floats");
+  JAGG_CHECK_ARG(f.dh % 8 == 0 && f.dh <= 256, "attention: head dim %d unsupported", f.dh);
+  const int64_t chunks = (int64_t)f.B * f.N * f.heads * f.dh / 8;
+  JAGG_CHECK_ARG(chunks < (1ll << 31), "attention: too many rows");
+  int tok = prof_start(s);
+  rowdot_zero_kernel<<<(int)((chunks + 255) / 256), 256, 0, s>>>(a);
   JAGG_LAUNCHED();
+  prof_stop(tok, s, PROF_ATTN_AUX, 0.0, 4.0 * f.B * f.N * f.heads * f.dh * 1.5);
   int st = JAGG_ERR_UNSUPPORTED;
   if (f.dtype == JAGG_DTYPE_BF16 && f.dh == 64)
     st = bwd_tc<64>(a, s);
@@ -567,8 +654,10 @@ int attention_bwd(const AttnBwdArgs& a, cudaStream_t s) {
     return st;
   }
   const int64_t total = (int64_t)f.B * f.N * f.heads * f.dh;
-  dq_store_kernel<<<(int)std::min<int64_t>((total + 255) / 256, 1 << 20), 256, 0, s>>>(a);
+  tok = prof_start(s);
+  dq_store_kernel<<<(int)((chunks + 255) / 256), 256, 0, s>>>(a);
   JAGG_LAUNCHED();
+  prof_stop(tok, s, PROF_ATTN_AUX, 0.0, 6.0 * total);
   return JAGG_OK;
 }
 

@@ -42,8 +42,11 @@ struct AttnBwdArgs {
 };
 
 int attention_fwd(const AttnArgs& a, cudaStream_t s);
-// Scratch: Dv and dq_acc as described above (sizes from attention_bwd_scratch_floats).
+// Scratch: Dv and dq_acc as described above.  dq_acc must be 16-byte aligned (it receives
+// 16-byte vector reductions); attention_bwd_scratch places both in one buffer of
+// attention_bwd_scratch_floats floats with dq_acc at a 256-byte boundary.
 int attention_bwd(const AttnBwdArgs& a, cudaStream_t s);
 int64_t attention_bwd_scratch_floats(int B, int N, int heads, int dh);
+void attention_bwd_scratch(float* scratch, int B, int N, int heads, float** Dv, float** dq_acc);
 
 }  // namespace jagg

@@ -112,7 +112,15 @@ int sm_count();
 // bracketed by CUDA events on their stream and attributed to a kernel family with their
 // algorithmic FLOPs and bytes.
 void count_launch();
-enum ProfFamily : int { PROF_GEMM_TC = 0, PROF_GEMM_SIMT, PROF_ATTN_FWD, PROF_ATTN_BWD, PROF_FAMILIES };
+enum ProfFamily : int {
+  PROF_GEMM_TC = 0,
+  PROF_GEMM_SIMT,
+  PROF_ATTN_FWD,
+  PROF_ATTN_BWD,
+  PROF_LN_BWD,     // LayerNorm + gate backward
+  PROF_ATTN_AUX,   // attention backward helpers (rowsum(dO O), dQ conversion)
+  PROF_FAMILIES
+};
 int prof_start(cudaStream_t s);  // returns a token, or -1 when profiling is off
 void prof_stop(int token, cudaStream_t s, int family, double flops, double bytes, int m = 0, int n = 0, int k = 0);
 

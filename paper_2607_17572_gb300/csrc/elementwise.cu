@@ -158,11 +158,7 @@ __global__ void ln_mod_fwd_kernel(LnModFwd a) {
   }
 }
 
-// Backward of LayerNorm + modulation and of the gated residual branch, in two passes:
-//   rows:    one warp per row forms the LayerNorm input-gradient (added to the residual
-//            gradient dh) and dy = gate * dh;
-//   columns: per sequence and column, sums over the sequence's rows give dshift, dscale,
-//            dgate and the bias gradient (sum_m dy = gate * sum_m dh), with coalesced loads.
+// Backward of LayerNorm + modulation and of a gated residual branch.
 __device__ __forceinline__ void load4(const void* p, int64_t i, int is_f32, float (&v)[4]) {
   if (is_f32) {
     const float4 f = *reinterpret_cast<const float4*>(static_cast<const float*>(p) + i);
@@ -186,108 +182,140 @@ __device__ __forceinline__ void store4(void* p, int64_t i, int is_f32, const flo
   }
 }
 
-__global__ void ln_gate_rows_kernel(LnGateBwd a) {
-  const int warps = blockDim.x / 32;
-  const int m = blockIdx.x * warps + threadIdx.x / 32;
-  const int lane = threadIdx.x & 31;
-  if (m >= a.M) return;
-  const int d = a.d;
-  const int64_t hr = seg_row(m, a.seg, a.seg_off, a.seg_stride);
-  const int b = m / a.rows_per_seq;
+// One pass per row tile: a block of 8 warps takes LNF_ROWS rows of one sequence, each warp
+// LNF_R of them.  Per row: the LayerNorm input-gradient (added to the residual gradient
+// dh) and dy = gate * dh.  The per-sequence column sums (dshift, dscale, dgate, and sum dh
+// for the bias gradient: sum_m dy = gate * sum_m dh) are summed over a warp's rows in
+// registers, then over the block in shared memory (laid out [quantity][element][d/4] so a
+// warp's atomics hit consecutive words), then flushed with one global atomic per column.
+constexpr int LNF_R = 4;
+constexpr int LNF_ROWS = 8 * LNF_R;
+
+__global__ void __launch_bounds__(256) ln_gate_fused_kernel(LnGateBwd a) {
+  extern __shared__ float part[];  // [4 quantities][4][d/4]
+  const int d = a.d, d4 = a.d / 4;
+  const int chunks = (a.rows_per_seq + LNF_ROWS - 1) / LNF_ROWS;
+  const int b = blockIdx.x / chunks;
+  const int r0 = (blockIdx.x % chunks) * LNF_ROWS;
+  for (int i = threadIdx.x; i < 4 * d; i += blockDim.x) part[i] = 0.f;
+  __syncthreads();
+  const int warp = threadIdx.x / 32, lane = threadIdx.x & 31;
   const int is_f32 = a.dtype == JAGG_DTYPE_F32;
   const int nv = (d + 127) / 128;
   const float* gate = a.do_gate ? a.gate + (int64_t)b * a.mod_stride : nullptr;
+  const float* sc = a.do_ln ? a.scale + (int64_t)b * a.mod_stride : nullptr;
+  int mrow[LNF_R];
+  int64_t hrow[LNF_R];
+  bool live[LNF_R];
+  float mu[LNF_R], rs[LNF_R], s1[LNF_R], s2[LNF_R];
+#pragma unroll
+  for (int k = 0; k < LNF_R; ++k) {
+    const int r = r0 + warp * LNF_R + k;
+    live[k] = r < a.rows_per_seq;
+    mrow[k] = b * a.rows_per_seq + (live[k] ? r : 0);
+    hrow[k] = seg_row(mrow[k], a.seg, a.seg_off, a.seg_stride);
+    mu[k] = rs[k] = s1[k] = s2[k] = 0.f;
+  }
   if (a.do_ln) {
-    const float mu = a.mean[m], rs = a.rstd[m];
-    const float* sc = a.scale + (int64_t)b * a.mod_stride;
-    float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+    for (int k = 0; k < LNF_R; ++k) {
+      if (live[k]) {
+        mu[k] = a.mean[mrow[k]];
+        rs[k] = a.rstd[mrow[k]];
+      }
+    }
     for (int i = 0; i < nv; ++i) {
       const int c = (i * 32 + lane) * 4;
-      if (c < d) {
+      if (c >= d) continue;
+      const float4 s4 = *reinterpret_cast<const float4*>(sc + c);
+      const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
+#pragma unroll
+      for (int k = 0; k < LNF_R; ++k) {
+        if (!live[k]) continue;
         float dm[4];
-        load4(a.dm, (int64_t)m * d + c, a.dm_f32, dm);
-        const float4 h4 = *reinterpret_cast<const float4*>(a.h + hr * d + c);
-        const float4 s4 = *reinterpret_cast<const float4*>(sc + c);
-        const float hv[4] = {h4.x, h4.y, h4.z, h4.w}, sv[4] = {s4.x, s4.y, s4.z, s4.w};
+        load4(a.dm, (int64_t)mrow[k] * d + c, a.dm_f32, dm);
+        const float4 h4 = *reinterpret_cast<const float4*>(a.h + hrow[k] * d + c);
+        const float hv[4] = {h4.x, h4.y, h4.z, h4.w};
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const float dxh = dm[e] * (1.f + sv[e]);
-          s1 += dxh;
-          s2 += dxh * (hv[e] - mu) * rs;
+          s1[k] += dxh;
+          s2[k] += dxh * (hv[e] - mu[k]) * rs[k];
         }
       }
     }
-    s1 = warp_sum(s1) / d;
-    s2 = warp_sum(s2) / d;
-    for (int i = 0; i < nv; ++i) {
-      const int c = (i * 32 + lane) * 4;
-      if (c < d) {
+#pragma unroll
+    for (int k = 0; k < LNF_R; ++k) {
+      s1[k] = warp_sum(s1[k]) / d;
+      s2[k] = warp_sum(s2[k]) / d;
+    }
+  }
+  for (int i = 0; i < nv; ++i) {
+    const int c = (i * 32 + lane) * 4;
+    if (c >= d) continue;
+    float acc[4][4];  // [quantity][element]
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) acc[q][e] = 0.f;
+    float sv[4] = {0.f, 0.f, 0.f, 0.f}, gv[4] = {0.f, 0.f, 0.f, 0.f};
+    if (a.do_ln) {
+      const float4 s4 = *reinterpret_cast<const float4*>(sc + c);
+      sv[0] = s4.x; sv[1] = s4.y; sv[2] = s4.z; sv[3] = s4.w;
+    }
+    if (gate) {
+      const float4 g4 = *reinterpret_cast<const float4*>(gate + c);
+      gv[0] = g4.x; gv[1] = g4.y; gv[2] = g4.z; gv[3] = g4.w;
+    }
+#pragma unroll
+    for (int k = 0; k < LNF_R; ++k) {
+      if (!live[k]) continue;
+      const float4 d4 = *reinterpret_cast<const float4*>(a.dh_in + hrow[k] * d + c);
+      float dh[4] = {d4.x, d4.y, d4.z, d4.w};
+      if (a.do_ln) {
         float dm[4];
-        load4(a.dm, (int64_t)m * d + c, a.dm_f32, dm);
-        const float4 h4 = *reinterpret_cast<const float4*>(a.h + hr * d + c);
-        const float4 s4 = *reinterpret_cast<const float4*>(sc + c);
-        const float4 d4 = *reinterpret_cast<const float4*>(a.dh_in + hr * d + c);
-        const float hv[4] = {h4.x, h4.y, h4.z, h4.w}, sv[4] = {s4.x, s4.y, s4.z, s4.w};
-        float dh[4] = {d4.x, d4.y, d4.z, d4.w};
+        load4(a.dm, (int64_t)mrow[k] * d + c, a.dm_f32, dm);
+        const float4 h4 = *reinterpret_cast<const float4*>(a.h + hrow[k] * d + c);
+        const float hv[4] = {h4.x, h4.y, h4.z, h4.w};
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          const float xh = (hv[e] - mu) * rs;
-          dh[e] += rs * (dm[e] * (1.f + sv[e]) - s1 - xh * s2);
+          const float xh = (hv[e] - mu[k]) * rs[k];
+          dh[e] += rs[k] * (dm[e] * (1.f + sv[e]) - s1[k] - xh * s2[k]);
+          acc[0][e] += dm[e];
+          acc[1][e] += dm[e] * xh;
         }
-        *reinterpret_cast<float4*>(a.dh_out + hr * d + c) = make_float4(dh[0], dh[1], dh[2], dh[3]);
-        if (gate) {
-          const float4 g4 = *reinterpret_cast<const float4*>(gate + c);
-          const float dy[4] = {g4.x * dh[0], g4.y * dh[1], g4.z * dh[2], g4.w * dh[3]};
-          store4(a.dy, (int64_t)m * d + c, is_f32, dy);
+        *reinterpret_cast<float4*>(a.dh_out + hrow[k] * d + c) = make_float4(dh[0], dh[1], dh[2], dh[3]);
+      }
+      if (gate) {
+        const float dy[4] = {gv[0] * dh[0], gv[1] * dh[1], gv[2] * dh[2], gv[3] * dh[3]};
+        store4(a.dy, (int64_t)mrow[k] * d + c, is_f32, dy);
+        float yv[4];
+        load4(a.y, (int64_t)mrow[k] * d + c, is_f32, yv);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          acc[2][e] += dh[e] * yv[e];
+          acc[3][e] += dh[e];
         }
       }
     }
-  } else if (gate) {
-    for (int i = 0; i < nv; ++i) {
-      const int c = (i * 32 + lane) * 4;
-      if (c < d) {
-        const float4 d4 = *reinterpret_cast<const float4*>(a.dh_in + hr * d + c);
-        const float4 g4 = *reinterpret_cast<const float4*>(gate + c);
-        const float dy[4] = {g4.x * d4.x, g4.y * d4.y, g4.z * d4.z, g4.w * d4.w};
-        store4(a.dy, (int64_t)m * d + c, is_f32, dy);
-      }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      if (q < 2 ? !a.do_ln : !gate) continue;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) atomicAdd(&part[(q * 4 + e) * d4 + c / 4], acc[q][e]);
     }
   }
-}
-
-constexpr int LNC_ROWS = 32;
-// grid: (ceil(d / 256), sequences, ceil(rows_per_seq / LNC_ROWS)); one thread per column.
-__global__ void ln_gate_cols_kernel(LnGateBwd a) {
-  const int c = blockIdx.x * blockDim.x + threadIdx.x;
-  const int b = blockIdx.y;
-  const int r0 = blockIdx.z * LNC_ROWS;
-  if (c >= a.d || r0 >= a.rows_per_seq) return;
-  const int r1 = min(r0 + LNC_ROWS, a.rows_per_seq);
-  const int d = a.d;
-  const int is_f32 = a.dtype == JAGG_DTYPE_F32;
-  const float* dh = a.do_ln ? a.dh_out : a.dh_in;
-  float psh = 0.f, psc = 0.f, pg = 0.f, pdh = 0.f;
-  for (int r = r0; r < r1; ++r) {
-    const int m = b * a.rows_per_seq + r;
-    const int64_t hr = seg_row(m, a.seg, a.seg_off, a.seg_stride);
+  __syncthreads();
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    auto P = [&](int q) { return part[(q * 4 + c % 4) * d4 + c / 4]; };
     if (a.do_ln) {
-      const float dmv = ldx(a.dm, (int64_t)m * d + c, a.dm_f32);
-      psh += dmv;
-      psc += dmv * (a.h[hr * d + c] - a.mean[m]) * a.rstd[m];
+      atomicAdd(a.dshift + (int64_t)b * a.dmod_stride + c, P(0));
+      atomicAdd(a.dscale + (int64_t)b * a.dmod_stride + c, P(1));
     }
     if (a.do_gate) {
-      const float g = dh[hr * d + c];
-      pg += g * ldx(a.y, (int64_t)m * d + c, is_f32);
-      pdh += g;
+      atomicAdd(a.dgate + (int64_t)b * a.dmod_stride + c, P(2));
+      if (a.dbias) atomicAdd(a.dbias + c, gate[c] * P(3));
     }
-  }
-  if (a.do_ln) {
-    atomicAdd(a.dshift + (int64_t)b * a.dmod_stride + c, psh);
-    atomicAdd(a.dscale + (int64_t)b * a.dmod_stride + c, psc);
-  }
-  if (a.do_gate) {
-    atomicAdd(a.dgate + (int64_t)b * a.dmod_stride + c, pg);
-    if (a.dbias) atomicAdd(a.dbias + c, a.gate[(int64_t)b * a.mod_stride + c] * pdh);
   }
 }
 
@@ -356,12 +384,10 @@ __device__ __forceinline__ void rope_angle(int n, int n_txt, int gw, int dh, int
   }
   const int tok = n - n_txt;
   const int axis = pair / npair, i = pair % npair;
-  const double pos = axis == 0 ? (double)(tok / gw) : (double)(tok % gw);
-  const double th = exp(-log(10000.0) * 2.0 * (double)i / (double)hd);
-  double s, c;
-  sincos(pos * th, &s, &c);
-  cs = (float)c;
-  sn = (float)s;
+  // f32: the angle pos * theta (pos < grid size) is off by a few 1e-6 rad at most
+  const float pos = axis == 0 ? (float)(tok / gw) : (float)(tok % gw);
+  const float th = exp2f(-13.287712379549449f * 2.f * (float)i / (float)hd);  // 10000^(-2i/hd)
+  sincosf(pos * th, &sn, &cs);
 }
 
 __global__ void qk_norm_rope_fwd_kernel(QkNormRope a) {
@@ -501,14 +527,24 @@ int launch_ln_mod_fwd(const LnModFwd& a, cudaStream_t s) {
   return JAGG_OK;
 }
 int launch_ln_gate_bwd(const LnGateBwd& a, cudaStream_t s) {
-  JAGG_CHECK_ARG(a.d % 4 == 0, "ln_gate_bwd: hidden %d not a multiple of 4", a.d);
+  JAGG_CHECK_ARG(a.d % 4 == 0 && a.d <= 3072, "ln_gate_bwd: hidden %d unsupported", a.d);
   JAGG_CHECK_ARG(a.M % a.rows_per_seq == 0, "ln_gate_bwd: rows not a whole number of sequences");
   if (!a.do_ln && !a.do_gate) return JAGG_OK;
-  ln_gate_rows_kernel<<<ceil_div(a.M, 8), 256, 0, s>>>(a);
+  const int smem = 4 * a.d * (int)sizeof(float);
+  static bool attr = false;
+  if (!attr) {
+    JAGG_CUDA_TRY(cudaFuncSetAttribute(ln_gate_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       4 * 3072 * (int)sizeof(float)));
+    attr = true;
+  }
+  const int blocks = (a.M / a.rows_per_seq) * ceil_div(a.rows_per_seq, LNF_ROWS);
+  const int tok = prof_start(s);
+  ln_gate_fused_kernel<<<blocks, 256, smem, s>>>(a);
   JAGG_LAUNCHED();
-  const dim3 grid(ceil_div(a.d, 256), a.M / a.rows_per_seq, ceil_div(a.rows_per_seq, LNC_ROWS));
-  ln_gate_cols_kernel<<<grid, 256, 0, s>>>(a);
-  JAGG_LAUNCHED();
+  // algorithmic bytes: dh read + write (f32), dm (f32), h (f32), y and dy (storage type)
+  const double elem = (double)a.M * a.d;
+  prof_stop(tok, s, PROF_LN_BWD, 0.0,
+            elem * ((a.do_ln ? 16.0 : 4.0) + (a.do_gate ? 2.0 * (a.dtype == JAGG_DTYPE_F32 ? 4 : 2) : 0.0)));
   return JAGG_OK;
 }
 int launch_colsum(const void* X, int x_f32, int dtype, int rows, int cols, int64_t ld, float* db, cudaStream_t s) {

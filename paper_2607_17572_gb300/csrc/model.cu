@@ -45,6 +45,20 @@ struct DitBlockW {
   int64_t mod_col;  // offset of this block's segment inside the stacked modulation output
 };
 
+// One stream (text or image) of an MMDiT double block.
+struct StreamW {
+  int64_t qkv_w, qkv_b, qn, kn, proj_w, proj_b, fc1_w, fc1_b, fc2_w, fc2_b;
+  int64_t mod_col;
+};
+struct DoubleW {
+  StreamW s[2];  // 0 = text, 1 = image
+};
+// Flux-style single block: lin1 -> [qkv | u], lin2 on [o | GELU(u)].
+struct SingleW {
+  int64_t lin1_w, lin1_b, qn, kn, lin2_w, lin2_b;
+  int64_t mod_col;
+};
+
 struct ParamTable {
   std::vector<TensorInfo> t;
   int64_t total = 0;
@@ -54,6 +68,8 @@ struct ParamTable {
   int64_t final_mod_col;
   int64_t out_w, out_b;
   std::vector<DitBlockW> blocks;
+  std::vector<DoubleW> doubles;
+  std::vector<SingleW> singles;
 };
 
 static int64_t align64(int64_t x) { return (x + 63) / 64 * 64; }
@@ -75,13 +91,27 @@ static bool build_table(const jagg_config& c, ParamTable& T) {
   T.t_b1 = add("t_embed.b1", d, 1);
   T.t_w2 = add("t_embed.w2", d, d);
   T.t_b2 = add("t_embed.b2", d, 1);
-  if (c.arch != JAGG_ARCH_DIT) return false;
-  // stacked modulation: every block's [6d, d] then the final layer's [2d, d]
+  const bool mm = c.arch == JAGG_ARCH_MMDIT;
+  const int64_t dh = c.hidden / c.heads;
+  // stacked modulation: every block's rows (DiT: [6d, d]; MMDiT: [6d, d] per stream of a
+  // double block, [3d, d] per single block), then the final layer's [2d, d]
   std::vector<std::string> mods;
   std::vector<int64_t> mrows;
-  for (int i = 0; i < c.depth; ++i) {
-    mods.push_back("blocks." + std::to_string(i) + ".mod");
-    mrows.push_back(6 * d);
+  if (!mm) {
+    for (int i = 0; i < c.depth; ++i) {
+      mods.push_back("blocks." + std::to_string(i) + ".mod");
+      mrows.push_back(6 * d);
+    }
+  } else {
+    for (int i = 0; i < c.depth_double; ++i)
+      for (const char* s : {"txt", "img"}) {
+        mods.push_back("double." + std::to_string(i) + "." + s + ".mod");
+        mrows.push_back(6 * d);
+      }
+    for (int i = 0; i < c.depth; ++i) {
+      mods.push_back("single." + std::to_string(i) + ".mod");
+      mrows.push_back(3 * d);
+    }
   }
   mods.push_back("final.mod");
   mrows.push_back(2 * d);
@@ -99,7 +129,41 @@ static bool build_table(const jagg_config& c, ParamTable& T) {
     if (i == 0) T.mod_b = o;
   }
   T.final_mod_col = mcol.back();
-  for (int i = 0; i < c.depth; ++i) {
+  if (mm) {
+    size_t mi = 0;
+    for (int i = 0; i < c.depth_double; ++i) {
+      DoubleW w;
+      for (int si = 0; si < 2; ++si) {
+        const std::string p = "double." + std::to_string(i) + (si == 0 ? ".txt." : ".img.");
+        StreamW& s = w.s[si];
+        s.mod_col = mcol[mi++];
+        s.qkv_w = add(p + "qkv.w", 3 * d, d);
+        s.qkv_b = add(p + "qkv.b", 3 * d, 1);
+        s.qn = add(p + "q_norm", dh, 1);
+        s.kn = add(p + "k_norm", dh, 1);
+        s.proj_w = add(p + "proj.w", d, d);
+        s.proj_b = add(p + "proj.b", d, 1);
+        s.fc1_w = add(p + "fc1.w", dm, d);
+        s.fc1_b = add(p + "fc1.b", dm, 1);
+        s.fc2_w = add(p + "fc2.w", d, dm);
+        s.fc2_b = add(p + "fc2.b", d, 1);
+      }
+      T.doubles.push_back(w);
+    }
+    for (int i = 0; i < c.depth; ++i) {
+      const std::string p = "single." + std::to_string(i) + ".";
+      SingleW w;
+      w.mod_col = mcol[mi++];
+      w.lin1_w = add(p + "lin1.w", 3 * d + dm, d);
+      w.lin1_b = add(p + "lin1.b", 3 * d + dm, 1);
+      w.qn = add(p + "q_norm", dh, 1);
+      w.kn = add(p + "k_norm", dh, 1);
+      w.lin2_w = add(p + "lin2.w", d, d + dm);
+      w.lin2_b = add(p + "lin2.b", d, 1);
+      T.singles.push_back(w);
+    }
+  }
+  for (int i = 0; i < (mm ? 0 : c.depth); ++i) {
     const std::string p = "blocks." + std::to_string(i) + ".";
     DitBlockW w;
     w.mod_col = mcol[i];
@@ -504,20 +568,27 @@ int vjp_impl(const jagg_model& m, const void* saved, int B, const float* cot, fl
     a.dtype = dt;
     JAGG_TRY(launch_ln_gate_bwd(a, s));
   }
+  // Gate of block l's MLP branch (dg2, dy2 = g2 dh, db_fc2): for the last block a pass of
+  // its own; for the others fused into the LayerNorm-1 backward of block l + 1, which
+  // produces exactly that gradient.
+  auto mlp_gate = [&](LnGateBwd& a, int l) {
+    const DitBlockW& bw = m.T.blocks[l];
+    a.do_gate = 1; a.y = S.blk[l].y2; a.gate = S.mod + bw.mod_col + 5 * d; a.mod_stride = Lm;
+    a.dgate = w.dmod + bw.mod_col + 5 * d; a.dmod_stride = Lm; a.dy = w.dy; a.dbias = grad + bw.fc2_b;
+  };
+  if (c.depth > 0) {
+    LnGateBwd a{};
+    a.M = M; a.d = d; a.rows_per_seq = N;
+    a.do_ln = 0; a.dh_in = w.dh; a.dh_out = w.dh; a.dtype = dt;
+    mlp_gate(a, c.depth - 1);
+    JAGG_TRY(launch_ln_gate_bwd(a, s));
+  }
   // blocks, last to first
   for (int l = c.depth - 1; l >= 0; --l) {
     const DitBlockW& bw = m.T.blocks[l];
     const DitSaved& k = S.blk[l];
     const float* mod = S.mod + bw.mod_col;
     float* dmod = w.dmod + bw.mod_col;
-    {  // gate of the MLP branch: dg2, dy2 = g2 dh, db_fc2
-      LnGateBwd a{};
-      a.M = M; a.d = d; a.rows_per_seq = N;
-      a.do_ln = 0; a.dh_in = w.dh; a.dh_out = w.dh;
-      a.do_gate = 1; a.y = k.y2; a.gate = mod + 5 * d; a.mod_stride = Lm; a.dgate = dmod + 5 * d;
-      a.dmod_stride = Lm; a.dy = w.dy; a.dbias = grad + bw.fc2_b; a.dtype = dt;
-      JAGG_TRY(launch_ln_gate_bwd(a, s));
-    }
     JAGG_TRY(gemm(dw_gemm(m, M, d, dmw, w.dy, d, k.gu, dmw, grad, bw.fc2_w), s));
     {
       GemmArgs g = dx_gemm(m, M, d, dmw, w.dy, d, bw.fc2_w);
@@ -556,8 +627,7 @@ int vjp_impl(const jagg_model& m, const void* saved, int B, const float* cot, fl
       at.o = seg_single(k.o, d, N);
       at.lse = k.lse; at.dtype = dt;
       ab.dO = seg_single(w.dO, d, N);
-      ab.Dv = w.attn;
-      ab.dq_acc = w.attn + (int64_t)B * m.heads * N;
+      attention_bwd_scratch(w.attn, B, N, m.heads, &ab.Dv, &ab.dq_acc);
       ab.dq = ab.dk = ab.dv = seg_single(w.dqkv, 3 * d, N);
       ab.dq_col0 = 0; ab.dk_col0 = d; ab.dv_col0 = 2 * d;
       JAGG_TRY(attention_bwd(ab, s));
@@ -569,12 +639,13 @@ int vjp_impl(const jagg_model& m, const void* saved, int B, const float* cot, fl
       g.C = w.dx32; g.ldc = d; g.c_dtype = JAGG_DTYPE_F32;
       JAGG_TRY(gemm(g, s));
     }
-    {  // LN1 + modulation backward
+    {  // LN1 + modulation backward, then the previous block's MLP gate
       LnGateBwd a{};
       a.M = M; a.d = d; a.rows_per_seq = N;
       a.do_ln = 1; a.dm = w.dx32; a.dm_f32 = 1; a.h = k.h_in; a.mean = k.st1; a.rstd = k.st1 + M;
       a.scale = mod + d; a.mod_stride = Lm; a.dshift = dmod; a.dscale = dmod + d; a.dmod_stride = Lm;
       a.dh_in = w.dh; a.dh_out = w.dh; a.dtype = dt;
+      if (l > 0) mlp_gate(a, l - 1);
       JAGG_TRY(launch_ln_gate_bwd(a, s));
     }
   }

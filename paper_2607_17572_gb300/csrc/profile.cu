@@ -33,7 +33,8 @@ cudaEvent_t get_event() {
   return e;
 }
 
-const char* kFamilyNames[PROF_FAMILIES] = {"gemm_tcgen05", "gemm_simt", "attention_fwd", "attention_bwd"};
+const char* kFamilyNames[PROF_FAMILIES] = {"gemm_tcgen05",  "gemm_simt",   "attention_fwd",
+                                           "attention_bwd", "ln_gate_bwd", "attention_bwd_aux"};
 
 }  // namespace
 
@@ -122,6 +123,7 @@ extern "C" int jagg_profile_launches(jagg_profile_launch* out, int cap, int* n_o
     o.k = r.k;
     o.ms = ms;
     o.flops = r.flops;
+    o.bytes = r.bytes;
   }
   *n_out = n;
   return JAGG_OK;

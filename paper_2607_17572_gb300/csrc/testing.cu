@@ -53,8 +53,7 @@ extern "C" int jagg_test_attention_bwd(const void* qkv, const void* o, const flo
   ab.f = make_args(qkv, B, N, heads, dh, dtype, const_cast<void*>(o), const_cast<float*>(lse));
   const int d = heads * dh;
   ab.dO = seg_single(const_cast<void*>(dO), d, N);
-  ab.Dv = static_cast<float*>(scratch);
-  ab.dq_acc = ab.Dv + (int64_t)B * heads * N;
+  attention_bwd_scratch(static_cast<float*>(scratch), B, N, heads, &ab.Dv, &ab.dq_acc);
   ab.dq = ab.dk = ab.dv = seg_single(dqkv, 3 * d, N);
   ab.dq_col0 = 0; ab.dk_col0 = d; ab.dv_col0 = 2 * d;
   return attention_bwd(ab, stream);
