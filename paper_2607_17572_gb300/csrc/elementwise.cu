@@ -390,95 +390,134 @@ __device__ __forceinline__ void rope_angle(int n, int n_txt, int gw, int dh, int
   sincosf(pos * th, &sn, &cs);
 }
 
-__global__ void qk_norm_rope_fwd_kernel(QkNormRope a) {
-  const int64_t w = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) / 32;
+// Grid-stride over (row, head) items, one warp per item; lane j owns the rotated pairs j
+// and j + 32 of the head.
+constexpr int QKN_THREADS = 256, QKN_WARPS = QKN_THREADS / 32;
+
+__global__ void __launch_bounds__(QKN_THREADS) qk_norm_rope_fwd_kernel(QkNormRope a) {
   const int lane = threadIdx.x & 31;
-  if (w >= (int64_t)a.M * a.heads) return;
-  const int hd = (int)(w % a.heads);
-  const int m = (int)(w / a.heads);
-  const int n = m % a.N;
   const int dh = a.d / a.heads;
   const int is_f32 = a.dtype == JAGG_DTYPE_F32;
-  const bool txt = n < a.n_txt;
-  for (int which = 0; which < 2; ++which) {
-    const void* scl = which == 0 ? (txt ? a.qscale_txt : a.qscale_img) : (txt ? a.kscale_txt : a.kscale_img);
-    const int64_t base = (int64_t)m * a.ld_qkv + which * a.d + hd * dh;
-    float x[4] = {0.f, 0.f, 0.f, 0.f};
-    float ss = 0.f;
-    for (int j = 0; j < 2; ++j) {
-      const int pair = lane + 32 * j;
-      if (2 * pair < dh) {
-        x[2 * j] = ldx(a.qkv, base + 2 * pair, is_f32);
-        x[2 * j + 1] = ldx(a.qkv, base + 2 * pair + 1, is_f32);
-        ss += x[2 * j] * x[2 * j] + x[2 * j + 1] * x[2 * j + 1];
+  const int64_t items = (int64_t)a.M * a.heads;
+  for (int64_t w = (int64_t)blockIdx.x * QKN_WARPS + threadIdx.x / 32; w < items;
+       w += (int64_t)gridDim.x * QKN_WARPS) {
+    const int hd = (int)(w % a.heads);
+    const int m = (int)(w / a.heads);
+    const int n = m % a.N;
+    const bool txt = n < a.n_txt;
+    for (int which = 0; which < 2; ++which) {
+      const void* scl = which == 0 ? (txt ? a.qscale_txt : a.qscale_img) : (txt ? a.kscale_txt : a.kscale_img);
+      const int64_t base = (int64_t)m * a.ld_qkv + which * a.d + hd * dh;
+      float x[4] = {0.f, 0.f, 0.f, 0.f};
+      float ss = 0.f;
+      for (int j = 0; j < 2; ++j) {
+        const int pair = lane + 32 * j;
+        if (2 * pair < dh) {
+          x[2 * j] = ldx(a.qkv, base + 2 * pair, is_f32);
+          x[2 * j + 1] = ldx(a.qkv, base + 2 * pair + 1, is_f32);
+          ss += x[2 * j] * x[2 * j] + x[2 * j + 1] * x[2 * j + 1];
+        }
       }
-    }
-    const float r = rsqrtf(warp_sum(ss) / dh + 1e-6f);
-    for (int j = 0; j < 2; ++j) {
-      const int pair = lane + 32 * j;
-      if (2 * pair < dh) {
-        const float y0 = x[2 * j] * r * ldx(scl, 2 * pair, is_f32);
-        const float y1 = x[2 * j + 1] * r * ldx(scl, 2 * pair + 1, is_f32);
-        float cs = 1.f, sn = 0.f;
-        if (a.rope) rope_angle(n, a.n_txt, a.gw, dh, pair, cs, sn);
-        const int64_t o = (int64_t)m * 2 * a.d + which * a.d + hd * dh + 2 * pair;
-        stx(a.qk_out, o, is_f32, y0 * cs - y1 * sn);
-        stx(a.qk_out, o + 1, is_f32, y0 * sn + y1 * cs);
+      const float r = rsqrtf(warp_sum(ss) / dh + 1e-6f);
+      for (int j = 0; j < 2; ++j) {
+        const int pair = lane + 32 * j;
+        if (2 * pair < dh) {
+          const float y0 = x[2 * j] * r * ldx(scl, 2 * pair, is_f32);
+          const float y1 = x[2 * j + 1] * r * ldx(scl, 2 * pair + 1, is_f32);
+          float cs = 1.f, sn = 0.f;
+          if (a.rope) rope_angle(n, a.n_txt, a.gw, dh, pair, cs, sn);
+          const int64_t o = (int64_t)m * 2 * a.d + which * a.d + hd * dh + 2 * pair;
+          stx(a.qk_out, o, is_f32, y0 * cs - y1 * sn);
+          stx(a.qk_out, o + 1, is_f32, y0 * sn + y1 * cs);
+        }
       }
+      if (lane == 0) (which == 0 ? a.rq : a.rk)[(int64_t)m * a.heads + hd] = r;
     }
-    if (lane == 0) (which == 0 ? a.rq : a.rk)[(int64_t)m * a.heads + hd] = r;
   }
 }
 
-__global__ void qk_norm_rope_bwd_kernel(QkNormRopeBwd b) {
+// The scale gradients sum over every (row, head): each lane keeps its elements' partial
+// sums in registers (q / k x text / image), the block adds its warps' partials in shared
+// memory and issues one atomic per element.
+__global__ void __launch_bounds__(QKN_THREADS) qk_norm_rope_bwd_kernel(QkNormRopeBwd b) {
   const QkNormRope& a = b.f;
-  const int64_t w = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) / 32;
-  const int lane = threadIdx.x & 31;
-  if (w >= (int64_t)a.M * a.heads) return;
-  const int hd = (int)(w % a.heads);
-  const int m = (int)(w / a.heads);
-  const int n = m % a.N;
+  __shared__ float part[QKN_WARPS][4][128];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x / 32;
   const int dh = a.d / a.heads;
   const int is_f32 = a.dtype == JAGG_DTYPE_F32;
-  const bool txt = n < a.n_txt;
-  for (int which = 0; which < 2; ++which) {
-    const void* scl = which == 0 ? (txt ? a.qscale_txt : a.qscale_img) : (txt ? a.kscale_txt : a.kscale_img);
-    float* dscl = which == 0 ? (txt ? b.dqs_txt : b.dqs_img) : (txt ? b.dks_txt : b.dks_img);
-    const float r = (which == 0 ? a.rq : a.rk)[(int64_t)m * a.heads + hd];
-    const int64_t xb = (int64_t)m * a.ld_qkv + which * a.d + hd * dh;
-    const int64_t gb = (int64_t)m * b.ld_dqk + which * a.d + hd * dh;
-    float x[4] = {0.f, 0.f, 0.f, 0.f}, u[4] = {0.f, 0.f, 0.f, 0.f}, gsc[4] = {0.f, 0.f, 0.f, 0.f};
-    float xu = 0.f;
-    for (int j = 0; j < 2; ++j) {
-      const int pair = lane + 32 * j;
-      if (2 * pair < dh) {
-        // undo the rotation of the incoming gradient (rotate by -angle)
-        const float g0 = ldx(b.dqk, gb + 2 * pair, is_f32), g1 = ldx(b.dqk, gb + 2 * pair + 1, is_f32);
-        float cs = 1.f, sn = 0.f;
-        if (a.rope) rope_angle(n, a.n_txt, a.gw, dh, pair, cs, sn);
-        const float dy0 = g0 * cs + g1 * sn;
-        const float dy1 = -g0 * sn + g1 * cs;
-        x[2 * j] = ldx(a.qkv, xb + 2 * pair, is_f32);
-        x[2 * j + 1] = ldx(a.qkv, xb + 2 * pair + 1, is_f32);
-        gsc[2 * j] = ldx(scl, 2 * pair, is_f32);
-        gsc[2 * j + 1] = ldx(scl, 2 * pair + 1, is_f32);
-        atomicAdd(dscl + 2 * pair, dy0 * x[2 * j] * r);
-        atomicAdd(dscl + 2 * pair + 1, dy1 * x[2 * j + 1] * r);
-        u[2 * j] = dy0 * gsc[2 * j];
-        u[2 * j + 1] = dy1 * gsc[2 * j + 1];
-        xu += x[2 * j] * u[2 * j] + x[2 * j + 1] * u[2 * j + 1];
+  float acc[4][4];  // [which * 2 + stream][element]
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) acc[i][e] = 0.f;
+  const int64_t items = (int64_t)a.M * a.heads;
+  for (int64_t w = (int64_t)blockIdx.x * QKN_WARPS + warp; w < items; w += (int64_t)gridDim.x * QKN_WARPS) {
+    const int hd = (int)(w % a.heads);
+    const int m = (int)(w / a.heads);
+    const int n = m % a.N;
+    const bool txt = n < a.n_txt;
+#pragma unroll
+    for (int which = 0; which < 2; ++which) {
+      const void* scl = which == 0 ? (txt ? a.qscale_txt : a.qscale_img) : (txt ? a.kscale_txt : a.kscale_img);
+      const float r = (which == 0 ? a.rq : a.rk)[(int64_t)m * a.heads + hd];
+      const int64_t xb = (int64_t)m * a.ld_qkv + which * a.d + hd * dh;
+      const int64_t gb = (int64_t)m * b.ld_dqk + which * a.d + hd * dh;
+      float x[4] = {0.f, 0.f, 0.f, 0.f}, u[4] = {0.f, 0.f, 0.f, 0.f}, dsc[4] = {0.f, 0.f, 0.f, 0.f};
+      float xu = 0.f;
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const int pair = lane + 32 * j;
+        if (2 * pair < dh) {
+          // undo the rotation of the incoming gradient (rotate by -angle)
+          const float g0 = ldx(b.dqk, gb + 2 * pair, is_f32), g1 = ldx(b.dqk, gb + 2 * pair + 1, is_f32);
+          float cs = 1.f, sn = 0.f;
+          if (a.rope) rope_angle(n, a.n_txt, a.gw, dh, pair, cs, sn);
+          const float dy0 = g0 * cs + g1 * sn;
+          const float dy1 = -g0 * sn + g1 * cs;
+          x[2 * j] = ldx(a.qkv, xb + 2 * pair, is_f32);
+          x[2 * j + 1] = ldx(a.qkv, xb + 2 * pair + 1, is_f32);
+          dsc[2 * j] = dy0 * x[2 * j] * r;
+          dsc[2 * j + 1] = dy1 * x[2 * j + 1] * r;
+          u[2 * j] = dy0 * ldx(scl, 2 * pair, is_f32);
+          u[2 * j + 1] = dy1 * ldx(scl, 2 * pair + 1, is_f32);
+          xu += x[2 * j] * u[2 * j] + x[2 * j + 1] * u[2 * j + 1];
+        }
       }
-    }
-    xu = warp_sum(xu);
-    for (int j = 0; j < 2; ++j) {
-      const int pair = lane + 32 * j;
-      if (2 * pair < dh) {
-        for (int e = 0; e < 2; ++e) {
-          const float dx = r * u[2 * j + e] - x[2 * j + e] * r * r * r * xu / dh;
-          stx(b.dqk, gb + 2 * pair + e, is_f32, dx);
+      const int slot = which * 2 + (txt ? 0 : 1);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) acc[slot][e] += dsc[e];
+      xu = warp_sum(xu);
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const int pair = lane + 32 * j;
+        if (2 * pair < dh) {
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const float dx = r * u[2 * j + e] - x[2 * j + e] * r * r * r * xu / dh;
+            stx(b.dqk, gb + 2 * pair + e, is_f32, dx);
+          }
         }
       }
     }
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const int pair = lane + 32 * j;
+      if (2 * pair < dh) {
+        part[warp][i][2 * pair] = acc[i][2 * j];
+        part[warp][i][2 * pair + 1] = acc[i][2 * j + 1];
+      }
+    }
+  __syncthreads();
+  float* dst[4] = {b.dqs_txt, b.dqs_img, b.dks_txt, b.dks_img};
+  for (int t = threadIdx.x; t < 4 * dh; t += QKN_THREADS) {
+    const int i = t / dh, c = t % dh;
+    float s = 0.f;
+#pragma unroll
+    for (int w = 0; w < QKN_WARPS; ++w) s += part[w][i][c];
+    if (s != 0.f) atomicAdd(dst[i] + c, s);
   }
 }
 
@@ -585,15 +624,24 @@ int launch_attn_rowdot(const void* dO, const void* O, int64_t ld, float* Dv, int
   return JAGG_OK;
 }
 int launch_qk_norm_rope_fwd(const QkNormRope& a, cudaStream_t s) {
-  JAGG_CHECK_ARG(a.d / a.heads <= 128, "qk_norm: head dim too large");
-  const int64_t warps = (int64_t)a.M * a.heads;
-  qk_norm_rope_fwd_kernel<<<grid_for(warps * 32, 256), 256, 0, s>>>(a);
+  JAGG_CHECK_ARG(a.heads > 0 && a.d % a.heads == 0 && a.d / a.heads <= 128 && (a.d / a.heads) % 2 == 0,
+                 "qk_norm: head dim unsupported");
+  if (a.M <= 0) return JAGG_OK;
+  const int64_t blocks = ((int64_t)a.M * a.heads + QKN_WARPS - 1) / QKN_WARPS;
+  qk_norm_rope_fwd_kernel<<<(int)(blocks < 65536 ? blocks : 65536), QKN_THREADS, 0, s>>>(a);
   JAGG_LAUNCHED();
   return JAGG_OK;
 }
 int launch_qk_norm_rope_bwd(const QkNormRopeBwd& a, cudaStream_t s) {
-  const int64_t warps = (int64_t)a.f.M * a.f.heads;
-  qk_norm_rope_bwd_kernel<<<grid_for(warps * 32, 256), 256, 0, s>>>(a);
+  const QkNormRope& f = a.f;
+  JAGG_CHECK_ARG(f.heads > 0 && f.d % f.heads == 0 && f.d / f.heads <= 128 && (f.d / f.heads) % 2 == 0,
+                 "qk_norm: head dim unsupported");
+  JAGG_CHECK_ARG(a.dqs_txt && a.dks_txt && a.dqs_img && a.dks_img, "qk_norm: null scale gradient");
+  if (f.M <= 0) return JAGG_OK;
+  // a few blocks per SM: each block ends in 4 dh atomics
+  const int64_t blocks = ((int64_t)f.M * f.heads + QKN_WARPS - 1) / QKN_WARPS;
+  const int cap = 4 * sm_count();
+  qk_norm_rope_bwd_kernel<<<(int)(blocks < cap ? blocks : cap), QKN_THREADS, 0, s>>>(a);
   JAGG_LAUNCHED();
   return JAGG_OK;
 }

@@ -199,10 +199,8 @@ static int check_config(const jagg_config* c) {
   const int dh = c->hidden / c->heads;
   JAGG_CHECK_ARG(dh == 16 || dh == 32 || dh == 64 || dh == 128, "head dim %d unsupported", dh);
   JAGG_CHECK_ARG(c->dtype == JAGG_DTYPE_F32 || dh >= 64, "bf16 needs head dim 64 or 128");
-  if (c->arch != JAGG_ARCH_DIT) {
-    set_last_error("arch %d not implemented in this build", c->arch);
-    return JAGG_ERR_UNSUPPORTED;
-  }
+  JAGG_CHECK_ARG(c->arch == JAGG_ARCH_DIT || c->arch == JAGG_ARCH_MMDIT, "unknown arch %d", c->arch);
+  JAGG_CHECK_ARG(c->arch == JAGG_ARCH_MMDIT || c->depth_double == 0, "a DiT has no double blocks");
   return JAGG_OK;
 }
 
@@ -251,6 +249,32 @@ struct DitSaved {
   void* y2;      // [M, d] fc2 output (before the gate)
   float* st1;    // [2, M] mean, rstd of LN1
   float* st2;
+  // MMDiT double-block streams only: q/k after RMSNorm + RoPE and the saved 1/rms
+  void* qk = nullptr;    // [M, 2d]
+  float* rq = nullptr;   // [M, heads]
+  float* rk = nullptr;
+};
+
+// An MMDiT double block: the text (0) and image (1) streams, each laid out as a DiT block
+// over its own rows, and the joint attention's log-sum-exp.
+struct DoubleSaved {
+  DitSaved s[2];
+  float* lse;  // [B, heads, N]
+};
+
+// A Flux-style single block.
+struct SingleSaved {
+  float* h_in;  // [M, d]
+  void* a;      // [M, d] LN + modulation
+  float* st1;   // [2, M]
+  void* qkv;    // [M, 3d] first 3d outputs of lin1
+  void* gp;     // [M, dm] GELU'(u) for the last dm outputs u of lin1
+  void* cat;    // [M, d + dm] [attention output | GELU(u)], the input of lin2
+  void* qk;     // [M, 2d]
+  float* rq;    // [M, heads]
+  float* rk;
+  float* lse;   // [B, heads, N]
+  void* y;      // [M, d] lin2 output (before the gate)
 };
 
 struct Saved {
@@ -266,6 +290,9 @@ struct Saved {
   void* sc_b;    // [B, d] silu(c) in the storage type (operand of the modulation products)
   float* mod;    // [B, Lmod]
   std::vector<DitSaved> blk;
+  std::vector<DoubleSaved> dbl;
+  std::vector<SingleSaved> sgl;
+  float* hD[2] = {nullptr, nullptr};  // outputs of the last double block per stream
   float* h_fin;  // [M, d]
   float* st_f;   // [2, B*Ni]
   void* mf;      // [B*Ni, d]
@@ -289,6 +316,49 @@ void carve_block(Carver& cv, const jagg_model& m, int B, DitSaved& s) {
   s.st2 = cv.f32(2 * M);
 }
 
+void carve_stream(Carver& cv, const jagg_model& m, int B, int Ns, DitSaved& q) {
+  const int64_t Ms = (int64_t)B * Ns;
+  const size_t e = m.esz;
+  q.h_in = cv.f32(Ms * m.d);
+  q.a = cv.take(Ms * m.d * e);
+  q.qkv = cv.take(Ms * 3 * m.d * e);
+  q.qk = cv.take(Ms * 2 * m.d * e);
+  q.rq = cv.f32(Ms * m.heads);
+  q.rk = cv.f32(Ms * m.heads);
+  q.o = cv.take(Ms * m.d * e);
+  q.lse = nullptr;
+  q.y1 = cv.take(Ms * m.d * e);
+  q.h_mid = cv.f32(Ms * m.d);
+  q.m = cv.take(Ms * m.d * e);
+  q.gp = cv.take(Ms * m.dm * e);
+  q.gu = cv.take(Ms * m.dm * e);
+  q.y2 = cv.take(Ms * m.d * e);
+  q.st1 = cv.f32(2 * Ms);
+  q.st2 = cv.f32(2 * Ms);
+}
+
+void carve_double(Carver& cv, const jagg_model& m, int B, DoubleSaved& k) {
+  carve_stream(cv, m, B, m.Nt, k.s[0]);
+  carve_stream(cv, m, B, m.Ni, k.s[1]);
+  k.lse = cv.f32((int64_t)B * m.heads * m.N);
+}
+
+void carve_single(Carver& cv, const jagg_model& m, int B, SingleSaved& k) {
+  const int64_t M = (int64_t)B * m.N;
+  const size_t e = m.esz;
+  k.h_in = cv.f32(M * m.d);
+  k.a = cv.take(M * m.d * e);
+  k.st1 = cv.f32(2 * M);
+  k.qkv = cv.take(M * 3 * m.d * e);
+  k.gp = cv.take(M * m.dm * e);
+  k.cat = cv.take(M * (m.d + m.dm) * e);
+  k.qk = cv.take(M * 2 * m.d * e);
+  k.rq = cv.f32(M * m.heads);
+  k.rk = cv.f32(M * m.heads);
+  k.lse = cv.f32((int64_t)B * m.heads * m.N);
+  k.y = cv.take(M * m.d * e);
+}
+
 // save == true: every block gets its own slots (the saved arena).  save == false: one set
 // of block slots reused by every block (a forward that keeps nothing).
 size_t carve_saved(const jagg_model& m, int B, void* base, bool save, Saved& s) {
@@ -305,6 +375,48 @@ size_t carve_saved(const jagg_model& m, int B, void* base, bool save, Saved& s) 
   s.sc = cv.f32((int64_t)B * m.d);
   s.sc_b = cv.take((size_t)B * m.d * m.esz);
   s.mod = cv.f32((int64_t)B * m.T.Lmod);
+  if (m.cfg.arch == JAGG_ARCH_MMDIT) {
+    const int Ld = m.cfg.depth_double, Ls = m.cfg.depth;
+    s.blk.clear();
+    s.dbl.assign(Ld, DoubleSaved());
+    s.sgl.assign(Ls, SingleSaved());
+    if (save) {
+      for (int l = 0; l < Ld; ++l) carve_double(cv, m, B, s.dbl[l]);
+      if (Ld > 0) {
+        s.hD[0] = cv.f32(Mt * m.d);
+        s.hD[1] = cv.f32(Mi * m.d);
+      }
+      for (int l = 0; l < Ls; ++l) carve_single(cv, m, B, s.sgl[l]);
+      s.h_fin = cv.f32(M * m.d);
+    } else {
+      // one set of slots per block type; residual streams ping-pong between two buffers
+      if (Ld > 0) {
+        DoubleSaved one;
+        carve_double(cv, m, B, one);
+        float* other[2] = {cv.f32(Mt * m.d), cv.f32(Mi * m.d)};
+        for (int l = 0; l < Ld; ++l) {
+          s.dbl[l] = one;
+          for (int si = 0; si < 2; ++si) s.dbl[l].s[si].h_in = (l % 2 == 0) ? one.s[si].h_in : other[si];
+        }
+        for (int si = 0; si < 2; ++si) s.hD[si] = (Ld % 2 == 0) ? one.s[si].h_in : other[si];
+      }
+      if (Ls > 0) {
+        SingleSaved one;
+        carve_single(cv, m, B, one);
+        float* other = cv.f32(M * m.d);
+        for (int l = 0; l < Ls; ++l) {
+          s.sgl[l] = one;
+          s.sgl[l].h_in = (l % 2 == 0) ? one.h_in : other;
+        }
+        s.h_fin = (Ls % 2 == 0) ? one.h_in : other;
+      } else {
+        s.h_fin = cv.f32(M * m.d);
+      }
+    }
+    s.st_f = cv.f32(2 * Mi);
+    s.mf = cv.take(Mi * m.d * m.esz);
+    return align256(cv.off);
+  }
   const int L = m.cfg.depth;
   s.blk.assign(L, DitSaved());
   if (save) {
@@ -333,7 +445,8 @@ struct VjpWs {
   void* du;     // [M, dm]
   float* dx32;  // [M, d] f32 input-gradients feeding LayerNorm backward
   void* dO;     // [M, d]
-  void* dqkv;   // [M, 3d]
+  void* dqkv;   // [M, 3d] (MMDiT: [M, 3d + dm], the gradient of a single block's lin1 output)
+  float* dhs[2] = {nullptr, nullptr};  // MMDiT double blocks: per-stream residual gradients
   float* attn;  // attention scratch
   float* dmod;  // [B, Lmod]
   void* dmod_b;  // [B, Lmod] in the storage type
@@ -353,7 +466,12 @@ size_t carve_vjp_ws(const jagg_model& m, int B, void* base, VjpWs& w) {
   w.du = cv.take(M * m.dm * e);
   w.dx32 = cv.f32(M * m.d);
   w.dO = cv.take(M * m.d * e);
-  w.dqkv = cv.take(M * 3 * m.d * e);
+  const bool mm = m.cfg.arch == JAGG_ARCH_MMDIT;
+  w.dqkv = cv.take(M * (3 * m.d + (mm ? m.dm : 0)) * e);
+  if (mm && m.cfg.depth_double > 0) {
+    w.dhs[0] = cv.f32(Mt * m.d);
+    w.dhs[1] = cv.f32(Mi * m.d);
+  }
   w.attn = cv.f32(attention_bwd_scratch_floats(B, m.N, m.heads, m.dh));
   w.dmod = cv.f32((int64_t)B * m.T.Lmod);
   w.dmod_b = cv.take((size_t)B * m.T.Lmod * m.esz);
@@ -388,11 +506,13 @@ GemmArgs fwd_gemm(const jagg_model& m, int M, int N, int K, const void* X, int64
   return g;
 }
 // dX[M, K] = dY[M, N] Wt[N, K]  (Wt stored [N, K] row-major: MN-major operand).
-GemmArgs dx_gemm(const jagg_model& m, int M, int N, int K, const void* dY, int64_t ldy, int64_t w_off) {
+// ldw: row pitch of Wt when the K columns are a slice of a wider matrix (0 = K).
+GemmArgs dx_gemm(const jagg_model& m, int M, int N, int K, const void* dY, int64_t ldy, int64_t w_off,
+                 int64_t ldw = 0) {
   GemmArgs g;
   g.M = M; g.N = K; g.K = N;
   g.A = dY; g.lda = ldy; g.a_mn = false; g.a_dtype = m.cfg.dtype;
-  g.B = W(m, w_off); g.ldb = K; g.b_mn = true; g.b_dtype = m.cfg.dtype;
+  g.B = W(m, w_off); g.ldb = ldw ? ldw : K; g.b_mn = true; g.b_dtype = m.cfg.dtype;
   g.c_dtype = m.cfg.dtype;
   return g;
 }
@@ -442,40 +562,40 @@ GemmArgs rows_dx(const jagg_model& m, int out, int in, int B, const void* dY, in
   return g;
 }
 
-int forward_impl(const jagg_model& m, const void* z, const float* t, const void* txt, int B, void* v_out,
-                 void* saved, void* ws, cudaStream_t s) {
-  const jagg_config& c = m.cfg;
-  const int dt = c.dtype;
-  const int d = m.d, N = m.N, Ni = m.Ni, Nt = m.Nt;
-  const int M = B * N, Mi = B * Ni, Mt = B * Nt;
-  const int64_t Lm = m.T.Lmod;
-  // With a saved arena every activation goes there; otherwise one block's worth of slots
-  // at the start of the workspace is reused by every block.
-  Saved S;
-  const size_t used = carve_saved(m, B, saved ? saved : ws, saved != nullptr, S);
-  void* vt = nullptr;
-  carve_fwd_ws(m, B, static_cast<uint8_t*>(ws) + (saved ? 0 : used), &vt);
-  float* hstart = S.blk.empty() ? S.h_fin : S.blk[0].h_in;
+// Row map of a token range inside the joint [txt; img] layout of B sequences of N rows:
+// row r of the range is (r / seg) * stride + off + r % seg (seg = 0: the identity).
+struct RowMap {
+  int seg, off;
+  int64_t stride;
+};
+RowMap img_rows_of(const jagg_model& m) { return RowMap{m.Ni, m.Nt, m.N}; }
+RowMap txt_rows_of(const jagg_model& m) { return RowMap{m.Nt, 0, m.N}; }
+constexpr RowMap kContiguous{0, 0, 0};
 
-  // embeddings into the joint [txt; img] residual stream
+// Phase 1 prologue: patch and text embeddings into the residual stream(s) (image rows at
+// h_img through mi, text rows at h_txt through mt), the t-embedding MLP and every block's
+// modulation at once from the stacked weights.
+int prologue_fwd(const jagg_model& m, const void* z, const float* t, const void* txt, int B, const Saved& S,
+                 float* h_img, RowMap mi, float* h_txt, RowMap mt, cudaStream_t s) {
+  const jagg_config& c = m.cfg;
+  const int dt = c.dtype, d = m.d;
+  const int Mi = B * m.Ni, Mt = B * m.Nt;
   JAGG_TRY(launch_patchify(z, dt == JAGG_DTYPE_F32, S.xp, dt == JAGG_DTYPE_F32, dt, B, c.in_channels, c.latent_h,
                            c.latent_w, c.patch, s));
   JAGG_CUDA_TRY(cudaMemcpyAsync(S.txt, txt, (size_t)Mt * c.txt_dim * m.esz, cudaMemcpyDeviceToDevice, s));
-  {
-    GemmArgs g = fwd_gemm(m, Mi, d, m.pd, S.xp, m.pd, m.T.x_w, m.T.x_b);
-    g.C = hstart; g.ldc = d; g.c_dtype = JAGG_DTYPE_F32;
-    g.remap_rows = Ni; g.remap_offset = Nt; g.remap_stride = N;
-    JAGG_TRY(gemm(g, s));
-    GemmArgs gt = fwd_gemm(m, Mt, d, c.txt_dim, S.txt, c.txt_dim, m.T.txt_w, m.T.txt_b);
-    gt.C = hstart; gt.ldc = d; gt.c_dtype = JAGG_DTYPE_F32;
-    gt.remap_rows = Nt; gt.remap_offset = 0; gt.remap_stride = N;
-    JAGG_TRY(gemm(gt, s));
-  }
-  JAGG_TRY(launch_add_pos_embed(hstart, B, N, Nt, m.gh, m.gw, d, s));
-  // t-embedding MLP and every block's modulation (per-sequence rows, f32 activations)
+  GemmArgs g = fwd_gemm(m, Mi, d, m.pd, S.xp, m.pd, m.T.x_w, m.T.x_b);
+  g.C = h_img; g.ldc = d; g.c_dtype = JAGG_DTYPE_F32;
+  g.remap_rows = mi.seg; g.remap_offset = mi.off; g.remap_stride = mi.stride;
+  JAGG_TRY(gemm(g, s));
+  GemmArgs gt = fwd_gemm(m, Mt, d, c.txt_dim, S.txt, c.txt_dim, m.T.txt_w, m.T.txt_b);
+  gt.C = h_txt; gt.ldc = d; gt.c_dtype = JAGG_DTYPE_F32;
+  gt.remap_rows = mt.seg; gt.remap_offset = mt.off; gt.remap_stride = mt.stride;
+  JAGG_TRY(gemm(gt, s));
+  // the single-stream DiT adds the fixed 2D sin-cos table; the MMDiT rotates q/k instead
+  if (c.arch == JAGG_ARCH_DIT) JAGG_TRY(launch_add_pos_embed(h_img, B, m.N, m.Nt, m.gh, m.gw, d, s));
+  // t-embedding MLP and every block's modulation (stacked weights): products with B
+  // per-sequence rows, each run as Y^T = W X^T so that the long dimension is M
   JAGG_TRY(launch_timestep_embedding(t, S.phi, B, c.freq_dim, s));
-  // t-embedding MLP and every block's modulation at once (stacked weights): products
-  // with B per-sequence rows, each run as Y^T = W X^T so that the long dimension is M
   JAGG_TRY(launch_gather_rows(S.phi, c.freq_dim, 0, 0, 0, S.phi_b, dt, B, c.freq_dim, s));
   JAGG_TRY(gemm(rows_gemm(m, d, c.freq_dim, B, S.phi_b, m.T.t_w1, m.T.t_b1, S.e1), s));
   JAGG_TRY(launch_silu(S.e1, S.se1, (int64_t)B * d, s));
@@ -483,177 +603,61 @@ int forward_impl(const jagg_model& m, const void* z, const float* t, const void*
   JAGG_TRY(gemm(rows_gemm(m, d, d, B, S.se1_b, m.T.t_w2, m.T.t_b2, S.c), s));
   JAGG_TRY(launch_silu(S.c, S.sc, (int64_t)B * d, s));
   JAGG_TRY(launch_gather_rows(S.sc, d, 0, 0, 0, S.sc_b, dt, B, d, s));
-  JAGG_TRY(gemm(rows_gemm(m, (int)Lm, d, B, S.sc_b, m.T.mod_w, m.T.mod_b, S.mod), s));
-  // blocks
-  for (int l = 0; l < c.depth; ++l) {
-    const DitBlockW& bw = m.T.blocks[l];
-    const DitSaved& k = S.blk[l];
-    float* h_out = (l + 1 < c.depth) ? S.blk[l + 1].h_in : S.h_fin;
-    const float* mod = S.mod + bw.mod_col;
-    LnModFwd ln{k.h_in, 0, 0, 0, M, d, N, mod, mod + d, Lm, k.a, dt, k.st1, k.st1 + M};
-    JAGG_TRY(launch_ln_mod_fwd(ln, s));
-    GemmArgs g = fwd_gemm(m, M, 3 * d, d, k.a, d, bw.qkv_w, bw.qkv_b);
-    g.C = k.qkv; g.ldc = 3 * d;
-    JAGG_TRY(gemm(g, s));
-    AttnArgs at;
-    at.B = B; at.N = N; at.heads = m.heads; at.dh = m.dh; at.scale = 1.f / sqrtf((float)m.dh);
-    at.q = at.k = at.v = seg_single(k.qkv, 3 * d, N);
-    at.q_col0 = 0; at.k_col0 = d; at.v_col0 = 2 * d;
-    at.o = seg_single(k.o, d, N);
-    at.lse = k.lse;
-    at.dtype = dt;
-    JAGG_TRY(attention_fwd(at, s));
-    g = fwd_gemm(m, M, d, d, k.o, d, bw.proj_w, bw.proj_b);
-    g.epi = EPI_GATE_RESID; g.C = k.y1; g.ldc = d;
-    g.C2 = k.h_mid; g.ldc2 = d; g.aux = k.h_in; g.ld_aux = d;
-    g.gate = mod + 2 * d; g.gate_stride = Lm; g.rows_per_seq = N;
-    JAGG_TRY(gemm(g, s));
-    LnModFwd ln2{k.h_mid, 0, 0, 0, M, d, N, mod + 3 * d, mod + 4 * d, Lm, k.m, dt, k.st2, k.st2 + M};
-    JAGG_TRY(launch_ln_mod_fwd(ln2, s));
-    g = fwd_gemm(m, M, m.dm, d, k.m, d, bw.fc1_w, bw.fc1_b);
-    g.epi = EPI_GELU; g.C = k.gp; g.ldc = m.dm; g.C2 = k.gu; g.ldc2 = m.dm;
-    JAGG_TRY(gemm(g, s));
-    g = fwd_gemm(m, M, d, m.dm, k.gu, m.dm, bw.fc2_w, bw.fc2_b);
-    g.epi = EPI_GATE_RESID; g.C = k.y2; g.ldc = d;
-    g.C2 = h_out; g.ldc2 = d; g.aux = k.h_mid; g.ld_aux = d;
-    g.gate = mod + 5 * d; g.gate_stride = Lm; g.rows_per_seq = N;
-    JAGG_TRY(gemm(g, s));
-  }
-  // final layer on the image tokens
+  JAGG_TRY(gemm(rows_gemm(m, (int)m.T.Lmod, d, B, S.sc_b, m.T.mod_w, m.T.mod_b, S.mod), s));
+  return JAGG_OK;
+}
+
+// Final layer on the image rows of the joint stream S.h_fin, then unpatchify.
+int final_fwd(const jagg_model& m, int B, const Saved& S, void* vt, void* v_out, cudaStream_t s) {
+  const jagg_config& c = m.cfg;
+  const int d = m.d, Mi = B * m.Ni;
   const float* fm = S.mod + m.T.final_mod_col;
-  LnModFwd lf{S.h_fin, Ni, Nt, N, Mi, d, Ni, fm, fm + d, Lm, S.mf, dt, S.st_f, S.st_f + Mi};
+  LnModFwd lf{S.h_fin, m.Ni, m.Nt, m.N, Mi, d, m.Ni, fm, fm + d, m.T.Lmod, S.mf, c.dtype, S.st_f, S.st_f + Mi};
   JAGG_TRY(launch_ln_mod_fwd(lf, s));
   GemmArgs g = fwd_gemm(m, Mi, m.pd, d, S.mf, d, m.T.out_w, m.T.out_b);
   g.C = vt; g.ldc = m.pd;
   JAGG_TRY(gemm(g, s));
-  JAGG_TRY(launch_unpatchify(vt, v_out, dt, B, c.in_channels, c.latent_h, c.latent_w, c.patch, s));
+  JAGG_TRY(launch_unpatchify(vt, v_out, c.dtype, B, c.in_channels, c.latent_h, c.latent_w, c.patch, s));
   return JAGG_OK;
 }
 
-int vjp_impl(const jagg_model& m, const void* saved, int B, const float* cot, float* grad, void* ws,
-             cudaStream_t s) {
+// Backward of the final layer: parameter gradients, and dh (joint layout, zeroed by the
+// caller) += the gradient reaching the image rows.
+int final_bwd(const jagg_model& m, int B, const Saved& S, const VjpWs& w, const float* cot, float* grad,
+              cudaStream_t s) {
   const jagg_config& c = m.cfg;
-  const int dt = c.dtype;
-  const int d = m.d, dmw = m.dm, N = m.N, Ni = m.Ni, Nt = m.Nt;
-  const int M = B * N, Mi = B * Ni, Mt = B * Nt;
+  const int dt = c.dtype, d = m.d, Mi = B * m.Ni;
   const int64_t Lm = m.T.Lmod;
-  Saved S;
-  carve_saved(m, B, const_cast<void*>(saved), true, S);
-  VjpWs w;
-  carve_vjp_ws(m, B, ws, w);
-  JAGG_CUDA_TRY(cudaMemsetAsync(w.dmod, 0, sizeof(float) * (size_t)B * Lm, s));
-  JAGG_CUDA_TRY(cudaMemsetAsync(w.dh, 0, sizeof(float) * (size_t)M * d, s));
-  JAGG_CUDA_TRY(cudaMemsetAsync(w.dsc, 0, sizeof(float) * (size_t)B * d, s));
-  JAGG_CUDA_TRY(cudaMemsetAsync(w.de1, 0, sizeof(float) * (size_t)B * d, s));
-
-  // final layer
   JAGG_TRY(launch_patchify(cot, 1, w.dvt, dt == JAGG_DTYPE_F32, dt, B, c.in_channels, c.latent_h, c.latent_w,
                            c.patch, s));
   JAGG_TRY(launch_colsum(w.dvt, dt == JAGG_DTYPE_F32, dt, Mi, m.pd, m.pd, grad + m.T.out_b, s));
   JAGG_TRY(gemm(dw_gemm(m, Mi, m.pd, d, w.dvt, m.pd, S.mf, d, grad, m.T.out_w), s));
-  {
-    GemmArgs g = dx_gemm(m, Mi, m.pd, d, w.dvt, m.pd, m.T.out_w);
-    g.C = w.dx32; g.ldc = d; g.c_dtype = JAGG_DTYPE_F32;
-    JAGG_TRY(gemm(g, s));
-  }
+  GemmArgs g = dx_gemm(m, Mi, m.pd, d, w.dvt, m.pd, m.T.out_w);
+  g.C = w.dx32; g.ldc = d; g.c_dtype = JAGG_DTYPE_F32;
+  JAGG_TRY(gemm(g, s));
   const float* fm = S.mod + m.T.final_mod_col;
   float* dfm = w.dmod + m.T.final_mod_col;
-  {
-    LnGateBwd a{};
-    a.M = Mi; a.d = d; a.rows_per_seq = Ni;
-    a.seg = Ni; a.seg_off = Nt; a.seg_stride = N;
-    a.do_ln = 1; a.dm = w.dx32; a.dm_f32 = 1; a.h = S.h_fin; a.mean = S.st_f; a.rstd = S.st_f + Mi;
-    a.scale = fm + d; a.mod_stride = Lm; a.dshift = dfm; a.dscale = dfm + d; a.dmod_stride = Lm;
-    a.dh_in = w.dh; a.dh_out = w.dh;
-    a.dtype = dt;
-    JAGG_TRY(launch_ln_gate_bwd(a, s));
-  }
-  // Gate of block l's MLP branch (dg2, dy2 = g2 dh, db_fc2): for the last block a pass of
-  // its own; for the others fused into the LayerNorm-1 backward of block l + 1, which
-  // produces exactly that gradient.
-  auto mlp_gate = [&](LnGateBwd& a, int l) {
-    const DitBlockW& bw = m.T.blocks[l];
-    a.do_gate = 1; a.y = S.blk[l].y2; a.gate = S.mod + bw.mod_col + 5 * d; a.mod_stride = Lm;
-    a.dgate = w.dmod + bw.mod_col + 5 * d; a.dmod_stride = Lm; a.dy = w.dy; a.dbias = grad + bw.fc2_b;
-  };
-  if (c.depth > 0) {
-    LnGateBwd a{};
-    a.M = M; a.d = d; a.rows_per_seq = N;
-    a.do_ln = 0; a.dh_in = w.dh; a.dh_out = w.dh; a.dtype = dt;
-    mlp_gate(a, c.depth - 1);
-    JAGG_TRY(launch_ln_gate_bwd(a, s));
-  }
-  // blocks, last to first
-  for (int l = c.depth - 1; l >= 0; --l) {
-    const DitBlockW& bw = m.T.blocks[l];
-    const DitSaved& k = S.blk[l];
-    const float* mod = S.mod + bw.mod_col;
-    float* dmod = w.dmod + bw.mod_col;
-    JAGG_TRY(gemm(dw_gemm(m, M, d, dmw, w.dy, d, k.gu, dmw, grad, bw.fc2_w), s));
-    {
-      GemmArgs g = dx_gemm(m, M, d, dmw, w.dy, d, bw.fc2_w);
-      g.epi = EPI_MUL_AUX; g.C = w.du; g.ldc = dmw; g.aux = k.gp; g.ld_aux = dmw;
-      JAGG_TRY(gemm(g, s));
-    }
-    JAGG_TRY(launch_colsum(w.du, dt == JAGG_DTYPE_F32, dt, M, dmw, dmw, grad + bw.fc1_b, s));
-    JAGG_TRY(gemm(dw_gemm(m, M, dmw, d, w.du, dmw, k.m, d, grad, bw.fc1_w), s));
-    {
-      GemmArgs g = dx_gemm(m, M, dmw, d, w.du, dmw, bw.fc1_w);
-      g.C = w.dx32; g.ldc = d; g.c_dtype = JAGG_DTYPE_F32;
-      JAGG_TRY(gemm(g, s));
-    }
-    {  // LN2 + modulation backward, then the attention branch's gate
-      LnGateBwd a{};
-      a.M = M; a.d = d; a.rows_per_seq = N;
-      a.do_ln = 1; a.dm = w.dx32; a.dm_f32 = 1; a.h = k.h_mid; a.mean = k.st2; a.rstd = k.st2 + M;
-      a.scale = mod + 4 * d; a.mod_stride = Lm; a.dshift = dmod + 3 * d; a.dscale = dmod + 4 * d;
-      a.dmod_stride = Lm; a.dh_in = w.dh; a.dh_out = w.dh;
-      a.do_gate = 1; a.y = k.y1; a.gate = mod + 2 * d; a.dgate = dmod + 2 * d; a.dy = w.dy;
-      a.dbias = grad + bw.proj_b; a.dtype = dt;
-      JAGG_TRY(launch_ln_gate_bwd(a, s));
-    }
-    JAGG_TRY(gemm(dw_gemm(m, M, d, d, w.dy, d, k.o, d, grad, bw.proj_w), s));
-    {
-      GemmArgs g = dx_gemm(m, M, d, d, w.dy, d, bw.proj_w);
-      g.C = w.dO; g.ldc = d;
-      JAGG_TRY(gemm(g, s));
-    }
-    {
-      AttnBwdArgs ab;
-      AttnArgs& at = ab.f;
-      at.B = B; at.N = N; at.heads = m.heads; at.dh = m.dh; at.scale = 1.f / sqrtf((float)m.dh);
-      at.q = at.k = at.v = seg_single(k.qkv, 3 * d, N);
-      at.q_col0 = 0; at.k_col0 = d; at.v_col0 = 2 * d;
-      at.o = seg_single(k.o, d, N);
-      at.lse = k.lse; at.dtype = dt;
-      ab.dO = seg_single(w.dO, d, N);
-      attention_bwd_scratch(w.attn, B, N, m.heads, &ab.Dv, &ab.dq_acc);
-      ab.dq = ab.dk = ab.dv = seg_single(w.dqkv, 3 * d, N);
-      ab.dq_col0 = 0; ab.dk_col0 = d; ab.dv_col0 = 2 * d;
-      JAGG_TRY(attention_bwd(ab, s));
-    }
-    JAGG_TRY(launch_colsum(w.dqkv, dt == JAGG_DTYPE_F32, dt, M, 3 * d, 3 * d, grad + bw.qkv_b, s));
-    JAGG_TRY(gemm(dw_gemm(m, M, 3 * d, d, w.dqkv, 3 * d, k.a, d, grad, bw.qkv_w), s));
-    {
-      GemmArgs g = dx_gemm(m, M, 3 * d, d, w.dqkv, 3 * d, bw.qkv_w);
-      g.C = w.dx32; g.ldc = d; g.c_dtype = JAGG_DTYPE_F32;
-      JAGG_TRY(gemm(g, s));
-    }
-    {  // LN1 + modulation backward, then the previous block's MLP gate
-      LnGateBwd a{};
-      a.M = M; a.d = d; a.rows_per_seq = N;
-      a.do_ln = 1; a.dm = w.dx32; a.dm_f32 = 1; a.h = k.h_in; a.mean = k.st1; a.rstd = k.st1 + M;
-      a.scale = mod + d; a.mod_stride = Lm; a.dshift = dmod; a.dscale = dmod + d; a.dmod_stride = Lm;
-      a.dh_in = w.dh; a.dh_out = w.dh; a.dtype = dt;
-      if (l > 0) mlp_gate(a, l - 1);
-      JAGG_TRY(launch_ln_gate_bwd(a, s));
-    }
-  }
-  // input projections (no gradient to z or txt)
-  JAGG_TRY(launch_gather_rows(w.dh, d, Ni, Nt, N, w.dxe, dt, Mi, d, s));
+  LnGateBwd a{};
+  a.M = Mi; a.d = d; a.rows_per_seq = m.Ni;
+  a.seg = m.Ni; a.seg_off = m.Nt; a.seg_stride = m.N;
+  a.do_ln = 1; a.dm = w.dx32; a.dm_f32 = 1; a.h = S.h_fin; a.mean = S.st_f; a.rstd = S.st_f + Mi;
+  a.scale = fm + d; a.mod_stride = Lm; a.dshift = dfm; a.dscale = dfm + d; a.dmod_stride = Lm;
+  a.dh_in = w.dh; a.dh_out = w.dh;
+  a.dtype = dt;
+  return launch_ln_gate_bwd(a, s);
+}
+
+// Backward of the embeddings (no gradient to z or txt) and of the stacked modulation and
+// the t-embedding MLP, from the residual gradients at the embedding outputs.
+int epilogue_bwd(const jagg_model& m, int B, const Saved& S, const VjpWs& w, const float* dh_img, RowMap mi,
+                 const float* dh_txt, RowMap mt, float* grad, cudaStream_t s) {
+  const jagg_config& c = m.cfg;
+  const int dt = c.dtype, d = m.d, Mi = B * m.Ni, Mt = B * m.Nt;
+  const int64_t Lm = m.T.Lmod;
+  JAGG_TRY(launch_gather_rows(dh_img, d, mi.seg, mi.off, mi.stride, w.dxe, dt, Mi, d, s));
   JAGG_TRY(launch_colsum(w.dxe, dt == JAGG_DTYPE_F32, dt, Mi, d, d, grad + m.T.x_b, s));
   JAGG_TRY(gemm(dw_gemm(m, Mi, d, m.pd, w.dxe, d, S.xp, m.pd, grad, m.T.x_w), s));
-  JAGG_TRY(launch_gather_rows(w.dh, d, Nt, 0, N, w.dxe, dt, Mt, d, s));
+  JAGG_TRY(launch_gather_rows(dh_txt, d, mt.seg, mt.off, mt.stride, w.dxe, dt, Mt, d, s));
   JAGG_TRY(launch_colsum(w.dxe, dt == JAGG_DTYPE_F32, dt, Mt, d, d, grad + m.T.txt_b, s));
   JAGG_TRY(gemm(dw_gemm(m, Mt, d, c.txt_dim, w.dxe, d, S.txt, c.txt_dim, grad, m.T.txt_w), s));
   // stacked modulation: dW += dmod^T silu(c), db += sum_b dmod, d silu(c) = dmod W
@@ -672,6 +676,425 @@ int vjp_impl(const jagg_model& m, const void* saved, int B, const float* cot, fl
   JAGG_TRY(launch_gather_rows(w.de1, d, 0, 0, 0, w.dc_b, dt, B, d, s));
   JAGG_TRY(gemm(rows_dw(m, d, c.freq_dim, B, w.dc_b, S.phi_b, grad, m.T.t_w1), s));
   return JAGG_OK;
+}
+
+int zero_vjp_accumulators(const jagg_model& m, int B, const VjpWs& w, cudaStream_t s) {
+  JAGG_CUDA_TRY(cudaMemsetAsync(w.dmod, 0, sizeof(float) * (size_t)B * m.T.Lmod, s));
+  JAGG_CUDA_TRY(cudaMemsetAsync(w.dh, 0, sizeof(float) * (size_t)B * m.N * m.d, s));
+  JAGG_CUDA_TRY(cudaMemsetAsync(w.dsc, 0, sizeof(float) * (size_t)B * m.d, s));
+  JAGG_CUDA_TRY(cudaMemsetAsync(w.de1, 0, sizeof(float) * (size_t)B * m.d, s));
+  return JAGG_OK;
+}
+
+// The MLP half of a block's backward, shared by DiT blocks and the streams of MMDiT
+// double blocks (Ms rows of Ns tokens per sequence): from dy = g2 dh (already formed)
+// through fc2, GELU, fc1 and LN2 + modulation, then the attention branch's gate, ending
+// with dO = dy1 Wproj.  dh accumulates in place.
+struct BranchW {
+  int64_t proj_w, proj_b, fc1_w, fc1_b, fc2_w, fc2_b, mod_col;
+};
+int mlp_and_proj_bwd(const jagg_model& m, int Ms, int Ns, const DitSaved& k, const BranchW& bw, const float* mod,
+                     float* dmod, float* dh, void* dy, void* dO, const VjpWs& w, float* grad, cudaStream_t s) {
+  const int dt = m.cfg.dtype, d = m.d, dmw = m.dm;
+  const int64_t Lm = m.T.Lmod;
+  JAGG_TRY(gemm(dw_gemm(m, Ms, d, dmw, dy, d, k.gu, dmw, grad, bw.fc2_w), s));
+  {
+    GemmArgs g = dx_gemm(m, Ms, d, dmw, dy, d, bw.fc2_w);
+    g.epi = EPI_MUL_AUX; g.C = w.du; g.ldc = dmw; g.aux = k.gp; g.ld_aux = dmw;
+    JAGG_TRY(gemm(g, s));
+  }
+  JAGG_TRY(launch_colsum(w.du, dt == JAGG_DTYPE_F32, dt, Ms, dmw, dmw, grad + bw.fc1_b, s));
+  JAGG_TRY(gemm(dw_gemm(m, Ms, dmw, d, w.du, dmw, k.m, d, grad, bw.fc1_w), s));
+  {
+    GemmArgs g = dx_gemm(m, Ms, dmw, d, w.du, dmw, bw.fc1_w);
+    g.C = w.dx32; g.ldc = d; g.c_dtype = JAGG_DTYPE_F32;
+    JAGG_TRY(gemm(g, s));
+  }
+  {  // LN2 + modulation backward, then the attention branch's gate
+    LnGateBwd a{};
+    a.M = Ms; a.d = d; a.rows_per_seq = Ns;
+    a.do_ln = 1; a.dm = w.dx32; a.dm_f32 = 1; a.h = k.h_mid; a.mean = k.st2; a.rstd = k.st2 + Ms;
+    a.scale = mod + 4 * d; a.mod_stride = Lm; a.dshift = dmod + 3 * d; a.dscale = dmod + 4 * d;
+    a.dmod_stride = Lm; a.dh_in = dh; a.dh_out = dh;
+    a.do_gate = 1; a.y = k.y1; a.gate = mod + 2 * d; a.dgate = dmod + 2 * d; a.dy = dy;
+    a.dbias = grad + bw.proj_b; a.dtype = dt;
+    JAGG_TRY(launch_ln_gate_bwd(a, s));
+  }
+  JAGG_TRY(gemm(dw_gemm(m, Ms, d, d, dy, d, k.o, d, grad, bw.proj_w), s));
+  GemmArgs g = dx_gemm(m, Ms, d, d, dy, d, bw.proj_w);
+  g.C = dO; g.ldc = d;
+  return gemm(g, s);
+}
+
+// The qkv half of a block's backward after attention: qkv bias / weight gradients, the
+// gradient into the LN1 input, and LN1 + modulation backward (dh accumulates in place).
+// `gate`, when given, fuses the gate backward of the previous block's last branch.
+int qkv_and_ln1_bwd(const jagg_model& m, int Ms, int Ns, const void* dqkv, int64_t ld_dqkv, int n_out,
+                    int64_t w_off, int64_t b_off, const void* a_in, const float* h_in, const float* st1,
+                    const float* mod, float* dmod, float* dh, const LnGateBwd* gate, const VjpWs& w, float* grad,
+                    cudaStream_t s) {
+  const int dt = m.cfg.dtype, d = m.d;
+  const int64_t Lm = m.T.Lmod;
+  JAGG_TRY(launch_colsum(dqkv, dt == JAGG_DTYPE_F32, dt, Ms, n_out, ld_dqkv, grad + b_off, s));
+  JAGG_TRY(gemm(dw_gemm(m, Ms, n_out, d, dqkv, ld_dqkv, a_in, d, grad, w_off), s));
+  {
+    GemmArgs g = dx_gemm(m, Ms, n_out, d, dqkv, ld_dqkv, w_off);
+    g.C = w.dx32; g.ldc = d; g.c_dtype = JAGG_DTYPE_F32;
+    JAGG_TRY(gemm(g, s));
+  }
+  LnGateBwd a = gate ? *gate : LnGateBwd{};
+  a.M = Ms; a.d = d; a.rows_per_seq = Ns;
+  a.do_ln = 1; a.dm = w.dx32; a.dm_f32 = 1; a.h = h_in; a.mean = st1; a.rstd = st1 + Ms;
+  a.scale = mod + d; a.mod_stride = Lm; a.dshift = dmod; a.dscale = dmod + d; a.dmod_stride = Lm;
+  a.dh_in = dh; a.dh_out = dh; a.dtype = dt;
+  return launch_ln_gate_bwd(a, s);
+}
+
+// Gate backward of a branch y with gate mod[gcol]: dgate += sum dh y; dy = gate dh; dbias.
+LnGateBwd gate_args(const jagg_model& m, int Ms, int Ns, float* dh, const void* y, const float* gate,
+                    float* dgate, void* dy, float* dbias) {
+  LnGateBwd a{};
+  a.M = Ms; a.d = m.d; a.rows_per_seq = Ns;
+  a.do_ln = 0; a.dh_in = dh; a.dh_out = dh;
+  a.do_gate = 1; a.y = y; a.gate = gate; a.mod_stride = m.T.Lmod; a.dgate = dgate; a.dmod_stride = m.T.Lmod;
+  a.dy = dy; a.dbias = dbias; a.dtype = m.cfg.dtype;
+  return a;
+}
+
+AttnArgs attn_args(const jagg_model& m, int B, SegRows qk, SegRows v, SegRows o, float* lse) {
+  AttnArgs at;
+  at.B = B; at.N = m.N; at.heads = m.heads; at.dh = m.dh; at.scale = 1.f / sqrtf((float)m.dh);
+  at.q = at.k = qk;
+  at.v = v;
+  at.o = o;
+  at.lse = lse;
+  at.dtype = m.cfg.dtype;
+  return at;
+}
+
+QkNormRope qk_args(const jagg_model& m, const void* qkv, int Ms, int Ns, int n_txt, int64_t qn, int64_t kn, void* qk,
+                   float* rq, float* rk) {
+  QkNormRope q{};
+  q.qkv = qkv; q.ld_qkv = 3 * m.d;
+  q.M = Ms; q.N = Ns; q.d = m.d; q.heads = m.heads; q.n_txt = n_txt; q.gw = m.gw;
+  q.qscale_txt = q.qscale_img = W(m, qn);
+  q.kscale_txt = q.kscale_img = W(m, kn);
+  q.rope = 1;
+  q.qk_out = qk; q.rq = rq; q.rk = rk;
+  q.dtype = m.cfg.dtype;
+  return q;
+}
+
+// ---------------------------------------------------------------- single-stream DiT
+int forward_dit(const jagg_model& m, const Saved& S, int B, cudaStream_t s) {
+  const jagg_config& c = m.cfg;
+  const int dt = c.dtype, d = m.d, N = m.N, M = B * N;
+  const int64_t Lm = m.T.Lmod;
+  for (int l = 0; l < c.depth; ++l) {
+    const DitBlockW& bw = m.T.blocks[l];
+    const DitSaved& k = S.blk[l];
+    float* h_out = (l + 1 < c.depth) ? S.blk[l + 1].h_in : S.h_fin;
+    const float* mod = S.mod + bw.mod_col;
+    LnModFwd ln{k.h_in, 0, 0, 0, M, d, N, mod, mod + d, Lm, k.a, dt, k.st1, k.st1 + M};
+    JAGG_TRY(launch_ln_mod_fwd(ln, s));
+    GemmArgs g = fwd_gemm(m, M, 3 * d, d, k.a, d, bw.qkv_w, bw.qkv_b);
+    g.C = k.qkv; g.ldc = 3 * d;
+    JAGG_TRY(gemm(g, s));
+    AttnArgs at = attn_args(m, B, seg_single(k.qkv, 3 * d, N), seg_single(k.qkv, 3 * d, N), seg_single(k.o, d, N),
+                            k.lse);
+    at.q_col0 = 0; at.k_col0 = d; at.v_col0 = 2 * d;
+    JAGG_TRY(attention_fwd(at, s));
+    g = fwd_gemm(m, M, d, d, k.o, d, bw.proj_w, bw.proj_b);
+    g.epi = EPI_GATE_RESID; g.C = k.y1; g.ldc = d;
+    g.C2 = k.h_mid; g.ldc2 = d; g.aux = k.h_in; g.ld_aux = d;
+    g.gate = mod + 2 * d; g.gate_stride = Lm; g.rows_per_seq = N;
+    JAGG_TRY(gemm(g, s));
+    LnModFwd ln2{k.h_mid, 0, 0, 0, M, d, N, mod + 3 * d, mod + 4 * d, Lm, k.m, dt, k.st2, k.st2 + M};
+    JAGG_TRY(launch_ln_mod_fwd(ln2, s));
+    g = fwd_gemm(m, M, m.dm, d, k.m, d, bw.fc1_w, bw.fc1_b);
+    g.epi = EPI_GELU; g.C = k.gp; g.ldc = m.dm; g.C2 = k.gu; g.ldc2 = m.dm;
+    JAGG_TRY(gemm(g, s));
+    g = fwd_gemm(m, M, d, m.dm, k.gu, m.dm, bw.fc2_w, bw.fc2_b);
+    g.epi = EPI_GATE_RESID; g.C = k.y2; g.ldc = d;
+    g.C2 = h_out; g.ldc2 = d; g.aux = k.h_mid; g.ld_aux = d;
+    g.gate = mod + 5 * d; g.gate_stride = Lm; g.rows_per_seq = N;
+    JAGG_TRY(gemm(g, s));
+  }
+  return JAGG_OK;
+}
+
+BranchW branch_of(const DitBlockW& b) {
+  return BranchW{b.proj_w, b.proj_b, b.fc1_w, b.fc1_b, b.fc2_w, b.fc2_b, b.mod_col};
+}
+BranchW branch_of(const StreamW& b) {
+  return BranchW{b.proj_w, b.proj_b, b.fc1_w, b.fc1_b, b.fc2_w, b.fc2_b, b.mod_col};
+}
+
+int vjp_dit(const jagg_model& m, const Saved& S, int B, const VjpWs& w, float* grad, cudaStream_t s) {
+  const jagg_config& c = m.cfg;
+  const int d = m.d, N = m.N, M = B * N;
+  // Gate of block l's MLP branch (dg2, dy2 = g2 dh, db_fc2): for the last block a pass of
+  // its own; for the others fused into the LayerNorm-1 backward of block l + 1, which
+  // produces exactly that gradient.
+  auto mlp_gate = [&](int l) {
+    const DitBlockW& bw = m.T.blocks[l];
+    return gate_args(m, M, N, w.dh, S.blk[l].y2, S.mod + bw.mod_col + 5 * d, w.dmod + bw.mod_col + 5 * d, w.dy,
+                     grad + bw.fc2_b);
+  };
+  if (c.depth > 0) JAGG_TRY(launch_ln_gate_bwd(mlp_gate(c.depth - 1), s));
+  for (int l = c.depth - 1; l >= 0; --l) {
+    const DitBlockW& bw = m.T.blocks[l];
+    const DitSaved& k = S.blk[l];
+    const float* mod = S.mod + bw.mod_col;
+    float* dmod = w.dmod + bw.mod_col;
+    JAGG_TRY(mlp_and_proj_bwd(m, M, N, k, branch_of(bw), mod, dmod, w.dh, w.dy, w.dO, w, grad, s));
+    AttnBwdArgs ab;
+    ab.f = attn_args(m, B, seg_single(k.qkv, 3 * d, N), seg_single(k.qkv, 3 * d, N), seg_single(k.o, d, N), k.lse);
+    ab.f.q_col0 = 0; ab.f.k_col0 = d; ab.f.v_col0 = 2 * d;
+    ab.dO = seg_single(w.dO, d, N);
+    attention_bwd_scratch(w.attn, B, N, m.heads, &ab.Dv, &ab.dq_acc);
+    ab.dq = ab.dk = ab.dv = seg_single(w.dqkv, 3 * d, N);
+    ab.dq_col0 = 0; ab.dk_col0 = d; ab.dv_col0 = 2 * d;
+    JAGG_TRY(attention_bwd(ab, s));
+    LnGateBwd prev{};
+    if (l > 0) prev = mlp_gate(l - 1);
+    JAGG_TRY(qkv_and_ln1_bwd(m, M, N, w.dqkv, 3 * d, 3 * d, bw.qkv_w, bw.qkv_b, k.a, k.h_in, k.st1, mod, dmod, w.dh,
+                             l > 0 ? &prev : nullptr, w, grad, s));
+  }
+  return JAGG_OK;
+}
+
+// ---------------------------------------------------------------- MMDiT
+// Double blocks run each stream as its own rows (Ms = B Ns, Ns = Nt or Ni tokens per
+// sequence) and meet only in the joint attention, which addresses the two streams'
+// buffers as one [txt; img] sequence.  Single blocks run on the joint layout.
+int forward_mmdit(const jagg_model& m, const Saved& S, int B, cudaStream_t s) {
+  const jagg_config& c = m.cfg;
+  const int dt = c.dtype, d = m.d, dm = m.dm, N = m.N, Nt = m.Nt, Ni = m.Ni, M = B * N;
+  const int Ld = c.depth_double, Ls = c.depth;
+  const int64_t Lm = m.T.Lmod;
+  for (int l = 0; l < Ld; ++l) {
+    const DoubleW& bw = m.T.doubles[l];
+    const DoubleSaved& k = S.dbl[l];
+    for (int si = 0; si < 2; ++si) {
+      const StreamW& sw = bw.s[si];
+      const DitSaved& q = k.s[si];
+      const int Ns = si ? Ni : Nt, Ms = B * Ns;
+      const float* mod = S.mod + sw.mod_col;
+      LnModFwd ln{q.h_in, 0, 0, 0, Ms, d, Ns, mod, mod + d, Lm, q.a, dt, q.st1, q.st1 + Ms};
+      JAGG_TRY(launch_ln_mod_fwd(ln, s));
+      GemmArgs g = fwd_gemm(m, Ms, 3 * d, d, q.a, d, sw.qkv_w, sw.qkv_b);
+      g.C = q.qkv; g.ldc = 3 * d;
+      JAGG_TRY(gemm(g, s));
+      // text tokens sit at RoPE position (0, 0): the whole text stream is unrotated
+      JAGG_TRY(launch_qk_norm_rope_fwd(qk_args(m, q.qkv, Ms, Ns, si ? 0 : Ns, sw.qn, sw.kn, q.qk, q.rq, q.rk), s));
+    }
+    AttnArgs at = attn_args(m, B, SegRows{k.s[0].qk, k.s[1].qk, 2 * d, 2 * d, Nt},
+                            SegRows{k.s[0].qkv, k.s[1].qkv, 3 * d, 3 * d, Nt},
+                            SegRows{k.s[0].o, k.s[1].o, d, d, Nt}, k.lse);
+    at.q_col0 = 0; at.k_col0 = d; at.v_col0 = 2 * d;
+    JAGG_TRY(attention_fwd(at, s));
+    for (int si = 0; si < 2; ++si) {
+      const StreamW& sw = bw.s[si];
+      const DitSaved& q = k.s[si];
+      const int Ns = si ? Ni : Nt, Ms = B * Ns;
+      const float* mod = S.mod + sw.mod_col;
+      float* h_out = (l + 1 < Ld) ? S.dbl[l + 1].s[si].h_in : S.hD[si];
+      GemmArgs g = fwd_gemm(m, Ms, d, d, q.o, d, sw.proj_w, sw.proj_b);
+      g.epi = EPI_GATE_RESID; g.C = q.y1; g.ldc = d;
+      g.C2 = q.h_mid; g.ldc2 = d; g.aux = q.h_in; g.ld_aux = d;
+      g.gate = mod + 2 * d; g.gate_stride = Lm; g.rows_per_seq = Ns;
+      JAGG_TRY(gemm(g, s));
+      LnModFwd ln2{q.h_mid, 0, 0, 0, Ms, d, Ns, mod + 3 * d, mod + 4 * d, Lm, q.m, dt, q.st2, q.st2 + Ms};
+      JAGG_TRY(launch_ln_mod_fwd(ln2, s));
+      g = fwd_gemm(m, Ms, dm, d, q.m, d, sw.fc1_w, sw.fc1_b);
+      g.epi = EPI_GELU; g.C = q.gp; g.ldc = dm; g.C2 = q.gu; g.ldc2 = dm;
+      JAGG_TRY(gemm(g, s));
+      g = fwd_gemm(m, Ms, d, dm, q.gu, dm, sw.fc2_w, sw.fc2_b);
+      g.epi = EPI_GATE_RESID; g.C = q.y2; g.ldc = d;
+      g.C2 = h_out; g.ldc2 = d; g.aux = q.h_mid; g.ld_aux = d;
+      g.gate = mod + 5 * d; g.gate_stride = Lm; g.rows_per_seq = Ns;
+      JAGG_TRY(gemm(g, s));
+    }
+  }
+  float* hj = Ls > 0 ? S.sgl[0].h_in : S.h_fin;
+  if (Ld > 0) {  // the two streams join into the [txt; img] layout
+    JAGG_TRY(launch_copy_rows(S.hD[0], d, 0, 0, 0, hj, d, Nt, 0, N, B * Nt, d, 4, s));
+    JAGG_TRY(launch_copy_rows(S.hD[1], d, 0, 0, 0, hj, d, Ni, Nt, N, B * Ni, d, 4, s));
+  }
+  const size_t e = m.esz;
+  for (int l = 0; l < Ls; ++l) {
+    const SingleW& sw = m.T.singles[l];
+    const SingleSaved& k = S.sgl[l];
+    float* h_out = (l + 1 < Ls) ? S.sgl[l + 1].h_in : S.h_fin;
+    const float* mod = S.mod + sw.mod_col;
+    LnModFwd ln{k.h_in, 0, 0, 0, M, d, N, mod, mod + d, Lm, k.a, dt, k.st1, k.st1 + M};
+    JAGG_TRY(launch_ln_mod_fwd(ln, s));
+    // lin1 = [qkv | u]: two products over the row blocks of its weight
+    GemmArgs g = fwd_gemm(m, M, 3 * d, d, k.a, d, sw.lin1_w, sw.lin1_b);
+    g.C = k.qkv; g.ldc = 3 * d;
+    JAGG_TRY(gemm(g, s));
+    g = fwd_gemm(m, M, dm, d, k.a, d, sw.lin1_w + (int64_t)3 * d * d, sw.lin1_b + 3 * d);
+    g.epi = EPI_GELU; g.C = k.gp; g.ldc = dm;
+    g.C2 = static_cast<uint8_t*>(k.cat) + (size_t)d * e; g.ldc2 = d + dm;
+    JAGG_TRY(gemm(g, s));
+    JAGG_TRY(launch_qk_norm_rope_fwd(qk_args(m, k.qkv, M, N, Nt, sw.qn, sw.kn, k.qk, k.rq, k.rk), s));
+    AttnArgs at = attn_args(m, B, seg_single(k.qk, 2 * d, N), seg_single(k.qkv, 3 * d, N),
+                            seg_single(k.cat, d + dm, N), k.lse);
+    at.q_col0 = 0; at.k_col0 = d; at.v_col0 = 2 * d;
+    JAGG_TRY(attention_fwd(at, s));
+    g = fwd_gemm(m, M, d, d + dm, k.cat, d + dm, sw.lin2_w, sw.lin2_b);
+    g.epi = EPI_GATE_RESID; g.C = k.y; g.ldc = d;
+    g.C2 = h_out; g.ldc2 = d; g.aux = k.h_in; g.ld_aux = d;
+    g.gate = mod + 2 * d; g.gate_stride = Lm; g.rows_per_seq = N;
+    JAGG_TRY(gemm(g, s));
+  }
+  return JAGG_OK;
+}
+
+int vjp_mmdit(const jagg_model& m, const Saved& S, int B, const VjpWs& w, float* grad, cudaStream_t s) {
+  const jagg_config& c = m.cfg;
+  const int d = m.d, dm = m.dm, N = m.N, Nt = m.Nt, Ni = m.Ni, M = B * N, Mt = B * Nt;
+  const int Ld = c.depth_double, Ls = c.depth;
+  const size_t e = m.esz;
+  auto at_byte = [](void* p, size_t off) { return static_cast<void*>(static_cast<uint8_t*>(p) + off); };
+  // single blocks, last to first, on the joint gradient w.dh
+  auto single_gate = [&](int l) {
+    const SingleW& sw = m.T.singles[l];
+    return gate_args(m, M, N, w.dh, S.sgl[l].y, S.mod + sw.mod_col + 2 * d, w.dmod + sw.mod_col + 2 * d, w.dy,
+                     grad + sw.lin2_b);
+  };
+  if (Ls > 0) JAGG_TRY(launch_ln_gate_bwd(single_gate(Ls - 1), s));
+  const int64_t ld1 = 3 * d + dm;  // w.dqkv holds d(lin1 output) = [dqkv | du]
+  for (int l = Ls - 1; l >= 0; --l) {
+    const SingleW& sw = m.T.singles[l];
+    const SingleSaved& k = S.sgl[l];
+    const float* mod = S.mod + sw.mod_col;
+    float* dmod = w.dmod + sw.mod_col;
+    JAGG_TRY(gemm(dw_gemm(m, M, d, d + dm, w.dy, d, k.cat, d + dm, grad, sw.lin2_w), s));
+    {  // d(cat) = dy Wlin2: the attention-output columns, then GELU's columns times GELU'
+      GemmArgs g = dx_gemm(m, M, d, d, w.dy, d, sw.lin2_w, d + dm);
+      g.C = w.dO; g.ldc = d;
+      JAGG_TRY(gemm(g, s));
+      g = dx_gemm(m, M, d, dm, w.dy, d, sw.lin2_w + d, d + dm);
+      g.epi = EPI_MUL_AUX; g.C = at_byte(w.dqkv, (size_t)3 * d * e); g.ldc = ld1; g.aux = k.gp; g.ld_aux = dm;
+      JAGG_TRY(gemm(g, s));
+    }
+    AttnBwdArgs ab;
+    ab.f = attn_args(m, B, seg_single(k.qk, 2 * d, N), seg_single(k.qkv, 3 * d, N), seg_single(k.cat, d + dm, N),
+                     k.lse);
+    ab.f.q_col0 = 0; ab.f.k_col0 = d; ab.f.v_col0 = 2 * d;
+    ab.dO = seg_single(w.dO, d, N);
+    attention_bwd_scratch(w.attn, B, N, m.heads, &ab.Dv, &ab.dq_acc);
+    ab.dq = ab.dk = ab.dv = seg_single(w.dqkv, ld1, N);
+    ab.dq_col0 = 0; ab.dk_col0 = d; ab.dv_col0 = 2 * d;
+    JAGG_TRY(attention_bwd(ab, s));
+    QkNormRopeBwd qb;
+    qb.f = qk_args(m, k.qkv, M, N, Nt, sw.qn, sw.kn, k.qk, k.rq, k.rk);
+    qb.dqk = w.dqkv; qb.ld_dqk = ld1;
+    qb.dqs_txt = qb.dqs_img = grad + sw.qn;
+    qb.dks_txt = qb.dks_img = grad + sw.kn;
+    JAGG_TRY(launch_qk_norm_rope_bwd(qb, s));
+    LnGateBwd prev{};
+    if (l > 0) prev = single_gate(l - 1);
+    JAGG_TRY(qkv_and_ln1_bwd(m, M, N, w.dqkv, ld1, (int)ld1, sw.lin1_w, sw.lin1_b, k.a, k.h_in, k.st1, mod, dmod,
+                             w.dh, l > 0 ? &prev : nullptr, w, grad, s));
+  }
+  if (Ld == 0) return JAGG_OK;
+  // the joint gradient splits into the two streams
+  JAGG_TRY(launch_copy_rows(w.dh, d, Nt, 0, N, w.dhs[0], d, 0, 0, 0, B * Nt, d, 4, s));
+  JAGG_TRY(launch_copy_rows(w.dh, d, Ni, Nt, N, w.dhs[1], d, 0, 0, 0, B * Ni, d, 4, s));
+  // per-stream regions of the gradient buffers: text rows first, image rows after
+  void* dy_s[2] = {w.dy, at_byte(w.dy, (size_t)Mt * d * e)};
+  void* dO_s[2] = {w.dO, at_byte(w.dO, (size_t)Mt * d * e)};
+  void* dqkv_s[2] = {w.dqkv, at_byte(w.dqkv, (size_t)Mt * 3 * d * e)};
+  auto mlp_gate = [&](int l, int si) {
+    const StreamW& sw = m.T.doubles[l].s[si];
+    const int Ns = si ? Ni : Nt;
+    return gate_args(m, B * Ns, Ns, w.dhs[si], S.dbl[l].s[si].y2, S.mod + sw.mod_col + 5 * d,
+                     w.dmod + sw.mod_col + 5 * d, dy_s[si], grad + sw.fc2_b);
+  };
+  for (int si = 0; si < 2; ++si) JAGG_TRY(launch_ln_gate_bwd(mlp_gate(Ld - 1, si), s));
+  for (int l = Ld - 1; l >= 0; --l) {
+    const DoubleW& bw = m.T.doubles[l];
+    const DoubleSaved& k = S.dbl[l];
+    for (int si = 0; si < 2; ++si) {
+      const int Ns = si ? Ni : Nt;
+      JAGG_TRY(mlp_and_proj_bwd(m, B * Ns, Ns, k.s[si], branch_of(bw.s[si]), S.mod + bw.s[si].mod_col,
+                                w.dmod + bw.s[si].mod_col, w.dhs[si], dy_s[si], dO_s[si], w, grad, s));
+    }
+    AttnBwdArgs ab;
+    ab.f = attn_args(m, B, SegRows{k.s[0].qk, k.s[1].qk, 2 * d, 2 * d, Nt},
+                     SegRows{k.s[0].qkv, k.s[1].qkv, 3 * d, 3 * d, Nt}, SegRows{k.s[0].o, k.s[1].o, d, d, Nt}, k.lse);
+    ab.f.q_col0 = 0; ab.f.k_col0 = d; ab.f.v_col0 = 2 * d;
+    ab.dO = SegRows{dO_s[0], dO_s[1], d, d, Nt};
+    attention_bwd_scratch(w.attn, B, N, m.heads, &ab.Dv, &ab.dq_acc);
+    ab.dq = ab.dk = ab.dv = SegRows{dqkv_s[0], dqkv_s[1], 3 * d, 3 * d, Nt};
+    ab.dq_col0 = 0; ab.dk_col0 = d; ab.dv_col0 = 2 * d;
+    JAGG_TRY(attention_bwd(ab, s));
+    for (int si = 0; si < 2; ++si) {
+      const StreamW& sw = bw.s[si];
+      const DitSaved& q = k.s[si];
+      const int Ns = si ? Ni : Nt, Ms = B * Ns;
+      QkNormRopeBwd qb;
+      qb.f = qk_args(m, q.qkv, Ms, Ns, si ? 0 : Ns, sw.qn, sw.kn, q.qk, q.rq, q.rk);
+      qb.dqk = dqkv_s[si]; qb.ld_dqk = 3 * d;
+      qb.dqs_txt = qb.dqs_img = grad + sw.qn;
+      qb.dks_txt = qb.dks_img = grad + sw.kn;
+      JAGG_TRY(launch_qk_norm_rope_bwd(qb, s));
+      LnGateBwd prev{};
+      if (l > 0) prev = mlp_gate(l - 1, si);
+      JAGG_TRY(qkv_and_ln1_bwd(m, Ms, Ns, dqkv_s[si], 3 * d, 3 * d, sw.qkv_w, sw.qkv_b, q.a, q.h_in, q.st1,
+                               S.mod + sw.mod_col, w.dmod + sw.mod_col, w.dhs[si], l > 0 ? &prev : nullptr, w, grad,
+                               s));
+    }
+  }
+  return JAGG_OK;
+}
+
+int forward_impl(const jagg_model& m, const void* z, const float* t, const void* txt, int B, void* v_out,
+                 void* saved, void* ws, cudaStream_t s) {
+  const jagg_config& c = m.cfg;
+  // With a saved arena every activation goes there; otherwise one block's worth of slots
+  // at the start of the workspace is reused by every block.
+  Saved S;
+  const size_t used = carve_saved(m, B, saved ? saved : ws, saved != nullptr, S);
+  void* vt = nullptr;
+  carve_fwd_ws(m, B, static_cast<uint8_t*>(ws) + (saved ? 0 : used), &vt);
+  if (c.arch == JAGG_ARCH_DIT) {
+    float* h0 = S.blk.empty() ? S.h_fin : S.blk[0].h_in;
+    JAGG_TRY(prologue_fwd(m, z, t, txt, B, S, h0, img_rows_of(m), h0, txt_rows_of(m), s));
+    JAGG_TRY(forward_dit(m, S, B, s));
+  } else {
+    if (c.depth_double > 0) {
+      JAGG_TRY(prologue_fwd(m, z, t, txt, B, S, S.dbl[0].s[1].h_in, kContiguous, S.dbl[0].s[0].h_in, kContiguous,
+                            s));
+    } else {
+      float* h0 = S.sgl.empty() ? S.h_fin : S.sgl[0].h_in;
+      JAGG_TRY(prologue_fwd(m, z, t, txt, B, S, h0, img_rows_of(m), h0, txt_rows_of(m), s));
+    }
+    JAGG_TRY(forward_mmdit(m, S, B, s));
+  }
+  return final_fwd(m, B, S, vt, v_out, s);
+}
+
+int vjp_impl(const jagg_model& m, const void* saved, int B, const float* cot, float* grad, void* ws,
+             cudaStream_t s) {
+  const jagg_config& c = m.cfg;
+  Saved S;
+  carve_saved(m, B, const_cast<void*>(saved), true, S);
+  VjpWs w;
+  carve_vjp_ws(m, B, ws, w);
+  JAGG_TRY(zero_vjp_accumulators(m, B, w, s));
+  JAGG_TRY(final_bwd(m, B, S, w, cot, grad, s));
+  if (c.arch == JAGG_ARCH_DIT) {
+    JAGG_TRY(vjp_dit(m, S, B, w, grad, s));
+  } else {
+    JAGG_TRY(vjp_mmdit(m, S, B, w, grad, s));
+    if (c.depth_double > 0)
+      return epilogue_bwd(m, B, S, w, w.dhs[1], kContiguous, w.dhs[0], kContiguous, grad, s);
+  }
+  return epilogue_bwd(m, B, S, w, w.dh, img_rows_of(m), w.dh, txt_rows_of(m), grad, s);
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }

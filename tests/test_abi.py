@@ -46,7 +46,7 @@ def test_main_entry_points_are_declared():
         assert n in names
 
 
-@pytest.mark.parametrize("name", ["tiny_dit_f32", "dit_b_bf16"])
+@pytest.mark.parametrize("name", sorted(synth.WORKLOADS))
 def test_param_table_matches_the_workload_shapes(jg, name):
     wl = synth.WORKLOADS[name]
     cfg = jg.Config.from_workload(wl)

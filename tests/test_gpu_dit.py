@@ -14,12 +14,28 @@ jg = pytest.importorskip("paper_2607_17572_gb300")
 TINY = synth.WORKLOADS["tiny_dit_f32"]
 DITB = synth.WORKLOADS["dit_b_bf16"]
 
+FLUX = synth.WORKLOADS["mmdit_flux512_bf16"]
+TINY_MM = synth.small_variant(TINY, name="tiny_mmdit", arch="mmdit", depth=2, depth_double=2, shift=3.0)
+
 CASES = [
     # (workload, rows B, forward tol, gradient tol)
     (TINY, 8, 1e-5, 1e-4),                                                    # 2G rows of the tiny config
     (synth.small_variant(TINY, name="tiny_odd", latent_h=6, latent_w=5, txt_len=3, txt_dim=40), 3, 1e-5, 1e-4),
     (synth.small_variant(DITB, name="ditb_2blocks", depth=2), 4, 2e-2, 1e-2),  # DiT-B width, 2 blocks
     (synth.small_variant(DITB, name="ditb_ragged", depth=1, latent_h=18, latent_w=22, txt_len=29), 3, 2e-2, 1e-2),
+    # MMDiT: double blocks (per-stream weights, QK RMSNorm, 2D RoPE, joint attention)
+    # followed by Flux-style single blocks
+    (TINY_MM, 8, 1e-5, 1e-4),
+    (synth.small_variant(TINY_MM, name="tiny_mmdit_odd", latent_h=6, latent_w=5, txt_len=3, txt_dim=40), 3,
+     1e-5, 1e-4),
+    (synth.small_variant(TINY_MM, name="tiny_mmdit_doubles_only", depth=0, depth_double=3), 4, 1e-5, 1e-4),
+    (synth.small_variant(TINY_MM, name="tiny_mmdit_singles_only", depth=3, depth_double=0), 4, 1e-5, 1e-4),
+    (synth.small_variant(TINY_MM, name="tiny_mmdit_dh32", hidden=128, heads=4, mlp=256), 2, 1e-5, 1e-4),
+    # bf16 at the Flux head dim (128) and at 64, reduced width and depth
+    (synth.small_variant(FLUX, name="mmdit_dh128_1d1s", hidden=512, heads=4, mlp=2048, depth=1, depth_double=1,
+                         latent_h=16, latent_w=20, txt_len=24, txt_dim=256), 2, 2e-2, 1e-2),
+    (synth.small_variant(FLUX, name="mmdit_dh64_2d1s", hidden=384, heads=6, mlp=1536, depth=1, depth_double=2,
+                         latent_h=14, latent_w=14, txt_len=37, txt_dim=128), 3, 2e-2, 1e-2),
 ]
 
 
@@ -62,8 +78,12 @@ def test_vjp_accumulates_and_is_linear_in_the_cotangent():
     assert rel_l2(grad.cpu().numpy(), 3.0 * g1.cpu().numpy()) < 1e-5
 
 
-def test_forward_without_saves_matches_saved_forward():
-    wl = synth.small_variant(DITB, name="ditb_2blocks", depth=2)
+@pytest.mark.parametrize("wl", [synth.small_variant(DITB, name="ditb_2blocks", depth=2),
+                                synth.small_variant(FLUX, name="mmdit_dh128_2d3s", hidden=512, heads=4, mlp=2048,
+                                                    depth=3, depth_double=2, latent_h=16, latent_w=16, txt_len=40,
+                                                    txt_dim=256)],
+                         ids=lambda w: w.name)
+def test_forward_without_saves_matches_saved_forward(wl):
     params = synth.make_params(wl)
     z, t, txt = model_inputs(wl, 4, 9)
     gm = GpuModel(jg, wl, params)
