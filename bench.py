@@ -50,7 +50,28 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--quick", action="store_true", help="skip the full-W, e2e and CPU legs")
+    p.add_argument("--G", type=int, default=0,
+                   help="override the workload's group size (small cases for profiler captures)")
+    p.add_argument("--vjp-rows", choices=["auto", "group", "window"], default="auto",
+                   help="one joint VJP per group (all windows' rows) or per window; auto picks the group "
+                        "when its saved activations fit in half of the free device memory")
     return p.parse_args()
+
+
+def workload(args):
+    wl = synth.WORKLOADS[args.workload]
+    if args.G:
+        wl = synth.small_variant(wl, name=f"{wl.name}_G{args.G}", G=args.G)
+    return wl
+
+
+def describe(wl) -> str:
+    if wl.arch == "dit":
+        blocks = f"DiT {wl.depth} blocks"
+    else:
+        blocks = f"MMDiT {wl.depth_double} double + {wl.depth} single blocks"
+    return (f"{wl.name}: {blocks} d={wl.hidden} h={wl.heads} mlp={wl.mlp}, {wl.n_img} img + {wl.txt_len} txt "
+            f"tokens, G={wl.G}, T={wl.T}, W={wl.W}, jagg_frac={wl.jagg_frac}")
 
 
 def peaks():
@@ -167,7 +188,11 @@ class Bench:
         self.sig_dev = torch.tensor(self.sig, **f64)
         self.rewards = torch.tensor(self.draws.rewards, dtype=torch.float32, device=dev)
         self.txt1 = torch.tensor(self.draws.txt, dtype=self.tdt, device=dev)
-        self.ws = jg.alloc_bytes(self.model.workspace_bytes(self.nw * W * G), dev)
+        # workspace for the largest single call: every window's W*G rows at once when they
+        # can be resident together, else one window's
+        total = torch.cuda.get_device_properties(dev).total_memory
+        ws_rows = self.nw * W * G if self.model.saved_bytes(self.nw * W * G) < 0.4 * total else W * G
+        self.ws = jg.alloc_bytes(self.model.workspace_bytes(ws_rows), dev)
         self.sws = jg.alloc_bytes(jg.signals_workspace_bytes(G, W, self.D), dev)
         self.gws = jg.alloc_bytes(jg.grad_reduce_workspace_bytes(self.P), dev)
         self.grad = torch.zeros(self.P, dtype=torch.float32, device=dev)
@@ -241,12 +266,27 @@ class Bench:
             r += n
         return out, r
 
-    def forward_saves(self, routes, batched):
-        """Phase 1 with saves for the rows of the plan.  batched: one arena holding every
-        window's rows (one joint VJP per group); otherwise one arena per window."""
+    def batch_group(self, routes, mode) -> bool:
+        """True: one saved arena (and one joint VJP) for every window of the group."""
+        if mode != "auto":
+            return mode == "group"
+        return self.fits(routes)
+
+    def fits(self, routes) -> bool:
+        """Every window's saved activations fit in half of the free device memory."""
+        _, rows = self.plan(routes)
+        free, _ = torch.cuda.mem_get_info(self.dev)
+        return self.model.saved_bytes(rows) < 0.5 * free
+
+    def forward_saves(self, routes, batched, windows=None):
+        """Phase 1 with saves for the rows of the plan (or of the listed windows only).
+        batched: one arena holding every window's rows (one joint VJP per group); otherwise
+        one arena per window."""
         wl = self.wl
         G, W = wl.G, wl.W
         plan, _ = self.plan(routes)
+        if windows is not None:
+            plan = [p for p in plan if p[0] in windows]
         rows = [self.rows(self.z[:, w * W:(w + 1) * W].reshape(G, W, *self.shape), w, jagg)
                 for (w, jagg, _, _) in plan]
         if batched:
@@ -263,8 +303,8 @@ class Bench:
         torch.cuda.synchronize()
         return arenas
 
-    def step(self, arenas):
-        """Phases 2-4 for every window of the group, then the gradient's squared norm."""
+    def step(self, arenas, reduce=True):
+        """Phases 2-4 for the windows of the arenas, then the gradient's squared norm."""
         jg, G, W, D = self.jg, self.wl.G, self.wl.W, self.D
         for saved, B, pl in arenas:
             row0 = pl[0][2]
@@ -275,7 +315,8 @@ class Bench:
                 else:
                     self.signals(w, self.lpo_win[w], s_out=dst.view(G, W, D))
             jg.dit_joint_vjp(self.model, saved, B, self.cot_all[row0:row0 + B], self.grad, self.ws)
-        jg.grad_reduce(self.grad, None, out3=self.out3, ws=self.gws)
+        if reduce:
+            jg.grad_reduce(self.grad, None, out3=self.out3, ws=self.gws)
 
 
 def time_steps(fn, steps, warmup, ws, use_graph):
@@ -301,11 +342,14 @@ def time_steps(fn, steps, warmup, ws, use_graph):
     barrier(ws)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    # the timed steps are the profiled range of `ncu --profile-from-start off`
+    torch.cuda.profiler.start()
     e0.record(stream)
     for _ in range(steps):
         run()
     e1.record(stream)
     torch.cuda.synchronize()
+    torch.cuda.profiler.stop()
     barrier(ws)
     return e0.elapsed_time(e1) / steps, graph
 
@@ -352,7 +396,7 @@ def threads_used():
 def run_reference(args, ws, rank):
     if rank != 0:
         return
-    wl = synth.WORKLOADS[args.workload]
+    wl = workload(args)
     G_sample = 2
     for _ in range(args.warmup):
         oracle_window_sample(wl, G_sample)
@@ -375,92 +419,120 @@ def run_reference(args, ws, rank):
 
 
 # ----------------------------------------------------------------------------- main leg
+def measure(b, routes, batched, args, ws, use_graph, profile=False):
+    """Device time of Phases 2-4 of one group step.
+
+    batched: one saved arena holding every window's rows and one joint VJP per group;
+    otherwise one arena and one joint VJP per window.  When every window's arena fits in
+    device memory at once, the whole step is one timed region; otherwise (MMDiT widths,
+    full-W) each window is timed with its own arena resident and the window times add,
+    the gradient norm counted once."""
+    jg = b.jg
+    res = {"ms": 0.0, "launches": 0, "prof": {}, "rows": 0, "vjps": 0, "saved_gb": 0.0, "resident": True}
+
+    def run_part(arenas, reduce):
+        n0 = jg.launch_count()
+        b.step(arenas, reduce)
+        torch.cuda.synchronize()
+        res["launches"] += jg.launch_count() - n0
+        assert jg.device_status() == 0, "device status set during the step"
+        ms, graph = time_steps(lambda: b.step(arenas, reduce), args.steps, args.warmup, ws, use_graph)
+        del graph
+        res["ms"] += ms
+        res["rows"] = max(res["rows"], max(a[1] for a in arenas))
+        res["vjps"] += len(arenas)
+        res["saved_gb"] = max(res["saved_gb"], sum(a[0].numel() for a in arenas) / 1e9)
+        if profile:  # per-family device time of the same work (events around each launch, eager)
+            jg.profile_enable(True)
+            for _ in range(args.steps):
+                b.step(arenas, reduce)
+            for k, v in jg.profile_read().items():
+                acc = res["prof"].setdefault(k, {"launches": 0.0, "ms": 0.0, "flops": 0.0, "bytes": 0.0})
+                for q in acc:
+                    acc[q] += v[q] / args.steps
+            jg.profile_enable(False)
+
+    if batched or b.fits(routes):
+        run_part(b.forward_saves(routes, batched=batched), True)
+    else:
+        res["resident"] = False
+        for w in range(b.nw):
+            arenas = b.forward_saves(routes, batched=False, windows=[w])
+            run_part(arenas, w == b.nw - 1)
+            del arenas
+            torch.cuda.empty_cache()
+    res["ms"] = max_over_ranks(res["ms"], ws)
+    return res
+
+
 def run_gpu(args, ws, rank):
     import paper_2607_17572_gb300 as jg
     dev = torch.device("cuda", torch.cuda.current_device())
-    wl = synth.WORKLOADS[args.workload]
+    wl = workload(args)
     b = Bench(wl, dev)
     b.rollout()
     routes, _ = jg.jagg_route(b.nw, wl.jagg_frac)
-    arenas = b.forward_saves(routes, batched=True)
-    B = arenas[0][1]
+    batched = b.batch_group(routes, args.vjp_rows)
     use_graph = not args.no_graph
     units = wl.G * wl.T
 
-    # ---- JAGG path, one joint VJP over every window's endpoint rows: timed region
-    n0 = jg.launch_count()
-    b.step(arenas)
-    torch.cuda.synchronize()
-    launches_per_step = jg.launch_count() - n0
-    assert jg.device_status() == 0, "device status set during the JAGG step"
+    # ---- JAGG path: timed region, then the per-family breakdown of the same work
     with ClockSampler(torch.cuda.current_device()) as clk:
-        ms, graph = time_steps(lambda: b.step(arenas), args.steps, args.warmup, ws, use_graph)
+        r = measure(b, routes, batched, args, ws, use_graph, profile=True)
     clocks = clk.summary()
-    ms = max_over_ranks(ms, ws)
+    ms = r["ms"]
     value = ws * units / (ms / 1000.0)
-    del graph
-
-    # ---- per-family device time of the same step (events around each launch, eager)
-    jg.profile_enable(True)
-    for _ in range(args.steps):
-        b.step(arenas)
-    prof = jg.profile_read()
-    jg.profile_enable(False)
     burst, sustained, hbm, src = peaks()
-    fam = {k: v for k, v in prof.items() if v["launches"]}
+    fam = {k: v for k, v in r["prof"].items() if v["launches"]}
     gt = fam.get("gemm_tcgen05", {"launches": 0, "ms": 0.0, "flops": 0.0})
     achieved = gt["flops"] / (gt["ms"] / 1000.0) / 1e12 if gt["ms"] > 0 else 0.0
     roofline = {"bound": "tensor", "achieved": achieved, "peak": sustained, "unit": "TFLOP/s",
                 "frac": achieved / sustained, "traffic": None,
                 "kernel": "gemm_tcgen05 (all dense products of the joint VJP)",
                 "peak_source": f"bf16_tflops_sustained of {src} peaks",
-                "launches_per_step": gt["launches"] / args.steps,
+                "launches_per_step": gt["launches"],
                 "flops_per_launch": gt["flops"] / max(gt["launches"], 1),
                 "ms_per_launch": gt["ms"] / max(gt["launches"], 1)}
-    step_flops = sum(v["flops"] for k, v in fam.items() if k != "gemm_simt") / args.steps
-    families = {k: {"launches_per_step": v["launches"] / args.steps, "ms_per_step": v["ms"] / args.steps,
+    step_flops = sum(v["flops"] for k, v in fam.items() if k != "gemm_simt")
+    families = {k: {"launches_per_step": v["launches"], "ms_per_step": v["ms"],
                     "tflops": (v["flops"] / (v["ms"] / 1000.0) / 1e12) if v["ms"] > 0 else None}
                 for k, v in fam.items()}
-
+    if batched:
+        batching = f"one joint VJP per group over all {b.nw} windows' endpoint rows"
+    else:
+        batching = f"one joint VJP per window ({b.nw} per step)" + (
+            "" if r["resident"] else ", each window timed with its own saved activations resident")
     out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-           "config": {"workload": (f"{wl.name}: DiT {wl.depth} blocks d={wl.hidden} h={wl.heads} mlp={wl.mlp}, "
-                                   f"{wl.n_img} img + {wl.txt_len} txt tokens, G={wl.G}, T={wl.T}, W={wl.W}, "
-                                   f"jagg_frac={wl.jagg_frac}"),
-                      "rows_per_vjp": B, "windows": b.nw, "cuda_graph": use_graph,
-                      "vjp_batching": f"one joint VJP per group over all {b.nw} windows' endpoint rows",
-                      "l2": "inputs larger than L2 (saved activations %.1f GB per step)" % (
-                          sum(a[0].numel() for a in arenas) / 1e9),
+           "config": {"workload": describe(wl), "rows_per_vjp": r["rows"], "windows": b.nw,
+                      "cuda_graph": use_graph, "vjp_batching": batching,
+                      "l2": "inputs larger than L2 (saved activations %.1f GB resident)" % r["saved_gb"],
                       "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU"},
            "roofline": roofline, "algorithmic_tflops_per_step": step_flops / 1e12,
            "step_tflops_per_s": step_flops / (ms / 1000.0) / 1e12, "families": families,
-           "gpu_launches": launches_per_step * args.steps, "clocks": clocks}
-    del arenas
+           "gpu_launches": r["launches"] * args.steps, "clocks": clocks}
     torch.cuda.empty_cache()
 
     if not args.quick:
         # ---- the same JAGG step with one joint VJP per window (Algorithm 1 as written)
-        arenas_w = b.forward_saves(routes, batched=False)
-        ms_w, graph = time_steps(lambda: b.step(arenas_w), args.steps, args.warmup, ws, use_graph)
-        ms_w = max_over_ranks(ms_w, ws)
-        out["per_window_vjp"] = {"value": ws * units / (ms_w / 1000.0), "unit": UNIT, "ms_per_step": ms_w,
-                                 "rows_per_vjp": arenas_w[0][1], "vjps_per_step": len(arenas_w)}
-        del graph, arenas_w
-        # ---- exact per-step path (jagg_frac = 0), batched like the headline
-        arenas_f = b.forward_saves([0] * b.nw, batched=True)
+        if batched:
+            rw = measure(b, routes, False, args, ws, use_graph)
+            out["per_window_vjp"] = {"value": ws * units / (rw["ms"] / 1000.0), "unit": UNIT,
+                                     "ms_per_step": rw["ms"], "rows_per_vjp": rw["rows"], "vjps_per_step": rw["vjps"]}
+        # ---- exact per-step path (jagg_frac = 0), batched like the headline when it fits
+        full = [0] * b.nw
         b.grad.zero_()
-        ms_f, graph = time_steps(lambda: b.step(arenas_f), args.steps, args.warmup, ws, use_graph)
-        ms_f = max_over_ranks(ms_f, ws)
-        out["full_w"] = {"value": ws * units / (ms_f / 1000.0), "unit": UNIT, "ms_per_step": ms_f,
-                         "rows_per_vjp": arenas_f[0][1]}
-        out["jagg_speedup_vs_full_w"] = ms_f / ms
+        rf = measure(b, full, b.batch_group(full, args.vjp_rows), args, ws, use_graph)
+        out["full_w"] = {"value": ws * units / (rf["ms"] / 1000.0), "unit": UNIT, "ms_per_step": rf["ms"],
+                         "rows_per_vjp": rf["rows"], "vjps_per_step": rf["vjps"]}
+        out["jagg_speedup_vs_full_w"] = rf["ms"] / ms
         out["ideal_speedup"] = wl.W / 2
-        del graph, arenas_f
         torch.cuda.empty_cache()
-        if not args.no_e2e:
+        if not args.no_e2e and batched:
             out["e2e"] = run_e2e(b, args, ws, routes)
-        if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        # the float64 oracle needs minutes per sequence at MMDiT width: DiT workloads only
+        if rank == 0 and ws == 1 and not args.no_cpu_baseline and wl.arch == "dit":
             G_sample = 2
             sec, u = oracle_window_sample(wl, G_sample)
             out["cpu_baseline"] = {"value": u / sec, "unit": UNIT, "cores": threads_used(), "kind": "oracle",

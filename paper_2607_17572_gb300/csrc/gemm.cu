@@ -170,8 +170,14 @@ __device__ __forceinline__ void epi_apply8(const EpiParams& e, int m, int n, con
 }
 
 // ------------------------------------------------------------------ tcgen05 kernel
+// Staged epilogues: the output tile goes through swizzled shared memory and leaves with
+// TMA stores (or TMA f32 reduce-adds), and the multiplier of EPI_MUL_AUX arrives in
+// shared memory by TMA before the accumulator is ready.
+enum : int { STAGED_NONE = 0, STAGED_STORE = 1, STAGED_MUL_AUX = 2, STAGED_ACCUM = 3 };
+
 struct TcParams {
   int tiles_m, tiles_n, splits, k_blocks;
+  int staged;  // STAGED_*
   EpiParams e;
 };
 
@@ -184,25 +190,41 @@ struct TcCfg {
   static constexpr int A_BYTES = TC_BM * TC_BK * 2;
   static constexpr int B_BYTES = BN * TC_BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int STAGES = (196608 / STAGE_BYTES) > 8 ? 8 : (196608 / STAGE_BYTES);
-  static constexpr int TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
+  // Per epilogue warp (32 rows): two staging chunks of 32 x 32 outputs (4 KB each for f32;
+  // the bf16 output of EPI_MUL_AUX uses 2 KB each), and for EPI_MUL_AUX the tile's
+  // multiplier rows, BN / 32 chunks of 32 x 32 bf16 after the bf16 staging chunks.
+  static constexpr int CHUNK_BF16 = 32 * 32 * 2;
+  static constexpr int EPI_WARP_BYTES = 2 * CHUNK_BF16 + (BN / 32) * CHUNK_BF16 > 4 * CHUNK_BF16
+                                            ? 2 * CHUNK_BF16 + (BN / 32) * CHUNK_BF16
+                                            : 4 * CHUNK_BF16;
+  static constexpr int EPI_BYTES = 4 * EPI_WARP_BYTES;
   // + 16 KB guard: every descriptor-addressed read stays inside the allocation even if
   // the two byte offsets of an MN-major descriptor were interpreted the other way round.
-  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/ + 16384;
+  static constexpr int FIXED = 1024 /*align*/ + 256 /*barriers*/ + 16384;
+  static constexpr int MAX_SMEM = 232448;
+  static constexpr int FIT = (MAX_SMEM - FIXED - EPI_BYTES) / STAGE_BYTES;
+  static constexpr int STAGES = FIT > 8 ? 8 : FIT;
+  static constexpr int TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EPI_BYTES + FIXED;
+  static_assert(STAGES >= 4, "pipeline too shallow");
+  static_assert(SMEM_BYTES <= MAX_SMEM, "shared memory budget");
 };
 
 template <int BN, bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(TC_THREADS, 1)
-    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, TcParams p) {
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmX, TcParams p) {
   using Cfg = TcCfg<BN>;
   constexpr int STAGES = Cfg::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * Cfg::STAGE_BYTES);
+  uint8_t* epi_smem = smem + STAGES * Cfg::STAGE_BYTES;  // 1024-byte aligned
+  uint64_t* full = reinterpret_cast<uint64_t*>(epi_smem + Cfg::EPI_BYTES);
   uint64_t* empty = full + STAGES;
   uint64_t* tfull = empty + STAGES;
   uint64_t* tempty = tfull + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  uint64_t* auxbar = tempty + 2;  // one per epilogue warp
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(auxbar + 4);
   __shared__ volatile int abort_flag;
 
   const int warp = threadIdx.x >> 5;
@@ -218,9 +240,12 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       ptx::mbar_init(&tfull[a], 1);
       ptx::mbar_init(&tempty[a], 4);
     }
+    for (int q = 0; q < 4; ++q) ptx::mbar_init(&auxbar[q], 1);
     ptx::fence_mbar_init();
     ptx::prefetch_tmap(&tmA);
     ptx::prefetch_tmap(&tmB);
+    if (p.staged != STAGED_NONE) ptx::prefetch_tmap(&tmC);
+    if (p.staged == STAGED_MUL_AUX) ptx::prefetch_tmap(&tmX);
   }
   if (warp == 1) {
     ptx::tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
@@ -315,6 +340,112 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         if (++acc == 2) { acc = 0; acc_phase ^= 1; }
       }
     }
+  } else if (p.staged != STAGED_NONE) {
+    // ---------------- staged epilogue, warps 2..5: TMEM lanes 32*(warp%4) .. +31.
+    // Thread = output row; per 32-column chunk: tcgen05.ld, the element-wise op, a write
+    // into a swizzled staging chunk (64-byte rows for bf16, 128-byte rows for f32, so the
+    // 16-byte writes of a warp hit distinct banks), then one TMA store / reduce-add of the
+    // 32 x 32 box by lane 0.  Two staging chunks alternate.
+    const int q = warp & 3;
+    const bool mul = p.staged == STAGED_MUL_AUX;
+    const bool out_f32 = !p.e.c_bf16;
+    const int chunk_bytes = out_f32 ? 4096 : Cfg::CHUNK_BF16;
+    uint8_t* stg = epi_smem + q * Cfg::EPI_WARP_BYTES;
+    uint8_t* auxs = stg + 2 * Cfg::CHUNK_BF16;  // EPI_MUL_AUX only (bf16 output)
+    int acc = 0, sbuf = 0;
+    uint32_t acc_phase = 0, aux_phase = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x) {
+      int tm, tn, ks;
+      decode(t, tm, tn, ks);
+      const int m0 = tm * TC_BM + q * 32;
+      // boxes wholly outside the output (rows past M, column chunks past N) are skipped
+      const bool rows_live = m0 < p.e.M;
+      const int live_chunks = min(BN / 32, (p.e.N - tn * BN + 31) / 32);
+      const bool aux_load = mul && rows_live;
+      if (aux_load) {
+        // the tile's multiplier rows; this warp finished reading the previous tile's
+        __syncwarp();
+        if (lane == 0) {
+          ptx::mbar_arrive_expect_tx(&auxbar[q], live_chunks * Cfg::CHUNK_BF16);
+          for (int c = 0; c < live_chunks; ++c)
+            ptx::tma_load_2d(auxs + c * Cfg::CHUNK_BF16, &tmX, &auxbar[q], tn * BN + c * 32, m0);
+        }
+      }
+      bool ok = ptx::mbar_wait(&tfull[acc], acc_phase);
+      if (aux_load) {
+        ok = ok && ptx::mbar_wait(&auxbar[q], aux_phase);
+        aux_phase ^= 1u;
+      }
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) { abort_flag = 1; break; }
+      ptx::tc_fence_after();
+#pragma unroll 1
+      for (int c = 0; c < (rows_live ? live_chunks : 0); ++c) {
+        uint32_t r[32];
+        ptx::tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c * 32, r);
+        ptx::tmem_ld_wait();
+        const int n0 = tn * BN + c * 32;
+        float v[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+        if (p.staged == STAGED_STORE && p.e.bias) {
+          if (n0 + 32 <= p.e.N) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] += ldv(p.e.bias, n0 + i, p.e.bias_bf16);
+          } else {
+            for (int i = 0; i < 32; ++i)
+              if (n0 + i < p.e.N) v[i] += ldv(p.e.bias, n0 + i, p.e.bias_bf16);
+          }
+        }
+        if (mul) {
+          const uint8_t* ar = auxs + c * Cfg::CHUNK_BF16 + lane * 64;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const uint4 raw = *reinterpret_cast<const uint4*>(ar + ((j ^ ((lane >> 1) & 3)) << 4));
+            const bf16* h = reinterpret_cast<const bf16*>(&raw);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) v[j * 8 + i] *= __bfloat162float(h[i]);
+          }
+        }
+        // the staging chunk written two chunks ago must have been read by its TMA
+        if (lane == 0) ptx::bulk_wait_read<1>();
+        __syncwarp();
+        uint8_t* sb = stg + sbuf * chunk_bytes;
+        if (out_f32) {
+          uint8_t* row = sb + lane * 128;
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            *reinterpret_cast<float4*>(row + ((j ^ (lane & 7)) << 4)) =
+                make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+        } else {
+          uint8_t* row = sb + lane * 64;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            uint4 raw;
+            __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&raw);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) h2[i] = __floats2bfloat162_rn(v[8 * j + 2 * i], v[8 * j + 2 * i + 1]);
+            *reinterpret_cast<uint4*>(row + ((j ^ ((lane >> 1) & 3)) << 4)) = raw;
+          }
+        }
+        ptx::fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          if (p.staged == STAGED_ACCUM)
+            ptx::tma_reduce_add_2d(&tmC, sb, n0, m0);
+          else
+            ptx::tma_store_2d(&tmC, sb, n0, m0);
+          ptx::bulk_commit();
+        }
+        sbuf ^= 1;
+      }
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(&tempty[acc]);
+      if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+    }
+    if (lane == 0) ptx::bulk_wait<0>();
+    __syncwarp();
   } else {
     // ---------------- epilogue warps 2..5: TMEM lanes 32*(warp%4) .. +31
     const int q = warp & 3;
@@ -454,20 +585,22 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// 2D bf16 tensor map over a row-major [rows, cols] matrix with row pitch `ld` elements.
-int make_tmap(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_cols, int box_rows) {
+// 2D tensor map over a row-major [rows, cols] matrix with row pitch `ld` elements (bf16,
+// or f32 when `f32`), boxes of box_rows x box_cols, the given shared-memory swizzle.
+int make_tmap(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_cols, int box_rows,
+              bool f32 = false, CUtensorMapSwizzle swz = CU_TENSOR_MAP_SWIZZLE_128B) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) {
     set_last_error("cuTensorMapEncodeTiled is not available from the driver");
     return JAGG_ERR_CUDA;
   }
   cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {(cuuint64_t)(ld * 2)};
+  cuuint64_t strides[1] = {(cuuint64_t)(ld * (f32 ? 4 : 2))};
   cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = fn(m, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                  const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
     set_last_error("cuTensorMapEncodeTiled failed (%d) rows=%lld cols=%lld ld=%lld box=%dx%d", (int)r,
                    (long long)rows, (long long)cols, (long long)ld, box_rows, box_cols);
@@ -508,6 +641,24 @@ EpiParams make_epi(const GemmArgs& g) {
   return e;
 }
 
+// Which staged epilogue (if any) serves the product: row-major outputs without row remap,
+// 16-byte aligned with 16-byte row pitches.
+int staged_mode(const GemmArgs& g) {
+  auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
+  if (g.c_trans || g.bias_m || g.remap_rows || !al16(g.C)) return STAGED_NONE;
+  const bool c_f32 = g.c_dtype == JAGG_DTYPE_F32;
+  if ((g.ldc * (c_f32 ? 4 : 2)) % 16) return STAGED_NONE;
+  switch (g.epi) {
+    case EPI_STORE:
+      return (!g.bias || al16(g.bias)) ? STAGED_STORE : STAGED_NONE;
+    case EPI_MUL_AUX:
+      return (!c_f32 && al16(g.aux) && g.ld_aux % 8 == 0) ? STAGED_MUL_AUX : STAGED_NONE;
+    case EPI_ACCUM:
+      return c_f32 ? STAGED_ACCUM : STAGED_NONE;
+  }
+  return STAGED_NONE;
+}
+
 int validate(const GemmArgs& g) {
   JAGG_CHECK_ARG(g.M > 0 && g.N > 0 && g.K > 0, "gemm: empty shape %dx%dx%d", g.M, g.N, g.K);
   JAGG_CHECK_ARG(g.A && g.B && g.C, "gemm: null operand");
@@ -532,6 +683,15 @@ int launch_tc(const GemmArgs& g, cudaStream_t stream) {
   else
     JAGG_TRY(make_tmap(&tb, g.B, g.K, g.N, g.ldb, 64, TC_BK));
   TcParams p;
+  p.staged = staged_mode(g);
+  CUtensorMap tc = ta, tx = ta;  // unused unless staged
+  if (p.staged != STAGED_NONE) {
+    const bool c_f32 = g.c_dtype == JAGG_DTYPE_F32;
+    JAGG_TRY(make_tmap(&tc, g.C, g.M, g.N, g.ldc, 32, 32, c_f32,
+                       c_f32 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B));
+  }
+  if (p.staged == STAGED_MUL_AUX)
+    JAGG_TRY(make_tmap(&tx, g.aux, g.M, g.N, g.ld_aux, 32, 32, false, CU_TENSOR_MAP_SWIZZLE_64B));
   p.tiles_m = ceil_div(g.M, TC_BM);
   p.tiles_n = ceil_div(g.N, BN);
   p.k_blocks = ceil_div(g.K, TC_BK);
@@ -557,7 +717,7 @@ int launch_tc(const GemmArgs& g, cudaStream_t stream) {
     attr_set = true;
   }
   const int tok = prof_start(stream);
-  gemm_tc_kernel<BN, A_MN, B_MN><<<grid, TC_THREADS, Cfg::SMEM_BYTES, stream>>>(ta, tb, p);
+  gemm_tc_kernel<BN, A_MN, B_MN><<<grid, TC_THREADS, Cfg::SMEM_BYTES, stream>>>(ta, tb, tc, tx, p);
   JAGG_LAUNCHED();
   prof_stop(tok, stream, PROF_GEMM_TC, 2.0 * g.M * g.N * g.K,
             2.0 * ((double)g.M * g.K + (double)g.N * g.K) + (double)g.M * g.N * (g.c_dtype == JAGG_DTYPE_F32 ? 4 : 2),

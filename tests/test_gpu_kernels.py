@@ -136,6 +136,46 @@ def test_gemm_accumulate_weight_gradient(split):
     assert _rel(G, ref) < 1e-5
 
 
+@pytest.mark.parametrize("M,N,K", [(300, 200, 192), (77, 1000, 320), (4099, 384, 512)])
+def test_gemm_outputs_inside_wider_buffers(M, N, K):
+    """Outputs written as a column block of a wider buffer (row pitch > N, 16-byte aligned
+    offset), the multiplier read likewise, bf16 stores with a bias and a ragged last column
+    chunk, and an accumulation into a sub-block: the shared-memory-staged epilogues."""
+    torch.manual_seed(M + 5 * N + K)
+    dev = "cuda"
+    A = torch.randn(M, K, device=dev).bfloat16()
+    B = (torch.randn(N, K, device=dev) / math.sqrt(K)).bfloat16()
+    bias = torch.randn(N, device=dev).bfloat16()
+    acc = A.float() @ B.float().t()
+    pad, off = 72, 24                      # columns before and after the block (16-byte multiples)
+    ld = off + N + pad
+    # bf16 store with bias into columns [off, off + N) of a [M, ld] buffer
+    big = torch.full((M, ld), 7.0, device=dev, dtype=torch.bfloat16)
+    view = big[:, off:]
+    jg.test_gemm(_desc(M, N, K, A, K, 0, B, K, 0, jg.DTYPE_BF16, view, ld, jg.DTYPE_BF16, bias=bias))
+    torch.cuda.synchronize()
+    assert _rel(big[:, off:off + N].float(), acc + bias.float()) < 5e-3
+    assert (big[:, :off] == 7.0).all() and (big[:, off + N:] == 7.0).all()
+    # multiply by a factor that is itself a column block of a wider buffer
+    auxbig = torch.randn(M, ld, device=dev).bfloat16()
+    out = torch.full((M, ld), 7.0, device=dev, dtype=torch.bfloat16)
+    jg.test_gemm(_desc(M, N, K, A, K, 0, B, K, 0, jg.DTYPE_BF16, out[:, off:], ld, jg.DTYPE_BF16, epi=3,
+                       aux=auxbig[:, off:], ld_aux=ld))
+    torch.cuda.synchronize()
+    assert _rel(out[:, off:off + N].float(), acc * auxbig[:, off:off + N].float()) < 5e-3
+    assert (out[:, :off] == 7.0).all() and (out[:, off + N:] == 7.0).all()
+    # f32 accumulation into a sub-block, with and without split-K
+    for split in (1, 4):
+        G0 = torch.randn(M, ld, device=dev)
+        G = G0.clone()
+        jg.test_gemm(_desc(M, N, K, A, K, 0, B, K, 0, jg.DTYPE_BF16, G[:, off:], ld, jg.DTYPE_F32, epi=4,
+                           split_k=split))
+        torch.cuda.synchronize()
+        assert _rel(G[:, off:off + N], G0[:, off:off + N] + acc) < 1e-5
+        assert torch.equal(G[:, :off], G0[:, :off]) and torch.equal(G[:, off + N:], G0[:, off + N:])
+    assert jg.device_status() == 0
+
+
 @pytest.mark.parametrize("M,N,K,a_mn,b_mn", [(16, 4608, 768, 0, 0), (16, 768, 56832, 0, 1), (56832, 768, 16, 1, 1),
                                               (40, 70, 33, 0, 0), (7, 9, 11, 1, 0)])
 def test_simt_gemm_f32(M, N, K, a_mn, b_mn):
