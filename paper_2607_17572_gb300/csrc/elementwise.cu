@@ -191,132 +191,170 @@ __device__ __forceinline__ void store4(void* p, int64_t i, int is_f32, const flo
 constexpr int LNF_R = 4;
 constexpr int LNF_ROWS = 8 * LNF_R;
 
-__global__ void __launch_bounds__(256) ln_gate_fused_kernel(LnGateBwd a) {
+// Persistent: the grid walks the (sequence, row-chunk) units, so no wave tail.  NVT > 0
+// fixes the number of float4 column groups per lane (d = 128 NVT) at compile time, so the
+// column loops unroll and a warp's loads for its rows are issued together.
+#ifndef LNF_MIN_BLOCKS
+#define LNF_MIN_BLOCKS 3
+#endif
+template <int NVT>
+__global__ void __launch_bounds__(256, LNF_MIN_BLOCKS) ln_gate_fused_kernel(LnGateBwd a) {
   extern __shared__ float part[];  // [4 quantities][4][d/4]
   const int d = a.d, d4 = a.d / 4;
   const int chunks = (a.rows_per_seq + LNF_ROWS - 1) / LNF_ROWS;
-  const int b = blockIdx.x / chunks;
-  const int r0 = (blockIdx.x % chunks) * LNF_ROWS;
-  for (int i = threadIdx.x; i < 4 * d; i += blockDim.x) part[i] = 0.f;
-  __syncthreads();
+  const int units = (a.M / a.rows_per_seq) * chunks;
   const int warp = threadIdx.x / 32, lane = threadIdx.x & 31;
   const int is_f32 = a.dtype == JAGG_DTYPE_F32;
-  const int nv = (d + 127) / 128;
-  const float* gate = a.do_gate ? a.gate + (int64_t)b * a.mod_stride : nullptr;
-  const float* sc = a.do_ln ? a.scale + (int64_t)b * a.mod_stride : nullptr;
-  int mrow[LNF_R];
-  int64_t hrow[LNF_R];
-  bool live[LNF_R];
-  float mu[LNF_R], rs[LNF_R], s1[LNF_R], s2[LNF_R];
-#pragma unroll
-  for (int k = 0; k < LNF_R; ++k) {
-    const int r = r0 + warp * LNF_R + k;
-    live[k] = r < a.rows_per_seq;
-    mrow[k] = b * a.rows_per_seq + (live[k] ? r : 0);
-    hrow[k] = seg_row(mrow[k], a.seg, a.seg_off, a.seg_stride);
-    mu[k] = rs[k] = s1[k] = s2[k] = 0.f;
-  }
-  if (a.do_ln) {
+  const int nv = NVT > 0 ? NVT : (d + 127) / 128;
+  for (int unit = blockIdx.x; unit < units; unit += gridDim.x) {
+    const int b = unit / chunks;
+    const int r0 = (unit % chunks) * LNF_ROWS;
+    for (int i = threadIdx.x; i < 4 * d; i += blockDim.x) part[i] = 0.f;
+    __syncthreads();
+    const float* gate = a.do_gate ? a.gate + (int64_t)b * a.mod_stride : nullptr;
+    const float* sc = a.do_ln ? a.scale + (int64_t)b * a.mod_stride : nullptr;
+    int mrow[LNF_R];
+    int64_t hrow[LNF_R];
+    bool live[LNF_R];
+    float mu[LNF_R], rs[LNF_R], s1[LNF_R], s2[LNF_R];
 #pragma unroll
     for (int k = 0; k < LNF_R; ++k) {
-      if (live[k]) {
-        mu[k] = a.mean[mrow[k]];
-        rs[k] = a.rstd[mrow[k]];
-      }
+      const int r = r0 + warp * LNF_R + k;
+      live[k] = r < a.rows_per_seq;
+      mrow[k] = b * a.rows_per_seq + (live[k] ? r : 0);
+      hrow[k] = seg_row(mrow[k], a.seg, a.seg_off, a.seg_stride);
+      mu[k] = rs[k] = s1[k] = s2[k] = 0.f;
     }
-    for (int i = 0; i < nv; ++i) {
-      const int c = (i * 32 + lane) * 4;
-      if (c >= d) continue;
-      const float4 s4 = *reinterpret_cast<const float4*>(sc + c);
-      const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
+    if (a.do_ln) {
 #pragma unroll
       for (int k = 0; k < LNF_R; ++k) {
-        if (!live[k]) continue;
-        float dm[4];
-        load4(a.dm, (int64_t)mrow[k] * d + c, a.dm_f32, dm);
-        const float4 h4 = *reinterpret_cast<const float4*>(a.h + hrow[k] * d + c);
-        const float hv[4] = {h4.x, h4.y, h4.z, h4.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float dxh = dm[e] * (1.f + sv[e]);
-          s1[k] += dxh;
-          s2[k] += dxh * (hv[e] - mu[k]) * rs[k];
+        if (live[k]) {
+          mu[k] = a.mean[mrow[k]];
+          rs[k] = a.rstd[mrow[k]];
         }
+      }
+#pragma unroll
+      for (int i = 0; i < (NVT > 0 ? NVT : 1); ++i) {
+        for (int ii = i; ii < (NVT > 0 ? i + 1 : nv); ++ii) {
+          const int c = (ii * 32 + lane) * 4;
+          if (c >= d) continue;
+          const float4 s4 = *reinterpret_cast<const float4*>(sc + c);
+          const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
+#pragma unroll
+          for (int k = 0; k < LNF_R; ++k) {
+            if (!live[k]) continue;
+            float dm[4];
+            load4(a.dm, (int64_t)mrow[k] * d + c, a.dm_f32, dm);
+            const float4 h4 = *reinterpret_cast<const float4*>(a.h + hrow[k] * d + c);
+            const float hv[4] = {h4.x, h4.y, h4.z, h4.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float dxh = dm[e] * (1.f + sv[e]);
+              s1[k] += dxh;
+              s2[k] += dxh * (hv[e] - mu[k]) * rs[k];
+            }
+          }
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < LNF_R; ++k) {
+        s1[k] = warp_sum(s1[k]) / d;
+        s2[k] = warp_sum(s2[k]) / d;
       }
     }
 #pragma unroll
-    for (int k = 0; k < LNF_R; ++k) {
-      s1[k] = warp_sum(s1[k]) / d;
-      s2[k] = warp_sum(s2[k]) / d;
-    }
-  }
-  for (int i = 0; i < nv; ++i) {
-    const int c = (i * 32 + lane) * 4;
-    if (c >= d) continue;
-    float acc[4][4];  // [quantity][element]
+    for (int i = 0; i < (NVT > 0 ? NVT : 1); ++i) {
+      for (int ii = i; ii < (NVT > 0 ? i + 1 : nv); ++ii) {
+        const int c = (ii * 32 + lane) * 4;
+        if (c >= d) continue;
+        float acc[4][4];  // [quantity][element]
 #pragma unroll
-    for (int q = 0; q < 4; ++q)
+        for (int q = 0; q < 4; ++q)
 #pragma unroll
-      for (int e = 0; e < 4; ++e) acc[q][e] = 0.f;
-    float sv[4] = {0.f, 0.f, 0.f, 0.f}, gv[4] = {0.f, 0.f, 0.f, 0.f};
-    if (a.do_ln) {
-      const float4 s4 = *reinterpret_cast<const float4*>(sc + c);
-      sv[0] = s4.x; sv[1] = s4.y; sv[2] = s4.z; sv[3] = s4.w;
-    }
-    if (gate) {
-      const float4 g4 = *reinterpret_cast<const float4*>(gate + c);
-      gv[0] = g4.x; gv[1] = g4.y; gv[2] = g4.z; gv[3] = g4.w;
-    }
+          for (int e = 0; e < 4; ++e) acc[q][e] = 0.f;
+        float sv[4] = {0.f, 0.f, 0.f, 0.f}, gv[4] = {0.f, 0.f, 0.f, 0.f};
+        if (a.do_ln) {
+          const float4 s4 = *reinterpret_cast<const float4*>(sc + c);
+          sv[0] = s4.x; sv[1] = s4.y; sv[2] = s4.z; sv[3] = s4.w;
+        }
+        if (gate) {
+          const float4 g4 = *reinterpret_cast<const float4*>(gate + c);
+          gv[0] = g4.x; gv[1] = g4.y; gv[2] = g4.z; gv[3] = g4.w;
+        }
 #pragma unroll
-    for (int k = 0; k < LNF_R; ++k) {
-      if (!live[k]) continue;
-      const float4 d4 = *reinterpret_cast<const float4*>(a.dh_in + hrow[k] * d + c);
-      float dh[4] = {d4.x, d4.y, d4.z, d4.w};
+        for (int k = 0; k < LNF_R; ++k) {
+          if (!live[k]) continue;
+          const float4 d4v = *reinterpret_cast<const float4*>(a.dh_in + hrow[k] * d + c);
+          float dh[4] = {d4v.x, d4v.y, d4v.z, d4v.w};
+          if (a.do_ln) {
+            float dm[4];
+            load4(a.dm, (int64_t)mrow[k] * d + c, a.dm_f32, dm);
+            const float4 h4 = *reinterpret_cast<const float4*>(a.h + hrow[k] * d + c);
+            const float hv[4] = {h4.x, h4.y, h4.z, h4.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float xh = (hv[e] - mu[k]) * rs[k];
+              dh[e] += rs[k] * (dm[e] * (1.f + sv[e]) - s1[k] - xh * s2[k]);
+              acc[0][e] += dm[e];
+              acc[1][e] += dm[e] * xh;
+            }
+            *reinterpret_cast<float4*>(a.dh_out + hrow[k] * d + c) = make_float4(dh[0], dh[1], dh[2], dh[3]);
+          }
+          if (gate) {
+            const float dy[4] = {gv[0] * dh[0], gv[1] * dh[1], gv[2] * dh[2], gv[3] * dh[3]};
+            store4(a.dy, (int64_t)mrow[k] * d + c, is_f32, dy);
+            float yv[4];
+            load4(a.y, (int64_t)mrow[k] * d + c, is_f32, yv);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              acc[2][e] += dh[e] * yv[e];
+              acc[3][e] += dh[e];
+            }
+          }
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          if (q < 2 ? !a.do_ln : !gate) continue;
+#pragma unroll
+          for (int e = 0; e < 4; ++e) atomicAdd(&part[(q * 4 + e) * d4 + c / 4], acc[q][e]);
+        }
+      }
+    }
+    __syncthreads();
+    for (int c = threadIdx.x; c < d; c += blockDim.x) {
+      auto P = [&](int q) { return part[(q * 4 + c % 4) * d4 + c / 4]; };
       if (a.do_ln) {
-        float dm[4];
-        load4(a.dm, (int64_t)mrow[k] * d + c, a.dm_f32, dm);
-        const float4 h4 = *reinterpret_cast<const float4*>(a.h + hrow[k] * d + c);
-        const float hv[4] = {h4.x, h4.y, h4.z, h4.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float xh = (hv[e] - mu[k]) * rs[k];
-          dh[e] += rs[k] * (dm[e] * (1.f + sv[e]) - s1[k] - xh * s2[k]);
-          acc[0][e] += dm[e];
-          acc[1][e] += dm[e] * xh;
-        }
-        *reinterpret_cast<float4*>(a.dh_out + hrow[k] * d + c) = make_float4(dh[0], dh[1], dh[2], dh[3]);
+        atomicAdd(a.dshift + (int64_t)b * a.dmod_stride + c, P(0));
+        atomicAdd(a.dscale + (int64_t)b * a.dmod_stride + c, P(1));
       }
-      if (gate) {
-        const float dy[4] = {gv[0] * dh[0], gv[1] * dh[1], gv[2] * dh[2], gv[3] * dh[3]};
-        store4(a.dy, (int64_t)mrow[k] * d + c, is_f32, dy);
-        float yv[4];
-        load4(a.y, (int64_t)mrow[k] * d + c, is_f32, yv);
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          acc[2][e] += dh[e] * yv[e];
-          acc[3][e] += dh[e];
-        }
+      if (a.do_gate) {
+        atomicAdd(a.dgate + (int64_t)b * a.dmod_stride + c, P(2));
+        if (a.dbias) atomicAdd(a.dbias + c, gate[c] * P(3));
       }
     }
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      if (q < 2 ? !a.do_ln : !gate) continue;
-#pragma unroll
-      for (int e = 0; e < 4; ++e) atomicAdd(&part[(q * 4 + e) * d4 + c / 4], acc[q][e]);
-    }
+    __syncthreads();  // the partials are re-zeroed by the next unit
   }
-  __syncthreads();
-  for (int c = threadIdx.x; c < d; c += blockDim.x) {
-    auto P = [&](int q) { return part[(q * 4 + c % 4) * d4 + c / 4]; };
-    if (a.do_ln) {
-      atomicAdd(a.dshift + (int64_t)b * a.dmod_stride + c, P(0));
-      atomicAdd(a.dscale + (int64_t)b * a.dmod_stride + c, P(1));
-    }
-    if (a.do_gate) {
-      atomicAdd(a.dgate + (int64_t)b * a.dmod_stride + c, P(2));
-      if (a.dbias) atomicAdd(a.dbias + c, gate[c] * P(3));
-    }
+}
+
+template <int NVT>
+int launch_ln_gate_nv(const LnGateBwd& a, int smem, cudaStream_t s) {
+  static bool attr = false;
+  if (!attr) {
+    JAGG_CUDA_TRY(cudaFuncSetAttribute(ln_gate_fused_kernel<NVT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       4 * 3072 * (int)sizeof(float)));
+    attr = true;
   }
+  static int per_sm = 0;
+  if (!per_sm) {
+    JAGG_CUDA_TRY(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ln_gate_fused_kernel<NVT>, 256,
+                                                                4 * 3072 * (int)sizeof(float)));
+    if (per_sm < 1) per_sm = 1;
+  }
+  const int units = (a.M / a.rows_per_seq) * ceil_div(a.rows_per_seq, LNF_ROWS);
+  const int cap = per_sm * sm_count();
+  ln_gate_fused_kernel<NVT><<<units < cap ? units : cap, 256, smem, s>>>(a);
+  JAGG_LAUNCHED();
+  return JAGG_OK;
 }
 
 // ------------------------------------------------------------------ reductions / copies
@@ -570,16 +608,18 @@ int launch_ln_gate_bwd(const LnGateBwd& a, cudaStream_t s) {
   JAGG_CHECK_ARG(a.M % a.rows_per_seq == 0, "ln_gate_bwd: rows not a whole number of sequences");
   if (!a.do_ln && !a.do_gate) return JAGG_OK;
   const int smem = 4 * a.d * (int)sizeof(float);
-  static bool attr = false;
-  if (!attr) {
-    JAGG_CUDA_TRY(cudaFuncSetAttribute(ln_gate_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       4 * 3072 * (int)sizeof(float)));
-    attr = true;
-  }
-  const int blocks = (a.M / a.rows_per_seq) * ceil_div(a.rows_per_seq, LNF_ROWS);
   const int tok = prof_start(s);
-  ln_gate_fused_kernel<<<blocks, 256, smem, s>>>(a);
-  JAGG_LAUNCHED();
+  int st;
+  switch (a.d % 128 == 0 ? a.d / 128 : 0) {
+    case 3: st = launch_ln_gate_nv<3>(a, smem, s); break;
+    case 4: st = launch_ln_gate_nv<4>(a, smem, s); break;
+    case 6: st = launch_ln_gate_nv<6>(a, smem, s); break;
+    case 8: st = launch_ln_gate_nv<8>(a, smem, s); break;
+    case 12: st = launch_ln_gate_nv<12>(a, smem, s); break;
+    case 24: st = launch_ln_gate_nv<24>(a, smem, s); break;
+    default: st = launch_ln_gate_nv<0>(a, smem, s); break;
+  }
+  JAGG_TRY(st);
   // algorithmic bytes: dh read + write (f32), dm (f32), h (f32), y and dy (storage type)
   const double elem = (double)a.M * a.d;
   prof_stop(tok, s, PROF_LN_BWD, 0.0,

@@ -185,7 +185,9 @@ constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;
 constexpr int TC_THREADS = 192;
 
-template <int BN>
+// AUX: the instance can run EPI_MUL_AUX (the input-gradient products, K-major A and
+// MN-major B); the others need no shared memory for a multiplier.
+template <int BN, bool AUX>
 struct TcCfg {
   static constexpr int A_BYTES = TC_BM * TC_BK * 2;
   static constexpr int B_BYTES = BN * TC_BK * 2;
@@ -194,13 +196,11 @@ struct TcCfg {
   // the bf16 output of EPI_MUL_AUX uses 2 KB each), and for EPI_MUL_AUX the tile's
   // multiplier rows, BN / 32 chunks of 32 x 32 bf16 after the bf16 staging chunks.
   static constexpr int CHUNK_BF16 = 32 * 32 * 2;
-  static constexpr int EPI_WARP_BYTES = 2 * CHUNK_BF16 + (BN / 32) * CHUNK_BF16 > 4 * CHUNK_BF16
-                                            ? 2 * CHUNK_BF16 + (BN / 32) * CHUNK_BF16
-                                            : 4 * CHUNK_BF16;
+  static constexpr int AUX_WARP_BYTES = 2 * CHUNK_BF16 + (BN / 32) * CHUNK_BF16;
+  static constexpr int EPI_WARP_BYTES =
+      AUX && AUX_WARP_BYTES > 4 * CHUNK_BF16 ? AUX_WARP_BYTES : 4 * CHUNK_BF16;
   static constexpr int EPI_BYTES = 4 * EPI_WARP_BYTES;
-  // + 16 KB guard: every descriptor-addressed read stays inside the allocation even if
-  // the two byte offsets of an MN-major descriptor were interpreted the other way round.
-  static constexpr int FIXED = 1024 /*align*/ + 256 /*barriers*/ + 16384;
+  static constexpr int FIXED = 1024 /*align*/ + 256 /*barriers*/;
   static constexpr int MAX_SMEM = 232448;
   static constexpr int FIT = (MAX_SMEM - FIXED - EPI_BYTES) / STAGE_BYTES;
   static constexpr int STAGES = FIT > 8 ? 8 : FIT;
@@ -214,7 +214,7 @@ template <int BN, bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(TC_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmX, TcParams p) {
-  using Cfg = TcCfg<BN>;
+  using Cfg = TcCfg<BN, !A_MN && B_MN>;
   constexpr int STAGES = Cfg::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -672,7 +672,7 @@ int validate(const GemmArgs& g) {
 
 template <int BN, bool A_MN, bool B_MN>
 int launch_tc(const GemmArgs& g, cudaStream_t stream) {
-  using Cfg = TcCfg<BN>;
+  using Cfg = TcCfg<BN, !A_MN && B_MN>;
   CUtensorMap ta, tb;
   if (!A_MN)
     JAGG_TRY(make_tmap(&ta, g.A, g.M, g.K, g.lda, TC_BK, TC_BM));
@@ -690,6 +690,7 @@ int launch_tc(const GemmArgs& g, cudaStream_t stream) {
     JAGG_TRY(make_tmap(&tc, g.C, g.M, g.N, g.ldc, 32, 32, c_f32,
                        c_f32 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B));
   }
+  if (p.staged == STAGED_MUL_AUX && (A_MN || !B_MN)) p.staged = STAGED_NONE;  // no multiplier space
   if (p.staged == STAGED_MUL_AUX)
     JAGG_TRY(make_tmap(&tx, g.aux, g.M, g.N, g.ld_aux, 32, 32, false, CU_TENSOR_MAP_SWIZZLE_64B));
   p.tiles_m = ceil_div(g.M, TC_BM);
