@@ -26,7 +26,9 @@ extern "C" {
  * MN-major (B[k*ldb + n]).  a_dtype/b_dtype/c_dtype/bias_dtype are JAGG_DTYPE_*; C2 and aux
  * follow c_dtype for gelu/dgelu and are f32 for gate.  force_simt selects the SIMT kernel
  * instead of the tcgen05 one (bf16 operands only take the tensor-core path).  For store and
- * accum, c_trans writes element (m, n) to C[n*ldc + m] and bias_m indexes the bias by m. */
+ * accum, c_trans writes element (m, n) to C[n*ldc + m] and bias_m indexes the bias by m.
+ * tile_n forces the tensor-core tile width (64, 128 or 256 columns; 0 = the library's
+ * choice); a width the product cannot use returns JAGG_ERR_ARG. */
 typedef struct jagg_gemm_desc {
   int32_t M, N, K;
   const void* A;
@@ -52,6 +54,7 @@ typedef struct jagg_gemm_desc {
   int32_t force_simt;
   int32_t c_trans;
   int32_t bias_m;
+  int32_t tile_n;
 } jagg_gemm_desc;
 
 int jagg_test_gemm(const jagg_gemm_desc* desc, cudaStream_t stream);

@@ -57,7 +57,8 @@ class GemmDesc(ctypes.Structure):
                 ("ldc2", ctypes.c_int64), ("aux", ctypes.c_void_p), ("ld_aux", ctypes.c_int64),
                 ("gate", ctypes.c_void_p), ("gate_stride", ctypes.c_int64),
                 ("rows_per_seq", ctypes.c_int32), ("split_k", ctypes.c_int32),
-                ("force_simt", ctypes.c_int32), ("c_trans", ctypes.c_int32), ("bias_m", ctypes.c_int32)]
+                ("force_simt", ctypes.c_int32), ("c_trans", ctypes.c_int32), ("bias_m", ctypes.c_int32),
+                ("tile_n", ctypes.c_int32)]
 
 
 class ProfileStat(ctypes.Structure):

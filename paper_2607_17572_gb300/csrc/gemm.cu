@@ -210,11 +210,11 @@ struct TcCfg {
   static_assert(SMEM_BYTES <= MAX_SMEM, "shared memory budget");
 };
 
-template <int BN, bool A_MN, bool B_MN>
+template <int BN, bool A_MN, bool B_MN, bool AUX>
 __global__ void __launch_bounds__(TC_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmX, TcParams p) {
-  using Cfg = TcCfg<BN, !A_MN && B_MN>;
+  using Cfg = TcCfg<BN, AUX>;
   constexpr int STAGES = Cfg::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -641,6 +641,30 @@ EpiParams make_epi(const GemmArgs& g) {
   return e;
 }
 
+// Split-K factor: accumulating products whose tiles do not cover the SMs split K.
+int choose_splits(const GemmArgs& g, int BN, int nsm) {
+  if (g.epi != EPI_ACCUM) return 1;
+  const int k_blocks = ceil_div(g.K, TC_BK);
+  const int tiles = ceil_div(g.M, TC_BM) * ceil_div(g.N, BN);
+  int splits = 1;
+  if (g.split_k > 0)
+    splits = g.split_k;
+  else if (tiles < nsm)
+    splits = (nsm + tiles - 1) / tiles;
+  if (splits > k_blocks) splits = k_blocks;
+  return splits < 1 ? 1 : splits;
+}
+
+// Relative duration of the product with BN-wide tiles: waves of work units times the
+// work per unit, over the tile's relative efficiency (FLOP per byte of operand traffic).
+double tile_cost(const GemmArgs& g, int BN, int nsm) {
+  const int splits = choose_splits(g, BN, nsm);
+  const long long units = (long long)ceil_div(g.M, TC_BM) * ceil_div(g.N, BN) * splits;
+  const double waves = (double)((units + nsm - 1) / nsm);
+  const double eff = BN >= 256 ? 1.33 : 1.0;
+  return waves * BN * ((double)ceil_div(g.K, TC_BK) / splits) / eff;
+}
+
 // Which staged epilogue (if any) serves the product: row-major outputs without row remap,
 // 16-byte aligned with 16-byte row pitches.
 int staged_mode(const GemmArgs& g) {
@@ -670,9 +694,9 @@ int validate(const GemmArgs& g) {
   return JAGG_OK;
 }
 
-template <int BN, bool A_MN, bool B_MN>
+template <int BN, bool A_MN, bool B_MN, bool AUX>
 int launch_tc(const GemmArgs& g, cudaStream_t stream) {
-  using Cfg = TcCfg<BN, !A_MN && B_MN>;
+  using Cfg = TcCfg<BN, AUX>;
   CUtensorMap ta, tb;
   if (!A_MN)
     JAGG_TRY(make_tmap(&ta, g.A, g.M, g.K, g.lda, TC_BK, TC_BM));
@@ -690,35 +714,25 @@ int launch_tc(const GemmArgs& g, cudaStream_t stream) {
     JAGG_TRY(make_tmap(&tc, g.C, g.M, g.N, g.ldc, 32, 32, c_f32,
                        c_f32 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B));
   }
-  if (p.staged == STAGED_MUL_AUX && (A_MN || !B_MN)) p.staged = STAGED_NONE;  // no multiplier space
+  if (p.staged == STAGED_MUL_AUX && !AUX) p.staged = STAGED_NONE;  // no multiplier space
   if (p.staged == STAGED_MUL_AUX)
     JAGG_TRY(make_tmap(&tx, g.aux, g.M, g.N, g.ld_aux, 32, 32, false, CU_TENSOR_MAP_SWIZZLE_64B));
   p.tiles_m = ceil_div(g.M, TC_BM);
   p.tiles_n = ceil_div(g.N, BN);
   p.k_blocks = ceil_div(g.K, TC_BK);
   const int nsm = sm_count();
-  int splits = 1;
-  if (g.epi == EPI_ACCUM) {
-    const int tiles = p.tiles_m * p.tiles_n;
-    if (g.split_k > 0)
-      splits = g.split_k;
-    else if (tiles < nsm)
-      splits = (nsm + tiles - 1) / tiles;
-    if (splits > p.k_blocks) splits = p.k_blocks;
-    if (splits < 1) splits = 1;
-  }
-  p.splits = splits;
+  p.splits = choose_splits(g, BN, nsm);
   p.e = make_epi(g);
   const int total = p.tiles_m * p.tiles_n * p.splits;
   const int grid = total < nsm ? total : nsm;
   static bool attr_set = false;  // one per template instance
   if (!attr_set) {
-    JAGG_CUDA_TRY(cudaFuncSetAttribute(gemm_tc_kernel<BN, A_MN, B_MN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    JAGG_CUDA_TRY(cudaFuncSetAttribute(gemm_tc_kernel<BN, A_MN, B_MN, AUX>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Cfg::SMEM_BYTES));
     attr_set = true;
   }
   const int tok = prof_start(stream);
-  gemm_tc_kernel<BN, A_MN, B_MN><<<grid, TC_THREADS, Cfg::SMEM_BYTES, stream>>>(ta, tb, tc, tx, p);
+  gemm_tc_kernel<BN, A_MN, B_MN, AUX><<<grid, TC_THREADS, Cfg::SMEM_BYTES, stream>>>(ta, tb, tc, tx, p);
   JAGG_LAUNCHED();
   prof_stop(tok, stream, PROF_GEMM_TC, 2.0 * g.M * g.N * g.K,
             2.0 * ((double)g.M * g.K + (double)g.N * g.K) + (double)g.M * g.N * (g.c_dtype == JAGG_DTYPE_F32 ? 4 : 2),
@@ -728,9 +742,25 @@ int launch_tc(const GemmArgs& g, cudaStream_t stream) {
 
 template <bool A_MN, bool B_MN>
 int dispatch_bn(const GemmArgs& g, cudaStream_t stream) {
-  // Every K-major box stays inside its tensor's outer extent (N >= BN).
-  if (g.N < 128) return launch_tc<64, A_MN, B_MN>(g, stream);
-  return launch_tc<128, A_MN, B_MN>(g, stream);
+  // The multiplier epilogue needs its own shared memory: the input-gradient instance
+  // (K-major A, MN-major B) with BN <= 128.
+  JAGG_CHECK_ARG(g.tile_n == 0 || g.tile_n == 64 || g.tile_n == 128 || g.tile_n == 256, "gemm: tile width %d",
+                 g.tile_n);
+  if constexpr (!A_MN && B_MN) {
+    if (staged_mode(g) == STAGED_MUL_AUX) {
+      JAGG_CHECK_ARG(g.tile_n != 256, "gemm: the multiplier epilogue uses tiles of at most 128 columns");
+      if (g.tile_n == 64 || (g.tile_n == 0 && g.N < 128)) return launch_tc<64, A_MN, B_MN, true>(g, stream);
+      return launch_tc<128, A_MN, B_MN, true>(g, stream);
+    }
+  }
+  if (g.tile_n == 64 || (g.tile_n == 0 && g.N < 128)) return launch_tc<64, A_MN, B_MN, false>(g, stream);
+  if (g.tile_n == 128) return launch_tc<128, A_MN, B_MN, false>(g, stream);
+  if (g.tile_n == 256) return launch_tc<256, A_MN, B_MN, false>(g, stream);
+  // Wider tiles halve the B-operand traffic per FLOP (the products are bound by L2
+  // bandwidth at 128 x 128), at the price of coarser waves over the SMs.
+  const int nsm = sm_count();
+  if (g.N >= 256 && tile_cost(g, 256, nsm) < tile_cost(g, 128, nsm)) return launch_tc<256, A_MN, B_MN, false>(g, stream);
+  return launch_tc<128, A_MN, B_MN, false>(g, stream);
 }
 
 bool tc_eligible(const GemmArgs& g) {

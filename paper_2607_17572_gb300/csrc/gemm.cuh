@@ -50,6 +50,7 @@ struct GemmArgs {
   // indexed by m instead of n.
   bool c_trans = false;
   bool bias_m = false;
+  int tile_n = 0;  // tensor-core tile width (64 / 128 / 256); 0 = chosen by the cost model
 };
 
 // Launches the product on `stream`.  bf16 x bf16 goes to the tcgen05 tensor-core kernel;

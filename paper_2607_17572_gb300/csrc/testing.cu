@@ -20,6 +20,7 @@ extern "C" int jagg_test_gemm(const jagg_gemm_desc* d, cudaStream_t stream) {
   g.split_k = d->split_k;
   g.c_trans = d->c_trans != 0;
   g.bias_m = d->bias_m != 0;
+  g.tile_n = d->tile_n;
   return d->force_simt ? gemm_simt(g, stream) : gemm(g, stream);
 }
 

@@ -1,0 +1,163 @@
+"""Parity at the workloads' full sizes (full width, depth and token count), where the
+float64 oracle is out of reach (minutes per sequence at Flux width):
+
+* the bf16 path against the same architecture assembled from PyTorch library routines
+  with autograd (tests/torch_backbone.py, pinned to the oracle at 1e-9 in float64), run in
+  float32 on the GPU (TF32 off) on the same bf16-representable weights and inputs;
+* additivity of the joint VJP over its rows: grad(rows a and b in one call) equals
+  grad(a) + grad(b) from separate forwards and VJPs -- the batching of every kernel;
+* the no-save forward equals the saving one.
+
+Weights are drawn on the device (Xavier-uniform per matrix, small biases, norm scales near
+1) from the library's own parameter table: no oracle is involved, so the host-side
+generator of `synth` (minutes for 2.5 B parameters) is not needed."""
+import math
+
+import pytest
+import torch
+
+import synth
+from torch_backbone import torch_backbone
+
+pytestmark = [pytest.mark.gpu, pytest.mark.slow]
+
+jg = pytest.importorskip("paper_2607_17572_gb300")
+
+
+def device_weights(cfg, seed):
+    """f32 weights with bf16-representable values, laid out by the parameter table."""
+    gen = torch.Generator(device="cuda").manual_seed(seed)
+    w = torch.zeros(jg.param_count(cfg), dtype=torch.float32, device="cuda")
+    for p in jg.param_table(cfg):
+        view = w[p.offset:p.offset + p.numel]
+        if p.name.endswith("q_norm") or p.name.endswith("k_norm"):
+            view.uniform_(0.9, 1.1, generator=gen)
+        elif p.cols == 1:
+            view.uniform_(-0.02, 0.02, generator=gen)
+        else:
+            a = math.sqrt(6.0 / (p.rows + p.cols))
+            view.uniform_(-a, a, generator=gen)
+    return w.bfloat16().float()
+
+
+def run(cfg, weights, z, t, txt, cot):
+    tdt = cfg.torch_dtype
+    model = jg.Model(cfg, weights.to(tdt).contiguous())
+    B = z.shape[0]
+    zt, xt = z.to(tdt).contiguous(), txt.to(tdt).contiguous()
+    v = torch.empty_like(zt)
+    ws = jg.alloc_bytes(model.workspace_bytes(B))
+    saved = jg.alloc_bytes(model.saved_bytes(B))
+    jg.dit_forward_save(model, zt, t, xt, v, saved=saved, ws=ws)
+    grad = torch.zeros(jg.param_count(cfg), dtype=torch.float32, device="cuda")
+    jg.dit_joint_vjp(model, saved, B, cot, grad, ws)
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    del saved, ws
+    return v.float(), grad
+
+
+def inputs(wl, B, seed):
+    gen = torch.Generator(device="cuda").manual_seed(seed)
+    z = torch.randn(B, wl.in_channels, wl.latent_h, wl.latent_w, device="cuda", generator=gen).bfloat16().float()
+    t = torch.rand(B, device="cuda", generator=gen) * 0.9 + 0.05
+    txt = torch.randn(B, wl.txt_len, wl.txt_dim, device="cuda", generator=gen).bfloat16().float()
+    cot = torch.randn(B, wl.in_channels, wl.latent_h, wl.latent_w, device="cuda", generator=gen)
+    return z, t, txt, cot
+
+
+def _sums(a, b, chunk=1 << 26):
+    """sum (a-b)^2, sum b^2, sum a b, sum a^2 in float64, in chunks (2.5 B elements)."""
+    a, b = a.reshape(-1), b.reshape(-1)
+    out = torch.zeros(4, dtype=torch.float64, device=a.device)
+    for i in range(0, a.numel(), chunk):
+        x, y = a[i:i + chunk].double(), b[i:i + chunk].double()
+        out += torch.stack([((x - y) ** 2).sum(), (y * y).sum(), (x * y).sum(), (x * x).sum()])
+    return out.tolist()
+
+
+def rel(a, b):
+    d2, b2, _, _ = _sums(a, b)
+    return math.sqrt(d2 / b2)
+
+
+def cos(a, b):
+    _, b2, ab, a2 = _sums(a, b)
+    return ab / math.sqrt(a2 * b2)
+
+
+FULL = [("mmdit_flux512_bf16", 2), ("mmdit_flux1024_bf16", 1), ("mmdit_qwen_sweep_bf16", 2), ("dit_b_bf16", 8)]
+
+
+def torch_reference(wl, cfg, w, z, t, txt, cot):
+    """v and the flat parameter gradient of the PyTorch float32 assembly."""
+    P = {}
+    for p in jg.param_table(cfg):
+        x = w[p.offset:p.offset + p.numel]
+        P[p.name] = (x.view(p.rows, p.cols) if p.cols > 1 else x.view(p.rows)).clone().requires_grad_()
+    prev = torch.backends.cuda.matmul.allow_tf32
+    torch.backends.cuda.matmul.allow_tf32 = False
+    try:
+        v = torch_backbone(wl, P, z, t, txt)
+        (v * cot).sum().backward()
+    finally:
+        torch.backends.cuda.matmul.allow_tf32 = prev
+    grad = torch.zeros_like(w)
+    for p in jg.param_table(cfg):
+        grad[p.offset:p.offset + p.numel] = P[p.name].grad.reshape(-1)
+    return v.detach(), grad
+
+
+@pytest.mark.parametrize("name,B", FULL, ids=[f[0] for f in FULL])
+def test_full_size_bf16_path_matches_torch_fp32(name, B):
+    wl = synth.WORKLOADS[name]
+    cfg = jg.Config.from_workload(wl)
+    w = device_weights(cfg, 42)
+    z, t, txt, cot = inputs(wl, B, 7)
+    v16, g16 = run(cfg, w, z, t, txt, cot)
+    torch.cuda.empty_cache()
+    v32, g32 = torch_reference(wl, cfg, w, z, t, txt, cot)
+    assert torch.isfinite(g16).all()
+    fv, fg, cg = rel(v16, v32), rel(g16, g32), cos(g16, g32)
+    per = {}
+    for p in jg.param_table(cfg):
+        a, b = g16[p.offset:p.offset + p.numel], g32[p.offset:p.offset + p.numel]
+        if _sums(a, b)[1] > 0:
+            per[p.name] = rel(a, b)
+    worst = max(per, key=per.get)
+    print(f"{name} B={B}: forward {fv:.2e}, grad rel L2 {fg:.2e}, cos {cg:.6f}, worst {worst} {per[worst]:.2e}")
+    assert fv <= 2e-2
+    assert fg <= 1e-2, f"gradient rel L2 {fg:.3e} (worst {worst}: {per[worst]:.3e})"
+    assert cg >= 0.999
+
+
+@pytest.mark.parametrize("name", ["mmdit_flux512_bf16", "mmdit_qwen_sweep_bf16"])
+def test_full_size_joint_vjp_is_additive_over_rows(name):
+    wl = synth.WORKLOADS[name]
+    cfg = jg.Config.from_workload(wl)
+    w = device_weights(cfg, 43)
+    z, t, txt, cot = inputs(wl, 2, 8)
+    v_joint, g_joint = run(cfg, w, z, t, txt, cot)
+    v0, g0 = run(cfg, w, z[:1], t[:1], txt[:1], cot[:1])
+    v1, g1 = run(cfg, w, z[1:], t[1:], txt[1:], cot[1:])
+    rv, rg = rel(v_joint, torch.cat([v0, v1])), rel(g_joint, g0 + g1)
+    print(f"{name}: joint vs single-row calls: forward rel L2 {rv:.2e}, gradient rel L2 {rg:.2e}")
+    # The tile width of each product is chosen from its row count, so a 1-row and a 2-row
+    # call may round their bf16 activations differently (a few 1e-3 relative); a batching
+    # error (a wrong row offset or sequence index) is of order 1.
+    assert rv <= 5e-3 and rg <= 5e-3
+
+
+def test_full_size_forward_without_saves_matches_saved_forward():
+    wl = synth.WORKLOADS["mmdit_flux512_bf16"]
+    cfg = jg.Config.from_workload(wl)
+    model = jg.Model(cfg, device_weights(cfg, 44).bfloat16().contiguous())
+    z, t, txt, _ = inputs(wl, 2, 9)
+    zt, xt = z.bfloat16().contiguous(), txt.bfloat16().contiguous()
+    ws = jg.alloc_bytes(model.workspace_bytes(2))
+    saved = jg.alloc_bytes(model.saved_bytes(2))
+    v1, v2 = torch.empty_like(zt), torch.empty_like(zt)
+    jg.dit_forward_save(model, zt, t, xt, v1, saved=saved, ws=ws)
+    jg.dit_forward_save(model, zt, t, xt, v2, ws=ws)
+    torch.cuda.synchronize()
+    assert torch.equal(v1, v2)

@@ -33,6 +33,37 @@ def _desc(M, N, K, A, lda, a_mn, B, ldb, b_mn, dt, C, ldc, c_dt, epi=0, **kw):
 SHAPES = [(256, 128, 128), (300, 200, 192), (128, 64, 64), (1000, 768, 768), (5328, 2304, 768), (777, 320, 1000)]
 
 
+@pytest.mark.parametrize("tile_n", [0, 64, 128, 256])
+@pytest.mark.parametrize("a_mn,b_mn", [(False, False), (False, True), (True, True), (True, False)])
+@pytest.mark.parametrize("M,N,K", [(300, 600, 192), (1000, 768, 520)])
+def test_tcgen05_tile_widths(M, N, K, a_mn, b_mn, tile_n):
+    """Every tile width on every operand layout, with a ragged last column tile, for a
+    plain store, a biased bf16 store and a split-K accumulation."""
+    torch.manual_seed(M + N + K + tile_n)
+    dev = "cuda"
+    A = torch.randn(M, K, device=dev).bfloat16()
+    B = (torch.randn(N, K, device=dev) / math.sqrt(K)).bfloat16()
+    As = A.t().contiguous() if a_mn else A
+    Bs = B.t().contiguous() if b_mn else B
+    lda, ldb = (M if a_mn else K), (N if b_mn else K)
+    ref = A.float() @ B.float().t()
+    C = torch.full((M, N), float("nan"), device=dev)
+    jg.test_gemm(_desc(M, N, K, As, lda, a_mn, Bs, ldb, b_mn, jg.DTYPE_BF16, C, N, jg.DTYPE_F32, tile_n=tile_n))
+    bias = torch.randn(N, device=dev).bfloat16()
+    Cb = torch.empty(M, N, device=dev, dtype=torch.bfloat16)
+    jg.test_gemm(_desc(M, N, K, As, lda, a_mn, Bs, ldb, b_mn, jg.DTYPE_BF16, Cb, N, jg.DTYPE_BF16, bias=bias,
+                       tile_n=tile_n))
+    G0 = torch.randn(M, N, device=dev)
+    G = G0.clone()
+    jg.test_gemm(_desc(M, N, K, As, lda, a_mn, Bs, ldb, b_mn, jg.DTYPE_BF16, G, N, jg.DTYPE_F32, epi=4, split_k=3,
+                       tile_n=tile_n))
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    assert _rel(C, ref) < 1e-5
+    assert _rel(Cb.float(), ref + bias.float()) < 5e-3
+    assert _rel(G, G0 + ref) < 1e-5
+
+
 @pytest.mark.parametrize("a_mn,b_mn", [(False, False), (False, True), (True, True), (True, False)])
 @pytest.mark.parametrize("M,N,K", SHAPES)
 def test_tcgen05_gemm_layouts(M, N, K, a_mn, b_mn):
