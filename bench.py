@@ -52,6 +52,9 @@ def parse():
     p.add_argument("--quick", action="store_true", help="skip the full-W, e2e and CPU legs")
     p.add_argument("--G", type=int, default=0,
                    help="override the workload's group size (small cases for profiler captures)")
+    p.add_argument("--kernel", choices=["attention_bwd"], default=None,
+                   help="time one kernel family alone on the workload's shapes instead of the step")
+    p.add_argument("--rows", type=int, default=0, help="sequences per call for --kernel (default 2G)")
     p.add_argument("--vjp-rows", choices=["auto", "group", "window"], default="auto",
                    help="one joint VJP per group (all windows' rows) or per window; auto picks the group "
                         "when its saved activations fit in half of the free device memory")
@@ -632,10 +635,70 @@ def run_e2e(b, args, ws, routes):
             "includes": "Phase 1 forwards (2G rows saved + (W-2)G rows unsaved per window), signals, one joint VJP"}
 
 
+def run_kernel_attention_bwd(args):
+    """The attention backward alone on the workload's joint attention (B sequences, the
+    text and image streams in their own buffers as in the MMDiT double blocks), timed with
+    CUDA events over the timed calls; the kernel's own device time comes from the
+    library's per-launch events."""
+    import paper_2607_17572_gb300 as jg
+    wl = workload(args)
+    dev = torch.device("cuda", torch.cuda.current_device())
+    B = args.rows or 2 * wl.G
+    N, H, dh = wl.n_tok, wl.heads, wl.head_dim
+    n0 = wl.txt_len if wl.arch == "mmdit" else N
+    d = H * dh
+    gen = torch.Generator(device=dev).manual_seed(synth.NOISE_SEED)
+    qkv = (torch.randn(B * N, 3 * d, device=dev, generator=gen) * 1.5).bfloat16()
+    o = torch.empty(B * N, d, device=dev, dtype=torch.bfloat16)
+    lse = torch.empty(B, H, N, device=dev)
+    jg.test_attention_fwd(qkv, B, N, H, dh, o, lse)
+    dO = torch.randn(B * N, d, device=dev, generator=gen).bfloat16()
+
+    def split(x):
+        x = x.view(B, N, -1)
+        return x[:, :n0].contiguous(), x[:, n0:].contiguous()
+    views = (split(qkv), split(o), split(dO))
+    dq = (torch.empty(B, n0, 3 * d, device=dev, dtype=torch.bfloat16),
+          torch.empty(B, N - n0, 3 * d, device=dev, dtype=torch.bfloat16))
+    call = lambda: jg.test_attention_bwd_streams(views[0], views[1], lse, views[2], B, N, n0, H, dh, dq)
+    for _ in range(args.warmup):
+        call()
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.profiler.start()
+    e0.record(stream)
+    for _ in range(args.steps):
+        call()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    torch.cuda.profiler.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+    jg.profile_enable(True)
+    for _ in range(args.steps):
+        call()
+    prof = jg.profile_read()
+    jg.profile_enable(False)
+    fam = prof["attention_bwd"]
+    flops = 8.0 * B * H * N * N * dh
+    kms = fam["ms"] / max(fam["launches"], 1)
+    burst, sustained, hbm, src = peaks()
+    tf = flops / (kms / 1000.0) / 1e12
+    print(json.dumps({"kernel": "attention_bwd", "workload": describe(wl), "rows": B, "heads": H, "head_dim": dh,
+                      "tokens": N, "text_tokens": n0 if n0 < N else 0, "steps": args.steps,
+                      "ms_per_call": ms, "kernel_ms": kms, "algorithmic_tflop": flops / 1e12,
+                      "roofline": {"bound": "tensor", "achieved": tf, "peak": burst, "unit": "TFLOP/s",
+                                   "frac": tf / burst, "peak_source": f"bf16_tflops (burst) of {src} peaks"},
+                      "aux_ms_per_call": prof["attention_bwd_aux"]["ms"] / args.steps}), flush=True)
+
+
 def main():
     args = parse()
     ws, rank = dist_setup()
-    if args.impl == "reference":
+    if args.kernel == "attention_bwd":
+        if rank == 0:
+            run_kernel_attention_bwd(args)
+    elif args.impl == "reference":
         run_reference(args, ws, rank)
     else:
         run_gpu(args, ws, rank)

@@ -67,6 +67,15 @@ int jagg_test_attention_fwd(const void* qkv, int B, int N, int heads, int dh, in
 int64_t jagg_test_attention_scratch_bytes(int B, int N, int heads, int dh);
 int jagg_test_attention_bwd(const void* qkv, const void* o, const float* lse, const void* dO, int B, int N,
                             int heads, int dh, int dtype, void* dqkv, void* scratch, cudaStream_t stream);
+/* The backward over two-stream views, as the MMDiT double blocks use it: the first n0
+ * tokens of every sequence live in qkv0 / o0 / dO0 / dqkv0 ([B*n0, 3d], [B*n0, d], ...),
+ * the remaining N - n0 in qkv1 / o1 / dO1 / dqkv1 (n0 = N: one buffer, the *1 pointers
+ * ignored).  impl: 0 the library's choice, 1 the warp-level MMA kernel, 2 the tcgen05
+ * kernel (JAGG_ERR_ARG when it does not serve the call). */
+int jagg_test_attention_bwd_streams(const void* qkv0, const void* qkv1, const void* o0, const void* o1,
+                                    const float* lse, const void* dO0, const void* dO1, int B, int N, int n0,
+                                    int heads, int dh, int dtype, void* dqkv0, void* dqkv1, void* scratch, int impl,
+                                    cudaStream_t stream);
 
 #ifdef __cplusplus
 }

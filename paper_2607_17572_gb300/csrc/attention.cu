@@ -637,7 +637,15 @@ int attention_bwd(const AttnBwdArgs& a, cudaStream_t s) {
   JAGG_LAUNCHED();
   prof_stop(tok, s, PROF_ATTN_AUX, 0.0, 4.0 * f.B * f.N * f.heads * f.dh * 1.5);
   int st = JAGG_ERR_UNSUPPORTED;
-  if (f.dtype == JAGG_DTYPE_BF16 && f.dh == 64)
+  JAGG_CHECK_ARG(a.impl >= 0 && a.impl <= 2, "attention: bad implementation %d", a.impl);
+  const bool tc = attention_bwd_tc_eligible(a);
+  JAGG_CHECK_ARG(a.impl != 2 || tc, "attention: the tcgen05 backward does not serve this call");
+  if (tc && a.impl != 1) {
+    tok = prof_start(s);
+    st = attention_bwd_tc(a, s);
+    prof_stop(tok, s, PROF_ATTN_BWD, 8.0 * f.B * f.heads * (double)f.N * f.N * f.dh,
+              2.0 * f.B * (double)f.N * f.heads * f.dh * 7);
+  } else if (f.dtype == JAGG_DTYPE_BF16 && f.dh == 64)
     st = bwd_tc<64>(a, s);
   else if (f.dtype == JAGG_DTYPE_BF16 && f.dh == 128)
     st = bwd_tc<128>(a, s);

@@ -39,9 +39,14 @@ struct AttnBwdArgs {
   float* dq_acc;  // f32 [B*N, heads*dh] scratch, zeroed by the launcher
   SegRows dq, dk, dv;  // outputs (dtype), columns dq_col0 + h * dh etc.
   int64_t dq_col0, dk_col0, dv_col0;
+  int impl = 0;  // 0: the library's choice; 1: warp-level MMA kernel; 2: tcgen05 kernel
 };
 
 int attention_fwd(const AttnArgs& a, cudaStream_t s);
+// The tcgen05 backward (attention_tc.cu): bf16, head dim 64 / 128, stream boundary on a
+// multiple of 128 tokens, 16-byte aligned views.
+bool attention_bwd_tc_eligible(const AttnBwdArgs& a);
+int attention_bwd_tc(const AttnBwdArgs& a, cudaStream_t s);
 // Scratch: Dv and dq_acc as described above.  dq_acc must be 16-byte aligned (it receives
 // 16-byte vector reductions); attention_bwd_scratch places both in one buffer of
 // attention_bwd_scratch_floats floats with dq_acc at a 256-byte boundary.

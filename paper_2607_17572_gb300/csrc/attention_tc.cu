@@ -1,0 +1,535 @@
+// Attention backward on the fifth-generation tensor cores (tcgen05, TMEM accumulators,
+// TMA-fed shared-memory operands), bf16, head dim 64 or 128 (appendix, Eqs. bwd_V ..
+// bwd_QK, with the softmax recomputed from the saved log-sum-exp).
+//
+// One CTA per (128-key tile, sequence, head) streams the sequence's query tiles:
+//   S^T = K Q^T, dP^T = V dO^T                      (128 x BQ, TMEM)
+//   P^T = exp(scale S^T - lse), dS^T = P^T (dP^T - rowsum(dO O))   (8 warps, -> bf16 smem)
+//   dV += P^T dO, dK += dS^T Q                      (128 x dh, TMEM, whole sequence)
+//   dQ  = dS K (head dim 64, BQ = 128) or dQ^T = K^T dS^T (head dim 128, BQ = 64)
+//        -> 4 warps -> TMA f32 reduce-add into the dQ accumulator.
+// Every product has M = 128.  Each shared tile serves as a K-major and an MN-major
+// operand through two descriptors of the same 128-byte-swizzled layout, so nothing is
+// transposed.  Warp roles: 0 TMA producer, 1 MMA issuer (one elected thread), 2-9 P / dS
+// (two warps per TMEM lane quarter, half the query columns each) and the final dK / dV,
+// 10-13 dQ.
+// Head dim 128: S^T, dP^T are double-buffered in TMEM and dQ^T of a tile is written over
+// its own (consumed) S^T columns, so S^T, dP^T of tile j + 1 are ready while P, dS of
+// tile j are formed (512 columns: 2 x (64 + 64) + 128 + 128).  Head dim 64: one S^T, dP^T
+// buffer (128 + 128 + 64 + 64 + 64 columns); the MMA warp issues S, dP of tile j + 1 before
+// dV, dK, dQ of tile j.
+// Ragged ends: 3D tensor maps [sequence][token][column] per stream buffer make TMA read
+// zeros past the last token and drop dQ rows past it.
+#include <cuda.h>
+
+#include "attention.cuh"
+#include "ptx.cuh"
+#include "tmap.cuh"
+
+namespace jagg {
+namespace {
+
+constexpr float kLog2eTc = 1.4426950408889634f;
+constexpr int FB_THREADS = 448;  // 14 warps
+
+template <int D>
+struct FbCfg {
+  static constexpr int BK = 128;                 // keys per CTA
+  static constexpr int BQ = D == 64 ? 128 : 64;  // queries per step
+  static constexpr bool DQT = D == 128;          // dQ^T = K^T dS^T (M = D)
+  static constexpr int NSB = DQT ? 2 : 1;        // S^T / dP^T TMEM buffers
+  static constexpr int CW = BQ / 2;              // query columns per P / dS warp
+  static constexpr int KV_BYTES = BK * D * 2;
+  static constexpr int QT_BYTES = BQ * D * 2;
+  static constexpr int PS_BYTES = BK * BQ * 2;
+  static constexpr int STAGES = 3;
+  static constexpr int DQ_WARP_BYTES = 32 * 32 * 4;  // one 32 x 32 f32 box, used twice per tile
+  static constexpr int OFF_K = 0;
+  static constexpr int OFF_V = OFF_K + KV_BYTES;
+  static constexpr int OFF_Q = OFF_V + KV_BYTES;
+  static constexpr int OFF_DO = OFF_Q + STAGES * QT_BYTES;
+  static constexpr int OFF_P = OFF_DO + STAGES * QT_BYTES;
+  static constexpr int OFF_DS = OFF_P + PS_BYTES;
+  static constexpr int OFF_DQ = OFF_DS + PS_BYTES;
+  static constexpr int OFF_LSE = OFF_DQ + 4 * DQ_WARP_BYTES;
+  static constexpr int OFF_RD = OFF_LSE + STAGES * BQ * 4;
+  static constexpr int OFF_BAR = OFF_RD + STAGES * BQ * 4;
+  static constexpr int SMEM = OFF_BAR + 256 + 1024;
+  // TMEM columns
+  static constexpr int T_DV = DQT ? 256 : 256, T_DK = DQT ? 384 : 320;
+  __host__ __device__ static constexpr int t_s(int b) { return DQT ? b * 64 : 0; }
+  __host__ __device__ static constexpr int t_dp(int b) { return DQT ? 128 + b * 64 : 128; }
+  __host__ __device__ static constexpr int t_dq(int b) { return DQT ? b * 64 : 384; }
+  static_assert(SMEM <= 232448, "shared memory budget");
+};
+
+// Tensor maps of one backward call: per stream buffer (0: the first n0 tokens of every
+// sequence, 1: the rest) the query, key, value and output-gradient views, and the dQ
+// accumulator.
+struct FbMaps {
+  CUtensorMap q[2], k[2], v[2], dO[2], dq;
+};
+
+struct FbParams {
+  int B, N, heads, n0;
+  float scale;
+  int64_t q_col0, k_col0, v_col0, dk_col0, dv_col0;
+  const float* lse;
+  const float* Dv;
+  SegRows dk, dv;
+};
+
+// Shared-memory descriptor of a 128-byte-swizzled operand; k-step `k` (16 elements of K).
+// K-major: `rows` rows of 128 B per 64-element K chunk, chunks rows * 128 B apart.
+// MN-major: the K dimension runs down the rows (8-row atoms 1024 B apart), 64-element MN
+// chunks `chunk_bytes` apart.
+__device__ __forceinline__ uint64_t kmajor_desc(uint32_t base, int rows, int k) {
+  return ptx::sdesc_sw128(base + (k >> 2) * (rows * 128) + (k & 3) * 32, 16, 1024);
+}
+__device__ __forceinline__ uint64_t mnmajor_desc(uint32_t base, int chunk_bytes, int k) {
+  return ptx::sdesc_sw128(base + k * 2048, chunk_bytes, 1024);
+}
+
+__device__ __forceinline__ uint32_t pack2_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// Writes columns c0 .. c0 + 31 of row r (16 packed bf16 pairs) into a K-major
+// 128-byte-swizzled tile of 64-column chunks, `rows` rows per chunk.
+__device__ __forceinline__ void st_row32_packed(uint8_t* tile, int rows, int r, int c0, const uint32_t* h) {
+  uint8_t* row = tile + (c0 >> 6) * (rows * 128) + r * 128;
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const int j16 = ((c0 & 63) >> 3) + u;
+    *reinterpret_cast<uint4*>(row + ((j16 ^ (r & 7)) << 4)) =
+        make_uint4(h[4 * u], h[4 * u + 1], h[4 * u + 2], h[4 * u + 3]);
+  }
+}
+
+// P^T, dS^T of 32 query columns of one key row from S^T, dP^T (f32 bit patterns).
+__device__ __forceinline__ void softmax32(const uint32_t* rs, const uint32_t* rp, const float* lse, const float* rd,
+                                          float scale, uint32_t* hp, uint32_t* hd) {
+#pragma unroll
+  for (int i = 0; i < 32; i += 4) {
+    const float4 l4 = *reinterpret_cast<const float4*>(lse + i);
+    const float4 r4 = *reinterpret_cast<const float4*>(rd + i);
+    const float p0 = ptx::ex2_approx((__uint_as_float(rs[i]) * scale - l4.x) * kLog2eTc);
+    const float p1 = ptx::ex2_approx((__uint_as_float(rs[i + 1]) * scale - l4.y) * kLog2eTc);
+    const float p2 = ptx::ex2_approx((__uint_as_float(rs[i + 2]) * scale - l4.z) * kLog2eTc);
+    const float p3 = ptx::ex2_approx((__uint_as_float(rs[i + 3]) * scale - l4.w) * kLog2eTc);
+    hp[i / 2] = pack2_bf16(p0, p1);
+    hp[i / 2 + 1] = pack2_bf16(p2, p3);
+    hd[i / 2] = pack2_bf16(p0 * (__uint_as_float(rp[i]) - r4.x), p1 * (__uint_as_float(rp[i + 1]) - r4.y));
+    hd[i / 2 + 1] = pack2_bf16(p2 * (__uint_as_float(rp[i + 2]) - r4.z), p3 * (__uint_as_float(rp[i + 3]) - r4.w));
+  }
+}
+
+template <int D>
+__global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_constant__ FbMaps maps, FbParams p) {
+  using C = FbCfg<D>;
+  constexpr int BK = C::BK, BQ = C::BQ, NS = C::STAGES, NSB = C::NSB, CW = C::CW;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sK = sm + C::OFF_K;
+  uint8_t* sV = sm + C::OFF_V;
+  uint8_t* sQ = sm + C::OFF_Q;
+  uint8_t* sdO = sm + C::OFF_DO;
+  uint8_t* sP = sm + C::OFF_P;
+  uint8_t* sdS = sm + C::OFF_DS;
+  uint8_t* sDQ = sm + C::OFF_DQ;
+  float* sLse = reinterpret_cast<float*>(sm + C::OFF_LSE);
+  float* sRd = reinterpret_cast<float*>(sm + C::OFF_RD);
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sm + C::OFF_BAR);
+  uint64_t* full = bar;                     // [NS] Q, dO, lse, rowsum of a stage landed
+  uint64_t* empty = full + NS;              // [NS] the stage's products are done
+  uint64_t* bar_s = empty + NS;             // [NSB] S^T, dP^T of a tile are in TMEM buffer b
+  uint64_t* bar_dq = bar_s + NSB;           // [NSB] dQ of a tile is in TMEM buffer b
+  uint64_t* bar_dqfree = bar_dq + NSB;      // [NSB] the dQ warps have read it
+  uint64_t* bar_kv = bar_dqfree + NSB;      // K, V landed
+  uint64_t* bar_p = bar_kv + 1;             // P^T, dS^T written (S^T, dP^T read) by the 8 warps
+  uint64_t* bar_pfree = bar_kv + 2;         // the products reading P^T, dS^T are done
+  uint64_t* bar_fin = bar_kv + 3;           // every product is done (dK, dV final)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_kv + 4);
+  __shared__ volatile int abort_flag;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int kt = blockIdx.x, bh = blockIdx.y;
+  const int b = bh / p.heads, h = bh % p.heads;
+  const int N = p.N;
+  const int k0 = kt * BK;
+  const int nq = (N + BQ - 1) / BQ;
+
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    for (int i = 0; i < NS; ++i) {
+      ptx::mbar_init(&full[i], 1 + 32);  // the TMA's expect-tx arrival + one per producer lane's copies
+      ptx::mbar_init(&empty[i], 1);
+    }
+    for (int i = 0; i < NSB; ++i) {
+      ptx::mbar_init(&bar_s[i], 1);
+      ptx::mbar_init(&bar_dq[i], 1);
+      ptx::mbar_init(&bar_dqfree[i], 4);
+    }
+    ptx::mbar_init(bar_kv, 1);
+    ptx::mbar_init(bar_p, 8);
+    ptx::mbar_init(bar_pfree, 1);
+    ptx::mbar_init(bar_fin, 1);
+    ptx::fence_mbar_init();
+    for (int sg = 0; sg < 2; ++sg) {
+      ptx::prefetch_tmap(&maps.q[sg]);
+      ptx::prefetch_tmap(&maps.k[sg]);
+      ptx::prefetch_tmap(&maps.v[sg]);
+      ptx::prefetch_tmap(&maps.dO[sg]);
+    }
+    ptx::prefetch_tmap(&maps.dq);
+  }
+  if (warp == 1) {
+    ptx::tmem_alloc(tmem_slot, 512);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  // row coordinates inside a stream buffer
+  auto seg_of = [&](int r) { return r < p.n0 ? 0 : 1; };
+  auto row_in = [&](int r) { return r < p.n0 ? r : r - p.n0; };
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      const int s = seg_of(k0), r = row_in(k0);
+      ptx::mbar_arrive_expect_tx(bar_kv, 2 * C::KV_BYTES);
+#pragma unroll
+      for (int c = 0; c < D / 64; ++c) {
+        ptx::tma_load_3d(sK + c * BK * 128, &maps.k[s], bar_kv, (int)(p.k_col0 + h * D + c * 64), r, b);
+        ptx::tma_load_3d(sV + c * BK * 128, &maps.v[s], bar_kv, (int)(p.v_col0 + h * D + c * 64), r, b);
+      }
+    }
+    for (int j = 0; j < nq; ++j) {
+      const int st = j % NS;
+      bool ok = true;
+      if (lane == 0) ok = ptx::mbar_wait(&empty[st], ((j / NS) & 1) ^ 1);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      if (!ok || abort_flag) { abort_flag = 1; break; }
+      const int q0 = j * BQ;
+      // lse and rowsum(dO O) of the tile's queries: asynchronous 4-byte copies (their
+      // addresses need not be 16-byte aligned) whose completion the stage barrier tracks;
+      // +inf / 0 past the last query
+      for (int i = lane; i < BQ; i += 32) {
+        const int q = q0 + i;
+        if (q < N) {
+          ptx::cp_async4(sLse + st * BQ + i, p.lse + (int64_t)bh * N + q);
+          ptx::cp_async4(sRd + st * BQ + i, p.Dv + (int64_t)bh * N + q);
+        } else {
+          sLse[st * BQ + i] = INFINITY;
+          sRd[st * BQ + i] = 0.f;
+        }
+      }
+      ptx::cp_async_arrive_noinc(&full[st]);
+      __syncwarp();
+      if (lane == 0) {
+        const int s = seg_of(q0), r = row_in(q0);
+        ptx::mbar_arrive_expect_tx(&full[st], 2 * C::QT_BYTES);
+#pragma unroll
+        for (int c = 0; c < D / 64; ++c) {
+          ptx::tma_load_3d(sQ + st * C::QT_BYTES + c * BQ * 128, &maps.q[s], &full[st],
+                           (int)(p.q_col0 + h * D + c * 64), r, b);
+          ptx::tma_load_3d(sdO + st * C::QT_BYTES + c * BQ * 128, &maps.dO[s], &full[st], h * D + c * 64, r, b);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (ptx::elect_one()) {
+      constexpr uint32_t id_s = ptx::idesc_bf16(128, BQ, false, false);
+      constexpr uint32_t id_acc = ptx::idesc_bf16(128, D, false, true);
+      constexpr uint32_t id_dq = ptx::idesc_bf16(128, 64, true, true);
+      const uint32_t aK = ptx::smem_u32(sK), aV = ptx::smem_u32(sV);
+      const uint32_t aP = ptx::smem_u32(sP), adS = ptx::smem_u32(sdS);
+      // S^T, dP^T of tile j into TMEM buffer j % NSB
+      auto issue_s = [&](int j) {
+        const int st = j % NS, bb = j % NSB;
+        const uint32_t aQ = ptx::smem_u32(sQ + st * C::QT_BYTES), adO = ptx::smem_u32(sdO + st * C::QT_BYTES);
+#pragma unroll
+        for (int k = 0; k < D / 16; ++k) {
+          ptx::umma_bf16(tmem + C::t_s(bb), kmajor_desc(aK, BK, k), kmajor_desc(aQ, BQ, k), id_s, k > 0);
+          ptx::umma_bf16(tmem + C::t_dp(bb), kmajor_desc(aV, BK, k), kmajor_desc(adO, BQ, k), id_s, k > 0);
+        }
+        ptx::umma_commit(&bar_s[bb]);
+      };
+      bool ok = ptx::mbar_wait(bar_kv, 0);
+      for (int j = 0; j < NSB && j < nq && ok; ++j) {
+        ok = ptx::mbar_wait(&full[j % NS], (j / NS) & 1);
+        if (ok) {
+          ptx::tc_fence_after();
+          issue_s(j);
+        }
+      }
+      for (int j = 0; j < nq && ok; ++j) {
+        const int st = j % NS, bb = j % NSB;
+        if (!ptx::mbar_wait(bar_p, j & 1)) { ok = false; break; }
+        ptx::tc_fence_after();
+        if constexpr (NSB == 1) {
+          // the single S^T / dP^T buffer is consumed: the next tile's products first
+          if (j + 1 < nq) {
+            if (!ptx::mbar_wait(&full[(j + 1) % NS], ((j + 1) / NS) & 1)) { ok = false; break; }
+            ptx::tc_fence_after();
+            issue_s(j + 1);
+          }
+        }
+        const uint32_t aQ = ptx::smem_u32(sQ + st * C::QT_BYTES), adO = ptx::smem_u32(sdO + st * C::QT_BYTES);
+#pragma unroll
+        for (int k = 0; k < BQ / 16; ++k) {
+          const uint32_t acc = (j > 0 || k > 0) ? 1u : 0u;
+          ptx::umma_bf16(tmem + C::T_DV, kmajor_desc(aP, BK, k), mnmajor_desc(adO, BQ * 128, k), id_acc, acc);
+          ptx::umma_bf16(tmem + C::T_DK, kmajor_desc(adS, BK, k), mnmajor_desc(aQ, BQ * 128, k), id_acc, acc);
+        }
+        if constexpr (NSB == 1) {
+          if (j > 0) {  // the dQ warps have read the previous tile's dQ
+            if (!ptx::mbar_wait(&bar_dqfree[0], (j - 1) & 1)) { ok = false; break; }
+            ptx::tc_fence_after();
+          }
+        }
+#pragma unroll
+        for (int k = 0; k < BK / 16; ++k) {
+          if constexpr (C::DQT)  // dQ^T[d][q] = sum_key K[key][d] dS^T[key][q], over this tile's S^T
+            ptx::umma_bf16(tmem + C::t_dq(bb), mnmajor_desc(aK, BK * 128, k), mnmajor_desc(adS, BK * 128, k),
+                           id_dq, k > 0);
+          else  // dQ[q][d] = sum_key dS^T[key][q] K[key][d]
+            ptx::umma_bf16(tmem + C::t_dq(bb), mnmajor_desc(adS, BK * 128, k), mnmajor_desc(aK, BK * 128, k),
+                           id_dq, k > 0);
+        }
+        ptx::umma_commit(&bar_dq[bb]);
+        ptx::umma_commit(&empty[st]);
+        ptx::umma_commit(bar_pfree);
+        if constexpr (NSB == 2) {
+          // S^T, dP^T of tile j + 2 go into this buffer once the dQ warps have read dQ^T
+          if (j + 2 < nq) {
+            if (!ptx::mbar_wait(&bar_dqfree[bb], (j >> 1) & 1)) { ok = false; break; }
+            if (!ptx::mbar_wait(&full[(j + 2) % NS], ((j + 2) / NS) & 1)) { ok = false; break; }
+            ptx::tc_fence_after();
+            issue_s(j + 2);
+          }
+        }
+      }
+      if (!ok) abort_flag = 1;
+      ptx::umma_commit(bar_fin);
+    }
+  } else if (warp < 10) {
+    // ---------------------------------------------------------------- P / dS, then dK, dV
+    const int quarter = warp & 3, half = (warp - 2) >> 2;
+    const int r = quarter * 32 + lane;  // key row of the tile = TMEM lane
+    const int c0 = half * CW;           // this warp's query columns
+    const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
+    bool ok = true;
+    for (int j = 0; j < nq; ++j) {
+      const int st = j % NS, bb = j % NSB;
+      ok = ptx::mbar_wait(&bar_s[bb], (j / NSB) & 1) && ptx::mbar_wait(&full[st], (j / NS) & 1);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok || abort_flag) { abort_flag = 1; break; }
+      ptx::tc_fence_after();
+      const float* lse = sLse + st * BQ + c0;
+      const float* rd = sRd + st * BQ + c0;
+      uint32_t hp[CW / 2], hd[CW / 2];
+#pragma unroll
+      for (int c = 0; c < CW / 32; ++c) {
+        uint32_t rs[32], rp[32];
+        ptx::tmem_ld_32x32b_x32(trow + C::t_s(bb) + c0 + c * 32, rs);
+        ptx::tmem_ld_32x32b_x32(trow + C::t_dp(bb) + c0 + c * 32, rp);
+        ptx::tmem_ld_wait();
+        softmax32(rs, rp, lse + c * 32, rd + c * 32, p.scale, hp + c * 16, hd + c * 16);
+      }
+      ptx::tc_fence_before();
+      if (j > 0) ok = ptx::mbar_wait(bar_pfree, (j - 1) & 1);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok || abort_flag) { abort_flag = 1; break; }
+#pragma unroll
+      for (int c = 0; c < CW / 32; ++c) {
+        st_row32_packed(sP, BK, r, c0 + c * 32, hp + c * 16);
+        st_row32_packed(sdS, BK, r, c0 + c * 32, hd + c * 16);
+      }
+      ptx::fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(bar_p);
+    }
+    ok = ok && ptx::mbar_wait(bar_fin, 0);
+    ok = __all_sync(0xffffffffu, ok);
+    if (ok) {
+      ptx::tc_fence_after();
+      const int key = k0 + r;
+#pragma unroll 1
+      for (int c = half * (D / 64); c < (half + 1) * (D / 64); ++c) {
+        uint32_t rv[32], rk[32];
+        ptx::tmem_ld_32x32b_x32(trow + C::T_DV + c * 32, rv);
+        ptx::tmem_ld_32x32b_x32(trow + C::T_DK + c * 32, rk);
+        ptx::tmem_ld_wait();
+        if (key < N) {
+          bf16* dv = static_cast<bf16*>(p.dv.base(key)) + p.dv.off(b, key, N, p.dv_col0 + h * D + c * 32);
+          bf16* dk = static_cast<bf16*>(p.dk.base(key)) + p.dk.off(b, key, N, p.dk_col0 + h * D + c * 32);
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            uint4 a, bb;
+            __nv_bfloat162* ha = reinterpret_cast<__nv_bfloat162*>(&a);
+            __nv_bfloat162* hb = reinterpret_cast<__nv_bfloat162*>(&bb);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              ha[i] = __floats2bfloat162_rn(__uint_as_float(rv[8 * u + 2 * i]), __uint_as_float(rv[8 * u + 2 * i + 1]));
+              hb[i] = __floats2bfloat162_rn(__uint_as_float(rk[8 * u + 2 * i]) * p.scale,
+                                            __uint_as_float(rk[8 * u + 2 * i + 1]) * p.scale);
+            }
+            *reinterpret_cast<uint4*>(dv + 8 * u) = a;
+            *reinterpret_cast<uint4*>(dk + 8 * u) = bb;
+          }
+        }
+      }
+    } else {
+      abort_flag = 1;
+    }
+  } else {
+    // ---------------------------------------------------------------- dQ -> f32 reduce-add
+    const int quarter = warp & 3;
+    const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
+    uint8_t* stg = sDQ + quarter * C::DQ_WARP_BYTES;
+    for (int j = 0; j < nq; ++j) {
+      const int bb = j % NSB;
+      bool ok = ptx::mbar_wait(&bar_dq[bb], (j / NSB) & 1);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok || abort_flag) { abort_flag = 1; break; }
+      ptx::tc_fence_after();
+      uint32_t rq[64];
+      ptx::tmem_ld_32x32b_x32(trow + C::t_dq(bb), *reinterpret_cast<uint32_t(*)[32]>(rq));
+      ptx::tmem_ld_32x32b_x32(trow + C::t_dq(bb) + 32, *reinterpret_cast<uint32_t(*)[32]>(rq + 32));
+      ptx::tmem_ld_wait();
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(&bar_dqfree[bb]);
+      const int q0 = j * BQ;
+      // two 32 x 32 boxes through one staging box: dQ^T (lane = head dim, columns = the
+      // tile's 64 queries: box rows = queries) or dQ (lane = query, columns = 64 head dims)
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        if (lane == 0) ptx::bulk_wait_read<0>();
+        __syncwarp();
+        if constexpr (C::DQT) {
+#pragma unroll
+          for (int q = 0; q < 32; ++q)
+            *reinterpret_cast<float*>(stg + q * 128 + (((lane >> 2) ^ (q & 7)) << 4) + (lane & 3) * 4) =
+                __uint_as_float(rq[hh * 32 + q]) * p.scale;
+        } else {
+          uint8_t* row = stg + lane * 128;
+#pragma unroll
+          for (int u = 0; u < 8; ++u)
+            *reinterpret_cast<float4*>(row + ((u ^ (lane & 7)) << 4)) =
+                make_float4(__uint_as_float(rq[hh * 32 + 4 * u]) * p.scale,
+                            __uint_as_float(rq[hh * 32 + 4 * u + 1]) * p.scale,
+                            __uint_as_float(rq[hh * 32 + 4 * u + 2]) * p.scale,
+                            __uint_as_float(rq[hh * 32 + 4 * u + 3]) * p.scale);
+        }
+        ptx::fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          const int col = C::DQT ? h * D + quarter * 32 : h * D + hh * 32;
+          const int row = C::DQT ? q0 + hh * 32 : q0 + quarter * 32;
+          if (row < N) {
+            ptx::tma_reduce_add_3d(&maps.dq, stg, col, row, b);
+            ptx::bulk_commit();
+          }
+        }
+      }
+    }
+    if (lane == 0) ptx::bulk_wait<0>();
+    __syncwarp();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, 512);
+  }
+}
+
+// 3D view [sequence][token][column] of a stream buffer (bf16), boxes of 64 columns x `rows`.
+int seg_map(CUtensorMap* m, const void* base, int64_t ld, int ntok, int B, int rows) {
+  const uint64_t dims[3] = {(uint64_t)ld, (uint64_t)ntok, (uint64_t)B};
+  const uint64_t strides[2] = {(uint64_t)ld * 2, (uint64_t)ld * 2 * ntok};
+  const uint32_t box[3] = {64, (uint32_t)rows, 1};
+  return encode_tmap(m, false, 3, base, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+template <int D>
+int launch(const AttnBwdArgs& a, cudaStream_t s) {
+  using C = FbCfg<D>;
+  const AttnArgs& f = a.f;
+  const int n0 = f.q.n0, N = f.N;
+  const int n1 = N - n0;
+  FbMaps maps;
+  for (int sg = 0; sg < 2; ++sg) {
+    const int nt = sg == 0 ? n0 : n1;
+    if (nt <= 0) {  // single stream: the second views are unused copies
+      maps.q[1] = maps.q[0];
+      maps.k[1] = maps.k[0];
+      maps.v[1] = maps.v[0];
+      maps.dO[1] = maps.dO[0];
+      break;
+    }
+    JAGG_TRY(seg_map(&maps.q[sg], sg ? f.q.p1 : f.q.p0, sg ? f.q.ld1 : f.q.ld0, nt, f.B, C::BQ));
+    JAGG_TRY(seg_map(&maps.k[sg], sg ? f.k.p1 : f.k.p0, sg ? f.k.ld1 : f.k.ld0, nt, f.B, C::BK));
+    JAGG_TRY(seg_map(&maps.v[sg], sg ? f.v.p1 : f.v.p0, sg ? f.v.ld1 : f.v.ld0, nt, f.B, C::BK));
+    JAGG_TRY(seg_map(&maps.dO[sg], sg ? a.dO.p1 : a.dO.p0, sg ? a.dO.ld1 : a.dO.ld0, nt, f.B, C::BQ));
+  }
+  {
+    const int64_t cols = (int64_t)f.heads * D;
+    const uint64_t dims[3] = {(uint64_t)cols, (uint64_t)N, (uint64_t)f.B};
+    const uint64_t strides[2] = {(uint64_t)cols * 4, (uint64_t)cols * 4 * N};
+    const uint32_t box[3] = {32, 32, 1};
+    JAGG_TRY(encode_tmap(&maps.dq, true, 3, a.dq_acc, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B));
+  }
+  FbParams p;
+  p.B = f.B; p.N = N; p.heads = f.heads; p.n0 = n0 > 0 && n0 < N ? n0 : N;
+  p.scale = f.scale;
+  p.q_col0 = f.q_col0; p.k_col0 = f.k_col0; p.v_col0 = f.v_col0;
+  p.dk_col0 = a.dk_col0; p.dv_col0 = a.dv_col0;
+  p.lse = f.lse; p.Dv = a.Dv;
+  p.dk = a.dk; p.dv = a.dv;
+  static bool attr = false;
+  if (!attr) {
+    JAGG_CUDA_TRY(cudaFuncSetAttribute(fa_bwd_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
+    attr = true;
+  }
+  dim3 grid(ceil_div(N, C::BK), f.B * f.heads);
+  fa_bwd_tc_kernel<D><<<grid, FB_THREADS, C::SMEM, s>>>(maps, p);
+  JAGG_LAUNCHED();
+  return JAGG_OK;
+}
+
+}  // namespace
+
+// Whether the tensor-core backward serves the call: bf16, head dim 64 / 128, the stream
+// boundary on a 128-token multiple, 16-byte aligned buffers with 16-byte row pitches.
+bool attention_bwd_tc_eligible(const AttnBwdArgs& a) {
+  const AttnArgs& f = a.f;
+  if (f.dtype != JAGG_DTYPE_BF16 || (f.dh != 64 && f.dh != 128)) return false;
+  const int n0 = f.q.n0;
+  const bool single = n0 >= f.N;
+  if (!single && (n0 <= 0 || n0 % 128)) return false;
+  const SegRows* views[4] = {&f.q, &f.k, &f.v, &a.dO};
+  for (const SegRows* v : views) {
+    if (v->n0 != n0) return false;
+    if (!aligned16(v->p0) || v->ld0 % 8) return false;
+    if (!single && (!aligned16(v->p1) || v->ld1 % 8)) return false;
+  }
+  if (f.q_col0 % 8 || f.k_col0 % 8 || f.v_col0 % 8) return false;
+  return aligned16(a.dq_acc) && (a.dk_col0 % 8 == 0) && (a.dv_col0 % 8 == 0) && a.dk.ld0 % 8 == 0 &&
+         a.dv.ld0 % 8 == 0 && (single || (a.dk.ld1 % 8 == 0 && a.dv.ld1 % 8 == 0));
+}
+
+int attention_bwd_tc(const AttnBwdArgs& a, cudaStream_t s) {
+  return a.f.dh == 64 ? launch<64>(a, s) : launch<128>(a, s);
+}
+
+}  // namespace jagg

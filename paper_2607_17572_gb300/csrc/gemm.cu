@@ -15,6 +15,7 @@
 
 #include "gemm.cuh"
 #include "ptx.cuh"
+#include "tmap.cuh"
 
 namespace jagg {
 
@@ -774,6 +775,32 @@ bool tc_eligible(const GemmArgs& g) {
 }
 
 }  // namespace
+
+int encode_tmap(CUtensorMap* m, bool f32, int rank, const void* base, const uint64_t* dims, const uint64_t* strides,
+                const uint32_t* box, CUtensorMapSwizzle swz) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) {
+    set_last_error("cuTensorMapEncodeTiled is not available from the driver");
+    return JAGG_ERR_CUDA;
+  }
+  cuuint64_t d[5], st[4];
+  cuuint32_t bx[5], estr[5];
+  for (int i = 0; i < rank; ++i) {
+    d[i] = dims[i];
+    bx[i] = box[i];
+    estr[i] = 1;
+    if (i + 1 < rank) st[i] = strides[i];
+  }
+  CUresult r = fn(m, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank,
+                  const_cast<void*>(base), d, st, bx, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    set_last_error("cuTensorMapEncodeTiled failed (%d): rank %d, dims %llu x %llu", (int)r, rank,
+                   (unsigned long long)dims[0], (unsigned long long)(rank > 1 ? dims[1] : 1));
+    return JAGG_ERR_CUDA;
+  }
+  return JAGG_OK;
+}
 
 int gemm_simt(const GemmArgs& g, cudaStream_t stream) {
   JAGG_TRY(validate(g));

@@ -59,3 +59,31 @@ extern "C" int jagg_test_attention_bwd(const void* qkv, const void* o, const flo
   ab.dq_col0 = 0; ab.dk_col0 = d; ab.dv_col0 = 2 * d;
   return attention_bwd(ab, stream);
 }
+
+extern "C" int jagg_test_attention_bwd_streams(const void* qkv0, const void* qkv1, const void* o0, const void* o1,
+                                               const float* lse, const void* dO0, const void* dO1, int B, int N,
+                                               int n0, int heads, int dh, int dtype, void* dqkv0, void* dqkv1,
+                                               void* scratch, int impl, cudaStream_t stream) {
+  JAGG_CHECK_ARG(qkv0 && o0 && lse && dO0 && dqkv0 && scratch, "jagg_test_attention_bwd_streams: null pointer");
+  JAGG_CHECK_ARG(n0 > 0 && n0 <= N, "jagg_test_attention_bwd_streams: n0 = %d", n0);
+  const bool two = n0 < N;
+  JAGG_CHECK_ARG(!two || (qkv1 && o1 && dO1 && dqkv1), "jagg_test_attention_bwd_streams: null second stream");
+  const int d = heads * dh;
+  auto view = [&](const void* p0, const void* p1, int64_t ld) {
+    return SegRows{const_cast<void*>(p0), const_cast<void*>(two ? p1 : p0), ld, ld, two ? n0 : N};
+  };
+  AttnBwdArgs ab;
+  AttnArgs& f = ab.f;
+  f.B = B; f.N = N; f.heads = heads; f.dh = dh; f.scale = 1.f / sqrtf((float)dh);
+  f.q = f.k = f.v = view(qkv0, qkv1, 3 * d);
+  f.q_col0 = 0; f.k_col0 = d; f.v_col0 = 2 * d;
+  f.o = view(o0, o1, d);
+  f.lse = const_cast<float*>(lse);
+  f.dtype = dtype;
+  ab.dO = view(dO0, dO1, d);
+  attention_bwd_scratch(static_cast<float*>(scratch), B, N, heads, &ab.Dv, &ab.dq_acc);
+  ab.dq = ab.dk = ab.dv = view(dqkv0, dqkv1, 3 * d);
+  ab.dq_col0 = 0; ab.dk_col0 = d; ab.dv_col0 = 2 * d;
+  ab.impl = impl;
+  return attention_bwd(ab, stream);
+}

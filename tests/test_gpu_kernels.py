@@ -258,3 +258,48 @@ def test_attention_forward_backward(dtype, dh, N, B, H):
     g = dqkv.float().view(B, N, 3, H, dh).permute(2, 0, 3, 1, 4)
     for i, t in enumerate((q, k, v)):
         assert _rel(g[i], t.grad) < (2e-2 if dtype == torch.bfloat16 else 1e-4), "qkv"[i]
+
+
+@pytest.mark.parametrize("impl", [1, 2])
+@pytest.mark.parametrize("dh,N,n0,B,H", [(64, 333, 333, 2, 3), (64, 256, 128, 2, 2), (64, 64, 64, 1, 1),
+                                         (64, 24, 24, 3, 2), (128, 1536, 512, 1, 2), (128, 200, 200, 1, 2),
+                                         (128, 700, 256, 2, 2), (128, 4608, 512, 1, 1)])
+def test_attention_backward_kernels_on_two_stream_views(dh, N, n0, B, H, impl):
+    """Both backward kernels (impl 1: warp-level MMA, 2: tcgen05) against PyTorch fp32 on
+    one buffer (n0 = N) and on the text/image stream split of the MMDiT double blocks."""
+    torch.manual_seed(N + dh + n0)
+    dev = "cuda"
+    d = H * dh
+    qkv = (torch.randn(B * N, 3 * d, device=dev) * 1.5).bfloat16()
+    o = torch.empty(B * N, d, device=dev, dtype=torch.bfloat16)
+    lse = torch.empty(B, H, N, device=dev)
+    jg.test_attention_fwd(qkv, B, N, H, dh, o, lse)
+    q, k, v = _attn_ref(qkv, B, N, H, dh)
+    q.requires_grad_(); k.requires_grad_(); v.requires_grad_()
+    ref_o = torch.softmax((q @ k.transpose(-1, -2)) / math.sqrt(dh), -1) @ v
+    dO = torch.randn(B * N, d, device=dev).bfloat16()
+    ref_o.backward(dO.float().view(B, N, H, dh).transpose(1, 2))
+
+    def split(x):
+        x = x.view(B, N, -1)
+        return x[:, :n0].contiguous(), x[:, n0:].contiguous()
+
+    dq0 = torch.full((B, n0, 3 * d), float("nan"), device=dev, dtype=torch.bfloat16)
+    dq1 = torch.full((B, N - n0, 3 * d), float("nan"), device=dev, dtype=torch.bfloat16)
+    jg.test_attention_bwd_streams(split(qkv), split(o), lse, split(dO), B, N, n0, H, dh, (dq0, dq1), impl=impl)
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    g = torch.cat([dq0, dq1], 1).float().view(B, N, 3, H, dh).permute(2, 0, 3, 1, 4)
+    for i, t in enumerate((q, k, v)):
+        assert _rel(g[i], t.grad) < 2e-2, "qkv"[i]
+
+
+def test_tcgen05_attention_backward_rejects_unaligned_streams():
+    B, N, n0, H, dh = 1, 300, 100, 2, 64
+    d = H * dh
+    x = lambda n, c: torch.zeros(B, n, c, device="cuda", dtype=torch.bfloat16)
+    lse = torch.zeros(B, H, N, device="cuda")
+    with pytest.raises(jg.JaggError):
+        jg.test_attention_bwd_streams((x(n0, 3 * d), x(N - n0, 3 * d)), (x(n0, d), x(N - n0, d)), lse,
+                                      (x(n0, d), x(N - n0, d)), B, N, n0, H, dh,
+                                      (x(n0, 3 * d), x(N - n0, 3 * d)), impl=2)
