@@ -336,6 +336,141 @@ __global__ void __launch_bounds__(256, LNF_MIN_BLOCKS) ln_gate_fused_kernel(LnGa
   }
 }
 
+// Row-in-registers variant for d = 128 NV <= 768: a warp issues every load of one row at
+// once (dm, h, dh, y: 4 float4-wide groups per 128 columns), forms the row statistics
+// with two warp reductions and updates the row without a second pass over dm and h.  The
+// per-sequence column sums go to a warp-private shared-memory slab ([4 quantities][d],
+// plain read-modify-write, no atomics), summed over the block's 8 warps per unit.
+constexpr int LNR_ROWS = 32;  // rows per (sequence, chunk) unit: 4 per warp
+template <int NV>
+__global__ void __launch_bounds__(256, 2) ln_gate_rowreg_kernel(LnGateBwd a) {
+  extern __shared__ float part[];  // [8 warps][4 quantities][d]
+  constexpr int d = 128 * NV;
+  const int warp = threadIdx.x / 32, lane = threadIdx.x & 31;
+  float* mine = part + warp * 4 * d;
+  const int chunks = (a.rows_per_seq + LNR_ROWS - 1) / LNR_ROWS;
+  const int units = (a.M / a.rows_per_seq) * chunks;
+  const int is_f32 = a.dtype == JAGG_DTYPE_F32;
+  for (int unit = blockIdx.x; unit < units; unit += gridDim.x) {
+    const int b = unit / chunks;
+    const int r0 = (unit % chunks) * LNR_ROWS;
+    for (int i = lane; i < 4 * d; i += 32) mine[i] = 0.f;
+    __syncwarp();
+    const float* gate = a.do_gate ? a.gate + (int64_t)b * a.mod_stride : nullptr;
+    const float* sc = a.do_ln ? a.scale + (int64_t)b * a.mod_stride : nullptr;
+#pragma unroll 1
+    for (int k = 0; k < 4; ++k) {
+      const int r = r0 + warp * 4 + k;
+      if (r >= a.rows_per_seq) break;
+      const int m = b * a.rows_per_seq + r;
+      const int64_t hr = seg_row(m, a.seg, a.seg_off, a.seg_stride);
+      float dm[NV][4], hv[NV][4], dh[NV][4], yv[NV][4];
+#pragma unroll
+      for (int i = 0; i < NV; ++i) {
+        const int c = (i * 32 + lane) * 4;
+        const float4 d4 = *reinterpret_cast<const float4*>(a.dh_in + hr * d + c);
+        dh[i][0] = d4.x; dh[i][1] = d4.y; dh[i][2] = d4.z; dh[i][3] = d4.w;
+        if (a.do_ln) {
+          load4(a.dm, (int64_t)m * d + c, a.dm_f32, dm[i]);
+          const float4 h4 = *reinterpret_cast<const float4*>(a.h + hr * d + c);
+          hv[i][0] = h4.x; hv[i][1] = h4.y; hv[i][2] = h4.z; hv[i][3] = h4.w;
+        }
+        if (gate) load4(a.y, (int64_t)m * d + c, is_f32, yv[i]);
+      }
+      if (a.do_ln) {
+        const float mu = a.mean[m], rs = a.rstd[m];
+        float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+        for (int i = 0; i < NV; ++i) {
+          const int c = (i * 32 + lane) * 4;
+          const float4 s4 = *reinterpret_cast<const float4*>(sc + c);
+          const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            hv[i][e] = (hv[i][e] - mu) * rs;  // now x-hat
+            const float dxh = dm[i][e] * (1.f + sv[e]);
+            s1 += dxh;
+            s2 += dxh * hv[i][e];
+          }
+        }
+        s1 = warp_sum(s1) / d;
+        s2 = warp_sum(s2) / d;
+#pragma unroll
+        for (int i = 0; i < NV; ++i) {
+          const int c = (i * 32 + lane) * 4;
+          const float4 s4 = *reinterpret_cast<const float4*>(sc + c);
+          const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) dh[i][e] += rs * (dm[i][e] * (1.f + sv[e]) - s1 - hv[i][e] * s2);
+          *reinterpret_cast<float4*>(a.dh_out + hr * d + c) = make_float4(dh[i][0], dh[i][1], dh[i][2], dh[i][3]);
+          float4* q0 = reinterpret_cast<float4*>(mine + c);
+          float4* q1 = reinterpret_cast<float4*>(mine + d + c);
+          float4 u = *q0, w = *q1;
+          u.x += dm[i][0]; u.y += dm[i][1]; u.z += dm[i][2]; u.w += dm[i][3];
+          w.x += dm[i][0] * hv[i][0]; w.y += dm[i][1] * hv[i][1]; w.z += dm[i][2] * hv[i][2];
+          w.w += dm[i][3] * hv[i][3];
+          *q0 = u;
+          *q1 = w;
+        }
+      }
+      if (gate) {
+#pragma unroll
+        for (int i = 0; i < NV; ++i) {
+          const int c = (i * 32 + lane) * 4;
+          const float4 g4 = *reinterpret_cast<const float4*>(gate + c);
+          const float dy[4] = {g4.x * dh[i][0], g4.y * dh[i][1], g4.z * dh[i][2], g4.w * dh[i][3]};
+          store4(a.dy, (int64_t)m * d + c, is_f32, dy);
+          float4* q2 = reinterpret_cast<float4*>(mine + 2 * d + c);
+          float4* q3 = reinterpret_cast<float4*>(mine + 3 * d + c);
+          float4 u = *q2, w = *q3;
+          u.x += dh[i][0] * yv[i][0]; u.y += dh[i][1] * yv[i][1]; u.z += dh[i][2] * yv[i][2];
+          u.w += dh[i][3] * yv[i][3];
+          w.x += dh[i][0]; w.y += dh[i][1]; w.z += dh[i][2]; w.w += dh[i][3];
+          *q2 = u;
+          *q3 = w;
+        }
+      }
+    }
+    __syncthreads();
+    for (int c = threadIdx.x; c < d; c += blockDim.x) {
+      float P[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int w = 0; w < 8; ++w)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) P[q] += part[(w * 4 + q) * d + c];
+      if (a.do_ln) {
+        atomicAdd(a.dshift + (int64_t)b * a.dmod_stride + c, P[0]);
+        atomicAdd(a.dscale + (int64_t)b * a.dmod_stride + c, P[1]);
+      }
+      if (a.do_gate) {
+        atomicAdd(a.dgate + (int64_t)b * a.dmod_stride + c, P[2]);
+        if (a.dbias) atomicAdd(a.dbias + c, gate[c] * P[3]);
+      }
+    }
+    __syncthreads();  // the slabs are re-zeroed by the next unit
+  }
+}
+
+template <int NV>
+int launch_ln_gate_rowreg(const LnGateBwd& a, cudaStream_t s) {
+  const int smem = 8 * 4 * 128 * NV * (int)sizeof(float);
+  static bool attr = false;
+  if (!attr) {
+    JAGG_CUDA_TRY(cudaFuncSetAttribute(ln_gate_rowreg_kernel<NV>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    attr = true;
+  }
+  static int per_sm = 0;
+  if (!per_sm) {
+    JAGG_CUDA_TRY(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ln_gate_rowreg_kernel<NV>, 256, smem));
+    if (per_sm < 1) per_sm = 1;
+  }
+  const int units = (a.M / a.rows_per_seq) * ceil_div(a.rows_per_seq, LNR_ROWS);
+  const int cap = per_sm * sm_count();
+  ln_gate_rowreg_kernel<NV><<<units < cap ? units : cap, 256, smem, s>>>(a);
+  JAGG_LAUNCHED();
+  return JAGG_OK;
+}
+
 template <int NVT>
 int launch_ln_gate_nv(const LnGateBwd& a, int smem, cudaStream_t s) {
   static bool attr = false;
@@ -611,9 +746,9 @@ int launch_ln_gate_bwd(const LnGateBwd& a, cudaStream_t s) {
   const int tok = prof_start(s);
   int st;
   switch (a.d % 128 == 0 ? a.d / 128 : 0) {
-    case 3: st = launch_ln_gate_nv<3>(a, smem, s); break;
-    case 4: st = launch_ln_gate_nv<4>(a, smem, s); break;
-    case 6: st = launch_ln_gate_nv<6>(a, smem, s); break;
+    case 3: st = launch_ln_gate_rowreg<3>(a, s); break;
+    case 4: st = launch_ln_gate_rowreg<4>(a, s); break;
+    case 6: st = launch_ln_gate_rowreg<6>(a, s); break;
     case 8: st = launch_ln_gate_nv<8>(a, smem, s); break;
     case 12: st = launch_ln_gate_nv<12>(a, smem, s); break;
     case 24: st = launch_ln_gate_nv<24>(a, smem, s); break;
