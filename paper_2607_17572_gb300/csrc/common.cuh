@@ -93,6 +93,15 @@ __device__ __forceinline__ void gelu_tanh_both(float u, float& g, float& dg) {
   g = 0.5f * u * (1.f + th);
   dg = 0.5f * (1.f + th) + 0.5f * u * (1.f - th * th) * c * (1.f + 3.f * a * u * u);
 }
+// The same pair with tanh from the hardware approximation (tanh.approx.f32, absolute
+// error below 2^-10): for outputs rounded to bf16 (the tensor-core path).
+__device__ __forceinline__ void gelu_tanh_both_approx(float u, float& g, float& dg) {
+  const float c = 0.7978845608028654f, a = 0.044715f;
+  float th;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(th) : "f"(c * (u + a * u * u * u)));
+  g = 0.5f * u * (1.f + th);
+  dg = 0.5f * (1.f + th) + 0.5f * u * (1.f - th * th) * c * (1.f + 3.f * a * u * u);
+}
 __device__ __forceinline__ float silu_f(float x) { return x / (1.f + expf(-x)); }
 __device__ __forceinline__ float silu_grad_f(float x) {
   float s = 1.f / (1.f + expf(-x));

@@ -3,7 +3,7 @@
 // bf16 x bf16 -> f32: a persistent, warp-specialised tcgen05 kernel.  One CTA per SM;
 // warp 0 issues TMA loads of 128-byte-swizzled tiles into a multi-stage shared-memory
 // ring, warp 1 (one elected thread) issues tcgen05.mma into a double-buffered TMEM
-// accumulator, warps 2-5 drain TMEM with tcgen05.ld and run the fused epilogue while
+// accumulator, warps 2-9 (two per TMEM lane quarter) drain TMEM with tcgen05.ld and run the fused epilogue while
 // the next tile's MMAs proceed.  Both operands may be K-major or MN-major, so the
 // forward (X W^T), input-gradient (dY W) and weight-gradient (dY^T X) products all read
 // their operands in place, without transposes.
@@ -174,7 +174,11 @@ __device__ __forceinline__ void epi_apply8(const EpiParams& e, int m, int n, con
 // Staged epilogues: the output tile goes through swizzled shared memory and leaves with
 // TMA stores (or TMA f32 reduce-adds), and the multiplier of EPI_MUL_AUX arrives in
 // shared memory by TMA before the accumulator is ready.
-enum : int { STAGED_NONE = 0, STAGED_STORE = 1, STAGED_MUL_AUX = 2, STAGED_ACCUM = 3 };
+// STAGED_ROWS: the other row-major epilogues (GELU, gated residual, row-remapped stores):
+// each 32 x 32 chunk goes through swizzled shared memory and back so that a lane holds 4
+// consecutive columns of one row, and every global load / store of the epilogue covers
+// contiguous 128-byte row segments.
+enum : int { STAGED_NONE = 0, STAGED_STORE = 1, STAGED_MUL_AUX = 2, STAGED_ACCUM = 3, STAGED_ROWS = 4 };
 
 struct TcParams {
   int tiles_m, tiles_n, splits, k_blocks;
@@ -184,23 +188,29 @@ struct TcParams {
 
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;
-constexpr int TC_THREADS = 192;
+// Epilogue warps EW: 4 (one per TMEM lane quarter, two staging chunks each: the TMA-staged
+// epilogues, whose stores overlap the next chunk) or 8 (two per quarter, alternate
+// chunks, one staging chunk each: the arithmetic-heavy row-coalesced epilogues).
+constexpr int TC_MAX_EPI_WARPS = 8;
+__host__ __device__ constexpr int tc_threads(int ew) { return 64 + 32 * ew; }
 
 // AUX: the instance can run EPI_MUL_AUX (the input-gradient products, K-major A and
 // MN-major B); the others need no shared memory for a multiplier.
-template <int BN, bool AUX>
+template <int BN, bool AUX, int EW>
 struct TcCfg {
+  static constexpr int SPLIT = EW / 4;           // chunk stride of an epilogue warp
+  static constexpr int NSTG = EW == 4 ? 2 : 1;   // staging chunks per epilogue warp
   static constexpr int A_BYTES = TC_BM * TC_BK * 2;
   static constexpr int B_BYTES = BN * TC_BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  // Per epilogue warp (32 rows): two staging chunks of 32 x 32 outputs (4 KB each for f32;
-  // the bf16 output of EPI_MUL_AUX uses 2 KB each), and for EPI_MUL_AUX the tile's
-  // multiplier rows, BN / 32 chunks of 32 x 32 bf16 after the bf16 staging chunks.
+  // Per epilogue warp (32 rows, every other 32-column chunk of the tile): one staging
+  // chunk of 32 x 32 outputs (4 KB as f32; the bf16 output of EPI_MUL_AUX uses 2 KB), and
+  // for EPI_MUL_AUX this warp's multiplier chunks (BN / 64 of 32 x 32 bf16) after it.
   static constexpr int CHUNK_BF16 = 32 * 32 * 2;
-  static constexpr int AUX_WARP_BYTES = 2 * CHUNK_BF16 + (BN / 32) * CHUNK_BF16;
+  static constexpr int AUX_WARP_BYTES = NSTG * CHUNK_BF16 + ((BN / 32 + SPLIT - 1) / SPLIT) * CHUNK_BF16;
   static constexpr int EPI_WARP_BYTES =
-      AUX && AUX_WARP_BYTES > 4 * CHUNK_BF16 ? AUX_WARP_BYTES : 4 * CHUNK_BF16;
-  static constexpr int EPI_BYTES = 4 * EPI_WARP_BYTES;
+      AUX && AUX_WARP_BYTES > NSTG * 2 * CHUNK_BF16 ? AUX_WARP_BYTES : NSTG * 2 * CHUNK_BF16;
+  static constexpr int EPI_BYTES = EW * EPI_WARP_BYTES;
   static constexpr int FIXED = 1024 /*align*/ + 256 /*barriers*/;
   static constexpr int MAX_SMEM = 232448;
   static constexpr int FIT = (MAX_SMEM - FIXED - EPI_BYTES) / STAGE_BYTES;
@@ -211,12 +221,13 @@ struct TcCfg {
   static_assert(SMEM_BYTES <= MAX_SMEM, "shared memory budget");
 };
 
-template <int BN, bool A_MN, bool B_MN, bool AUX>
-__global__ void __launch_bounds__(TC_THREADS, 1)
+template <int BN, bool A_MN, bool B_MN, bool AUX, int EW>
+__global__ void __launch_bounds__(tc_threads(EW), 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmX, TcParams p) {
-  using Cfg = TcCfg<BN, AUX>;
+  using Cfg = TcCfg<BN, AUX, EW>;
   constexpr int STAGES = Cfg::STAGES;
+  constexpr int SPLIT = Cfg::SPLIT;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* epi_smem = smem + STAGES * Cfg::STAGE_BYTES;  // 1024-byte aligned
@@ -225,7 +236,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   uint64_t* tfull = empty + STAGES;
   uint64_t* tempty = tfull + 2;
   uint64_t* auxbar = tempty + 2;  // one per epilogue warp
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(auxbar + 4);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(auxbar + TC_MAX_EPI_WARPS);
   __shared__ volatile int abort_flag;
 
   const int warp = threadIdx.x >> 5;
@@ -239,13 +250,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       ptx::mbar_init(&tfull[a], 1);
-      ptx::mbar_init(&tempty[a], 4);
+      ptx::mbar_init(&tempty[a], EW);
     }
-    for (int q = 0; q < 4; ++q) ptx::mbar_init(&auxbar[q], 1);
+    for (int q = 0; q < EW; ++q) ptx::mbar_init(&auxbar[q], 1);
     ptx::fence_mbar_init();
     ptx::prefetch_tmap(&tmA);
     ptx::prefetch_tmap(&tmB);
-    if (p.staged != STAGED_NONE) ptx::prefetch_tmap(&tmC);
+    if (p.staged != STAGED_NONE && p.staged != STAGED_ROWS) ptx::prefetch_tmap(&tmC);
     if (p.staged == STAGED_MUL_AUX) ptx::prefetch_tmap(&tmX);
   }
   if (warp == 1) {
@@ -341,18 +352,138 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         if (++acc == 2) { acc = 0; acc_phase ^= 1; }
       }
     }
+  } else if constexpr (EW == 8) {
+    // ---------------- row-coalesced epilogue (the only epilogue of the 8-warp instances), warps 2..9: TMEM lanes 32*(warp%4) .. +31, alternate chunks
+    const int q = warp & 3, half = (warp - 2) >> 2, ew = warp - 2;  // half < SPLIT
+    float* xch = reinterpret_cast<float*>(epi_smem + ew * Cfg::EPI_WARP_BYTES);  // one 32 x 32 f32 chunk
+    const EpiParams& e = p.e;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    const int sub = lane >> 3, c4 = lane & 7;  // read-back: rows sub, sub + 4, ...; columns 4 c4 .. +3
+    for (int t = blockIdx.x; t < total; t += gridDim.x) {
+      int tm, tn, ks;
+      decode(t, tm, tn, ks);
+      bool ok = ptx::mbar_wait(&tfull[acc], acc_phase);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) { abort_flag = 1; break; }
+      ptx::tc_fence_after();
+      const int m0 = tm * TC_BM + q * 32;
+      const int live_chunks = (m0 < e.M) ? min(BN / 32, (e.N - tn * BN + 31) / 32) : 0;
+#pragma unroll 1
+      for (int c = half; c < live_chunks; c += SPLIT) {
+        uint32_t r[32];
+        ptx::tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c * 32, r);
+        ptx::tmem_ld_wait();
+        __syncwarp();  // the previous chunk's read-back is done
+        uint8_t* row = reinterpret_cast<uint8_t*>(xch) + lane * 128;
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          *reinterpret_cast<uint4*>(row + ((u ^ (lane & 7)) << 4)) =
+              make_uint4(r[4 * u], r[4 * u + 1], r[4 * u + 2], r[4 * u + 3]);
+        __syncwarp();
+        const int n = tn * BN + c * 32 + 4 * c4;
+        float b4[4] = {0.f, 0.f, 0.f, 0.f};
+        if (e.bias && e.epi != EPI_MUL_AUX && n < e.N) {
+          if (e.bias_bf16) {
+            const uint2 raw = *reinterpret_cast<const uint2*>(static_cast<const bf16*>(e.bias) + n);
+            const bf16* hb = reinterpret_cast<const bf16*>(&raw);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) b4[i] = __bfloat162float(hb[i]);
+          } else {
+            const float4 f = *reinterpret_cast<const float4*>(static_cast<const float*>(e.bias) + n);
+            b4[0] = f.x; b4[1] = f.y; b4[2] = f.z; b4[3] = f.w;
+          }
+        }
+        // every global operand of the chunk first (8 rows per lane), then the stores
+        float4 av[8], xa[8], xg[8];
+#pragma unroll
+        for (int it = 0; it < 8; ++it) {
+          const int rr = it * 4 + sub;
+          const int m = m0 + rr;
+          av[it] = *reinterpret_cast<const float4*>(reinterpret_cast<uint8_t*>(xch) + rr * 128 + ((c4 ^ (rr & 7)) << 4));
+          xa[it] = make_float4(0.f, 0.f, 0.f, 0.f);
+          xg[it] = xa[it];
+          if (m < e.M && n < e.N) {
+            if (e.epi == EPI_GATE_RESID) {
+              xg[it] = *reinterpret_cast<const float4*>(e.gate + (int64_t)(m / e.rows_per_seq) * e.gate_stride + n);
+              xa[it] = *reinterpret_cast<const float4*>(static_cast<const float*>(e.aux) + (int64_t)m * e.ld_aux + n);
+            } else if (e.epi == EPI_MUL_AUX) {
+              if (e.c_bf16) {
+                const uint2 raw =
+                    *reinterpret_cast<const uint2*>(static_cast<const bf16*>(e.aux) + (int64_t)m * e.ld_aux + n);
+                const bf16* hb = reinterpret_cast<const bf16*>(&raw);
+                xa[it] = make_float4(__bfloat162float(hb[0]), __bfloat162float(hb[1]), __bfloat162float(hb[2]),
+                                     __bfloat162float(hb[3]));
+              } else {
+                xa[it] = *reinterpret_cast<const float4*>(static_cast<const float*>(e.aux) + (int64_t)m * e.ld_aux + n);
+              }
+            }
+          }
+        }
+        __syncwarp();  // the chunk buffer is free for the next chunk
+        auto st4 = [&](void* base, int64_t idx, int is_bf16, const float (&x)[4]) {
+          if (is_bf16) {
+            __nv_bfloat162 lo = __floats2bfloat162_rn(x[0], x[1]), hi = __floats2bfloat162_rn(x[2], x[3]);
+            uint2 raw;
+            raw.x = *reinterpret_cast<uint32_t*>(&lo);
+            raw.y = *reinterpret_cast<uint32_t*>(&hi);
+            *reinterpret_cast<uint2*>(static_cast<bf16*>(base) + idx) = raw;
+          } else {
+            *reinterpret_cast<float4*>(static_cast<float*>(base) + idx) = make_float4(x[0], x[1], x[2], x[3]);
+          }
+        };
+#pragma unroll
+        for (int it = 0; it < 8; ++it) {
+          const int m = m0 + it * 4 + sub;
+          if (m >= e.M || n >= e.N) continue;
+          const float4 a4 = av[it];
+          float v[4] = {a4.x + b4[0], a4.y + b4[1], a4.z + b4[2], a4.w + b4[3]};
+          const int64_t cr = epi_crow(e, m);
+          switch (e.epi) {
+            case EPI_STORE:
+              st4(e.C, cr * e.ldc + n, e.c_bf16, v);
+              break;
+            case EPI_GELU: {
+              float g[4], dg[4];
+#pragma unroll
+              for (int i = 0; i < 4; ++i) gelu_tanh_both_approx(v[i], g[i], dg[i]);
+              st4(e.C, cr * e.ldc + n, e.c_bf16, dg);
+              st4(e.C2, cr * e.ldc2 + n, e.c_bf16, g);
+            } break;
+            case EPI_GATE_RESID: {
+              st4(e.C, cr * e.ldc + n, e.c_bf16, v);
+              const float4 g4 = xg[it], h4 = xa[it];
+              const float o[4] = {h4.x + g4.x * v[0], h4.y + g4.y * v[1], h4.z + g4.z * v[2], h4.w + g4.w * v[3]};
+              st4(e.C2, (int64_t)m * e.ldc2 + n, 0, o);
+            } break;
+            case EPI_MUL_AUX: {
+              const float4 u4 = xa[it];
+              const float o[4] = {a4.x * u4.x, a4.y * u4.y, a4.z * u4.z, a4.w * u4.w};
+              st4(e.C, cr * e.ldc + n, e.c_bf16, o);
+            } break;
+            case EPI_ACCUM:
+              ptx::red_add_v4(static_cast<float*>(e.C) + cr * e.ldc + n, a4.x, a4.y, a4.z, a4.w);
+              break;
+          }
+        }
+      }
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(&tempty[acc]);
+      if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+    }
   } else if (p.staged != STAGED_NONE) {
-    // ---------------- staged epilogue, warps 2..5: TMEM lanes 32*(warp%4) .. +31.
+    // ---------------- staged epilogue (4-warp instances), warps 2..5: TMEM lanes 32*(warp%4) .. +31.
     // Thread = output row; per 32-column chunk: tcgen05.ld, the element-wise op, a write
     // into a swizzled staging chunk (64-byte rows for bf16, 128-byte rows for f32, so the
     // 16-byte writes of a warp hit distinct banks), then one TMA store / reduce-add of the
-    // 32 x 32 box by lane 0.  Two staging chunks alternate.
-    const int q = warp & 3;
+    // 32 x 32 box by lane 0.  The two warps of a lane quarter take alternate chunks.
+    const int q = warp & 3, half = (warp - 2) >> 2, ew = warp - 2;  // half < SPLIT
     const bool mul = p.staged == STAGED_MUL_AUX;
     const bool out_f32 = !p.e.c_bf16;
     const int chunk_bytes = out_f32 ? 4096 : Cfg::CHUNK_BF16;
-    uint8_t* stg = epi_smem + q * Cfg::EPI_WARP_BYTES;
-    uint8_t* auxs = stg + 2 * Cfg::CHUNK_BF16;  // EPI_MUL_AUX only (bf16 output)
+    uint8_t* stg = epi_smem + ew * Cfg::EPI_WARP_BYTES;
+    uint8_t* auxs = stg + Cfg::NSTG * Cfg::CHUNK_BF16;  // EPI_MUL_AUX only (bf16 output)
     int acc = 0, sbuf = 0;
     uint32_t acc_phase = 0, aux_phase = 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
@@ -362,26 +493,28 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       // boxes wholly outside the output (rows past M, column chunks past N) are skipped
       const bool rows_live = m0 < p.e.M;
       const int live_chunks = min(BN / 32, (p.e.N - tn * BN + 31) / 32);
-      const bool aux_load = mul && rows_live;
+      const int my_chunks = live_chunks > half ? (live_chunks - half + SPLIT - 1) / SPLIT : 0;
+      const bool aux_load = mul && rows_live && my_chunks > 0;
       if (aux_load) {
-        // the tile's multiplier rows; this warp finished reading the previous tile's
+        // this warp's multiplier chunks of the tile; it finished reading the previous tile's
         __syncwarp();
         if (lane == 0) {
-          ptx::mbar_arrive_expect_tx(&auxbar[q], live_chunks * Cfg::CHUNK_BF16);
-          for (int c = 0; c < live_chunks; ++c)
-            ptx::tma_load_2d(auxs + c * Cfg::CHUNK_BF16, &tmX, &auxbar[q], tn * BN + c * 32, m0);
+          ptx::mbar_arrive_expect_tx(&auxbar[ew], my_chunks * Cfg::CHUNK_BF16);
+          for (int i = 0; i < my_chunks; ++i)
+            ptx::tma_load_2d(auxs + i * Cfg::CHUNK_BF16, &tmX, &auxbar[ew], tn * BN + (half + SPLIT * i) * 32,
+                             m0);
         }
       }
       bool ok = ptx::mbar_wait(&tfull[acc], acc_phase);
       if (aux_load) {
-        ok = ok && ptx::mbar_wait(&auxbar[q], aux_phase);
+        ok = ok && ptx::mbar_wait(&auxbar[ew], aux_phase);
         aux_phase ^= 1u;
       }
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) { abort_flag = 1; break; }
       ptx::tc_fence_after();
 #pragma unroll 1
-      for (int c = 0; c < (rows_live ? live_chunks : 0); ++c) {
+      for (int c = half; c < (rows_live ? live_chunks : 0); c += SPLIT) {
         uint32_t r[32];
         ptx::tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c * 32, r);
         ptx::tmem_ld_wait();
@@ -399,7 +532,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           }
         }
         if (mul) {
-          const uint8_t* ar = auxs + c * Cfg::CHUNK_BF16 + lane * 64;
+          const uint8_t* ar = auxs + (c / SPLIT) * Cfg::CHUNK_BF16 + lane * 64;
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
             const uint4 raw = *reinterpret_cast<const uint4*>(ar + ((j ^ ((lane >> 1) & 3)) << 4));
@@ -408,8 +541,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             for (int i = 0; i < 8; ++i) v[j * 8 + i] *= __bfloat162float(h[i]);
           }
         }
-        // the staging chunk written two chunks ago must have been read by its TMA
-        if (lane == 0) ptx::bulk_wait_read<1>();
+        // the staging chunk's previous TMA has read it
+        if (lane == 0) {
+          if constexpr (Cfg::NSTG == 2)
+            ptx::bulk_wait_read<1>();
+          else
+            ptx::bulk_wait_read<0>();
+        }
         __syncwarp();
         uint8_t* sb = stg + sbuf * chunk_bytes;
         if (out_f32) {
@@ -438,7 +576,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             ptx::tma_store_2d(&tmC, sb, n0, m0);
           ptx::bulk_commit();
         }
-        sbuf ^= 1;
+        sbuf = (sbuf + 1) % Cfg::NSTG;
       }
       ptx::tc_fence_before();
       __syncwarp();
@@ -448,8 +586,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     if (lane == 0) ptx::bulk_wait<0>();
     __syncwarp();
   } else {
-    // ---------------- epilogue warps 2..5: TMEM lanes 32*(warp%4) .. +31
-    const int q = warp & 3;
+    // ---------------- epilogue warps 2..9: TMEM lanes 32*(warp%4) .. +31, alternate chunks
+    const int q = warp & 3, half = (warp - 2) >> 2;
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
@@ -461,7 +599,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       ptx::tc_fence_after();
       const int m = tm * TC_BM + q * 32 + lane;
 #pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
+      for (int c = half; c < BN / 32; c += SPLIT) {
         uint32_t r[32];
         ptx::tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c * 32, r);
         ptx::tmem_ld_wait();
@@ -670,7 +808,15 @@ double tile_cost(const GemmArgs& g, int BN, int nsm) {
 // 16-byte aligned with 16-byte row pitches.
 int staged_mode(const GemmArgs& g) {
   auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
-  if (g.c_trans || g.bias_m || g.remap_rows || !al16(g.C)) return STAGED_NONE;
+  if (g.c_trans || g.bias_m || !al16(g.C)) return STAGED_NONE;
+  if (g.remap_rows || g.epi == EPI_GELU || g.epi == EPI_GATE_RESID) {
+    // row-coalesced path: 4-column groups, 16-byte aligned rows of every operand
+    bool ok = g.N % 4 == 0 && g.ldc % 4 == 0 && (!g.bias || al16(g.bias));
+    if (g.epi == EPI_GELU || g.epi == EPI_GATE_RESID) ok = ok && g.C2 && al16(g.C2) && g.ldc2 % 4 == 0;
+    if (g.epi == EPI_GATE_RESID || g.epi == EPI_MUL_AUX) ok = ok && al16(g.aux) && g.ld_aux % 4 == 0;
+    if (g.epi == EPI_GATE_RESID) ok = ok && g.gate_stride % 4 == 0 && al16(g.gate);
+    return ok ? STAGED_ROWS : STAGED_NONE;
+  }
   const bool c_f32 = g.c_dtype == JAGG_DTYPE_F32;
   if ((g.ldc * (c_f32 ? 4 : 2)) % 16) return STAGED_NONE;
   switch (g.epi) {
@@ -695,9 +841,9 @@ int validate(const GemmArgs& g) {
   return JAGG_OK;
 }
 
-template <int BN, bool A_MN, bool B_MN, bool AUX>
+template <int BN, bool A_MN, bool B_MN, bool AUX, int EW = 4>
 int launch_tc(const GemmArgs& g, cudaStream_t stream) {
-  using Cfg = TcCfg<BN, AUX>;
+  using Cfg = TcCfg<BN, AUX, EW>;
   CUtensorMap ta, tb;
   if (!A_MN)
     JAGG_TRY(make_tmap(&ta, g.A, g.M, g.K, g.lda, TC_BK, TC_BM));
@@ -709,8 +855,11 @@ int launch_tc(const GemmArgs& g, cudaStream_t stream) {
     JAGG_TRY(make_tmap(&tb, g.B, g.K, g.N, g.ldb, 64, TC_BK));
   TcParams p;
   p.staged = staged_mode(g);
-  CUtensorMap tc = ta, tx = ta;  // unused unless staged
-  if (p.staged != STAGED_NONE) {
+  // the row-coalesced epilogue exists in the 8-warp instances only; elsewhere the
+  // per-thread epilogue serves those requests
+  if ((p.staged == STAGED_ROWS) != (EW == 8)) p.staged = EW == 8 ? STAGED_ROWS : STAGED_NONE;
+  CUtensorMap tc = ta, tx = ta;  // unused unless staged through TMA
+  if (p.staged != STAGED_NONE && p.staged != STAGED_ROWS) {
     const bool c_f32 = g.c_dtype == JAGG_DTYPE_F32;
     JAGG_TRY(make_tmap(&tc, g.C, g.M, g.N, g.ldc, 32, 32, c_f32,
                        c_f32 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B));
@@ -728,12 +877,12 @@ int launch_tc(const GemmArgs& g, cudaStream_t stream) {
   const int grid = total < nsm ? total : nsm;
   static bool attr_set = false;  // one per template instance
   if (!attr_set) {
-    JAGG_CUDA_TRY(cudaFuncSetAttribute(gemm_tc_kernel<BN, A_MN, B_MN, AUX>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    JAGG_CUDA_TRY(cudaFuncSetAttribute(gemm_tc_kernel<BN, A_MN, B_MN, AUX, EW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Cfg::SMEM_BYTES));
     attr_set = true;
   }
   const int tok = prof_start(stream);
-  gemm_tc_kernel<BN, A_MN, B_MN, AUX><<<grid, TC_THREADS, Cfg::SMEM_BYTES, stream>>>(ta, tb, tc, tx, p);
+  gemm_tc_kernel<BN, A_MN, B_MN, AUX, EW><<<grid, tc_threads(EW), Cfg::SMEM_BYTES, stream>>>(ta, tb, tc, tx, p);
   JAGG_LAUNCHED();
   prof_stop(tok, stream, PROF_GEMM_TC, 2.0 * g.M * g.N * g.K,
             2.0 * ((double)g.M * g.K + (double)g.N * g.K) + (double)g.M * g.N * (g.c_dtype == JAGG_DTYPE_F32 ? 4 : 2),
@@ -752,6 +901,17 @@ int dispatch_bn(const GemmArgs& g, cudaStream_t stream) {
       JAGG_CHECK_ARG(g.tile_n != 256, "gemm: the multiplier epilogue uses tiles of at most 128 columns");
       if (g.tile_n == 64 || (g.tile_n == 0 && g.N < 128)) return launch_tc<64, A_MN, B_MN, true>(g, stream);
       return launch_tc<128, A_MN, B_MN, true>(g, stream);
+    }
+  }
+  if constexpr (!A_MN && !B_MN) {
+    // the forward products' arithmetic-heavy epilogues (GELU, gated residual) on 8 warps
+    if (staged_mode(g) == STAGED_ROWS) {
+      const int nsm = sm_count();
+      if (g.tile_n == 64 || (g.tile_n == 0 && g.N < 128)) return launch_tc<64, false, false, false, 8>(g, stream);
+      if (g.tile_n == 128) return launch_tc<128, false, false, false, 8>(g, stream);
+      if (g.tile_n == 256 || (g.tile_n == 0 && g.N >= 256 && tile_cost(g, 256, nsm) < tile_cost(g, 128, nsm)))
+        return launch_tc<256, false, false, false, 8>(g, stream);
+      return launch_tc<128, false, false, false, 8>(g, stream);
     }
   }
   if (g.tile_n == 64 || (g.tile_n == 0 && g.N < 128)) return launch_tc<64, A_MN, B_MN, false>(g, stream);
