@@ -2,7 +2,8 @@
 // TMA-fed shared-memory operands), bf16, head dim 64 or 128 (appendix, Eqs. bwd_V ..
 // bwd_QK, with the softmax recomputed from the saved log-sum-exp).
 //
-// One CTA per (128-key tile, sequence, head) streams the sequence's query tiles:
+// Persistent: each CTA walks (128-key tile, sequence, head) units; per unit it streams the
+// sequence's query tiles:
 //   S^T = K Q^T, dP^T = V dO^T                      (128 x BQ, TMEM)
 //   P^T = exp(scale S^T - lse), dS^T = P^T (dP^T - rowsum(dO O))   (8 warps, -> bf16 smem)
 //   dV += P^T dO, dK += dS^T Q                      (128 x dh, TMEM, whole sequence)
@@ -18,6 +19,9 @@
 // tile j are formed (512 columns: 2 x (64 + 64) + 128 + 128).  Head dim 64: one S^T, dP^T
 // buffer (128 + 128 + 64 + 64 + 64 columns); the MMA warp issues S, dP of tile j + 1 before
 // dV, dK, dQ of tile j.
+// Tile-level barrier phases run on across units, so the next unit's K, V loads and first
+// products overlap the previous unit's last tiles and its dQ drain (head dim 64 keeps two
+// K, V buffers for that).
 // Ragged ends: 3D tensor maps [sequence][token][column] per stream buffer make TMA read
 // zeros past the last token and drop dQ rows past it.
 #include <cuda.h>
@@ -42,11 +46,14 @@ struct FbCfg {
   static constexpr int KV_BYTES = BK * D * 2;
   static constexpr int QT_BYTES = BQ * D * 2;
   static constexpr int PS_BYTES = BK * BQ * 2;
-  static constexpr int STAGES = 3;
+  // head dim 64 (short sequences in practice): K, V double-buffered across the CTA's
+  // units, two Q / dO stages; head dim 128: one K, V buffer, three stages
+  static constexpr int KVB = D == 64 ? 2 : 1;
+  static constexpr int STAGES = D == 64 ? 2 : 3;
   static constexpr int DQ_WARP_BYTES = 32 * 32 * 4;  // one 32 x 32 f32 box, used twice per tile
-  static constexpr int OFF_K = 0;
-  static constexpr int OFF_V = OFF_K + KV_BYTES;
-  static constexpr int OFF_Q = OFF_V + KV_BYTES;
+  static constexpr int OFF_K = 0;                       // KVB buffers
+  static constexpr int OFF_V = OFF_K + KVB * KV_BYTES;    // KVB buffers
+  static constexpr int OFF_Q = OFF_V + KVB * KV_BYTES;
   static constexpr int OFF_DO = OFF_Q + STAGES * QT_BYTES;
   static constexpr int OFF_P = OFF_DO + STAGES * QT_BYTES;
   static constexpr int OFF_DS = OFF_P + PS_BYTES;
@@ -128,7 +135,7 @@ __device__ __forceinline__ void softmax32(const uint32_t* rs, const uint32_t* rp
 template <int D>
 __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_constant__ FbMaps maps, FbParams p) {
   using C = FbCfg<D>;
-  constexpr int BK = C::BK, BQ = C::BQ, NS = C::STAGES, NSB = C::NSB, CW = C::CW;
+  constexpr int BK = C::BK, BQ = C::BQ, NS = C::STAGES, NSB = C::NSB, CW = C::CW, KVB = C::KVB;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sK = sm + C::OFF_K;
@@ -146,19 +153,26 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
   uint64_t* bar_s = empty + NS;             // [NSB] S^T, dP^T of a tile are in TMEM buffer b
   uint64_t* bar_dq = bar_s + NSB;           // [NSB] dQ of a tile is in TMEM buffer b
   uint64_t* bar_dqfree = bar_dq + NSB;      // [NSB] the dQ warps have read it
-  uint64_t* bar_kv = bar_dqfree + NSB;      // K, V landed
-  uint64_t* bar_p = bar_kv + 1;             // P^T, dS^T written (S^T, dP^T read) by the 8 warps
-  uint64_t* bar_pfree = bar_kv + 2;         // the products reading P^T, dS^T are done
-  uint64_t* bar_fin = bar_kv + 3;           // every product is done (dK, dV final)
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_kv + 4);
+  uint64_t* bar_kv = bar_dqfree + NSB;      // [KVB] a unit's K, V landed
+  uint64_t* kv_free = bar_kv + KVB;         // [KVB] a unit's products are done (K, V reusable)
+  uint64_t* bar_p = kv_free + KVB;          // P^T, dS^T written (S^T, dP^T read) by the 8 warps
+  uint64_t* bar_pfree = bar_p + 1;          // the products reading P^T, dS^T are done
+  uint64_t* bar_fin = bar_p + 2;            // a unit's products are done (dK, dV final)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_p + 3);
   __shared__ volatile int abort_flag;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int kt = blockIdx.x, bh = blockIdx.y;
-  const int b = bh / p.heads, h = bh % p.heads;
   const int N = p.N;
-  const int k0 = kt * BK;
+  const int nkt = (N + BK - 1) / BK;
+  const int units = nkt * p.B * p.heads;
   const int nq = (N + BQ - 1) / BQ;
+  // unit u: key tile u % nkt of sequence-head u / nkt
+  auto unit_of = [&](int u, int& k0, int& b, int& h) {
+    const int bh = u / nkt;
+    k0 = (u % nkt) * BK;
+    b = bh / p.heads;
+    h = bh % p.heads;
+  };
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
@@ -171,7 +185,10 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
       ptx::mbar_init(&bar_dq[i], 1);
       ptx::mbar_init(&bar_dqfree[i], 4);
     }
-    ptx::mbar_init(bar_kv, 1);
+    for (int i = 0; i < KVB; ++i) {
+      ptx::mbar_init(&bar_kv[i], 1);
+      ptx::mbar_init(&kv_free[i], 1);
+    }
     ptx::mbar_init(bar_p, 8);
     ptx::mbar_init(bar_pfree, 1);
     ptx::mbar_init(bar_fin, 1);
@@ -199,45 +216,61 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
 
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA producer
-    if (lane == 0) {
-      const int s = seg_of(k0), r = row_in(k0);
-      ptx::mbar_arrive_expect_tx(bar_kv, 2 * C::KV_BYTES);
-#pragma unroll
-      for (int c = 0; c < D / 64; ++c) {
-        ptx::tma_load_3d(sK + c * BK * 128, &maps.k[s], bar_kv, (int)(p.k_col0 + h * D + c * 64), r, b);
-        ptx::tma_load_3d(sV + c * BK * 128, &maps.v[s], bar_kv, (int)(p.v_col0 + h * D + c * 64), r, b);
-      }
-    }
-    for (int j = 0; j < nq; ++j) {
-      const int st = j % NS;
+    int i = 0;
+    for (int u = blockIdx.x; u < units && !abort_flag; u += gridDim.x, ++i) {
+      int k0, b, h;
+      unit_of(u, k0, b, h);
+      const int bh = b * p.heads + h;
+      const int kvb = i % KVB;
       bool ok = true;
-      if (lane == 0) ok = ptx::mbar_wait(&empty[st], ((j / NS) & 1) ^ 1);
-      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-      if (!ok || abort_flag) { abort_flag = 1; break; }
-      const int q0 = j * BQ;
-      // lse and rowsum(dO O) of the tile's queries: asynchronous 4-byte copies (their
-      // addresses need not be 16-byte aligned) whose completion the stage barrier tracks;
-      // +inf / 0 past the last query
-      for (int i = lane; i < BQ; i += 32) {
-        const int q = q0 + i;
-        if (q < N) {
-          ptx::cp_async4(sLse + st * BQ + i, p.lse + (int64_t)bh * N + q);
-          ptx::cp_async4(sRd + st * BQ + i, p.Dv + (int64_t)bh * N + q);
-        } else {
-          sLse[st * BQ + i] = INFINITY;
-          sRd[st * BQ + i] = 0.f;
+      if (lane == 0) {
+        if (i >= KVB) ok = ptx::mbar_wait(&kv_free[kvb], ((i / KVB) & 1) ^ 1);
+        if (ok) {
+          const int s = seg_of(k0), r = row_in(k0);
+          ptx::mbar_arrive_expect_tx(&bar_kv[kvb], 2 * C::KV_BYTES);
+#pragma unroll
+          for (int c = 0; c < D / 64; ++c) {
+            ptx::tma_load_3d(sK + kvb * C::KV_BYTES + c * BK * 128, &maps.k[s], &bar_kv[kvb],
+                             (int)(p.k_col0 + h * D + c * 64), r, b);
+            ptx::tma_load_3d(sV + kvb * C::KV_BYTES + c * BK * 128, &maps.v[s], &bar_kv[kvb],
+                             (int)(p.v_col0 + h * D + c * 64), r, b);
+          }
         }
       }
-      ptx::cp_async_arrive_noinc(&full[st]);
-      __syncwarp();
-      if (lane == 0) {
-        const int s = seg_of(q0), r = row_in(q0);
-        ptx::mbar_arrive_expect_tx(&full[st], 2 * C::QT_BYTES);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      if (!ok) { abort_flag = 1; break; }
+      for (int j = 0; j < nq; ++j) {
+        const int g = i * nq + j;
+        const int st = g % NS;
+        if (lane == 0) ok = ptx::mbar_wait(&empty[st], ((g / NS) & 1) ^ 1);
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        if (!ok || abort_flag) { abort_flag = 1; break; }
+        const int q0 = j * BQ;
+        // lse and rowsum(dO O) of the tile's queries: asynchronous 4-byte copies (their
+        // addresses need not be 16-byte aligned) whose completion the stage barrier tracks;
+        // +inf / 0 past the last query
+        for (int t = lane; t < BQ; t += 32) {
+          const int q = q0 + t;
+          if (q < N) {
+            ptx::cp_async4(sLse + st * BQ + t, p.lse + (int64_t)bh * N + q);
+            ptx::cp_async4(sRd + st * BQ + t, p.Dv + (int64_t)bh * N + q);
+          } else {
+            sLse[st * BQ + t] = INFINITY;
+            sRd[st * BQ + t] = 0.f;
+          }
+        }
+        ptx::cp_async_arrive_noinc(&full[st]);
+        __syncwarp();
+        if (lane == 0) {
+          const int s = seg_of(q0), r = row_in(q0);
+          ptx::mbar_arrive_expect_tx(&full[st], 2 * C::QT_BYTES);
 #pragma unroll
-        for (int c = 0; c < D / 64; ++c) {
-          ptx::tma_load_3d(sQ + st * C::QT_BYTES + c * BQ * 128, &maps.q[s], &full[st],
-                           (int)(p.q_col0 + h * D + c * 64), r, b);
-          ptx::tma_load_3d(sdO + st * C::QT_BYTES + c * BQ * 128, &maps.dO[s], &full[st], h * D + c * 64, r, b);
+          for (int c = 0; c < D / 64; ++c) {
+            ptx::tma_load_3d(sQ + st * C::QT_BYTES + c * BQ * 128, &maps.q[s], &full[st],
+                             (int)(p.q_col0 + h * D + c * 64), r, b);
+            ptx::tma_load_3d(sdO + st * C::QT_BYTES + c * BQ * 128, &maps.dO[s], &full[st], h * D + c * 64, r,
+                             b);
+          }
         }
       }
     }
@@ -247,76 +280,87 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
       constexpr uint32_t id_s = ptx::idesc_bf16(128, BQ, false, false);
       constexpr uint32_t id_acc = ptx::idesc_bf16(128, D, false, true);
       constexpr uint32_t id_dq = ptx::idesc_bf16(128, 64, true, true);
-      const uint32_t aK = ptx::smem_u32(sK), aV = ptx::smem_u32(sV);
       const uint32_t aP = ptx::smem_u32(sP), adS = ptx::smem_u32(sdS);
-      // S^T, dP^T of tile j into TMEM buffer j % NSB
-      auto issue_s = [&](int j) {
-        const int st = j % NS, bb = j % NSB;
-        const uint32_t aQ = ptx::smem_u32(sQ + st * C::QT_BYTES), adO = ptx::smem_u32(sdO + st * C::QT_BYTES);
+      bool ok = true;
+      int i = 0;
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++i) {
+        const int kvb = i % KVB;
+        const uint32_t aK = ptx::smem_u32(sK + kvb * C::KV_BYTES), aV = ptx::smem_u32(sV + kvb * C::KV_BYTES);
+        // S^T, dP^T of global tile g into TMEM buffer g % NSB
+        auto issue_s = [&](int g) {
+          const int st = g % NS, bb = g % NSB;
+          const uint32_t aQ = ptx::smem_u32(sQ + st * C::QT_BYTES), adO = ptx::smem_u32(sdO + st * C::QT_BYTES);
 #pragma unroll
-        for (int k = 0; k < D / 16; ++k) {
-          ptx::umma_bf16(tmem + C::t_s(bb), kmajor_desc(aK, BK, k), kmajor_desc(aQ, BQ, k), id_s, k > 0);
-          ptx::umma_bf16(tmem + C::t_dp(bb), kmajor_desc(aV, BK, k), kmajor_desc(adO, BQ, k), id_s, k > 0);
-        }
-        ptx::umma_commit(&bar_s[bb]);
-      };
-      bool ok = ptx::mbar_wait(bar_kv, 0);
-      for (int j = 0; j < NSB && j < nq && ok; ++j) {
-        ok = ptx::mbar_wait(&full[j % NS], (j / NS) & 1);
-        if (ok) {
+          for (int k = 0; k < D / 16; ++k) {
+            ptx::umma_bf16(tmem + C::t_s(bb), kmajor_desc(aK, BK, k), kmajor_desc(aQ, BQ, k), id_s, k > 0);
+            ptx::umma_bf16(tmem + C::t_dp(bb), kmajor_desc(aV, BK, k), kmajor_desc(adO, BQ, k), id_s, k > 0);
+          }
+          ptx::umma_commit(&bar_s[bb]);
+        };
+        if (!ptx::mbar_wait(&bar_kv[kvb], (i / KVB) & 1)) { ok = false; break; }
+        for (int j = 0; j < NSB && j < nq; ++j) {
+          const int g = i * nq + j;
+          // head dim 128: the buffer's previous tile (an earlier unit's) has been drained
+          if (NSB == 2 && g >= NSB && !ptx::mbar_wait(&bar_dqfree[g % NSB], ((g - NSB) / NSB) & 1)) {
+            ok = false;
+            break;
+          }
+          if (!ptx::mbar_wait(&full[g % NS], (g / NS) & 1)) { ok = false; break; }
           ptx::tc_fence_after();
-          issue_s(j);
+          issue_s(g);
         }
-      }
-      for (int j = 0; j < nq && ok; ++j) {
-        const int st = j % NS, bb = j % NSB;
-        if (!ptx::mbar_wait(bar_p, j & 1)) { ok = false; break; }
-        ptx::tc_fence_after();
-        if constexpr (NSB == 1) {
-          // the single S^T / dP^T buffer is consumed: the next tile's products first
-          if (j + 1 < nq) {
-            if (!ptx::mbar_wait(&full[(j + 1) % NS], ((j + 1) / NS) & 1)) { ok = false; break; }
-            ptx::tc_fence_after();
-            issue_s(j + 1);
+        for (int j = 0; j < nq && ok; ++j) {
+          const int g = i * nq + j;
+          const int st = g % NS, bb = g % NSB;
+          if (!ptx::mbar_wait(bar_p, g & 1)) { ok = false; break; }
+          ptx::tc_fence_after();
+          if constexpr (NSB == 1) {
+            // the single S^T / dP^T buffer is consumed: the next tile's products first
+            if (j + 1 < nq) {
+              if (!ptx::mbar_wait(&full[(g + 1) % NS], ((g + 1) / NS) & 1)) { ok = false; break; }
+              ptx::tc_fence_after();
+              issue_s(g + 1);
+            }
           }
-        }
-        const uint32_t aQ = ptx::smem_u32(sQ + st * C::QT_BYTES), adO = ptx::smem_u32(sdO + st * C::QT_BYTES);
+          const uint32_t aQ = ptx::smem_u32(sQ + st * C::QT_BYTES), adO = ptx::smem_u32(sdO + st * C::QT_BYTES);
 #pragma unroll
-        for (int k = 0; k < BQ / 16; ++k) {
-          const uint32_t acc = (j > 0 || k > 0) ? 1u : 0u;
-          ptx::umma_bf16(tmem + C::T_DV, kmajor_desc(aP, BK, k), mnmajor_desc(adO, BQ * 128, k), id_acc, acc);
-          ptx::umma_bf16(tmem + C::T_DK, kmajor_desc(adS, BK, k), mnmajor_desc(aQ, BQ * 128, k), id_acc, acc);
-        }
-        if constexpr (NSB == 1) {
-          if (j > 0) {  // the dQ warps have read the previous tile's dQ
-            if (!ptx::mbar_wait(&bar_dqfree[0], (j - 1) & 1)) { ok = false; break; }
-            ptx::tc_fence_after();
+          for (int k = 0; k < BQ / 16; ++k) {
+            const uint32_t acc = (j > 0 || k > 0) ? 1u : 0u;
+            ptx::umma_bf16(tmem + C::T_DV, kmajor_desc(aP, BK, k), mnmajor_desc(adO, BQ * 128, k), id_acc, acc);
+            ptx::umma_bf16(tmem + C::T_DK, kmajor_desc(adS, BK, k), mnmajor_desc(aQ, BQ * 128, k), id_acc, acc);
           }
-        }
+          if constexpr (NSB == 1) {
+            if (g > 0) {  // the dQ warps have read the previous tile's dQ
+              if (!ptx::mbar_wait(&bar_dqfree[0], (g - 1) & 1)) { ok = false; break; }
+              ptx::tc_fence_after();
+            }
+          }
 #pragma unroll
-        for (int k = 0; k < BK / 16; ++k) {
-          if constexpr (C::DQT)  // dQ^T[d][q] = sum_key K[key][d] dS^T[key][q], over this tile's S^T
-            ptx::umma_bf16(tmem + C::t_dq(bb), mnmajor_desc(aK, BK * 128, k), mnmajor_desc(adS, BK * 128, k),
-                           id_dq, k > 0);
-          else  // dQ[q][d] = sum_key dS^T[key][q] K[key][d]
-            ptx::umma_bf16(tmem + C::t_dq(bb), mnmajor_desc(adS, BK * 128, k), mnmajor_desc(aK, BK * 128, k),
-                           id_dq, k > 0);
-        }
-        ptx::umma_commit(&bar_dq[bb]);
-        ptx::umma_commit(&empty[st]);
-        ptx::umma_commit(bar_pfree);
-        if constexpr (NSB == 2) {
-          // S^T, dP^T of tile j + 2 go into this buffer once the dQ warps have read dQ^T
-          if (j + 2 < nq) {
-            if (!ptx::mbar_wait(&bar_dqfree[bb], (j >> 1) & 1)) { ok = false; break; }
-            if (!ptx::mbar_wait(&full[(j + 2) % NS], ((j + 2) / NS) & 1)) { ok = false; break; }
-            ptx::tc_fence_after();
-            issue_s(j + 2);
+          for (int k = 0; k < BK / 16; ++k) {
+            if constexpr (C::DQT)  // dQ^T[d][q] = sum_key K[key][d] dS^T[key][q], over this tile's S^T
+              ptx::umma_bf16(tmem + C::t_dq(bb), mnmajor_desc(aK, BK * 128, k), mnmajor_desc(adS, BK * 128, k),
+                             id_dq, k > 0);
+            else  // dQ[q][d] = sum_key dS^T[key][q] K[key][d]
+              ptx::umma_bf16(tmem + C::t_dq(bb), mnmajor_desc(adS, BK * 128, k), mnmajor_desc(aK, BK * 128, k),
+                             id_dq, k > 0);
+          }
+          ptx::umma_commit(&bar_dq[bb]);
+          ptx::umma_commit(&empty[st]);
+          ptx::umma_commit(bar_pfree);
+          if constexpr (NSB == 2) {
+            // S^T, dP^T of tile g + 2 go into this buffer once the dQ warps have read dQ^T
+            if (j + 2 < nq) {
+              if (!ptx::mbar_wait(&bar_dqfree[bb], (g / NSB) & 1)) { ok = false; break; }
+              if (!ptx::mbar_wait(&full[(g + 2) % NS], ((g + 2) / NS) & 1)) { ok = false; break; }
+              ptx::tc_fence_after();
+              issue_s(g + 2);
+            }
           }
         }
+        ptx::umma_commit(&kv_free[kvb]);
+        ptx::umma_commit(bar_fin);
       }
       if (!ok) abort_flag = 1;
-      ptx::umma_commit(bar_fin);
     }
   } else if (warp < 10) {
     // ---------------------------------------------------------------- P / dS, then dK, dV
@@ -325,39 +369,47 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
     const int c0 = half * CW;           // this warp's query columns
     const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
     bool ok = true;
-    for (int j = 0; j < nq; ++j) {
-      const int st = j % NS, bb = j % NSB;
-      ok = ptx::mbar_wait(&bar_s[bb], (j / NSB) & 1) && ptx::mbar_wait(&full[st], (j / NS) & 1);
-      ok = __all_sync(0xffffffffu, ok);
-      if (!ok || abort_flag) { abort_flag = 1; break; }
-      ptx::tc_fence_after();
-      const float* lse = sLse + st * BQ + c0;
-      const float* rd = sRd + st * BQ + c0;
-      uint32_t hp[CW / 2], hd[CW / 2];
+    int i = 0;
+    for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++i) {
+      int k0, b, h;
+      unit_of(u, k0, b, h);
+      for (int j = 0; j < nq; ++j) {
+        const int g = i * nq + j;
+        const int st = g % NS, bb = g % NSB;
+        ok = ptx::mbar_wait(&bar_s[bb], (g / NSB) & 1) && ptx::mbar_wait(&full[st], (g / NS) & 1);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok || abort_flag) { ok = false; abort_flag = 1; break; }
+        ptx::tc_fence_after();
+        const float* lse = sLse + st * BQ + c0;
+        const float* rd = sRd + st * BQ + c0;
+        uint32_t hp[CW / 2], hd[CW / 2];
 #pragma unroll
-      for (int c = 0; c < CW / 32; ++c) {
-        uint32_t rs[32], rp[32];
-        ptx::tmem_ld_32x32b_x32(trow + C::t_s(bb) + c0 + c * 32, rs);
-        ptx::tmem_ld_32x32b_x32(trow + C::t_dp(bb) + c0 + c * 32, rp);
-        ptx::tmem_ld_wait();
-        softmax32(rs, rp, lse + c * 32, rd + c * 32, p.scale, hp + c * 16, hd + c * 16);
-      }
-      ptx::tc_fence_before();
-      if (j > 0) ok = ptx::mbar_wait(bar_pfree, (j - 1) & 1);
-      ok = __all_sync(0xffffffffu, ok);
-      if (!ok || abort_flag) { abort_flag = 1; break; }
+        for (int c = 0; c < CW / 32; ++c) {
+          uint32_t rs[32], rp[32];
+          ptx::tmem_ld_32x32b_x32(trow + C::t_s(bb) + c0 + c * 32, rs);
+          ptx::tmem_ld_32x32b_x32(trow + C::t_dp(bb) + c0 + c * 32, rp);
+          ptx::tmem_ld_wait();
+          softmax32(rs, rp, lse + c * 32, rd + c * 32, p.scale, hp + c * 16, hd + c * 16);
+        }
+        ptx::tc_fence_before();
+        if (g > 0) ok = ptx::mbar_wait(bar_pfree, (g - 1) & 1);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok || abort_flag) { ok = false; abort_flag = 1; break; }
 #pragma unroll
-      for (int c = 0; c < CW / 32; ++c) {
-        st_row32_packed(sP, BK, r, c0 + c * 32, hp + c * 16);
-        st_row32_packed(sdS, BK, r, c0 + c * 32, hd + c * 16);
+        for (int c = 0; c < CW / 32; ++c) {
+          st_row32_packed(sP, BK, r, c0 + c * 32, hp + c * 16);
+          st_row32_packed(sdS, BK, r, c0 + c * 32, hd + c * 16);
+        }
+        ptx::fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(bar_p);
       }
-      ptx::fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) ptx::mbar_arrive(bar_p);
-    }
-    ok = ok && ptx::mbar_wait(bar_fin, 0);
-    ok = __all_sync(0xffffffffu, ok);
-    if (ok) {
+      if (!ok) break;
+      // the unit's dK, dV; the next unit's first dV, dK products are issued only after
+      // these warps' next P arrival, i.e. after these reads
+      ok = ptx::mbar_wait(bar_fin, i & 1);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) { abort_flag = 1; break; }
       ptx::tc_fence_after();
       const int key = k0 + r;
 #pragma unroll 1
@@ -370,72 +422,79 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
           bf16* dv = static_cast<bf16*>(p.dv.base(key)) + p.dv.off(b, key, N, p.dv_col0 + h * D + c * 32);
           bf16* dk = static_cast<bf16*>(p.dk.base(key)) + p.dk.off(b, key, N, p.dk_col0 + h * D + c * 32);
 #pragma unroll
-          for (int u = 0; u < 4; ++u) {
+          for (int v = 0; v < 4; ++v) {
             uint4 a, bb;
             __nv_bfloat162* ha = reinterpret_cast<__nv_bfloat162*>(&a);
             __nv_bfloat162* hb = reinterpret_cast<__nv_bfloat162*>(&bb);
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              ha[i] = __floats2bfloat162_rn(__uint_as_float(rv[8 * u + 2 * i]), __uint_as_float(rv[8 * u + 2 * i + 1]));
-              hb[i] = __floats2bfloat162_rn(__uint_as_float(rk[8 * u + 2 * i]) * p.scale,
-                                            __uint_as_float(rk[8 * u + 2 * i + 1]) * p.scale);
+            for (int t = 0; t < 4; ++t) {
+              ha[t] = __floats2bfloat162_rn(__uint_as_float(rv[8 * v + 2 * t]), __uint_as_float(rv[8 * v + 2 * t + 1]));
+              hb[t] = __floats2bfloat162_rn(__uint_as_float(rk[8 * v + 2 * t]) * p.scale,
+                                            __uint_as_float(rk[8 * v + 2 * t + 1]) * p.scale);
             }
-            *reinterpret_cast<uint4*>(dv + 8 * u) = a;
-            *reinterpret_cast<uint4*>(dk + 8 * u) = bb;
+            *reinterpret_cast<uint4*>(dv + 8 * v) = a;
+            *reinterpret_cast<uint4*>(dk + 8 * v) = bb;
           }
         }
       }
-    } else {
-      abort_flag = 1;
+      ptx::tc_fence_before();
     }
   } else {
     // ---------------------------------------------------------------- dQ -> f32 reduce-add
     const int quarter = warp & 3;
     const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
     uint8_t* stg = sDQ + quarter * C::DQ_WARP_BYTES;
-    for (int j = 0; j < nq; ++j) {
-      const int bb = j % NSB;
-      bool ok = ptx::mbar_wait(&bar_dq[bb], (j / NSB) & 1);
-      ok = __all_sync(0xffffffffu, ok);
-      if (!ok || abort_flag) { abort_flag = 1; break; }
-      ptx::tc_fence_after();
-      uint32_t rq[64];
-      ptx::tmem_ld_32x32b_x32(trow + C::t_dq(bb), *reinterpret_cast<uint32_t(*)[32]>(rq));
-      ptx::tmem_ld_32x32b_x32(trow + C::t_dq(bb) + 32, *reinterpret_cast<uint32_t(*)[32]>(rq + 32));
-      ptx::tmem_ld_wait();
-      ptx::tc_fence_before();
-      __syncwarp();
-      if (lane == 0) ptx::mbar_arrive(&bar_dqfree[bb]);
-      const int q0 = j * BQ;
-      // two 32 x 32 boxes through one staging box: dQ^T (lane = head dim, columns = the
-      // tile's 64 queries: box rows = queries) or dQ (lane = query, columns = 64 head dims)
-#pragma unroll
-      for (int hh = 0; hh < 2; ++hh) {
-        if (lane == 0) ptx::bulk_wait_read<0>();
+    bool ok = true;
+    int i = 0;
+    for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++i) {
+      int k0, b, h;
+      unit_of(u, k0, b, h);
+      (void)k0;
+      for (int j = 0; j < nq; ++j) {
+        const int g = i * nq + j;
+        const int bb = g % NSB;
+        ok = ptx::mbar_wait(&bar_dq[bb], (g / NSB) & 1);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok || abort_flag) { ok = false; abort_flag = 1; break; }
+        ptx::tc_fence_after();
+        uint32_t rq[64];
+        ptx::tmem_ld_32x32b_x32(trow + C::t_dq(bb), *reinterpret_cast<uint32_t(*)[32]>(rq));
+        ptx::tmem_ld_32x32b_x32(trow + C::t_dq(bb) + 32, *reinterpret_cast<uint32_t(*)[32]>(rq + 32));
+        ptx::tmem_ld_wait();
+        ptx::tc_fence_before();
         __syncwarp();
-        if constexpr (C::DQT) {
+        if (lane == 0) ptx::mbar_arrive(&bar_dqfree[bb]);
+        const int q0 = j * BQ;
+        // two 32 x 32 boxes through one staging box: dQ^T (lane = head dim, columns = the
+        // tile's 64 queries: box rows = queries) or dQ (lane = query, columns = 64 head dims)
 #pragma unroll
-          for (int q = 0; q < 32; ++q)
-            *reinterpret_cast<float*>(stg + q * 128 + (((lane >> 2) ^ (q & 7)) << 4) + (lane & 3) * 4) =
-                __uint_as_float(rq[hh * 32 + q]) * p.scale;
-        } else {
-          uint8_t* row = stg + lane * 128;
+        for (int hh = 0; hh < 2; ++hh) {
+          if (lane == 0) ptx::bulk_wait_read<0>();
+          __syncwarp();
+          if constexpr (C::DQT) {
 #pragma unroll
-          for (int u = 0; u < 8; ++u)
-            *reinterpret_cast<float4*>(row + ((u ^ (lane & 7)) << 4)) =
-                make_float4(__uint_as_float(rq[hh * 32 + 4 * u]) * p.scale,
-                            __uint_as_float(rq[hh * 32 + 4 * u + 1]) * p.scale,
-                            __uint_as_float(rq[hh * 32 + 4 * u + 2]) * p.scale,
-                            __uint_as_float(rq[hh * 32 + 4 * u + 3]) * p.scale);
-        }
-        ptx::fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) {
-          const int col = C::DQT ? h * D + quarter * 32 : h * D + hh * 32;
-          const int row = C::DQT ? q0 + hh * 32 : q0 + quarter * 32;
-          if (row < N) {
-            ptx::tma_reduce_add_3d(&maps.dq, stg, col, row, b);
-            ptx::bulk_commit();
+            for (int q = 0; q < 32; ++q)
+              *reinterpret_cast<float*>(stg + q * 128 + (((lane >> 2) ^ (q & 7)) << 4) + (lane & 3) * 4) =
+                  __uint_as_float(rq[hh * 32 + q]) * p.scale;
+          } else {
+            uint8_t* row = stg + lane * 128;
+#pragma unroll
+            for (int v = 0; v < 8; ++v)
+              *reinterpret_cast<float4*>(row + ((v ^ (lane & 7)) << 4)) =
+                  make_float4(__uint_as_float(rq[hh * 32 + 4 * v]) * p.scale,
+                              __uint_as_float(rq[hh * 32 + 4 * v + 1]) * p.scale,
+                              __uint_as_float(rq[hh * 32 + 4 * v + 2]) * p.scale,
+                              __uint_as_float(rq[hh * 32 + 4 * v + 3]) * p.scale);
+          }
+          ptx::fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            const int col = C::DQT ? h * D + quarter * 32 : h * D + hh * 32;
+            const int row = C::DQT ? q0 + hh * 32 : q0 + quarter * 32;
+            if (row < N) {
+              ptx::tma_reduce_add_3d(&maps.dq, stg, col, row, b);
+              ptx::bulk_commit();
+            }
           }
         }
       }
@@ -501,8 +560,9 @@ int launch(const AttnBwdArgs& a, cudaStream_t s) {
     JAGG_CUDA_TRY(cudaFuncSetAttribute(fa_bwd_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
     attr = true;
   }
-  dim3 grid(ceil_div(N, C::BK), f.B * f.heads);
-  fa_bwd_tc_kernel<D><<<grid, FB_THREADS, C::SMEM, s>>>(maps, p);
+  const int units = ceil_div(N, C::BK) * f.B * f.heads;
+  const int nsm = sm_count();
+  fa_bwd_tc_kernel<D><<<units < nsm ? units : nsm, FB_THREADS, C::SMEM, s>>>(maps, p);
   JAGG_LAUNCHED();
   return JAGG_OK;
 }
