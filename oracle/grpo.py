@@ -114,6 +114,35 @@ def aggregate(s, t_window):
     return np.concatenate([base, corr], axis=0)
 
 
+def aggregate_span(s, t_steps, t_first, t_last):
+    """Eq. s_base_corr restricted to some of a window's steps, with alpha taken against the
+    window's own endpoint times (Eq. alpha): alpha_j = (t_first - t_j) / (t_first - t_last).
+
+    The sequential-graph variant (Sec. 3.4, Algorithm 2) forms s_base from steps 0 .. W-2
+    before step W-1 is computed (alpha_{W-1} = 1 contributes nothing to s_base) and adds
+    the last step to s_corr later (alpha_0 = 0 contributes nothing to s_corr).
+    s [G, n, D] -> [2G, D] partial sums (rows 0..G-1 base, G..2G-1 corr)."""
+    s = np.asarray(s, np.float64)
+    G, n, D = s.shape
+    t = np.asarray(t_steps, np.float64)
+    al = (t_first - t) / (t_first - t_last)
+    base = np.zeros((G, D))
+    corr = np.zeros((G, D))
+    for j in range(n):
+        base += (1.0 - al[j]) * s[:, j]
+        corr += al[j] * s[:, j]
+    return np.concatenate([base, corr], axis=0)
+
+
+def aggregate_ablate(s):
+    """The endpoint-only ablation of Sec. 4: only s_0 and s_{W-1} are kept and each is
+    back-propagated through its own endpoint with weight 1 (the intermediate steps are
+    discarded and no t-weighting is applied).  s [G, W, D] -> [2G, D]: rows 0..G-1 = s_0,
+    rows G..2G-1 = s_{W-1}."""
+    s = np.asarray(s, np.float64)
+    return np.concatenate([s[:, 0], s[:, -1]], axis=0)
+
+
 def route_schedule(n_windows, jagg_frac):
     """jagg_frac routing (Sec. 3.3, "High-noise vs. low-noise scheduling"): the first
     floor(jagg_frac n + 1e-9) windows (highest noise first) take JAGG."""

@@ -142,3 +142,42 @@ def test_grad_stats_against_numpy():
     assert cos == pytest.approx(np.dot(a, b) / np.linalg.norm(a) / np.linalg.norm(b))
     assert rho == pytest.approx(np.linalg.norm(a) / np.linalg.norm(b))
     assert grpo.grad_stats(a, 2 * a)[3] == pytest.approx(1.0)
+
+
+def test_span_aggregation_reassembles_the_window():
+    """Spans of a window's steps, each with alpha against the window's endpoint times, add up
+    to the whole-window aggregation; the sequential-graph split (steps 0..W-2 before the
+    last step is known, then the last step alone) in particular."""
+    rng = np.random.Generator(np.random.PCG64(81))
+    G, W, D = 3, 5, 7
+    s = rng.standard_normal((G, W, D))
+    t = synth.time_grid(20, 3.0)[6:6 + W]
+    full = grpo.aggregate(s, t)
+    np.testing.assert_allclose(grpo.aggregate_span(s, t, t[0], t[-1]), full, atol=1e-14)
+    first = grpo.aggregate_span(s[:, :-1], t[:-1], t[0], t[-1])
+    last = grpo.aggregate_span(s[:, -1:], t[-1:], t[0], t[-1])
+    np.testing.assert_allclose(first + last, full, atol=1e-14)
+    # the last step adds only to the correction rows, the first only to the base rows
+    np.testing.assert_array_equal(last[:G], 0.0)
+    np.testing.assert_array_equal(grpo.aggregate_span(s[:, :1], t[:1], t[0], t[-1])[G:], 0.0)
+    # any partition of the steps works
+    parts = [grpo.aggregate_span(s[:, a:b], t[a:b], t[0], t[-1]) for a, b in ((0, 2), (2, 3), (3, 5))]
+    np.testing.assert_allclose(sum(parts), full, atol=1e-14)
+
+
+def test_ablation_keeps_the_endpoint_signals():
+    """The endpoint-only ablation: s_0 and s_{W-1} unweighted; it coincides with JAGG exactly
+    when the window has no middle steps (W = 2), and equals the span aggregation over the
+    two endpoint steps."""
+    rng = np.random.Generator(np.random.PCG64(82))
+    G, W, D = 2, 4, 6
+    s = rng.standard_normal((G, W, D))
+    t = synth.time_grid(16, 3.0)[:W]
+    ab = grpo.aggregate_ablate(s)
+    np.testing.assert_array_equal(ab[:G], s[:, 0])
+    np.testing.assert_array_equal(ab[G:], s[:, -1])
+    np.testing.assert_array_equal(grpo.aggregate_ablate(s[:, :2]), grpo.aggregate(s[:, :2], t[:2]))
+    ends = np.stack([s[:, 0], s[:, -1]], axis=1)
+    np.testing.assert_allclose(grpo.aggregate_span(ends, [t[0], t[-1]], t[0], t[-1]), ab, atol=1e-15)
+    # with middle steps the two differ (the ablation discards s_1 .. s_{W-2})
+    assert np.abs(ab - grpo.aggregate(s, t)).max() > 1e-3

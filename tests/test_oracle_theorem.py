@@ -83,3 +83,39 @@ def test_w2_jagg_is_exact_for_the_dit():
     ge = path.window_gradient(model, zw, t_win, txt, s, jagg=False)
     for k in gj:
         np.testing.assert_allclose(gj[k], ge[k], rtol=1e-12, atol=1e-14)
+
+
+def test_sequential_graph_variant_equals_the_joint_backward():
+    """Algorithm 2 (Sec. 3.4): two VJPs of G rows, the first with s_base formed from steps
+    0..W-2 only, the second with s_corr completed by the last step, give the same
+    gradient as the joint backward over 2G rows (the VJP is linear in the rows)."""
+    rng = np.random.Generator(np.random.PCG64(19))
+    D, k, G, W = 12, 5, 3, 4
+    model = LinearVelocity(D, k, rng)
+    t_win = synth.time_grid(16, 3.0)[4:4 + W]
+    z = _affine_window(rng, t_win, D, G)
+    s = rng.standard_normal((G, W, D))
+    zr, tr = path.window_rows(z, t_win, jagg=True)
+    joint = model.vjp(zr, tr, grpo.aggregate(s, t_win))
+    part = grpo.aggregate_span(s[:, :-1], t_win[:-1], t_win[0], t_win[-1])
+    g0 = model.vjp(z[:, 0], np.full(G, t_win[0]), part[:G])
+    corr = part[G:] + grpo.aggregate_span(s[:, -1:], t_win[-1:], t_win[0], t_win[-1])[G:]
+    g1 = model.vjp(z[:, -1], np.full(G, t_win[-1]), corr)
+    assert np.linalg.norm(g0 + g1 - joint) <= 1e-12 * np.linalg.norm(joint)
+
+
+def test_ablation_is_not_exact_where_jagg_is():
+    """On the theorem's linear model with W > 2 the endpoint-only ablation misses the middle
+    steps' contribution (JAGG recovers it exactly); with W = 2 both are exact."""
+    rng = np.random.Generator(np.random.PCG64(20))
+    D, k, G = 12, 5, 3
+    model = LinearVelocity(D, k, rng)
+    for W, exact_expected in ((4, False), (2, True)):
+        t_win = synth.time_grid(16, 3.0)[4:4 + W]
+        z = _affine_window(rng, t_win, D, G)
+        s = rng.standard_normal((G, W, D))
+        exact = sum(model.vjp(z[:, j], np.full(G, t_win[j]), s[:, j]) for j in range(W))
+        zr, tr = path.window_rows(z, t_win, jagg=True)
+        ab = model.vjp(zr, tr, grpo.aggregate_ablate(s))
+        err = np.linalg.norm(ab - exact) / np.linalg.norm(exact)
+        assert (err <= 1e-10) == exact_expected, (W, err)
