@@ -8,6 +8,11 @@ Readings of passages the paper leaves open (each is also listed in the design doc):
   * log-prob: the isotropic Gaussian density of the whole latent, i.e. the normalising
     term is D * log(sqrt(2 pi) sigma_j) (it cancels in the ratio); the mean is the
     rectified-flow Euler step mu = z_j + v_j (t_{j+1} - t_j) exactly as Eq. logprob states;
+  * epsilon-prediction mean: Eq. logprob writes sigma_{t_j} both for the step's noise scale
+    and for the diffusion schedule inside the DDIM mean; the oracle keeps them apart (the
+    schedule (alpha_t, sigma_t) of z_t = alpha_t x + sigma_t eps enters the mean only, the
+    step's scale the density only), and takes the mean exactly as printed (the deterministic
+    DDIM step) whatever the step's noise scale;
   * PPO clip: the gradient follows the max() of Eq. grpo_loss: a step contributes zero
     only when the clipped branch is strictly larger (A > 0 and rho > 1 + eps, or A < 0 and
     rho < 1 - eps); at a tie the step counts as unclipped.  The remark after Phase 2
@@ -89,6 +94,71 @@ def step_signals(v_hat, z, t, sigma, logp_old, A, clip_eps, scale):
                 clipped[i, j] = 1
                 continue
             s[i, j] = scale * (-a) * rho * r * dt / sigma[j] ** 2
+    return s, logp, ratio, clipped
+
+
+def ddim_mean(z_cur, eps_hat, a_cur, a_next, s_cur, s_next):
+    """Eq. logprob, epsilon-prediction case: the mean of the transition is the deterministic
+    DDIM step of the schedule (alpha_t, sigma_t) of z_t = alpha_t x + sigma_t eps,
+        mu = alpha_{t_{j+1}} (z_j / alpha_{t_j} - (sigma_{t_j} / alpha_{t_j}
+                                                   - sigma_{t_{j+1}} / alpha_{t_{j+1}}) eps_hat_j).
+    a_cur, a_next, s_cur, s_next are alpha_{t_j}, alpha_{t_{j+1}}, sigma_{t_j}, sigma_{t_{j+1}}
+    (schedule values, not the step's noise scale)."""
+    z_cur = np.asarray(z_cur, np.float64)
+    eps_hat = np.asarray(eps_hat, np.float64)
+    return a_next * (z_cur / a_cur - (s_cur / a_cur - s_next / a_next) * eps_hat)
+
+
+def step_logprob_eps(z_next, z_cur, eps_hat, a_cur, a_next, s_cur, s_next, sigma):
+    """Eq. logprob with the epsilon-prediction mean (ddim_mean); sigma is the step's noise
+    scale, as in step_logprob."""
+    z_next = np.asarray(z_next, np.float64).ravel()
+    mu = ddim_mean(z_cur, eps_hat, a_cur, a_next, s_cur, s_next).ravel()
+    D = z_next.size
+    return -((z_next - mu) ** 2).sum() / (2.0 * sigma ** 2) - D * math.log(math.sqrt(2.0 * math.pi) * sigma)
+
+
+def window_loss_eps(eps_hat, z, sched_alpha, sched_sigma, sigma, logp_old, A, clip_eps, scale):
+    """window_loss for an epsilon-prediction backbone.  eps_hat [W, D], z [W+1, D],
+    sched_alpha / sched_sigma [W+1] = alpha_{t_j}, sigma_{t_j} at the window's times."""
+    al, sg = sched_alpha, sched_sigma
+    total = 0.0
+    for j in range(eps_hat.shape[0]):
+        lp = step_logprob_eps(z[j + 1], z[j], eps_hat[j], al[j], al[j + 1], sg[j], sg[j + 1], sigma[j])
+        total += ppo_step_loss(A, math.exp(lp - logp_old[j]), clip_eps)
+    return scale * total
+
+
+def step_signals_eps(eps_hat, z, sched_alpha, sched_sigma, sigma, logp_old, A, clip_eps, scale):
+    """Phase 2 for an epsilon-prediction backbone: s_ij = dL_ij / d eps_hat_ij (Sec. 3.3,
+    Phase 2; Eq. logprob, epsilon case; Eq. grpo_loss).  Shapes as step_signals, with
+    sched_alpha / sched_sigma [W+1] in place of t.
+
+    mu is affine in eps_hat with slope c_j = -alpha_{t_{j+1}} (sigma_{t_j} / alpha_{t_j}
+    - sigma_{t_{j+1}} / alpha_{t_{j+1}}), so d logp / d eps_hat = (z_{j+1} - mu) c_j / sigma_j^2
+    and the unclipped branch -A rho has gradient -A rho (z_{j+1} - mu) c_j / sigma_j^2."""
+    eps_hat = np.asarray(eps_hat, np.float64)
+    z = np.asarray(z, np.float64)
+    al = np.asarray(sched_alpha, np.float64)
+    sg = np.asarray(sched_sigma, np.float64)
+    G, W, D = eps_hat.shape
+    s = np.zeros((G, W, D))
+    logp = np.zeros((G, W))
+    ratio = np.zeros((G, W))
+    clipped = np.zeros((G, W), np.uint8)
+    for i in range(G):
+        for j in range(W):
+            mu = ddim_mean(z[i, j], eps_hat[i, j], al[j], al[j + 1], sg[j], sg[j + 1])
+            c = -al[j + 1] * (sg[j] / al[j] - sg[j + 1] / al[j + 1])
+            logp[i, j] = step_logprob_eps(z[i, j + 1], z[i, j], eps_hat[i, j], al[j], al[j + 1], sg[j], sg[j + 1],
+                                          sigma[j])
+            rho = math.exp(logp[i, j] - logp_old[i, j])
+            ratio[i, j] = rho
+            a = A[i]
+            if (a > 0 and rho > 1.0 + clip_eps) or (a < 0 and rho < 1.0 - clip_eps):
+                clipped[i, j] = 1
+                continue
+            s[i, j] = scale * (-a) * rho * (z[i, j + 1] - mu) * c / sigma[j] ** 2
     return s, logp, ratio, clipped
 
 

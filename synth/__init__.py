@@ -228,6 +228,13 @@ def sigma_schedule(t: np.ndarray, eta: float) -> np.ndarray:
     return eta * np.sqrt(np.abs(np.diff(t)))
 
 
+def vp_schedule(t: np.ndarray):
+    """A variance-preserving diffusion schedule (alpha_t, sigma_t) = (cos(pi t / 2),
+    sin(pi t / 2)) at the times t, for epsilon-prediction inputs."""
+    t = np.asarray(t, np.float64)
+    return np.cos(0.5 * np.pi * t), np.sin(0.5 * np.pi * t)
+
+
 # ----------------------------------------------------------------------------------
 # Random draws.
 # ----------------------------------------------------------------------------------

@@ -181,3 +181,93 @@ def test_ablation_keeps_the_endpoint_signals():
     np.testing.assert_allclose(grpo.aggregate_span(ends, [t[0], t[-1]], t[0], t[-1]), ab, atol=1e-15)
     # with middle steps the two differ (the ablation discards s_1 .. s_{W-2})
     assert np.abs(ab - grpo.aggregate(s, t)).max() > 1e-3
+
+
+# ------------------------------------------------------------------ epsilon-prediction mean
+def _eps_case(seed, G=3, W=3, D=6):
+    rng = np.random.Generator(np.random.PCG64(seed))
+    t = synth.time_grid(W, shift=3.0) * 0.9 + 0.05     # keep alpha_t, sigma_t away from 0
+    al, sg = synth.vp_schedule(t)
+    sig = synth.sigma_schedule(t, 0.7)
+    z = rng.standard_normal((G, W + 1, D))
+    e = rng.standard_normal((G, W, D))
+    return t, al, sg, sig, z, e
+
+
+def test_ddim_mean_on_the_flow_schedule_is_the_euler_step():
+    """With alpha_t = 1 - t, sigma_t = t (the rectified-flow interpolation) the epsilon
+    model eps_hat is the velocity model v_hat = (eps_hat - z) / (1 - t): the DDIM mean then
+    equals the Euler step z + v_hat (t_{j+1} - t_j), and the step log-probs agree."""
+    rng = np.random.Generator(np.random.PCG64(90))
+    D = 23
+    z, zn, e = rng.standard_normal((3, D))
+    t0, t1, sig = 0.8, 0.7375, 0.31
+    v = (e - z) / (1.0 - t0)
+    np.testing.assert_allclose(grpo.ddim_mean(z, e, 1 - t0, 1 - t1, t0, t1), z + v * (t1 - t0), rtol=1e-12,
+                               atol=1e-14)
+    assert grpo.step_logprob_eps(zn, z, e, 1 - t0, 1 - t1, t0, t1, sig) == pytest.approx(
+        grpo.step_logprob(zn, z, v, t0, t1, sig), rel=1e-13)
+
+
+def test_eps_signals_follow_the_chain_rule_through_the_flow_signals():
+    """On the rectified-flow schedule d v_hat / d eps_hat = 1 / (1 - t_j), so the epsilon
+    signals are the (independently pinned) velocity signals divided by 1 - t_j, with the
+    same log-probs, ratios and clip decisions."""
+    rng = np.random.Generator(np.random.PCG64(91))
+    G, W, D = 3, 4, 9
+    t = synth.time_grid(W, shift=3.0) * 0.9 + 0.05
+    sig = synth.sigma_schedule(t, 0.7)
+    z = rng.standard_normal((G, W + 1, D))
+    e = rng.standard_normal((G, W, D))
+    v = (e - z[:, :W]) / (1.0 - t[:W])[None, :, None]
+    lp = np.array([[grpo.step_logprob(z[i, j + 1], z[i, j], v[i, j], t[j], t[j + 1], sig[j]) for j in range(W)]
+                   for i in range(G)])
+    lpo = lp + rng.uniform(-0.3, 0.3, size=(G, W))
+    A = np.array([1.3, -0.7, 0.4])
+    sv, lv, rv, cv = grpo.step_signals(v, z, t, sig, lpo, A, 0.1, 0.37)
+    se, le, re_, ce = grpo.step_signals_eps(e, z, 1.0 - t, t, sig, lpo, A, 0.1, 0.37)
+    np.testing.assert_allclose(le, lv, rtol=1e-12)
+    np.testing.assert_allclose(re_, rv, rtol=1e-10)
+    np.testing.assert_array_equal(ce, cv)
+    np.testing.assert_allclose(se, sv / (1.0 - t[:W])[None, :, None], rtol=1e-9, atol=1e-15)
+    assert ce.any() and not ce.all()
+
+
+def test_ddim_mean_recovers_the_noised_sample():
+    """For z_j = alpha_j x + sigma_j eps and the true noise eps_hat = eps, the DDIM mean is the
+    same sample noised to the next time: alpha_{j+1} x + sigma_{j+1} eps (variance-preserving
+    and variance-exploding schedules)."""
+    rng = np.random.Generator(np.random.PCG64(92))
+    x, eps = rng.standard_normal((2, 31))
+    t = np.array([0.9, 0.55])
+    al, sg = synth.vp_schedule(t)
+    for a, s in ((al, sg), (np.ones(2), np.array([4.0, 1.5]))):
+        z = a[0] * x + s[0] * eps
+        np.testing.assert_allclose(grpo.ddim_mean(z, eps, a[0], a[1], s[0], s[1]), a[1] * x + s[1] * eps,
+                                   rtol=1e-12, atol=1e-13)
+
+
+@pytest.mark.parametrize("seed", [93, 94])
+def test_eps_signals_are_the_gradient_of_the_window_loss(seed):
+    """s_ij equals the central difference of the epsilon window loss in eps_hat_ij."""
+    clip, scale = 0.1, 0.37
+    t, al, sg, sig, z, e = _eps_case(seed)
+    G, W, D = e.shape
+    lp = np.array([[grpo.step_logprob_eps(z[i, j + 1], z[i, j], e[i, j], al[j], al[j + 1], sg[j], sg[j + 1], sig[j])
+                    for j in range(W)] for i in range(G)])
+    rng = np.random.Generator(np.random.PCG64(seed + 100))
+    lpo = lp + rng.uniform(-0.3, 0.3, size=(G, W))
+    A = np.array([1.3, -0.7, 0.4])
+    s, _, ratio, clipped = grpo.step_signals_eps(e, z, al, sg, sig, lpo, A, clip, scale)
+    h = 1e-6
+    for i in range(G):
+        for j in range(W):
+            if abs(abs(ratio[i, j] - 1.0) - clip) < 1e-4:
+                continue
+            for k in range(D):
+                ep = e[i].copy(); ep[j, k] += h
+                em = e[i].copy(); em[j, k] -= h
+                fd = (grpo.window_loss_eps(ep, z[i], al, sg, sig, lpo[i], A[i], clip, scale)
+                      - grpo.window_loss_eps(em, z[i], al, sg, sig, lpo[i], A[i], clip, scale)) / (2 * h)
+                assert fd == pytest.approx(s[i, j, k], rel=1e-6, abs=1e-9)
+    assert clipped.any() and not clipped.all()
