@@ -485,6 +485,77 @@ def measure(b, routes, batched, args, ws, use_graph, profile=False):
     return res
 
 
+def graph_variants(b, args, ws, use_graph):
+    """The sequential-graph variant (Algorithm 2: per window, endpoint 0 forward into one
+    G-row arena, its VJP, endpoint W-1 forward into the same arena, its VJP) against the
+    joint variant (one 2G-row forward and VJP per window), same scope: the endpoint forwards
+    with saves and the VJPs, on the cotangents of the JAGG step (signals excluded, they are
+    the same for both)."""
+    jg, wl, dev = b.jg, b.wl, b.dev
+    G, W = wl.G, wl.W
+    rows = [b.rows(b.z[:, w * W:(w + 1) * W].reshape(G, W, *b.shape), w, True) for w in range(b.nw)]
+    txt1, txt2 = b.txt_rows(G), b.txt_rows(2 * G)
+    arena = jg.alloc_bytes(b.model.saved_bytes(G), dev)
+    v1 = torch.empty(G, *b.shape, dtype=b.tdt, device=dev)
+
+    def sequential():
+        for w, (z, t) in enumerate(rows):
+            for e in range(2):
+                sl = slice(e * G, (e + 1) * G)
+                jg.dit_forward_save(b.model, z[sl], t[sl], txt1, v1, saved=arena, ws=b.ws)
+                jg.dit_joint_vjp(b.model, arena, G, b.cot_all[w * 2 * G + e * G:w * 2 * G + (e + 1) * G], b.grad,
+                                 b.ws)
+    ms_s, graph = time_steps(sequential, args.steps, args.warmup, ws, use_graph)
+    del graph
+    seq_gb = arena.numel() / 1e9
+    del arena
+    torch.cuda.empty_cache()
+    arena2 = jg.alloc_bytes(b.model.saved_bytes(2 * G), dev)
+    v2 = torch.empty(2 * G, *b.shape, dtype=b.tdt, device=dev)
+
+    def joint():
+        for w, (z, t) in enumerate(rows):
+            jg.dit_forward_save(b.model, z, t, txt2, v2, saved=arena2, ws=b.ws)
+            jg.dit_joint_vjp(b.model, arena2, 2 * G, b.cot_all[w * 2 * G:(w + 1) * 2 * G], b.grad, b.ws)
+    ms_j, graph = time_steps(joint, args.steps, args.warmup, ws, use_graph)
+    del graph
+    joint_gb = arena2.numel() / 1e9
+    del arena2
+    torch.cuda.empty_cache()
+    units = wl.G * wl.T
+    return {"sequential": {"value": ws * units / (ms_s / 1000.0), "unit": UNIT, "ms_per_step": max_over_ranks(ms_s, ws),
+                           "saved_gb": seq_gb},
+            "joint": {"value": ws * units / (ms_j / 1000.0), "unit": UNIT, "ms_per_step": max_over_ranks(ms_j, ws),
+                      "saved_gb": joint_gb},
+            "scope": "per window: endpoint forwards with saves + VJPs on the JAGG cotangents (signals excluded)"}
+
+
+def ablate_step(b, args, ws, use_graph):
+    """The endpoint-only ablation (Sec. 4): per window the step signals, then s_0 and s_{W-1}
+    read in place as the two cotangent rows (no t-weighting), then the joint VJP over every
+    window's endpoint rows -- the headline step with the aggregation swapped."""
+    jg, wl, dev = b.jg, b.wl, b.dev
+    G, W, D = wl.G, wl.W, b.D
+    arenas = b.forward_saves([1] * b.nw, batched=True)
+    s_win = torch.empty(G, W, D, dtype=torch.float32, device=dev)
+
+    def step():
+        for w in range(b.nw):
+            b.signals(w, b.lpo_win[w], s_out=s_win)
+            tw = b.t_dev[w * W:(w + 1) * W]
+            cot = b.cot_all[w * 2 * G:(w + 1) * 2 * G]
+            t0, t1 = float(b.t[w * W]), float(b.t[w * W + W - 1])
+            jg.jagg_aggregate_span(s_win, tw[:1], t0, t1, cot, steps=(0, 1))
+            jg.jagg_aggregate_span(s_win, tw[W - 1:], t0, t1, cot, accumulate=True, steps=(W - 1, 1))
+        saved, B, _ = arenas[0]
+        jg.dit_joint_vjp(b.model, saved, B, b.cot_all[:B], b.grad, b.ws)
+        jg.grad_reduce(b.grad, None, out3=b.out3, ws=b.gws)
+    ms, graph = time_steps(step, args.steps, args.warmup, ws, use_graph)
+    del graph, arenas
+    torch.cuda.empty_cache()
+    return {"value": ws * wl.G * wl.T / (ms / 1000.0), "unit": UNIT, "ms_per_step": max_over_ranks(ms, ws)}
+
+
 def run_gpu(args, ws, rank):
     import paper_2607_17572_gb300 as jg
     dev = torch.device("cuda", torch.cuda.current_device())
@@ -549,6 +620,9 @@ def run_gpu(args, ws, rank):
         out["jagg_speedup_vs_full_w"] = rf["ms"] / ms
         out["ideal_speedup"] = wl.W / 2
         torch.cuda.empty_cache()
+        if batched:
+            out["graph_variants"] = graph_variants(b, args, ws, use_graph)
+            out["ablate"] = ablate_step(b, args, ws, use_graph)
         if not args.no_e2e and batched:
             out["e2e"] = run_e2e(b, args, ws, routes)
         # the float64 oracle needs minutes per sequence at MMDiT width: DiT workloads only

@@ -8,6 +8,7 @@
  *
  *   dit_forward_save   Phase 1: v = DiT(z, t, txt), keeping what Phase 4 needs
  *   grpo_step_signals  Phase 2: s_j = dL_j/dv_j through Eq. logprob and Eq. grpo_loss
+ *                      (grpo_step_signals_eps: the same for an epsilon-prediction model)
  *   jagg_aggregate     Phase 3: Eq. alpha and Eq. s_base_corr
  *   jagg_route         jagg_frac routing (Sec. 3.3 and the gradient-quality appendix)
  *   dit_joint_vjp      Phase 4: grad += sum_rows J(z_row, t_row)^T cot_row
@@ -195,6 +196,27 @@ int grpo_step_signals(const void* v_hat, int v_dtype, const float* z, const doub
                       double* logp_new, double* ratio, uint8_t* clipped, double* adv_out,
                       void* ws, size_t ws_bytes, cudaStream_t stream);
 
+/* Phase 2 for an epsilon-prediction backbone (Eq. logprob, epsilon case): the transition
+ * mean is the deterministic DDIM step of the diffusion schedule (alpha_t, sigma_t),
+ *   mu_ij = alpha_{j+1} (z_{i,j} / alpha_j - (sigma_j / alpha_j - sigma_{j+1} / alpha_{j+1}) eps_ij)
+ *         = a_j z_{i,j} + c_j eps_ij,
+ * and every other quantity is as in grpo_step_signals with r_ij = z_{i,j+1} - mu_ij and
+ *   s_ij = scale * (-A_i) rho r_ij c_j / sigma_j^2 (0 when clipped),
+ * the derivative with respect to the model output eps_ij.  The schedule's sigma_t is the noise
+ * level of z_t = alpha_t x + sigma_t eps; sigma (the step's noise scale) enters the density
+ * only.  t is used for the aggregation weights alone (cot_out).
+ *   eps_hat      device [G, W, D] (eps_dtype)   noise predictions of the window's steps
+ *   sched_alpha  device [W+1] f64 alpha_t at t_0 .. t_W, all > 0 (checked on device: otherwise
+ *                JAGG_DEV_STATUS_BADARG is set and the outputs are meaningless)
+ *   sched_sigma  device [W+1] f64 sigma_t at t_0 .. t_W
+ * Workspace: jagg_signals_workspace_bytes(G, W, D), as for grpo_step_signals.           */
+int grpo_step_signals_eps(const void* eps_hat, int eps_dtype, const float* z, const double* t,
+                          const double* sched_alpha, const double* sched_sigma, const double* sigma,
+                          const double* logp_old, const float* rewards, int G, int W, int64_t D,
+                          double clip_eps, double adv_clip, double adv_eps, double scale, float* s_out,
+                          float* cot_out, double* logp_new, double* ratio, uint8_t* clipped,
+                          double* adv_out, void* ws, size_t ws_bytes, cudaStream_t stream);
+
 /* grpo_step_signals for callers that cannot allocate device memory (no counterpart in the
  * paper: an interface convenience of this library).  Some callers have no way to obtain a
  * workspace: code that runs where cudaMalloc is not allowed or not wanted, such as an
@@ -226,6 +248,23 @@ int grpo_step_signals_static(const void* v_hat, int v_dtype, const float* z, con
  *   a zero denominator sets JAGG_DEV_STATUS_BADARG and writes zeros).                */
 int jagg_aggregate(const float* s, const double* t_window, int G, int W, int64_t D,
                    float* cot, cudaStream_t stream);
+
+/* Phase 3 over a span of a window's steps, alpha taken against the window's endpoint times
+ * (Eq. alpha, Eq. s_base_corr): alpha_j = (t_first - t_j) / (t_first - t_last),
+ *   cot[i]     (+)= sum_j (1 - alpha_j) s[i, j]
+ *   cot[G + i] (+)= sum_j alpha_j s[i, j]          over the n steps given.
+ * Serves the sequential-graph variant (Sec. 3.4, Algorithm 2: s_base from steps 0..W-2 is
+ * complete before the last step's forward, whose s_{W-1} then adds to s_corr alone) and the
+ * endpoint-only ablation of Sec. 4 (the span {0, W-1} with t_first = t_0, t_last = t_{W-1}
+ * maps s_0 and s_{W-1} to the two rows unweighted).  jagg_aggregate is the span of all W
+ * steps with accumulate = 0.
+ *   s        device f32, step j of sample i at s[i * s_sample_stride + j * D] (s_sample_stride =
+ *            0: n * D, a [G, n, D] array; W * D addresses n steps inside a [G, W, D] window)
+ *   t_steps  device [n] f64 network-input times of the steps
+ *   t_first, t_last  host f64 window endpoint times (must differ: JAGG_ERR_ARG otherwise)
+ *   cot      device [2G, D] f32, overwritten (accumulate = 0) or added to (accumulate != 0) */
+int jagg_aggregate_span(const float* s, int64_t s_sample_stride, const double* t_steps, double t_first,
+                        double t_last, int G, int n, int64_t D, float* cot, int accumulate, cudaStream_t stream);
 
 /* jagg_frac routing (Sec. 3.3 "High-noise vs. low-noise scheduling"; rule of the
  * gradient-quality appendix).  Host-only, synchronous.

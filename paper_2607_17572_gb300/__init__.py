@@ -99,9 +99,12 @@ _SIGNATURES = {
     "jagg_signals_workspace_bytes": (_I64, [_I, _I, _I64]),
     "grpo_step_signals": (_I, [_P, _I, _P, _P, _P, _P, _P, _I, _I, _I64, _D, _D, _D, _D, _P, _P, _P, _P,
                                _P, _P, _P, _SZ, _P]),
+    "grpo_step_signals_eps": (_I, [_P, _I, _P, _P, _P, _P, _P, _P, _P, _I, _I, _I64, _D, _D, _D, _D, _P, _P, _P,
+                                   _P, _P, _P, _P, _SZ, _P]),
     "grpo_step_signals_static": (_I, [_P, _I, _P, _P, _P, _P, _P, _I, _I, _I64, _D, _D, _D, _D, _P, _P, _P, _P,
                                       _P, _P, _P]),
     "jagg_aggregate": (_I, [_P, _P, _I, _I, _I64, _P, _P]),
+    "jagg_aggregate_span": (_I, [_P, _I64, _P, _D, _D, _I, _I, _I64, _P, _I, _P]),
     "jagg_route": (_I, [_I, _D, _P, _D, _P, _P]),
     "jagg_grad_reduce_workspace_bytes": (_I64, [_I64]),
     "grad_reduce": (_I, [_P, _P, _I64, ctypes.c_float, _P, _P, _P, _SZ, _P]),
@@ -270,6 +273,23 @@ def grpo_step_signals(v_hat, z, t, sigma, logp_old, rewards, clip_eps, adv_clip,
                                    _stream(stream)), "grpo_step_signals")
 
 
+def grpo_step_signals_eps(eps_hat, z, t, sched_alpha, sched_sigma, sigma, logp_old, rewards, clip_eps, adv_clip,
+                          adv_eps, scale, logp_new, ratio, clipped, adv_out, ws, s_out=None, cot_out=None,
+                          stream=None):
+    """Phase 2 for an epsilon-prediction backbone: the DDIM mean of the schedule
+    (sched_alpha, sched_sigma) [W+1] f64 (device) replaces the flow Euler step."""
+    _need_cuda(eps_hat, z, t, sched_alpha, sched_sigma, sigma, logp_old, rewards, logp_new, ratio, clipped, adv_out,
+               ws, s_out, cot_out)
+    G, W = eps_hat.shape[0], eps_hat.shape[1]
+    D = eps_hat[0, 0].numel()
+    vd = DTYPE_BF16 if eps_hat.dtype == torch.bfloat16 else DTYPE_F32
+    _check(lib().grpo_step_signals_eps(_ptr(eps_hat), vd, _ptr(z), _ptr(t), _ptr(sched_alpha), _ptr(sched_sigma),
+                                       _ptr(sigma), _ptr(logp_old), _ptr(rewards), G, W, D, clip_eps, adv_clip,
+                                       adv_eps, scale, _ptr(s_out), _ptr(cot_out), _ptr(logp_new), _ptr(ratio),
+                                       _ptr(clipped), _ptr(adv_out), _ptr(ws), ws.numel(), _stream(stream)),
+           "grpo_step_signals_eps")
+
+
 def grpo_step_signals_static(v_hat, z, t, sigma, logp_old, rewards, clip_eps, adv_clip, adv_eps, scale,
                              logp_new, ratio, clipped, adv_out, s_out=None, cot_out=None, stream=None):
     """grpo_step_signals without a workspace: scratch comes from an array compiled into the
@@ -289,6 +309,21 @@ def jagg_aggregate(s, t_window, cot, stream=None):
     G, W = s.shape[0], s.shape[1]
     D = s[0, 0].numel()
     _check(lib().jagg_aggregate(_ptr(s), _ptr(t_window), G, W, D, _ptr(cot), _stream(stream)), "jagg_aggregate")
+
+
+def jagg_aggregate_span(s, t_steps, t_first: float, t_last: float, cot, accumulate: bool = False, steps=None,
+                        stream=None):
+    """Phase 3 over a span of steps.  s [G, W, ...] f32 window signals; `steps` = (first, n)
+    selects n consecutive steps (default: all), read in place; t_steps [n] f64 (device);
+    cot [2G, ...] f32."""
+    _need_cuda(s, t_steps, cot)
+    G, W = s.shape[0], s.shape[1]
+    D = s[0, 0].numel()
+    j0, n = steps if steps is not None else (0, W)
+    assert s.is_contiguous() and 0 <= j0 and j0 + n <= W
+    ptr = s.data_ptr() + j0 * D * s.element_size()
+    _check(lib().jagg_aggregate_span(ptr, W * D, _ptr(t_steps), float(t_first), float(t_last), G, n, D, _ptr(cot),
+                                     1 if accumulate else 0, _stream(stream)), "jagg_aggregate_span")
 
 
 def jagg_route(n_windows: int, jagg_frac: float = 1.0, cos=None, tau: float = 0.5):

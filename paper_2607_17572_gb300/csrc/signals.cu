@@ -1,12 +1,20 @@
 // GRPO step signals (Phase 2), JAGG aggregation (Phase 3) and gradient reductions.
 //
+// Both backbone families of Eq. logprob have a transition mean that is affine in the model
+// output y_j (the velocity v_j or the noise prediction eps_j): mu_j = a_j z_j + c_j y_j, with
+//   rectified flow       a_j = 1,                        c_j = t_{j+1} - t_j;
+//   epsilon prediction   a_j = alpha_{j+1} / alpha_j,    c_j = -alpha_{j+1} (sigma_j / alpha_j
+//                                                               - sigma_{j+1} / alpha_{j+1})
+// ((alpha, sigma) the diffusion schedule at the window's times).  So r_ij = z_{j+1} - mu_j and
+// d logp / d y_ij = r_ij c_j / sigma_j^2 for both, and one set of kernels serves both.
+//
 // grpo_step_signals runs in three launches:
-//   1. advantages A_i (Eq. advantage) from the group's rewards;
-//   2. ||r_ij||^2 with r_ij = z_{j+1} - z_j - v_ij dt_j, one CTA per (i, j, chunk of D),
-//      partial sums in f64 written to the workspace (fixed order: deterministic);
+//   1. advantages A_i (Eq. advantage) from the group's rewards, and the W pairs (a_j, c_j);
+//   2. ||r_ij||^2, one CTA per (i, j, chunk of D), partial sums in f64 written to the
+//      workspace (fixed order: deterministic);
 //   3. per (i, j): log-prob (Eq. logprob), ratio, clip decision (Eq. grpo_loss), the
-//      coefficient c_ij = scale (-A_i) rho_ij dt_j / sigma_j^2 (0 when clipped); then one
-//      elementwise pass writes s_ij = c_ij r_ij and/or the aggregated cotangents
+//      coefficient k_ij = scale (-A_i) rho_ij c_j / sigma_j^2 (0 when clipped); then one
+//      elementwise pass writes s_ij = k_ij r_ij and/or the aggregated cotangents
 //      sum_j (1 - alpha_j) s_ij and sum_j alpha_j s_ij (Eq. alpha, Eq. s_base_corr).
 // The v-hat / z tiles of a window are read twice; at the paper's shapes they fit in L2.
 #include <mutex>
@@ -27,8 +35,47 @@ __device__ __forceinline__ float ldv_any(const void* p, int64_t i, int is_f32) {
   return is_f32 ? static_cast<const float*>(p)[i] : __bfloat162float(static_cast<const bf16*>(p)[i]);
 }
 
-__global__ void advantage_kernel(const float* rewards, int G, double adv_eps, double adv_clip, double* adv) {
-  if (threadIdx.x != 0 || blockIdx.x != 0) return;
+// An f64 mean coefficient as an unevaluated sum of two floats (hi + lo).  Rounding a_j or c_j
+// to one float shifts r_ij by the same relative amount at every element, an error that does
+// not average out over D and reaches the log-prob as ~1e-7 * sqrt(D) |z| |r| / sigma^2.
+struct Coef2 {
+  float hi, lo;
+};
+__device__ __forceinline__ Coef2 split_coef(double x) {
+  const float hi = (float)x;
+  return Coef2{hi, (float)(x - (double)hi)};
+}
+// r = z1 - a z0 - c y: the hi products cancel most of z1 exactly inside the first two fmas; the
+// lo terms are small corrections.
+__device__ __forceinline__ float resid(float z1, float z0, float y, Coef2 a, Coef2 c) {
+  float r = fmaf(-a.hi, z0, z1);
+  r = fmaf(-c.hi, y, r);
+  r = fmaf(-a.lo, z0, r);
+  return fmaf(-c.lo, y, r);
+}
+
+// One warp.  Lane 0: the advantages.  All lanes: the mean coefficients mc[j] = a_j,
+// mc[W + j] = c_j; sched_alpha == nullptr selects the rectified-flow step.
+__global__ void prep_kernel(const float* rewards, int G, double adv_eps, double adv_clip, double* adv, const double* t,
+                            const double* sched_alpha, const double* sched_sigma, int W, double* mc) {
+  if (blockIdx.x != 0) return;
+  for (int j = threadIdx.x; j < W; j += 32) {
+    double a = 1.0, c = t[j + 1] - t[j];
+    if (sched_alpha) {
+      const double a0 = sched_alpha[j], a1 = sched_alpha[j + 1];
+      if (a0 > 0.0 && a1 > 0.0) {
+        a = a1 / a0;
+        c = -a1 * (sched_sigma[j] / a0 - sched_sigma[j + 1] / a1);
+      } else {
+        set_device_status(JAGG_DEV_BADARG);
+        a = 0.0;
+        c = 0.0;
+      }
+    }
+    mc[j] = a;
+    mc[W + j] = c;
+  }
+  if (threadIdx.x != 0) return;
   double mu = 0.0;
   for (int i = 0; i < G; ++i) mu += (double)rewards[i];
   mu /= G;
@@ -47,10 +94,10 @@ __global__ void advantage_kernel(const float* rewards, int G, double adv_eps, do
 
 // grid: (chunks, G*W)
 __global__ void __launch_bounds__(SIG_THREADS) resid_norm_kernel(const void* v, int v_f32, const float* z,
-                                                                 const double* t, int W, int64_t D, double* partial) {
+                                                                 const double* mc, int W, int64_t D, double* partial) {
   const int ij = blockIdx.y;
   const int i = ij / W, j = ij % W;
-  const float dt = (float)(t[j + 1] - t[j]);
+  const Coef2 a = split_coef(mc[j]), c = split_coef(mc[W + j]);
   const float* z0 = z + ((int64_t)i * (W + 1) + j) * D;
   const float* z1 = z0 + D;
   const int64_t vb = ((int64_t)i * W + j) * D;
@@ -61,7 +108,7 @@ __global__ void __launch_bounds__(SIG_THREADS) resid_norm_kernel(const void* v, 
   for (int u = 0; u < SIG_PER_THREAD; ++u) {
     const int64_t k = k0 + threadIdx.x + (int64_t)u * SIG_THREADS;
     if (k < D) {
-      const float r = z1[k] - z0[k] - ldv_any(v, vb + k, v_f32) * dt;
+      const float r = resid(z1[k], z0[k], ldv_any(v, vb + k, v_f32), a, c);
       part = fmaf(r, r, part);
     }
     if ((u & 7) == 7) {  // fold every 8 terms into the f64 accumulator
@@ -82,7 +129,7 @@ __global__ void __launch_bounds__(SIG_THREADS) resid_norm_kernel(const void* v, 
 }
 
 // One thread per (i, j).
-__global__ void logprob_kernel(const double* partial, int chunks, const double* t, const double* sigma,
+__global__ void logprob_kernel(const double* partial, int chunks, const double* mc, const double* sigma,
                                const double* logp_old, const double* adv, int G, int W, int64_t D, double clip_eps,
                                double scale, double* logp_new, double* ratio, uint8_t* clipped, float* coef) {
   const int ij = blockIdx.x * blockDim.x + threadIdx.x;
@@ -91,7 +138,7 @@ __global__ void logprob_kernel(const double* partial, int chunks, const double* 
   double rr = 0.0;
   for (int c = 0; c < chunks; ++c) rr += partial[(int64_t)ij * chunks + c];
   const double sg = sigma[j];
-  const double dt = t[j + 1] - t[j];
+  const double c = mc[W + j];
   const double lp = -rr / (2.0 * sg * sg) - (double)D * log(sqrt(2.0 * 3.14159265358979323846) * sg);
   const double rho = exp(lp - logp_old[ij]);
   const double a = adv[i];
@@ -99,20 +146,20 @@ __global__ void logprob_kernel(const double* partial, int chunks, const double* 
   logp_new[ij] = lp;
   ratio[ij] = rho;
   clipped[ij] = clip ? 1 : 0;
-  coef[ij] = clip ? 0.f : (float)(scale * (-a) * rho * dt / (sg * sg));
+  coef[ij] = clip ? 0.f : (float)(scale * (-a) * rho * c / (sg * sg));
 }
 
 // grid: (ceil(D / SIG_THREADS / 4), G).  Each thread: 4 consecutive elements of D.
 __global__ void __launch_bounds__(SIG_THREADS) apply_kernel(const void* v, int v_f32, const float* z, const double* t,
-                                                            const float* coef, int G, int W, int64_t D, float* s_out,
-                                                            float* cot_out) {
+                                                            const double* mc, const float* coef, int G, int W,
+                                                            int64_t D, float* s_out, float* cot_out) {
   const int i = blockIdx.y;
   const int64_t kbase = ((int64_t)blockIdx.x * SIG_THREADS + threadIdx.x) * 4;
   if (kbase >= D) return;
   const double den = t[0] - t[W - 1];
   float base[4] = {0.f, 0.f, 0.f, 0.f}, corr[4] = {0.f, 0.f, 0.f, 0.f};
   for (int j = 0; j < W; ++j) {
-    const float dt = (float)(t[j + 1] - t[j]);
+    const Coef2 ma = split_coef(mc[j]), mcj = split_coef(mc[W + j]);
     const float c = coef[i * W + j];
     const float al = cot_out ? (den != 0.0 ? (float)((t[0] - t[j]) / den) : 0.f) : 0.f;
     const float* z0 = z + ((int64_t)i * (W + 1) + j) * D;
@@ -122,7 +169,7 @@ __global__ void __launch_bounds__(SIG_THREADS) apply_kernel(const void* v, int v
     for (int e = 0; e < 4; ++e) {
       const int64_t k = kbase + e;
       if (k < D) {
-        const float r = z1[k] - z0[k] - ldv_any(v, vb + k, v_f32) * dt;
+        const float r = resid(z1[k], z0[k], ldv_any(v, vb + k, v_f32), ma, mcj);
         const float s = c * r;
         if (s_out) s_out[vb + k] = s;
         base[e] += (1.f - al) * s;
@@ -162,6 +209,30 @@ __global__ void aggregate_kernel(const float* s, const double* t, int G, int W, 
   }
   cot[(int64_t)i * D + k] = base;
   cot[((int64_t)G + i) * D + k] = corr;
+}
+
+__global__ void aggregate_span_kernel(const float* s, int64_t ld, const double* t, double t_first, double t_last, int G,
+                                      int n, int64_t D, float* cot, int accumulate) {
+  const int i = blockIdx.y;
+  const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= D) return;
+  const double den = t_first - t_last;
+  float base = 0.f, corr = 0.f;
+  for (int j = 0; j < n; ++j) {
+    const float al = (float)((t_first - t[j]) / den);
+    const float v = s[(int64_t)i * ld + (int64_t)j * D + k];
+    base += (1.f - al) * v;
+    corr += al * v;
+  }
+  float* b = cot + (int64_t)i * D + k;
+  float* c = cot + ((int64_t)G + i) * D + k;
+  if (accumulate) {
+    *b += base;
+    *c += corr;
+  } else {
+    *b = base;
+    *c = corr;
+  }
 }
 
 // ------------------------------------------------------------------ grad_reduce
@@ -240,6 +311,9 @@ __global__ void grad_reduce_final(const double* partial, double* out3) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
+// The (a_j, c_j) pairs at the head of the signals workspace, padded to 16 bytes.
+int64_t mean_coef_bytes(int W) { return ((int64_t)2 * W * 8 + 15) / 16 * 16; }
+
 }  // namespace
 
 }  // namespace jagg
@@ -250,37 +324,39 @@ using namespace jagg;
 extern "C" int64_t jagg_signals_workspace_bytes(int G, int W, int64_t D) {
   if (G <= 0 || W <= 0 || D <= 0) return 0;
   const int64_t chunks = (D + SIG_CHUNK - 1) / SIG_CHUNK;
-  return (int64_t)G * W * chunks * 8 + (int64_t)G * W * 4 + 64;
+  return mean_coef_bytes(W) + (int64_t)G * W * chunks * 8 + (int64_t)G * W * 4 + 64;
 }
 
-extern "C" int grpo_step_signals(const void* v_hat, int v_dtype, const float* z, const double* t, const double* sigma,
-                                 const double* logp_old, const float* rewards, int G, int W, int64_t D,
-                                 double clip_eps, double adv_clip, double adv_eps, double scale, float* s_out,
-                                 float* cot_out, double* logp_new, double* ratio, uint8_t* clipped, double* adv_out,
-                                 void* ws, size_t ws_bytes, cudaStream_t stream) {
-  JAGG_CHECK_ARG(G > 0 && W > 0 && D > 0, "grpo_step_signals: G=%d W=%d D=%lld must be positive", G, W,
-                 (long long)D);
-  JAGG_CHECK_ARG(G <= 65535 && (int64_t)G * W <= 65535, "grpo_step_signals: G*W too large");
-  JAGG_CHECK_ARG(v_dtype == JAGG_DTYPE_F32 || v_dtype == JAGG_DTYPE_BF16, "grpo_step_signals: bad v_dtype");
+namespace jagg {
+namespace {
+int step_signals(const char* name, const void* v_hat, int v_dtype, const float* z, const double* t,
+                 const double* sched_alpha, const double* sched_sigma, const double* sigma, const double* logp_old,
+                 const float* rewards, int G, int W, int64_t D, double clip_eps, double adv_clip, double adv_eps,
+                 double scale, float* s_out, float* cot_out, double* logp_new, double* ratio, uint8_t* clipped,
+                 double* adv_out, void* ws, size_t ws_bytes, cudaStream_t stream) {
+  JAGG_CHECK_ARG(G > 0 && W > 0 && D > 0, "%s: G=%d W=%d D=%lld must be positive", name, G, W, (long long)D);
+  JAGG_CHECK_ARG(G <= 65535 && (int64_t)G * W <= 65535, "%s: G*W too large", name);
+  JAGG_CHECK_ARG(v_dtype == JAGG_DTYPE_F32 || v_dtype == JAGG_DTYPE_BF16, "%s: bad v_dtype", name);
   JAGG_CHECK_ARG(v_hat && z && t && sigma && logp_old && rewards && logp_new && ratio && clipped && adv_out && ws,
-                 "grpo_step_signals: null pointer");
-  JAGG_CHECK_ARG(!cot_out || W >= 2, "grpo_step_signals: aggregation needs W >= 2");
-  JAGG_CHECK_ARG(clip_eps >= 0.0 && adv_clip >= 0.0 && adv_eps >= 0.0, "grpo_step_signals: negative constant");
+                 "%s: null pointer", name);
+  JAGG_CHECK_ARG(!cot_out || W >= 2, "%s: aggregation needs W >= 2", name);
+  JAGG_CHECK_ARG(clip_eps >= 0.0 && adv_clip >= 0.0 && adv_eps >= 0.0, "%s: negative constant", name);
   const int64_t need = jagg_signals_workspace_bytes(G, W, D);
   if ((int64_t)ws_bytes < need) {
-    set_last_error("grpo_step_signals: workspace %zu < %lld bytes", ws_bytes, (long long)need);
+    set_last_error("%s: workspace %zu < %lld bytes", name, ws_bytes, (long long)need);
     return JAGG_ERR_WORKSPACE;
   }
-  JAGG_CHECK_ARG(aligned16(ws), "grpo_step_signals: workspace not 16-byte aligned");
+  JAGG_CHECK_ARG(aligned16(ws), "%s: workspace not 16-byte aligned", name);
   const int chunks = (int)((D + SIG_CHUNK - 1) / SIG_CHUNK);
-  double* partial = static_cast<double*>(ws);
+  double* mc = static_cast<double*>(ws);
+  double* partial = reinterpret_cast<double*>(static_cast<char*>(ws) + mean_coef_bytes(W));
   float* coef = reinterpret_cast<float*>(partial + (int64_t)G * W * chunks);
   const int vf32 = v_dtype == JAGG_DTYPE_F32;
-  advantage_kernel<<<1, 32, 0, stream>>>(rewards, G, adv_eps, adv_clip, adv_out);
+  prep_kernel<<<1, 32, 0, stream>>>(rewards, G, adv_eps, adv_clip, adv_out, t, sched_alpha, sched_sigma, W, mc);
   JAGG_LAUNCHED();
-  resid_norm_kernel<<<dim3(chunks, G * W), SIG_THREADS, 0, stream>>>(v_hat, vf32, z, t, W, D, partial);
+  resid_norm_kernel<<<dim3(chunks, G * W), SIG_THREADS, 0, stream>>>(v_hat, vf32, z, mc, W, D, partial);
   JAGG_LAUNCHED();
-  logprob_kernel<<<ceil_div((int64_t)G * W, 128), 128, 0, stream>>>(partial, chunks, t, sigma, logp_old, adv_out, G,
+  logprob_kernel<<<ceil_div((int64_t)G * W, 128), 128, 0, stream>>>(partial, chunks, mc, sigma, logp_old, adv_out, G,
                                                                      W, D, clip_eps, scale, logp_new, ratio, clipped,
                                                                      coef);
   JAGG_LAUNCHED();
@@ -290,10 +366,35 @@ extern "C" int grpo_step_signals(const void* v_hat, int v_dtype, const float* z,
       JAGG_LAUNCHED();
     }
     const int gx = ceil_div(D, (int64_t)SIG_THREADS * 4);
-    apply_kernel<<<dim3(gx, G), SIG_THREADS, 0, stream>>>(v_hat, vf32, z, t, coef, G, W, D, s_out, cot_out);
+    apply_kernel<<<dim3(gx, G), SIG_THREADS, 0, stream>>>(v_hat, vf32, z, t, mc, coef, G, W, D, s_out,
+                                                          cot_out);
     JAGG_LAUNCHED();
   }
   return JAGG_OK;
+}
+}  // namespace
+}  // namespace jagg
+
+extern "C" int grpo_step_signals(const void* v_hat, int v_dtype, const float* z, const double* t, const double* sigma,
+                                 const double* logp_old, const float* rewards, int G, int W, int64_t D,
+                                 double clip_eps, double adv_clip, double adv_eps, double scale, float* s_out,
+                                 float* cot_out, double* logp_new, double* ratio, uint8_t* clipped, double* adv_out,
+                                 void* ws, size_t ws_bytes, cudaStream_t stream) {
+  return step_signals("grpo_step_signals", v_hat, v_dtype, z, t, nullptr, nullptr, sigma, logp_old, rewards, G, W, D,
+                      clip_eps, adv_clip, adv_eps, scale, s_out, cot_out, logp_new, ratio, clipped, adv_out, ws,
+                      ws_bytes, stream);
+}
+
+extern "C" int grpo_step_signals_eps(const void* eps_hat, int eps_dtype, const float* z, const double* t,
+                                     const double* sched_alpha, const double* sched_sigma, const double* sigma,
+                                     const double* logp_old, const float* rewards, int G, int W, int64_t D,
+                                     double clip_eps, double adv_clip, double adv_eps, double scale, float* s_out,
+                                     float* cot_out, double* logp_new, double* ratio, uint8_t* clipped,
+                                     double* adv_out, void* ws, size_t ws_bytes, cudaStream_t stream) {
+  JAGG_CHECK_ARG(sched_alpha && sched_sigma, "grpo_step_signals_eps: null schedule");
+  return step_signals("grpo_step_signals_eps", eps_hat, eps_dtype, z, t, sched_alpha, sched_sigma, sigma, logp_old,
+                      rewards, G, W, D, clip_eps, adv_clip, adv_eps, scale, s_out, cot_out, logp_new, ratio, clipped,
+                      adv_out, ws, ws_bytes, stream);
 }
 
 extern "C" int jagg_aggregate(const float* s, const double* t_window, int G, int W, int64_t D, float* cot,
@@ -304,6 +405,21 @@ extern "C" int jagg_aggregate(const float* s, const double* t_window, int G, int
   check_alpha_kernel<<<1, 32, 0, stream>>>(t_window, W);
   JAGG_LAUNCHED();
   aggregate_kernel<<<dim3(ceil_div(D, 256), G), 256, 0, stream>>>(s, t_window, G, W, D, cot);
+  JAGG_LAUNCHED();
+  return JAGG_OK;
+}
+
+extern "C" int jagg_aggregate_span(const float* s, int64_t s_sample_stride, const double* t_steps, double t_first,
+                                   double t_last, int G, int n, int64_t D, float* cot, int accumulate,
+                                   cudaStream_t stream) {
+  JAGG_CHECK_ARG(s && t_steps && cot, "jagg_aggregate_span: null pointer");
+  JAGG_CHECK_ARG(G > 0 && G <= 65535 && n > 0 && D > 0, "jagg_aggregate_span: bad G=%d, n=%d or D=%lld", G, n,
+                 (long long)D);
+  JAGG_CHECK_ARG(t_first != t_last, "jagg_aggregate_span: the window endpoints must differ");
+  const int64_t ld = s_sample_stride ? s_sample_stride : (int64_t)n * D;
+  JAGG_CHECK_ARG(ld >= (int64_t)n * D, "jagg_aggregate_span: sample stride %lld below n * D", (long long)ld);
+  aggregate_span_kernel<<<dim3(ceil_div(D, 256), G), 256, 0, stream>>>(s, ld, t_steps, t_first, t_last, G, n, D, cot,
+                                                                       accumulate);
   JAGG_LAUNCHED();
   return JAGG_OK;
 }

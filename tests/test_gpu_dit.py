@@ -97,3 +97,33 @@ def test_forward_without_saves_matches_saved_forward(wl):
 def test_dit_b_full_depth_joint_vjp():
     """DiT-B (12 blocks, 333 tokens) at its JAGG batch of 2G = 16 rows."""
     _check(DITB, 2 * DITB.G, 2e-2, 1e-2, seed=11)
+
+
+@pytest.mark.parametrize("wl,G,tol", [(TINY, 4, 1e-5), (synth.small_variant(DITB, name="ditb_2blocks", depth=2), 4,
+                                                        5e-3)], ids=["tiny_f32", "ditb_2blocks_bf16"])
+def test_sequential_graph_variant_matches_the_joint_vjp(wl, G, tol):
+    """Algorithm 2: forward of endpoint 0 into one G-row arena, VJP with s_base, forward of
+    endpoint W-1 into the same arena, VJP with s_corr -- the same gradient as one joint VJP
+    over 2G rows, with half the saved activations.  (bf16: a G-row and a 2G-row product may
+    pick different tile widths and round differently, a few 1e-3 relative.)"""
+    params = synth.make_params(wl)
+    z, t, txt = model_inputs(wl, 2 * G, 21)
+    t[:G], t[G:] = 0.8, 0.55
+    rng = np.random.Generator(np.random.PCG64(22))
+    cot = rng.standard_normal(z.shape)
+    gm = GpuModel(jg, wl, params)
+    v, saved, ws = gm.forward(z, t, txt)
+    g_joint = gm.vjp(saved, ws, 2 * G, cot)
+    assert gm.model.saved_bytes(G) <= 0.51 * gm.model.saved_bytes(2 * G)
+    g_seq = torch.zeros_like(g_joint)
+    arena = jg.alloc_bytes(gm.model.saved_bytes(G))      # the one arena of both endpoints
+    ws1 = jg.alloc_bytes(gm.model.workspace_bytes(G))
+    for part in (slice(0, G), slice(G, 2 * G)):
+        zt = gm.tensor(z[part])
+        jg.dit_forward_save(gm.model, zt, torch.tensor(t[part], dtype=torch.float32, device="cuda"),
+                            gm.tensor(txt[part]), torch.empty_like(zt), saved=arena, ws=ws1)
+        gm.vjp(arena, ws1, G, cot[part], grad=g_seq)
+    torch.cuda.synchronize()
+    r = rel_l2(g_seq.cpu().numpy(), g_joint.cpu().numpy())
+    print(f"{wl.name}: sequential vs joint rel L2 {r:.2e}")
+    assert r <= tol

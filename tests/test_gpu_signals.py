@@ -87,6 +87,82 @@ def test_step_signals_and_aggregation_match_oracle(G, W, D, v_dtype, eps, shift)
         assert _rel(cot2.cpu().numpy(), grpo.aggregate(s.cpu().numpy(), t[:W])) < 1e-6
 
 
+def _eps_case(G, W, D, e_dtype, clip_eps, seed):
+    """An epsilon-prediction window on the variance-preserving cosine schedule: eps-hat from
+    N(0,1), z_{j+1} = (DDIM mean of z_j, eps_j) + sigma_j xi, old log-probs as in _case."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    t = synth.time_grid(4 * W, 3.0)[W:2 * W + 1] * 0.9 + 0.05
+    al, sg = synth.vp_schedule(t)
+    sig = synth.sigma_schedule(t, 0.5)
+    e = synth.storage_round(rng.standard_normal((G, W, D)), e_dtype)
+    z = np.zeros((G, W + 1, D))
+    z[:, 0] = rng.standard_normal((G, D))
+    for j in range(W):
+        mu = grpo.ddim_mean(z[:, j], e[:, j], al[j], al[j + 1], sg[j], sg[j + 1])
+        z[:, j + 1] = mu + sig[j] * rng.standard_normal((G, D))
+    z = z.astype(np.float32).astype(np.float64)
+    lp = np.array([[grpo.step_logprob_eps(z[i, j + 1], z[i, j], e[i, j], al[j], al[j + 1], sg[j], sg[j + 1], sig[j])
+                    for j in range(W)] for i in range(G)])
+    inside = rng.uniform(-0.3 * clip_eps, 0.3 * clip_eps, (G, W))
+    outside = rng.uniform(2 * clip_eps, 3 * clip_eps, (G, W)) * rng.choice([-1.0, 1.0], (G, W))
+    delta = np.where(rng.uniform(size=(G, W)) < 0.5, inside, outside)
+    rewards = synth.storage_round(rng.standard_normal(G), "f32")
+    return e, z, t, al, sg, sig, lp + delta, rewards
+
+
+def _run_eps(e, z, t, al, sg, sig, lpo, rewards, eps, scale, e_dtype, with_cot=True):
+    dev = "cuda"
+    G, W, D = e.shape
+    f64 = dict(dtype=torch.float64, device=dev)
+    out = dict(logp_new=torch.empty(G, W, **f64), ratio=torch.empty(G, W, **f64),
+               clipped=torch.empty(G, W, dtype=torch.uint8, device=dev), adv_out=torch.empty(G, **f64))
+    s = torch.full((G, W, D), float("nan"), device=dev)
+    cot = torch.full((2 * G, D), float("nan"), device=dev) if with_cot else None
+    ws = jg.alloc_bytes(jg.signals_workspace_bytes(G, W, D))
+    te = torch.tensor(e, dtype=torch.bfloat16 if e_dtype == "bf16" else torch.float32, device=dev)
+    jg.grpo_step_signals_eps(te, torch.tensor(z, dtype=torch.float32, device=dev), torch.tensor(t, **f64),
+                             torch.tensor(al, **f64), torch.tensor(sg, **f64), torch.tensor(sig, **f64),
+                             torch.tensor(lpo, **f64), torch.tensor(rewards, dtype=torch.float32, device=dev), eps,
+                             5.0, 1e-8, scale, ws=ws, s_out=s, cot_out=cot, **out)
+    torch.cuda.synchronize()
+    return s, cot, out
+
+
+@pytest.mark.parametrize("G,W,D,e_dtype,eps", [
+    (4, 4, 64, "f32", 1e-4),
+    (8, 4, 16384, "bf16", 0.1),
+    (3, 2, 12345, "bf16", 0.1),       # ragged D, W = 2
+    (5, 3, 8193, "f32", 0.05),        # D one past a CTA chunk
+])
+def test_eps_prediction_signals_match_oracle(G, W, D, e_dtype, eps):
+    """grpo_step_signals_eps (the DDIM mean of Eq. logprob) against the oracle, element by
+    element, with the same bars as the velocity path."""
+    e, z, t, al, sg, sig, lpo, rewards = _eps_case(G, W, D, e_dtype, eps, seed=7 * G + D)
+    scale = 1.0 / (G * 16)
+    A = grpo.advantages(rewards)
+    s_o, lp_o, ratio_o, clip_o = grpo.step_signals_eps(e, z, al, sg, sig, lpo, A, eps, scale)
+    jg.device_status(clear=True)
+    s, cot, out = _run_eps(e, z, t, al, sg, sig, lpo, rewards, eps, scale, e_dtype)
+    assert jg.device_status() == 0
+    lp_tol = 1e-6 * max(10.0, D / 50)
+    assert np.max(np.abs(out["logp_new"].cpu().numpy() - lp_o)) < lp_tol
+    np.testing.assert_allclose(out["ratio"].cpu().numpy(), ratio_o, rtol=2 * lp_tol)
+    np.testing.assert_array_equal(out["clipped"].cpu().numpy(), clip_o)
+    assert _rel(s.cpu().numpy(), s_o) < 1e-4
+    assert _rel(cot.cpu().numpy(), grpo.aggregate(s_o, t[:W])) < 1e-4
+
+
+def test_eps_prediction_rejects_a_nonpositive_alpha():
+    """alpha_t <= 0 makes the DDIM mean undefined: the device status reports it."""
+    e, z, t, al, sg, sig, lpo, rewards = _eps_case(2, 3, 100, "f32", 0.1, seed=5)
+    al = al.copy()
+    al[3] = 0.0
+    jg.device_status(clear=True)
+    _run_eps(e, z, t, al, sg, sig, lpo, rewards, 0.1, 0.1, "f32", with_cot=False)
+    assert jg.device_status() & 2
+    jg.device_status(clear=True)
+
+
 def test_aggregate_rejects_degenerate_window():
     dev = "cuda"
     s = torch.ones(2, 3, 10, device=dev)
@@ -119,3 +195,35 @@ def test_grad_reduce_matches_numpy(P):
     ab, aa, bb = out3.cpu().numpy()
     ro = grpo.grad_stats(a.cpu().numpy(), b.cpu().numpy())
     assert abs(ab / np.sqrt(aa * bb) - ro[3]) < 1e-6
+
+
+@pytest.mark.parametrize("G,W,D", [(4, 4, 64), (8, 5, 3000), (3, 8, 1 << 16)])
+def test_span_aggregation_and_ablation_match_oracle(G, W, D):
+    """The sequential-graph split (steps 0..W-2, then the last step accumulated) and the
+    endpoint-only ablation (span over {0, W-1}) against the oracle's definitions."""
+    dev = "cuda"
+    rng = np.random.Generator(np.random.PCG64(G * 100 + W))
+    s = rng.standard_normal((G, W, D)).astype(np.float32)
+    t = synth.time_grid(16, 3.0)[2:2 + W]
+    f64 = dict(dtype=torch.float64, device=dev)
+    st = torch.tensor(s, device=dev)
+    cot = torch.full((2 * G, D), float("nan"), device=dev)
+    jg.jagg_aggregate_span(st, torch.tensor(t[:-1], **f64), t[0], t[-1], cot, steps=(0, W - 1))
+    jg.jagg_aggregate_span(st, torch.tensor(t[-1:], **f64), t[0], t[-1], cot, accumulate=True, steps=(W - 1, 1))
+    ref = grpo.aggregate(s.astype(np.float64), t)
+    torch.cuda.synchronize()
+    assert np.abs(cot.cpu().numpy() - ref).max() <= 1e-5 * max(1.0, np.abs(ref).max())
+    # ablation: step 0 and step W-1 read in place, each over its own span (bit-exact pair)
+    ab = torch.empty(2 * G, D, device=dev)
+    jg.jagg_aggregate_span(st, torch.tensor(t[:1], **f64), t[0], t[-1], ab, steps=(0, 1))
+    jg.jagg_aggregate_span(st, torch.tensor(t[-1:], **f64), t[0], t[-1], ab, accumulate=True, steps=(W - 1, 1))
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(ab.cpu().numpy(), grpo.aggregate_ablate(s).astype(np.float32))
+    # a contiguous [G, 2, D] pair over the span {t_0, t_{W-1}} gives the same rows
+    ends = torch.stack([st[:, 0], st[:, -1]], 1).contiguous()
+    ab2 = torch.empty(2 * G, D, device=dev)
+    jg.jagg_aggregate_span(ends, torch.tensor([t[0], t[-1]], **f64), t[0], t[-1], ab2)
+    torch.cuda.synchronize()
+    assert torch.equal(ab, ab2)
+    with pytest.raises(jg.JaggError):
+        jg.jagg_aggregate_span(ends, torch.tensor([t[0], t[0]], **f64), t[0], t[0], ab)
