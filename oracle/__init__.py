@@ -13,7 +13,8 @@ Contents (each function cites the passage of the paper it follows):
                       Eq. alpha / Eq. s_base_corr aggregation, jagg_frac routing,
                       cosine / norm-ratio reductions
   linear_velocity.py  a velocity model linear in (z, t) for the exactness theorem
-  rollout.py          flow-SDE rollout that produces trajectories and old log-probs
+  rollout.py          one sampler step (flow Euler-Maruyama or stochastic DDIM) with the
+                      log-prob of its sample; the flow-SDE rollout built from it
   path.py             JAGG and full per-step window gradients (Algorithm 1)
 
 Every function computes in float64 with numpy; library matmuls are the only primitives.

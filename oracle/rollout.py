@@ -1,4 +1,5 @@
-"""Flow-SDE rollout producing trajectories and old log-probs for synthetic workloads.
+"""Stochastic sampler steps and the flow-SDE rollout producing trajectories and old
+log-probs for synthetic workloads.
 
 TEST INFRASTRUCTURE ONLY (see oracle/__init__.py).
 
@@ -13,7 +14,35 @@ from __future__ import annotations
 
 import numpy as np
 
-from .grpo import step_logprob
+from .grpo import ddim_mean, step_logprob, step_logprob_eps
+
+
+def sampler_step(z_cur, y_hat, xi, t_cur, t_next, sigma, sched=None):
+    """One step of the stochastic sampler whose Gaussian transition Eq. logprob scores, and
+    the log-probability of the sample it draws (the rollout's old log-prob):
+        z_{j+1} = mu_theta(z_j, t_j) + sigma_j xi_j,   xi_j ~ N(0, I) (passed in),
+    with mu the rectified-flow Euler step z_j + v_j (t_{j+1} - t_j) when sched is None, else
+    the DDIM mean of an epsilon-prediction model (ddim_mean) with
+    sched = (alpha_{t_j}, alpha_{t_{j+1}}, sigma_{t_j}, sigma_{t_{j+1}}).
+
+    z_next is rounded to float32, the precision trajectories are stored in, before its
+    log-probability is taken (the update stage scores the stored sample).  Arrays of D
+    elements (or [G, D] with the log-prob per row)."""
+    z_cur = np.asarray(z_cur, np.float64)
+    y_hat = np.asarray(y_hat, np.float64)
+    if sched is None:
+        mu = z_cur + y_hat * (t_next - t_cur)
+    else:
+        mu = ddim_mean(z_cur, y_hat, *sched)
+    z_next = (mu + sigma * np.asarray(xi, np.float64)).astype(np.float32).astype(np.float64)
+    rows = z_next.reshape(-1, z_next.shape[-1]) if z_next.ndim > 1 else z_next[None]
+    zc = z_cur.reshape(rows.shape)
+    yh = y_hat.reshape(rows.shape)
+    if sched is None:
+        lp = [step_logprob(rows[i], zc[i], yh[i], t_cur, t_next, sigma) for i in range(rows.shape[0])]
+    else:
+        lp = [step_logprob_eps(rows[i], zc[i], yh[i], *sched, sigma) for i in range(rows.shape[0])]
+    return z_next, (np.array(lp) if z_next.ndim > 1 else lp[0])
 
 
 def rollout(model, wl, draws, t, sigma, n_steps=None, storage_round=None):
@@ -32,8 +61,8 @@ def rollout(model, wl, draws, t, sigma, n_steps=None, storage_round=None):
         if storage_round is not None:
             vj = storage_round(vj)
         v[:, j] = vj
-        znext = z[:, j] + vj * (t[j + 1] - t[j]) + sigma[j] * draws.xi[:, j]
-        z[:, j + 1] = znext.astype(np.float32).astype(np.float64)
-        for i in range(G):
-            logp[i, j] = step_logprob(z[i, j + 1], z[i, j], v[i, j], t[j], t[j + 1], sigma[j])
+        xi = draws.xi[:, j].reshape(G, -1)
+        zn, lp = sampler_step(z[:, j].reshape(G, -1), vj.reshape(G, -1), xi, t[j], t[j + 1], sigma[j])
+        z[:, j + 1] = zn.reshape((G,) + shape)
+        logp[:, j] = lp
     return z, v, logp

@@ -271,3 +271,38 @@ def test_eps_signals_are_the_gradient_of_the_window_loss(seed):
                       - grpo.window_loss_eps(em, z[i], al, sg, sig, lpo[i], A[i], clip, scale)) / (2 * h)
                 assert fd == pytest.approx(s[i, j, k], rel=1e-6, abs=1e-9)
     assert clipped.any() and not clipped.all()
+
+
+# ------------------------------------------------------------------ sampler step (rollout)
+from oracle import rollout as oracle_rollout  # noqa: E402
+
+
+@pytest.mark.parametrize("eps_model", [False, True])
+def test_sampler_step_logprob_is_the_density_of_its_noise(eps_model):
+    """z_{j+1} - mu = sigma xi up to the float32 storage of z_{j+1}, so the log-prob of the
+    drawn sample is the standard-normal density of xi rescaled: -||xi||^2 / 2 - D log(sqrt(2 pi)
+    sigma) (scipy), within the storage rounding."""
+    rng = np.random.Generator(np.random.PCG64(95))
+    G, D = 3, 40
+    z, y, xi = rng.standard_normal((3, G, D))
+    t0, t1, sig = 0.7, 0.62, 0.2
+    sched = tuple(np.concatenate(synth.vp_schedule([t0, t1]))[[0, 1, 2, 3]]) if eps_model else None
+    zn, lp = oracle_rollout.sampler_step(z, y, xi, t0, t1, sig, sched)
+    ref = stats.norm.logpdf(xi, scale=1.0).sum(axis=1) - D * math.log(sig)
+    np.testing.assert_allclose(lp, ref, rtol=0, atol=1e-4)
+    assert zn.dtype == np.float64 and np.array_equal(zn, zn.astype(np.float32).astype(np.float64))
+
+
+def test_sampler_step_without_noise_follows_the_flow():
+    """sigma -> 0: the flow step is the Euler step of dz/dt = v (exact for a constant field:
+    z moves by v (t_{j+1} - t_j)); the epsilon step on the rectified-flow schedule with
+    eps = z + (1 - t) v is the same step."""
+    rng = np.random.Generator(np.random.PCG64(96))
+    D = 17
+    z, v, xi = rng.standard_normal((3, D))
+    t0, t1 = 0.9, 0.75
+    zn, _ = oracle_rollout.sampler_step(z, v, xi, t0, t1, 1e-12)
+    np.testing.assert_allclose(zn, z + v * (t1 - t0), atol=1e-6)
+    e = z + (1 - t0) * v
+    zn2, _ = oracle_rollout.sampler_step(z, e, xi, t0, t1, 1e-12, sched=(1 - t0, 1 - t1, t0, t1))
+    np.testing.assert_allclose(zn2, zn, atol=1e-6)
