@@ -13,7 +13,9 @@ The metric is trajectory-steps of gradient per second: G * T (sample, step) pair
 
 Also timed: the same step with one joint VJP per window (Algorithm 1 as written), the
 exact per-step path (jagg_frac = 0: the VJP over all W*G step inputs of every window with
-their own s_j), and `e2e`, the update stage through the public API from pinned host
+their own s_j), the sequential-graph variant and the endpoint-only ablation, the update
+stage (forwards on the stored experience + backward, JAGG against the exact path), the
+rollout sampler, and `e2e`, the update stage through the public API from pinned host
 buffers (Phase 1 forwards included).  `--impl reference` times the float64 CPU oracle.
 """
 from __future__ import annotations
@@ -214,6 +216,7 @@ class Bench:
         ws_rows = self.nw * W * G if self.model.saved_bytes(self.nw * W * G) < 0.4 * total else W * G
         self.ws = jg.alloc_bytes(self.model.workspace_bytes(ws_rows), dev)
         self.sws = jg.alloc_bytes(jg.signals_workspace_bytes(G, W, self.D), dev)
+        self.rws = jg.alloc_bytes(jg.rollout_workspace_bytes(G, self.D), dev)
         self.gws = jg.alloc_bytes(jg.grad_reduce_workspace_bytes(self.P), dev)
         self.grad = torch.zeros(self.P, dtype=torch.float32, device=dev)
         self.out3 = torch.zeros(3, **f64)
@@ -237,34 +240,45 @@ class Bench:
     def txt_rows(self, B):
         return self.txt1.unsqueeze(0).expand(B, -1, -1).contiguous()
 
-    def rollout(self):
-        """Synthetic trajectories from the model itself (theta_old = theta): Euler-Maruyama
-        steps z_{j+1} = z_j + v dt + sigma xi, old log-probs = rollout log-probs + delta."""
+    def sampler(self):
+        """The group's rollout on the device (theta_old = theta): per step, the forward without
+        saves on the G current samples, then the fused sampler step (Euler-Maruyama draw with
+        the passed-in noise, f32 trajectory store, the next forward's bf16 input and the old
+        log-prob).  Returns the closure and its buffers."""
         jg, wl, dev = self.jg, self.wl, self.dev
-        G, T, W = wl.G, wl.T, wl.W
+        G, T = wl.G, wl.T
         z = torch.zeros(G, T + 1, self.D, dtype=torch.float32, device=dev)
-        z[:, 0] = torch.tensor(self.draws.z0.reshape(-1), dtype=torch.float32, device=dev)
-        xi = torch.tensor(self.draws.xi.reshape(G, T, -1), dtype=torch.float32, device=dev)
-        v_all = torch.empty(G, T, self.D, dtype=self.tdt, device=dev)
+        z0 = torch.tensor(self.draws.z0.reshape(-1), dtype=torch.float32, device=dev)
+        xi = torch.tensor(np.ascontiguousarray(self.draws.xi.reshape(G, T, -1).transpose(1, 0, 2)),
+                          dtype=torch.float32, device=dev)            # [T, G, D]: xi[j] contiguous
+        v_all = torch.empty(T, G, *self.shape, dtype=self.tdt, device=dev)
+        zin = torch.empty(G, *self.shape, dtype=self.tdt, device=dev)
+        lp = torch.empty(G, T, dtype=torch.float64, device=dev)
         txt = self.txt_rows(G)
-        v = torch.empty(G, *self.shape, dtype=self.tdt, device=dev)
-        for j in range(T):
-            zin = z[:, j].reshape(G, *self.shape).to(self.tdt).contiguous()
-            tin = torch.full((G,), float(self.t[j]), dtype=torch.float32, device=dev)
-            jg.dit_forward_save(self.model, zin, tin, txt, v, ws=self.ws)
-            v_all[:, j] = v.reshape(G, -1)
-            z[:, j + 1] = z[:, j] + v.reshape(G, -1).float() * float(self.t[j + 1] - self.t[j]) + float(self.sig[j]) * xi[:, j]
+        tin = [torch.full((G,), float(self.t[j]), dtype=torch.float32, device=dev) for j in range(T)]
+
+        def run():
+            z[:, 0].copy_(z0.unsqueeze(0).expand(G, -1))
+            zin.copy_(z[:, 0].reshape(G, *self.shape))
+            for j in range(T):
+                jg.dit_forward_save(self.model, zin, tin[j], txt, v_all[j], ws=self.ws)
+                jg.jagg_rollout_step(v_all[j], z, j, xi[j], self.t[j], self.t[j + 1], self.sig[j], lp, self.rws,
+                                     z_model=zin)
+        return run, z, v_all, lp
+
+    def rollout(self):
+        """Synthetic trajectories from the model itself: the device sampler; old log-probs =
+        the rollout's log-probs + delta."""
+        wl, dev = self.wl, self.dev
+        G, T, W = wl.G, wl.T, wl.W
+        run, z, v_all, lp = self.sampler()
+        run()
         self.z = z
-        self.v_all = v_all
+        self.v_all = v_all.transpose(0, 1).reshape(G, T, -1).contiguous()
         self.v_win = [self.v_all[:, w * W:(w + 1) * W].contiguous() for w in range(self.nw)]
         self.z_win = [self.z[:, w * W:w * W + W + 1].contiguous() for w in range(self.nw)]
-        # old log-probs: the rollout's log-probs (from the library's own log-prob) + delta
-        self.logp_old = torch.zeros(G, T, dtype=torch.float64, device=dev)
-        zero = torch.zeros(G, W, dtype=torch.float64, device=dev)
-        for w in range(self.nw):
-            self.signals(w, zero)
-            self.logp_old[:, w * W:(w + 1) * W] = self.sig_out["logp_new"]
-        self.logp_old += torch.tensor(self.draws.delta, dtype=torch.float64, device=dev)
+        self.logp_rollout = lp.clone()
+        self.logp_old = lp + torch.tensor(self.draws.delta, dtype=torch.float64, device=dev)
         self.lpo_win = [self.logp_old[:, w * W:(w + 1) * W].contiguous() for w in range(self.nw)]
         torch.cuda.synchronize()
 
@@ -623,6 +637,8 @@ def run_gpu(args, ws, rank):
         if batched:
             out["graph_variants"] = graph_variants(b, args, ws, use_graph)
             out["ablate"] = ablate_step(b, args, ws, use_graph)
+            out["update_stage"] = update_stage(b, args, ws, use_graph)
+        out["rollout"] = rollout_leg(b, args, ws, use_graph)
         if not args.no_e2e and batched:
             out["e2e"] = run_e2e(b, args, ws, routes)
         # the float64 oracle needs minutes per sequence at MMDiT width: DiT workloads only
@@ -637,11 +653,13 @@ def run_gpu(args, ws, rank):
         print(json.dumps(out), flush=True)
 
 
-def run_e2e(b, args, ws, routes):
-    """The update stage through the public API from pinned host buffers: per step, copy the
-    group's trajectory, old log-probs and rewards to the device, run every window's Phase 1
-    forwards (endpoints saved, middle steps without saves) and Phases 2-4, and copy the
-    new log-probs and the gradient norm back."""
+def jagg_update(b, host):
+    """The JAGG update stage of one group (the paper's "update": forwards on the stored
+    experience, then the backward): every window's Phase 1 forwards (endpoints saved, middle
+    steps without saves), Phases 2-3 per window, one joint VJP over every window's endpoint
+    rows, the gradient norm.  host=True: the step starts by copying the group's trajectory,
+    old log-probs and rewards from pinned host buffers and ends by reading the new log-probs
+    and the gradient norm back.  Returns (step, h2d bytes, d2h bytes)."""
     jg, wl, dev = b.jg, b.wl, b.dev
     G, W = wl.G, wl.W
     h_z = b.z.cpu().pin_memory()
@@ -664,9 +682,10 @@ def run_e2e(b, args, ws, routes):
     z_mid = torch.empty(max(Bm, 1), *b.shape, dtype=b.tdt, device=dev)
 
     def step():
-        b.z.copy_(h_z, non_blocking=True)
-        b.logp_old.copy_(h_lpo, non_blocking=True)
-        b.rewards.copy_(h_rw, non_blocking=True)
+        if host:
+            b.z.copy_(h_z, non_blocking=True)
+            b.logp_old.copy_(h_lpo, non_blocking=True)
+            b.rewards.copy_(h_rw, non_blocking=True)
         for w in range(nw):
             zw = b.z[:, w * W:(w + 1) * W].reshape(G, W, *b.shape)
             z_end[w * 2 * G:w * 2 * G + G].copy_(zw[:, 0])
@@ -687,13 +706,91 @@ def run_e2e(b, args, ws, routes):
                 vw[:, 1:W - 1].copy_(v_mid[w * (W - 2) * G:(w + 1) * (W - 2) * G].reshape(G, W - 2, -1))
             # Phases 2-3
             b.signals(w, b.lpo_win[w], cot_out=b.cot_all[w * 2 * G:(w + 1) * 2 * G])
-            h_lpn[:, w * W:(w + 1) * W].copy_(b.sig_out["logp_new"], non_blocking=True)
+            if host:
+                h_lpn[:, w * W:(w + 1) * W].copy_(b.sig_out["logp_new"], non_blocking=True)
         # Phase 4 for the whole group
         jg.dit_joint_vjp(b.model, saved, B, b.cot_all[:B], b.grad, b.ws)
         jg.grad_reduce(b.grad, None, out3=b.out3, ws=b.gws)
-        h_out3.copy_(b.out3, non_blocking=True)
-        torch.cuda.current_stream().synchronize()
+        if host:
+            h_out3.copy_(b.out3, non_blocking=True)
+            torch.cuda.current_stream().synchronize()
 
+    h2d = h_z.numel() * 4 + h_lpo.numel() * 8 + h_rw.numel() * 4
+    d2h = h_lpn.numel() * 8 + h_out3.numel() * 8
+    return step, h2d, d2h
+
+
+def full_w_update(b):
+    """The exact per-step update stage of one group (jagg_frac = 0): the forward with saves of
+    every step of every window, each step's own signal, one VJP over all W*G rows of every
+    window, the gradient norm.  Returns the step, or None when its saved activations do
+    not fit."""
+    jg, wl, dev = b.jg, b.wl, b.dev
+    G, W, D = wl.G, wl.W, b.D
+    full = [0] * b.nw
+    if not b.fits(full):
+        return None
+    B = b.nw * W * G
+    saved = jg.alloc_bytes(b.model.saved_bytes(B), dev)
+    z_all = torch.empty(B, *b.shape, dtype=b.tdt, device=dev)
+    v_all = torch.empty(B, *b.shape, dtype=b.tdt, device=dev)
+    t_all = torch.tensor(np.concatenate([np.tile(b.t[w * W:(w + 1) * W], G) for w in range(b.nw)]),
+                         dtype=torch.float32, device=dev)
+    txt = b.txt_rows(B)
+
+    def step():
+        for w in range(b.nw):      # sample-major rows of each window, matching s [G, W, D]
+            z_all[w * W * G:(w + 1) * W * G].copy_(b.z[:, w * W:(w + 1) * W].reshape(G * W, *b.shape))
+        jg.dit_forward_save(b.model, z_all, t_all, txt, v_all, saved=saved, ws=b.ws)
+        for w in range(b.nw):
+            b.z_win[w].copy_(b.z[:, w * W:w * W + W + 1])
+            b.v_win[w].copy_(v_all[w * W * G:(w + 1) * W * G].reshape(G, W, D))
+            b.signals(w, b.lpo_win[w], s_out=b.cot_all[w * W * G:(w + 1) * W * G].view(G, W, D))
+        jg.dit_joint_vjp(b.model, saved, B, b.cot_all[:B], b.grad, b.ws)
+        jg.grad_reduce(b.grad, None, out3=b.out3, ws=b.gws)
+    return step
+
+
+def update_stage(b, args, ws, use_graph):
+    """The update time the paper reports for its efficiency analysis (forwards on the stored
+    experience + backward), device-resident, JAGG against the exact per-step path."""
+    wl = b.wl
+    units = wl.G * wl.T
+    step, _, _ = jagg_update(b, host=False)
+    ms_j, graph = time_steps(step, args.steps, args.warmup, ws, use_graph)
+    del graph, step
+    torch.cuda.empty_cache()
+    out = {"jagg": {"value": ws * units / (ms_j / 1000.0), "unit": UNIT, "ms_per_step": max_over_ranks(ms_j, ws)}}
+    fstep = full_w_update(b)
+    if fstep is not None:
+        ms_f, graph = time_steps(fstep, args.steps, args.warmup, ws, use_graph)
+        del graph, fstep
+        torch.cuda.empty_cache()
+        out["full_w"] = {"value": ws * units / (ms_f / 1000.0), "unit": UNIT, "ms_per_step": max_over_ranks(ms_f, ws)}
+        out["speedup"] = ms_f / ms_j
+        # forward = 1 unit, backward = 2: W * 3 units exact against W + 2 * 2 with JAGG
+        out["ideal_speedup"] = 3.0 * wl.W / (wl.W + 4.0)
+    out["scope"] = ("per group: the forwards on the stored trajectories (JAGG: endpoints saved, middle steps "
+                    "without; exact: every step saved), the step signals, the VJP(s), the gradient norm")
+    return out
+
+
+def rollout_leg(b, args, ws, use_graph):
+    """The rollout sampler on the device: per step the G forwards without saves and the fused
+    sampler step; G * T trajectory-steps per run."""
+    wl = b.wl
+    run, _, _, _ = b.sampler()
+    ms, graph = time_steps(run, args.steps, args.warmup, ws, use_graph)
+    del graph
+    return {"value": ws * wl.G * wl.T / (ms / 1000.0), "unit": "trajectory-steps/s (sampled)",
+            "ms_per_step": max_over_ranks(ms, ws)}
+
+
+def run_e2e(b, args, ws, routes):
+    """The JAGG update stage through the public API from pinned host buffers (jagg_update
+    with host=True), timed on the host clock."""
+    wl = b.wl
+    step, h2d, d2h = jagg_update(b, host=True)
     steps = max(2, args.steps // 2)
     for _ in range(max(1, args.warmup // 2)):
         step()
@@ -702,8 +799,6 @@ def run_e2e(b, args, ws, routes):
     for _ in range(steps):
         step()
     sec = max_over_ranks((time.perf_counter() - t0) / steps, ws)
-    h2d = h_z.numel() * 4 + h_lpo.numel() * 8 + h_rw.numel() * 4
-    d2h = h_lpn.numel() * 8 + h_out3.numel() * 8
     return {"value": ws * wl.G * wl.T / sec, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "ms_per_step": 1000 * sec, "steps": steps,
             "includes": "Phase 1 forwards (2G rows saved + (W-2)G rows unsaved per window), signals, one joint VJP"}

@@ -11,6 +11,7 @@
  *                      (grpo_step_signals_eps: the same for an epsilon-prediction model)
  *   jagg_aggregate     Phase 3: Eq. alpha and Eq. s_base_corr
  *   jagg_route         jagg_frac routing (Sec. 3.3 and the gradient-quality appendix)
+ *   jagg_rollout_step  one rollout sampler step with the log-prob of its sample
  *   dit_joint_vjp      Phase 4: grad += sum_rows J(z_row, t_row)^T cot_row
  *   grad_reduce        gradient accumulation and the cosine / norm-ratio reductions
  *
@@ -265,6 +266,34 @@ int jagg_aggregate(const float* s, const double* t_window, int G, int W, int64_t
  *   cot      device [2G, D] f32, overwritten (accumulate = 0) or added to (accumulate != 0) */
 int jagg_aggregate_span(const float* s, int64_t s_sample_stride, const double* t_steps, double t_first,
                         double t_last, int G, int n, int64_t D, float* cot, int accumulate, cudaStream_t stream);
+
+/* One step of the rollout sampler (the stochastic transition that Eq. logprob scores, Sec. 3.1
+ * and Sec. 3.2), fused with the log-probability of the sample it draws (the rollout's old
+ * log-prob that Eq. grpo_loss divides by):
+ *   z_next_i = mu_i + sigma xi_i,  mu_i = a z_cur_i + c y_i,  stored in f32;
+ *   logp_i   = -||z_next_i - mu_i||^2 / (2 sigma^2) - D log(sqrt(2 pi) sigma)
+ * with (a, c) = (1, t_next - t_cur) for a rectified-flow velocity y (Euler-Maruyama step),
+ * or the DDIM step of grpo_step_signals_eps for a noise prediction y when sched is given.
+ * The residual and its sum are evaluated by the same device code as grpo_step_signals, so
+ * scoring the stored step there with the same y gives exactly this logp (ratio exactly 1).
+ *   y_hat    device [G, D] (y_dtype) model outputs at z_cur, row i at y_hat + i * y_sample_stride
+ *   z_cur    device f32, row i at z_cur + i * z_sample_stride; z_next likewise (may be the next
+ *            step of the same [G, T+1, D] trajectory buffer: z_sample_stride = (T+1) D)
+ *   xi       device f32 standard-normal draws, row i at xi + i * xi_sample_stride
+ *            (a stride of 0 means D for y_hat, z and xi)
+ *   t_cur, t_next, sigma  host f64 (sigma > 0)
+ *   sched    host [4] f64 = {alpha_cur, alpha_next, sigma_cur, sigma_next} or NULL (flow);
+ *            an alpha <= 0 sets JAGG_DEV_STATUS_BADARG (outputs then meaningless)
+ *   logp     device f64, sample i at logp[i * logp_stride]
+ *   z_model  device [G, D] (z_model_dtype) or NULL: z_next rounded to the model's storage type,
+ *            the input of the next step's forward
+ *   ws       device workspace of >= jagg_rollout_workspace_bytes(G, D) bytes            */
+int64_t jagg_rollout_workspace_bytes(int G, int64_t D);
+int jagg_rollout_step(const void* y_hat, int y_dtype, int64_t y_sample_stride, const float* z_cur,
+                      float* z_next, int64_t z_sample_stride, const float* xi, int64_t xi_sample_stride,
+                      int G, int64_t D, double t_cur, double t_next, double sigma, const double* sched,
+                      double* logp, int64_t logp_stride, void* z_model, int z_model_dtype, void* ws,
+                      size_t ws_bytes, cudaStream_t stream);
 
 /* jagg_frac routing (Sec. 3.3 "High-noise vs. low-noise scheduling"; rule of the
  * gradient-quality appendix).  Host-only, synchronous.

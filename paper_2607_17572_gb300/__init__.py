@@ -101,6 +101,9 @@ _SIGNATURES = {
                                _P, _P, _P, _SZ, _P]),
     "grpo_step_signals_eps": (_I, [_P, _I, _P, _P, _P, _P, _P, _P, _P, _I, _I, _I64, _D, _D, _D, _D, _P, _P, _P,
                                    _P, _P, _P, _P, _SZ, _P]),
+    "jagg_rollout_workspace_bytes": (_I64, [_I, _I64]),
+    "jagg_rollout_step": (_I, [_P, _I, _I64, _P, _P, _I64, _P, _I64, _I, _I64, _D, _D, _D, _P, _P, _I64, _P, _I,
+                               _P, _SZ, _P]),
     "grpo_step_signals_static": (_I, [_P, _I, _P, _P, _P, _P, _P, _I, _I, _I64, _D, _D, _D, _D, _P, _P, _P, _P,
                                       _P, _P, _P]),
     "jagg_aggregate": (_I, [_P, _P, _I, _I, _I64, _P, _P]),
@@ -302,6 +305,33 @@ def grpo_step_signals_static(v_hat, z, t, sigma, logp_old, rewards, clip_eps, ad
                                           _ptr(rewards), G, W, D, clip_eps, adv_clip, adv_eps, scale, _ptr(s_out),
                                           _ptr(cot_out), _ptr(logp_new), _ptr(ratio), _ptr(clipped), _ptr(adv_out),
                                           _stream(stream)), "grpo_step_signals_static")
+
+
+def rollout_workspace_bytes(G: int, D: int) -> int:
+    return lib().jagg_rollout_workspace_bytes(G, D)
+
+
+def jagg_rollout_step(y_hat, z, j: int, xi, t_cur: float, t_next: float, sigma: float, logp, ws, sched=None,
+                      z_model=None, stream=None):
+    """One sampler step of G trajectories in place: z [G, T+1, ...] f32 (step j -> j+1),
+    y_hat [G, ...] model outputs at z[:, j], xi [G, ...] f32 noise, logp [G, T] f64 (column j
+    written).  sched = (alpha_cur, alpha_next, sigma_cur, sigma_next) for a noise-prediction
+    model, None for a velocity model.  z_model [G, ...] (bf16 or f32), if given, receives
+    z[:, j+1] in its dtype (the next forward's input)."""
+    _need_cuda(y_hat, z, xi, logp, ws, z_model)
+    G = z.shape[0]
+    D = z[0, 0].numel()
+    assert z.is_contiguous() and y_hat.is_contiguous() and xi.is_contiguous() and logp.is_contiguous()
+    assert y_hat[0].numel() == D and xi[0].numel() == D and 0 <= j < z.shape[1] - 1
+    es = z.element_size()
+    zc = z.data_ptr() + j * D * es
+    yd = DTYPE_BF16 if y_hat.dtype == torch.bfloat16 else DTYPE_F32
+    sch = (_D * 4)(*[float(x) for x in sched]) if sched is not None else None
+    _check(lib().jagg_rollout_step(_ptr(y_hat), yd, D, zc, zc + D * es, z.shape[1] * D, _ptr(xi), D, G, D,
+                                   float(t_cur), float(t_next), float(sigma), sch, logp.data_ptr() + j * 8,
+                                   logp.shape[1], _ptr(z_model),
+                                   DTYPE_BF16 if z_model is not None and z_model.dtype == torch.bfloat16
+                                   else DTYPE_F32, _ptr(ws), ws.numel(), _stream(stream)), "jagg_rollout_step")
 
 
 def jagg_aggregate(s, t_window, cot, stream=None):

@@ -54,24 +54,38 @@ __device__ __forceinline__ float resid(float z1, float z0, float y, Coef2 a, Coe
   return fmaf(-c.lo, y, r);
 }
 
+// The mean coefficients (a_j, c_j) of one step: the flow Euler step, or (eps) the DDIM step
+// of the schedule values a0 = alpha_j, a1 = alpha_{j+1}, s0 = sigma_j, s1 = sigma_{j+1}.
+// False (and a = c = 0) when an alpha is not positive.  The step signals and the rollout
+// sampler both take their coefficients from here, so both see the same f64 values.
+__device__ __forceinline__ bool mean_coef(double t0, double t1, bool eps, double a0, double a1, double s0, double s1,
+                                          double* a, double* c) {
+  if (!eps) {
+    *a = 1.0;
+    *c = t1 - t0;
+    return true;
+  }
+  if (a0 > 0.0 && a1 > 0.0) {
+    *a = a1 / a0;
+    *c = -a1 * (s0 / a0 - s1 / a1);
+    return true;
+  }
+  *a = 0.0;
+  *c = 0.0;
+  return false;
+}
+
 // One warp.  Lane 0: the advantages.  All lanes: the mean coefficients mc[j] = a_j,
 // mc[W + j] = c_j; sched_alpha == nullptr selects the rectified-flow step.
 __global__ void prep_kernel(const float* rewards, int G, double adv_eps, double adv_clip, double* adv, const double* t,
                             const double* sched_alpha, const double* sched_sigma, int W, double* mc) {
   if (blockIdx.x != 0) return;
   for (int j = threadIdx.x; j < W; j += 32) {
-    double a = 1.0, c = t[j + 1] - t[j];
-    if (sched_alpha) {
-      const double a0 = sched_alpha[j], a1 = sched_alpha[j + 1];
-      if (a0 > 0.0 && a1 > 0.0) {
-        a = a1 / a0;
-        c = -a1 * (sched_sigma[j] / a0 - sched_sigma[j + 1] / a1);
-      } else {
-        set_device_status(JAGG_DEV_BADARG);
-        a = 0.0;
-        c = 0.0;
-      }
-    }
+    const bool eps = sched_alpha != nullptr;
+    double a, c;
+    if (!mean_coef(t[j], t[j + 1], eps, eps ? sched_alpha[j] : 0.0, eps ? sched_alpha[j + 1] : 0.0,
+                   eps ? sched_sigma[j] : 0.0, eps ? sched_sigma[j + 1] : 0.0, &a, &c))
+      set_device_status(JAGG_DEV_BADARG);
     mc[j] = a;
     mc[W + j] = c;
   }
@@ -92,15 +106,11 @@ __global__ void prep_kernel(const float* rewards, int G, double adv_eps, double 
   }
 }
 
-// grid: (chunks, G*W)
-__global__ void __launch_bounds__(SIG_THREADS) resid_norm_kernel(const void* v, int v_f32, const float* z,
-                                                                 const double* mc, int W, int64_t D, double* partial) {
-  const int ij = blockIdx.y;
-  const int i = ij / W, j = ij % W;
-  const Coef2 a = split_coef(mc[j]), c = split_coef(mc[W + j]);
-  const float* z0 = z + ((int64_t)i * (W + 1) + j) * D;
-  const float* z1 = z0 + D;
-  const int64_t vb = ((int64_t)i * W + j) * D;
+// sum of r(k)^2 over the CTA's chunk of D (k = blockIdx.x * SIG_CHUNK + ...), valid in thread
+// 0: f32 partial sums folded into f64 every 8 terms, then a fixed-order block reduction.  The
+// rollout sampler and the step signals share it, so equal residuals give equal log-probs.
+template <class R>
+__device__ __forceinline__ double chunk_sq_sum(int64_t D, R r_at) {
   const int64_t k0 = (int64_t)blockIdx.x * SIG_CHUNK;
   double acc = 0.0;
   float part = 0.f;
@@ -108,7 +118,7 @@ __global__ void __launch_bounds__(SIG_THREADS) resid_norm_kernel(const void* v, 
   for (int u = 0; u < SIG_PER_THREAD; ++u) {
     const int64_t k = k0 + threadIdx.x + (int64_t)u * SIG_THREADS;
     if (k < D) {
-      const float r = resid(z1[k], z0[k], ldv_any(v, vb + k, v_f32), a, c);
+      const float r = r_at(k);
       part = fmaf(r, r, part);
     }
     if ((u & 7) == 7) {  // fold every 8 terms into the f64 accumulator
@@ -121,11 +131,33 @@ __global__ void __launch_bounds__(SIG_THREADS) resid_norm_kernel(const void* v, 
   __shared__ double red[SIG_THREADS / 32];
   if ((threadIdx.x & 31) == 0) red[threadIdx.x / 32] = acc;
   __syncthreads();
-  if (threadIdx.x == 0) {
-    double s = 0.0;
+  double s = 0.0;
+  if (threadIdx.x == 0)
     for (int w = 0; w < SIG_THREADS / 32; ++w) s += red[w];
-    partial[(int64_t)ij * gridDim.x + blockIdx.x] = s;
-  }
+  return s;
+}
+
+// Eq. logprob from the squared residual norm.  Written with explicitly rounded operations so
+// that no call site contracts it into a different fused multiply-add: the rollout sampler
+// and the step signals must agree to the last bit.
+__device__ __forceinline__ double gauss_logp(double rr, double sg, int64_t D) {
+  const double quad = __ddiv_rn(rr, __dmul_rn(2.0, __dmul_rn(sg, sg)));
+  const double norm = __dmul_rn((double)D, log(__dmul_rn(sqrt(2.0 * 3.14159265358979323846), sg)));
+  return __dsub_rn(-quad, norm);
+}
+
+// grid: (chunks, G*W)
+__global__ void __launch_bounds__(SIG_THREADS) resid_norm_kernel(const void* v, int v_f32, const float* z,
+                                                                 const double* mc, int W, int64_t D, double* partial) {
+  const int ij = blockIdx.y;
+  const int i = ij / W, j = ij % W;
+  const Coef2 a = split_coef(mc[j]), c = split_coef(mc[W + j]);
+  const float* z0 = z + ((int64_t)i * (W + 1) + j) * D;
+  const float* z1 = z0 + D;
+  const int64_t vb = ((int64_t)i * W + j) * D;
+  const double s =
+      chunk_sq_sum(D, [&](int64_t k) { return resid(z1[k], z0[k], ldv_any(v, vb + k, v_f32), a, c); });
+  if (threadIdx.x == 0) partial[(int64_t)ij * gridDim.x + blockIdx.x] = s;
 }
 
 // One thread per (i, j).
@@ -139,7 +171,7 @@ __global__ void logprob_kernel(const double* partial, int chunks, const double* 
   for (int c = 0; c < chunks; ++c) rr += partial[(int64_t)ij * chunks + c];
   const double sg = sigma[j];
   const double c = mc[W + j];
-  const double lp = -rr / (2.0 * sg * sg) - (double)D * log(sqrt(2.0 * 3.14159265358979323846) * sg);
+  const double lp = gauss_logp(rr, sg, D);
   const double rho = exp(lp - logp_old[ij]);
   const double a = adv[i];
   const bool clip = (a > 0.0 && rho > 1.0 + clip_eps) || (a < 0.0 && rho < 1.0 - clip_eps);
@@ -187,6 +219,61 @@ __global__ void __launch_bounds__(SIG_THREADS) apply_kernel(const void* v, int v
       }
     }
   }
+}
+
+// Rollout sampler step.  grid: (chunks, G).  z_{j+1} = a z_j + c y + sigma xi, rounded to f32
+// and stored, then its residual against the mean enters the same chunk sums as the signals.
+struct RolloutStep {
+  const void* y;
+  int y_f32;
+  const float* z_cur;
+  const float* xi;
+  float* z_next;
+  void* z_model;  // optional dense [G, D] copy of z_next in the model's dtype (next forward's input)
+  int zm_f32;
+  int64_t D, z_ld, y_ld, xi_ld;
+  double t0, t1, sigma, a0, a1, s0, s1;
+  int eps;
+  double* partial;
+};
+
+__global__ void __launch_bounds__(SIG_THREADS) rollout_step_kernel(RolloutStep p) {
+  const int i = blockIdx.y;
+  double ad, cd;
+  if (!mean_coef(p.t0, p.t1, p.eps != 0, p.a0, p.a1, p.s0, p.s1, &ad, &cd) && blockIdx.x == 0 && i == 0 &&
+      threadIdx.x == 0)
+    set_device_status(JAGG_DEV_BADARG);
+  const Coef2 a = split_coef(ad), c = split_coef(cd);
+  const float sg = (float)p.sigma;
+  const float* z0 = p.z_cur + (int64_t)i * p.z_ld;
+  float* z1 = p.z_next + (int64_t)i * p.z_ld;
+  const float* xi = p.xi + (int64_t)i * p.xi_ld;
+  const int64_t yb = (int64_t)i * p.y_ld;
+  const double s = chunk_sq_sum(p.D, [&](int64_t k) {
+    const float zk = z0[k], yk = ldv_any(p.y, yb + k, p.y_f32);
+    float m = fmaf(a.lo, zk, c.lo * yk);
+    m = fmaf(c.hi, yk, m);
+    m = fmaf(a.hi, zk, m);
+    const float zn = fmaf(sg, xi[k], m);
+    z1[k] = zn;
+    if (p.z_model) {
+      if (p.zm_f32)
+        static_cast<float*>(p.z_model)[(int64_t)i * p.D + k] = zn;
+      else
+        static_cast<bf16*>(p.z_model)[(int64_t)i * p.D + k] = __float2bfloat16_rn(zn);
+    }
+    return resid(zn, zk, yk, a, c);
+  });
+  if (threadIdx.x == 0) p.partial[(int64_t)i * gridDim.x + blockIdx.x] = s;
+}
+
+__global__ void rollout_logp_kernel(const double* partial, int chunks, double sigma, int G, int64_t D,
+                                    double* logp, int64_t logp_ld) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= G) return;
+  double rr = 0.0;
+  for (int c = 0; c < chunks; ++c) rr += partial[(int64_t)i * chunks + c];
+  logp[(int64_t)i * logp_ld] = gauss_logp(rr, sigma, D);
 }
 
 __global__ void check_alpha_kernel(const double* t, int W) {
@@ -395,6 +482,45 @@ extern "C" int grpo_step_signals_eps(const void* eps_hat, int eps_dtype, const f
   return step_signals("grpo_step_signals_eps", eps_hat, eps_dtype, z, t, sched_alpha, sched_sigma, sigma, logp_old,
                       rewards, G, W, D, clip_eps, adv_clip, adv_eps, scale, s_out, cot_out, logp_new, ratio, clipped,
                       adv_out, ws, ws_bytes, stream);
+}
+
+extern "C" int64_t jagg_rollout_workspace_bytes(int G, int64_t D) {
+  if (G <= 0 || D <= 0) return 0;
+  return (int64_t)G * ((D + SIG_CHUNK - 1) / SIG_CHUNK) * 8 + 64;
+}
+
+extern "C" int jagg_rollout_step(const void* y_hat, int y_dtype, int64_t y_sample_stride, const float* z_cur,
+                                 float* z_next, int64_t z_sample_stride, const float* xi, int64_t xi_sample_stride,
+                                 int G, int64_t D, double t_cur, double t_next, double sigma, const double* sched,
+                                 double* logp, int64_t logp_stride, void* z_model, int z_model_dtype, void* ws,
+                                 size_t ws_bytes, cudaStream_t stream) {
+  JAGG_CHECK_ARG(y_hat && z_cur && z_next && xi && logp && ws, "jagg_rollout_step: null pointer");
+  JAGG_CHECK_ARG(G > 0 && G <= 65535 && D > 0, "jagg_rollout_step: bad G=%d or D=%lld", G, (long long)D);
+  JAGG_CHECK_ARG(y_dtype == JAGG_DTYPE_F32 || y_dtype == JAGG_DTYPE_BF16, "jagg_rollout_step: bad y_dtype");
+  JAGG_CHECK_ARG(sigma > 0.0, "jagg_rollout_step: sigma %g must be positive", sigma);
+  const int64_t zl = z_sample_stride ? z_sample_stride : D, yl = y_sample_stride ? y_sample_stride : D,
+                xl = xi_sample_stride ? xi_sample_stride : D;
+  JAGG_CHECK_ARG(zl >= D && yl >= D && xl >= D, "jagg_rollout_step: a sample stride is below D");
+  JAGG_CHECK_ARG(logp_stride >= 1, "jagg_rollout_step: logp_stride must be >= 1");
+  JAGG_CHECK_ARG(!z_model || z_model_dtype == JAGG_DTYPE_F32 || z_model_dtype == JAGG_DTYPE_BF16,
+                 "jagg_rollout_step: bad z_model_dtype");
+  const int64_t need = jagg_rollout_workspace_bytes(G, D);
+  if ((int64_t)ws_bytes < need) {
+    set_last_error("jagg_rollout_step: workspace %zu < %lld bytes", ws_bytes, (long long)need);
+    return JAGG_ERR_WORKSPACE;
+  }
+  JAGG_CHECK_ARG(aligned16(ws), "jagg_rollout_step: workspace not 16-byte aligned");
+  const int chunks = (int)((D + SIG_CHUNK - 1) / SIG_CHUNK);
+  RolloutStep p{y_hat, y_dtype == JAGG_DTYPE_F32, z_cur, xi, z_next, z_model, z_model_dtype == JAGG_DTYPE_F32,
+                D, zl, yl, xl, t_cur, t_next, sigma,
+                sched ? sched[0] : 0.0, sched ? sched[1] : 0.0, sched ? sched[2] : 0.0, sched ? sched[3] : 0.0,
+                sched ? 1 : 0, static_cast<double*>(ws)};
+  rollout_step_kernel<<<dim3(chunks, G), SIG_THREADS, 0, stream>>>(p);
+  JAGG_LAUNCHED();
+  rollout_logp_kernel<<<ceil_div((int64_t)G, 128), 128, 0, stream>>>(static_cast<double*>(ws), chunks, sigma, G, D,
+                                                                      logp, logp_stride);
+  JAGG_LAUNCHED();
+  return JAGG_OK;
 }
 
 extern "C" int jagg_aggregate(const float* s, const double* t_window, int G, int W, int64_t D, float* cot,

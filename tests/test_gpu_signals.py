@@ -227,3 +227,111 @@ def test_span_aggregation_and_ablation_match_oracle(G, W, D):
     assert torch.equal(ab, ab2)
     with pytest.raises(jg.JaggError):
         jg.jagg_aggregate_span(ends, torch.tensor([t[0], t[0]], **f64), t[0], t[0], ab)
+
+
+# ------------------------------------------------------------------ rollout sampler step
+from oracle import rollout as oracle_rollout  # noqa: E402
+
+
+def _sched(eps_model, t):
+    if not eps_model:
+        return None
+    al, sg = synth.vp_schedule(np.asarray(t))
+    return al, sg
+
+
+@pytest.mark.parametrize("G,T,D,y_dtype,eps_model", [
+    (4, 3, 64, "f32", False),
+    (8, 4, 16384, "bf16", False),      # DiT-B latent
+    (3, 2, 12345, "bf16", True),       # ragged D, noise prediction
+    (5, 3, 8193, "f32", True),         # D one past a CTA chunk
+])
+def test_rollout_step_matches_oracle(G, T, D, y_dtype, eps_model):
+    """jagg_rollout_step against the oracle's sampler step, writing step j -> j+1 of a
+    [G, T+1, D] trajectory buffer in place: the stored sample to float32 rounding of the
+    f32 mean, the log-prob with the signals' bar."""
+    dev = "cuda"
+    rng = np.random.Generator(np.random.PCG64(G * 31 + D))
+    t = synth.time_grid(4 * T, 3.0)[T:2 * T + 1] * 0.9 + 0.05
+    sig = synth.sigma_schedule(t, 0.7)
+    sch = _sched(eps_model, t)
+    z = torch.zeros(G, T + 1, D, device=dev)
+    z[:, 0] = torch.tensor(rng.standard_normal((G, D)), dtype=torch.float32, device=dev)
+    logp = torch.full((G, T), float("nan"), dtype=torch.float64, device=dev)
+    ws = jg.alloc_bytes(jg.rollout_workspace_bytes(G, D))
+    jg.device_status(clear=True)
+    for j in range(T):
+        y = synth.storage_round(rng.standard_normal((G, D)), y_dtype)
+        xi = rng.standard_normal((G, D)).astype(np.float32)
+        sched_j = None if sch is None else (sch[0][j], sch[0][j + 1], sch[1][j], sch[1][j + 1])
+        z_cur = z[:, j].cpu().numpy().astype(np.float64)
+        yt = torch.tensor(y, dtype=torch.bfloat16 if y_dtype == "bf16" else torch.float32, device=dev)
+        zm = torch.empty(G, D, dtype=torch.bfloat16, device=dev)
+        jg.jagg_rollout_step(yt, z, j, torch.tensor(xi, device=dev), t[j], t[j + 1], sig[j], logp, ws, sched=sched_j,
+                             z_model=zm)
+        torch.cuda.synchronize()
+        assert torch.equal(zm, z[:, j + 1].bfloat16())      # the next forward's input, RNE-rounded
+        zn_o, lp_o = oracle_rollout.sampler_step(z_cur, y, xi, t[j], t[j + 1], sig[j], sched_j)
+        zn = z[:, j + 1].cpu().numpy().astype(np.float64)
+        assert np.max(np.abs(zn - zn_o)) <= 4e-7 * max(1.0, np.abs(zn_o).max())
+        # the log-prob of the sample the GPU stored, by the oracle's Eq. logprob
+        if sched_j is None:
+            lp_ref = [grpo.step_logprob(zn[i], z_cur[i], y[i], t[j], t[j + 1], sig[j]) for i in range(G)]
+        else:
+            lp_ref = [grpo.step_logprob_eps(zn[i], z_cur[i], y[i], *sched_j, sig[j]) for i in range(G)]
+        lp_tol = 1e-6 * max(10.0, D / 50)
+        lp = logp[:, j].cpu().numpy()
+        assert np.max(np.abs(lp - np.array(lp_ref))) < lp_tol
+        # and the oracle's own sample scores alike (the two samples differ by f32 roundings)
+        assert np.max(np.abs(lp - lp_o)) < lp_tol + 1e-3
+    assert jg.device_status() == 0
+
+
+@pytest.mark.parametrize("eps_model", [False, True])
+def test_rollout_logprobs_are_reproduced_exactly_by_the_step_signals(eps_model):
+    """theta = theta_old: scoring the stored rollout with the same model outputs gives the
+    rollout's own log-probs bit for bit, so every ratio is exactly 1 and no step is clipped."""
+    dev = "cuda"
+    G, W, D = 6, 4, 20000
+    rng = np.random.Generator(np.random.PCG64(11 + eps_model))
+    t = synth.time_grid(4 * W, 3.0)[W:2 * W + 1] * 0.9 + 0.05
+    sig = synth.sigma_schedule(t, 0.7)
+    sch = _sched(eps_model, t)
+    f64 = dict(dtype=torch.float64, device=dev)
+    z = torch.zeros(G, W + 1, D, device=dev)
+    z[:, 0] = torch.tensor(rng.standard_normal((G, D)), dtype=torch.float32, device=dev)
+    y = torch.tensor(rng.standard_normal((G, W, D)), dtype=torch.bfloat16, device=dev)
+    xi = torch.tensor(rng.standard_normal((G, W, D)), dtype=torch.float32, device=dev)
+    logp = torch.empty(G, W, **f64)
+    ws = jg.alloc_bytes(jg.rollout_workspace_bytes(G, D))
+    for j in range(W):
+        sched_j = None if sch is None else (sch[0][j], sch[0][j + 1], sch[1][j], sch[1][j + 1])
+        jg.jagg_rollout_step(y[:, j].contiguous(), z, j, xi[:, j].contiguous(), t[j], t[j + 1], sig[j], logp, ws,
+                             sched=sched_j)
+    out = dict(logp_new=torch.empty(G, W, **f64), ratio=torch.empty(G, W, **f64),
+               clipped=torch.empty(G, W, dtype=torch.uint8, device=dev), adv_out=torch.empty(G, **f64))
+    sws = jg.alloc_bytes(jg.signals_workspace_bytes(G, W, D))
+    rewards = torch.tensor(rng.standard_normal(G), dtype=torch.float32, device=dev)
+    args = (torch.tensor(sig[:W], **f64), logp, rewards, 0.1, 5.0, 1e-8, 1.0)
+    if eps_model:
+        jg.grpo_step_signals_eps(y, z, torch.tensor(t, **f64), torch.tensor(sch[0], **f64),
+                                 torch.tensor(sch[1], **f64), *args, ws=sws, **out)
+    else:
+        jg.grpo_step_signals(y, z, torch.tensor(t, **f64), *args, ws=sws, **out)
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    assert torch.equal(out["logp_new"], logp)
+    assert torch.all(out["ratio"] == 1.0)
+    assert not out["clipped"].any()
+
+
+def test_rollout_step_rejects_bad_arguments():
+    dev = "cuda"
+    z = torch.zeros(2, 3, 10, device=dev)
+    y = torch.zeros(2, 10, device=dev)
+    logp = torch.empty(2, 2, dtype=torch.float64, device=dev)
+    ws = jg.alloc_bytes(jg.rollout_workspace_bytes(2, 10))
+    with pytest.raises(jg.JaggError):
+        jg.jagg_rollout_step(y, z, 0, y, 0.5, 0.4, 0.0, logp, ws)     # sigma must be positive
+    with pytest.raises(jg.JaggError):
+        jg.jagg_rollout_step(y, z, 0, y, 0.5, 0.4, 0.1, logp, jg.alloc_bytes(8))   # workspace too small
