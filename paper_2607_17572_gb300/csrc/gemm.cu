@@ -182,6 +182,7 @@ enum : int { STAGED_NONE = 0, STAGED_STORE = 1, STAGED_MUL_AUX = 2, STAGED_ACCUM
 
 struct TcParams {
   int tiles_m, tiles_n, splits, k_blocks;
+  int raster_n;  // 1: consecutive tile indices walk N first (see tile_order)
   int staged;  // STAGED_*
   EpiParams e;
 };
@@ -269,12 +270,19 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
   const uint32_t tmem_base = *tmem_slot;
 
   const int total = p.tiles_m * p.tiles_n * p.splits;
-  // tile index -> (m tile, n tile, split); m fastest so consecutive CTAs share B tiles.
+  // tile index -> (m tile, n tile, split), the faster of m and n chosen by the host.
   auto decode = [&](int t, int& tm, int& tn, int& ks) {
-    tm = t % p.tiles_m;
-    int r = t / p.tiles_m;
-    tn = r % p.tiles_n;
-    ks = r / p.tiles_n;
+    if (p.raster_n) {
+      tn = t % p.tiles_n;
+      const int r = t / p.tiles_n;
+      tm = r % p.tiles_m;
+      ks = r / p.tiles_m;
+    } else {
+      tm = t % p.tiles_m;
+      const int r = t / p.tiles_m;
+      tn = r % p.tiles_n;
+      ks = r / p.tiles_n;
+    }
   };
   auto krange = [&](int ks, int& kb0, int& kb1) {
     kb0 = (int)((long long)p.k_blocks * ks / p.splits);
@@ -804,6 +812,13 @@ double tile_cost(const GemmArgs& g, int BN, int nsm) {
   return waves * BN * ((double)ceil_div(g.K, TC_BK) / splits) / eff;
 }
 
+// Tile order.  The CTAs resident at one time work on consecutive tile indices, so the
+// operand panel that those tiles share is read from DRAM once and from L2 after that.  With
+// N fastest, tiles_n neighbours share one 128-row panel of A; with M fastest, tiles_m
+// neighbours share one panel of B.  Sharing the panel of the larger operand saves the
+// more DRAM traffic: the tall products (rows x d outputs, A = activations) walk N first.
+int tile_order_n_first(const GemmArgs& g) { return (long long)g.M > (long long)g.N ? 1 : 0; }
+
 // Which staged epilogue (if any) serves the product: row-major outputs without row remap,
 // 16-byte aligned with 16-byte row pitches.
 int staged_mode(const GemmArgs& g) {
@@ -870,6 +885,7 @@ int launch_tc(const GemmArgs& g, cudaStream_t stream) {
   p.tiles_m = ceil_div(g.M, TC_BM);
   p.tiles_n = ceil_div(g.N, BN);
   p.k_blocks = ceil_div(g.K, TC_BK);
+  p.raster_n = tile_order_n_first(g);
   const int nsm = sm_count();
   p.splits = choose_splits(g, BN, nsm);
   p.e = make_epi(g);
