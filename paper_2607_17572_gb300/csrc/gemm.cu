@@ -788,18 +788,26 @@ EpiParams make_epi(const GemmArgs& g) {
   return e;
 }
 
-// Split-K factor: accumulating products whose tiles do not cover the SMs split K.
+// Split-K factor of an accumulating product (the partial sums meet in the f32 output through
+// reduce-adds): the split count with the fewest waves of units times k-blocks per unit, each
+// unit charged two k-blocks for its pipeline fill and epilogue.  Products with few tiles and a
+// long K (the weight gradients, K = rows) split so that their units fill whole waves.
 int choose_splits(const GemmArgs& g, int BN, int nsm) {
   if (g.epi != EPI_ACCUM) return 1;
   const int k_blocks = ceil_div(g.K, TC_BK);
-  const int tiles = ceil_div(g.M, TC_BM) * ceil_div(g.N, BN);
-  int splits = 1;
-  if (g.split_k > 0)
-    splits = g.split_k;
-  else if (tiles < nsm)
-    splits = (nsm + tiles - 1) / tiles;
-  if (splits > k_blocks) splits = k_blocks;
-  return splits < 1 ? 1 : splits;
+  if (g.split_k > 0) return g.split_k < k_blocks ? g.split_k : k_blocks;
+  const long long tiles = (long long)ceil_div(g.M, TC_BM) * ceil_div(g.N, BN);
+  int best = 1;
+  double best_cost = 0.0;
+  for (int s = 1; s <= k_blocks && s <= 32; ++s) {
+    const double waves = (double)((tiles * s + nsm - 1) / nsm);
+    const double cost = waves * (ceil_div(k_blocks, s) + 2.0);
+    if (s == 1 || cost < 0.999 * best_cost) {
+      best = s;
+      best_cost = cost;
+    }
+  }
+  return best;
 }
 
 // Relative duration of the product with BN-wide tiles: waves of work units times the
