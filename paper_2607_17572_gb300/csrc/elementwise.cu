@@ -340,29 +340,27 @@ __global__ void __launch_bounds__(256, LNF_MIN_BLOCKS) ln_gate_fused_kernel(LnGa
 // once (dm, h, dh, y: 4 float4-wide groups per 128 columns), forms the row statistics
 // with two warp reductions and updates the row without a second pass over dm and h.  The
 // per-sequence column sums go to a warp-private shared-memory slab ([4 quantities][d],
-// plain read-modify-write, no atomics), summed over the block's 8 warps per unit.
-constexpr int LNR_ROWS = 32;  // rows per (sequence, chunk) unit: 4 per warp
+// plain read-modify-write, no atomics), summed over the block's 8 warps and flushed with
+// atomics once per sequence segment.  Each CTA owns a contiguous, equal share of the rows
+// (at most a few sequence segments), so every CTA finishes at the same time.
 template <int NV>
 __global__ void __launch_bounds__(256, 2) ln_gate_rowreg_kernel(LnGateBwd a) {
   extern __shared__ float part[];  // [8 warps][4 quantities][d]
   constexpr int d = 128 * NV;
   const int warp = threadIdx.x / 32, lane = threadIdx.x & 31;
   float* mine = part + warp * 4 * d;
-  const int chunks = (a.rows_per_seq + LNR_ROWS - 1) / LNR_ROWS;
-  const int units = (a.M / a.rows_per_seq) * chunks;
   const int is_f32 = a.dtype == JAGG_DTYPE_F32;
-  for (int unit = blockIdx.x; unit < units; unit += gridDim.x) {
-    const int b = unit / chunks;
-    const int r0 = (unit % chunks) * LNR_ROWS;
+  const int row_begin = (int)((int64_t)a.M * blockIdx.x / gridDim.x);
+  const int row_end = (int)((int64_t)a.M * (blockIdx.x + 1) / gridDim.x);
+  for (int seg0 = row_begin; seg0 < row_end;) {
+    const int b = seg0 / a.rows_per_seq;
+    const int seg1 = min(row_end, (b + 1) * a.rows_per_seq);
     for (int i = lane; i < 4 * d; i += 32) mine[i] = 0.f;
     __syncwarp();
     const float* gate = a.do_gate ? a.gate + (int64_t)b * a.mod_stride : nullptr;
     const float* sc = a.do_ln ? a.scale + (int64_t)b * a.mod_stride : nullptr;
 #pragma unroll 1
-    for (int k = 0; k < 4; ++k) {
-      const int r = r0 + warp * 4 + k;
-      if (r >= a.rows_per_seq) break;
-      const int m = b * a.rows_per_seq + r;
+    for (int m = seg0 + warp; m < seg1; m += 8) {
       const int64_t hr = seg_row(m, a.seg, a.seg_off, a.seg_stride);
       float dm[NV][4], hv[NV][4], dh[NV][4], yv[NV][4];
 #pragma unroll
@@ -447,7 +445,8 @@ __global__ void __launch_bounds__(256, 2) ln_gate_rowreg_kernel(LnGateBwd a) {
         if (a.dbias) atomicAdd(a.dbias + c, gate[c] * P[3]);
       }
     }
-    __syncthreads();  // the slabs are re-zeroed by the next unit
+    __syncthreads();  // the slabs are re-zeroed for the next segment
+    seg0 = seg1;
   }
 }
 
@@ -464,9 +463,10 @@ int launch_ln_gate_rowreg(const LnGateBwd& a, cudaStream_t s) {
     JAGG_CUDA_TRY(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ln_gate_rowreg_kernel<NV>, 256, smem));
     if (per_sm < 1) per_sm = 1;
   }
-  const int units = (a.M / a.rows_per_seq) * ceil_div(a.rows_per_seq, LNR_ROWS);
+  // equal row shares of at least 16 rows per CTA, at most one wave of resident CTAs
   const int cap = per_sm * sm_count();
-  ln_gate_rowreg_kernel<NV><<<units < cap ? units : cap, 256, smem, s>>>(a);
+  const int want = ceil_div(a.M, 16);
+  ln_gate_rowreg_kernel<NV><<<want < cap ? want : cap, 256, smem, s>>>(a);
   JAGG_LAUNCHED();
   return JAGG_OK;
 }
