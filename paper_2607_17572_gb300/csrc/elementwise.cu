@@ -336,96 +336,101 @@ __global__ void __launch_bounds__(256, LNF_MIN_BLOCKS) ln_gate_fused_kernel(LnGa
   }
 }
 
-// Row-in-registers variant for d = 128 NV <= 768: a warp issues every load of one row at
-// once (dm, h, dh, y: 4 float4-wide groups per 128 columns), forms the row statistics
-// with two warp reductions and updates the row without a second pass over dm and h.  The
+// Row-in-registers variant for d = 128 NV <= 768, with the LayerNorm part always present and
+// dm in f32 (GATE: the gate part too; YBF: y and dy in bf16).  A warp issues every load of
+// one row at once (dh, dm, h, y: float4-wide groups per 128 columns), forms the row
+// statistics with two warp reductions and updates the row without a second pass.  The
+// sequence's scale and gate vectors sit in shared memory for the whole segment.  The
 // per-sequence column sums go to a warp-private shared-memory slab ([4 quantities][d],
 // plain read-modify-write, no atomics), summed over the block's 8 warps and flushed with
 // atomics once per sequence segment.  Each CTA owns a contiguous, equal share of the rows
 // (at most a few sequence segments), so every CTA finishes at the same time.
-template <int NV>
+template <int NV, bool GATE, bool YBF>
 __global__ void __launch_bounds__(256, 2) ln_gate_rowreg_kernel(LnGateBwd a) {
-  extern __shared__ float part[];  // [8 warps][4 quantities][d]
+  extern __shared__ float part[];  // [8 warps][4 quantities][d], then scale[d], gate[d]
   constexpr int d = 128 * NV;
   const int warp = threadIdx.x / 32, lane = threadIdx.x & 31;
   float* mine = part + warp * 4 * d;
-  const int is_f32 = a.dtype == JAGG_DTYPE_F32;
+  float* sc_s = part + 8 * 4 * d;
+  float* gt_s = sc_s + d;
   const int row_begin = (int)((int64_t)a.M * blockIdx.x / gridDim.x);
   const int row_end = (int)((int64_t)a.M * (blockIdx.x + 1) / gridDim.x);
   for (int seg0 = row_begin; seg0 < row_end;) {
     const int b = seg0 / a.rows_per_seq;
     const int seg1 = min(row_end, (b + 1) * a.rows_per_seq);
     for (int i = lane; i < 4 * d; i += 32) mine[i] = 0.f;
-    __syncwarp();
-    const float* gate = a.do_gate ? a.gate + (int64_t)b * a.mod_stride : nullptr;
-    const float* sc = a.do_ln ? a.scale + (int64_t)b * a.mod_stride : nullptr;
+    for (int c = threadIdx.x; c < d; c += blockDim.x) {
+      sc_s[c] = 1.f + a.scale[(int64_t)b * a.mod_stride + c];
+      if (GATE) gt_s[c] = a.gate[(int64_t)b * a.mod_stride + c];
+    }
+    __syncthreads();
 #pragma unroll 1
     for (int m = seg0 + warp; m < seg1; m += 8) {
       const int64_t hr = seg_row(m, a.seg, a.seg_off, a.seg_stride);
-      float dm[NV][4], hv[NV][4], dh[NV][4], yv[NV][4];
+      const float mu = a.mean[m], rs = a.rstd[m];
+      float4 dh[NV], dm[NV], hv[NV];
+      uint2 yb[NV];
+      float4 yf[NV];
 #pragma unroll
       for (int i = 0; i < NV; ++i) {
         const int c = (i * 32 + lane) * 4;
-        const float4 d4 = *reinterpret_cast<const float4*>(a.dh_in + hr * d + c);
-        dh[i][0] = d4.x; dh[i][1] = d4.y; dh[i][2] = d4.z; dh[i][3] = d4.w;
-        if (a.do_ln) {
-          load4(a.dm, (int64_t)m * d + c, a.dm_f32, dm[i]);
-          const float4 h4 = *reinterpret_cast<const float4*>(a.h + hr * d + c);
-          hv[i][0] = h4.x; hv[i][1] = h4.y; hv[i][2] = h4.z; hv[i][3] = h4.w;
+        dh[i] = *reinterpret_cast<const float4*>(a.dh_in + hr * d + c);
+        dm[i] = *reinterpret_cast<const float4*>(static_cast<const float*>(a.dm) + (int64_t)m * d + c);
+        hv[i] = *reinterpret_cast<const float4*>(a.h + hr * d + c);
+        if (GATE) {
+          if (YBF)
+            yb[i] = *reinterpret_cast<const uint2*>(static_cast<const bf16*>(a.y) + (int64_t)m * d + c);
+          else
+            yf[i] = *reinterpret_cast<const float4*>(static_cast<const float*>(a.y) + (int64_t)m * d + c);
         }
-        if (gate) load4(a.y, (int64_t)m * d + c, is_f32, yv[i]);
       }
-      if (a.do_ln) {
-        const float mu = a.mean[m], rs = a.rstd[m];
-        float s1 = 0.f, s2 = 0.f;
+      float s1 = 0.f, s2 = 0.f;
 #pragma unroll
-        for (int i = 0; i < NV; ++i) {
-          const int c = (i * 32 + lane) * 4;
-          const float4 s4 = *reinterpret_cast<const float4*>(sc + c);
-          const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
+      for (int i = 0; i < NV; ++i) {
+        const float4 sv = *reinterpret_cast<const float4*>(sc_s + (i * 32 + lane) * 4);
+        hv[i].x = (hv[i].x - mu) * rs; hv[i].y = (hv[i].y - mu) * rs;  // now x-hat
+        hv[i].z = (hv[i].z - mu) * rs; hv[i].w = (hv[i].w - mu) * rs;
+        const float e0 = dm[i].x * sv.x, e1 = dm[i].y * sv.y, e2 = dm[i].z * sv.z, e3 = dm[i].w * sv.w;
+        s1 += (e0 + e1) + (e2 + e3);
+        s2 += (e0 * hv[i].x + e1 * hv[i].y) + (e2 * hv[i].z + e3 * hv[i].w);
+      }
+      s1 = warp_sum(s1) / d;
+      s2 = warp_sum(s2) / d;
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            hv[i][e] = (hv[i][e] - mu) * rs;  // now x-hat
-            const float dxh = dm[i][e] * (1.f + sv[e]);
-            s1 += dxh;
-            s2 += dxh * hv[i][e];
+      for (int i = 0; i < NV; ++i) {
+        const int c = (i * 32 + lane) * 4;
+        const float4 sv = *reinterpret_cast<const float4*>(sc_s + c);
+        dh[i].x += rs * (dm[i].x * sv.x - s1 - hv[i].x * s2);
+        dh[i].y += rs * (dm[i].y * sv.y - s1 - hv[i].y * s2);
+        dh[i].z += rs * (dm[i].z * sv.z - s1 - hv[i].z * s2);
+        dh[i].w += rs * (dm[i].w * sv.w - s1 - hv[i].w * s2);
+        *reinterpret_cast<float4*>(a.dh_out + hr * d + c) = dh[i];
+        float4* q0 = reinterpret_cast<float4*>(mine + c);
+        float4* q1 = reinterpret_cast<float4*>(mine + d + c);
+        float4 u = *q0, w = *q1;
+        u.x += dm[i].x; u.y += dm[i].y; u.z += dm[i].z; u.w += dm[i].w;
+        w.x += dm[i].x * hv[i].x; w.y += dm[i].y * hv[i].y; w.z += dm[i].z * hv[i].z; w.w += dm[i].w * hv[i].w;
+        *q0 = u;
+        *q1 = w;
+        if (GATE) {
+          float y0, y1, y2, y3;
+          if (YBF) {
+            const bf16* h = reinterpret_cast<const bf16*>(&yb[i]);
+            y0 = __bfloat162float(h[0]); y1 = __bfloat162float(h[1]);
+            y2 = __bfloat162float(h[2]); y3 = __bfloat162float(h[3]);
+          } else {
+            y0 = yf[i].x; y1 = yf[i].y; y2 = yf[i].z; y3 = yf[i].w;
           }
-        }
-        s1 = warp_sum(s1) / d;
-        s2 = warp_sum(s2) / d;
-#pragma unroll
-        for (int i = 0; i < NV; ++i) {
-          const int c = (i * 32 + lane) * 4;
-          const float4 s4 = *reinterpret_cast<const float4*>(sc + c);
-          const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
-#pragma unroll
-          for (int e = 0; e < 4; ++e) dh[i][e] += rs * (dm[i][e] * (1.f + sv[e]) - s1 - hv[i][e] * s2);
-          *reinterpret_cast<float4*>(a.dh_out + hr * d + c) = make_float4(dh[i][0], dh[i][1], dh[i][2], dh[i][3]);
-          float4* q0 = reinterpret_cast<float4*>(mine + c);
-          float4* q1 = reinterpret_cast<float4*>(mine + d + c);
-          float4 u = *q0, w = *q1;
-          u.x += dm[i][0]; u.y += dm[i][1]; u.z += dm[i][2]; u.w += dm[i][3];
-          w.x += dm[i][0] * hv[i][0]; w.y += dm[i][1] * hv[i][1]; w.z += dm[i][2] * hv[i][2];
-          w.w += dm[i][3] * hv[i][3];
-          *q0 = u;
-          *q1 = w;
-        }
-      }
-      if (gate) {
-#pragma unroll
-        for (int i = 0; i < NV; ++i) {
-          const int c = (i * 32 + lane) * 4;
-          const float4 g4 = *reinterpret_cast<const float4*>(gate + c);
-          const float dy[4] = {g4.x * dh[i][0], g4.y * dh[i][1], g4.z * dh[i][2], g4.w * dh[i][3]};
-          store4(a.dy, (int64_t)m * d + c, is_f32, dy);
+          const float4 g4 = *reinterpret_cast<const float4*>(gt_s + c);
+          const float dy[4] = {g4.x * dh[i].x, g4.y * dh[i].y, g4.z * dh[i].z, g4.w * dh[i].w};
+          store4(a.dy, (int64_t)m * d + c, !YBF, dy);
           float4* q2 = reinterpret_cast<float4*>(mine + 2 * d + c);
           float4* q3 = reinterpret_cast<float4*>(mine + 3 * d + c);
-          float4 u = *q2, w = *q3;
-          u.x += dh[i][0] * yv[i][0]; u.y += dh[i][1] * yv[i][1]; u.z += dh[i][2] * yv[i][2];
-          u.w += dh[i][3] * yv[i][3];
-          w.x += dh[i][0]; w.y += dh[i][1]; w.z += dh[i][2]; w.w += dh[i][3];
-          *q2 = u;
-          *q3 = w;
+          float4 u2 = *q2, w2 = *q3;
+          u2.x += dh[i].x * y0; u2.y += dh[i].y * y1; u2.z += dh[i].z * y2; u2.w += dh[i].w * y3;
+          w2.x += dh[i].x; w2.y += dh[i].y; w2.z += dh[i].z; w2.w += dh[i].w;
+          *q2 = u2;
+          *q3 = w2;
         }
       }
     }
@@ -435,38 +440,38 @@ __global__ void __launch_bounds__(256, 2) ln_gate_rowreg_kernel(LnGateBwd a) {
 #pragma unroll
       for (int w = 0; w < 8; ++w)
 #pragma unroll
-        for (int q = 0; q < 4; ++q) P[q] += part[(w * 4 + q) * d + c];
-      if (a.do_ln) {
-        atomicAdd(a.dshift + (int64_t)b * a.dmod_stride + c, P[0]);
-        atomicAdd(a.dscale + (int64_t)b * a.dmod_stride + c, P[1]);
-      }
-      if (a.do_gate) {
+        for (int q = 0; q < (GATE ? 4 : 2); ++q) P[q] += part[(w * 4 + q) * d + c];
+      atomicAdd(a.dshift + (int64_t)b * a.dmod_stride + c, P[0]);
+      atomicAdd(a.dscale + (int64_t)b * a.dmod_stride + c, P[1]);
+      if (GATE) {
         atomicAdd(a.dgate + (int64_t)b * a.dmod_stride + c, P[2]);
-        if (a.dbias) atomicAdd(a.dbias + c, gate[c] * P[3]);
+        if (a.dbias) atomicAdd(a.dbias + c, gt_s[c] * P[3]);
       }
     }
-    __syncthreads();  // the slabs are re-zeroed for the next segment
+    __syncthreads();  // the slabs and vectors are rewritten for the next segment
     seg0 = seg1;
   }
 }
 
-template <int NV>
-int launch_ln_gate_rowreg(const LnGateBwd& a, cudaStream_t s) {
-  const int smem = 8 * 4 * 128 * NV * (int)sizeof(float);
+template <int NV, bool GATE, bool YBF>
+int launch_ln_gate_rowreg_t(const LnGateBwd& a, cudaStream_t s) {
+  const int smem = (8 * 4 + 2) * 128 * NV * (int)sizeof(float);
   static bool attr = false;
   if (!attr) {
-    JAGG_CUDA_TRY(cudaFuncSetAttribute(ln_gate_rowreg_kernel<NV>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    JAGG_CUDA_TRY(cudaFuncSetAttribute(ln_gate_rowreg_kernel<NV, GATE, YBF>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
     attr = true;
   }
   static int per_sm = 0;
   if (!per_sm) {
-    JAGG_CUDA_TRY(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ln_gate_rowreg_kernel<NV>, 256, smem));
+    JAGG_CUDA_TRY(
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ln_gate_rowreg_kernel<NV, GATE, YBF>, 256, smem));
     if (per_sm < 1) per_sm = 1;
   }
   // equal row shares of at least 16 rows per CTA, at most one wave of resident CTAs
   const int cap = per_sm * sm_count();
   const int want = ceil_div(a.M, 16);
-  ln_gate_rowreg_kernel<NV><<<want < cap ? want : cap, 256, smem, s>>>(a);
+  ln_gate_rowreg_kernel<NV, GATE, YBF><<<want < cap ? want : cap, 256, smem, s>>>(a);
   JAGG_LAUNCHED();
   return JAGG_OK;
 }
@@ -738,6 +743,16 @@ int launch_ln_mod_fwd(const LnModFwd& a, cudaStream_t s) {
   JAGG_LAUNCHED();
   return JAGG_OK;
 }
+// The row-in-registers kernel serves LayerNorm backwards with an f32 dm (with or without the
+// gate); the rest go to the persistent kernel.
+template <int NV>
+int launch_ln_gate_rowreg(const LnGateBwd& a, int smem_fused, cudaStream_t s) {
+  if (!a.do_ln || !a.dm_f32) return launch_ln_gate_nv<0>(a, smem_fused, s);
+  if (!a.do_gate) return launch_ln_gate_rowreg_t<NV, false, false>(a, s);
+  return a.dtype == JAGG_DTYPE_F32 ? launch_ln_gate_rowreg_t<NV, true, false>(a, s)
+                                   : launch_ln_gate_rowreg_t<NV, true, true>(a, s);
+}
+
 int launch_ln_gate_bwd(const LnGateBwd& a, cudaStream_t s) {
   JAGG_CHECK_ARG(a.d % 4 == 0 && a.d <= 3072, "ln_gate_bwd: hidden %d unsupported", a.d);
   JAGG_CHECK_ARG(a.M % a.rows_per_seq == 0, "ln_gate_bwd: rows not a whole number of sequences");
@@ -746,9 +761,9 @@ int launch_ln_gate_bwd(const LnGateBwd& a, cudaStream_t s) {
   const int tok = prof_start(s);
   int st;
   switch (a.d % 128 == 0 ? a.d / 128 : 0) {
-    case 3: st = launch_ln_gate_rowreg<3>(a, s); break;
-    case 4: st = launch_ln_gate_rowreg<4>(a, s); break;
-    case 6: st = launch_ln_gate_rowreg<6>(a, s); break;
+    case 3: st = launch_ln_gate_rowreg<3>(a, smem, s); break;
+    case 4: st = launch_ln_gate_rowreg<4>(a, smem, s); break;
+    case 6: st = launch_ln_gate_rowreg<6>(a, smem, s); break;
     case 8: st = launch_ln_gate_nv<8>(a, smem, s); break;
     case 12: st = launch_ln_gate_nv<12>(a, smem, s); break;
     case 24: st = launch_ln_gate_nv<24>(a, smem, s); break;
