@@ -68,7 +68,7 @@ __device__ __forceinline__ void epi_apply1(const EpiParams& e, int m, int n, flo
     case EPI_GELU: {
       float g, dg;
       gelu_tanh_both(acc + (e.bias ? ldv(e.bias, n, e.bias_bf16) : 0.f), g, dg);
-      stv(e.C, cr * e.ldc + n, e.c_bf16, dg);
+      if (e.C) stv(e.C, cr * e.ldc + n, e.c_bf16, dg);
       stv(e.C2, cr * e.ldc2 + n, e.c_bf16, g);
     } break;
     case EPI_GATE_RESID: {
@@ -134,7 +134,7 @@ __device__ __forceinline__ void epi_apply8(const EpiParams& e, int m, int n, con
       float gv[8], dv[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) gelu_tanh_both(v[i], gv[i], dv[i]);
-      store8(e.C, cr * e.ldc + n, e.c_bf16, dv);
+      if (e.C) store8(e.C, cr * e.ldc + n, e.c_bf16, dv);
       store8(e.C2, cr * e.ldc2 + n, e.c_bf16, gv);
     } break;
     case EPI_GATE_RESID: {
@@ -178,7 +178,7 @@ __device__ __forceinline__ void epi_apply8(const EpiParams& e, int m, int n, con
 // each 32 x 32 chunk goes through swizzled shared memory and back so that a lane holds 4
 // consecutive columns of one row, and every global load / store of the epilogue covers
 // contiguous 128-byte row segments.
-enum : int { STAGED_NONE = 0, STAGED_STORE = 1, STAGED_MUL_AUX = 2, STAGED_ACCUM = 3, STAGED_ROWS = 4 };
+enum : int { STAGED_NONE = 0, STAGED_STORE = 1, STAGED_MUL_AUX = 2, STAGED_ACCUM = 3, STAGED_ROWS = 4, STAGED_GELU = 5 };
 
 struct TcParams {
   int tiles_m, tiles_n, splits, k_blocks;
@@ -258,7 +258,7 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
     ptx::prefetch_tmap(&tmA);
     ptx::prefetch_tmap(&tmB);
     if (p.staged != STAGED_NONE && p.staged != STAGED_ROWS) ptx::prefetch_tmap(&tmC);
-    if (p.staged == STAGED_MUL_AUX) ptx::prefetch_tmap(&tmX);
+    if (p.staged == STAGED_MUL_AUX || p.staged == STAGED_GELU) ptx::prefetch_tmap(&tmX);
   }
   if (warp == 1) {
     ptx::tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
@@ -455,7 +455,7 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
               float g[4], dg[4];
 #pragma unroll
               for (int i = 0; i < 4; ++i) gelu_tanh_both_approx(v[i], g[i], dg[i]);
-              st4(e.C, cr * e.ldc + n, e.c_bf16, dg);
+              if (e.C) st4(e.C, cr * e.ldc + n, e.c_bf16, dg);
               st4(e.C2, cr * e.ldc2 + n, e.c_bf16, g);
             } break;
             case EPI_GATE_RESID: {
@@ -488,7 +488,11 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
     // 32 x 32 box by lane 0.  The two warps of a lane quarter take alternate chunks.
     const int q = warp & 3, half = (warp - 2) >> 2, ew = warp - 2;  // half < SPLIT
     const bool mul = p.staged == STAGED_MUL_AUX;
-    const bool out_f32 = !p.e.c_bf16;
+    // STAGED_GELU: two bf16 outputs per chunk, GELU'(u) to C (when given, tmC) and GELU(u)
+    // to C2 (tmX), both staged in one slot (a slot holds a 32 x 32 f32 box)
+    const bool gelu = p.staged == STAGED_GELU;
+    const bool gelu_d = gelu && p.e.C != nullptr;
+    const bool out_f32 = !p.e.c_bf16 && !gelu;
     const int chunk_bytes = out_f32 ? 4096 : Cfg::CHUNK_BF16;
     uint8_t* stg = epi_smem + ew * Cfg::EPI_WARP_BYTES;
     uint8_t* auxs = stg + Cfg::NSTG * Cfg::CHUNK_BF16;  // EPI_MUL_AUX only (bf16 output)
@@ -530,7 +534,7 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
         float v[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-        if (p.staged == STAGED_STORE && p.e.bias) {
+        if ((p.staged == STAGED_STORE || gelu) && p.e.bias) {
           if (n0 + 32 <= p.e.N) {
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] += ldv(p.e.bias, n0 + i, p.e.bias_bf16);
@@ -557,8 +561,28 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
             ptx::bulk_wait_read<0>();
         }
         __syncwarp();
-        uint8_t* sb = stg + sbuf * chunk_bytes;
-        if (out_f32) {
+        uint8_t* sb = stg + sbuf * (gelu ? 2 * Cfg::CHUNK_BF16 : chunk_bytes);
+        if (gelu) {
+          uint8_t* row_d = sb + lane * 64;
+          uint8_t* row_g = sb + Cfg::CHUNK_BF16 + lane * 64;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            uint4 rd, rg;
+            __nv_bfloat162* hd = reinterpret_cast<__nv_bfloat162*>(&rd);
+            __nv_bfloat162* hg = reinterpret_cast<__nv_bfloat162*>(&rg);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              float g0, d0, g1, d1;
+              gelu_tanh_both_approx(v[8 * j + 2 * i], g0, d0);
+              gelu_tanh_both_approx(v[8 * j + 2 * i + 1], g1, d1);
+              hd[i] = __floats2bfloat162_rn(d0, d1);
+              hg[i] = __floats2bfloat162_rn(g0, g1);
+            }
+            const int off = (j ^ ((lane >> 1) & 3)) << 4;
+            if (gelu_d) *reinterpret_cast<uint4*>(row_d + off) = rd;
+            *reinterpret_cast<uint4*>(row_g + off) = rg;
+          }
+        } else if (out_f32) {
           uint8_t* row = sb + lane * 128;
 #pragma unroll
           for (int j = 0; j < 8; ++j)
@@ -578,10 +602,14 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
         ptx::fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) {
-          if (p.staged == STAGED_ACCUM)
+          if (p.staged == STAGED_ACCUM) {
             ptx::tma_reduce_add_2d(&tmC, sb, n0, m0);
-          else
+          } else if (gelu) {
+            if (gelu_d) ptx::tma_store_2d(&tmC, sb, n0, m0);
+            ptx::tma_store_2d(&tmX, sb + Cfg::CHUNK_BF16, n0, m0);
+          } else {
             ptx::tma_store_2d(&tmC, sb, n0, m0);
+          }
           ptx::bulk_commit();
         }
         sbuf = (sbuf + 1) % Cfg::NSTG;
@@ -831,7 +859,11 @@ int tile_order_n_first(const GemmArgs& g) { return (long long)g.M > (long long)g
 // 16-byte aligned with 16-byte row pitches.
 int staged_mode(const GemmArgs& g) {
   auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
-  if (g.c_trans || g.bias_m || !al16(g.C)) return STAGED_NONE;
+  if (g.c_trans || g.bias_m || (g.C && !al16(g.C))) return STAGED_NONE;
+  if (g.epi == EPI_GELU && !g.remap_rows && g.c_dtype == JAGG_DTYPE_BF16 && g.C2 && al16(g.C2) &&
+      g.ldc2 % 8 == 0 && (!g.C || g.ldc % 8 == 0) && (!g.bias || al16(g.bias)))
+    return STAGED_GELU;
+  if (!g.C) return STAGED_NONE;
   if (g.remap_rows || g.epi == EPI_GELU || g.epi == EPI_GATE_RESID) {
     // row-coalesced path: 4-column groups, 16-byte aligned rows of every operand
     bool ok = g.N % 4 == 0 && g.ldc % 4 == 0 && (!g.bias || al16(g.bias));
@@ -855,7 +887,7 @@ int staged_mode(const GemmArgs& g) {
 
 int validate(const GemmArgs& g) {
   JAGG_CHECK_ARG(g.M > 0 && g.N > 0 && g.K > 0, "gemm: empty shape %dx%dx%d", g.M, g.N, g.K);
-  JAGG_CHECK_ARG(g.A && g.B && g.C, "gemm: null operand");
+  JAGG_CHECK_ARG(g.A && g.B && (g.C || (g.epi == EPI_GELU && g.C2)), "gemm: null operand");
   JAGG_CHECK_ARG(g.epi >= EPI_STORE && g.epi <= EPI_ACCUM, "gemm: bad epilogue %d", g.epi);
   JAGG_CHECK_ARG(g.epi != EPI_ACCUM || g.c_dtype == JAGG_DTYPE_F32, "gemm: accumulation needs an f32 output");
   JAGG_CHECK_ARG(g.epi != EPI_GELU || g.C2, "gemm: GELU epilogue needs C2");
@@ -882,11 +914,13 @@ int launch_tc(const GemmArgs& g, cudaStream_t stream) {
   // per-thread epilogue serves those requests
   if ((p.staged == STAGED_ROWS) != (EW == 8)) p.staged = EW == 8 ? STAGED_ROWS : STAGED_NONE;
   CUtensorMap tc = ta, tx = ta;  // unused unless staged through TMA
-  if (p.staged != STAGED_NONE && p.staged != STAGED_ROWS) {
+  if (p.staged != STAGED_NONE && p.staged != STAGED_ROWS && g.C) {
     const bool c_f32 = g.c_dtype == JAGG_DTYPE_F32;
     JAGG_TRY(make_tmap(&tc, g.C, g.M, g.N, g.ldc, 32, 32, c_f32,
                        c_f32 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B));
   }
+  if (p.staged == STAGED_GELU)
+    JAGG_TRY(make_tmap(&tx, g.C2, g.M, g.N, g.ldc2, 32, 32, false, CU_TENSOR_MAP_SWIZZLE_64B));
   if (p.staged == STAGED_MUL_AUX && !AUX) p.staged = STAGED_NONE;  // no multiplier space
   if (p.staged == STAGED_MUL_AUX)
     JAGG_TRY(make_tmap(&tx, g.aux, g.M, g.N, g.ld_aux, 32, 32, false, CU_TENSOR_MAP_SWIZZLE_64B));

@@ -8,7 +8,7 @@ namespace jagg {
 
 enum GemmEpi : int {
   EPI_STORE = 0,       // C = acc (+ bias[n])                     (C: dtype or f32)
-  EPI_GELU = 1,        // u = acc + bias; C = gelu'(u); C2 = gelu(u)   (both dtype)
+  EPI_GELU = 1,        // u = acc + bias; C = gelu'(u) (C may be null); C2 = gelu(u)  (both dtype)
   EPI_GATE_RESID = 2,  // C = y = acc + bias; C2 = aux + gate[seq(m), n] * y  (C2, aux f32)
   EPI_MUL_AUX = 3,     // C = acc * aux                              (aux dtype)
   EPI_ACCUM = 4,       // C += acc (f32, atomic reduction; allows split-K)

@@ -294,6 +294,7 @@ struct Saved {
   std::vector<SingleSaved> sgl;
   float* hD[2] = {nullptr, nullptr};  // outputs of the last double block per stream
   float* h_fin;  // [M, d]
+  bool keep = true;  // a saving forward; false: nothing is kept, so GELU'(u) is not formed
   float* st_f;   // [2, B*Ni]
   void* mf;      // [B*Ni, d]
 };
@@ -364,6 +365,7 @@ void carve_single(Carver& cv, const jagg_model& m, int B, SingleSaved& k) {
 size_t carve_saved(const jagg_model& m, int B, void* base, bool save, Saved& s) {
   Carver cv(base);
   const int64_t M = (int64_t)B * m.N, Mi = (int64_t)B * m.Ni, Mt = (int64_t)B * m.Nt;
+  s.keep = save;
   s.xp = cv.take(Mi * m.pd * m.esz);
   s.txt = cv.take(Mt * m.cfg.txt_dim * m.esz);
   s.phi = cv.f32((int64_t)B * m.cfg.freq_dim);
@@ -812,7 +814,7 @@ int forward_dit(const jagg_model& m, const Saved& S, int B, cudaStream_t s) {
     LnModFwd ln2{k.h_mid, 0, 0, 0, M, d, N, mod + 3 * d, mod + 4 * d, Lm, k.m, dt, k.st2, k.st2 + M};
     JAGG_TRY(launch_ln_mod_fwd(ln2, s));
     g = fwd_gemm(m, M, m.dm, d, k.m, d, bw.fc1_w, bw.fc1_b);
-    g.epi = EPI_GELU; g.C = k.gp; g.ldc = m.dm; g.C2 = k.gu; g.ldc2 = m.dm;
+    g.epi = EPI_GELU; g.C = S.keep ? k.gp : nullptr; g.ldc = m.dm; g.C2 = k.gu; g.ldc2 = m.dm;
     JAGG_TRY(gemm(g, s));
     g = fwd_gemm(m, M, d, m.dm, k.gu, m.dm, bw.fc2_w, bw.fc2_b);
     g.epi = EPI_GATE_RESID; g.C = k.y2; g.ldc = d;
@@ -908,7 +910,7 @@ int forward_mmdit(const jagg_model& m, const Saved& S, int B, cudaStream_t s) {
       LnModFwd ln2{q.h_mid, 0, 0, 0, Ms, d, Ns, mod + 3 * d, mod + 4 * d, Lm, q.m, dt, q.st2, q.st2 + Ms};
       JAGG_TRY(launch_ln_mod_fwd(ln2, s));
       g = fwd_gemm(m, Ms, dm, d, q.m, d, sw.fc1_w, sw.fc1_b);
-      g.epi = EPI_GELU; g.C = q.gp; g.ldc = dm; g.C2 = q.gu; g.ldc2 = dm;
+      g.epi = EPI_GELU; g.C = S.keep ? q.gp : nullptr; g.ldc = dm; g.C2 = q.gu; g.ldc2 = dm;
       JAGG_TRY(gemm(g, s));
       g = fwd_gemm(m, Ms, d, dm, q.gu, dm, sw.fc2_w, sw.fc2_b);
       g.epi = EPI_GATE_RESID; g.C = q.y2; g.ldc = d;
@@ -935,7 +937,7 @@ int forward_mmdit(const jagg_model& m, const Saved& S, int B, cudaStream_t s) {
     g.C = k.qkv; g.ldc = 3 * d;
     JAGG_TRY(gemm(g, s));
     g = fwd_gemm(m, M, dm, d, k.a, d, sw.lin1_w + (int64_t)3 * d * d, sw.lin1_b + 3 * d);
-    g.epi = EPI_GELU; g.C = k.gp; g.ldc = dm;
+    g.epi = EPI_GELU; g.C = S.keep ? k.gp : nullptr; g.ldc = dm;
     g.C2 = static_cast<uint8_t*>(k.cat) + (size_t)d * e; g.ldc2 = d + dm;
     JAGG_TRY(gemm(g, s));
     JAGG_TRY(launch_qk_norm_rope_fwd(qk_args(m, k.qkv, M, N, Nt, sw.qn, sw.kn, k.qk, k.rq, k.rk), s));

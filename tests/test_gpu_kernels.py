@@ -131,6 +131,13 @@ def test_gemm_epilogues(M, N, K):
     gelu_u.sum().backward()
     assert _rel(GU.float(), gelu_u.detach()) < 5e-3
     assert _rel(DU.float(), u.grad) < 5e-3
+    # GELU alone (no derivative output: the forwards that keep nothing), into a wider buffer
+    GW = torch.full((M, N + 8), 7.0, device=dev, dtype=torch.bfloat16)
+    d = _desc(M, N, K, A, K, 0, B, K, 0, jg.DTYPE_BF16, DU, N, jg.DTYPE_BF16, epi=1, bias=bias, C2=GW, ldc2=N + 8)
+    d.C = None
+    jg.test_gemm(d)
+    torch.cuda.synchronize()
+    assert torch.equal(GW[:, :N], GU) and torch.all(GW[:, N:] == 7.0)
     u = u.detach()
     # gated residual: y = acc + bias; h_out = h_in + gate[seq] * y
     rows = 37
