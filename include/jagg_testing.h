@@ -72,6 +72,10 @@ int jagg_test_attention_bwd(const void* qkv, const void* o, const float* lse, co
  * the remaining N - n0 in qkv1 / o1 / dO1 / dqkv1 (n0 = N: one buffer, the *1 pointers
  * ignored).  impl: 0 the library's choice, 1 the warp-level MMA kernel, 2 the tcgen05
  * kernel (JAGG_ERR_ARG when it does not serve the call). */
+/* The forward over two-stream views (same layout and impl codes as the backward below):
+ * o0 / o1 receive the output rows of each stream, lse [B, heads, N]. */
+int jagg_test_attention_fwd_streams(const void* qkv0, const void* qkv1, void* o0, void* o1, float* lse, int B,
+                                    int N, int n0, int heads, int dh, int dtype, int impl, cudaStream_t stream);
 int jagg_test_attention_bwd_streams(const void* qkv0, const void* qkv1, const void* o0, const void* o1,
                                     const float* lse, const void* dO0, const void* dO1, int B, int N, int n0,
                                     int heads, int dh, int dtype, void* dqkv0, void* dqkv1, void* scratch, int impl,

@@ -115,6 +115,7 @@ _SIGNATURES = {
     "jagg_test_attention_fwd": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _P]),
     "jagg_test_attention_scratch_bytes": (_I64, [_I, _I, _I, _I]),
     "jagg_test_attention_bwd": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _P]),
+    "jagg_test_attention_fwd_streams": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
     "jagg_test_attention_bwd_streams": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _I,
                                              _P]),
 }
@@ -426,6 +427,16 @@ def test_attention_bwd(qkv, o, lse, dO, B, N, heads, dh, dqkv, stream=None):
     scratch = alloc_bytes(lib().jagg_test_attention_scratch_bytes(B, N, heads, dh), qkv.device)
     _check(lib().jagg_test_attention_bwd(_ptr(qkv), _ptr(o), _ptr(lse), _ptr(dO), B, N, heads, dh, dt, _ptr(dqkv),
                                          _ptr(scratch), _stream(stream)), "jagg_test_attention_bwd")
+
+
+def test_attention_fwd_streams(qkv, o, lse, B, N, n0, heads, dh, impl=0, stream=None):
+    """Forward over two-stream views: qkv and o given as pairs (first n0 tokens of every
+    sequence, the rest), contiguous; n0 = N uses the first only."""
+    dt = DTYPE_BF16 if qkv[0].dtype == torch.bfloat16 else DTYPE_F32
+    second = lambda pair: _ptr(pair[1]) if n0 < N else None
+    _check(lib().jagg_test_attention_fwd_streams(_ptr(qkv[0]), second(qkv), _ptr(o[0]), second(o), _ptr(lse), B, N,
+                                                 n0, heads, dh, dt, impl, _stream(stream)),
+           "jagg_test_attention_fwd_streams")
 
 
 def test_attention_bwd_streams(qkv, o, lse, dO, B, N, n0, heads, dh, dqkv, impl=0, stream=None):

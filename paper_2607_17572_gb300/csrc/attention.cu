@@ -610,6 +610,17 @@ void attention_bwd_scratch(float* scratch, int B, int N, int heads, float** Dv, 
 
 int attention_fwd(const AttnArgs& a, cudaStream_t s) {
   JAGG_CHECK_ARG(a.B > 0 && a.N > 0 && a.heads > 0, "attention: empty shape");
+  JAGG_CHECK_ARG(a.impl >= 0 && a.impl <= 2, "attention: bad implementation %d", a.impl);
+  const bool tc = attention_fwd_tc_eligible(a);
+  JAGG_CHECK_ARG(a.impl != 2 || tc, "attention: the tcgen05 forward does not serve this call");
+  if (tc && a.impl != 1) {
+    const int tok = prof_start(s);
+    JAGG_TRY(attention_fwd_tc(a, s));
+    // QK^T and PV: 2 N^2 d multiply-adds per (sequence, head); the second S pass is not counted
+    prof_stop(tok, s, PROF_ATTN_FWD, 4.0 * a.B * a.heads * (double)a.N * a.N * a.dh,
+              2.0 * a.B * (double)a.N * a.heads * a.dh * 4);
+    return JAGG_OK;
+  }
   if (a.dtype == JAGG_DTYPE_BF16) {
     if (a.dh == 64) return fwd_tc<64>(a, s);
     if (a.dh == 128) return fwd_tc<128>(a, s);

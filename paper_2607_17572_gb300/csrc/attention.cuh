@@ -30,6 +30,7 @@ struct AttnArgs {
   SegRows o;  // output, col h * dh
   float* lse;  // [B, heads, N] natural-log log-sum-exp of the scaled scores
   int dtype;
+  int impl = 0;  // forward: 0 the library's choice; 1 warp-level MMA kernel; 2 tcgen05 kernel
 };
 
 struct AttnBwdArgs {
@@ -43,6 +44,10 @@ struct AttnBwdArgs {
 };
 
 int attention_fwd(const AttnArgs& a, cudaStream_t s);
+// The tcgen05 forward (attention_tc.cu): bf16, head dim 64 / 128, stream boundary on a
+// multiple of 128 tokens, 16-byte aligned views.
+bool attention_fwd_tc_eligible(const AttnArgs& a);
+int attention_fwd_tc(const AttnArgs& a, cudaStream_t s);
 // The tcgen05 backward (attention_tc.cu): bf16, head dim 64 / 128, stream boundary on a
 // multiple of 128 tokens, 16-byte aligned views.
 bool attention_bwd_tc_eligible(const AttnBwdArgs& a);

@@ -510,6 +510,337 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
   }
 }
 
+// ================================================================== forward
+// Persistent over (128-query tile, sequence, head) units, two passes over the sequence's
+// 128-key tiles per unit:
+//   pass 1   S = Q K^T (TMEM), the exact row maximum m of the scaled scores;
+//   pass 2   S again, P = exp(scale (S - m)) (f32 row sums l; bf16 P to shared memory),
+//            O += P V (TMEM, never rescaled);
+//   then     O / l -> bf16 output, lse = scale m + ln l.
+// The extra S product (half the forward's tensor work again) buys a softmax with no running
+// rescale of O.  Warp roles: 0 TMA producer (Q once per unit, K in pass 1, K and V in pass 2),
+// 1 MMA issuer, 2-9 softmax and output (two warps per TMEM lane quarter = 32 query rows,
+// 64 key columns each; they exchange row maxima and sums through shared memory).
+constexpr int FF_THREADS = 320;  // 10 warps
+
+template <int D>
+struct FfCfg {
+  static constexpr int BQ = 128, BK = 128;
+  static constexpr int NS = D == 64 ? 3 : 2;  // K (pass 1) / K, V (pass 2) stages
+  static constexpr int NP = D == 64 ? 2 : 1;  // P buffers
+  static constexpr int Q_BYTES = BQ * D * 2;
+  static constexpr int KV_BYTES = BK * D * 2;
+  static constexpr int P_BYTES = BQ * BK * 2;
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_K = OFF_Q + Q_BYTES;
+  static constexpr int OFF_V = OFF_K + NS * KV_BYTES;
+  static constexpr int OFF_P = OFF_V + NS * KV_BYTES;
+  static constexpr int OFF_RED = OFF_P + NP * P_BYTES;  // [2: max, sum][2 halves][128 rows] f32
+  static constexpr int OFF_BAR = OFF_RED + 2 * 2 * 128 * 4;
+  static constexpr int SMEM = OFF_BAR + 256 + 1024;
+  static constexpr int T_O = 256;  // TMEM: S buffers at columns 0 and 128, O at 256
+  static_assert(SMEM <= 232448, "shared memory budget");
+};
+
+struct FfMaps {
+  CUtensorMap q[2], k[2], v[2];
+};
+
+struct FfParams {
+  int B, N, heads, n0;
+  float scale;
+  int64_t q_col0, k_col0, v_col0;
+  SegRows o;
+  float* lse;
+};
+
+__device__ __forceinline__ void named_bar(int id, int threads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+
+template <int D>
+__global__ void __launch_bounds__(FF_THREADS, 1) fa_fwd_tc_kernel(const __grid_constant__ FfMaps maps, FfParams p) {
+  using C = FfCfg<D>;
+  constexpr int BQ = C::BQ, BK = C::BK, NS = C::NS, NP = C::NP;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = sm + C::OFF_Q;
+  uint8_t* sK = sm + C::OFF_K;
+  uint8_t* sV = sm + C::OFF_V;
+  uint8_t* sP = sm + C::OFF_P;
+  float* red = reinterpret_cast<float*>(sm + C::OFF_RED);
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sm + C::OFF_BAR);
+  uint64_t* full = bar;              // [NS] a K (and V) stage landed
+  uint64_t* empty = full + NS;       // [NS] its products are done
+  uint64_t* qfull = empty + NS;      // the unit's Q landed
+  uint64_t* qfree = qfull + 1;       // the unit's last S product is done
+  uint64_t* bar_s = qfree + 1;       // [2] S in TMEM buffer b
+  uint64_t* sfree = bar_s + 2;       // [2] the 8 warps have read it
+  uint64_t* pready = sfree + 2;      // [NP] P written by the 8 warps
+  uint64_t* pfree = pready + NP;     // [NP] the product reading P is done
+  uint64_t* bar_o = pfree + NP;      // the unit's O is complete
+  uint64_t* ofree = bar_o + 1;       // the 8 warps have read O
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(ofree + 1);
+  __shared__ volatile int abort_flag;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int N = p.N;
+  const int nk = (N + BK - 1) / BK;
+  const int nq = (N + BQ - 1) / BQ;
+  const int units = nq * p.B * p.heads;
+  // unit u: query tile u % nq of sequence-head u / nq
+  auto unit_of = [&](int u, int& q0, int& b, int& h) {
+    const int bh = u / nq;
+    q0 = (u % nq) * BQ;
+    b = bh / p.heads;
+    h = bh % p.heads;
+  };
+  auto seg_of = [&](int r) { return r < p.n0 ? 0 : 1; };
+  auto row_in = [&](int r) { return r < p.n0 ? r : r - p.n0; };
+
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    for (int i = 0; i < NS; ++i) {
+      ptx::mbar_init(&full[i], 1);
+      ptx::mbar_init(&empty[i], 1);
+    }
+    ptx::mbar_init(qfull, 1);
+    ptx::mbar_init(qfree, 1);
+    for (int i = 0; i < 2; ++i) {
+      ptx::mbar_init(&bar_s[i], 1);
+      ptx::mbar_init(&sfree[i], 8);
+    }
+    for (int i = 0; i < NP; ++i) {
+      ptx::mbar_init(&pready[i], 8);
+      ptx::mbar_init(&pfree[i], 1);
+    }
+    ptx::mbar_init(bar_o, 1);
+    ptx::mbar_init(ofree, 8);
+    ptx::fence_mbar_init();
+    for (int sg = 0; sg < 2; ++sg) {
+      ptx::prefetch_tmap(&maps.q[sg]);
+      ptx::prefetch_tmap(&maps.k[sg]);
+      ptx::prefetch_tmap(&maps.v[sg]);
+    }
+  }
+  if (warp == 1) {
+    ptx::tmem_alloc(tmem_slot, 512);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      int g = 0, i = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < units && ok && !abort_flag; u += gridDim.x, ++i) {
+        int q0, b, h;
+        unit_of(u, q0, b, h);
+        if (i > 0 && !ptx::mbar_wait(qfree, (i - 1) & 1)) { ok = false; break; }
+        ptx::mbar_arrive_expect_tx(qfull, C::Q_BYTES);
+#pragma unroll
+        for (int c = 0; c < D / 64; ++c)
+          ptx::tma_load_3d(sQ + c * BQ * 128, &maps.q[seg_of(q0)], qfull, (int)(p.q_col0 + h * D + c * 64),
+                           row_in(q0), b);
+        for (int pass = 0; pass < 2 && ok; ++pass) {
+          for (int j = 0; j < nk; ++j, ++g) {
+            const int st = g % NS;
+            if (g >= NS && !ptx::mbar_wait(&empty[st], ((g / NS) & 1) ^ 1)) { ok = false; break; }
+            const int k0 = j * BK, sg = seg_of(k0), r = row_in(k0);
+            ptx::mbar_arrive_expect_tx(&full[st], (pass + 1) * C::KV_BYTES);
+#pragma unroll
+            for (int c = 0; c < D / 64; ++c) {
+              ptx::tma_load_3d(sK + st * C::KV_BYTES + c * BK * 128, &maps.k[sg], &full[st],
+                               (int)(p.k_col0 + h * D + c * 64), r, b);
+              if (pass == 1)
+                ptx::tma_load_3d(sV + st * C::KV_BYTES + c * BK * 128, &maps.v[sg], &full[st],
+                                 (int)(p.v_col0 + h * D + c * 64), r, b);
+            }
+          }
+        }
+      }
+      if (!ok) abort_flag = 1;
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (ptx::elect_one()) {
+      constexpr uint32_t id_s = ptx::idesc_bf16(128, BK, false, false);
+      constexpr uint32_t id_o = ptx::idesc_bf16(128, D, false, true);
+      const uint32_t aQ = ptx::smem_u32(sQ);
+      bool ok = true;
+      int g = 0, sc = 0, pc = 0, i = 0;
+      auto issue_s = [&](int st) {  // S of the stage's key tile into TMEM buffer sc % 2
+        const int sb = sc & 1;
+        if (sc >= 2 && !ptx::mbar_wait(&sfree[sb], ((sc >> 1) & 1) ^ 1)) return false;
+        ptx::tc_fence_after();
+        const uint32_t aK = ptx::smem_u32(sK + st * C::KV_BYTES);
+#pragma unroll
+        for (int k = 0; k < D / 16; ++k)
+          ptx::umma_bf16(tmem + sb * 128, kmajor_desc(aQ, BQ, k), kmajor_desc(aK, BK, k), id_s, k > 0);
+        ptx::umma_commit(&bar_s[sb]);
+        ++sc;
+        return true;
+      };
+      auto issue_pv = [&](int st, bool first) {  // O += P V of the stage's value tile
+        const int pb = pc % NP;
+        if (!ptx::mbar_wait(&pready[pb], (pc / NP) & 1)) return false;
+        ptx::tc_fence_after();
+        const uint32_t aP = ptx::smem_u32(sP + pb * C::P_BYTES);
+        const uint32_t aV = ptx::smem_u32(sV + st * C::KV_BYTES);
+#pragma unroll
+        for (int k = 0; k < BK / 16; ++k)
+          ptx::umma_bf16(tmem + C::T_O, kmajor_desc(aP, BQ, k), mnmajor_desc(aV, BK * 128, k), id_o,
+                         (!first || k > 0) ? 1u : 0u);
+        ptx::umma_commit(&pfree[pb]);
+        ptx::umma_commit(&empty[st]);
+        ++pc;
+        return true;
+      };
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++i) {
+        if (!ptx::mbar_wait(qfull, i & 1)) { ok = false; break; }
+        // pass 1
+        for (int j = 0; j < nk && ok; ++j, ++g) {
+          const int st = g % NS;
+          if (!ptx::mbar_wait(&full[st], (g / NS) & 1)) { ok = false; break; }
+          ok = issue_s(st);
+          ptx::umma_commit(&empty[st]);
+        }
+        // pass 2: S of tile j, then P V of tile j - 1
+        int prev_st = -1;
+        for (int j = 0; j < nk && ok; ++j, ++g) {
+          const int st = g % NS;
+          if (!ptx::mbar_wait(&full[st], (g / NS) & 1)) { ok = false; break; }
+          if (!issue_s(st)) { ok = false; break; }
+          if (j == nk - 1) ptx::umma_commit(qfree);
+          if (j > 0) {
+            if (j == 1 && i > 0 && !ptx::mbar_wait(ofree, (i - 1) & 1)) { ok = false; break; }
+            if (!issue_pv(prev_st, j == 1)) { ok = false; break; }
+          }
+          prev_st = st;
+        }
+        if (!ok) break;
+        if (nk == 1 && i > 0 && !ptx::mbar_wait(ofree, (i - 1) & 1)) { ok = false; break; }
+        if (!issue_pv(prev_st, nk == 1)) { ok = false; break; }
+        ptx::umma_commit(bar_o);
+      }
+      if (!ok) abort_flag = 1;
+    }
+  } else {
+    // ---------------------------------------------------------------- softmax, output
+    // The two warps of a lane quarter meet at named barriers, so neither leaves the unit
+    // loop early: after a failed (timed-out) wait a warp runs on without waiting.
+    const int quarter = warp & 3, half = (warp - 2) >> 2;
+    const int r = quarter * 32 + lane;  // query row of the tile = TMEM lane
+    const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
+    const float c2 = p.scale * kLog2eTc;
+    float* red_m = red;
+    float* red_l = red + 2 * 128;
+    bool ok = true;
+    auto wait = [&](uint64_t* b, uint32_t phase) {
+      if (ok) ok = __all_sync(0xffffffffu, ptx::mbar_wait(b, phase));
+      if (!ok) abort_flag = 1;
+    };
+    int sc = 0, pc = 0, i = 0;
+    for (int u = blockIdx.x; u < units; u += gridDim.x, ++i) {
+      int q0, b, h;
+      unit_of(u, q0, b, h);
+      // pass 1: the row maximum over the valid keys
+      float m = -INFINITY;
+      for (int j = 0; j < nk; ++j, ++sc) {
+        const int sb = sc & 1;
+        wait(&bar_s[sb], (sc >> 1) & 1);
+        ptx::tc_fence_after();
+        uint32_t rs[64];
+        ptx::tmem_ld_32x32b_x32(trow + sb * 128 + half * 64, *reinterpret_cast<uint32_t(*)[32]>(rs));
+        ptx::tmem_ld_32x32b_x32(trow + sb * 128 + half * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(rs + 32));
+        ptx::tmem_ld_wait();
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0 && ok) ptx::mbar_arrive(&sfree[sb]);
+        const int kv = N - (j * BK + half * 64);  // valid keys among this warp's 64
+#pragma unroll
+        for (int c = 0; c < 64; ++c)
+          if (c < kv) m = fmaxf(m, __uint_as_float(rs[c]));
+      }
+      red_m[half * 128 + r] = m;
+      named_bar(1 + quarter, 64);
+      m = fmaxf(m, red_m[(1 - half) * 128 + r]);
+      // pass 2: P, its row sums, O += P V
+      float l = 0.f;
+      for (int j = 0; j < nk; ++j, ++sc, ++pc) {
+        const int sb = sc & 1, pb = pc % NP;
+        wait(&bar_s[sb], (sc >> 1) & 1);
+        ptx::tc_fence_after();
+        uint32_t hp[32];
+        const int kv = N - (j * BK + half * 64);
+#pragma unroll
+        for (int cc = 0; cc < 2; ++cc) {
+          uint32_t rs[32];
+          ptx::tmem_ld_32x32b_x32(trow + sb * 128 + half * 64 + cc * 32, rs);
+          ptx::tmem_ld_wait();
+#pragma unroll
+          for (int c = 0; c < 32; c += 2) {
+            const float p0 = cc * 32 + c < kv ? ptx::ex2_approx((__uint_as_float(rs[c]) - m) * c2) : 0.f;
+            const float p1 = cc * 32 + c + 1 < kv ? ptx::ex2_approx((__uint_as_float(rs[c + 1]) - m) * c2) : 0.f;
+            l += p0 + p1;
+            hp[cc * 16 + c / 2] = pack2_bf16(p0, p1);
+          }
+        }
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0 && ok) ptx::mbar_arrive(&sfree[sb]);
+        if (pc >= NP) wait(&pfree[pb], ((pc - NP) / NP) & 1);
+        uint8_t* tile = sP + pb * C::P_BYTES;
+        st_row32_packed(tile, BQ, r, half * 64, hp);
+        st_row32_packed(tile, BQ, r, half * 64 + 32, hp + 16);
+        ptx::fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0 && ok) ptx::mbar_arrive(&pready[pb]);
+      }
+      red_l[half * 128 + r] = l;
+      named_bar(1 + quarter, 64);
+      l += red_l[(1 - half) * 128 + r];
+      // the unit's output: O / l, and the log-sum-exp
+      wait(bar_o, i & 1);
+      ptx::tc_fence_after();
+      const int q = q0 + r;
+      const float inv = 1.f / l;
+#pragma unroll
+      for (int cc = 0; cc < D / 64; ++cc) {
+        uint32_t ro[32];
+        ptx::tmem_ld_32x32b_x32(trow + C::T_O + half * (D / 2) + cc * 32, ro);
+        ptx::tmem_ld_wait();
+        if (q < N && ok) {
+          bf16* o = static_cast<bf16*>(p.o.base(q)) + p.o.off(b, q, N, (int64_t)h * D + half * (D / 2) + cc * 32);
+#pragma unroll
+          for (int v = 0; v < 4; ++v) {
+            uint4 w;
+            w.x = pack2_bf16(__uint_as_float(ro[8 * v]) * inv, __uint_as_float(ro[8 * v + 1]) * inv);
+            w.y = pack2_bf16(__uint_as_float(ro[8 * v + 2]) * inv, __uint_as_float(ro[8 * v + 3]) * inv);
+            w.z = pack2_bf16(__uint_as_float(ro[8 * v + 4]) * inv, __uint_as_float(ro[8 * v + 5]) * inv);
+            w.w = pack2_bf16(__uint_as_float(ro[8 * v + 6]) * inv, __uint_as_float(ro[8 * v + 7]) * inv);
+            *reinterpret_cast<uint4*>(o + 8 * v) = w;
+          }
+        }
+      }
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0 && ok) ptx::mbar_arrive(ofree);
+      if (half == 0 && q < N && ok) p.lse[((int64_t)b * p.heads + h) * N + q] = p.scale * m + logf(l);
+    }
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, 512);
+  }
+}
+
 // 3D view [sequence][token][column] of a stream buffer (bf16), boxes of 64 columns x `rows`.
 int seg_map(CUtensorMap* m, const void* base, int64_t ld, int ntok, int B, int rows) {
   const uint64_t dims[3] = {(uint64_t)ld, (uint64_t)ntok, (uint64_t)B};
@@ -567,7 +898,63 @@ int launch(const AttnBwdArgs& a, cudaStream_t s) {
   return JAGG_OK;
 }
 
+template <int D>
+int launch_fwd(const AttnArgs& f, cudaStream_t s) {
+  using C = FfCfg<D>;
+  const int n0 = f.q.n0, N = f.N;
+  const int n1 = N - n0;
+  FfMaps maps;
+  for (int sg = 0; sg < 2; ++sg) {
+    const int nt = sg == 0 ? n0 : n1;
+    if (nt <= 0) {  // single stream: the second views are unused copies
+      maps.q[1] = maps.q[0];
+      maps.k[1] = maps.k[0];
+      maps.v[1] = maps.v[0];
+      break;
+    }
+    JAGG_TRY(seg_map(&maps.q[sg], sg ? f.q.p1 : f.q.p0, sg ? f.q.ld1 : f.q.ld0, nt, f.B, C::BQ));
+    JAGG_TRY(seg_map(&maps.k[sg], sg ? f.k.p1 : f.k.p0, sg ? f.k.ld1 : f.k.ld0, nt, f.B, C::BK));
+    JAGG_TRY(seg_map(&maps.v[sg], sg ? f.v.p1 : f.v.p0, sg ? f.v.ld1 : f.v.ld0, nt, f.B, C::BK));
+  }
+  FfParams p;
+  p.B = f.B; p.N = N; p.heads = f.heads; p.n0 = n0 > 0 && n0 < N ? n0 : N;
+  p.scale = f.scale;
+  p.q_col0 = f.q_col0; p.k_col0 = f.k_col0; p.v_col0 = f.v_col0;
+  p.o = f.o;
+  p.lse = f.lse;
+  static bool attr = false;
+  if (!attr) {
+    JAGG_CUDA_TRY(cudaFuncSetAttribute(fa_fwd_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
+    attr = true;
+  }
+  const int units = ceil_div(N, C::BQ) * f.B * f.heads;
+  const int nsm = sm_count();
+  fa_fwd_tc_kernel<D><<<units < nsm ? units : nsm, FF_THREADS, C::SMEM, s>>>(maps, p);
+  JAGG_LAUNCHED();
+  return JAGG_OK;
+}
+
 }  // namespace
+
+// Whether the tensor-core forward serves the call: bf16, head dim 64 / 128, the stream
+// boundary on a 128-token multiple, 16-byte aligned operands and output rows.
+bool attention_fwd_tc_eligible(const AttnArgs& f) {
+  if (f.dtype != JAGG_DTYPE_BF16 || (f.dh != 64 && f.dh != 128) || !f.lse) return false;
+  const int n0 = f.q.n0;
+  const bool single = n0 >= f.N;
+  if (!single && (n0 <= 0 || n0 % 128)) return false;
+  const SegRows* views[4] = {&f.q, &f.k, &f.v, &f.o};
+  for (const SegRows* v : views) {
+    if (v->n0 != n0) return false;
+    if (!aligned16(v->p0) || v->ld0 % 8) return false;
+    if (!single && (!aligned16(v->p1) || v->ld1 % 8)) return false;
+  }
+  return f.q_col0 % 8 == 0 && f.k_col0 % 8 == 0 && f.v_col0 % 8 == 0;
+}
+
+int attention_fwd_tc(const AttnArgs& f, cudaStream_t s) {
+  return f.dh == 64 ? launch_fwd<64>(f, s) : launch_fwd<128>(f, s);
+}
 
 // Whether the tensor-core backward serves the call: bf16, head dim 64 / 128, the stream
 // boundary on a 128-token multiple, 16-byte aligned buffers with 16-byte row pitches.

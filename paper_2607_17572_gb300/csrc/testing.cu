@@ -60,6 +60,28 @@ extern "C" int jagg_test_attention_bwd(const void* qkv, const void* o, const flo
   return attention_bwd(ab, stream);
 }
 
+extern "C" int jagg_test_attention_fwd_streams(const void* qkv0, const void* qkv1, void* o0, void* o1, float* lse,
+                                               int B, int N, int n0, int heads, int dh, int dtype, int impl,
+                                               cudaStream_t stream) {
+  JAGG_CHECK_ARG(qkv0 && o0 && lse, "jagg_test_attention_fwd_streams: null pointer");
+  JAGG_CHECK_ARG(n0 > 0 && n0 <= N, "jagg_test_attention_fwd_streams: n0 = %d", n0);
+  const bool two = n0 < N;
+  JAGG_CHECK_ARG(!two || (qkv1 && o1), "jagg_test_attention_fwd_streams: null second stream");
+  const int d = heads * dh;
+  auto view = [&](const void* p0, const void* p1, int64_t ld) {
+    return SegRows{const_cast<void*>(p0), const_cast<void*>(two ? p1 : p0), ld, ld, two ? n0 : N};
+  };
+  AttnArgs f;
+  f.B = B; f.N = N; f.heads = heads; f.dh = dh; f.scale = 1.f / sqrtf((float)dh);
+  f.q = f.k = f.v = view(qkv0, qkv1, 3 * d);
+  f.q_col0 = 0; f.k_col0 = d; f.v_col0 = 2 * d;
+  f.o = view(o0, o1, d);
+  f.lse = lse;
+  f.dtype = dtype;
+  f.impl = impl;
+  return attention_fwd(f, stream);
+}
+
 extern "C" int jagg_test_attention_bwd_streams(const void* qkv0, const void* qkv1, const void* o0, const void* o1,
                                                const float* lse, const void* dO0, const void* dO1, int B, int N,
                                                int n0, int heads, int dh, int dtype, void* dqkv0, void* dqkv1,

@@ -301,6 +301,37 @@ def test_attention_backward_kernels_on_two_stream_views(dh, N, n0, B, H, impl):
         assert _rel(g[i], t.grad) < 2e-2, "qkv"[i]
 
 
+@pytest.mark.parametrize("impl", [1, 2])
+@pytest.mark.parametrize("dh,N,n0,B,H", [(64, 333, 333, 2, 3), (64, 256, 128, 2, 2), (64, 64, 64, 1, 1),
+                                         (64, 24, 24, 3, 2), (64, 1000, 1000, 1, 2), (128, 1536, 512, 1, 2),
+                                         (128, 200, 200, 1, 2), (128, 700, 256, 2, 2), (128, 4608, 512, 1, 1)])
+def test_attention_forward_kernels_on_two_stream_views(dh, N, n0, B, H, impl):
+    """Both forward kernels (impl 1: warp-level MMA, 2: tcgen05) against PyTorch fp32 on one
+    buffer and on the text/image stream split: output and log-sum-exp, ragged last tiles."""
+    torch.manual_seed(N + dh + n0 + 1)
+    dev = "cuda"
+    d = H * dh
+    qkv = (torch.randn(B * N, 3 * d, device=dev) * 1.5).bfloat16()
+    q, k, v = _attn_ref(qkv, B, N, H, dh)
+    s = (q @ k.transpose(-1, -2)) / math.sqrt(dh)
+    ref_lse = torch.logsumexp(s, -1)
+    ref_o = torch.softmax(s, -1) @ v
+
+    def split(x):
+        x = x.view(B, N, -1)
+        return x[:, :n0].contiguous(), x[:, n0:].contiguous()
+
+    o0 = torch.full((B, n0, d), float("nan"), device=dev, dtype=torch.bfloat16)
+    o1 = torch.full((B, N - n0, d), float("nan"), device=dev, dtype=torch.bfloat16)
+    lse = torch.full((B, H, N), float("nan"), device=dev)
+    jg.test_attention_fwd_streams(split(qkv), (o0, o1), lse, B, N, n0, H, dh, impl=impl)
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    o = torch.cat([o0, o1], 1).float().view(B, N, H, dh).transpose(1, 2)
+    assert _rel(o, ref_o) < 1e-2
+    assert (lse - ref_lse).abs().max().item() < 1e-2
+
+
 def test_tcgen05_attention_backward_rejects_unaligned_streams():
     B, N, n0, H, dh = 1, 300, 100, 2, 64
     d = H * dh
