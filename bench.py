@@ -54,8 +54,11 @@ def parse():
     p.add_argument("--quick", action="store_true", help="skip the full-W, e2e and CPU legs")
     p.add_argument("--G", type=int, default=0,
                    help="override the workload's group size (small cases for profiler captures)")
-    p.add_argument("--kernel", choices=["attention_bwd"], default=None,
+    p.add_argument("--kernel", choices=["attention_bwd", "gemm"], default=None,
                    help="time one kernel family alone on the workload's shapes instead of the step")
+    p.add_argument("--product", default="all",
+                   help="for --kernel gemm: one of the block's backward products (fc2_dx, fc1_dx, qkv_dx, "
+                        "proj_dx, fc2_dw, fc1_dw, qkv_dw, proj_dw) or all")
     p.add_argument("--rows", type=int, default=0, help="sequences per call for --kernel (default 2G)")
     p.add_argument("--vjp-rows", choices=["auto", "group", "window"], default="auto",
                    help="one joint VJP per group (all windows' rows) or per window; auto picks the group "
@@ -861,12 +864,93 @@ def run_kernel_attention_bwd(args):
                       "aux_ms_per_call": prof["attention_bwd_aux"]["ms"] / args.steps}), flush=True)
 
 
+def gemm_products(wl, rows):
+    """The dense products of one block's backward at `rows` token rows, in the operand layouts
+    of the joint VJP: name -> (M, N, K, a_mn, b_mn, epilogue).  Input gradients dX = dY W
+    (K-major dY, MN-major W; the fc2 one times GELU'(u), the multiplier epilogue), weight
+    gradients dW += dY^T X (both MN-major, f32 accumulation)."""
+    d, f = wl.hidden, wl.mlp
+    return {"fc2_dx": (rows, f, d, False, True, "mul_aux"), "fc1_dx": (rows, d, f, False, True, "store"),
+            "qkv_dx": (rows, d, 3 * d, False, True, "store"), "proj_dx": (rows, d, d, False, True, "store"),
+            "fc2_dw": (d, f, rows, True, True, "accum"), "fc1_dw": (f, d, rows, True, True, "accum"),
+            "qkv_dw": (3 * d, d, rows, True, True, "accum"), "proj_dw": (d, d, rows, True, True, "accum")}
+
+
+def run_kernel_gemm(args):
+    """The block's backward products alone at the step's VJP rows (2G rows per window, every
+    window: the joint VJP's token rows), each timed with CUDA events over the timed calls and
+    by the library's per-launch events, on random bf16 operands (a few hundred MB at most)."""
+    import paper_2607_17572_gb300 as jg
+    wl = workload(args)
+    dev = torch.device("cuda", torch.cuda.current_device())
+    rows = (args.rows or 2 * wl.G * (wl.T // wl.W)) * wl.n_tok
+    prods = gemm_products(wl, rows)
+    names = list(prods) if args.product == "all" else [args.product]
+    gen = torch.Generator(device=dev).manual_seed(synth.NOISE_SEED)
+    burst, sustained, hbm, src = peaks()
+    out = {}
+    for name in names:
+        M, N, K, a_mn, b_mn, epi = prods[name]
+        A = torch.randn(K, M, device=dev, generator=gen).bfloat16() if a_mn else \
+            torch.randn(M, K, device=dev, generator=gen).bfloat16()
+        B = (torch.randn(K, N, device=dev, generator=gen) if b_mn else
+             torch.randn(N, K, device=dev, generator=gen)).mul_(K ** -0.5).bfloat16()
+        d = jg.GemmDesc()
+        d.M, d.N, d.K = M, N, K
+        d.A, d.lda, d.a_mn, d.a_dtype = A.data_ptr(), M if a_mn else K, int(a_mn), jg.DTYPE_BF16
+        d.B, d.ldb, d.b_mn, d.b_dtype = B.data_ptr(), N if b_mn else K, int(b_mn), jg.DTYPE_BF16
+        d.rows_per_seq = 1
+        keep = [A, B]
+        if epi == "accum":
+            C = torch.zeros(M, N, device=dev)
+            d.epi, d.C, d.ldc, d.c_dtype = 4, C.data_ptr(), N, jg.DTYPE_F32
+        else:
+            C = torch.empty(M, N, device=dev, dtype=torch.bfloat16)
+            d.epi, d.C, d.ldc, d.c_dtype = (3 if epi == "mul_aux" else 0), C.data_ptr(), N, jg.DTYPE_BF16
+            if epi == "mul_aux":
+                X = torch.rand(M, N, device=dev, generator=gen).bfloat16()
+                d.aux, d.ld_aux = X.data_ptr(), N
+                keep.append(X)
+        keep.append(C)
+        call = lambda: jg.test_gemm(d)
+        for _ in range(args.warmup):
+            call()
+        torch.cuda.synchronize()
+        stream = torch.cuda.current_stream()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.profiler.start()
+        e0.record(stream)
+        for _ in range(args.steps):
+            call()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        torch.cuda.profiler.stop()
+        ms = e0.elapsed_time(e1) / args.steps
+        jg.profile_enable(True)
+        for _ in range(args.steps):
+            call()
+        fam = jg.profile_read()["gemm_tcgen05"]
+        jg.profile_enable(False)
+        kms = fam["ms"] / max(fam["launches"], 1)
+        tf = 2.0 * M * N * K / (kms / 1000.0) / 1e12
+        out[name] = {"M": M, "N": N, "K": K, "epilogue": epi, "ms_per_call": ms, "kernel_ms": kms, "tflops": tf,
+                     "frac_of_burst": tf / burst}
+        del keep, C
+        torch.cuda.empty_cache()
+    print(json.dumps({"kernel": "gemm", "workload": describe(wl), "rows": rows, "steps": args.steps,
+                      "peak": {"tflops": burst, "source": f"bf16_tflops (burst) of {src} peaks"},
+                      "products": out}), flush=True)
+
+
 def main():
     args = parse()
     ws, rank = dist_setup()
     if args.kernel == "attention_bwd":
         if rank == 0:
             run_kernel_attention_bwd(args)
+    elif args.kernel == "gemm":
+        if rank == 0:
+            run_kernel_gemm(args)
     elif args.impl == "reference":
         run_reference(args, ws, rank)
     else:

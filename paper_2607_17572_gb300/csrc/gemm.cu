@@ -490,7 +490,10 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
     const bool mul = p.staged == STAGED_MUL_AUX;
     // STAGED_GELU: two bf16 outputs per chunk, GELU'(u) to C (when given, tmC) and GELU(u)
     // to C2 (tmX), both staged in one slot (a slot holds a 32 x 32 f32 box)
-    const bool gelu = p.staged == STAGED_GELU;
+    // (the forward-only GELU epilogue is compiled into the forward-layout instances alone, so
+    // the backward products keep their register budget)
+    constexpr bool FWD = !A_MN && !B_MN;
+    const bool gelu = FWD && p.staged == STAGED_GELU;
     const bool gelu_d = gelu && p.e.C != nullptr;
     const bool out_f32 = !p.e.c_bf16 && !gelu;
     const int chunk_bytes = out_f32 ? 4096 : Cfg::CHUNK_BF16;
