@@ -530,20 +530,22 @@ GemmArgs dw_gemm(const jagg_model& m, int M, int N, int K, const void* dY, int64
   return g;
 }
 
-// Products over the B per-sequence rows (t-embedding MLP, stacked modulation), in the
-// transposed form whose M is a feature dimension:
-//   rows_gemm: C[B, out] (f32) = X[B, in] W[out, in]^T + b   as  C^T = W X^T
+// Products over the B per-sequence rows (t-embedding MLP, stacked modulation).  B is small
+// (a few dozen rows: one 128-row tile, the rest of it zero-filled by TMA), and the products
+// are bound by reading W, so they keep the plain row-major output with the staged
+// epilogues:
+//   rows_gemm: C[B, out] (f32) = X[B, in] W[out, in]^T + b
 //   rows_dw:   grad[out, in] += dY[B, out]^T X[B, in]        (K = B)
-//   rows_dx:   dX[B, in] += dY[B, out] W[out, in]             as  dX^T = W^T dY^T
-// X / dY are in the storage type; dX accumulates in f32 (split over out).
+//   rows_dx:   dX[B, in] += dY[B, out] W[out, in]             (split over out)
+// X / dY are in the storage type; dX accumulates in f32.
 GemmArgs rows_gemm(const jagg_model& m, int out, int in, int B, const void* X, int64_t w_off, int64_t b_off,
                    float* C) {
   GemmArgs g;
-  g.M = out; g.N = B; g.K = in;
-  g.A = W(m, w_off); g.lda = in; g.a_dtype = m.cfg.dtype;
-  g.B = X; g.ldb = in; g.b_dtype = m.cfg.dtype;
-  g.bias = W(m, b_off); g.bias_dtype = m.cfg.dtype; g.bias_m = true;
-  g.C = C; g.ldc = out; g.c_dtype = JAGG_DTYPE_F32; g.c_trans = true;
+  g.M = B; g.N = out; g.K = in;
+  g.A = X; g.lda = in; g.a_dtype = m.cfg.dtype;
+  g.B = W(m, w_off); g.ldb = in; g.b_dtype = m.cfg.dtype;
+  g.bias = W(m, b_off); g.bias_dtype = m.cfg.dtype;
+  g.C = C; g.ldc = out; g.c_dtype = JAGG_DTYPE_F32;
   return g;
 }
 GemmArgs rows_dw(const jagg_model& m, int out, int in, int B, const void* dY, const void* X, float* grad,
@@ -557,10 +559,10 @@ GemmArgs rows_dw(const jagg_model& m, int out, int in, int B, const void* dY, co
 }
 GemmArgs rows_dx(const jagg_model& m, int out, int in, int B, const void* dY, int64_t w_off, float* dX) {
   GemmArgs g;
-  g.M = in; g.N = B; g.K = out;
-  g.A = W(m, w_off); g.lda = in; g.a_mn = true; g.a_dtype = m.cfg.dtype;
-  g.B = dY; g.ldb = out; g.b_mn = false; g.b_dtype = m.cfg.dtype;
-  g.epi = EPI_ACCUM; g.C = dX; g.ldc = in; g.c_dtype = JAGG_DTYPE_F32; g.c_trans = true;
+  g.M = B; g.N = in; g.K = out;
+  g.A = dY; g.lda = out; g.a_mn = false; g.a_dtype = m.cfg.dtype;
+  g.B = W(m, w_off); g.ldb = in; g.b_mn = true; g.b_dtype = m.cfg.dtype;
+  g.epi = EPI_ACCUM; g.C = dX; g.ldc = in; g.c_dtype = JAGG_DTYPE_F32;
   return g;
 }
 
