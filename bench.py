@@ -82,6 +82,12 @@ def describe(wl) -> str:
             f"tokens, G={wl.G}, T={wl.T}, W={wl.W}, jagg_frac={wl.jagg_frac}")
 
 
+# DRAM bytes (read + write) per launch of the dense-product kernel in the timed step, from
+# one ncu capture of the step's launch list (profiles/ditb_jagg_step_launches.md: kernel
+# revision 91655fa); None for workloads without such a capture.
+TRAFFIC_PER_LAUNCH = {"dit_b_bf16": 134.7e6}
+
+
 def peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -595,7 +601,8 @@ def run_gpu(args, ws, rank):
     gt = fam.get("gemm_tcgen05", {"launches": 0, "ms": 0.0, "flops": 0.0})
     achieved = gt["flops"] / (gt["ms"] / 1000.0) / 1e12 if gt["ms"] > 0 else 0.0
     roofline = {"bound": "tensor", "achieved": achieved, "peak": sustained, "unit": "TFLOP/s",
-                "frac": achieved / sustained, "traffic": None,
+                "frac": achieved / sustained, "traffic": TRAFFIC_PER_LAUNCH.get(wl.name),
+                "algorithmic_bytes_per_launch": gt.get("bytes", 0.0) / max(gt["launches"], 1),
                 "kernel": "gemm_tcgen05 (all dense products of the joint VJP)",
                 "peak_source": f"bf16_tflops_sustained of {src} peaks",
                 "launches_per_step": gt["launches"],
