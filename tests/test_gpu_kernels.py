@@ -62,6 +62,17 @@ def test_tcgen05_tile_widths(M, N, K, a_mn, b_mn, tile_n):
     assert _rel(C, ref) < 1e-5
     assert _rel(Cb.float(), ref + bias.float()) < 5e-3
     assert _rel(G, G0 + ref) < 1e-5
+    if not a_mn and b_mn and tile_n != 256:
+        # the multiplier epilogue of the input-gradient products (tiles of at most 128
+        # columns), bf16 output into a wider buffer
+        X = torch.rand(M, N, device=dev).bfloat16()
+        O = torch.full((M, N + 8), 3.0, device=dev, dtype=torch.bfloat16)
+        jg.test_gemm(_desc(M, N, K, As, lda, a_mn, Bs, ldb, b_mn, jg.DTYPE_BF16, O, N + 8, jg.DTYPE_BF16, epi=3,
+                           aux=X, ld_aux=N, tile_n=tile_n))
+        torch.cuda.synchronize()
+        assert jg.device_status() == 0
+        assert _rel(O[:, :N].float(), ref * X.float()) < 5e-3
+        assert torch.all(O[:, N:] == 3.0)
 
 
 @pytest.mark.parametrize("a_mn,b_mn", [(False, False), (False, True), (True, True), (True, False)])
