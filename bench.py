@@ -54,7 +54,7 @@ def parse():
     p.add_argument("--quick", action="store_true", help="skip the full-W, e2e and CPU legs")
     p.add_argument("--G", type=int, default=0,
                    help="override the workload's group size (small cases for profiler captures)")
-    p.add_argument("--kernel", choices=["attention_bwd", "gemm"], default=None,
+    p.add_argument("--kernel", choices=["attention_bwd", "attention_fwd", "gemm"], default=None,
                    help="time one kernel family alone on the workload's shapes instead of the step")
     p.add_argument("--product", default="all",
                    help="for --kernel gemm: one of the block's backward products (fc2_dx, fc1_dx, qkv_dx, "
@@ -815,7 +815,7 @@ def run_e2e(b, args, ws, routes):
 
 
 def run_kernel_attention_bwd(args):
-    """The attention backward alone on the workload's joint attention (B sequences, the
+    """The attention backward (or forward) alone on the workload's joint attention (B sequences, the
     text and image streams in their own buffers as in the MMDiT double blocks), timed with
     CUDA events over the timed calls; the kernel's own device time comes from the
     library's per-launch events."""
@@ -839,7 +839,12 @@ def run_kernel_attention_bwd(args):
     views = (split(qkv), split(o), split(dO))
     dq = (torch.empty(B, n0, 3 * d, device=dev, dtype=torch.bfloat16),
           torch.empty(B, N - n0, 3 * d, device=dev, dtype=torch.bfloat16))
-    call = lambda: jg.test_attention_bwd_streams(views[0], views[1], lse, views[2], B, N, n0, H, dh, dq)
+    fwd = args.kernel == "attention_fwd"
+    family = "attention_fwd" if fwd else "attention_bwd"
+    if fwd:  # the forward on the same views: o and lse rewritten each call
+        call = lambda: jg.test_attention_fwd_streams(views[0], views[1], lse, B, N, n0, H, dh)
+    else:
+        call = lambda: jg.test_attention_bwd_streams(views[0], views[1], lse, views[2], B, N, n0, H, dh, dq)
     for _ in range(args.warmup):
         call()
     torch.cuda.synchronize()
@@ -858,17 +863,17 @@ def run_kernel_attention_bwd(args):
         call()
     prof = jg.profile_read()
     jg.profile_enable(False)
-    fam = prof["attention_bwd"]
-    flops = 8.0 * B * H * N * N * dh
+    fam = prof[family]
+    flops = (4.0 if fwd else 8.0) * B * H * N * N * dh
     kms = fam["ms"] / max(fam["launches"], 1)
     burst, sustained, hbm, src = peaks()
     tf = flops / (kms / 1000.0) / 1e12
-    print(json.dumps({"kernel": "attention_bwd", "workload": describe(wl), "rows": B, "heads": H, "head_dim": dh,
+    print(json.dumps({"kernel": family, "workload": describe(wl), "rows": B, "heads": H, "head_dim": dh,
                       "tokens": N, "text_tokens": n0 if n0 < N else 0, "steps": args.steps,
                       "ms_per_call": ms, "kernel_ms": kms, "algorithmic_tflop": flops / 1e12,
                       "roofline": {"bound": "tensor", "achieved": tf, "peak": burst, "unit": "TFLOP/s",
                                    "frac": tf / burst, "peak_source": f"bf16_tflops (burst) of {src} peaks"},
-                      "aux_ms_per_call": prof["attention_bwd_aux"]["ms"] / args.steps}), flush=True)
+                      "aux_ms_per_call": 0.0 if fwd else prof["attention_bwd_aux"]["ms"] / args.steps}), flush=True)
 
 
 def gemm_products(wl, rows):
@@ -952,7 +957,7 @@ def run_kernel_gemm(args):
 def main():
     args = parse()
     ws, rank = dist_setup()
-    if args.kernel == "attention_bwd":
+    if args.kernel in ("attention_bwd", "attention_fwd"):
         if rank == 0:
             run_kernel_attention_bwd(args)
     elif args.kernel == "gemm":
