@@ -118,12 +118,19 @@ def barrier(ws):
 
 
 def max_over_ranks(x: float, ws: int) -> float:
+    """The slowest rank's time (the whole job's step time); host tensors under gloo."""
     if ws == 1:
         return x
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def job_rate(units_per_rank: float, ms_per_step: float, ws: int) -> float:
+    """Whole-job throughput: every rank's units over the slowest rank's step time."""
+    return ws * units_per_rank / (ms_per_step / 1000.0)
 
 
 # ----------------------------------------------------------------------------- clocks
@@ -595,7 +602,7 @@ def run_gpu(args, ws, rank):
         r = measure(b, routes, batched, args, ws, use_graph, profile=True)
     clocks = clk.summary()
     ms = r["ms"]
-    value = ws * units / (ms / 1000.0)
+    value = job_rate(units, ms, ws)
     burst, sustained, hbm, src = peaks()
     fam = {k: v for k, v in r["prof"].items() if v["launches"]}
     gt = fam.get("gemm_tcgen05", {"launches": 0, "ms": 0.0, "flops": 0.0})
