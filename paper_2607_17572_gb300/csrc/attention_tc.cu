@@ -158,7 +158,8 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
   uint64_t* bar_p = kv_free + KVB;          // P^T, dS^T written (S^T, dP^T read) by the 8 warps
   uint64_t* bar_pfree = bar_p + 1;          // the products reading P^T, dS^T are done
   uint64_t* bar_fin = bar_p + 2;            // a unit's products are done (dK, dV final)
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_p + 3);
+  uint64_t* bar_kvout = bar_p + 3;          // the dQ warps have read the unit's dK, dV
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_p + 4);
   __shared__ volatile int abort_flag;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -192,6 +193,7 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
     ptx::mbar_init(bar_p, 8);
     ptx::mbar_init(bar_pfree, 1);
     ptx::mbar_init(bar_fin, 1);
+    ptx::mbar_init(bar_kvout, 4);
     ptx::fence_mbar_init();
     for (int sg = 0; sg < 2; ++sg) {
       ptx::prefetch_tmap(&maps.q[sg]);
@@ -323,6 +325,12 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
             }
           }
           const uint32_t aQ = ptx::smem_u32(sQ + st * C::QT_BYTES), adO = ptx::smem_u32(sdO + st * C::QT_BYTES);
+          // the first dV, dK products of a unit overwrite the accumulators: the dQ warps have
+          // read the previous unit's
+          if (j == 0 && i > 0) {
+            if (!ptx::mbar_wait(bar_kvout, (i - 1) & 1)) { ok = false; break; }
+            ptx::tc_fence_after();
+          }
 #pragma unroll
           for (int k = 0; k < BQ / 16; ++k) {
             const uint32_t acc = (j > 0 || k > 0) ? 1u : 0u;
@@ -405,39 +413,6 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
         if (lane == 0) ptx::mbar_arrive(bar_p);
       }
       if (!ok) break;
-      // the unit's dK, dV; the next unit's first dV, dK products are issued only after
-      // these warps' next P arrival, i.e. after these reads
-      ok = ptx::mbar_wait(bar_fin, i & 1);
-      ok = __all_sync(0xffffffffu, ok);
-      if (!ok) { abort_flag = 1; break; }
-      ptx::tc_fence_after();
-      const int key = k0 + r;
-#pragma unroll 1
-      for (int c = half * (D / 64); c < (half + 1) * (D / 64); ++c) {
-        uint32_t rv[32], rk[32];
-        ptx::tmem_ld_32x32b_x32(trow + C::T_DV + c * 32, rv);
-        ptx::tmem_ld_32x32b_x32(trow + C::T_DK + c * 32, rk);
-        ptx::tmem_ld_wait();
-        if (key < N) {
-          bf16* dv = static_cast<bf16*>(p.dv.base(key)) + p.dv.off(b, key, N, p.dv_col0 + h * D + c * 32);
-          bf16* dk = static_cast<bf16*>(p.dk.base(key)) + p.dk.off(b, key, N, p.dk_col0 + h * D + c * 32);
-#pragma unroll
-          for (int v = 0; v < 4; ++v) {
-            uint4 a, bb;
-            __nv_bfloat162* ha = reinterpret_cast<__nv_bfloat162*>(&a);
-            __nv_bfloat162* hb = reinterpret_cast<__nv_bfloat162*>(&bb);
-#pragma unroll
-            for (int t = 0; t < 4; ++t) {
-              ha[t] = __floats2bfloat162_rn(__uint_as_float(rv[8 * v + 2 * t]), __uint_as_float(rv[8 * v + 2 * t + 1]));
-              hb[t] = __floats2bfloat162_rn(__uint_as_float(rk[8 * v + 2 * t]) * p.scale,
-                                            __uint_as_float(rk[8 * v + 2 * t + 1]) * p.scale);
-            }
-            *reinterpret_cast<uint4*>(dv + 8 * v) = a;
-            *reinterpret_cast<uint4*>(dk + 8 * v) = bb;
-          }
-        }
-      }
-      ptx::tc_fence_before();
     }
   } else {
     // ---------------------------------------------------------------- dQ -> f32 reduce-add
@@ -449,7 +424,6 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
     for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++i) {
       int k0, b, h;
       unit_of(u, k0, b, h);
-      (void)k0;
       for (int j = 0; j < nq; ++j) {
         const int g = i * nq + j;
         const int bb = g % NSB;
@@ -498,6 +472,41 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
           }
         }
       }
+      if (!ok) break;
+      // the unit's dK, dV (key rows of this warp's lane quarter): the P / dS warps move on to
+      // the next unit meanwhile
+      ok = __all_sync(0xffffffffu, ptx::mbar_wait(bar_fin, i & 1));
+      if (!ok || abort_flag) { ok = false; abort_flag = 1; break; }
+      ptx::tc_fence_after();
+      const int key = k0 + quarter * 32 + lane;
+#pragma unroll 1
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t rv[32], rk[32];
+        ptx::tmem_ld_32x32b_x32(trow + C::T_DV + c * 32, rv);
+        ptx::tmem_ld_32x32b_x32(trow + C::T_DK + c * 32, rk);
+        ptx::tmem_ld_wait();
+        if (key < N) {
+          bf16* dv = static_cast<bf16*>(p.dv.base(key)) + p.dv.off(b, key, N, p.dv_col0 + h * D + c * 32);
+          bf16* dk = static_cast<bf16*>(p.dk.base(key)) + p.dk.off(b, key, N, p.dk_col0 + h * D + c * 32);
+#pragma unroll
+          for (int v = 0; v < 4; ++v) {
+            uint4 a, bb;
+            __nv_bfloat162* ha = reinterpret_cast<__nv_bfloat162*>(&a);
+            __nv_bfloat162* hb = reinterpret_cast<__nv_bfloat162*>(&bb);
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+              ha[t] = __floats2bfloat162_rn(__uint_as_float(rv[8 * v + 2 * t]), __uint_as_float(rv[8 * v + 2 * t + 1]));
+              hb[t] = __floats2bfloat162_rn(__uint_as_float(rk[8 * v + 2 * t]) * p.scale,
+                                            __uint_as_float(rk[8 * v + 2 * t + 1]) * p.scale);
+            }
+            *reinterpret_cast<uint4*>(dv + 8 * v) = a;
+            *reinterpret_cast<uint4*>(dk + 8 * v) = bb;
+          }
+        }
+      }
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(bar_kvout);
     }
     if (lane == 0) ptx::bulk_wait<0>();
     __syncwarp();
