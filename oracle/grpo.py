@@ -2,7 +2,7 @@
 
 TEST INFRASTRUCTURE ONLY (see oracle/__init__.py).
 
-Readings of passages the paper leaves open (each is also listed in the design doc):
+Readings of passages the paper leaves open:
   * advantage: eps = 1e-8, unbiased (Bessel) group std, clamp to +-adv_clip (5.0 in the
     hyper-parameter table);
   * log-prob: the isotropic Gaussian density of the whole latent, i.e. the normalising
