@@ -87,3 +87,29 @@ def test_route_argument_errors(jg):
     route = (ctypes.c_uint8 * 4)()
     assert jg.lib().jagg_route(4, 1.5, None, 0.5, route, None) == -1
     assert jg.lib().jagg_route(0, 0.5, None, 0.5, route, None) == -1
+
+
+def test_host_argument_checks_of_the_signal_and_sampler_entry_points(jg):
+    """Argument errors are caught on the host before any launch (so these calls run without a
+    device): a missing schedule, a non-positive noise scale, too small a workspace, strides
+    below the row length, a span whose endpoint times coincide."""
+    L = jg.lib()
+    fake = 1 << 20                                   # never dereferenced: every call fails first
+    ws = 256
+    # grpo_step_signals_eps without a schedule
+    st = L.grpo_step_signals_eps(fake, 0, fake, fake, None, None, fake, fake, fake, 2, 3, 100, 0.1, 5.0, 1e-8,
+                                 1.0, None, None, fake, fake, fake, fake, fake, ws, None)
+    assert st < 0 and "schedule" in L.jagg_last_error().decode()
+    # jagg_rollout_step: sigma must be positive; workspace size; strides
+    args = lambda sigma, zs, wsb: (fake, 0, 0, fake, fake, zs, fake, 0, 2, 100, 0.9, 0.8, sigma, None, fake, 1, None,
+                                   0, fake, wsb, None)
+    assert L.jagg_rollout_step(*args(0.0, 0, 1 << 20)) < 0
+    assert "sigma" in L.jagg_last_error().decode()
+    assert L.jagg_rollout_step(*args(0.1, 0, 8)) == -5        # JAGG_ERR_WORKSPACE
+    assert "workspace" in L.jagg_last_error().decode()
+    assert L.jagg_rollout_step(*args(0.1, 50, 1 << 20)) < 0
+    assert "stride" in L.jagg_last_error().decode()
+    assert L.jagg_rollout_workspace_bytes(2, 100) >= 2 * 8
+    # jagg_aggregate_span with equal endpoint times
+    assert L.jagg_aggregate_span(fake, 0, fake, 0.5, 0.5, 2, 3, 100, fake, 0, None) < 0
+    assert "endpoints" in L.jagg_last_error().decode()
