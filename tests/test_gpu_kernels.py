@@ -169,6 +169,33 @@ def test_gemm_epilogues(M, N, K):
     assert jg.device_status() == 0
 
 
+@pytest.mark.parametrize("tile_n", [0, 64, 128])
+@pytest.mark.parametrize("M,N,K,rows", [(300, 100, 192, 37), (1000, 768, 256, 333), (129, 264, 64, 129)])
+def test_gated_residual_epilogue(M, N, K, rows, tile_n):
+    """y = X W^T + b to C (bf16) and h_out = h_in + gate[seq(m)] * y (f32) to C2, with the
+    residual input TMA-loaded per 32 x 32 chunk: ragged rows and columns, sequences that
+    start inside a tile, outputs inside wider buffers."""
+    torch.manual_seed(M + N + K + tile_n)
+    dev = "cuda"
+    A = torch.randn(M, K, device=dev).bfloat16()
+    B = (torch.randn(N, K, device=dev) / math.sqrt(K)).bfloat16()
+    bias = torch.randn(N, device=dev).bfloat16()
+    gate = torch.randn((M + rows - 1) // rows, N + 4, device=dev)
+    hin = torch.randn(M, N + 4, device=dev)
+    Y = torch.full((M, N + 8), 5.0, device=dev, dtype=torch.bfloat16)
+    H = torch.full((M, N + 4), 7.0, device=dev)
+    jg.test_gemm(_desc(M, N, K, A, K, 0, B, K, 0, jg.DTYPE_BF16, Y, N + 8, jg.DTYPE_BF16, epi=2, bias=bias, C2=H,
+                       ldc2=N + 4, aux=hin, ld_aux=N + 4, gate=gate, gate_stride=N + 4, rows_per_seq=rows,
+                       tile_n=tile_n))
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    y = A.float() @ B.float().t() + bias.float()
+    g = gate[torch.arange(M, device=dev) // rows, :N]
+    assert _rel(Y[:, :N].float(), y) < 5e-3
+    assert _rel(H[:, :N], hin[:, :N] + g * y) < 1e-5
+    assert torch.all(Y[:, N:] == 5.0) and torch.all(H[:, N:] == 7.0)
+
+
 @pytest.mark.parametrize("split", [0, 1, 3])
 def test_gemm_accumulate_weight_gradient(split):
     """dW += dY^T X with both operands MN-major, accumulated into an existing f32 buffer."""
