@@ -226,10 +226,12 @@ class Bench:
         self.sig_dev = torch.tensor(self.sig, **f64)
         self.rewards = torch.tensor(self.draws.rewards, dtype=torch.float32, device=dev)
         self.txt1 = torch.tensor(self.draws.txt, dtype=self.tdt, device=dev)
-        # workspace for the largest single call: every window's W*G rows at once when they
-        # can be resident together, else one window's
+        # workspace for the largest single call: one window's W*G rows, or the batched calls
+        # over every window (2G endpoint rows each, or W*G step rows each) when their saved
+        # activations can be resident (the test `fits` applies, against free memory)
         total = torch.cuda.get_device_properties(dev).total_memory
-        ws_rows = self.nw * W * G if self.model.saved_bytes(self.nw * W * G) < 0.4 * total else W * G
+        cands = [W * G] + [r for r in (2 * G * self.nw, W * G * self.nw) if self.model.saved_bytes(r) < 0.5 * total]
+        ws_rows = max(cands)
         self.ws = jg.alloc_bytes(self.model.workspace_bytes(ws_rows), dev)
         self.sws = jg.alloc_bytes(jg.signals_workspace_bytes(G, W, self.D), dev)
         self.rws = jg.alloc_bytes(jg.rollout_workspace_bytes(G, self.D), dev)
