@@ -231,8 +231,8 @@ class Bench:
         # activations can be resident (the test `fits` applies, against free memory)
         total = torch.cuda.get_device_properties(dev).total_memory
         cands = [W * G] + [r for r in (2 * G * self.nw, W * G * self.nw) if self.model.saved_bytes(r) < 0.5 * total]
-        ws_rows = max(cands)
-        self.ws = jg.alloc_bytes(self.model.workspace_bytes(ws_rows), dev)
+        self.ws_rows = max(cands)
+        self.ws = jg.alloc_bytes(self.model.workspace_bytes(self.ws_rows), dev)
         self.sws = jg.alloc_bytes(jg.signals_workspace_bytes(G, W, self.D), dev)
         self.rws = jg.alloc_bytes(jg.rollout_workspace_bytes(G, self.D), dev)
         self.gws = jg.alloc_bytes(jg.grad_reduce_workspace_bytes(self.P), dev)
@@ -325,10 +325,11 @@ class Bench:
         return self.fits(routes)
 
     def fits(self, routes) -> bool:
-        """Every window's saved activations fit in half of the free device memory."""
+        """Every window's saved activations fit in half of the free device memory (and the
+        workspace covers that many rows)."""
         _, rows = self.plan(routes)
         free, _ = torch.cuda.mem_get_info(self.dev)
-        return self.model.saved_bytes(rows) < 0.5 * free
+        return rows <= self.ws_rows and self.model.saved_bytes(rows) < 0.5 * free
 
     def forward_saves(self, routes, batched, windows=None):
         """Phase 1 with saves for the rows of the plan (or of the listed windows only).
