@@ -10,6 +10,7 @@
  *   grpo_step_signals  Phase 2: s_j = dL_j/dv_j through Eq. logprob and Eq. grpo_loss
  *                      (grpo_step_signals_eps: the same for an epsilon-prediction model)
  *   jagg_aggregate     Phase 3: Eq. alpha and Eq. s_base_corr
+ *                      (jagg_aggregate_span: over a span of a window's steps)
  *   jagg_route         jagg_frac routing (Sec. 3.3 and the gradient-quality appendix)
  *   jagg_rollout_step  one rollout sampler step with the log-prob of its sample
  *   dit_joint_vjp      Phase 4: grad += sum_rows J(z_row, t_row)^T cot_row
