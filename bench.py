@@ -98,15 +98,21 @@ def peaks():
 
 
 # ----------------------------------------------------------------------------- distributed
-def dist_setup():
+def dist_setup(need_gpu: bool = True):
+    """One rank per GPU (NCCL).  The reference arm (the float64 oracle on the host cores)
+    needs no GPU: without one its ranks meet over gloo."""
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
+    gpu = need_gpu or torch.cuda.is_available()
     if ws > 1:
         import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    else:
+        if gpu:
+            torch.cuda.set_device(local)
+            dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        else:
+            dist.init_process_group("gloo")
+    elif gpu:
         torch.cuda.set_device(0)
     return ws, rank
 
@@ -966,7 +972,7 @@ def run_kernel_gemm(args):
 
 def main():
     args = parse()
-    ws, rank = dist_setup()
+    ws, rank = dist_setup(need_gpu=args.impl != "reference" or args.kernel is not None)
     if args.kernel in ("attention_bwd", "attention_fwd"):
         if rank == 0:
             run_kernel_attention_bwd(args)
