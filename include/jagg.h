@@ -46,7 +46,7 @@ extern "C" {
 /* ----------------------------------------------------------------- status codes */
 #define JAGG_OK 0
 #define JAGG_ERR_ARG (-1)          /* invalid pointer, size, alignment or config     */
-#define JAGG_ERR_UNSUPPORTED (-2)  /* valid request this build does not implement     */
+#define JAGG_ERR_UNSUPPORTED (-2)  /* valid request the library does not implement   */
 #define JAGG_ERR_CUDA (-3)         /* a CUDA runtime/driver call failed               */
 #define JAGG_ERR_TIMEOUT (-4)      /* a bounded device wait gave up                   */
 #define JAGG_ERR_WORKSPACE (-5)    /* workspace or saved arena smaller than required  */
