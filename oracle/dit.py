@@ -143,26 +143,46 @@ def rms_bwd(dy, x, r, g):
     return dx, dg
 
 
-def attention(q, k, v):
-    """q, k, v: [B, N, h, dh] -> o [B, N, h, dh], probabilities P [B, h, N, N]."""
-    dh = q.shape[-1]
-    S = np.einsum("bnhd,bmhd->bhnm", q, k) / np.sqrt(dh)
+def softmax_probs(qh, kh):
+    """P = softmax(qh kh^T / sqrt(dh)) row by row, for one (sequence, head): qh, kh [N, dh]
+    -> P [N, N] (row n: the weights query n gives the keys)."""
+    S = qh @ kh.T / np.sqrt(qh.shape[-1])
     S = S - S.max(-1, keepdims=True)
     P = np.exp(S)
     P /= P.sum(-1, keepdims=True)
-    o = np.einsum("bhnm,bmhd->bnhd", P, v)
-    return o, P
+    return P
 
 
-def attention_bwd(do, q, k, v, P):
+def attention(q, k, v, keep_probs=False):
+    """q, k, v: [B, N, h, dh] -> o [B, N, h, dh] (and the probabilities P [B, h, N, N] if
+    keep_probs), one (sequence, head) at a time: o = P v."""
+    B, N, h, _ = q.shape
+    o = np.empty(v.shape)
+    P_all = np.empty((B, h, N, N)) if keep_probs else None
+    for b in range(B):
+        for j in range(h):
+            P = softmax_probs(q[b, :, j], k[b, :, j])
+            o[b, :, j] = P @ v[b, :, j]
+            if keep_probs:
+                P_all[b, j] = P
+    return o, P_all
+
+
+def attention_bwd(do, q, k, v):
     """dV = P^T dO, dP = dO V^T, dS = P*(dP - rowsum(dP*P)), dQ = dS K/sqrt(dh),
-    dK = dS^T Q/sqrt(dh)  (appendix, Eqs. bwd_V .. bwd_QK)."""
-    dh = q.shape[-1]
-    dv = np.einsum("bhnm,bnhd->bmhd", P, do)
-    dP = np.einsum("bnhd,bmhd->bhnm", do, v)
-    dS = P * (dP - (dP * P).sum(-1, keepdims=True))
-    dq = np.einsum("bhnm,bmhd->bnhd", dS, k) / np.sqrt(dh)
-    dk = np.einsum("bhnm,bnhd->bmhd", dS, q) / np.sqrt(dh)
+    dK = dS^T Q/sqrt(dh)  (appendix, Eqs. bwd_V .. bwd_QK), one (sequence, head) at a time;
+    P is formed again from q and k exactly as the forward formed it."""
+    B, N, h, dh = q.shape
+    dq, dk, dv = np.empty(q.shape), np.empty(k.shape), np.empty(v.shape)
+    for b in range(B):
+        for j in range(h):
+            qh, kh, vh, doh = q[b, :, j], k[b, :, j], v[b, :, j], do[b, :, j]
+            P = softmax_probs(qh, kh)
+            dv[b, :, j] = P.T @ doh
+            dP = doh @ vh.T
+            dS = P * (dP - (dP * P).sum(-1, keepdims=True))
+            dq[b, :, j] = dS @ kh / np.sqrt(dh)
+            dk[b, :, j] = dS.T @ qh / np.sqrt(dh)
     return dq, dk, dv
 
 
@@ -218,8 +238,8 @@ class Backbone:
         if wl.rope:
             q = rope_apply(q, self.ang)
             k = rope_apply(k, self.ang)
-        o, P = attention(q, k, v)
-        cache.update(q=q, k=k, v=v, P=P)
+        o, _ = attention(q, k, v)
+        cache.update(q=q, k=k, v=v)
         return o.reshape(B, N, d), cache
 
     def _attn_bwd(self, do, cache, qn=None, kn=None):
@@ -227,7 +247,7 @@ class Backbone:
         wl = self.wl
         B, N, d = do.shape
         h, dh = wl.heads, wl.head_dim
-        dq, dk, dv = attention_bwd(do.reshape(B, N, h, dh), cache["q"], cache["k"], cache["v"], cache["P"])
+        dq, dk, dv = attention_bwd(do.reshape(B, N, h, dh), cache["q"], cache["k"], cache["v"])
         if wl.rope:
             dq = rope_apply(dq, self.ang, inverse=True)
             dk = rope_apply(dk, self.ang, inverse=True)
