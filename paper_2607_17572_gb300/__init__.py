@@ -197,12 +197,13 @@ def param_count(cfg: Config) -> int:
 
 
 def pack_params(cfg: Config, arrays: dict, device="cuda") -> torch.Tensor:
-    """Places named parameter arrays into one flat buffer in the library's layout."""
-    flat = torch.zeros(param_count(cfg), dtype=cfg.torch_dtype)
+    """Places named parameter arrays (host arrays or device tensors) into one flat buffer in
+    the library's layout on `device`."""
+    flat = torch.zeros(param_count(cfg), dtype=cfg.torch_dtype, device=device)
     for p in param_table(cfg):
         a = torch.as_tensor(arrays[p.name]).reshape(-1)
-        flat[p.offset:p.offset + p.numel] = a.to(cfg.torch_dtype)
-    return flat.to(device)
+        flat[p.offset:p.offset + p.numel] = a.to(device=device, dtype=cfg.torch_dtype)
+    return flat
 
 
 def unpack_grads(cfg: Config, grad: torch.Tensor) -> dict:

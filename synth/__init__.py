@@ -127,9 +127,11 @@ def small_variant(wl: Workload, **over) -> Workload:
 # same representable numbers.
 # ----------------------------------------------------------------------------------
 def bf16_bits(x) -> np.ndarray:
+    """Bit patterns of the nearest bf16 values (ties to even) of finite inputs.  The sum
+    stays below 2^32 for every finite or infinite float32 (NaN is never rounded here)."""
     f = np.ascontiguousarray(np.asarray(x, dtype=np.float32))
-    u = f.view(np.uint32).astype(np.uint64)
-    rounded = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    u = f.view(np.uint32)
+    rounded = (u + np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1))) >> np.uint32(16)
     return rounded.astype(np.uint16)
 
 
@@ -208,6 +210,28 @@ def make_params(wl: Workload, seed: int = WEIGHT_SEED, bias_scale: float = 0.02)
         else:
             v = rng.uniform(-bias_scale, bias_scale, size=shape)
         params[name] = storage_round(v, wl.dtype)
+    return params
+
+
+def device_params(wl: Workload, seed: int = WEIGHT_SEED, device="cuda", bias_scale: float = 0.02):
+    """The draws of make_params (Xavier-uniform matrices, small uniform biases, RMSNorm
+    scales near 1, rounded to the storage type) made by torch's generator on a device:
+    seconds for the 2.5 B parameters of the Flux-width models, where the host generator
+    takes minutes.  Returns {name: float32 device tensor}.  A different stream of numbers
+    from make_params with the same seed; both sides of a comparison take the one dict."""
+    import torch
+    gen = torch.Generator(device=device).manual_seed(seed)
+    params = {}
+    for name, shape in param_shapes(wl):
+        v = torch.empty(shape, dtype=torch.float32, device=device)
+        if len(shape) == 2:
+            bound = math.sqrt(6.0 / (shape[0] + shape[1]))
+            v.uniform_(-bound, bound, generator=gen)
+        elif name.endswith("_norm"):
+            v.uniform_(0.9, 1.1, generator=gen)
+        else:
+            v.uniform_(-bias_scale, bias_scale, generator=gen)
+        params[name] = v.bfloat16().float() if wl.dtype == "bf16" else v
     return params
 
 

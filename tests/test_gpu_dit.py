@@ -6,6 +6,7 @@ import torch
 
 import synth
 from gpu_cases import GpuModel, cosine, flat, model_inputs, oracle_vjp, rel_l2
+from oracle import dit, path
 
 pytestmark = pytest.mark.gpu
 
@@ -61,6 +62,10 @@ def _check(wl, B, ftol, gtol, seed=5):
     print(f"{wl.name}: forward {fv:.2e}, grad rel L2 {tot:.2e}, cos {cs:.6f}, worst {worst} {per[worst]:.2e}")
     assert tot <= gtol, f"gradient rel L2 {tot:.3e} (worst {worst}: {per[worst]:.3e})"
     assert cs >= 0.999
+    # every tensor on its own, so that a wrong gradient of a small tensor (a bias, a norm
+    # scale, the final layer) cannot hide under the norm of the large ones
+    bad = {k: e for k, e in per.items() if e > 5 * gtol}
+    assert not bad, f"tensors beyond {5 * gtol:.0e}: {bad}"
     return grad, gm, saved, ws, cot
 
 
@@ -127,3 +132,52 @@ def test_sequential_graph_variant_matches_the_joint_vjp(wl, G, tol):
     r = rel_l2(g_seq.cpu().numpy(), g_joint.cpu().numpy())
     print(f"{wl.name}: sequential vs joint rel L2 {r:.2e}")
     assert r <= tol
+
+
+@pytest.mark.parametrize("wl,G,tol", [(TINY, 4, 1e-4), (synth.small_variant(DITB, name="ditb_2blocks", depth=2), 4,
+                                                        1e-2)], ids=["tiny_f32", "ditb_2blocks_bf16"])
+def test_sequential_graph_variant_matches_oracle(wl, G, tol):
+    """Algorithm 2 against the oracle's JAGG window gradient.  In the variant's order: the
+    signals of steps 0..W-2 are aggregated (jagg_aggregate_span against the window's endpoint
+    times) into both rows; endpoint 0 is forwarded into the one G-row arena and its VJP
+    takes s_base; the last step's signal is added to s_corr; endpoint W-1 is forwarded into
+    the same arena and its VJP takes s_corr.  The oracle: path.window_gradient (Eq.
+    s_base_corr, one joint VJP over both endpoints) on the same signals."""
+    W = wl.W
+    params = synth.make_params(wl)
+    rng = np.random.Generator(np.random.PCG64(31))
+    z_win = synth.storage_round(rng.standard_normal((G, W, wl.in_channels, wl.latent_h, wl.latent_w)), wl.dtype)
+    txt = synth.storage_round(rng.standard_normal((wl.txt_len, wl.txt_dim)), wl.dtype)
+    t = synth.time_grid(8, 3.0)[1:W + 1].astype(np.float32).astype(np.float64)    # shifted: alpha != j/(W-1)
+    s = rng.standard_normal((G, W) + z_win.shape[2:]).astype(np.float32).astype(np.float64)
+    gm = GpuModel(jg, wl, params)
+    dev = "cuda"
+    f64 = dict(dtype=torch.float64, device=dev)
+    st = torch.tensor(s.reshape(G, W, -1), dtype=torch.float32, device=dev)
+    cot = torch.empty(2 * G, st.shape[-1], dtype=torch.float32, device=dev)
+    arena = jg.alloc_bytes(gm.model.saved_bytes(G))
+    ws = jg.alloc_bytes(gm.model.workspace_bytes(G))
+    grad = torch.zeros(jg.param_count(gm.cfg), dtype=torch.float32, device=dev)
+    txt_g = gm.tensor(np.broadcast_to(txt, (G,) + txt.shape))
+    jg.jagg_aggregate_span(st, torch.tensor(t[:W - 1], **f64), t[0], t[W - 1], cot, steps=(0, W - 1))
+    for e, j in enumerate((0, W - 1)):
+        if e == 1:
+            jg.jagg_aggregate_span(st, torch.tensor(t[W - 1:], **f64), t[0], t[W - 1], cot, accumulate=True,
+                                   steps=(W - 1, 1))
+        zt = gm.tensor(z_win[:, j])
+        jg.dit_forward_save(gm.model, zt, torch.full((G,), float(t[j]), dtype=torch.float32, device=dev), txt_g,
+                            torch.empty_like(zt), saved=arena, ws=ws)
+        jg.dit_joint_vjp(gm.model, arena, G, cot[e * G:(e + 1) * G].reshape(G, *z_win.shape[2:]).contiguous(),
+                         grad, ws)
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    g_o = path.window_gradient(dit.Backbone(wl, params), z_win, t, txt, s, jagg=True)
+    g_gpu = jg.unpack_grads(gm.cfg, grad)
+    names = list(g_o)
+    err, cs = rel_l2(flat(g_gpu, names), flat(g_o, names)), cosine(flat(g_gpu, names), flat(g_o, names))
+    per = {k: rel_l2(g_gpu[k], g_o[k]) for k in names}
+    worst = max(per, key=per.get)
+    print(f"{wl.name}: sequential graph vs oracle rel L2 {err:.2e}, cos {cs:.7f}, worst {worst} {per[worst]:.2e}")
+    assert err <= tol and cs >= 0.999
+    bad = {k: e for k, e in per.items() if e > 5 * tol}
+    assert not bad, f"tensors beyond {5 * tol:.0e}: {bad}"

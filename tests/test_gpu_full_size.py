@@ -129,6 +129,8 @@ def test_full_size_bf16_path_matches_torch_fp32(name, B):
     assert fv <= 2e-2
     assert fg <= 1e-2, f"gradient rel L2 {fg:.3e} (worst {worst}: {per[worst]:.3e})"
     assert cg >= 0.999
+    bad = {k: e for k, e in per.items() if e > 5e-2}
+    assert not bad, f"tensors beyond 5e-2: {bad}"
 
 
 @pytest.mark.parametrize("name", ["mmdit_flux512_bf16", "mmdit_qwen_sweep_bf16"])

@@ -335,3 +335,87 @@ def test_rollout_step_rejects_bad_arguments():
         jg.jagg_rollout_step(y, z, 0, y, 0.5, 0.4, 0.0, logp, ws)     # sigma must be positive
     with pytest.raises(jg.JaggError):
         jg.jagg_rollout_step(y, z, 0, y, 0.5, 0.4, 0.1, logp, jg.alloc_bytes(8))   # workspace too small
+
+
+# ------------------------------------------------------------------ clip decisions at the boundary
+def _dyadic_case(G, W, D, v_dtype, seed):
+    """A window whose residuals r = z_{j+1} - z_j - v_j dt_j are computed exactly by both
+    sides: a uniform grid (dt = -1/8), v multiples of 2^-4 in [-4, 4] (exact in bf16), noise
+    multiples of 2^-8 in [-1/2, 1/2].  Every partial sum of r^2 is then exact in float32, so
+    the library's log-prob equals the oracle's to the rounding of the f64 normaliser."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    q = lambda x, step, lim: np.clip(np.round(x / step) * step, -lim, lim)
+    t = synth.time_grid(2 * W, 1.0)[:W + 1]
+    sig = synth.sigma_schedule(t, 0.7)
+    v = q(rng.standard_normal((G, W, D)), 2.0 ** -4, 4.0)
+    z = np.zeros((G, W + 1, D))
+    z[:, 0] = q(rng.standard_normal((G, D)), 2.0 ** -8, 4.0)
+    for j in range(W):
+        z[:, j + 1] = z[:, j] + v[:, j] * (t[j + 1] - t[j]) + q(sig[j] * rng.standard_normal((G, D)), 2.0 ** -8, 0.5)
+    assert np.array_equal(z.astype(np.float32), z)
+    lp = np.array([[grpo.step_logprob(z[i, j + 1], z[i, j], v[i, j], t[j], t[j + 1], sig[j]) for j in range(W)]
+                   for i in range(G)])
+    rewards = synth.storage_round(rng.standard_normal(G), "f32")
+    return v, z, t, sig, lp, rewards, rng
+
+
+def _signals_call(v, z, t, sig, lpo, rewards, eps, scale, v_dtype):
+    dev = "cuda"
+    G, W, D = v.shape
+    f64 = dict(dtype=torch.float64, device=dev)
+    out = dict(logp_new=torch.empty(G, W, **f64), ratio=torch.empty(G, W, **f64),
+               clipped=torch.empty(G, W, dtype=torch.uint8, device=dev), adv_out=torch.empty(G, **f64))
+    s = torch.full((G, W, D), float("nan"), device=dev)
+    ws = jg.alloc_bytes(jg.signals_workspace_bytes(G, W, D))
+    jg.grpo_step_signals(torch.tensor(v, dtype=torch.bfloat16 if v_dtype == "bf16" else torch.float32, device=dev),
+                         torch.tensor(z, dtype=torch.float32, device=dev), torch.tensor(t, **f64),
+                         torch.tensor(sig, **f64), torch.tensor(lpo, **f64),
+                         torch.tensor(rewards, dtype=torch.float32, device=dev), eps, 5.0, 1e-8, scale, ws=ws,
+                         s_out=s, **out)
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    return s.cpu().numpy(), {k: x.cpu().numpy() for k, x in out.items()}
+
+
+@pytest.mark.parametrize("D,v_dtype", [(4096, "f32"), (65536, "bf16")])
+def test_clip_mask_near_the_boundary_matches_oracle(D, v_dtype):
+    """log rho placed within (1e-6, 1e-3) of log(1 + eps) or log(1 - eps), on either side
+    (log-uniform distances): the clip decisions agree with the oracle bit for bit."""
+    G, W, eps = 8, 4, 0.1
+    v, z, t, sig, lp, rewards, rng = _dyadic_case(G, W, D, v_dtype, seed=D + 1)
+    bound = np.where(rng.uniform(size=(G, W)) < 0.5, np.log1p(eps), np.log1p(-eps))
+    margin = 10.0 ** rng.uniform(-6, -3, (G, W)) * rng.choice([-1.0, 1.0], (G, W))
+    lpo = lp - (bound + margin)
+    scale = 1.0 / (G * 16)
+    A = grpo.advantages(rewards)
+    s_o, lp_o, ratio_o, clip_o = grpo.step_signals(v, z, t, sig, lpo, A, eps, scale)
+    s, out = _signals_call(v, z, t, sig, lpo, rewards, eps, scale, v_dtype)
+    assert np.max(np.abs(out["logp_new"] - lp_o)) <= 1e-9 * max(1.0, np.abs(lp_o).max())
+    np.testing.assert_array_equal(out["clipped"], clip_o)
+    assert 0 < clip_o.sum() < G * W            # both outcomes occur
+    assert _rel(s, s_o) < 1e-6
+
+
+def test_clip_tie_counts_as_unclipped_on_the_device():
+    """rho = 1 + eps with A > 0 (and rho = 1 - eps with A < 0) exactly, eps formed in float64
+    from the library's own ratio: the step keeps its gradient, bit-equal to the one it gets
+    under a wide clip range; one ulp of rho past the tie it is clipped."""
+    G, W, D = 6, 4, 4096
+    v, z, t, sig, lp, rewards, rng = _dyadic_case(G, W, D, "f32", seed=77)
+    lpo = lp - rng.uniform(-0.08, 0.08, (G, W))
+    scale = 1.0 / (G * 16)
+    A = grpo.advantages(rewards)
+    s_wide, out = _signals_call(v, z, t, sig, lpo, rewards, 0.5, scale, "f32")
+    assert not out["clipped"].any()
+    rho = out["ratio"]
+    for sign in (1.0, -1.0):
+        cand = [(i, j) for i in range(G) for j in range(W) if A[i] * sign > 0 and (rho[i, j] - 1.0) * sign > 0]
+        i, j = cand[0]
+        eps_tie = (rho[i, j] - 1.0) * sign                   # exact: 1 +- eps_tie == rho[i, j]
+        assert 1.0 + sign * eps_tie == rho[i, j]
+        s_tie, o_tie = _signals_call(v, z, t, sig, lpo, rewards, eps_tie, scale, "f32")
+        assert o_tie["clipped"][i, j] == 0 and o_tie["ratio"][i, j] == rho[i, j]
+        np.testing.assert_array_equal(s_tie[i, j], s_wide[i, j])
+        assert np.abs(s_tie[i, j]).sum() > 0
+        _, o_past = _signals_call(v, z, t, sig, lpo, rewards, eps_tie - np.spacing(rho[i, j]), scale, "f32")
+        assert o_past["clipped"][i, j] == 1

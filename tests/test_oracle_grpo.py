@@ -306,3 +306,26 @@ def test_sampler_step_without_noise_follows_the_flow():
     e = z + (1 - t0) * v
     zn2, _ = oracle_rollout.sampler_step(z, e, xi, t0, t1, 1e-12, sched=(1 - t0, 1 - t1, t0, t1))
     np.testing.assert_allclose(zn2, zn, atol=1e-6)
+
+
+def test_clip_tie_counts_as_unclipped():
+    """At rho = 1 + eps (A > 0) or rho = 1 - eps (A < 0) exactly, both branches of the max()
+    in Eq. grpo_loss have the same value; the step keeps its gradient, which equals the one
+    it has under a wider clip range."""
+    G, W = 2, 1
+    v, z, t, sig, lp, _ = _signals_case(6, W=W, G=G, rho_shift=np.zeros((G, W)), eps=0.1)
+    for A, log_rho in [(1.0, 0.07), (-1.0, -0.07)]:
+        lpo = lp - log_rho
+        _, _, ratio, _ = grpo.step_signals(v, z, t, sig, lpo, np.array([A, A]), 0.5, 1.0)
+        rho = ratio[0, 0]
+        eps_tie = rho - 1.0 if A > 0 else 1.0 - rho     # exact (Sterbenz): 1 +- eps_tie == rho
+        assert (1.0 + eps_tie == rho) if A > 0 else (1.0 - eps_tie == rho)
+        s_tie, _, _, clipped = grpo.step_signals(v, z, t, sig, lpo, np.array([A, A]), eps_tie, 1.0)
+        s_wide, _, _, _ = grpo.step_signals(v, z, t, sig, lpo, np.array([A, A]), 0.5, 1.0)
+        assert clipped[0, 0] == 0
+        np.testing.assert_array_equal(s_tie[0], s_wide[0])
+        assert np.abs(s_tie[0]).sum() > 0
+        # one ulp of rho past the tie the clipped branch is strictly larger
+        past = eps_tie - np.spacing(rho)
+        _, _, _, clipped = grpo.step_signals(v, z, t, sig, lpo, np.array([A, A]), past, 1.0)
+        assert clipped[0, 0] == 1
