@@ -229,8 +229,11 @@ int grpo_step_signals_eps(const void* eps_hat, int eps_dtype, const float* z, co
  * the library until the process exits).  It allocates nothing.
  *   - Requests whose scratch need (jagg_signals_workspace_bytes(G, W, D)) exceeds
  *     JAGG_SIGNALS_STATIC_SCRATCH_BYTES fail with JAGG_ERR_WORKSPACE before any launch.
+ *   - The stream must belong to the current device (JAGG_ERR_ARG otherwise).
  *   - The first call on a device looks up the array's device address (a synchronous
- *     runtime query); make that first call before any stream capture on that device.
+ *     runtime query) and keeps it for the life of the process; make that first call before
+ *     any stream capture on that device.  A device reset (cudaDeviceReset) after it is not
+ *     supported: the kept address would be stale.
  *   - Every call shares the one array: calls whose kernels may overlap on the GPU (on
  *     different streams without ordering between them) race and give wrong results.
  *     Nothing in the array needs to start at zero; each call overwrites what it reads. */

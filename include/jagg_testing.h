@@ -81,6 +81,15 @@ int jagg_test_attention_bwd_streams(const void* qkv0, const void* qkv1, const vo
                                     int heads, int dh, int dtype, void* dqkv0, void* dqkv1, void* scratch, int impl,
                                     cudaStream_t stream);
 
+/* Failure detection of the bounded waits (every mbarrier wait of the library gives up after
+ * a wall-clock limit instead of hanging): one CTA waits on an mbarrier that nothing arrives
+ * at, with the limit limit_ns (0 < limit_ns <= 2 s, else JAGG_ERR_ARG) in place of the
+ * library's 2 s.  The wait gives up, sets JAGG_DEV_STATUS_TIMEOUT in the device status word
+ * (read and cleared by jagg_device_status) and the kernel returns; no copy or MMA is in
+ * flight.  out device [2] u64: out[0] = 1 when the wait gave up, out[1] = the nanoseconds
+ * it waited. */
+int jagg_test_wait_timeout(unsigned long long limit_ns, unsigned long long* out, cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

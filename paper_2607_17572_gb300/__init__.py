@@ -112,6 +112,7 @@ _SIGNATURES = {
     "jagg_grad_reduce_workspace_bytes": (_I64, [_I64]),
     "grad_reduce": (_I, [_P, _P, _I64, ctypes.c_float, _P, _P, _P, _SZ, _P]),
     "jagg_test_gemm": (_I, [ctypes.POINTER(GemmDesc), _P]),
+    "jagg_test_wait_timeout": (_I, [ctypes.c_ulonglong, _P, _P]),
     "jagg_test_attention_fwd": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _P]),
     "jagg_test_attention_scratch_bytes": (_I64, [_I, _I, _I, _I]),
     "jagg_test_attention_bwd": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _P]),
@@ -449,3 +450,10 @@ def test_attention_bwd_streams(qkv, o, lse, dO, B, N, n0, heads, dh, dqkv, impl=
     _check(lib().jagg_test_attention_bwd_streams(
         _ptr(qkv[0]), second(qkv), _ptr(o[0]), second(o), _ptr(lse), _ptr(dO[0]), second(dO), B, N, n0, heads, dh,
         dt, _ptr(dqkv[0]), second(dqkv), _ptr(scratch), impl, _stream(stream)), "jagg_test_attention_bwd_streams")
+
+
+def test_wait_timeout(limit_ns: int, out, stream=None):
+    """A bounded mbarrier wait that nothing satisfies, with the given limit: out [2] u64 device
+    (int64 tensor) receives (gave up, nanoseconds waited)."""
+    _need_cuda(out)
+    _check(lib().jagg_test_wait_timeout(int(limit_ns), _ptr(out), _stream(stream)), "jagg_test_wait_timeout")

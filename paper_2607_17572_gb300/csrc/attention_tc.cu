@@ -31,6 +31,8 @@
 #include "tmap.cuh"
 
 namespace jagg {
+
+int unit_status_attention_tc(unsigned* v, int clear) { return read_unit_status(v, clear); }
 namespace {
 
 constexpr float kLog2eTc = 1.4426950408889634f;
@@ -159,7 +161,8 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
   uint64_t* bar_pfree = bar_p + 1;          // the products reading P^T, dS^T are done
   uint64_t* bar_fin = bar_p + 2;            // a unit's products are done (dK, dV final)
   uint64_t* bar_kvout = bar_p + 3;          // the dQ warps have read the unit's dK, dV
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_p + 4);
+  uint64_t* bar_drain = bar_p + 4;          // the MMA thread's drain after a give-up
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_p + 5);
   __shared__ volatile int abort_flag;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -194,6 +197,7 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
     ptx::mbar_init(bar_pfree, 1);
     ptx::mbar_init(bar_fin, 1);
     ptx::mbar_init(bar_kvout, 4);
+    ptx::mbar_init(bar_drain, 1);
     ptx::fence_mbar_init();
     for (int sg = 0; sg < 2; ++sg) {
       ptx::prefetch_tmap(&maps.q[sg]);
@@ -219,6 +223,7 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA producer
     int i = 0;
+    int i_last = -1, g_last = -1;  // the last unit whose K, V and the last tile whose Q, dO were issued
     for (int u = blockIdx.x; u < units && !abort_flag; u += gridDim.x, ++i) {
       int k0, b, h;
       unit_of(u, k0, b, h);
@@ -237,6 +242,7 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
             ptx::tma_load_3d(sV + kvb * C::KV_BYTES + c * BK * 128, &maps.v[s], &bar_kv[kvb],
                              (int)(p.v_col0 + h * D + c * 64), r, b);
           }
+          i_last = i;
         }
       }
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
@@ -274,7 +280,16 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
                              b);
           }
         }
+        g_last = g;
       }
+    }
+    // After a give-up anywhere in the CTA, copies already issued may still be landing in
+    // shared memory: wait (bounded) for the last phase of every buffer before exiting.
+    if (abort_flag && lane == 0) {
+      for (int k = 0; k < KVB && i_last - k >= 0; ++k)
+        ptx::mbar_wait(&bar_kv[(i_last - k) % KVB], ((i_last - k) / KVB) & 1);
+      for (int k = 0; k < NS && g_last - k >= 0; ++k)
+        ptx::mbar_wait(&full[(g_last - k) % NS], ((g_last - k) / NS) & 1);
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
@@ -369,6 +384,10 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
         ptx::umma_commit(bar_fin);
       }
       if (!ok) abort_flag = 1;
+      if (abort_flag) {  // MMAs of this thread may still run: drain them before TMEM is freed
+        ptx::umma_commit(bar_drain);
+        ptx::mbar_wait(bar_drain, 0);
+      }
     }
   } else if (warp < 10) {
     // ---------------------------------------------------------------- P / dS, then dK, dV
@@ -589,7 +608,8 @@ __global__ void __launch_bounds__(FF_THREADS, 1) fa_fwd_tc_kernel(const __grid_c
   uint64_t* pfree = pready + NP;     // [NP] the product reading P is done
   uint64_t* bar_o = pfree + NP;      // the unit's O is complete
   uint64_t* ofree = bar_o + 1;       // the 8 warps have read O
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(ofree + 1);
+  uint64_t* bar_drain = ofree + 1;   // the MMA thread's drain after a give-up
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_drain + 1);
   __shared__ volatile int abort_flag;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -625,6 +645,7 @@ __global__ void __launch_bounds__(FF_THREADS, 1) fa_fwd_tc_kernel(const __grid_c
     }
     ptx::mbar_init(bar_o, 1);
     ptx::mbar_init(ofree, 8);
+    ptx::mbar_init(bar_drain, 1);
     ptx::fence_mbar_init();
     for (int sg = 0; sg < 2; ++sg) {
       ptx::prefetch_tmap(&maps.q[sg]);
@@ -644,12 +665,13 @@ __global__ void __launch_bounds__(FF_THREADS, 1) fa_fwd_tc_kernel(const __grid_c
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA producer
     if (lane == 0) {
-      int g = 0, i = 0;
+      int g = 0, i = 0, iq_last = -1;  // g: K / V tiles issued; iq_last: the last unit whose Q was issued
       bool ok = true;
       for (int u = blockIdx.x; u < units && ok && !abort_flag; u += gridDim.x, ++i) {
         int q0, b, h;
         unit_of(u, q0, b, h);
         if (i > 0 && !ptx::mbar_wait(qfree, (i - 1) & 1)) { ok = false; break; }
+        iq_last = i;
         ptx::mbar_arrive_expect_tx(qfull, C::Q_BYTES);
 #pragma unroll
         for (int c = 0; c < D / 64; ++c)
@@ -673,6 +695,11 @@ __global__ void __launch_bounds__(FF_THREADS, 1) fa_fwd_tc_kernel(const __grid_c
         }
       }
       if (!ok) abort_flag = 1;
+      // after a give-up: wait (bounded) for the copies still landing before exiting
+      if (abort_flag) {
+        if (iq_last >= 0) ptx::mbar_wait(qfull, iq_last & 1);
+        for (int k = 0; k < NS && g - 1 - k >= 0; ++k) ptx::mbar_wait(&full[(g - 1 - k) % NS], ((g - 1 - k) / NS) & 1);
+      }
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
@@ -737,6 +764,10 @@ __global__ void __launch_bounds__(FF_THREADS, 1) fa_fwd_tc_kernel(const __grid_c
         ptx::umma_commit(bar_o);
       }
       if (!ok) abort_flag = 1;
+      if (abort_flag) {  // MMAs of this thread may still run: drain them before TMEM is freed
+        ptx::umma_commit(bar_drain);
+        ptx::mbar_wait(bar_drain, 0);
+      }
     }
   } else {
     // ---------------------------------------------------------------- softmax, output

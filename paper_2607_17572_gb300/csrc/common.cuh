@@ -32,6 +32,8 @@ static inline int read_unit_status(unsigned* v, int clear) {
 }
 int unit_status_gemm(unsigned* v, int clear);
 int unit_status_signals(unsigned* v, int clear);
+int unit_status_attention_tc(unsigned* v, int clear);
+int unit_status_testing(unsigned* v, int clear);
 
 __device__ __forceinline__ void set_device_status(unsigned bits) { atomicOr(&g_device_status, bits); }
 

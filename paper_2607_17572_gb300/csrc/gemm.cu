@@ -219,6 +219,7 @@ struct TcCfg {
   static constexpr int TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
   static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EPI_BYTES + FIXED;
   static_assert(STAGES >= 4, "pipeline too shallow");
+  static_assert((2 * STAGES + 4 + TC_MAX_EPI_WARPS + 1) * 8 + 4 <= 256, "barrier region");
   static_assert(SMEM_BYTES <= MAX_SMEM, "shared memory budget");
 };
 
@@ -237,7 +238,8 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
   uint64_t* tfull = empty + STAGES;
   uint64_t* tempty = tfull + 2;
   uint64_t* auxbar = tempty + 2;  // one per epilogue warp
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(auxbar + TC_MAX_EPI_WARPS);
+  uint64_t* drainbar = auxbar + TC_MAX_EPI_WARPS;  // the MMA thread's drain after a give-up
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drainbar + 1);
   __shared__ volatile int abort_flag;
 
   const int warp = threadIdx.x >> 5;
@@ -254,6 +256,7 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
       ptx::mbar_init(&tempty[a], EW);
     }
     for (int q = 0; q < EW; ++q) ptx::mbar_init(&auxbar[q], 1);
+    ptx::mbar_init(drainbar, 1);
     ptx::fence_mbar_init();
     ptx::prefetch_tmap(&tmA);
     ptx::prefetch_tmap(&tmB);
@@ -294,6 +297,7 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
       // ---------------- TMA producer
       int stage = 0;
       uint32_t phase = 0;
+      uint32_t issued = 0, issued_parity = 0;  // per stage: a load was issued, and its phase
       for (int t = blockIdx.x; t < total && !abort_flag; t += gridDim.x) {
         int tm, tn, ks, kb0, kb1;
         decode(t, tm, tn, ks);
@@ -317,9 +321,16 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
             for (int c = 0; c < BN / 64; ++c)
               ptx::tma_load_2d(sB + c * (64 * TC_BK * 2), &tmB, &full[stage], tn * BN + c * 64, kb * TC_BK);
           }
+          issued |= 1u << stage;
+          issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
         }
       }
+      // After a give-up anywhere in the CTA, the loads already issued may still be landing
+      // in shared memory: wait (bounded) for the last phase of every stage before exiting.
+      if (abort_flag)
+        for (int s = 0; s < STAGES; ++s)
+          if (issued & (1u << s)) ptx::mbar_wait(&full[s], (issued_parity >> s) & 1u);
     }
   } else if (warp == 1) {
     if (ptx::elect_one()) {
@@ -358,6 +369,12 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
         if (!ok) { abort_flag = 1; break; }
         ptx::umma_commit(&tfull[acc]);
         if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+      }
+      // After a give-up, MMAs of this thread may still be running on TMEM and shared
+      // memory: commit them to the drain barrier and wait (bounded) before the CTA frees TMEM.
+      if (abort_flag) {
+        ptx::umma_commit(drainbar);
+        ptx::mbar_wait(drainbar, 0);
       }
     }
   } else if constexpr (EW == 8) {
@@ -521,8 +538,8 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
         }
       }
       bool ok = ptx::mbar_wait(&tfull[acc], acc_phase);
-      if (aux_load) {
-        ok = ok && ptx::mbar_wait(&auxbar[ew], aux_phase);
+      if (aux_load) {  // waited for even after a give-up: the multiplier load is in flight
+        ok = ptx::mbar_wait(&auxbar[ew], aux_phase) && ok;
         aux_phase ^= 1u;
       }
       ok = __all_sync(0xffffffffu, ok);

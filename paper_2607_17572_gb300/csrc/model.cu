@@ -1116,12 +1116,13 @@ extern "C" const char* jagg_last_error(void) { return jagg::last_error_text(); }
 extern "C" int jagg_device_status(unsigned* status_out, int clear) {
   JAGG_CHECK_ARG(status_out, "jagg_device_status: null output");
   JAGG_CUDA_TRY(cudaDeviceSynchronize());
-  unsigned a = 0, b = 0;
-  if (jagg::unit_status_gemm(&a, clear) || jagg::unit_status_signals(&b, clear)) {
+  unsigned a = 0, b = 0, c = 0, d = 0;
+  if (jagg::unit_status_gemm(&a, clear) || jagg::unit_status_signals(&b, clear) ||
+      jagg::unit_status_attention_tc(&c, clear) || jagg::unit_status_testing(&d, clear)) {
     set_last_error("jagg_device_status: reading the status word failed");
     return JAGG_ERR_CUDA;
   }
-  *status_out = a | b;
+  *status_out = a | b | c | d;
   return JAGG_OK;
 }
 

@@ -610,11 +610,15 @@ constexpr int kMaxDevices = 64;
 std::mutex g_scratch_mu;
 void* g_scratch_ptr[kMaxDevices] = {};
 
-// The array's device address for the current device, looked up once per device.  In host
-// code `g_signals_scratch` names a host-side stand-in, never the device memory itself.
-int scratch_for_current_device(void** out) {
-  int dev = 0;
+// The array's device address for the device of `stream`, which must be the current device
+// (the address comes from a runtime query on the current device), looked up once per device.
+// In host code `g_signals_scratch` names a host-side stand-in, never the device memory itself.
+int scratch_for_stream(cudaStream_t stream, void** out) {
+  int dev = 0, sdev = 0;
   JAGG_CUDA_TRY(cudaGetDevice(&dev));
+  JAGG_CUDA_TRY(cudaStreamGetDevice(stream, &sdev));
+  JAGG_CHECK_ARG(sdev == dev, "grpo_step_signals_static: the stream belongs to device %d, the current device is %d",
+                 sdev, dev);
   JAGG_CHECK_ARG(dev >= 0 && dev < kMaxDevices, "grpo_step_signals_static: device %d out of range", dev);
   std::lock_guard<std::mutex> lk(g_scratch_mu);
   if (!g_scratch_ptr[dev]) {
@@ -641,8 +645,8 @@ extern "C" int grpo_step_signals_static(const void* v_hat, int v_dtype, const fl
     return JAGG_ERR_WORKSPACE;
   }
   void* scratch = nullptr;
-  JAGG_TRY(scratch_for_current_device(&scratch));
-  return grpo_step_signals(v_hat, v_dtype, z, t, sigma, logp_old, rewards, G, W, D, clip_eps, adv_clip, adv_eps,
-                           scale, s_out, cot_out, logp_new, ratio, clipped, adv_out, scratch,
-                           (size_t)JAGG_SIGNALS_STATIC_SCRATCH_BYTES, stream);
+  JAGG_TRY(scratch_for_stream(stream, &scratch));
+  return jagg::step_signals("grpo_step_signals_static", v_hat, v_dtype, z, t, nullptr, nullptr, sigma, logp_old,
+                            rewards, G, W, D, clip_eps, adv_clip, adv_eps, scale, s_out, cot_out, logp_new, ratio,
+                            clipped, adv_out, scratch, (size_t)JAGG_SIGNALS_STATIC_SCRATCH_BYTES, stream);
 }

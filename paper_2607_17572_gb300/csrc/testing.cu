@@ -2,8 +2,38 @@
 #include "../../include/jagg_testing.h"
 #include "attention.cuh"
 #include "gemm.cuh"
+#include "ptx.cuh"
+
+namespace jagg {
+int unit_status_testing(unsigned* v, int clear) { return read_unit_status(v, clear); }
+}  // namespace jagg
 
 using namespace jagg;
+
+namespace {
+// One mbarrier that nothing ever arrives at: the library's bounded wait on it gives up after
+// limit_ns, sets JAGG_DEV_TIMEOUT and returns.  No copy or MMA is in flight.
+__global__ void wait_timeout_kernel(unsigned long long limit_ns, unsigned long long* out) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x == 0) {
+    ptx::mbar_init(&bar, 1);
+    ptx::fence_mbar_init();
+    const unsigned long long t0 = globaltimer_ns();
+    const bool ok = ptx::mbar_wait_for(&bar, 0, limit_ns);
+    out[0] = ok ? 0ull : 1ull;
+    out[1] = globaltimer_ns() - t0;
+  }
+}
+}  // namespace
+
+extern "C" int jagg_test_wait_timeout(unsigned long long limit_ns, unsigned long long* out, cudaStream_t stream) {
+  JAGG_CHECK_ARG(out, "jagg_test_wait_timeout: null output");
+  JAGG_CHECK_ARG(limit_ns > 0 && limit_ns <= kWaitLimitNs, "jagg_test_wait_timeout: limit %llu ns outside (0, %llu]",
+                 limit_ns, kWaitLimitNs);
+  wait_timeout_kernel<<<1, 32, 0, stream>>>(limit_ns, out);
+  JAGG_LAUNCHED();
+  return JAGG_OK;
+}
 
 extern "C" int jagg_test_gemm(const jagg_gemm_desc* d, cudaStream_t stream) {
   JAGG_CHECK_ARG(d, "jagg_test_gemm: null descriptor");

@@ -113,3 +113,22 @@ def test_host_argument_checks_of_the_signal_and_sampler_entry_points(jg):
     # jagg_aggregate_span with equal endpoint times
     assert L.jagg_aggregate_span(fake, 0, fake, 0.5, 0.5, 2, 3, 100, fake, 0, None) < 0
     assert "endpoints" in L.jagg_last_error().decode()
+
+
+def test_static_signals_argument_errors_name_the_static_entry_point(jg):
+    """grpo_step_signals_static reports its argument errors under its own name (checked
+    before any device call)."""
+    L = jg.lib()
+    st = L.grpo_step_signals_static(None, 0, None, None, None, None, None, 0, 4, 64, 0.1, 5.0, 1e-8, 1.0, None, None,
+                                    None, None, None, None, None)
+    assert st == -1
+    assert L.jagg_last_error().decode().startswith("grpo_step_signals_static")
+
+
+def test_wait_timeout_rejects_limits_outside_its_range(jg):
+    """The bounded-wait test entry point takes a limit in (0, 2 s]; others are argument
+    errors returned before any launch."""
+    L = jg.lib()
+    for bad in (0, 2_000_000_001):
+        assert L.jagg_test_wait_timeout(bad, ctypes.c_void_p(16), None) == -1
+        assert "limit" in L.jagg_last_error().decode()

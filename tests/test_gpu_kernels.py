@@ -379,3 +379,22 @@ def test_tcgen05_attention_backward_rejects_unaligned_streams():
         jg.test_attention_bwd_streams((x(n0, 3 * d), x(N - n0, 3 * d)), (x(n0, d), x(N - n0, d)), lse,
                                       (x(n0, d), x(N - n0, d)), B, N, n0, H, dh,
                                       (x(n0, 3 * d), x(N - n0, 3 * d)), impl=2)
+
+
+# ------------------------------------------------------------------ bounded waits
+@pytest.mark.parametrize("limit_ns", [1_000_000, 20_000_000])
+def test_bounded_wait_gives_up_and_reports_timeout(limit_ns):
+    """A wait on an mbarrier that nothing arrives at ends after its limit: the kernel returns,
+    the device status word reads JAGG_DEV_STATUS_TIMEOUT (then clears), and the context
+    stays usable for the next call."""
+    assert jg.device_status() == 0
+    out = torch.zeros(2, dtype=torch.int64, device="cuda")
+    jg.test_wait_timeout(limit_ns, out)
+    torch.cuda.synchronize()
+    gave_up, waited = out.tolist()
+    assert gave_up == 1
+    assert limit_ns <= waited < limit_ns + 50_000_000
+    assert jg.device_status() == 1          # JAGG_DEV_STATUS_TIMEOUT, cleared by the read
+    assert jg.device_status() == 0
+    x = torch.randn(256, 256, device="cuda")
+    assert torch.isfinite(x @ x).all()      # the context still works

@@ -87,3 +87,32 @@ def test_static_scratch_rejects_requests_beyond_its_size():
                                                v.data_ptr(), v.data_ptr(), v.data_ptr(), v.data_ptr(),
                                                torch.cuda.current_stream().cuda_stream)
         jg._check(st, "grpo_step_signals_static")
+
+
+def test_static_scratch_entry_point_allocates_nothing():
+    """What the entry point is for: after a first call on the device (which looks up the
+    array's address), further calls change neither PyTorch's allocated bytes nor the
+    device's free memory (cudaMemGetInfo)."""
+    G, W, D = 4, 4, 8192
+    v, z, t, sig, rewards = _window(G, W, D, seed=3)
+    out, s, cot = _outputs(G, W, D)
+    logp_old = torch.zeros(G, W, dtype=torch.float64, device="cuda")
+    args = (v, z, t, sig, logp_old, rewards, 0.1, 5.0, 1e-8, 1.0 / (G * 16))
+    jg.grpo_step_signals_static(*args, s_out=s, cot_out=cot, **out)
+    torch.cuda.synchronize()
+    alloc0, free0 = torch.cuda.memory_allocated(), torch.cuda.mem_get_info()[0]
+    for _ in range(2):
+        jg.grpo_step_signals_static(*args, s_out=s, cot_out=cot, **out)
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    assert torch.cuda.memory_allocated() == alloc0
+    assert torch.cuda.mem_get_info()[0] == free0
+
+
+def test_static_scratch_errors_name_the_static_entry_point():
+    v = torch.zeros(16, device="cuda")
+    p = v.data_ptr()
+    st = jg.lib().grpo_step_signals_static(p, 0, p, p, p, p, p, 2, 2, 64, 0.1, 5.0, 1e-8, 1.0, None, None,
+                                           None, p, p, p, torch.cuda.current_stream().cuda_stream)   # null logp_new
+    assert st == -1
+    assert jg.lib().jagg_last_error().decode().startswith("grpo_step_signals_static")
