@@ -1,22 +1,27 @@
 #!/usr/bin/env python3
 """Throughput of the JAGG backward path on GB300.
 
-One step = the whole update-stage backward of one GRPO group on the DiT-B workload
-(12 single-stream blocks, d = 768, 256 image + 77 text tokens; G = 8 samples, T = 16
-sampling steps, windows of W = 4, jagg_frac = 1): for every window, the step signals with
-the fused t-weighted aggregation (Phases 2-3); then one joint VJP over the 2G endpoint rows
-of every window of the group at once, accumulating the fp32 parameter gradient (Phase 4;
-the window gradients add, so this equals one joint VJP per window); then the gradient's
-squared norm.  The forward passes of Phase 1 (endpoints saved, middle steps without
-saves) run before the timed region: their saved activations are inputs resident in HBM.
-The metric is trajectory-steps of gradient per second: G * T (sample, step) pairs per step.
+One step = the whole update-stage backward of one GRPO group.  Default workload: the
+Flux-width MMDiT at 1024^2 (4 double-stream + 8 single-stream blocks, d = 3072, 24 heads
+of 128, MLP 12288; 4096 image + 512 text tokens; G = 4 samples, T = 16 sampling steps,
+windows of W = 4, jagg_frac = 1).  Per window: the step signals with the fused t-weighted
+aggregation (Phases 2-3), then the joint VJP over the window's 2G endpoint rows,
+accumulating the fp32 parameter gradient (Phase 4, Algorithm 1); after the last window the
+gradient's squared norm.  When the whole group's saved activations fit in HBM at once the
+step is one timed region; smaller models batch every window's endpoint rows into one
+joint VJP (the window gradients add).  The forward passes of Phase 1 (endpoints saved,
+middle steps without saves) run before the timed region: their saved activations are
+inputs resident in HBM.  The metric is trajectory-steps of gradient per second: G * T
+(sample, step) pairs per step.
 
-Also timed: the same step with one joint VJP per window (Algorithm 1 as written), the
-exact per-step path (jagg_frac = 0: the VJP over all W*G step inputs of every window with
-their own s_j), the sequential-graph variant and the endpoint-only ablation, the update
-stage (forwards on the stored experience + backward, JAGG against the exact path), the
-rollout sampler, and `e2e`, the update stage through the public API from pinned host
-buffers (Phase 1 forwards included).  `--impl reference` times the float64 CPU oracle.
+Also timed: the exact per-step path (jagg_frac = 0: the VJP over all W*G step inputs of
+every window with their own s_j), the sequential-graph variant and the endpoint-only
+ablation, the update stage (forwards on the stored experience + backward, JAGG against
+the exact path), the rollout sampler, and `e2e`, the update stage through the public API
+from pinned host buffers (Phase 1 forwards included).  `--sweep` times the routing and
+window sweep (W in {2, 4, 8} x jagg_frac in {0, 0.5, 1}) on the Qwen-width MMDiT with the
+per-window gradient cosines behind each routing decision.  `--impl reference` times the
+float64 CPU oracle.
 """
 from __future__ import annotations
 
@@ -47,7 +52,10 @@ def parse():
     p.add_argument("--steps", type=int, default=10)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["jagg", "reference"], default="jagg")
-    p.add_argument("--workload", default="dit_b_bf16")
+    p.add_argument("--workload", default=None,
+                   help="default mmdit_flux1024_bf16 (mmdit_qwen_sweep_bf16 with --sweep)")
+    p.add_argument("--sweep", action="store_true",
+                   help="the routing and window sweep: W in {2, 4, 8} x jagg_frac in {0, 0.5, 1}")
     p.add_argument("--no-graph", action="store_true", help="launch eagerly instead of replaying a CUDA graph")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
@@ -57,8 +65,9 @@ def parse():
     p.add_argument("--kernel", choices=["attention_bwd", "attention_fwd", "gemm"], default=None,
                    help="time one kernel family alone on the workload's shapes instead of the step")
     p.add_argument("--product", default="all",
-                   help="for --kernel gemm: one of the block's backward products (fc2_dx, fc1_dx, qkv_dx, "
-                        "proj_dx, fc2_dw, fc1_dw, qkv_dw, proj_dw) or all")
+                   help="for --kernel gemm: one of the block's backward products (gemm_products: DiT fc2_dx, "
+                        "fc1_dx, qkv_dx, proj_dx, fc2_dw, fc1_dw, qkv_dw, proj_dw; MMDiT lin2_dx_o, lin2_dx_u, "
+                        "lin1_dx, lin2_dw, lin1_dw and the img_ products of a double block) or all")
     p.add_argument("--rows", type=int, default=0, help="sequences per call for --kernel (default 2G)")
     p.add_argument("--vjp-rows", choices=["auto", "group", "window"], default="auto",
                    help="one joint VJP per group (all windows' rows) or per window; auto picks the group "
@@ -67,7 +76,8 @@ def parse():
 
 
 def workload(args):
-    wl = synth.WORKLOADS[args.workload]
+    name = args.workload or ("mmdit_qwen_sweep_bf16" if getattr(args, "sweep", False) else "mmdit_flux1024_bf16")
+    wl = synth.WORKLOADS[name]
     if args.G:
         wl = synth.small_variant(wl, name=f"{wl.name}_G{args.G}", G=args.G)
     return wl
@@ -82,10 +92,11 @@ def describe(wl) -> str:
             f"tokens, G={wl.G}, T={wl.T}, W={wl.W}, jagg_frac={wl.jagg_frac}")
 
 
-# DRAM bytes (read + write) per launch of the dense-product kernel in the timed step, from
-# one ncu capture of the step's launch list (profiles/ditb_jagg_step_launches.md: kernel
-# revision 91655fa); None for workloads without such a capture.
-TRAFFIC_PER_LAUNCH = {"dit_b_bf16": 134.7e6}
+# DRAM bytes (read + write) per launch of the dense-product kernel over its algorithmic
+# bytes, from one ncu capture of the kernel alone (`--kernel gemm`) on the workload's
+# backward products at the step's rows; the roofline's `traffic` is this ratio times the
+# step's algorithmic bytes per launch.  Absent: no capture of the current kernel.
+TRAFFIC_RATIO = {}
 
 
 def peaks():
@@ -234,7 +245,8 @@ class Bench:
         self.txt1 = torch.tensor(self.draws.txt, dtype=self.tdt, device=dev)
         # workspace for the largest single call: one window's W*G rows, or the batched calls
         # over every window (2G endpoint rows each, or W*G step rows each) when their saved
-        # activations can be resident (the test `fits` applies, against free memory)
+        # activations take at most half of the device (the test `fits` applies, against
+        # free memory)
         total = torch.cuda.get_device_properties(dev).total_memory
         cands = [W * G] + [r for r in (2 * G * self.nw, W * G * self.nw) if self.model.saved_bytes(r) < 0.5 * total]
         self.ws_rows = max(cands)
@@ -328,14 +340,18 @@ class Bench:
         """True: one saved arena (and one joint VJP) for every window of the group."""
         if mode != "auto":
             return mode == "group"
-        return self.fits(routes)
+        return self.fits(routes, batched=True)
 
-    def fits(self, routes) -> bool:
-        """Every window's saved activations fit in half of the free device memory (and the
-        workspace covers that many rows)."""
-        _, rows = self.plan(routes)
+    def fits(self, routes, batched) -> bool:
+        """Every window's saved activations can be resident at once.  batched (one arena,
+        one joint VJP over the group): the workspace covers the group's rows and the arena
+        takes at most half of the free memory; otherwise (one arena per window) the arenas
+        together take at most 85 % of it."""
+        plan, rows = self.plan(routes)
         free, _ = torch.cuda.mem_get_info(self.dev)
-        return rows <= self.ws_rows and self.model.saved_bytes(rows) < 0.5 * free
+        if batched:
+            return rows <= self.ws_rows and self.model.saved_bytes(rows) < 0.5 * free
+        return sum(self.model.saved_bytes(n) for (_, _, _, n) in plan) < 0.85 * free
 
     def forward_saves(self, routes, batched, windows=None):
         """Phase 1 with saves for the rows of the plan (or of the listed windows only).
@@ -414,31 +430,61 @@ def time_steps(fn, steps, warmup, ws, use_graph):
 
 
 # ----------------------------------------------------------------------------- oracle legs
-def oracle_window_sample(wl, G_sample):
-    """One JAGG window of the workload on the float64 oracle for G_sample samples:
-    the endpoint forwards with their caches, the step signals of the window (on synthetic
-    v-hat), the t-weighted aggregation and the joint VJP.  Returns (seconds, traj-steps)."""
+def oracle_sample_plan(wl):
+    """What the float64 oracle runs as a bounded sample of the workload, and what it stands
+    for.  DiT widths: one JAGG window of 2 samples through the whole model (4 endpoint
+    rows).  MMDiT widths, where the whole model takes the oracle minutes per sequence: one
+    endpoint row through one block at the workload's full width and token count (a Flux-style
+    single block when the model has them, else one double-stream block) with the model's
+    embeddings and final layer, its time scaled to one sample's JAGG window (2 endpoint rows
+    through the whole model) by the algorithmic FLOPs of flops_per_sequence.
+    Returns (sample workload, rows, samples the run stands for, scale)."""
+    if wl.arch == "dit":
+        return wl, 4, 2, 1.0
+    sub = synth.small_variant(wl, depth=min(wl.depth, 1), depth_double=0 if wl.depth else 1)
+    full = sum(flops_per_sequence(wl)) * 2
+    part = sum(flops_per_sequence(sub))
+    return sub, 1, 1, full / part
+
+
+def oracle_sample(wl):
+    """One bounded sample of the workload on the float64 oracle (oracle_sample_plan): the step
+    signals of one window on synthetic v-hat, the t-weighted aggregation, the forward of the
+    sample's rows with caches and the VJP.  Returns (seconds measured, trajectory-steps the
+    sample stands for, seconds scaled to them, description)."""
     from oracle import dit, grpo
-    params = synth.make_params(wl)
-    model = dit.Backbone(wl, params)
+    sub, rows, n_samples, scale = oracle_sample_plan(wl)
+    params = synth.make_params(sub)
+    model = dit.Backbone(sub, params)
     rng = np.random.Generator(np.random.PCG64(5))
     W = wl.W
     shape = (wl.in_channels, wl.latent_h, wl.latent_w)
     t = synth.time_grid(wl.T, wl.shift)[:W + 1]
     sig = synth.sigma_schedule(t, wl.eta)
-    z = synth.storage_round(rng.standard_normal((G_sample, W + 1) + shape), wl.dtype)
-    v = synth.storage_round(rng.standard_normal((G_sample, W) + shape), wl.dtype)
-    lpo = np.zeros((G_sample, W))
-    txt = np.broadcast_to(synth.draw_group(wl).txt, (2 * G_sample, wl.txt_len, wl.txt_dim))
+    z = synth.storage_round(rng.standard_normal((n_samples, W + 1) + shape), wl.dtype)
+    v = synth.storage_round(rng.standard_normal((n_samples, W) + shape), wl.dtype)
+    lpo = np.zeros((n_samples, W))
+    txt = np.broadcast_to(synth.draw_group(wl).txt, (rows, wl.txt_len, wl.txt_dim))
     t0 = time.perf_counter()
-    s, _, _, _ = grpo.step_signals(v.reshape(G_sample, W, -1), z.reshape(G_sample, W + 1, -1), t, sig, lpo,
-                                   grpo.advantages(rng.standard_normal(G_sample)), wl.clip_eps, 1.0 / (wl.G * wl.T))
-    cot = grpo.aggregate(s, t[:W]).reshape((2 * G_sample,) + shape)
-    zr = np.concatenate([z[:, 0], z[:, W - 1]])
-    tr = np.concatenate([np.full(G_sample, t[0]), np.full(G_sample, t[W - 1])])
+    s, _, _, _ = grpo.step_signals(v.reshape(n_samples, W, -1), z.reshape(n_samples, W + 1, -1), t, sig, lpo,
+                                   grpo.advantages(rng.standard_normal(n_samples)), wl.clip_eps,
+                                   1.0 / (wl.G * wl.T))
+    cot = grpo.aggregate(s, t[:W]).reshape((2 * n_samples,) + shape)[:rows]
+    zr = np.concatenate([z[:, 0], z[:, W - 1]])[:rows]
+    tr = np.concatenate([np.full(n_samples, t[0]), np.full(n_samples, t[W - 1])])[:rows]
     _, cache = model.forward(zr, tr, txt)
     model.vjp(cache, cot)
-    return time.perf_counter() - t0, G_sample * W
+    sec = time.perf_counter() - t0
+    if scale == 1.0:
+        desc = (f"one JAGG window (W={W}) of {wl.name} for {n_samples} of the G={wl.G} samples: step signals, "
+                f"aggregation, endpoint forwards with caches and the joint VJP over {rows} rows")
+    else:
+        kind = "Flux-style single block" if sub.depth else "double-stream block"
+        desc = (f"{rows} endpoint row of {wl.name} through one {kind} at full width and {wl.n_tok} tokens "
+                f"(+ embeddings, final layer, one window's step signals and aggregation): forward with caches "
+                f"and VJP, {sec:.1f} s measured, scaled by algorithmic FLOPs x{scale:.1f} to one sample's JAGG "
+                f"window (2 endpoint rows through all {wl.depth_double} double + {wl.depth} single blocks)")
+    return sec, n_samples * W, sec * scale, desc
 
 
 def threads_used():
@@ -453,26 +499,27 @@ def threads_used():
 
 
 def run_reference(args, ws, rank):
+    """The reference arm: the float64 oracle on the host cores, each step one bounded sample
+    of the workload (oracle_sample), rank 0 only."""
     if rank != 0:
         return
     wl = workload(args)
-    G_sample = 2
     for _ in range(args.warmup):
-        oracle_window_sample(wl, G_sample)
-    tot, units = 0.0, 0
+        oracle_sample(wl)
+    tot, units, measured = 0.0, 0, 0.0
     for _ in range(args.steps):
-        sec, u = oracle_window_sample(wl, G_sample)
-        tot += sec
+        sec, u, scaled, desc = oracle_sample(wl)
+        measured += sec
+        tot += scaled
         units += u
     value = units / tot
-    sample = (f"one JAGG window (W={wl.W}) of {wl.name} for {G_sample} of the G={wl.G} samples per step: "
-              f"endpoint forwards with caches, step signals, aggregation, joint VJP over {2 * G_sample} rows")
     cores = threads_used()
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * tot / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": wl.name},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+            "config": {"workload": describe(wl)},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc,
+                             "measured_s_per_step": measured / args.steps},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -511,7 +558,7 @@ def measure(b, routes, batched, args, ws, use_graph, profile=False):
                     acc[q] += v[q] / args.steps
             jg.profile_enable(False)
 
-    if batched or b.fits(routes):
+    if batched or b.fits(routes, batched=False):
         run_part(b.forward_saves(routes, batched=batched), True)
     else:
         res["resident"] = False
@@ -569,30 +616,69 @@ def graph_variants(b, args, ws, use_graph):
             "scope": "per window: endpoint forwards with saves + VJPs on the JAGG cotangents (signals excluded)"}
 
 
-def ablate_step(b, args, ws, use_graph):
+def ablate_step(b, args, ws, use_graph, batched, steps, warmup):
     """The endpoint-only ablation (Sec. 4): per window the step signals, then s_0 and s_{W-1}
-    read in place as the two cotangent rows (no t-weighting), then the joint VJP over every
-    window's endpoint rows -- the headline step with the aggregation swapped."""
+    read in place as the two cotangent rows (no t-weighting), then the joint VJP(s) over the
+    endpoint rows, batched like the headline -- the headline step with the aggregation
+    swapped.  None when the endpoint arenas do not fit at once."""
     jg, wl, dev = b.jg, b.wl, b.dev
     G, W, D = wl.G, wl.W, b.D
-    arenas = b.forward_saves([1] * b.nw, batched=True)
+    routes = [1] * b.nw
+    if not (batched or b.fits(routes, batched=False)):
+        return None
+    arenas = b.forward_saves(routes, batched=batched)
     s_win = torch.empty(G, W, D, dtype=torch.float32, device=dev)
 
     def step():
-        for w in range(b.nw):
-            b.signals(w, b.lpo_win[w], s_out=s_win)
-            tw = b.t_dev[w * W:(w + 1) * W]
-            cot = b.cot_all[w * 2 * G:(w + 1) * 2 * G]
-            t0, t1 = float(b.t[w * W]), float(b.t[w * W + W - 1])
-            jg.jagg_aggregate_span(s_win, tw[:1], t0, t1, cot, steps=(0, 1))
-            jg.jagg_aggregate_span(s_win, tw[W - 1:], t0, t1, cot, accumulate=True, steps=(W - 1, 1))
-        saved, B, _ = arenas[0]
-        jg.dit_joint_vjp(b.model, saved, B, b.cot_all[:B], b.grad, b.ws)
+        for saved, B, pl in arenas:
+            row0 = pl[0][2]
+            for (w, _, r, _) in pl:
+                b.signals(w, b.lpo_win[w], s_out=s_win)
+                tw = b.t_dev[w * W:(w + 1) * W]
+                cot = b.cot_all[r:r + 2 * G]
+                t0, t1 = float(b.t[w * W]), float(b.t[w * W + W - 1])
+                jg.jagg_aggregate_span(s_win, tw[:1], t0, t1, cot, steps=(0, 1))
+                jg.jagg_aggregate_span(s_win, tw[W - 1:], t0, t1, cot, accumulate=True, steps=(W - 1, 1))
+            jg.dit_joint_vjp(b.model, saved, B, b.cot_all[row0:row0 + B], b.grad, b.ws)
         jg.grad_reduce(b.grad, None, out3=b.out3, ws=b.gws)
-    ms, graph = time_steps(step, args.steps, args.warmup, ws, use_graph)
+    ms, graph = time_steps(step, steps, warmup, ws, use_graph)
     del graph, arenas
     torch.cuda.empty_cache()
-    return {"value": ws * wl.G * wl.T / (ms / 1000.0), "unit": UNIT, "ms_per_step": max_over_ranks(ms, ws)}
+    return {"value": ws * wl.G * wl.T / (ms / 1000.0), "unit": UNIT, "ms_per_step": max_over_ranks(ms, ws),
+            "steps": steps, "warmup": warmup}
+
+
+def flops_per_sequence(wl):
+    """Algorithmic FLOPs (2 per multiply-add) of one sequence through the backbone:
+    (forward, backward).  Per block the four dense products of every token (4 d^2 + 2 d dm
+    multiply-adds: qkv, proj, fc1, fc2 -- or lin1, lin2 of a single block), attention
+    4 N^2 d, the modulation product; embeddings and final layer.  Backward: the input and
+    weight gradients of every product (2x, weight gradient only for the input embeddings,
+    which pass no gradient to z or the text), 8 N^2 d for attention (recomputing S is not
+    counted)."""
+    d, dm, N = wl.hidden, wl.mlp, wl.n_tok
+    blocks = wl.depth + wl.depth_double
+    lin = 2.0 * N * (4 * d * d + 2 * d * dm)
+    att = 4.0 * N * N * d
+    mod_rows = (6 * d * wl.depth if wl.arch == "dit" else 12 * d * wl.depth_double + 3 * d * wl.depth) + 2 * d
+    mod = 2.0 * d * mod_rows + 2.0 * (wl.freq_dim * d + d * d)
+    emb_in = 2.0 * d * (wl.n_img * wl.patch_dim + wl.txt_len * wl.txt_dim)
+    emb_out = 2.0 * d * wl.n_img * wl.patch_dim
+    fwd = blocks * (lin + att) + mod + emb_in + emb_out
+    bwd = blocks * (2 * lin + 2 * att) + 2 * mod + emb_in + 2 * emb_out
+    return fwd, bwd
+
+
+def family_roofline(fam, name, peak, src, label):
+    """Roofline object of one kernel family over the step's launches: algorithmic FLOPs
+    per launch over its average launch duration (events around each launch)."""
+    f = fam.get(name, {"launches": 0, "ms": 0.0, "flops": 0.0, "bytes": 0.0})
+    n = max(f["launches"], 1)
+    achieved = f["flops"] / (f["ms"] / 1000.0) / 1e12 if f["ms"] > 0 else 0.0
+    return {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+            "kernel": label, "peak_source": src, "launches_per_step": f["launches"],
+            "flops_per_launch": f["flops"] / n, "algorithmic_bytes_per_launch": f.get("bytes", 0.0) / n,
+            "ms_per_launch": f["ms"] / n}
 
 
 def run_gpu(args, ws, rank):
@@ -605,6 +691,10 @@ def run_gpu(args, ws, rank):
     batched = b.batch_group(routes, args.vjp_rows)
     use_graph = not args.no_graph
     units = wl.G * wl.T
+    # the legs beside the headline: at most 5 timed steps on the MMDiT widths (seconds each)
+    leg_steps = args.steps if wl.arch == "dit" else min(args.steps, 5)
+    leg_warm = max(3, args.warmup) if wl.arch == "dit" else 3
+    lg = argparse.Namespace(steps=leg_steps, warmup=leg_warm)
 
     # ---- JAGG path: timed region, then the per-family breakdown of the same work
     with ClockSampler(torch.cuda.current_device()) as clk:
@@ -614,16 +704,15 @@ def run_gpu(args, ws, rank):
     value = job_rate(units, ms, ws)
     burst, sustained, hbm, src = peaks()
     fam = {k: v for k, v in r["prof"].items() if v["launches"]}
-    gt = fam.get("gemm_tcgen05", {"launches": 0, "ms": 0.0, "flops": 0.0})
-    achieved = gt["flops"] / (gt["ms"] / 1000.0) / 1e12 if gt["ms"] > 0 else 0.0
-    roofline = {"bound": "tensor", "achieved": achieved, "peak": sustained, "unit": "TFLOP/s",
-                "frac": achieved / sustained, "traffic": TRAFFIC_PER_LAUNCH.get(wl.name),
-                "algorithmic_bytes_per_launch": gt.get("bytes", 0.0) / max(gt["launches"], 1),
-                "kernel": "gemm_tcgen05 (all dense products of the joint VJP)",
-                "peak_source": f"bf16_tflops_sustained of {src} peaks",
-                "launches_per_step": gt["launches"],
-                "flops_per_launch": gt["flops"] / max(gt["launches"], 1),
-                "ms_per_launch": gt["ms"] / max(gt["launches"], 1)}
+    # the products and attention run back to back for the seconds of a step: sustained peak
+    psrc = f"bf16_tflops_sustained of {src} peaks"
+    roofline = family_roofline(fam, "gemm_tcgen05", sustained, psrc,
+                               "gemm_tc_kernel (all dense products of the joint VJP)")
+    ratio = TRAFFIC_RATIO.get(wl.name)
+    roofline["traffic"] = ratio * roofline["algorithmic_bytes_per_launch"] if ratio else None
+    roofline["frac_of_burst"] = roofline["achieved"] / burst
+    att = family_roofline(fam, "attention_bwd", sustained, psrc, "fa_bwd_tc_kernel (attention backward)")
+    att["frac_of_burst"] = att["achieved"] / burst
     step_flops = sum(v["flops"] for k, v in fam.items() if k != "gemm_simt")
     families = {k: {"launches_per_step": v["launches"], "ms_per_step": v["ms"],
                     "tflops": (v["flops"] / (v["ms"] / 1000.0) / 1e12) if v["ms"] > 0 else None}
@@ -632,7 +721,8 @@ def run_gpu(args, ws, rank):
         batching = f"one joint VJP per group over all {b.nw} windows' endpoint rows"
     else:
         batching = f"one joint VJP per window ({b.nw} per step)" + (
-            "" if r["resident"] else ", each window timed with its own saved activations resident")
+            ", every window's saved activations resident" if r["resident"] else
+            ", each window timed with its own saved activations resident, the window times added")
     out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
@@ -640,7 +730,8 @@ def run_gpu(args, ws, rank):
                       "cuda_graph": use_graph, "vjp_batching": batching,
                       "l2": "inputs larger than L2 (saved activations %.1f GB resident)" % r["saved_gb"],
                       "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU"},
-           "roofline": roofline, "algorithmic_tflops_per_step": step_flops / 1e12,
+           "roofline": roofline, "roofline_attention_bwd": att,
+           "algorithmic_tflops_per_step": step_flops / 1e12,
            "step_tflops_per_s": step_flops / (ms / 1000.0) / 1e12, "families": families,
            "gpu_launches": r["launches"] * args.steps, "clocks": clocks}
     torch.cuda.empty_cache()
@@ -648,94 +739,135 @@ def run_gpu(args, ws, rank):
     if not args.quick:
         # ---- the same JAGG step with one joint VJP per window (Algorithm 1 as written)
         if batched:
-            rw = measure(b, routes, False, args, ws, use_graph)
+            rw = measure(b, routes, False, lg, ws, use_graph)
             out["per_window_vjp"] = {"value": ws * units / (rw["ms"] / 1000.0), "unit": UNIT,
                                      "ms_per_step": rw["ms"], "rows_per_vjp": rw["rows"], "vjps_per_step": rw["vjps"]}
         # ---- exact per-step path (jagg_frac = 0), batched like the headline when it fits
         full = [0] * b.nw
-        b.grad.zero_()
-        rf = measure(b, full, b.batch_group(full, args.vjp_rows), args, ws, use_graph)
+        rf = measure(b, full, b.batch_group(full, args.vjp_rows), lg, ws, use_graph)
         out["full_w"] = {"value": ws * units / (rf["ms"] / 1000.0), "unit": UNIT, "ms_per_step": rf["ms"],
-                         "rows_per_vjp": rf["rows"], "vjps_per_step": rf["vjps"]}
+                         "rows_per_vjp": rf["rows"], "vjps_per_step": rf["vjps"], "steps": lg.steps,
+                         "resident": ("every window" if rf["resident"] else
+                                      "one window at a time, the window times added")}
         out["jagg_speedup_vs_full_w"] = rf["ms"] / ms
         out["ideal_speedup"] = wl.W / 2
         torch.cuda.empty_cache()
-        if batched:
-            out["graph_variants"] = graph_variants(b, args, ws, use_graph)
-            out["ablate"] = ablate_step(b, args, ws, use_graph)
-            out["update_stage"] = update_stage(b, args, ws, use_graph)
-        out["rollout"] = rollout_leg(b, args, ws, use_graph)
-        if not args.no_e2e and batched:
-            out["e2e"] = run_e2e(b, args, ws, routes)
-        # the float64 oracle needs minutes per sequence at MMDiT width: DiT workloads only
-        if rank == 0 and ws == 1 and not args.no_cpu_baseline and wl.arch == "dit":
-            G_sample = 2
-            sec, u = oracle_window_sample(wl, G_sample)
-            out["cpu_baseline"] = {"value": u / sec, "unit": UNIT, "cores": threads_used(), "kind": "oracle",
-                                   "sample": (f"one JAGG window (W={wl.W}) of {wl.name} for {G_sample} samples: "
-                                              f"endpoint forwards with caches, step signals, aggregation, joint "
-                                              f"VJP over {2 * G_sample} rows; {sec:.1f} s")}
+        out["graph_variants"] = graph_variants(b, lg, ws, use_graph)
+        ab = ablate_step(b, args, ws, use_graph, batched, lg.steps, lg.warmup)
+        if ab is not None:
+            out["ablate"] = ab
+        out["update_stage"] = update_stage(b, args, ws, use_graph, lg.steps, lg.warmup)
+        out["rollout"] = rollout_leg(b, lg, ws, use_graph)
+    if not args.no_e2e:
+        out["e2e"] = run_e2e(b, args, ws, routes, steps=lg.steps, warmup=lg.warmup)
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        sec, u, scaled, desc = oracle_sample(wl)
+        out["cpu_baseline"] = {"value": u / scaled, "unit": UNIT, "cores": threads_used(), "kind": "oracle",
+                               "sample": desc, "measured_s": sec}
     if rank == 0:
         print(json.dumps(out), flush=True)
 
 
-def jagg_update(b, host):
-    """The JAGG update stage of one group (the paper's "update": forwards on the stored
-    experience, then the backward): every window's Phase 1 forwards (endpoints saved, middle
-    steps without saves), Phases 2-3 per window, one joint VJP over every window's endpoint
-    rows, the gradient norm.  host=True: the step starts by copying the group's trajectory,
-    old log-probs and rewards from pinned host buffers and ends by reading the new log-probs
+def update_chunks(b, routes):
+    """Windows per Phase-4 call of the update stage: every window at once when the group's
+    saved activations fit (one arena, one joint VJP over the group), else one window at a
+    time through one arena (Algorithm 1's loop over windows)."""
+    G, W = b.wl.G, b.wl.W
+    mid = sum((W - 2) * G for w in range(b.nw) if routes[w])
+    if b.fits(routes, batched=True) and mid <= b.ws_rows:
+        return [list(range(b.nw))]
+    return [[w] for w in range(b.nw)]
+
+
+def update_step(b, routes, host):
+    """The update stage of one group (the paper's "update": forwards on the stored
+    experience, then the backward).  Per window routed to JAGG: the endpoint forwards with
+    saves, the middle steps' forwards without, the step signals with the aggregation, the
+    joint VJP over the 2G endpoint rows; per exact window: every step's forward with saves,
+    each step's own signal, the VJP over its W*G rows.  Windows share one VJP call when the
+    group's saved activations fit (update_chunks).  After the last window, the gradient's
+    squared norm.  host=True: the step starts by copying the group's trajectory, old
+    log-probs and rewards from pinned host buffers and ends by reading the new log-probs
     and the gradient norm back.  Returns (step, h2d bytes, d2h bytes)."""
     jg, wl, dev = b.jg, b.wl, b.dev
-    G, W = wl.G, wl.W
+    G, W, D = wl.G, wl.W, b.D
     h_z = b.z.cpu().pin_memory()
     h_lpo = b.logp_old.cpu().pin_memory()
     h_rw = b.rewards.cpu().pin_memory()
     h_lpn = torch.empty(G, wl.T, dtype=torch.float64).pin_memory()
     h_out3 = torch.empty(3, dtype=torch.float64).pin_memory()
-    nw = b.nw
-    B = nw * 2 * G                       # every window's two endpoints, saved
-    Bm = nw * (W - 2) * G                # every window's middle steps, not saved
-    saved = jg.alloc_bytes(b.model.saved_bytes(B), dev)
-    v_end = torch.empty(B, *b.shape, dtype=b.tdt, device=dev)
-    v_mid = torch.empty(max(Bm, 1), *b.shape, dtype=b.tdt, device=dev)
-    txt_mid, txt_end = b.txt_rows(max(Bm, 1)), b.txt_rows(B)
-    t_end = torch.tensor(np.concatenate([np.repeat([b.t[w * W], b.t[w * W + W - 1]], G) for w in range(nw)]),
-                         dtype=torch.float32, device=dev)
-    t_mid = torch.tensor(np.concatenate([np.tile(b.t[w * W + 1:w * W + W - 1], G) for w in range(nw)]),
-                         dtype=torch.float32, device=dev)
-    z_end = torch.empty(B, *b.shape, dtype=b.tdt, device=dev)
-    z_mid = torch.empty(max(Bm, 1), *b.shape, dtype=b.tdt, device=dev)
+    chunks = update_chunks(b, routes)
+
+    def rows_of(c):
+        sv = sum(2 * G if routes[w] else W * G for w in c)
+        mid = sum((W - 2) * G for w in c if routes[w])
+        return sv, mid
+    n_sv = max(rows_of(c)[0] for c in chunks)
+    n_mid = max(max(rows_of(c)[1] for c in chunks), 1)
+    saved = jg.alloc_bytes(b.model.saved_bytes(n_sv), dev)
+    z_sv = torch.empty(n_sv, *b.shape, dtype=b.tdt, device=dev)
+    v_sv = torch.empty_like(z_sv)
+    z_mid = torch.empty(n_mid, *b.shape, dtype=b.tdt, device=dev)
+    v_mid = torch.empty_like(z_mid)
+    txt_sv, txt_mid = b.txt_rows(n_sv), b.txt_rows(n_mid)
+    t_sv, t_mid = [], []
+    for c in chunks:
+        ts, tm = [], []
+        for w in c:
+            tw = b.t[w * W:(w + 1) * W]
+            if routes[w]:
+                ts.append(np.repeat([tw[0], tw[W - 1]], G))
+                tm.append(np.tile(tw[1:W - 1], G))
+            else:
+                ts.append(np.tile(tw, G))       # sample-major, matching s [G, W, D]
+        t_sv.append(torch.tensor(np.concatenate(ts), dtype=torch.float32, device=dev))
+        t_mid.append(torch.tensor(np.concatenate(tm), dtype=torch.float32, device=dev) if tm else None)
 
     def step():
         if host:
             b.z.copy_(h_z, non_blocking=True)
             b.logp_old.copy_(h_lpo, non_blocking=True)
             b.rewards.copy_(h_rw, non_blocking=True)
-        for w in range(nw):
-            zw = b.z[:, w * W:(w + 1) * W].reshape(G, W, *b.shape)
-            z_end[w * 2 * G:w * 2 * G + G].copy_(zw[:, 0])
-            z_end[w * 2 * G + G:(w + 1) * 2 * G].copy_(zw[:, W - 1])
-            if W > 2:
-                z_mid[w * (W - 2) * G:(w + 1) * (W - 2) * G].copy_(zw[:, 1:W - 1].reshape(-1, *b.shape))
-        # Phase 1: endpoints of every window with saves, middle steps without
-        jg.dit_forward_save(b.model, z_end, t_end, txt_end, v_end, saved=saved, ws=b.ws)
-        if W > 2:
-            jg.dit_forward_save(b.model, z_mid[:Bm], t_mid, txt_mid[:Bm], v_mid[:Bm], ws=b.ws)
-        for w in range(nw):
-            b.z_win[w].copy_(b.z[:, w * W:w * W + W + 1])
-            b.lpo_win[w].copy_(b.logp_old[:, w * W:(w + 1) * W])
-            vw = b.v_win[w]
-            vw[:, 0].copy_(v_end[w * 2 * G:w * 2 * G + G].reshape(G, -1))
-            vw[:, W - 1].copy_(v_end[w * 2 * G + G:(w + 1) * 2 * G].reshape(G, -1))
-            if W > 2:
-                vw[:, 1:W - 1].copy_(v_mid[w * (W - 2) * G:(w + 1) * (W - 2) * G].reshape(G, W - 2, -1))
-            # Phases 2-3
-            b.signals(w, b.lpo_win[w], cot_out=b.cot_all[w * 2 * G:(w + 1) * 2 * G])
-            if host:
-                h_lpn[:, w * W:(w + 1) * W].copy_(b.sig_out["logp_new"], non_blocking=True)
-        # Phase 4 for the whole group
-        jg.dit_joint_vjp(b.model, saved, B, b.cot_all[:B], b.grad, b.ws)
+        for ci, c in enumerate(chunks):
+            r = m = 0
+            for w in c:
+                zw = b.z[:, w * W:(w + 1) * W].reshape(G, W, *b.shape)
+                if routes[w]:
+                    z_sv[r:r + G].copy_(zw[:, 0])
+                    z_sv[r + G:r + 2 * G].copy_(zw[:, W - 1])
+                    r += 2 * G
+                    if W > 2:
+                        z_mid[m:m + (W - 2) * G].copy_(zw[:, 1:W - 1].reshape(-1, *b.shape))
+                        m += (W - 2) * G
+                else:
+                    z_sv[r:r + W * G].copy_(zw.reshape(G * W, *b.shape))
+                    r += W * G
+            # Phase 1: saved rows (endpoints, or every step of an exact window), middle steps without saves
+            jg.dit_forward_save(b.model, z_sv[:r], t_sv[ci], txt_sv[:r], v_sv[:r], saved=saved, ws=b.ws)
+            if m:
+                jg.dit_forward_save(b.model, z_mid[:m], t_mid[ci], txt_mid[:m], v_mid[:m], ws=b.ws)
+            r = m = 0
+            for w in c:
+                b.z_win[w].copy_(b.z[:, w * W:w * W + W + 1])
+                b.lpo_win[w].copy_(b.logp_old[:, w * W:(w + 1) * W])
+                vw = b.v_win[w]
+                if routes[w]:
+                    vw[:, 0].copy_(v_sv[r:r + G].reshape(G, -1))
+                    vw[:, W - 1].copy_(v_sv[r + G:r + 2 * G].reshape(G, -1))
+                    if W > 2:
+                        vw[:, 1:W - 1].copy_(v_mid[m:m + (W - 2) * G].reshape(G, W - 2, -1))
+                        m += (W - 2) * G
+                    # Phases 2-3
+                    b.signals(w, b.lpo_win[w], cot_out=b.cot_all[r:r + 2 * G])
+                    r += 2 * G
+                else:
+                    vw.copy_(v_sv[r:r + W * G].reshape(G, W, D))
+                    b.signals(w, b.lpo_win[w], s_out=b.cot_all[r:r + W * G].view(G, W, D))
+                    r += W * G
+                if host:
+                    h_lpn[:, w * W:(w + 1) * W].copy_(b.sig_out["logp_new"], non_blocking=True)
+            # Phase 4
+            jg.dit_joint_vjp(b.model, saved, r, b.cot_all[:r], b.grad, b.ws)
         jg.grad_reduce(b.grad, None, out3=b.out3, ws=b.gws)
         if host:
             h_out3.copy_(b.out3, non_blocking=True)
@@ -743,59 +875,31 @@ def jagg_update(b, host):
 
     h2d = h_z.numel() * 4 + h_lpo.numel() * 8 + h_rw.numel() * 4
     d2h = h_lpn.numel() * 8 + h_out3.numel() * 8
-    return step, h2d, d2h
+    return step, h2d, d2h, len(chunks) == 1
 
 
-def full_w_update(b):
-    """The exact per-step update stage of one group (jagg_frac = 0): the forward with saves of
-    every step of every window, each step's own signal, one VJP over all W*G rows of every
-    window, the gradient norm.  Returns the step, or None when its saved activations do
-    not fit."""
-    jg, wl, dev = b.jg, b.wl, b.dev
-    G, W, D = wl.G, wl.W, b.D
-    full = [0] * b.nw
-    if not b.fits(full):
-        return None
-    B = b.nw * W * G
-    saved = jg.alloc_bytes(b.model.saved_bytes(B), dev)
-    z_all = torch.empty(B, *b.shape, dtype=b.tdt, device=dev)
-    v_all = torch.empty(B, *b.shape, dtype=b.tdt, device=dev)
-    t_all = torch.tensor(np.concatenate([np.tile(b.t[w * W:(w + 1) * W], G) for w in range(b.nw)]),
-                         dtype=torch.float32, device=dev)
-    txt = b.txt_rows(B)
-
-    def step():
-        for w in range(b.nw):      # sample-major rows of each window, matching s [G, W, D]
-            z_all[w * W * G:(w + 1) * W * G].copy_(b.z[:, w * W:(w + 1) * W].reshape(G * W, *b.shape))
-        jg.dit_forward_save(b.model, z_all, t_all, txt, v_all, saved=saved, ws=b.ws)
-        for w in range(b.nw):
-            b.z_win[w].copy_(b.z[:, w * W:w * W + W + 1])
-            b.v_win[w].copy_(v_all[w * W * G:(w + 1) * W * G].reshape(G, W, D))
-            b.signals(w, b.lpo_win[w], s_out=b.cot_all[w * W * G:(w + 1) * W * G].view(G, W, D))
-        jg.dit_joint_vjp(b.model, saved, B, b.cot_all[:B], b.grad, b.ws)
-        jg.grad_reduce(b.grad, None, out3=b.out3, ws=b.gws)
-    return step
-
-
-def update_stage(b, args, ws, use_graph):
+def update_stage(b, args, ws, use_graph, steps, warmup):
     """The update time the paper reports for its efficiency analysis (forwards on the stored
     experience + backward), device-resident, JAGG against the exact per-step path."""
     wl = b.wl
     units = wl.G * wl.T
-    step, _, _ = jagg_update(b, host=False)
-    ms_j, graph = time_steps(step, args.steps, args.warmup, ws, use_graph)
+    lg = argparse.Namespace(steps=steps, warmup=warmup)
+    step, _, _, one = update_step(b, [1] * b.nw, host=False)
+    ms_j, graph = time_steps(step, lg.steps, lg.warmup, ws, use_graph)
     del graph, step
     torch.cuda.empty_cache()
-    out = {"jagg": {"value": ws * units / (ms_j / 1000.0), "unit": UNIT, "ms_per_step": max_over_ranks(ms_j, ws)}}
-    fstep = full_w_update(b)
-    if fstep is not None:
-        ms_f, graph = time_steps(fstep, args.steps, args.warmup, ws, use_graph)
-        del graph, fstep
-        torch.cuda.empty_cache()
-        out["full_w"] = {"value": ws * units / (ms_f / 1000.0), "unit": UNIT, "ms_per_step": max_over_ranks(ms_f, ws)}
-        out["speedup"] = ms_f / ms_j
-        # forward = 1 unit, backward = 2: W * 3 units exact against W + 2 * 2 with JAGG
-        out["ideal_speedup"] = 3.0 * wl.W / (wl.W + 4.0)
+    out = {"jagg": {"value": ws * units / (ms_j / 1000.0), "unit": UNIT, "ms_per_step": max_over_ranks(ms_j, ws),
+                    "vjp_calls": 1 if one else b.nw}}
+    fstep, _, _, one = update_step(b, [0] * b.nw, host=False)
+    ms_f, graph = time_steps(fstep, lg.steps, lg.warmup, ws, use_graph)
+    del graph, fstep
+    torch.cuda.empty_cache()
+    out["full_w"] = {"value": ws * units / (ms_f / 1000.0), "unit": UNIT, "ms_per_step": max_over_ranks(ms_f, ws),
+                     "vjp_calls": 1 if one else b.nw}
+    out["speedup"] = ms_f / ms_j
+    # forward = 1 unit, backward = 2: W * 3 units exact against W + 2 * 2 with JAGG
+    out["ideal_speedup"] = 3.0 * wl.W / (wl.W + 4.0)
+    out["steps"], out["warmup"] = steps, warmup
     out["scope"] = ("per group: the forwards on the stored trajectories (JAGG: endpoints saved, middle steps "
                     "without; exact: every step saved), the step signals, the VJP(s), the gradient norm")
     return out
@@ -812,22 +916,107 @@ def rollout_leg(b, args, ws, use_graph):
             "ms_per_step": max_over_ranks(ms, ws)}
 
 
-def run_e2e(b, args, ws, routes):
-    """The JAGG update stage through the public API from pinned host buffers (jagg_update
+def run_e2e(b, args, ws, routes, steps, warmup):
+    """The JAGG update stage through the public API from pinned host buffers (update_step
     with host=True), timed on the host clock."""
     wl = b.wl
-    step, h2d, d2h = jagg_update(b, host=True)
-    steps = max(2, args.steps // 2)
-    for _ in range(max(1, args.warmup // 2)):
+    step, h2d, d2h, one = update_step(b, routes, host=True)
+    for _ in range(warmup):
         step()
     barrier(ws)
     t0 = time.perf_counter()
     for _ in range(steps):
         step()
     sec = max_over_ranks((time.perf_counter() - t0) / steps, ws)
+    del step
+    torch.cuda.empty_cache()
     return {"value": ws * wl.G * wl.T / sec, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-            "ms_per_step": 1000 * sec, "steps": steps,
-            "includes": "Phase 1 forwards (2G rows saved + (W-2)G rows unsaved per window), signals, one joint VJP"}
+            "ms_per_step": 1000 * sec, "steps": steps, "warmup": warmup,
+            "includes": ("H2D of the group's trajectory, old log-probs and rewards; per window the Phase 1 "
+                         "forwards (2G endpoint rows saved, (W-2)G middle rows unsaved), signals with aggregation; "
+                         + ("one joint VJP over the group" if one else "one joint VJP per window") +
+                         "; gradient norm; D2H of the new log-probs and the norm")}
+
+
+def window_cosines(b):
+    """Per window, the cosine between its JAGG gradient (the 2G endpoint rows with the
+    aggregated cotangents) and its exact per-step gradient (all W*G rows with their own
+    s_j), each accumulated into its own zeroed buffer and compared by grad_reduce: the
+    quantity the gradient-quality appendix routes on (cos >= 0.5)."""
+    jg, wl, dev = b.jg, b.wl, b.dev
+    G, W, D = wl.G, wl.W, b.D
+    g_j = torch.empty(b.P, dtype=torch.float32, device=dev)
+    g_e = torch.empty(b.P, dtype=torch.float32, device=dev)
+    out3 = torch.empty(3, dtype=torch.float64, device=dev)
+    cos = []
+    for w in range(b.nw):
+        g_j.zero_()
+        g_e.zero_()
+        zw = b.z[:, w * W:(w + 1) * W].reshape(G, W, *b.shape)
+        for jagg, g in ((True, g_j), (False, g_e)):
+            z, t = b.rows(zw, w, jagg)
+            B = z.shape[0]
+            saved = jg.alloc_bytes(b.model.saved_bytes(B), dev)
+            v = torch.empty_like(z)
+            jg.dit_forward_save(b.model, z, t, b.txt_rows(B), v, saved=saved, ws=b.ws)
+            cot = b.cot_all[:B]
+            if jagg:
+                b.signals(w, b.lpo_win[w], cot_out=cot)
+            else:
+                b.signals(w, b.lpo_win[w], s_out=cot.view(G, W, D))
+            jg.dit_joint_vjp(b.model, saved, B, cot, g, b.ws)
+            torch.cuda.synchronize()
+            del saved, v
+        jg.grad_reduce(g_j, g_e, out3=out3, ws=b.gws)
+        ab, aa, bb = out3.tolist()
+        cos.append(ab / (aa * bb) ** 0.5 if aa > 0 and bb > 0 else 0.0)
+    del g_j, g_e
+    torch.cuda.empty_cache()
+    return cos
+
+
+def run_sweep(args, ws, rank):
+    """The routing and window sweep on the Qwen-width MMDiT (8 double-stream blocks, d = 3072,
+    1024 image + 256 text tokens, G = 8, T = 16): for W in {2, 4, 8} and jagg_frac in
+    {0, 0.5, 1} (schedule routing, n_jagg = floor(jagg_frac n_w)), the group step of
+    Phases 2-4 with one joint VJP per window (Algorithm 1), every window's saved activations
+    resident; the speed-up over jagg_frac = 0 against the ideal ratio of VJP rows (W/2 when
+    every window is routed); per window the cosine between the JAGG and exact gradients
+    and the routes the calibration rule (cos >= 0.5) derives from them."""
+    import paper_2607_17572_gb300 as jg
+    dev = torch.device("cuda", torch.cuda.current_device())
+    base = workload(args)
+    use_graph = not args.no_graph
+    burst, sustained, hbm, src = peaks()
+    table, t_start = {}, time.perf_counter()
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        for W in (2, 4, 8):
+            wl = synth.small_variant(base, W=W)
+            b = Bench(wl, dev)
+            b.rollout()
+            cells = {}
+            for frac in (0.0, 0.5, 1.0):
+                routes, _ = jg.jagg_route(b.nw, frac)
+                r = measure(b, routes, False, args, ws, use_graph)
+                rows = sum(2 * wl.G if x else W * wl.G for x in routes)
+                cells[str(frac)] = {"value": job_rate(wl.G * wl.T, r["ms"], ws), "ms_per_step": r["ms"],
+                                    "routes": routes, "vjp_rows_per_step": rows,
+                                    "resident": r["resident"]}
+                torch.cuda.empty_cache()
+            full_rows = cells["0.0"]["vjp_rows_per_step"]
+            for c in cells.values():
+                c["speedup_vs_full_w"] = cells["0.0"]["ms_per_step"] / c["ms_per_step"]
+                c["ideal_speedup"] = full_rows / c["vjp_rows_per_step"]
+            cos = window_cosines(b)
+            calib, derived = jg.jagg_route(b.nw, 1.0, cos=cos, tau=0.5)
+            table[f"W={W}"] = {"windows": b.nw, "cells": cells, "window_cos": cos, "calibrated_routes": calib,
+                               "derived_jagg_frac": derived}
+            del b
+            torch.cuda.empty_cache()
+    if rank == 0:
+        print(json.dumps({"metric": METRIC, "unit": UNIT, "sweep": "W x jagg_frac", "workload": describe(base),
+                          "steps": args.steps, "warmup": args.warmup, "cuda_graph": use_graph, "table": table,
+                          "clocks": clk.summary(), "wall_s": time.perf_counter() - t_start}), flush=True)
 
 
 def run_kernel_attention_bwd(args):
@@ -895,13 +1084,30 @@ def run_kernel_attention_bwd(args):
 def gemm_products(wl, rows):
     """The dense products of one block's backward at `rows` token rows, in the operand layouts
     of the joint VJP: name -> (M, N, K, a_mn, b_mn, epilogue).  Input gradients dX = dY W
-    (K-major dY, MN-major W; the fc2 one times GELU'(u), the multiplier epilogue), weight
-    gradients dW += dY^T X (both MN-major, f32 accumulation)."""
+    (K-major dY, MN-major W; the ones into GELU's input times GELU'(u), the multiplier
+    epilogue), weight gradients dW += dY^T X (both MN-major, f32 accumulation).  DiT: one
+    block.  MMDiT: a Flux-style single block at the joint rows (lin2's two input-gradient
+    parts, [o] and [GELU(u)]; lin1 over [qkv | u]) and a double block's image-stream
+    products at its image rows."""
     d, f = wl.hidden, wl.mlp
-    return {"fc2_dx": (rows, f, d, False, True, "mul_aux"), "fc1_dx": (rows, d, f, False, True, "store"),
-            "qkv_dx": (rows, d, 3 * d, False, True, "store"), "proj_dx": (rows, d, d, False, True, "store"),
-            "fc2_dw": (d, f, rows, True, True, "accum"), "fc1_dw": (f, d, rows, True, True, "accum"),
-            "qkv_dw": (3 * d, d, rows, True, True, "accum"), "proj_dw": (d, d, rows, True, True, "accum")}
+
+    def block(r, pre=""):
+        return {pre + "fc2_dx": (r, f, d, False, True, "mul_aux"), pre + "fc1_dx": (r, d, f, False, True, "store"),
+                pre + "qkv_dx": (r, d, 3 * d, False, True, "store"), pre + "proj_dx": (r, d, d, False, True, "store"),
+                pre + "fc2_dw": (d, f, r, True, True, "accum"), pre + "fc1_dw": (f, d, r, True, True, "accum"),
+                pre + "qkv_dw": (3 * d, d, r, True, True, "accum"), pre + "proj_dw": (d, d, r, True, True, "accum")}
+    if wl.arch == "dit":
+        return block(rows)
+    out = {}
+    if wl.depth:
+        out.update({"lin2_dx_o": (rows, d, d, False, True, "store"),
+                    "lin2_dx_u": (rows, f, d, False, True, "mul_aux"),
+                    "lin1_dx": (rows, d, 3 * d + f, False, True, "store"),
+                    "lin2_dw": (d, d + f, rows, True, True, "accum"),
+                    "lin1_dw": (3 * d + f, d, rows, True, True, "accum")})
+    if wl.depth_double:
+        out.update(block(rows * wl.n_img // wl.n_tok, "img_"))
+    return out
 
 
 def run_kernel_gemm(args):
@@ -981,6 +1187,8 @@ def main():
             run_kernel_gemm(args)
     elif args.impl == "reference":
         run_reference(args, ws, rank)
+    elif args.sweep:
+        run_sweep(args, ws, rank)
     else:
         run_gpu(args, ws, rank)
     if ws > 1:
