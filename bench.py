@@ -348,7 +348,10 @@ class Bench:
         takes at most half of the free memory; otherwise (one arena per window) the arenas
         together take at most 85 % of it."""
         plan, rows = self.plan(routes)
+        torch.cuda.empty_cache()
         free, _ = torch.cuda.mem_get_info(self.dev)
+        self.last_fit = {"free_gb": free / 1e9, "saved_gb_needed": (self.model.saved_bytes(rows) if batched else sum(
+            self.model.saved_bytes(n) for (_, _, _, n) in plan)) / 1e9}
         if batched:
             return rows <= self.ws_rows and self.model.saved_bytes(rows) < 0.5 * free
         return sum(self.model.saved_bytes(n) for (_, _, _, n) in plan) < 0.85 * free
@@ -447,6 +450,9 @@ def oracle_sample_plan(wl):
     return sub, 1, 1, full / part
 
 
+_ORACLE_MODEL = {}   # the sample's backbone, built once per process
+
+
 def oracle_sample(wl):
     """One bounded sample of the workload on the float64 oracle (oracle_sample_plan): the step
     signals of one window on synthetic v-hat, the t-weighted aggregation, the forward of the
@@ -454,8 +460,9 @@ def oracle_sample(wl):
     sample stands for, seconds scaled to them, description)."""
     from oracle import dit, grpo
     sub, rows, n_samples, scale = oracle_sample_plan(wl)
-    params = synth.make_params(sub)
-    model = dit.Backbone(sub, params)
+    if _ORACLE_MODEL.get("name") != sub.name:
+        _ORACLE_MODEL.update(name=sub.name, model=dit.Backbone(sub, synth.make_params(sub)))
+    model = _ORACLE_MODEL["model"]
     rng = np.random.Generator(np.random.PCG64(5))
     W = wl.W
     shape = (wl.in_channels, wl.latent_h, wl.latent_w)
@@ -715,7 +722,9 @@ def run_gpu(args, ws, rank):
     att["frac_of_burst"] = att["achieved"] / burst
     step_flops = sum(v["flops"] for k, v in fam.items() if k != "gemm_simt")
     families = {k: {"launches_per_step": v["launches"], "ms_per_step": v["ms"],
-                    "tflops": (v["flops"] / (v["ms"] / 1000.0) / 1e12) if v["ms"] > 0 else None}
+                    "tflops": (v["flops"] / (v["ms"] / 1000.0) / 1e12) if v["ms"] > 0 else None,
+                    "algorithmic_gb_per_step": v["bytes"] / 1e9,
+                    "gbs": (v["bytes"] / (v["ms"] / 1000.0) / 1e9) if v["ms"] > 0 else None}
                 for k, v in fam.items()}
     if batched:
         batching = f"one joint VJP per group over all {b.nw} windows' endpoint rows"
@@ -729,6 +738,7 @@ def run_gpu(args, ws, rank):
            "config": {"workload": describe(wl), "rows_per_vjp": r["rows"], "windows": b.nw,
                       "cuda_graph": use_graph, "vjp_batching": batching,
                       "l2": "inputs larger than L2 (saved activations %.1f GB resident)" % r["saved_gb"],
+                      "memory_plan": getattr(b, "last_fit", None),
                       "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU"},
            "roofline": roofline, "roofline_attention_bwd": att,
            "algorithmic_tflops_per_step": step_flops / 1e12,

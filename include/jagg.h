@@ -71,11 +71,15 @@ int jagg_device_status(unsigned* status_out, int clear);
 int64_t jagg_launch_count(void);
 
 /* Kernel timing by family.  jagg_profile_enable(1) clears earlier records and starts
- * bracketing every dense-product and attention launch with CUDA events on its stream
- * (this adds two event records per launch); jagg_profile_enable(0) stops.
- * jagg_profile_read synchronises the device and fills up to `cap` entries, one per
- * family: launches, summed device milliseconds, summed algorithmic FLOPs (2 per
- * multiply-add of the products the operation defines) and algorithmic bytes. */
+ * bracketing the launches of the path's kernels with CUDA events on their stream (this
+ * adds two event records per launch); jagg_profile_enable(0) stops.  Families, in this
+ * order: gemm_tcgen05, gemm_simt, attention_fwd, attention_bwd, ln_gate_bwd,
+ * attention_bwd_aux, qk_norm_rope_bwd, colsum, copy_rows, step_signals, grad_reduce,
+ * ln_mod_fwd, qk_norm_rope_fwd (step_signals and grad_reduce cover a whole call of the
+ * entry point).  jagg_profile_read synchronises the device and fills up to `cap` entries,
+ * one per family: launches, summed device milliseconds, summed algorithmic FLOPs (2 per
+ * multiply-add of the products the operation defines) and algorithmic bytes (each input
+ * read once, each output written once). */
 typedef struct jagg_profile_stat {
   char family[32];
   int64_t launches;

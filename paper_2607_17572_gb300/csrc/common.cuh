@@ -119,9 +119,9 @@ int sm_count();
 
 // ------------------------------------------------------------------ launch accounting
 // Every kernel launch of the library is counted (jagg_launch_count).  While profiling is
-// enabled (jagg_profile_enable), the dense-product and attention launches are also
-// bracketed by CUDA events on their stream and attributed to a kernel family with their
-// algorithmic FLOPs and bytes.
+// enabled (jagg_profile_enable), the launches of the path's kernels are also bracketed by
+// CUDA events on their stream and attributed to a kernel family with their algorithmic
+// FLOPs and bytes.
 void count_launch();
 enum ProfFamily : int {
   PROF_GEMM_TC = 0,
@@ -130,6 +130,13 @@ enum ProfFamily : int {
   PROF_ATTN_BWD,
   PROF_LN_BWD,     // LayerNorm + gate backward
   PROF_ATTN_AUX,   // attention backward helpers (rowsum(dO O), dQ conversion)
+  PROF_QKN_BWD,    // per-head RMSNorm + RoPE backward
+  PROF_COLSUM,     // bias gradients (column sums)
+  PROF_COPY,       // row copies between the stream and joint layouts
+  PROF_SIGNALS,    // the step signals (with the aggregation when fused)
+  PROF_GRAD_REDUCE,
+  PROF_LN_FWD,     // LayerNorm + modulation forward
+  PROF_QKN_FWD,    // per-head RMSNorm + RoPE forward
   PROF_FAMILIES
 };
 int prof_start(cudaStream_t s);  // returns a token, or -1 when profiling is off

@@ -771,8 +771,12 @@ int launch_add_pos_embed(float* h, int B, int rows_per_seq, int row0, int gh, in
 int launch_ln_mod_fwd(const LnModFwd& a, cudaStream_t s) {
   JAGG_CHECK_ARG(a.d % 4 == 0 && a.d <= 128 * LN_MAXV, "ln_mod: hidden %d unsupported", a.d);
   const int warps = 8;
+  const int tok = prof_start(s);
   ln_mod_fwd_kernel<<<ceil_div(a.M, warps), warps * 32, 0, s>>>(a);
   JAGG_LAUNCHED();
+  // algorithmic bytes: h read (f32), the modulated output written (storage type), statistics
+  prof_stop(tok, s, PROF_LN_FWD, 0.0,
+            (double)a.M * (a.d * (4.0 + (a.dtype == JAGG_DTYPE_F32 ? 4.0 : 2.0)) + 8.0));
   return JAGG_OK;
 }
 // The row-in-registers kernel serves LayerNorm backwards with an f32 dm (with or without the
@@ -810,15 +814,20 @@ int launch_ln_gate_bwd(const LnGateBwd& a, cudaStream_t s) {
 }
 int launch_colsum(const void* X, int x_f32, int dtype, int rows, int cols, int64_t ld, float* db, cudaStream_t s) {
   (void)dtype;
+  const int tok = prof_start(s);
+  // algorithmic bytes: X read once, db read and written
+  const double bytes = (double)rows * cols * (x_f32 ? 4 : 2) + 8.0 * cols;
   if (!x_f32 && cols % 8 == 0 && ld % 8 == 0 && (reinterpret_cast<uintptr_t>(X) & 15) == 0) {
     dim3 grid(ceil_div(cols, 256), ceil_div(rows, CSV_ROWS));
     colsum_bf16x8_kernel<<<grid, 256, 0, s>>>(static_cast<const bf16*>(X), rows, cols, ld, db);
     JAGG_LAUNCHED();
+    prof_stop(tok, s, PROF_COLSUM, 0.0, bytes);
     return JAGG_OK;
   }
   dim3 grid(ceil_div(cols, 256), ceil_div(rows, CS_ROWS));
   colsum_kernel<<<grid, 256, 0, s>>>(X, x_f32, rows, cols, ld, db);
   JAGG_LAUNCHED();
+  prof_stop(tok, s, PROF_COLSUM, 0.0, bytes);
   return JAGG_OK;
 }
 int launch_gather_rows(const float* in, int64_t ld_in, int seg, int seg_off, int64_t seg_stride, void* out,
@@ -832,6 +841,7 @@ int launch_copy_rows(const void* in, int64_t ld_in, int in_seg, int in_seg_off, 
                      int64_t ld_out, int out_seg, int out_seg_off, int64_t out_seg_stride, int rows, int cols,
                      int elem_bytes, cudaStream_t s) {
   const int g = grid_for((int64_t)rows * cols, 256);
+  const int tok = prof_start(s);
   if (elem_bytes == 4)
     copy_rows_kernel<float><<<g, 256, 0, s>>>(static_cast<const float*>(in), ld_in, in_seg, in_seg_off, in_seg_stride,
                                              static_cast<float*>(out), ld_out, out_seg, out_seg_off, out_seg_stride,
@@ -841,6 +851,7 @@ int launch_copy_rows(const void* in, int64_t ld_in, int in_seg, int in_seg_off, 
                                                 in_seg_stride, static_cast<uint16_t*>(out), ld_out, out_seg,
                                                 out_seg_off, out_seg_stride, rows, cols);
   JAGG_LAUNCHED();
+  prof_stop(tok, s, PROF_COPY, 0.0, 2.0 * rows * cols * elem_bytes);
   return JAGG_OK;
 }
 int launch_attn_rowdot(const void* dO, const void* O, int64_t ld, float* Dv, int B, int N, int heads, int dh,
@@ -856,8 +867,12 @@ int launch_qk_norm_rope_fwd(const QkNormRope& a, cudaStream_t s) {
                  "qk_norm: head dim unsupported");
   if (a.M <= 0) return JAGG_OK;
   const int64_t blocks = ((int64_t)a.M * a.heads + QKN_WARPS - 1) / QKN_WARPS;
+  const int tok = prof_start(s);
   qk_norm_rope_fwd_kernel<<<(int)(blocks < 65536 ? blocks : 65536), QKN_THREADS, 0, s>>>(a);
   JAGG_LAUNCHED();
+  // algorithmic bytes: raw q, k read, transformed q, k written (storage type), 1/rms of both
+  const double esz = a.dtype == JAGG_DTYPE_F32 ? 4.0 : 2.0;
+  prof_stop(tok, s, PROF_QKN_FWD, 0.0, (double)a.M * (4.0 * a.d * esz + 8.0 * a.heads));
   return JAGG_OK;
 }
 int launch_qk_norm_rope_bwd(const QkNormRopeBwd& a, cudaStream_t s) {
@@ -869,8 +884,12 @@ int launch_qk_norm_rope_bwd(const QkNormRopeBwd& a, cudaStream_t s) {
   // a few blocks per SM: each block ends in 4 dh atomics
   const int64_t blocks = ((int64_t)f.M * f.heads + QKN_WARPS - 1) / QKN_WARPS;
   const int cap = 4 * sm_count();
+  const int tok = prof_start(s);
   qk_norm_rope_bwd_kernel<<<(int)(blocks < cap ? blocks : cap), QKN_THREADS, 0, s>>>(a);
   JAGG_LAUNCHED();
+  // algorithmic bytes: dq, dk read and rewritten in place, raw q, k read (storage type), 1/rms
+  const double esz = f.dtype == JAGG_DTYPE_F32 ? 4.0 : 2.0;
+  prof_stop(tok, s, PROF_QKN_BWD, 0.0, (double)f.M * (6.0 * f.d * esz + 8.0 * f.heads));
   return JAGG_OK;
 }
 

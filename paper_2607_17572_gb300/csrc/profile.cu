@@ -33,8 +33,10 @@ cudaEvent_t get_event() {
   return e;
 }
 
-const char* kFamilyNames[PROF_FAMILIES] = {"gemm_tcgen05",  "gemm_simt",   "attention_fwd",
-                                           "attention_bwd", "ln_gate_bwd", "attention_bwd_aux"};
+const char* kFamilyNames[PROF_FAMILIES] = {"gemm_tcgen05",     "gemm_simt",   "attention_fwd", "attention_bwd",
+                                           "ln_gate_bwd",      "attention_bwd_aux", "qk_norm_rope_bwd",
+                                           "colsum",           "copy_rows",   "step_signals",  "grad_reduce",
+                                           "ln_mod_fwd",       "qk_norm_rope_fwd"};
 
 }  // namespace
 

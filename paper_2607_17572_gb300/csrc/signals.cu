@@ -439,6 +439,7 @@ int step_signals(const char* name, const void* v_hat, int v_dtype, const float* 
   double* partial = reinterpret_cast<double*>(static_cast<char*>(ws) + mean_coef_bytes(W));
   float* coef = reinterpret_cast<float*>(partial + (int64_t)G * W * chunks);
   const int vf32 = v_dtype == JAGG_DTYPE_F32;
+  const int tok = prof_start(stream);
   prep_kernel<<<1, 32, 0, stream>>>(rewards, G, adv_eps, adv_clip, adv_out, t, sched_alpha, sched_sigma, W, mc);
   JAGG_LAUNCHED();
   resid_norm_kernel<<<dim3(chunks, G * W), SIG_THREADS, 0, stream>>>(v_hat, vf32, z, mc, W, D, partial);
@@ -457,6 +458,11 @@ int step_signals(const char* name, const void* v_hat, int v_dtype, const float* 
                                                           cot_out);
     JAGG_LAUNCHED();
   }
+  // algorithmic bytes: v-hat and the W + 1 latents of every sample read once, the signals
+  // (G W rows) or the cotangents (2G rows) written in f32
+  const double out_rows = s_out ? (double)G * W : (cot_out ? 2.0 * G : 0.0);
+  prof_stop(tok, stream, PROF_SIGNALS, 0.0,
+            (double)D * ((double)G * W * (vf32 ? 4.0 : 2.0) + (double)G * (W + 1) * 4.0 + out_rows * 4.0));
   return JAGG_OK;
 }
 }  // namespace
@@ -591,6 +597,7 @@ extern "C" int grad_reduce(const float* a, const float* b, int64_t P, float alph
       return JAGG_ERR_WORKSPACE;
     }
   }
+  const int tok = prof_start(stream);
   grad_reduce_kernel<<<GR_BLOCKS, GR_THREADS, 0, stream>>>(a, b, P, alpha, acc,
                                                            out3 ? static_cast<double*>(ws) : nullptr);
   JAGG_LAUNCHED();
@@ -598,6 +605,8 @@ extern "C" int grad_reduce(const float* a, const float* b, int64_t P, float alph
     grad_reduce_final<<<1, 32, 0, stream>>>(static_cast<const double*>(ws), out3);
     JAGG_LAUNCHED();
   }
+  // algorithmic bytes: a (and b) read, acc read and written
+  prof_stop(tok, stream, PROF_GRAD_REDUCE, 0.0, 4.0 * P * (1.0 + (b ? 1.0 : 0.0) + (acc ? 2.0 : 0.0)));
   return JAGG_OK;
 }
 
