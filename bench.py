@@ -346,7 +346,7 @@ class Bench:
         """Every window's saved activations can be resident at once.  batched (one arena,
         one joint VJP over the group): the workspace covers the group's rows and the arena
         takes at most half of the free memory; otherwise (one arena per window) the arenas
-        together take at most 85 % of it."""
+        together take at most 90 % of it."""
         plan, rows = self.plan(routes)
         torch.cuda.empty_cache()
         free, _ = torch.cuda.mem_get_info(self.dev)
@@ -354,7 +354,7 @@ class Bench:
             self.model.saved_bytes(n) for (_, _, _, n) in plan)) / 1e9}
         if batched:
             return rows <= self.ws_rows and self.model.saved_bytes(rows) < 0.5 * free
-        return sum(self.model.saved_bytes(n) for (_, _, _, n) in plan) < 0.85 * free
+        return sum(self.model.saved_bytes(n) for (_, _, _, n) in plan) < 0.9 * free
 
     def forward_saves(self, routes, batched, windows=None):
         """Phase 1 with saves for the rows of the plan (or of the listed windows only).

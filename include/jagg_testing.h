@@ -81,6 +81,23 @@ int jagg_test_attention_bwd_streams(const void* qkv0, const void* qkv1, const vo
                                     int heads, int dh, int dtype, void* dqkv0, void* dqkv1, void* scratch, int impl,
                                     cudaStream_t stream);
 
+/* LayerNorm + modulation backward fused with the gate backward of the branch before it (the
+ * per-row kernels of the joint VJP; the paper's Phase 4 reverse mode through adaLN), on M
+ * rows of rows_per_seq rows per sequence, hidden size d (d % 4 == 0, d <= 3072).  Row m of
+ * sequence b = m / rows_per_seq, all buffers row-major and contiguous (f32 unless noted):
+ *   do_ln:   xh = (h - mean[m]) rstd[m]; e = dm (1 + scale[b]);
+ *            dh_out = dh_in + rstd (e - mean_row(e) - xh mean_row(e xh));
+ *            dshift[b] += sum_m dm, dscale[b] += sum_m dm xh   (dm [M, d] f32)
+ *   do_gate: dy = gate[b] dh (dh = dh_out, or dh_in without do_ln); dgate[b] += sum_m dh y;
+ *            dbias (nullable) += sum_b gate[b] sum_{m in b} dh   (y, dy [M, d] in `dtype`)
+ * scale, gate: [M / rows_per_seq, d]; dshift, dscale, dgate: [M / rows_per_seq, d],
+ * accumulated.  dh_out may alias dh_in.  JAGG_ERR_ARG for an unsupported d or rows that are
+ * not whole sequences. */
+int jagg_test_ln_gate_bwd(int M, int d, int rows_per_seq, int do_ln, int do_gate, const float* dm, const float* h,
+                          const float* mean, const float* rstd, const float* scale, float* dshift, float* dscale,
+                          const float* dh_in, float* dh_out, const void* y, const float* gate, float* dgate,
+                          void* dy, float* dbias, int dtype, cudaStream_t stream);
+
 /* Failure detection of the bounded waits (every mbarrier wait of the library gives up after
  * a wall-clock limit instead of hanging): one CTA waits on an mbarrier that nothing arrives
  * at, with the limit limit_ns (0 < limit_ns <= 2 s, else JAGG_ERR_ARG) in place of the

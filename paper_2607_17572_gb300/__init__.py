@@ -117,6 +117,8 @@ _SIGNATURES = {
     "jagg_test_attention_scratch_bytes": (_I64, [_I, _I, _I, _I]),
     "jagg_test_attention_bwd": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _P]),
     "jagg_test_attention_fwd_streams": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
+    "jagg_test_ln_gate_bwd": (_I, [_I, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P,
+                                   _I, _P]),
     "jagg_test_attention_bwd_streams": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _I,
                                              _P]),
 }
@@ -450,6 +452,18 @@ def test_attention_bwd_streams(qkv, o, lse, dO, B, N, n0, heads, dh, dqkv, impl=
     _check(lib().jagg_test_attention_bwd_streams(
         _ptr(qkv[0]), second(qkv), _ptr(o[0]), second(o), _ptr(lse), _ptr(dO[0]), second(dO), B, N, n0, heads, dh,
         dt, _ptr(dqkv[0]), second(dqkv), _ptr(scratch), impl, _stream(stream)), "jagg_test_attention_bwd_streams")
+
+
+def test_ln_gate_bwd(M, d, rows_per_seq, dh_in, dh_out, dm=None, h=None, mean=None, rstd=None, scale=None,
+                     dshift=None, dscale=None, y=None, gate=None, dgate=None, dy=None, dbias=None, stream=None):
+    """LayerNorm + modulation and gate backward on contiguous rows (jagg_test_ln_gate_bwd);
+    the LayerNorm part runs when dm is given, the gate part when y is given."""
+    do_ln, do_gate = dm is not None, y is not None
+    dt = DTYPE_BF16 if (y is not None and y.dtype == torch.bfloat16) else DTYPE_F32
+    _check(lib().jagg_test_ln_gate_bwd(M, d, rows_per_seq, int(do_ln), int(do_gate), _ptr(dm), _ptr(h), _ptr(mean),
+                                       _ptr(rstd), _ptr(scale), _ptr(dshift), _ptr(dscale), _ptr(dh_in),
+                                       _ptr(dh_out), _ptr(y), _ptr(gate), _ptr(dgate), _ptr(dy), _ptr(dbias), dt,
+                                       _stream(stream)), "jagg_test_ln_gate_bwd")
 
 
 def test_wait_timeout(limit_ns: int, out, stream=None):

@@ -453,6 +453,160 @@ __global__ void __launch_bounds__(256, 2) ln_gate_rowreg_kernel(LnGateBwd a) {
   }
 }
 
+// Row-per-CTA variant for d = 1024 NV4 (d = 3072 at the Flux and Qwen widths; bf16 y and
+// dy, dm in f32 when the LayerNorm part is present).  The 256 threads of a block take one row at a time,
+// each holding NV4 float4 column groups of every operand in registers, so every row is read
+// once and written once.  The row statistics are two block reductions: warp shuffles, then
+// the 8 warp partials through a shared slot double-buffered by row parity (one barrier per
+// row).  Each CTA owns a contiguous, equal share of the rows and each thread the same columns
+// for all of them, so the per-sequence column sums (dshift, dscale, dgate, sum dh for the
+// bias gradient) stay in registers and leave by one global atomic per column and quantity
+// at each sequence boundary.
+template <int NV4, bool LN, bool GATE>
+__global__ void __launch_bounds__(256, 2) ln_gate_rowcta_kernel(LnGateBwd a) {
+  constexpr int d = 1024 * NV4;
+  __shared__ float red[2][2][8];  // [row parity][s1, s2][warp]
+  __shared__ __align__(16) float sc_s[LN ? d : 4], gt_s[GATE ? d : 4];  // 1 + scale, gate of the sequence
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int row_begin = (int)((int64_t)a.M * blockIdx.x / gridDim.x);
+  const int row_end = (int)((int64_t)a.M * (blockIdx.x + 1) / gridDim.x);
+  int parity = 0;
+  for (int seg0 = row_begin; seg0 < row_end;) {
+    const int b = seg0 / a.rows_per_seq;
+    const int seg1 = min(row_end, (b + 1) * a.rows_per_seq);
+    float4 acc[4][NV4];
+    __syncthreads();  // the previous segment's readers of the vectors are done
+#pragma unroll
+    for (int i = 0; i < NV4; ++i) {
+      const int c = (i * 256 + tid) * 4;
+      if (LN) {
+        float4 v = *reinterpret_cast<const float4*>(a.scale + (int64_t)b * a.mod_stride + c);
+        v.x += 1.f; v.y += 1.f; v.z += 1.f; v.w += 1.f;
+        *reinterpret_cast<float4*>(sc_s + c) = v;
+      }
+      if (GATE) *reinterpret_cast<float4*>(gt_s + c) = *reinterpret_cast<const float4*>(a.gate + (int64_t)b * a.mod_stride + c);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) acc[q][i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    __syncthreads();
+#pragma unroll 1
+    for (int m = seg0; m < seg1; ++m) {
+      const int64_t hr = seg_row(m, a.seg, a.seg_off, a.seg_stride);
+      float4 dh[NV4], dm[NV4], hv[NV4];
+      uint2 yb[NV4];  // y in bf16
+#pragma unroll
+      for (int i = 0; i < NV4; ++i) {
+        const int c = (i * 256 + tid) * 4;
+        dh[i] = *reinterpret_cast<const float4*>(a.dh_in + hr * d + c);
+        if (LN) {
+          dm[i] = *reinterpret_cast<const float4*>(static_cast<const float*>(a.dm) + (int64_t)m * d + c);
+          hv[i] = *reinterpret_cast<const float4*>(a.h + hr * d + c);
+        }
+        if (GATE) yb[i] = *reinterpret_cast<const uint2*>(static_cast<const bf16*>(a.y) + (int64_t)m * d + c);
+      }
+      if (LN) {
+        const float mu = a.mean[m], rs = a.rstd[m];
+        float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+        for (int i = 0; i < NV4; ++i) {
+          hv[i].x = (hv[i].x - mu) * rs; hv[i].y = (hv[i].y - mu) * rs;  // now x-hat
+          hv[i].z = (hv[i].z - mu) * rs; hv[i].w = (hv[i].w - mu) * rs;
+          const float4 sv = *reinterpret_cast<const float4*>(sc_s + (i * 256 + tid) * 4);
+          const float e0 = dm[i].x * sv.x, e1 = dm[i].y * sv.y, e2 = dm[i].z * sv.z, e3 = dm[i].w * sv.w;
+          s1 += (e0 + e1) + (e2 + e3);
+          s2 += (e0 * hv[i].x + e1 * hv[i].y) + (e2 * hv[i].z + e3 * hv[i].w);
+        }
+        s1 = warp_sum(s1);
+        s2 = warp_sum(s2);
+        if (lane == 0) {
+          red[parity][0][warp] = s1;
+          red[parity][1][warp] = s2;
+        }
+        __syncthreads();
+        s1 = 0.f;
+        s2 = 0.f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) {
+          s1 += red[parity][0][w];
+          s2 += red[parity][1][w];
+        }
+        s1 /= d;
+        s2 /= d;
+        parity ^= 1;
+#pragma unroll
+        for (int i = 0; i < NV4; ++i) {
+          const int c = (i * 256 + tid) * 4;
+          const float4 sv = *reinterpret_cast<const float4*>(sc_s + c);
+          dh[i].x += rs * (dm[i].x * sv.x - s1 - hv[i].x * s2);
+          dh[i].y += rs * (dm[i].y * sv.y - s1 - hv[i].y * s2);
+          dh[i].z += rs * (dm[i].z * sv.z - s1 - hv[i].z * s2);
+          dh[i].w += rs * (dm[i].w * sv.w - s1 - hv[i].w * s2);
+          *reinterpret_cast<float4*>(a.dh_out + hr * d + c) = dh[i];
+          acc[0][i].x += dm[i].x; acc[0][i].y += dm[i].y; acc[0][i].z += dm[i].z; acc[0][i].w += dm[i].w;
+          acc[1][i].x += dm[i].x * hv[i].x; acc[1][i].y += dm[i].y * hv[i].y;
+          acc[1][i].z += dm[i].z * hv[i].z; acc[1][i].w += dm[i].w * hv[i].w;
+        }
+      }
+      if (GATE) {
+#pragma unroll
+        for (int i = 0; i < NV4; ++i) {
+          const int c = (i * 256 + tid) * 4;
+          const float4 g4 = *reinterpret_cast<const float4*>(gt_s + c);
+          const float dy[4] = {g4.x * dh[i].x, g4.y * dh[i].y, g4.z * dh[i].z, g4.w * dh[i].w};
+          store4(a.dy, (int64_t)m * d + c, 0, dy);
+          const bf16* yh = reinterpret_cast<const bf16*>(&yb[i]);
+          acc[2][i].x += dh[i].x * __bfloat162float(yh[0]); acc[2][i].y += dh[i].y * __bfloat162float(yh[1]);
+          acc[2][i].z += dh[i].z * __bfloat162float(yh[2]); acc[2][i].w += dh[i].w * __bfloat162float(yh[3]);
+          acc[3][i].x += dh[i].x; acc[3][i].y += dh[i].y; acc[3][i].z += dh[i].z; acc[3][i].w += dh[i].w;
+        }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < NV4; ++i) {
+      const int c = (i * 256 + tid) * 4;
+      const float* q0 = &acc[0][i].x;
+      const float* q1 = &acc[1][i].x;
+      const float* q2 = &acc[2][i].x;
+      const float* q3 = &acc[3][i].x;
+      const float* g4 = gt_s + c;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        if (LN) {
+          atomicAdd(a.dshift + (int64_t)b * a.dmod_stride + c + e, q0[e]);
+          atomicAdd(a.dscale + (int64_t)b * a.dmod_stride + c + e, q1[e]);
+        }
+        if (GATE) {
+          atomicAdd(a.dgate + (int64_t)b * a.dmod_stride + c + e, q2[e]);
+          if (a.dbias) atomicAdd(a.dbias + c + e, g4[e] * q3[e]);
+        }
+      }
+    }
+    seg0 = seg1;
+  }
+}
+
+template <int NV4, bool LN, bool GATE>
+int launch_ln_gate_rowcta_t(const LnGateBwd& a, cudaStream_t s) {
+  static int per_sm = 0;
+  if (!per_sm) {
+    JAGG_CUDA_TRY(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ln_gate_rowcta_kernel<NV4, LN, GATE>, 256, 0));
+    if (per_sm < 1) per_sm = 1;
+  }
+  // equal row shares of at least 8 rows per CTA, at most one wave of resident CTAs
+  const int cap = per_sm * sm_count();
+  const int want = ceil_div(a.M, 8);
+  ln_gate_rowcta_kernel<NV4, LN, GATE><<<want < cap ? want : cap, 256, 0, s>>>(a);
+  JAGG_LAUNCHED();
+  return JAGG_OK;
+}
+
+template <int NV4>
+int launch_ln_gate_rowcta(const LnGateBwd& a, cudaStream_t s) {
+  if (a.do_ln) return a.do_gate ? launch_ln_gate_rowcta_t<NV4, true, true>(a, s)
+                                : launch_ln_gate_rowcta_t<NV4, true, false>(a, s);
+  return launch_ln_gate_rowcta_t<NV4, false, true>(a, s);
+}
+
 template <int NV, bool GATE, bool YBF>
 int launch_ln_gate_rowreg_t(const LnGateBwd& a, cudaStream_t s) {
   const int smem = (8 * 4 + 2) * 128 * NV * (int)sizeof(float);
@@ -731,6 +885,175 @@ __global__ void __launch_bounds__(QKN_THREADS) qk_norm_rope_bwd_kernel(QkNormRop
   }
 }
 
+// Head dim 128 in bf16 (the Flux and Qwen widths): lane l owns the 4 consecutive elements
+// [4l, 4l + 4) of q and of k, i.e. the rotated pairs 2l and 2l + 1, so every operand moves
+// in 8-byte vectors and each lane's RMSNorm scales and RoPE frequencies are fixed for the
+// whole kernel.  The angles are the ones rope_angle forms (same expressions), so the forward
+// rotation and its inverse in the backward agree bit for bit.  Two (row, head) items per
+// warp iteration keep 2 KB of loads in flight per warp.
+constexpr int QKV_ITEMS = 2;
+
+__device__ __forceinline__ void bf16x4_load(const bf16* p, float (&v)[4]) {
+  const uint2 raw = *reinterpret_cast<const uint2*>(p);
+  const bf16* h = reinterpret_cast<const bf16*>(&raw);
+  v[0] = __bfloat162float(h[0]); v[1] = __bfloat162float(h[1]);
+  v[2] = __bfloat162float(h[2]); v[3] = __bfloat162float(h[3]);
+}
+__device__ __forceinline__ void bf16x4_store(bf16* p, const float (&v)[4]) {
+  __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]), b = __floats2bfloat162_rn(v[2], v[3]);
+  uint2 raw;
+  raw.x = *reinterpret_cast<uint32_t*>(&a);
+  raw.y = *reinterpret_cast<uint32_t*>(&b);
+  *reinterpret_cast<uint2*>(p) = raw;
+}
+// cos / sin of the lane's two pairs for token n (identity for text tokens)
+__device__ __forceinline__ void rope_lane(const QkNormRope& a, int n, int lane, float (&cs)[2], float (&sn)[2]) {
+#pragma unroll
+  for (int e = 0; e < 2; ++e) {
+    cs[e] = 1.f;
+    sn[e] = 0.f;
+    if (a.rope) rope_angle(n, a.n_txt, a.gw, 128, 2 * lane + e, cs[e], sn[e]);
+  }
+}
+
+__global__ void __launch_bounds__(QKN_THREADS) qk_norm_rope_fwd_v_kernel(QkNormRope a) {
+  const int lane = threadIdx.x & 31;
+  float scl[4][4];  // q txt, q img, k txt, k img: this lane's 4 elements
+  bf16x4_load(static_cast<const bf16*>(a.qscale_txt) + 4 * lane, scl[0]);
+  bf16x4_load(static_cast<const bf16*>(a.qscale_img) + 4 * lane, scl[1]);
+  bf16x4_load(static_cast<const bf16*>(a.kscale_txt) + 4 * lane, scl[2]);
+  bf16x4_load(static_cast<const bf16*>(a.kscale_img) + 4 * lane, scl[3]);
+  const int64_t items = (int64_t)a.M * a.heads;
+  const int64_t stride = (int64_t)gridDim.x * QKN_WARPS * QKV_ITEMS;
+  for (int64_t w0 = ((int64_t)blockIdx.x * QKN_WARPS + threadIdx.x / 32) * QKV_ITEMS; w0 < items; w0 += stride) {
+    float x[QKV_ITEMS][2][4];
+#pragma unroll
+    for (int it = 0; it < QKV_ITEMS; ++it) {
+      const int64_t w = w0 + it < items ? w0 + it : w0;
+      const int hd = (int)(w % a.heads), m = (int)(w / a.heads);
+#pragma unroll
+      for (int which = 0; which < 2; ++which)
+        bf16x4_load(static_cast<const bf16*>(a.qkv) + (int64_t)m * a.ld_qkv + which * a.d + hd * 128 + 4 * lane,
+                    x[it][which]);
+    }
+#pragma unroll
+    for (int it = 0; it < QKV_ITEMS; ++it) {
+      const int64_t w = w0 + it;
+      if (w >= items) break;
+      const int hd = (int)(w % a.heads), m = (int)(w / a.heads);
+      const int n = m % a.N;
+      const bool txt = n < a.n_txt;
+      float cs[2], sn[2];
+      rope_lane(a, n, lane, cs, sn);
+#pragma unroll
+      for (int which = 0; which < 2; ++which) {
+        float sc[4];  // selected per element: the array index stays a compile-time constant
+#pragma unroll
+        for (int e = 0; e < 4; ++e) sc[e] = txt ? scl[which * 2][e] : scl[which * 2 + 1][e];
+        const float* xv = x[it][which];
+        const float r = rsqrtf(warp_sum(xv[0] * xv[0] + xv[1] * xv[1] + xv[2] * xv[2] + xv[3] * xv[3]) / 128.f +
+                               1e-6f);
+        float o[4];
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const float y0 = xv[2 * e] * r * sc[2 * e], y1 = xv[2 * e + 1] * r * sc[2 * e + 1];
+          o[2 * e] = y0 * cs[e] - y1 * sn[e];
+          o[2 * e + 1] = y0 * sn[e] + y1 * cs[e];
+        }
+        bf16x4_store(static_cast<bf16*>(a.qk_out) + (int64_t)m * 2 * a.d + which * a.d + hd * 128 + 4 * lane, o);
+        if (lane == 0) (which == 0 ? a.rq : a.rk)[(int64_t)m * a.heads + hd] = r;
+      }
+    }
+  }
+}
+
+__global__ void __launch_bounds__(QKN_THREADS) qk_norm_rope_bwd_v_kernel(QkNormRopeBwd b) {
+  const QkNormRope& a = b.f;
+  __shared__ float part[QKN_WARPS][4][128];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x / 32;
+  float scl[4][4];  // q txt, q img, k txt, k img: this lane's 4 elements
+  bf16x4_load(static_cast<const bf16*>(a.qscale_txt) + 4 * lane, scl[0]);
+  bf16x4_load(static_cast<const bf16*>(a.qscale_img) + 4 * lane, scl[1]);
+  bf16x4_load(static_cast<const bf16*>(a.kscale_txt) + 4 * lane, scl[2]);
+  bf16x4_load(static_cast<const bf16*>(a.kscale_img) + 4 * lane, scl[3]);
+  float acc[4][4];  // scale gradients, [which * 2 + stream][element]
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) acc[i][e] = 0.f;
+  const int64_t items = (int64_t)a.M * a.heads;
+  const int64_t stride = (int64_t)gridDim.x * QKN_WARPS * QKV_ITEMS;
+  for (int64_t w0 = ((int64_t)blockIdx.x * QKN_WARPS + warp) * QKV_ITEMS; w0 < items; w0 += stride) {
+    float x[QKV_ITEMS][2][4], g[QKV_ITEMS][2][4];
+#pragma unroll
+    for (int it = 0; it < QKV_ITEMS; ++it) {
+      const int64_t w = w0 + it < items ? w0 + it : w0;
+      const int hd = (int)(w % a.heads), m = (int)(w / a.heads);
+#pragma unroll
+      for (int which = 0; which < 2; ++which) {
+        bf16x4_load(static_cast<const bf16*>(a.qkv) + (int64_t)m * a.ld_qkv + which * a.d + hd * 128 + 4 * lane,
+                    x[it][which]);
+        bf16x4_load(static_cast<const bf16*>(b.dqk) + (int64_t)m * b.ld_dqk + which * a.d + hd * 128 + 4 * lane,
+                    g[it][which]);
+      }
+    }
+#pragma unroll
+    for (int it = 0; it < QKV_ITEMS; ++it) {
+      const int64_t w = w0 + it;
+      if (w >= items) break;
+      const int hd = (int)(w % a.heads), m = (int)(w / a.heads);
+      const int n = m % a.N;
+      const bool txt = n < a.n_txt;
+      float cs[2], sn[2];
+      rope_lane(a, n, lane, cs, sn);
+#pragma unroll
+      for (int which = 0; which < 2; ++which) {
+        float sc[4];  // selected per element: the array index stays a compile-time constant
+#pragma unroll
+        for (int e = 0; e < 4; ++e) sc[e] = txt ? scl[which * 2][e] : scl[which * 2 + 1][e];
+        const float* xv = x[it][which];
+        const float r = (which == 0 ? a.rq : a.rk)[(int64_t)m * a.heads + hd];
+        float u[4], dy[4];
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {  // undo the rotation of the incoming gradient
+          const float g0 = g[it][which][2 * e], g1 = g[it][which][2 * e + 1];
+          dy[2 * e] = g0 * cs[e] + g1 * sn[e];
+          dy[2 * e + 1] = -g0 * sn[e] + g1 * cs[e];
+        }
+        float xu = 0.f;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float ds = dy[e] * xv[e] * r;
+          if (txt)
+            acc[which * 2][e] += ds;
+          else
+            acc[which * 2 + 1][e] += ds;
+          u[e] = dy[e] * sc[e];
+          xu += xv[e] * u[e];
+        }
+        xu = warp_sum(xu);
+        float dx[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) dx[e] = r * u[e] - xv[e] * r * r * r * xu / 128.f;
+        bf16x4_store(static_cast<bf16*>(b.dqk) + (int64_t)m * b.ld_dqk + which * a.d + hd * 128 + 4 * lane, dx);
+      }
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) part[warp][i][4 * lane + e] = acc[i][e];
+  __syncthreads();
+  for (int t = threadIdx.x; t < 4 * 128; t += QKN_THREADS) {
+    const int i = t / 128, c = t % 128;
+    float s = 0.f;
+#pragma unroll
+    for (int w = 0; w < QKN_WARPS; ++w) s += part[w][i][c];
+    float* dst = i == 0 ? b.dqs_txt : i == 1 ? b.dqs_img : i == 2 ? b.dks_txt : b.dks_img;
+    if (s != 0.f) atomicAdd(dst + c, s);
+  }
+}
+
 }  // namespace
 
 // ------------------------------------------------------------------ launchers
@@ -802,7 +1125,10 @@ int launch_ln_gate_bwd(const LnGateBwd& a, cudaStream_t s) {
     case 6: st = launch_ln_gate_rowreg<6>(a, smem, s); break;
     case 8: st = launch_ln_gate_nv<8>(a, smem, s); break;
     case 12: st = launch_ln_gate_nv<12>(a, smem, s); break;
-    case 24: st = launch_ln_gate_nv<24>(a, smem, s); break;
+    case 24:
+      st = (!a.do_ln || a.dm_f32) && a.dtype == JAGG_DTYPE_BF16 ? launch_ln_gate_rowcta<3>(a, s)
+                                                                  : launch_ln_gate_nv<24>(a, smem, s);
+      break;
     default: st = launch_ln_gate_nv<0>(a, smem, s); break;
   }
   JAGG_TRY(st);
@@ -862,13 +1188,26 @@ int launch_attn_rowdot(const void* dO, const void* O, int64_t ld, float* Dv, int
   JAGG_LAUNCHED();
   return JAGG_OK;
 }
+// The vectorised kernels serve head dim 128 in bf16 with 8-byte aligned rows and scales.
+static bool aligned8(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 7) == 0; }
+static bool qkn_vector(const QkNormRope& a) {
+  return a.dtype == JAGG_DTYPE_BF16 && a.heads > 0 && a.d == 128 * a.heads && a.ld_qkv % 4 == 0 &&
+         aligned8(a.qkv) && aligned8(a.qk_out) && aligned8(a.qscale_txt) && aligned8(a.qscale_img) &&
+         aligned8(a.kscale_txt) && aligned8(a.kscale_img);
+}
 int launch_qk_norm_rope_fwd(const QkNormRope& a, cudaStream_t s) {
   JAGG_CHECK_ARG(a.heads > 0 && a.d % a.heads == 0 && a.d / a.heads <= 128 && (a.d / a.heads) % 2 == 0,
                  "qk_norm: head dim unsupported");
   if (a.M <= 0) return JAGG_OK;
   const int64_t blocks = ((int64_t)a.M * a.heads + QKN_WARPS - 1) / QKN_WARPS;
   const int tok = prof_start(s);
-  qk_norm_rope_fwd_kernel<<<(int)(blocks < 65536 ? blocks : 65536), QKN_THREADS, 0, s>>>(a);
+  if (qkn_vector(a)) {
+    const int64_t vb = ceil_div((int64_t)a.M * a.heads, (int64_t)QKN_WARPS * QKV_ITEMS);
+    const int cap = 16 * sm_count();
+    qk_norm_rope_fwd_v_kernel<<<(int)(vb < cap ? vb : cap), QKN_THREADS, 0, s>>>(a);
+  } else {
+    qk_norm_rope_fwd_kernel<<<(int)(blocks < 65536 ? blocks : 65536), QKN_THREADS, 0, s>>>(a);
+  }
   JAGG_LAUNCHED();
   // algorithmic bytes: raw q, k read, transformed q, k written (storage type), 1/rms of both
   const double esz = a.dtype == JAGG_DTYPE_F32 ? 4.0 : 2.0;
@@ -885,7 +1224,14 @@ int launch_qk_norm_rope_bwd(const QkNormRopeBwd& a, cudaStream_t s) {
   const int64_t blocks = ((int64_t)f.M * f.heads + QKN_WARPS - 1) / QKN_WARPS;
   const int cap = 4 * sm_count();
   const int tok = prof_start(s);
-  qk_norm_rope_bwd_kernel<<<(int)(blocks < cap ? blocks : cap), QKN_THREADS, 0, s>>>(a);
+  if (qkn_vector(f) && a.ld_dqk % 4 == 0 && aligned8(a.dqk)) {
+    // a few blocks per SM: each block ends in 4 x 128 scale-gradient atomics
+    const int64_t vb = ceil_div((int64_t)f.M * f.heads, (int64_t)QKN_WARPS * QKV_ITEMS);
+    const int vcap = 8 * sm_count();
+    qk_norm_rope_bwd_v_kernel<<<(int)(vb < vcap ? vb : vcap), QKN_THREADS, 0, s>>>(a);
+  } else {
+    qk_norm_rope_bwd_kernel<<<(int)(blocks < cap ? blocks : cap), QKN_THREADS, 0, s>>>(a);
+  }
   JAGG_LAUNCHED();
   // algorithmic bytes: dq, dk read and rewritten in place, raw q, k read (storage type), 1/rms
   const double esz = f.dtype == JAGG_DTYPE_F32 ? 4.0 : 2.0;

@@ -1,6 +1,7 @@
 // Kernel-level entry points for the library's tests (include/jagg_testing.h).
 #include "../../include/jagg_testing.h"
 #include "attention.cuh"
+#include "elementwise.cuh"
 #include "gemm.cuh"
 #include "ptx.cuh"
 
@@ -138,4 +139,25 @@ extern "C" int jagg_test_attention_bwd_streams(const void* qkv0, const void* qkv
   ab.dq_col0 = 0; ab.dk_col0 = d; ab.dv_col0 = 2 * d;
   ab.impl = impl;
   return attention_bwd(ab, stream);
+}
+
+extern "C" int jagg_test_ln_gate_bwd(int M, int d, int rows_per_seq, int do_ln, int do_gate, const float* dm,
+                                     const float* h, const float* mean, const float* rstd, const float* scale,
+                                     float* dshift, float* dscale, const float* dh_in, float* dh_out, const void* y,
+                                     const float* gate, float* dgate, void* dy, float* dbias, int dtype,
+                                     cudaStream_t stream) {
+  JAGG_CHECK_ARG(M > 0 && rows_per_seq > 0, "jagg_test_ln_gate_bwd: M=%d rows_per_seq=%d", M, rows_per_seq);
+  JAGG_CHECK_ARG(dtype == JAGG_DTYPE_F32 || dtype == JAGG_DTYPE_BF16, "jagg_test_ln_gate_bwd: bad dtype");
+  JAGG_CHECK_ARG(!do_ln || (dm && h && mean && rstd && scale && dshift && dscale && dh_out),
+                 "jagg_test_ln_gate_bwd: null LayerNorm operand");
+  JAGG_CHECK_ARG(!do_gate || (y && gate && dgate && dy), "jagg_test_ln_gate_bwd: null gate operand");
+  JAGG_CHECK_ARG(dh_in, "jagg_test_ln_gate_bwd: null dh_in");
+  LnGateBwd a{};
+  a.M = M; a.d = d; a.rows_per_seq = rows_per_seq;
+  a.do_ln = do_ln; a.dm = dm; a.dm_f32 = 1; a.h = h; a.mean = mean; a.rstd = rstd;
+  a.scale = scale; a.mod_stride = d; a.dshift = dshift; a.dscale = dscale; a.dmod_stride = d;
+  a.dh_in = dh_in; a.dh_out = dh_out;
+  a.do_gate = do_gate; a.y = y; a.gate = gate; a.dgate = dgate; a.dy = dy; a.dbias = dbias;
+  a.dtype = dtype;
+  return launch_ln_gate_bwd(a, stream);
 }

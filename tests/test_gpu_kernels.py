@@ -398,3 +398,58 @@ def test_bounded_wait_gives_up_and_reports_timeout(limit_ns):
     assert jg.device_status() == 0
     x = torch.randn(256, 256, device="cuda")
     assert torch.isfinite(x @ x).all()      # the context still works
+
+
+@pytest.mark.parametrize("d,M,rps,ln,gate,dtype", [
+    (3072, 4608 * 2, 4608, True, True, torch.bfloat16),   # Flux single block: row-per-CTA kernel
+    (3072, 512 * 3, 512, True, False, torch.bfloat16),    # LayerNorm only
+    (3072, 1024 * 2 + 0, 1024, False, True, torch.bfloat16),  # gate only
+    (3072, 333 * 3, 333, True, True, torch.bfloat16),     # sequences that straddle CTA row shares
+    (3072, 40, 8, True, True, torch.float32),             # f32 y: the persistent kernel
+    (768, 333 * 4, 333, True, True, torch.bfloat16),      # DiT-B width: row-in-registers kernel
+    (1024, 300, 100, True, True, torch.bfloat16),
+    (64, 24 * 4, 24, True, True, torch.float32)])
+def test_ln_gate_backward_kernels(d, M, rps, ln, gate, dtype):
+    """LayerNorm + modulation backward fused with the gate backward (every kernel variant the
+    dispatcher picks: row per CTA at d = 3072, row in registers up to 768, the persistent
+    kernel otherwise) against PyTorch fp32 on the same inputs, including the per-sequence
+    column sums (dshift, dscale, dgate) and the bias gradient."""
+    torch.manual_seed(d + M)
+    dev = "cuda"
+    S = M // rps
+    f = dict(device=dev, dtype=torch.float32)
+    h = torch.randn(M, d, **f) * 2 + 0.5
+    mean, rstd = h.mean(1), torch.rsqrt(h.var(1, unbiased=False) + 1e-6)
+    dm = torch.randn(M, d, **f)
+    scale = torch.randn(S, d, **f) * 0.3
+    gate_v = torch.randn(S, d, **f)
+    y = torch.randn(M, d, **f).to(dtype)
+    dh_in = torch.randn(M, d, **f)
+    dh_out = torch.empty_like(dh_in) if ln else None
+    dshift, dscale, dgate = (torch.full((S, d), 0.25, **f) for _ in range(3))
+    dbias = torch.full((d,), -0.5, **f)
+    dy = torch.empty(M, d, device=dev, dtype=dtype)
+    kw = {}
+    if ln:
+        kw.update(dm=dm, h=h, mean=mean, rstd=rstd, scale=scale, dshift=dshift, dscale=dscale)
+    if gate:
+        kw.update(y=y, gate=gate_v, dgate=dgate, dy=dy, dbias=dbias)
+    jg.test_ln_gate_bwd(M, d, rps, dh_in, dh_out, **kw)
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    seq = torch.arange(M, device=dev) // rps
+    xh = (h - mean[:, None]) * rstd[:, None]
+    if ln:
+        e = dm * (1 + scale[seq])
+        dh_ref = dh_in + rstd[:, None] * (e - e.mean(1, keepdim=True) - xh * (e * xh).mean(1, keepdim=True))
+        assert _rel(dh_out, dh_ref) < 1e-5
+        assert _rel(dshift - 0.25, torch.zeros(S, d, **f).index_add_(0, seq, dm)) < 1e-5
+        assert _rel(dscale - 0.25, torch.zeros(S, d, **f).index_add_(0, seq, dm * xh)) < 1e-5
+    else:
+        dh_ref = dh_in
+    if gate:
+        yf = y.float()
+        assert _rel(dy.float(), gate_v[seq] * dh_ref) < (1e-2 if dtype == torch.bfloat16 else 1e-6)
+        assert _rel(dgate - 0.25, torch.zeros(S, d, **f).index_add_(0, seq, dh_ref * yf)) < 1e-5
+        sums = torch.zeros(S, d, **f).index_add_(0, seq, dh_ref)
+        assert _rel(dbias + 0.5, (gate_v * sums).sum(0)) < 1e-5
