@@ -538,6 +538,448 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
   }
 }
 
+// ================================================================== backward, head dim 128
+// 128-key x 64-query tiles with S^T and dP^T double-buffered in tensor memory.  One CTA per
+// SM, persistent over (128-key tile, sequence, head) units; per unit the sequence's query
+// tiles stream through three Q / dO stages.  Tensor memory (512 columns), buffer b = tile % 2:
+//   S_b   [128 b, 128 b + 64)        S^T (f32); P^T written over it (bf16, two per column)
+//   dP_b  [128 b + 64, 128 b + 128)  dP^T (f32); dS^T written over it; then dQ^T (f32)
+//   [256, 384) dV, [384, 512) dK     accumulated over the whole sequence
+// Products of tile g (buffer b), in issue order (one thread; the tensor pipe runs them in
+// order):
+//   dV += P^T dO, dK += dS^T Q        A from tensor memory, B (dO, Q) from shared memory
+//   dQ^T = K^T dS^T                   both from shared memory (dS^T in a double-buffered
+//                                     shared tile); over dS^T in dP_b
+//   S^T(g+2) = K Q^T                  over P^T(g) in S_b
+//   dP^T(g+2) = V dO^T                once the dQ warps have read dQ^T(g) out of dP_b
+// The 8 P / dS warps form P^T of tile g+1 as soon as its S^T lands and dS^T once its dP^T
+// lands, while the products of tile g run; each writes only over the f32 columns it has read
+// (32 keys x 32 queries per warp), so no warp waits for another and nothing waits for a
+// product to release a shared P / dS tile.  The 4 dQ warps move dQ^T through shared memory
+// into TMA f32 reduce-adds and store each unit's dK, dV at its end.
+constexpr int FB2_THREADS = 448;  // 14 warps
+
+struct Fb2 {
+  static constexpr int D = 128, BK = 128, BQ = 64, NS = 3;
+  static constexpr int KV_BYTES = BK * D * 2;  // 32 KB: two 64-column chunks
+  static constexpr int QT_BYTES = BQ * D * 2;  // 16 KB
+  static constexpr int DS_BYTES = BK * BQ * 2; // 16 KB
+  static constexpr int DQ_WARP_BYTES = 32 * 32 * 4;
+  static constexpr int OFF_K = 0;
+  static constexpr int OFF_V = OFF_K + KV_BYTES;
+  static constexpr int OFF_Q = OFF_V + KV_BYTES;         // NS stages
+  static constexpr int OFF_DO = OFF_Q + NS * QT_BYTES;   // NS stages
+  static constexpr int OFF_DS = OFF_DO + NS * QT_BYTES;  // 2 buffers
+  static constexpr int OFF_DQ = OFF_DS + 2 * DS_BYTES;
+  static constexpr int OFF_LSE = OFF_DQ + 4 * DQ_WARP_BYTES;
+  static constexpr int OFF_RD = OFF_LSE + NS * BQ * 4;
+  static constexpr int OFF_BAR = OFF_RD + NS * BQ * 4;
+  static constexpr int NBAR = 24;
+  static constexpr int SMEM = OFF_BAR + NBAR * 8 + 16 + 1024;  // + alignment of the base to 1024 bytes
+  static_assert(SMEM <= 232448, "shared memory budget");
+  __host__ __device__ static constexpr uint32_t t_s(int b) { return 128u * b; }
+  __host__ __device__ static constexpr uint32_t t_dp(int b) { return 128u * b + 64u; }
+  static constexpr uint32_t T_DV = 256, T_DK = 384;
+};
+
+__global__ void __launch_bounds__(FB2_THREADS, 1) fa_bwd_tc128_kernel(const __grid_constant__ FbMaps maps,
+                                                                      FbParams p) {
+  using C = Fb2;
+  constexpr int BK = C::BK, BQ = C::BQ, D = C::D, NS = C::NS;
+  extern __shared__ uint8_t smem_fb2[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_fb2) + 1023) & ~uintptr_t(1023));
+  uint8_t* sK = sm + C::OFF_K;
+  uint8_t* sV = sm + C::OFF_V;
+  uint8_t* sQ = sm + C::OFF_Q;
+  uint8_t* sdO = sm + C::OFF_DO;
+  uint8_t* sdS = sm + C::OFF_DS;
+  uint8_t* sDQ = sm + C::OFF_DQ;
+  float* sLse = reinterpret_cast<float*>(sm + C::OFF_LSE);
+  float* sRd = reinterpret_cast<float*>(sm + C::OFF_RD);
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sm + C::OFF_BAR);
+  uint64_t* full = bar;              // [NS] Q, dO, lse, rowsum(dO O) of a stage landed
+  uint64_t* empty = bar + NS;        // [NS] the stage's products are done
+  uint64_t* bar_s = bar + 2 * NS;    // [2] S^T of a tile in S_b
+  uint64_t* bar_dp = bar_s + 2;      // [2] dP^T of a tile in dP_b
+  uint64_t* bar_p = bar_s + 4;       // [2] P^T written (8 warps)
+  uint64_t* bar_ds = bar_s + 6;      // [2] dS^T written to TMEM and shared memory (8 warps)
+  uint64_t* bar_dq = bar_s + 8;      // [2] dQ^T of a tile in dP_b
+  uint64_t* dqfree = bar_s + 10;     // [2] the dQ warps have read it (4 warps)
+  uint64_t* bar_kv = bar_s + 12;     // a unit's K, V landed
+  uint64_t* kv_free = bar_s + 13;    // a unit's products are done (K, V reusable)
+  uint64_t* bar_fin = bar_s + 14;    // a unit's dK, dV are final
+  uint64_t* kvout = bar_s + 15;      // the dQ warps have read them (4 warps)
+  uint64_t* bar_drain = bar_s + 16;  // the MMA thread's drain after a give-up
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar + C::NBAR);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int N = p.N;
+  const int nkt = (N + BK - 1) / BK;
+  const int units = nkt * p.B * p.heads;
+  const int nq = (N + BQ - 1) / BQ;
+  // unit u: key tile u % nkt of sequence-head u / nkt
+  auto unit_of = [&](int u, int& k0, int& b, int& h) {
+    const int bh = u / nkt;
+    k0 = (u % nkt) * BK;
+    b = bh / p.heads;
+    h = bh % p.heads;
+  };
+  auto seg_of = [&](int r) { return r < p.n0 ? 0 : 1; };
+  auto row_in = [&](int r) { return r < p.n0 ? r : r - p.n0; };
+
+  if (threadIdx.x == 0) {
+    *abort_flag = 0;
+    for (int i = 0; i < NS; ++i) {
+      ptx::mbar_init(&full[i], 1 + 32);  // the TMA's expect-tx arrival + one per producer lane's copies
+      ptx::mbar_init(&empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      ptx::mbar_init(&bar_s[i], 1);
+      ptx::mbar_init(&bar_dp[i], 1);
+      ptx::mbar_init(&bar_p[i], 8);
+      ptx::mbar_init(&bar_ds[i], 8);
+      ptx::mbar_init(&bar_dq[i], 1);
+      ptx::mbar_init(&dqfree[i], 4);
+    }
+    ptx::mbar_init(bar_kv, 1);
+    ptx::mbar_init(kv_free, 1);
+    ptx::mbar_init(bar_fin, 1);
+    ptx::mbar_init(kvout, 4);
+    ptx::mbar_init(bar_drain, 1);
+    ptx::fence_mbar_init();
+    for (int sg = 0; sg < 2; ++sg) {
+      ptx::prefetch_tmap(&maps.q[sg]);
+      ptx::prefetch_tmap(&maps.k[sg]);
+      ptx::prefetch_tmap(&maps.v[sg]);
+      ptx::prefetch_tmap(&maps.dO[sg]);
+    }
+    ptx::prefetch_tmap(&maps.dq);
+  }
+  if (warp == 1) {
+    ptx::tmem_alloc(tmem_slot, 512);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    int i = 0;
+    int i_last = -1, g_last = -1;  // the last unit whose K, V and the last tile whose Q, dO were issued
+    for (int u = blockIdx.x; u < units && !*abort_flag; u += gridDim.x, ++i) {
+      int k0, b, h;
+      unit_of(u, k0, b, h);
+      const int bh = b * p.heads + h;
+      bool ok = true;
+      if (lane == 0) {
+        ok = ptx::mbar_wait(kv_free, (i & 1) ^ 1);
+        if (ok) {
+          const int sg = seg_of(k0), r = row_in(k0);
+          ptx::mbar_arrive_expect_tx(bar_kv, 2 * C::KV_BYTES);
+#pragma unroll
+          for (int c = 0; c < D / 64; ++c) {
+            ptx::tma_load_3d(sK + c * BK * 128, &maps.k[sg], bar_kv, (int)(p.k_col0 + h * D + c * 64), r, b);
+            ptx::tma_load_3d(sV + c * BK * 128, &maps.v[sg], bar_kv, (int)(p.v_col0 + h * D + c * 64), r, b);
+          }
+          i_last = i;
+        }
+      }
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      if (!ok) { *abort_flag = 1; break; }
+      for (int j = 0; j < nq; ++j) {
+        const int g = i * nq + j;
+        const int st = g % NS;
+        if (lane == 0) ok = ptx::mbar_wait(&empty[st], ((g / NS) & 1) ^ 1);
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        if (!ok || *abort_flag) { *abort_flag = 1; break; }
+        const int q0 = j * BQ;
+        // lse and rowsum(dO O) of the tile's queries by 4-byte copies the stage barrier tracks
+        // (their rows need not be 16-byte aligned); +inf / 0 past the last query
+        for (int t = lane; t < BQ; t += 32) {
+          const int q = q0 + t;
+          if (q < N) {
+            ptx::cp_async4(sLse + st * BQ + t, p.lse + (int64_t)bh * N + q);
+            ptx::cp_async4(sRd + st * BQ + t, p.Dv + (int64_t)bh * N + q);
+          } else {
+            sLse[st * BQ + t] = INFINITY;
+            sRd[st * BQ + t] = 0.f;
+          }
+        }
+        ptx::cp_async_arrive_noinc(&full[st]);
+        __syncwarp();
+        if (lane == 0) {
+          const int sg = seg_of(q0), r = row_in(q0);
+          ptx::mbar_arrive_expect_tx(&full[st], 2 * C::QT_BYTES);
+#pragma unroll
+          for (int c = 0; c < D / 64; ++c) {
+            ptx::tma_load_3d(sQ + st * C::QT_BYTES + c * BQ * 128, &maps.q[sg], &full[st],
+                             (int)(p.q_col0 + h * D + c * 64), r, b);
+            ptx::tma_load_3d(sdO + st * C::QT_BYTES + c * BQ * 128, &maps.dO[sg], &full[st], h * D + c * 64, r,
+                             b);
+          }
+        }
+        g_last = g;
+      }
+      if (*abort_flag) break;
+    }
+    // After a give-up anywhere in the CTA, copies already issued may still be landing in
+    // shared memory: wait (bounded) for the last phase of every buffer before exiting.
+    if (*abort_flag && lane == 0) {
+      if (i_last >= 0) ptx::mbar_wait(bar_kv, i_last & 1);
+      for (int k = 0; k < NS && g_last - k >= 0; ++k)
+        ptx::mbar_wait(&full[(g_last - k) % NS], ((g_last - k) / NS) & 1);
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (ptx::elect_one()) {
+      constexpr uint32_t id_s = ptx::idesc_bf16(128, BQ, false, false);  // S^T, dP^T
+      constexpr uint32_t id_acc = ptx::idesc_bf16(128, D, false, true);  // dV, dK (A from TMEM)
+      constexpr uint32_t id_dq = ptx::idesc_bf16(128, BQ, true, true);   // dQ^T
+      const uint32_t aK = ptx::smem_u32(sK), aV = ptx::smem_u32(sV);
+      auto issue_s = [&](int g) {  // S^T = K Q^T into S_b
+        const uint32_t aQ = ptx::smem_u32(sQ + (g % NS) * C::QT_BYTES);
+#pragma unroll
+        for (int k = 0; k < D / 16; ++k)
+          ptx::umma_bf16(tmem + C::t_s(g & 1), kmajor_desc(aK, BK, k), kmajor_desc(aQ, BQ, k), id_s, k > 0);
+        ptx::umma_commit(&bar_s[g & 1]);
+      };
+      auto issue_dp = [&](int g) {  // dP^T = V dO^T into dP_b
+        const uint32_t adO = ptx::smem_u32(sdO + (g % NS) * C::QT_BYTES);
+#pragma unroll
+        for (int k = 0; k < D / 16; ++k)
+          ptx::umma_bf16(tmem + C::t_dp(g & 1), kmajor_desc(aV, BK, k), kmajor_desc(adO, BQ, k), id_s, k > 0);
+        ptx::umma_commit(&bar_dp[g & 1]);
+      };
+      bool ok = true;
+      int i = 0;
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++i) {
+        if (!ptx::mbar_wait(bar_kv, i & 1)) { ok = false; break; }
+        // the unit's first two tiles
+        for (int j = 0; j < 2 && j < nq && ok; ++j) {
+          const int g = i * nq + j;
+          if (!ptx::mbar_wait(&full[g % NS], (g / NS) & 1)) { ok = false; break; }
+          ptx::tc_fence_after();
+          issue_s(g);
+          // dP_b held dQ^T of the buffer's previous tile (an earlier unit's): drained
+          if (g >= 2 && !ptx::mbar_wait(&dqfree[g & 1], ((g - 2) >> 1) & 1)) { ok = false; break; }
+          ptx::tc_fence_after();
+          issue_dp(g);
+        }
+        for (int j = 0; j < nq && ok; ++j) {
+          const int g = i * nq + j;
+          const int st = g % NS, bb = g & 1;
+          const uint32_t aQ = ptx::smem_u32(sQ + st * C::QT_BYTES), adO = ptx::smem_u32(sdO + st * C::QT_BYTES);
+          const uint32_t adS = ptx::smem_u32(sdS + bb * C::DS_BYTES);
+          if (!ptx::mbar_wait(&bar_p[bb], (g >> 1) & 1)) { ok = false; break; }
+          ptx::tc_fence_after();
+          // the first dV, dK products of a unit overwrite the accumulators: the dQ warps have
+          // read the previous unit's
+          if (j == 0 && i > 0) {
+            if (!ptx::mbar_wait(kvout, (i - 1) & 1)) { ok = false; break; }
+            ptx::tc_fence_after();
+          }
+          // P^T of queries [32 hf, 32 hf + 32) sits in columns S_b + 32 hf + [0, 16)
+#pragma unroll
+          for (int k = 0; k < BQ / 16; ++k)
+            ptx::umma_bf16_ts(tmem + C::T_DV, tmem + C::t_s(bb) + (k >> 1) * 32 + (k & 1) * 8,
+                              mnmajor_desc(adO, BQ * 128, k), id_acc, (j > 0 || k > 0) ? 1u : 0u);
+          if (!ptx::mbar_wait(&bar_ds[bb], (g >> 1) & 1)) { ok = false; break; }
+          ptx::tc_fence_after();
+#pragma unroll
+          for (int k = 0; k < BQ / 16; ++k)
+            ptx::umma_bf16_ts(tmem + C::T_DK, tmem + C::t_dp(bb) + (k >> 1) * 32 + (k & 1) * 8,
+                              mnmajor_desc(aQ, BQ * 128, k), id_acc, (j > 0 || k > 0) ? 1u : 0u);
+          ptx::umma_commit(&empty[st]);
+          // dQ^T[d][q] = sum_key K[key][d] dS^T[key][q], over dS^T in dP_b
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            ptx::umma_bf16(tmem + C::t_dp(bb), mnmajor_desc(aK, BK * 128, k), mnmajor_desc(adS, BK * 128, k),
+                           id_dq, k > 0);
+          ptx::umma_commit(&bar_dq[bb]);
+          if (j + 2 < nq) {
+            const int g2 = g + 2;
+            if (!ptx::mbar_wait(&full[g2 % NS], (g2 / NS) & 1)) { ok = false; break; }
+            ptx::tc_fence_after();
+            issue_s(g2);
+            if (!ptx::mbar_wait(&dqfree[bb], (g >> 1) & 1)) { ok = false; break; }
+            ptx::tc_fence_after();
+            issue_dp(g2);
+          }
+        }
+        ptx::umma_commit(kv_free);
+        ptx::umma_commit(bar_fin);
+      }
+      if (!ok) *abort_flag = 1;
+      if (*abort_flag) {  // MMAs of this thread may still run: drain them before TMEM is freed
+        ptx::umma_commit(bar_drain);
+        ptx::mbar_wait(bar_drain, 0);
+      }
+    }
+  } else if (warp < 10) {
+    // ---------------------------------------------------------------- P / dS
+    const int quarter = warp & 3, hf = (warp - 2) >> 2;
+    const int r = quarter * 32 + lane;  // key row of the tile = TMEM lane
+    const int c0 = hf * 32;             // this warp's query columns
+    const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
+    const float c1 = p.scale * kLog2eTc;
+    bool ok = true;
+    int i = 0;
+    for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++i) {
+      for (int j = 0; j < nq; ++j) {
+        const int g = i * nq + j;
+        const int st = g % NS, bb = g & 1;
+        ok = ptx::mbar_wait(&bar_s[bb], (g >> 1) & 1) && ptx::mbar_wait(&full[st], (g / NS) & 1);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok || *abort_flag) { ok = false; *abort_flag = 1; break; }
+        ptx::tc_fence_after();
+        const float* lse = sLse + st * BQ + c0;
+        const float* rd = sRd + st * BQ + c0;
+        uint32_t hp[16];  // P^T of this thread's 32 queries, bf16 pairs
+        {
+          uint32_t rs[32];
+          ptx::tmem_ld_32x32b_x32(trow + C::t_s(bb) + c0, rs);
+          ptx::tmem_ld_wait();
+#pragma unroll
+          for (int e = 0; e < 32; e += 4) {
+            const float4 l4 = *reinterpret_cast<const float4*>(lse + e);
+            const float p0 = ptx::ex2_approx(fmaf(__uint_as_float(rs[e]), c1, -l4.x * kLog2eTc));
+            const float p1 = ptx::ex2_approx(fmaf(__uint_as_float(rs[e + 1]), c1, -l4.y * kLog2eTc));
+            const float p2 = ptx::ex2_approx(fmaf(__uint_as_float(rs[e + 2]), c1, -l4.z * kLog2eTc));
+            const float p3 = ptx::ex2_approx(fmaf(__uint_as_float(rs[e + 3]), c1, -l4.w * kLog2eTc));
+            hp[e / 2] = pack2_bf16(p0, p1);
+            hp[e / 2 + 1] = pack2_bf16(p2, p3);
+          }
+        }
+        // over this warp's own S^T columns, read already
+        ptx::tmem_st_32x32b_x16(trow + C::t_s(bb) + c0, hp);
+        ptx::tmem_st_wait();
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(&bar_p[bb]);
+        ok = __all_sync(0xffffffffu, ptx::mbar_wait(&bar_dp[bb], (g >> 1) & 1));
+        if (!ok || *abort_flag) { ok = false; *abort_flag = 1; break; }
+        ptx::tc_fence_after();
+        uint32_t hd[16];
+        {
+          uint32_t rp[32];
+          ptx::tmem_ld_32x32b_x32(trow + C::t_dp(bb) + c0, rp);
+          ptx::tmem_ld_wait();
+#pragma unroll
+          for (int e = 0; e < 32; e += 4) {
+            const float4 r4 = *reinterpret_cast<const float4*>(rd + e);
+            const uint32_t a = hp[e / 2], a2 = hp[e / 2 + 1];
+            hd[e / 2] = pack2_bf16(__uint_as_float(a << 16) * (__uint_as_float(rp[e]) - r4.x),
+                                   __uint_as_float(a & 0xffff0000u) * (__uint_as_float(rp[e + 1]) - r4.y));
+            hd[e / 2 + 1] = pack2_bf16(__uint_as_float(a2 << 16) * (__uint_as_float(rp[e + 2]) - r4.z),
+                                       __uint_as_float(a2 & 0xffff0000u) * (__uint_as_float(rp[e + 3]) - r4.w));
+          }
+        }
+        ptx::tmem_st_32x32b_x16(trow + C::t_dp(bb) + c0, hd);
+        // the B operand of dQ^T: row = key, columns = queries (the product that read this
+        // buffer two tiles ago finished before this tile's dP^T)
+        st_row32_packed(sdS + bb * C::DS_BYTES, BK, r, c0, hd);
+        ptx::tmem_st_wait();
+        ptx::fence_proxy_async_smem();
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(&bar_ds[bb]);
+      }
+      if (!ok) break;
+    }
+  } else {
+    // ---------------------------------------------------------------- dQ -> f32 reduce-add; dK, dV
+    const int quarter = warp & 3;
+    const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
+    uint8_t* stg = sDQ + quarter * C::DQ_WARP_BYTES;
+    bool ok = true;
+    int i = 0;
+    for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++i) {
+      int k0, b, h;
+      unit_of(u, k0, b, h);
+      for (int j = 0; j < nq; ++j) {
+        const int g = i * nq + j;
+        const int bb = g & 1;
+        ok = __all_sync(0xffffffffu, ptx::mbar_wait(&bar_dq[bb], (g >> 1) & 1));
+        if (!ok || *abort_flag) { ok = false; *abort_flag = 1; break; }
+        ptx::tc_fence_after();
+        uint32_t rq[64];
+        ptx::tmem_ld_32x32b_x32(trow + C::t_dp(bb), *reinterpret_cast<uint32_t(*)[32]>(rq));
+        ptx::tmem_ld_32x32b_x32(trow + C::t_dp(bb) + 32, *reinterpret_cast<uint32_t(*)[32]>(rq + 32));
+        ptx::tmem_ld_wait();
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(&dqfree[bb]);
+        const int q0 = j * BQ;
+        // dQ^T: lane = head-dim index, columns = the tile's 64 queries; two 32 x 32 boxes
+        // (box rows = queries) through one staging box
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+          if (lane == 0) ptx::bulk_wait_read<0>();
+          __syncwarp();
+#pragma unroll
+          for (int q = 0; q < 32; ++q)
+            *reinterpret_cast<float*>(stg + q * 128 + (((lane >> 2) ^ (q & 7)) << 4) + (lane & 3) * 4) =
+                __uint_as_float(rq[hh * 32 + q]) * p.scale;
+          ptx::fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            const int row = q0 + hh * 32;
+            if (row < N) {
+              ptx::tma_reduce_add_3d(&maps.dq, stg, h * D + quarter * 32, row, b);
+              ptx::bulk_commit();
+            }
+          }
+        }
+      }
+      if (!ok) break;
+      // the unit's dK, dV (key rows of this warp's lane quarter)
+      ok = __all_sync(0xffffffffu, ptx::mbar_wait(bar_fin, i & 1));
+      if (!ok || *abort_flag) { ok = false; *abort_flag = 1; break; }
+      ptx::tc_fence_after();
+      const int key = k0 + quarter * 32 + lane;
+#pragma unroll 1
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t rv[32], rk[32];
+        ptx::tmem_ld_32x32b_x32(trow + C::T_DV + c * 32, rv);
+        ptx::tmem_ld_32x32b_x32(trow + C::T_DK + c * 32, rk);
+        ptx::tmem_ld_wait();
+        if (key < N) {
+          bf16* dv = static_cast<bf16*>(p.dv.base(key)) + p.dv.off(b, key, N, p.dv_col0 + h * D + c * 32);
+          bf16* dk = static_cast<bf16*>(p.dk.base(key)) + p.dk.off(b, key, N, p.dk_col0 + h * D + c * 32);
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            uint4 a, bb;
+            a.x = pack2_bf16(__uint_as_float(rv[8 * t]), __uint_as_float(rv[8 * t + 1]));
+            a.y = pack2_bf16(__uint_as_float(rv[8 * t + 2]), __uint_as_float(rv[8 * t + 3]));
+            a.z = pack2_bf16(__uint_as_float(rv[8 * t + 4]), __uint_as_float(rv[8 * t + 5]));
+            a.w = pack2_bf16(__uint_as_float(rv[8 * t + 6]), __uint_as_float(rv[8 * t + 7]));
+            bb.x = pack2_bf16(__uint_as_float(rk[8 * t]) * p.scale, __uint_as_float(rk[8 * t + 1]) * p.scale);
+            bb.y = pack2_bf16(__uint_as_float(rk[8 * t + 2]) * p.scale, __uint_as_float(rk[8 * t + 3]) * p.scale);
+            bb.z = pack2_bf16(__uint_as_float(rk[8 * t + 4]) * p.scale, __uint_as_float(rk[8 * t + 5]) * p.scale);
+            bb.w = pack2_bf16(__uint_as_float(rk[8 * t + 6]) * p.scale, __uint_as_float(rk[8 * t + 7]) * p.scale);
+            *reinterpret_cast<uint4*>(dv + 8 * t) = a;
+            *reinterpret_cast<uint4*>(dk + 8 * t) = bb;
+          }
+        }
+      }
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(kvout);
+    }
+    if (lane == 0) ptx::bulk_wait<0>();
+    __syncwarp();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, 512);
+  }
+}
+
 // ================================================================== forward
 // Persistent over (128-query tile, sequence, head) units, two passes over the sequence's
 // 128-key tiles per unit:
@@ -938,6 +1380,53 @@ int launch(const AttnBwdArgs& a, cudaStream_t s) {
   return JAGG_OK;
 }
 
+// The head-dim-128 backward (fa_bwd_tc128_kernel).
+int launch128(const AttnBwdArgs& a, cudaStream_t s) {
+  using C = Fb2;
+  const AttnArgs& f = a.f;
+  const int n0 = f.q.n0, N = f.N;
+  const int n1 = N - n0;
+  FbMaps maps;
+  for (int sg = 0; sg < 2; ++sg) {
+    const int nt = sg == 0 ? n0 : n1;
+    if (nt <= 0) {  // single stream: the second views are unused copies
+      maps.q[1] = maps.q[0];
+      maps.k[1] = maps.k[0];
+      maps.v[1] = maps.v[0];
+      maps.dO[1] = maps.dO[0];
+      break;
+    }
+    JAGG_TRY(seg_map(&maps.q[sg], sg ? f.q.p1 : f.q.p0, sg ? f.q.ld1 : f.q.ld0, nt, f.B, C::BQ));
+    JAGG_TRY(seg_map(&maps.k[sg], sg ? f.k.p1 : f.k.p0, sg ? f.k.ld1 : f.k.ld0, nt, f.B, C::BK));
+    JAGG_TRY(seg_map(&maps.v[sg], sg ? f.v.p1 : f.v.p0, sg ? f.v.ld1 : f.v.ld0, nt, f.B, C::BK));
+    JAGG_TRY(seg_map(&maps.dO[sg], sg ? a.dO.p1 : a.dO.p0, sg ? a.dO.ld1 : a.dO.ld0, nt, f.B, C::BQ));
+  }
+  {
+    const int64_t cols = (int64_t)f.heads * C::D;
+    const uint64_t dims[3] = {(uint64_t)cols, (uint64_t)N, (uint64_t)f.B};
+    const uint64_t strides[2] = {(uint64_t)cols * 4, (uint64_t)cols * 4 * N};
+    const uint32_t box[3] = {32, 32, 1};
+    JAGG_TRY(encode_tmap(&maps.dq, true, 3, a.dq_acc, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B));
+  }
+  FbParams p;
+  p.B = f.B; p.N = N; p.heads = f.heads; p.n0 = n0 > 0 && n0 < N ? n0 : N;
+  p.scale = f.scale;
+  p.q_col0 = f.q_col0; p.k_col0 = f.k_col0; p.v_col0 = f.v_col0;
+  p.dk_col0 = a.dk_col0; p.dv_col0 = a.dv_col0;
+  p.lse = f.lse; p.Dv = a.Dv;
+  p.dk = a.dk; p.dv = a.dv;
+  static bool attr = false;
+  if (!attr) {
+    JAGG_CUDA_TRY(cudaFuncSetAttribute(fa_bwd_tc128_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
+    attr = true;
+  }
+  const int units = ceil_div(N, C::BK) * f.B * f.heads;
+  const int nsm = sm_count();
+  fa_bwd_tc128_kernel<<<units < nsm ? units : nsm, FB2_THREADS, C::SMEM, s>>>(maps, p);
+  JAGG_LAUNCHED();
+  return JAGG_OK;
+}
+
 template <int D>
 int launch_fwd(const AttnArgs& f, cudaStream_t s) {
   using C = FfCfg<D>;
@@ -1016,7 +1505,7 @@ bool attention_bwd_tc_eligible(const AttnBwdArgs& a) {
 }
 
 int attention_bwd_tc(const AttnBwdArgs& a, cudaStream_t s) {
-  return a.f.dh == 64 ? launch<64>(a, s) : launch<128>(a, s);
+  return a.f.dh == 64 ? launch<64>(a, s) : launch128(a, s);
 }
 
 }  // namespace jagg

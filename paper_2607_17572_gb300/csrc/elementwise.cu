@@ -906,17 +906,42 @@ __device__ __forceinline__ void bf16x4_store(bf16* p, const float (&v)[4]) {
   raw.y = *reinterpret_cast<uint32_t*>(&b);
   *reinterpret_cast<uint2*>(p) = raw;
 }
-// cos / sin of the lane's two pairs for token n (identity for text tokens)
-__device__ __forceinline__ void rope_lane(const QkNormRope& a, int n, int lane, float (&cs)[2], float (&sn)[2]) {
-#pragma unroll
-  for (int e = 0; e < 2; ++e) {
-    cs[e] = 1.f;
-    sn[e] = 0.f;
-    if (a.rope) rope_angle(n, a.n_txt, a.gw, 128, 2 * lane + e, cs[e], sn[e]);
+// RoPE angles of head dim 128 as a table in shared memory, filled by each block: entry
+// [pos][i] = (cos, sin) of pos * theta_i for the 32 frequencies of one axis, pos below the
+// larger grid side; the values are rope_angle's (same expressions), so the forward rotation
+// and its inverse agree bit for bit.  QKN_TABLE_MAX bounds the grid side the table serves.
+constexpr int QKN_TABLE_MAX = 128;
+__device__ __forceinline__ int rope_table_side(const QkNormRope& a) {
+  const int gh = (a.N - a.n_txt) / a.gw;
+  return gh > a.gw ? gh : a.gw;
+}
+__device__ __forceinline__ void rope_table_fill(const QkNormRope& a, float2* tab) {
+  const int side = rope_table_side(a);
+  for (int t = threadIdx.x; t < side * 32; t += blockDim.x) {
+    const int pos = t / 32, i = t % 32;
+    const float th = exp2f(-13.287712379549449f * 2.f * (float)i / 64.f);  // 10000^(-2i/64)
+    float sn, cs;
+    sincosf((float)pos * th, &sn, &cs);
+    tab[t] = make_float2(cs, sn);
   }
+}
+// cos / sin of the lane's two pairs (2 lane, 2 lane + 1: axis lane / 16, frequencies
+// 2 lane % 32 and + 1) for token n; identity for text tokens
+__device__ __forceinline__ void rope_lane(const QkNormRope& a, const float2* tab, int n, int lane, float (&cs)[2],
+                                          float (&sn)[2]) {
+  cs[0] = cs[1] = 1.f;
+  sn[0] = sn[1] = 0.f;
+  if (!a.rope || n < a.n_txt) return;
+  const int tok = n - a.n_txt;
+  const int pos = lane < 16 ? tok / a.gw : tok % a.gw;
+  const float4 v = *reinterpret_cast<const float4*>(tab + pos * 32 + ((2 * lane) & 31));
+  cs[0] = v.x; sn[0] = v.y; cs[1] = v.z; sn[1] = v.w;
 }
 
 __global__ void __launch_bounds__(QKN_THREADS) qk_norm_rope_fwd_v_kernel(QkNormRope a) {
+  extern __shared__ __align__(16) float2 rope_tab[];  // [side][32] when a.rope
+  if (a.rope) rope_table_fill(a, rope_tab);
+  __syncthreads();
   const int lane = threadIdx.x & 31;
   float scl[4][4];  // q txt, q img, k txt, k img: this lane's 4 elements
   bf16x4_load(static_cast<const bf16*>(a.qscale_txt) + 4 * lane, scl[0]);
@@ -944,7 +969,7 @@ __global__ void __launch_bounds__(QKN_THREADS) qk_norm_rope_fwd_v_kernel(QkNormR
       const int n = m % a.N;
       const bool txt = n < a.n_txt;
       float cs[2], sn[2];
-      rope_lane(a, n, lane, cs, sn);
+      rope_lane(a, rope_tab, n, lane, cs, sn);
 #pragma unroll
       for (int which = 0; which < 2; ++which) {
         float sc[4];  // selected per element: the array index stays a compile-time constant
@@ -967,15 +992,18 @@ __global__ void __launch_bounds__(QKN_THREADS) qk_norm_rope_fwd_v_kernel(QkNormR
   }
 }
 
-__global__ void __launch_bounds__(QKN_THREADS) qk_norm_rope_bwd_v_kernel(QkNormRopeBwd b) {
+__global__ void __launch_bounds__(QKN_THREADS, 3) qk_norm_rope_bwd_v_kernel(QkNormRopeBwd b) {
   const QkNormRope& a = b.f;
   __shared__ float part[QKN_WARPS][4][128];
+  extern __shared__ __align__(16) float2 rope_tab[];  // [side][32] when a.rope
+  if (a.rope) rope_table_fill(a, rope_tab);
+  __syncthreads();
   const int lane = threadIdx.x & 31, warp = threadIdx.x / 32;
-  float scl[4][4];  // q txt, q img, k txt, k img: this lane's 4 elements
-  bf16x4_load(static_cast<const bf16*>(a.qscale_txt) + 4 * lane, scl[0]);
-  bf16x4_load(static_cast<const bf16*>(a.qscale_img) + 4 * lane, scl[1]);
-  bf16x4_load(static_cast<const bf16*>(a.kscale_txt) + 4 * lane, scl[2]);
-  bf16x4_load(static_cast<const bf16*>(a.kscale_img) + 4 * lane, scl[3]);
+  __shared__ __align__(16) float scl[4][128];  // q txt, q img, k txt, k img
+  for (int t = threadIdx.x; t < 4 * 128; t += QKN_THREADS) {
+    const void* p = t < 128 ? a.qscale_txt : t < 256 ? a.qscale_img : t < 384 ? a.kscale_txt : a.kscale_img;
+    scl[t / 128][t % 128] = __bfloat162float(static_cast<const bf16*>(p)[t % 128]);
+  }
   float acc[4][4];  // scale gradients, [which * 2 + stream][element]
 #pragma unroll
   for (int i = 0; i < 4; ++i)
@@ -1005,12 +1033,11 @@ __global__ void __launch_bounds__(QKN_THREADS) qk_norm_rope_bwd_v_kernel(QkNormR
       const int n = m % a.N;
       const bool txt = n < a.n_txt;
       float cs[2], sn[2];
-      rope_lane(a, n, lane, cs, sn);
+      rope_lane(a, rope_tab, n, lane, cs, sn);
 #pragma unroll
       for (int which = 0; which < 2; ++which) {
-        float sc[4];  // selected per element: the array index stays a compile-time constant
-#pragma unroll
-        for (int e = 0; e < 4; ++e) sc[e] = txt ? scl[which * 2][e] : scl[which * 2 + 1][e];
+        const float4 sc4 = *reinterpret_cast<const float4*>(&scl[which * 2 + (txt ? 0 : 1)][4 * lane]);
+        const float sc[4] = {sc4.x, sc4.y, sc4.z, sc4.w};
         const float* xv = x[it][which];
         const float r = (which == 0 ? a.rq : a.rk)[(int64_t)m * a.heads + hd];
         float u[4], dy[4];
@@ -1190,7 +1217,15 @@ int launch_attn_rowdot(const void* dO, const void* O, int64_t ld, float* Dv, int
 }
 // The vectorised kernels serve head dim 128 in bf16 with 8-byte aligned rows and scales.
 static bool aligned8(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 7) == 0; }
+static int qkn_table_bytes(const QkNormRope& a) {
+  if (!a.rope) return 0;
+  const int gh = (a.N - a.n_txt) / a.gw;
+  return (gh > a.gw ? gh : a.gw) * 32 * (int)sizeof(float2);
+}
 static bool qkn_vector(const QkNormRope& a) {
+  if (a.rope && (a.gw <= 0 || (a.N - a.n_txt) % a.gw || (a.N - a.n_txt) / a.gw > QKN_TABLE_MAX ||
+                 a.gw > QKN_TABLE_MAX))
+    return false;
   return a.dtype == JAGG_DTYPE_BF16 && a.heads > 0 && a.d == 128 * a.heads && a.ld_qkv % 4 == 0 &&
          aligned8(a.qkv) && aligned8(a.qk_out) && aligned8(a.qscale_txt) && aligned8(a.qscale_img) &&
          aligned8(a.kscale_txt) && aligned8(a.kscale_img);
@@ -1204,7 +1239,7 @@ int launch_qk_norm_rope_fwd(const QkNormRope& a, cudaStream_t s) {
   if (qkn_vector(a)) {
     const int64_t vb = ceil_div((int64_t)a.M * a.heads, (int64_t)QKN_WARPS * QKV_ITEMS);
     const int cap = 16 * sm_count();
-    qk_norm_rope_fwd_v_kernel<<<(int)(vb < cap ? vb : cap), QKN_THREADS, 0, s>>>(a);
+    qk_norm_rope_fwd_v_kernel<<<(int)(vb < cap ? vb : cap), QKN_THREADS, qkn_table_bytes(a), s>>>(a);
   } else {
     qk_norm_rope_fwd_kernel<<<(int)(blocks < 65536 ? blocks : 65536), QKN_THREADS, 0, s>>>(a);
   }
@@ -1227,8 +1262,8 @@ int launch_qk_norm_rope_bwd(const QkNormRopeBwd& a, cudaStream_t s) {
   if (qkn_vector(f) && a.ld_dqk % 4 == 0 && aligned8(a.dqk)) {
     // a few blocks per SM: each block ends in 4 x 128 scale-gradient atomics
     const int64_t vb = ceil_div((int64_t)f.M * f.heads, (int64_t)QKN_WARPS * QKV_ITEMS);
-    const int vcap = 8 * sm_count();
-    qk_norm_rope_bwd_v_kernel<<<(int)(vb < vcap ? vb : vcap), QKN_THREADS, 0, s>>>(a);
+    const int vcap = 3 * sm_count();  // the resident blocks (80 registers, 3 per SM)
+    qk_norm_rope_bwd_v_kernel<<<(int)(vb < vcap ? vb : vcap), QKN_THREADS, qkn_table_bytes(f), s>>>(a);
   } else {
     qk_norm_rope_bwd_kernel<<<(int)(blocks < cap ? blocks : cap), QKN_THREADS, 0, s>>>(a);
   }
