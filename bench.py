@@ -62,7 +62,7 @@ def parse():
     p.add_argument("--quick", action="store_true", help="skip the full-W, e2e and CPU legs")
     p.add_argument("--G", type=int, default=0,
                    help="override the workload's group size (small cases for profiler captures)")
-    p.add_argument("--kernel", choices=["attention_bwd", "attention_fwd", "gemm"], default=None,
+    p.add_argument("--kernel", choices=["attention_bwd", "attention_fwd", "gemm", "hbm"], default=None,
                    help="time one kernel family alone on the workload's shapes instead of the step")
     p.add_argument("--product", default="all",
                    help="for --kernel gemm: one of the block's backward products (gemm_products: DiT fc2_dx, "
@@ -96,7 +96,7 @@ def describe(wl) -> str:
 # bytes, from one ncu capture of the kernel alone (`--kernel gemm`) on the workload's
 # backward products at the step's rows; the roofline's `traffic` is this ratio times the
 # step's algorithmic bytes per launch.  Absent: no capture of the current kernel.
-TRAFFIC_RATIO = {}
+TRAFFIC_RATIO = {"mmdit_flux1024_bf16": 2.96}
 
 
 def peaks():
@@ -1186,6 +1186,103 @@ def run_kernel_gemm(args):
                       "products": out}), flush=True)
 
 
+def run_kernel_hbm(args):
+    """The bandwidth-bound kernels of the joint VJP alone at the workload's per-window shapes
+    (rows = 2G sequences of one window by default) on random operands, each timed by the
+    library's per-launch events over the timed calls and reported against the measured HBM
+    copy bandwidth: the LayerNorm + modulation and gate backward (a single block's rows), the
+    QK-norm + RoPE forward and backward, the bias column sums (a single block's lin1 output
+    gradient), the step signals with the fused aggregation, grad_reduce (a 256 M-parameter
+    slice: the norm and a dot with a second gradient).  Every operand a few hundred MB."""
+    import paper_2607_17572_gb300 as jg
+    wl = workload(args)
+    dev = torch.device("cuda", torch.cuda.current_device())
+    seqs = args.rows or 2 * wl.G
+    N, d, dm, H = wl.n_tok, wl.hidden, wl.mlp, wl.heads
+    M = seqs * N
+    gen = torch.Generator(device=dev).manual_seed(synth.NOISE_SEED)
+    bf = torch.bfloat16
+    f = dict(device=dev, dtype=torch.float32)
+    burst, sustained, hbm, src = peaks()
+    out = {}
+
+    def run(name, family, fn):
+        for _ in range(args.warmup):
+            fn()
+        torch.cuda.synchronize()
+        torch.cuda.profiler.start()
+        jg.profile_enable(True)
+        for _ in range(args.steps):
+            fn()
+        prof = jg.profile_read()
+        jg.profile_enable(False)
+        torch.cuda.profiler.stop()
+        fam = prof[family]
+        ms = fam["ms"] / max(fam["launches"], 1)
+        gbs = fam["bytes"] / max(fam["launches"], 1) / (ms / 1000.0) / 1e9
+        out[name] = {"family": family, "ms_per_launch": ms, "algorithmic_mb_per_launch": fam["bytes"] / max(fam["launches"], 1) / 1e6,
+                     "gbs": gbs, "frac_of_hbm": gbs / hbm}
+
+    # LayerNorm + modulation and gate backward over a single block's rows
+    h = torch.randn(M, d, **f, generator=gen)
+    mean, rstd = h.mean(1), torch.rsqrt(h.var(1, unbiased=False) + 1e-6)
+    dmv = torch.randn(M, d, **f, generator=gen)
+    dh = torch.randn(M, d, **f, generator=gen)
+    y = torch.randn(M, d, **f, generator=gen).to(bf)
+    dy = torch.empty(M, d, device=dev, dtype=bf)
+    scale, gate = torch.randn(seqs, d, **f, generator=gen), torch.randn(seqs, d, **f, generator=gen)
+    acc3 = [torch.zeros(seqs, d, **f) for _ in range(3)]
+    dbias = torch.zeros(d, **f)
+    run("ln_gate_bwd", "ln_gate_bwd",
+        lambda: jg.test_ln_gate_bwd(M, d, N, dh, dh, dm=dmv, h=h, mean=mean, rstd=rstd, scale=scale, dshift=acc3[0],
+                                    dscale=acc3[1], y=y, gate=gate, dgate=acc3[2], dy=dy, dbias=dbias))
+    del h, mean, rstd, dmv, dh, y, dy
+    torch.cuda.empty_cache()
+    if wl.arch == "mmdit":
+        dh_ = wl.head_dim
+        qkv = (torch.randn(M, 3 * d, **f, generator=gen) * 2).to(bf)
+        qs, ks = torch.ones(dh_, device=dev, dtype=bf), torch.ones(dh_, device=dev, dtype=bf)
+        qk = torch.empty(M, 2 * d, device=dev, dtype=bf)
+        rq, rk = torch.empty(M, H, **f), torch.empty(M, H, **f)
+        gw = wl.latent_w // wl.patch
+        run("qk_norm_rope_fwd", "qk_norm_rope_fwd",
+            lambda: jg.test_qk_norm_rope_fwd(qkv, M, N, H, wl.txt_len, gw, qs, ks, qk, rq, rk))
+        dqk = torch.randn(M, 3 * d + dm, **f, generator=gen).to(bf)
+        dqs, dks = torch.zeros(dh_, **f), torch.zeros(dh_, **f)
+        run("qk_norm_rope_bwd", "qk_norm_rope_bwd",
+            lambda: jg.test_qk_norm_rope_bwd(qkv, M, N, H, wl.txt_len, gw, qs, ks, rq, rk, dqk, dqs, dks))
+        del qkv, qk, rq, rk
+        X = dqk
+    else:
+        X = torch.randn(M, 3 * d, **f, generator=gen).to(bf)
+    db = torch.zeros(X.shape[1], **f)
+    run("colsum", "colsum", lambda: jg.test_colsum(X, db))
+    del X
+    torch.cuda.empty_cache()
+    # the step signals of one window with the fused aggregation (Phases 2-3)
+    G, W, D = wl.G, wl.W, wl.D
+    v = torch.randn(G, W, D, **f, generator=gen).to(bf)
+    z = torch.randn(G, W + 1, D, **f, generator=gen)
+    t = synth.time_grid(wl.T, wl.shift)
+    sig = synth.sigma_schedule(t, wl.eta)
+    f64 = dict(dtype=torch.float64, device=dev)
+    so = dict(logp_new=torch.empty(G, W, **f64), ratio=torch.empty(G, W, **f64),
+              clipped=torch.empty(G, W, dtype=torch.uint8, device=dev), adv_out=torch.empty(G, **f64))
+    cot = torch.empty(2 * G, D, **f)
+    sws = jg.alloc_bytes(jg.signals_workspace_bytes(G, W, D), dev)
+    targs = (v, z, torch.tensor(t[:W + 1], **f64), torch.tensor(sig[:W], **f64), torch.zeros(G, W, **f64),
+             torch.randn(G, **f, generator=gen), wl.clip_eps, wl.adv_clip, wl.adv_eps, 1.0 / (G * wl.T))
+    run("step_signals", "step_signals", lambda: jg.grpo_step_signals(*targs, ws=sws, cot_out=cot, **so))
+    # grad_reduce on a 256 M-parameter slice: |a|^2 and <a, b>
+    P = 256 * 1024 * 1024
+    ga, gb = torch.randn(P, **f, generator=gen), torch.randn(P, **f, generator=gen)
+    out3 = torch.zeros(3, **f64)
+    gws = jg.alloc_bytes(jg.grad_reduce_workspace_bytes(P), dev)
+    run("grad_reduce_dot", "grad_reduce", lambda: jg.grad_reduce(ga, gb, out3=out3, ws=gws))
+    print(json.dumps({"kernel": "hbm", "workload": describe(wl), "rows": M, "sequences": seqs, "steps": args.steps,
+                      "peak": {"hbm_gbs": hbm, "source": f"hbm_gbs of {src} peaks"}, "kernels": out}), flush=True)
+
+
 def main():
     args = parse()
     ws, rank = dist_setup(need_gpu=args.impl != "reference" or args.kernel is not None)
@@ -1195,6 +1292,9 @@ def main():
     elif args.kernel == "gemm":
         if rank == 0:
             run_kernel_gemm(args)
+    elif args.kernel == "hbm":
+        if rank == 0:
+            run_kernel_hbm(args)
     elif args.impl == "reference":
         run_reference(args, ws, rank)
     elif args.sweep:

@@ -98,6 +98,27 @@ int jagg_test_ln_gate_bwd(int M, int d, int rows_per_seq, int do_ln, int do_gate
                           const float* dh_in, float* dh_out, const void* y, const float* gate, float* dgate,
                           void* dy, float* dbias, int dtype, cudaStream_t stream);
 
+/* Per-head RMSNorm of q and k (learned scale [dh], eps 1e-6) followed by 2D RoPE (the MMDiT
+ * blocks' QK normalisation; the backbone reading of the paper's Flux / Qwen-Image models), on
+ * M rows of N tokens per sequence whose first n_txt tokens are text (not rotated) and whose
+ * image tokens lie on a grid gw wide.  qkv [M, ld_qkv] holds q at column 0 and k at column d
+ * (d = heads * dh, dh <= 128 even), in `dtype`; qscale, kscale [dh] in `dtype`.
+ * Forward: qk_out [M, 2d] = the normalised, rotated q then k; rq, rk [M, heads] f32 the
+ * inverse RMS of each (row, head).  rope = 0 skips the rotation. */
+int jagg_test_qk_norm_rope_fwd(const void* qkv, int64_t ld_qkv, int M, int N, int d, int heads, int n_txt, int gw,
+                               const void* qscale, const void* kscale, int rope, void* qk_out, float* rq, float* rk,
+                               int dtype, cudaStream_t stream);
+/* Backward of the above: dqk [M, ld_dqk] (dtype) holds the gradient of the rotated q at column
+ * 0 and of k at column d on entry and the gradient of the raw q, k on exit; dqscale,
+ * dkscale [dh] f32 accumulate the scale gradients.  rq, rk from the forward. */
+int jagg_test_qk_norm_rope_bwd(const void* qkv, int64_t ld_qkv, int M, int N, int d, int heads, int n_txt, int gw,
+                               const void* qscale, const void* kscale, int rope, const float* rq, const float* rk,
+                               void* dqk, int64_t ld_dqk, float* dqscale, float* dkscale, int dtype,
+                               cudaStream_t stream);
+/* Column sums db[c] += sum_r X[r * ld + c] (r < rows, c < cols; X f32 when x_f32 else bf16):
+ * the bias gradients of the joint VJP. */
+int jagg_test_colsum(const void* X, int x_f32, int rows, int cols, int64_t ld, float* db, cudaStream_t stream);
+
 /* Failure detection of the bounded waits (every mbarrier wait of the library gives up after
  * a wall-clock limit instead of hanging): one CTA waits on an mbarrier that nothing arrives
  * at, with the limit limit_ns (0 < limit_ns <= 2 s, else JAGG_ERR_ARG) in place of the

@@ -119,6 +119,10 @@ _SIGNATURES = {
     "jagg_test_attention_fwd_streams": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
     "jagg_test_ln_gate_bwd": (_I, [_I, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P,
                                    _I, _P]),
+    "jagg_test_qk_norm_rope_fwd": (_I, [_P, _I64, _I, _I, _I, _I, _I, _I, _P, _P, _I, _P, _P, _P, _I, _P]),
+    "jagg_test_qk_norm_rope_bwd": (_I, [_P, _I64, _I, _I, _I, _I, _I, _I, _P, _P, _I, _P, _P, _P, _I64, _P, _P, _I,
+                                        _P]),
+    "jagg_test_colsum": (_I, [_P, _I, _I, _I, _I64, _P, _P]),
     "jagg_test_attention_bwd_streams": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _I,
                                              _P]),
 }
@@ -464,6 +468,32 @@ def test_ln_gate_bwd(M, d, rows_per_seq, dh_in, dh_out, dm=None, h=None, mean=No
                                        _ptr(rstd), _ptr(scale), _ptr(dshift), _ptr(dscale), _ptr(dh_in),
                                        _ptr(dh_out), _ptr(y), _ptr(gate), _ptr(dgate), _ptr(dy), _ptr(dbias), dt,
                                        _stream(stream)), "jagg_test_ln_gate_bwd")
+
+
+def test_qk_norm_rope_fwd(qkv, M, N, heads, n_txt, gw, qscale, kscale, qk_out, rq, rk, rope=True, stream=None):
+    """Per-head RMSNorm + 2D RoPE of q, k (jagg_test_qk_norm_rope_fwd); qkv [M, >= 2d]."""
+    d = qk_out.shape[-1] // 2
+    dt = DTYPE_BF16 if qkv.dtype == torch.bfloat16 else DTYPE_F32
+    _check(lib().jagg_test_qk_norm_rope_fwd(_ptr(qkv), qkv.stride(0), M, N, d, heads, n_txt, gw, _ptr(qscale),
+                                            _ptr(kscale), int(rope), _ptr(qk_out), _ptr(rq), _ptr(rk), dt,
+                                            _stream(stream)), "jagg_test_qk_norm_rope_fwd")
+
+
+def test_qk_norm_rope_bwd(qkv, M, N, heads, n_txt, gw, qscale, kscale, rq, rk, dqk, dqscale, dkscale, rope=True,
+                          stream=None):
+    """Its backward in place on dqk [M, >= 2d] (jagg_test_qk_norm_rope_bwd)."""
+    d = qscale.numel() * heads
+    dt = DTYPE_BF16 if qkv.dtype == torch.bfloat16 else DTYPE_F32
+    _check(lib().jagg_test_qk_norm_rope_bwd(_ptr(qkv), qkv.stride(0), M, N, d, heads, n_txt, gw, _ptr(qscale),
+                                            _ptr(kscale), int(rope), _ptr(rq), _ptr(rk), _ptr(dqk), dqk.stride(0),
+                                            _ptr(dqscale), _ptr(dkscale), dt, _stream(stream)),
+           "jagg_test_qk_norm_rope_bwd")
+
+
+def test_colsum(X, db, stream=None):
+    """db += column sums of X [rows, cols] (f32 or bf16) (jagg_test_colsum)."""
+    _check(lib().jagg_test_colsum(_ptr(X), int(X.dtype == torch.float32), X.shape[0], X.shape[1], X.stride(0),
+                                  _ptr(db), _stream(stream)), "jagg_test_colsum")
 
 
 def test_wait_timeout(limit_ns: int, out, stream=None):

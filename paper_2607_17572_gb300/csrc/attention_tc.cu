@@ -1,27 +1,22 @@
 // Attention backward on the fifth-generation tensor cores (tcgen05, TMEM accumulators,
-// TMA-fed shared-memory operands), bf16, head dim 64 or 128 (appendix, Eqs. bwd_V ..
-// bwd_QK, with the softmax recomputed from the saved log-sum-exp).
+// TMA-fed shared-memory operands), bf16 (appendix, Eqs. bwd_V .. bwd_QK, with the softmax
+// recomputed from the saved log-sum-exp).  Head dim 64: fa_bwd_tc_kernel below; head dim
+// 128: fa_bwd_tc128_kernel further down.
 //
-// Persistent: each CTA walks (128-key tile, sequence, head) units; per unit it streams the
-// sequence's query tiles:
-//   S^T = K Q^T, dP^T = V dO^T                      (128 x BQ, TMEM)
+// Head dim 64.  Persistent: each CTA walks (128-key tile, sequence, head) units; per unit it
+// streams the sequence's 128-query tiles:
+//   S^T = K Q^T, dP^T = V dO^T                      (128 x 128, TMEM)
 //   P^T = exp(scale S^T - lse), dS^T = P^T (dP^T - rowsum(dO O))   (8 warps, -> bf16 smem)
-//   dV += P^T dO, dK += dS^T Q                      (128 x dh, TMEM, whole sequence)
-//   dQ  = dS K (head dim 64, BQ = 128) or dQ^T = K^T dS^T (head dim 128, BQ = 64)
-//        -> 4 warps -> TMA f32 reduce-add into the dQ accumulator.
+//   dV += P^T dO, dK += dS^T Q                      (128 x 64, TMEM, whole sequence)
+//   dQ  = dS K  -> 4 warps -> TMA f32 reduce-add into the dQ accumulator.
 // Every product has M = 128.  Each shared tile serves as a K-major and an MN-major
 // operand through two descriptors of the same 128-byte-swizzled layout, so nothing is
 // transposed.  Warp roles: 0 TMA producer, 1 MMA issuer (one elected thread), 2-9 P / dS
-// (two warps per TMEM lane quarter, half the query columns each) and the final dK / dV,
-// 10-13 dQ.
-// Head dim 128: S^T, dP^T are double-buffered in TMEM and dQ^T of a tile is written over
-// its own (consumed) S^T columns, so S^T, dP^T of tile j + 1 are ready while P, dS of
-// tile j are formed (512 columns: 2 x (64 + 64) + 128 + 128).  Head dim 64: one S^T, dP^T
-// buffer (128 + 128 + 64 + 64 + 64 columns); the MMA warp issues S, dP of tile j + 1 before
-// dV, dK, dQ of tile j.
-// Tile-level barrier phases run on across units, so the next unit's K, V loads and first
-// products overlap the previous unit's last tiles and its dQ drain (head dim 64 keeps two
-// K, V buffers for that).
+// (two warps per TMEM lane quarter, half the query columns each), 10-13 dQ and the final
+// dK / dV.  One S^T, dP^T buffer (128 + 128 + 64 + 64 + 64 columns); the MMA warp issues S,
+// dP of tile j + 1 before dV, dK, dQ of tile j.
+// Tile-level barrier phases run on across units, and two K, V buffers let the next unit's K,
+// V loads and first products overlap the previous unit's last tiles and its dQ drain.
 // Ragged ends: 3D tensor maps [sequence][token][column] per stream buffer make TMA read
 // zeros past the last token and drop dQ rows past it.
 #include <cuda.h>
@@ -40,18 +35,18 @@ constexpr int FB_THREADS = 448;  // 14 warps
 
 template <int D>
 struct FbCfg {
+  static_assert(D == 64, "head dim 128 has fa_bwd_tc128_kernel");
   static constexpr int BK = 128;                 // keys per CTA
-  static constexpr int BQ = D == 64 ? 128 : 64;  // queries per step
-  static constexpr bool DQT = D == 128;          // dQ^T = K^T dS^T (M = D)
-  static constexpr int NSB = DQT ? 2 : 1;        // S^T / dP^T TMEM buffers
+  static constexpr int BQ = 128;                 // queries per step
+  static constexpr int NSB = 1;                  // S^T / dP^T TMEM buffers
   static constexpr int CW = BQ / 2;              // query columns per P / dS warp
   static constexpr int KV_BYTES = BK * D * 2;
   static constexpr int QT_BYTES = BQ * D * 2;
   static constexpr int PS_BYTES = BK * BQ * 2;
-  // head dim 64 (short sequences in practice): K, V double-buffered across the CTA's
-  // units, two Q / dO stages; head dim 128: one K, V buffer, three stages
-  static constexpr int KVB = D == 64 ? 2 : 1;
-  static constexpr int STAGES = D == 64 ? 2 : 3;
+  // short sequences in practice: K, V double-buffered across the CTA's units, two Q / dO
+  // stages
+  static constexpr int KVB = 2;
+  static constexpr int STAGES = 2;
   static constexpr int DQ_WARP_BYTES = 32 * 32 * 4;  // one 32 x 32 f32 box, used twice per tile
   static constexpr int OFF_K = 0;                       // KVB buffers
   static constexpr int OFF_V = OFF_K + KVB * KV_BYTES;    // KVB buffers
@@ -64,11 +59,11 @@ struct FbCfg {
   static constexpr int OFF_RD = OFF_LSE + STAGES * BQ * 4;
   static constexpr int OFF_BAR = OFF_RD + STAGES * BQ * 4;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;
-  // TMEM columns
-  static constexpr int T_DV = DQT ? 256 : 256, T_DK = DQT ? 384 : 320;
-  __host__ __device__ static constexpr int t_s(int b) { return DQT ? b * 64 : 0; }
-  __host__ __device__ static constexpr int t_dp(int b) { return DQT ? 128 + b * 64 : 128; }
-  __host__ __device__ static constexpr int t_dq(int b) { return DQT ? b * 64 : 384; }
+  // TMEM columns: S^T [0, 128), dP^T [128, 256), dV, dK, dQ
+  static constexpr int T_DV = 256, T_DK = 320;
+  __host__ __device__ static constexpr int t_s(int) { return 0; }
+  __host__ __device__ static constexpr int t_dp(int) { return 128; }
+  __host__ __device__ static constexpr int t_dq(int) { return 384; }
   static_assert(SMEM <= 232448, "shared memory budget");
 };
 
@@ -317,11 +312,6 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
         if (!ptx::mbar_wait(&bar_kv[kvb], (i / KVB) & 1)) { ok = false; break; }
         for (int j = 0; j < NSB && j < nq; ++j) {
           const int g = i * nq + j;
-          // head dim 128: the buffer's previous tile (an earlier unit's) has been drained
-          if (NSB == 2 && g >= NSB && !ptx::mbar_wait(&bar_dqfree[g % NSB], ((g - NSB) / NSB) & 1)) {
-            ok = false;
-            break;
-          }
           if (!ptx::mbar_wait(&full[g % NS], (g / NS) & 1)) { ok = false; break; }
           ptx::tc_fence_after();
           issue_s(g);
@@ -331,13 +321,11 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
           const int st = g % NS, bb = g % NSB;
           if (!ptx::mbar_wait(bar_p, g & 1)) { ok = false; break; }
           ptx::tc_fence_after();
-          if constexpr (NSB == 1) {
-            // the single S^T / dP^T buffer is consumed: the next tile's products first
-            if (j + 1 < nq) {
-              if (!ptx::mbar_wait(&full[(g + 1) % NS], ((g + 1) / NS) & 1)) { ok = false; break; }
-              ptx::tc_fence_after();
-              issue_s(g + 1);
-            }
+          // the single S^T / dP^T buffer is consumed: the next tile's products first
+          if (j + 1 < nq) {
+            if (!ptx::mbar_wait(&full[(g + 1) % NS], ((g + 1) / NS) & 1)) { ok = false; break; }
+            ptx::tc_fence_after();
+            issue_s(g + 1);
           }
           const uint32_t aQ = ptx::smem_u32(sQ + st * C::QT_BYTES), adO = ptx::smem_u32(sdO + st * C::QT_BYTES);
           // the first dV, dK products of a unit overwrite the accumulators: the dQ warps have
@@ -352,33 +340,17 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
             ptx::umma_bf16(tmem + C::T_DV, kmajor_desc(aP, BK, k), mnmajor_desc(adO, BQ * 128, k), id_acc, acc);
             ptx::umma_bf16(tmem + C::T_DK, kmajor_desc(adS, BK, k), mnmajor_desc(aQ, BQ * 128, k), id_acc, acc);
           }
-          if constexpr (NSB == 1) {
-            if (g > 0) {  // the dQ warps have read the previous tile's dQ
-              if (!ptx::mbar_wait(&bar_dqfree[0], (g - 1) & 1)) { ok = false; break; }
-              ptx::tc_fence_after();
-            }
+          if (g > 0) {  // the dQ warps have read the previous tile's dQ
+            if (!ptx::mbar_wait(&bar_dqfree[0], (g - 1) & 1)) { ok = false; break; }
+            ptx::tc_fence_after();
           }
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k) {
-            if constexpr (C::DQT)  // dQ^T[d][q] = sum_key K[key][d] dS^T[key][q], over this tile's S^T
-              ptx::umma_bf16(tmem + C::t_dq(bb), mnmajor_desc(aK, BK * 128, k), mnmajor_desc(adS, BK * 128, k),
-                             id_dq, k > 0);
-            else  // dQ[q][d] = sum_key dS^T[key][q] K[key][d]
-              ptx::umma_bf16(tmem + C::t_dq(bb), mnmajor_desc(adS, BK * 128, k), mnmajor_desc(aK, BK * 128, k),
-                             id_dq, k > 0);
-          }
+          for (int k = 0; k < BK / 16; ++k)  // dQ[q][d] = sum_key dS^T[key][q] K[key][d]
+            ptx::umma_bf16(tmem + C::t_dq(bb), mnmajor_desc(adS, BK * 128, k), mnmajor_desc(aK, BK * 128, k),
+                           id_dq, k > 0);
           ptx::umma_commit(&bar_dq[bb]);
           ptx::umma_commit(&empty[st]);
           ptx::umma_commit(bar_pfree);
-          if constexpr (NSB == 2) {
-            // S^T, dP^T of tile g + 2 go into this buffer once the dQ warps have read dQ^T
-            if (j + 2 < nq) {
-              if (!ptx::mbar_wait(&bar_dqfree[bb], (g / NSB) & 1)) { ok = false; break; }
-              if (!ptx::mbar_wait(&full[(g + 2) % NS], ((g + 2) / NS) & 1)) { ok = false; break; }
-              ptx::tc_fence_after();
-              issue_s(g + 2);
-            }
-          }
         }
         ptx::umma_commit(&kv_free[kvb]);
         ptx::umma_commit(bar_fin);
@@ -458,32 +430,24 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
         __syncwarp();
         if (lane == 0) ptx::mbar_arrive(&bar_dqfree[bb]);
         const int q0 = j * BQ;
-        // two 32 x 32 boxes through one staging box: dQ^T (lane = head dim, columns = the
-        // tile's 64 queries: box rows = queries) or dQ (lane = query, columns = 64 head dims)
+        // two 32 x 32 boxes (lane = query, columns = 64 head dims) through one staging box
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
           if (lane == 0) ptx::bulk_wait_read<0>();
           __syncwarp();
-          if constexpr (C::DQT) {
+          uint8_t* srow = stg + lane * 128;
 #pragma unroll
-            for (int q = 0; q < 32; ++q)
-              *reinterpret_cast<float*>(stg + q * 128 + (((lane >> 2) ^ (q & 7)) << 4) + (lane & 3) * 4) =
-                  __uint_as_float(rq[hh * 32 + q]) * p.scale;
-          } else {
-            uint8_t* row = stg + lane * 128;
-#pragma unroll
-            for (int v = 0; v < 8; ++v)
-              *reinterpret_cast<float4*>(row + ((v ^ (lane & 7)) << 4)) =
-                  make_float4(__uint_as_float(rq[hh * 32 + 4 * v]) * p.scale,
-                              __uint_as_float(rq[hh * 32 + 4 * v + 1]) * p.scale,
-                              __uint_as_float(rq[hh * 32 + 4 * v + 2]) * p.scale,
-                              __uint_as_float(rq[hh * 32 + 4 * v + 3]) * p.scale);
-          }
+          for (int v = 0; v < 8; ++v)
+            *reinterpret_cast<float4*>(srow + ((v ^ (lane & 7)) << 4)) =
+                make_float4(__uint_as_float(rq[hh * 32 + 4 * v]) * p.scale,
+                            __uint_as_float(rq[hh * 32 + 4 * v + 1]) * p.scale,
+                            __uint_as_float(rq[hh * 32 + 4 * v + 2]) * p.scale,
+                            __uint_as_float(rq[hh * 32 + 4 * v + 3]) * p.scale);
           ptx::fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) {
-            const int col = C::DQT ? h * D + quarter * 32 : h * D + hh * 32;
-            const int row = C::DQT ? q0 + hh * 32 : q0 + quarter * 32;
+            const int col = h * D + hh * 32;
+            const int row = q0 + quarter * 32;
             if (row < N) {
               ptx::tma_reduce_add_3d(&maps.dq, stg, col, row, b);
               ptx::bulk_commit();

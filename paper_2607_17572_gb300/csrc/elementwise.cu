@@ -889,8 +889,8 @@ __global__ void __launch_bounds__(QKN_THREADS) qk_norm_rope_bwd_kernel(QkNormRop
 // [4l, 4l + 4) of q and of k, i.e. the rotated pairs 2l and 2l + 1, so every operand moves
 // in 8-byte vectors and each lane's RMSNorm scales and RoPE frequencies are fixed for the
 // whole kernel.  The angles are the ones rope_angle forms (same expressions), so the forward
-// rotation and its inverse in the backward agree bit for bit.  Two (row, head) items per
-// warp iteration keep 2 KB of loads in flight per warp.
+// rotation and its inverse in the backward agree bit for bit.  A warp walks rows, each row's
+// heads two at a time (2 KB of loads in flight per warp in the backward).
 constexpr int QKV_ITEMS = 2;
 
 __device__ __forceinline__ void bf16x4_load(const bf16* p, float (&v)[4]) {
@@ -948,45 +948,44 @@ __global__ void __launch_bounds__(QKN_THREADS) qk_norm_rope_fwd_v_kernel(QkNormR
   bf16x4_load(static_cast<const bf16*>(a.qscale_img) + 4 * lane, scl[1]);
   bf16x4_load(static_cast<const bf16*>(a.kscale_txt) + 4 * lane, scl[2]);
   bf16x4_load(static_cast<const bf16*>(a.kscale_img) + 4 * lane, scl[3]);
-  const int64_t items = (int64_t)a.M * a.heads;
-  const int64_t stride = (int64_t)gridDim.x * QKN_WARPS * QKV_ITEMS;
-  for (int64_t w0 = ((int64_t)blockIdx.x * QKN_WARPS + threadIdx.x / 32) * QKV_ITEMS; w0 < items; w0 += stride) {
-    float x[QKV_ITEMS][2][4];
+  // one row per warp, its heads two at a time: the token's stream and angles once per row
+  for (int m = blockIdx.x * QKN_WARPS + threadIdx.x / 32; m < a.M; m += gridDim.x * QKN_WARPS) {
+    const int n = m % a.N;
+    const bool txt = n < a.n_txt;
+    float cs[2], sn[2];
+    rope_lane(a, rope_tab, n, lane, cs, sn);
+    const bf16* row = static_cast<const bf16*>(a.qkv) + (int64_t)m * a.ld_qkv + 4 * lane;
+    bf16* out = static_cast<bf16*>(a.qk_out) + (int64_t)m * 2 * a.d + 4 * lane;
+    for (int h0 = 0; h0 < a.heads; h0 += QKV_ITEMS) {
+      float x[QKV_ITEMS][2][4];
 #pragma unroll
-    for (int it = 0; it < QKV_ITEMS; ++it) {
-      const int64_t w = w0 + it < items ? w0 + it : w0;
-      const int hd = (int)(w % a.heads), m = (int)(w / a.heads);
+      for (int it = 0; it < QKV_ITEMS; ++it) {
+        const int hd = h0 + it < a.heads ? h0 + it : h0;
 #pragma unroll
-      for (int which = 0; which < 2; ++which)
-        bf16x4_load(static_cast<const bf16*>(a.qkv) + (int64_t)m * a.ld_qkv + which * a.d + hd * 128 + 4 * lane,
-                    x[it][which]);
-    }
+        for (int which = 0; which < 2; ++which) bf16x4_load(row + which * a.d + hd * 128, x[it][which]);
+      }
 #pragma unroll
-    for (int it = 0; it < QKV_ITEMS; ++it) {
-      const int64_t w = w0 + it;
-      if (w >= items) break;
-      const int hd = (int)(w % a.heads), m = (int)(w / a.heads);
-      const int n = m % a.N;
-      const bool txt = n < a.n_txt;
-      float cs[2], sn[2];
-      rope_lane(a, rope_tab, n, lane, cs, sn);
+      for (int it = 0; it < QKV_ITEMS; ++it) {
+        const int hd = h0 + it;
+        if (hd >= a.heads) break;
 #pragma unroll
-      for (int which = 0; which < 2; ++which) {
-        float sc[4];  // selected per element: the array index stays a compile-time constant
+        for (int which = 0; which < 2; ++which) {
+          float sc[4];  // selected per element: the array index stays a compile-time constant
 #pragma unroll
-        for (int e = 0; e < 4; ++e) sc[e] = txt ? scl[which * 2][e] : scl[which * 2 + 1][e];
-        const float* xv = x[it][which];
-        const float r = rsqrtf(warp_sum(xv[0] * xv[0] + xv[1] * xv[1] + xv[2] * xv[2] + xv[3] * xv[3]) / 128.f +
-                               1e-6f);
-        float o[4];
+          for (int e = 0; e < 4; ++e) sc[e] = txt ? scl[which * 2][e] : scl[which * 2 + 1][e];
+          const float* xv = x[it][which];
+          const float r =
+              rsqrtf(warp_sum(xv[0] * xv[0] + xv[1] * xv[1] + xv[2] * xv[2] + xv[3] * xv[3]) / 128.f + 1e-6f);
+          float o[4];
 #pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const float y0 = xv[2 * e] * r * sc[2 * e], y1 = xv[2 * e + 1] * r * sc[2 * e + 1];
-          o[2 * e] = y0 * cs[e] - y1 * sn[e];
-          o[2 * e + 1] = y0 * sn[e] + y1 * cs[e];
+          for (int e = 0; e < 2; ++e) {
+            const float y0 = xv[2 * e] * r * sc[2 * e], y1 = xv[2 * e + 1] * r * sc[2 * e + 1];
+            o[2 * e] = y0 * cs[e] - y1 * sn[e];
+            o[2 * e + 1] = y0 * sn[e] + y1 * cs[e];
+          }
+          bf16x4_store(out + which * a.d + hd * 128, o);
+          if (lane == 0) (which == 0 ? a.rq : a.rk)[(int64_t)m * a.heads + hd] = r;
         }
-        bf16x4_store(static_cast<bf16*>(a.qk_out) + (int64_t)m * 2 * a.d + which * a.d + hd * 128 + 4 * lane, o);
-        if (lane == 0) (which == 0 ? a.rq : a.rk)[(int64_t)m * a.heads + hd] = r;
       }
     }
   }
@@ -997,79 +996,76 @@ __global__ void __launch_bounds__(QKN_THREADS, 3) qk_norm_rope_bwd_v_kernel(QkNo
   __shared__ float part[QKN_WARPS][4][128];
   extern __shared__ __align__(16) float2 rope_tab[];  // [side][32] when a.rope
   if (a.rope) rope_table_fill(a, rope_tab);
-  __syncthreads();
   const int lane = threadIdx.x & 31, warp = threadIdx.x / 32;
   __shared__ __align__(16) float scl[4][128];  // q txt, q img, k txt, k img
   for (int t = threadIdx.x; t < 4 * 128; t += QKN_THREADS) {
     const void* p = t < 128 ? a.qscale_txt : t < 256 ? a.qscale_img : t < 384 ? a.kscale_txt : a.kscale_img;
     scl[t / 128][t % 128] = __bfloat162float(static_cast<const bf16*>(p)[t % 128]);
   }
-  float acc[4][4];  // scale gradients, [which * 2 + stream][element]
+  // scale gradients of the warp's rows, [which * 2 + stream][element]: one read-modify-write
+  // of the lane's 4 elements per row
+  float4* wpart = reinterpret_cast<float4*>(&part[warp][0][0]);
 #pragma unroll
-  for (int i = 0; i < 4; ++i)
+  for (int i = 0; i < 4; ++i) wpart[i * 32 + lane] = make_float4(0.f, 0.f, 0.f, 0.f);
+  __syncthreads();
+  // one row per warp, its heads two at a time: the token's stream and angles once per row
+  for (int m = blockIdx.x * QKN_WARPS + warp; m < a.M; m += gridDim.x * QKN_WARPS) {
+    const int n = m % a.N;
+    const bool txt = n < a.n_txt;
+    float cs[2], sn[2];
+    rope_lane(a, rope_tab, n, lane, cs, sn);
+    const bf16* xrow = static_cast<const bf16*>(a.qkv) + (int64_t)m * a.ld_qkv + 4 * lane;
+    bf16* grow = static_cast<bf16*>(b.dqk) + (int64_t)m * b.ld_dqk + 4 * lane;
+    float rowacc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};  // q, k scale gradients of the row
+    for (int h0 = 0; h0 < a.heads; h0 += QKV_ITEMS) {
+      float x[QKV_ITEMS][2][4], g[QKV_ITEMS][2][4];
 #pragma unroll
-    for (int e = 0; e < 4; ++e) acc[i][e] = 0.f;
-  const int64_t items = (int64_t)a.M * a.heads;
-  const int64_t stride = (int64_t)gridDim.x * QKN_WARPS * QKV_ITEMS;
-  for (int64_t w0 = ((int64_t)blockIdx.x * QKN_WARPS + warp) * QKV_ITEMS; w0 < items; w0 += stride) {
-    float x[QKV_ITEMS][2][4], g[QKV_ITEMS][2][4];
+      for (int it = 0; it < QKV_ITEMS; ++it) {
+        const int hd = h0 + it < a.heads ? h0 + it : h0;
 #pragma unroll
-    for (int it = 0; it < QKV_ITEMS; ++it) {
-      const int64_t w = w0 + it < items ? w0 + it : w0;
-      const int hd = (int)(w % a.heads), m = (int)(w / a.heads);
+        for (int which = 0; which < 2; ++which) {
+          bf16x4_load(xrow + which * a.d + hd * 128, x[it][which]);
+          bf16x4_load(grow + which * a.d + hd * 128, g[it][which]);
+        }
+      }
 #pragma unroll
-      for (int which = 0; which < 2; ++which) {
-        bf16x4_load(static_cast<const bf16*>(a.qkv) + (int64_t)m * a.ld_qkv + which * a.d + hd * 128 + 4 * lane,
-                    x[it][which]);
-        bf16x4_load(static_cast<const bf16*>(b.dqk) + (int64_t)m * b.ld_dqk + which * a.d + hd * 128 + 4 * lane,
-                    g[it][which]);
+      for (int it = 0; it < QKV_ITEMS; ++it) {
+        const int hd = h0 + it;
+        if (hd >= a.heads) break;
+#pragma unroll
+        for (int which = 0; which < 2; ++which) {
+          const float4 sc4 = *reinterpret_cast<const float4*>(&scl[which * 2 + (txt ? 0 : 1)][4 * lane]);
+          const float sc[4] = {sc4.x, sc4.y, sc4.z, sc4.w};
+          const float* xv = x[it][which];
+          const float r = (which == 0 ? a.rq : a.rk)[(int64_t)m * a.heads + hd];
+          float u[4], dy[4];
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {  // undo the rotation of the incoming gradient
+            const float g0 = g[it][which][2 * e], g1 = g[it][which][2 * e + 1];
+            dy[2 * e] = g0 * cs[e] + g1 * sn[e];
+            dy[2 * e + 1] = -g0 * sn[e] + g1 * cs[e];
+          }
+          float xu = 0.f;
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            rowacc[which][e] += dy[e] * xv[e] * r;
+            u[e] = dy[e] * sc[e];
+            xu += xv[e] * u[e];
+          }
+          xu = warp_sum(xu);
+          float dx[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) dx[e] = r * u[e] - xv[e] * r * r * r * xu / 128.f;
+          bf16x4_store(grow + which * a.d + hd * 128, dx);
+        }
       }
     }
 #pragma unroll
-    for (int it = 0; it < QKV_ITEMS; ++it) {
-      const int64_t w = w0 + it;
-      if (w >= items) break;
-      const int hd = (int)(w % a.heads), m = (int)(w / a.heads);
-      const int n = m % a.N;
-      const bool txt = n < a.n_txt;
-      float cs[2], sn[2];
-      rope_lane(a, rope_tab, n, lane, cs, sn);
-#pragma unroll
-      for (int which = 0; which < 2; ++which) {
-        const float4 sc4 = *reinterpret_cast<const float4*>(&scl[which * 2 + (txt ? 0 : 1)][4 * lane]);
-        const float sc[4] = {sc4.x, sc4.y, sc4.z, sc4.w};
-        const float* xv = x[it][which];
-        const float r = (which == 0 ? a.rq : a.rk)[(int64_t)m * a.heads + hd];
-        float u[4], dy[4];
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {  // undo the rotation of the incoming gradient
-          const float g0 = g[it][which][2 * e], g1 = g[it][which][2 * e + 1];
-          dy[2 * e] = g0 * cs[e] + g1 * sn[e];
-          dy[2 * e + 1] = -g0 * sn[e] + g1 * cs[e];
-        }
-        float xu = 0.f;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float ds = dy[e] * xv[e] * r;
-          if (txt)
-            acc[which * 2][e] += ds;
-          else
-            acc[which * 2 + 1][e] += ds;
-          u[e] = dy[e] * sc[e];
-          xu += xv[e] * u[e];
-        }
-        xu = warp_sum(xu);
-        float dx[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) dx[e] = r * u[e] - xv[e] * r * r * r * xu / 128.f;
-        bf16x4_store(static_cast<bf16*>(b.dqk) + (int64_t)m * b.ld_dqk + which * a.d + hd * 128 + 4 * lane, dx);
-      }
+    for (int which = 0; which < 2; ++which) {
+      float4& q = wpart[(which * 2 + (txt ? 0 : 1)) * 32 + lane];
+      q.x += rowacc[which][0]; q.y += rowacc[which][1]; q.z += rowacc[which][2]; q.w += rowacc[which][3];
     }
   }
-#pragma unroll
-  for (int i = 0; i < 4; ++i)
-#pragma unroll
-    for (int e = 0; e < 4; ++e) part[warp][i][4 * lane + e] = acc[i][e];
   __syncthreads();
   for (int t = threadIdx.x; t < 4 * 128; t += QKN_THREADS) {
     const int i = t / 128, c = t % 128;
@@ -1237,8 +1233,8 @@ int launch_qk_norm_rope_fwd(const QkNormRope& a, cudaStream_t s) {
   const int64_t blocks = ((int64_t)a.M * a.heads + QKN_WARPS - 1) / QKN_WARPS;
   const int tok = prof_start(s);
   if (qkn_vector(a)) {
-    const int64_t vb = ceil_div((int64_t)a.M * a.heads, (int64_t)QKN_WARPS * QKV_ITEMS);
-    const int cap = 16 * sm_count();
+    const int64_t vb = ceil_div((int64_t)a.M, (int64_t)QKN_WARPS);
+    const int cap = 4 * sm_count();  // the resident blocks (4 per SM)
     qk_norm_rope_fwd_v_kernel<<<(int)(vb < cap ? vb : cap), QKN_THREADS, qkn_table_bytes(a), s>>>(a);
   } else {
     qk_norm_rope_fwd_kernel<<<(int)(blocks < 65536 ? blocks : 65536), QKN_THREADS, 0, s>>>(a);
@@ -1261,7 +1257,7 @@ int launch_qk_norm_rope_bwd(const QkNormRopeBwd& a, cudaStream_t s) {
   const int tok = prof_start(s);
   if (qkn_vector(f) && a.ld_dqk % 4 == 0 && aligned8(a.dqk)) {
     // a few blocks per SM: each block ends in 4 x 128 scale-gradient atomics
-    const int64_t vb = ceil_div((int64_t)f.M * f.heads, (int64_t)QKN_WARPS * QKV_ITEMS);
+    const int64_t vb = ceil_div((int64_t)f.M, (int64_t)QKN_WARPS);
     const int vcap = 3 * sm_count();  // the resident blocks (80 registers, 3 per SM)
     qk_norm_rope_bwd_v_kernel<<<(int)(vb < vcap ? vb : vcap), QKN_THREADS, qkn_table_bytes(f), s>>>(a);
   } else {

@@ -161,3 +161,57 @@ extern "C" int jagg_test_ln_gate_bwd(int M, int d, int rows_per_seq, int do_ln, 
   a.dtype = dtype;
   return launch_ln_gate_bwd(a, stream);
 }
+
+static QkNormRope qkn_args(const void* qkv, int64_t ld_qkv, int M, int N, int d, int heads, int n_txt, int gw,
+                           const void* qscale, const void* kscale, int rope, int dtype) {
+  QkNormRope q{};
+  q.qkv = qkv; q.ld_qkv = ld_qkv;
+  q.M = M; q.N = N; q.d = d; q.heads = heads; q.n_txt = n_txt; q.gw = gw;
+  q.qscale_txt = q.qscale_img = qscale;
+  q.kscale_txt = q.kscale_img = kscale;
+  q.rope = rope;
+  q.dtype = dtype;
+  return q;
+}
+
+static int qkn_check(const char* name, int M, int N, int d, int heads, int n_txt, int gw, int rope, int dtype) {
+  JAGG_CHECK_ARG(M > 0 && N > 0 && M % N == 0, "%s: M=%d not a whole number of %d-token sequences", name, M, N);
+  JAGG_CHECK_ARG(dtype == JAGG_DTYPE_F32 || dtype == JAGG_DTYPE_BF16, "%s: bad dtype", name);
+  JAGG_CHECK_ARG(n_txt >= 0 && n_txt <= N, "%s: n_txt=%d outside [0, %d]", name, n_txt, N);
+  JAGG_CHECK_ARG(!rope || (gw > 0 && (N - n_txt) % gw == 0), "%s: %d image tokens not a grid %d wide", name,
+                 N - n_txt, gw);
+  (void)d; (void)heads;
+  return JAGG_OK;
+}
+
+extern "C" int jagg_test_qk_norm_rope_fwd(const void* qkv, int64_t ld_qkv, int M, int N, int d, int heads, int n_txt,
+                                          int gw, const void* qscale, const void* kscale, int rope, void* qk_out,
+                                          float* rq, float* rk, int dtype, cudaStream_t stream) {
+  JAGG_TRY(qkn_check("jagg_test_qk_norm_rope_fwd", M, N, d, heads, n_txt, gw, rope, dtype));
+  JAGG_CHECK_ARG(qkv && qscale && kscale && qk_out && rq && rk, "jagg_test_qk_norm_rope_fwd: null pointer");
+  QkNormRope q = qkn_args(qkv, ld_qkv, M, N, d, heads, n_txt, gw, qscale, kscale, rope, dtype);
+  q.qk_out = qk_out; q.rq = rq; q.rk = rk;
+  return launch_qk_norm_rope_fwd(q, stream);
+}
+
+extern "C" int jagg_test_qk_norm_rope_bwd(const void* qkv, int64_t ld_qkv, int M, int N, int d, int heads, int n_txt,
+                                          int gw, const void* qscale, const void* kscale, int rope, const float* rq,
+                                          const float* rk, void* dqk, int64_t ld_dqk, float* dqscale, float* dkscale,
+                                          int dtype, cudaStream_t stream) {
+  JAGG_TRY(qkn_check("jagg_test_qk_norm_rope_bwd", M, N, d, heads, n_txt, gw, rope, dtype));
+  JAGG_CHECK_ARG(qkv && qscale && kscale && rq && rk && dqk && dqscale && dkscale,
+                 "jagg_test_qk_norm_rope_bwd: null pointer");
+  QkNormRopeBwd b{};
+  b.f = qkn_args(qkv, ld_qkv, M, N, d, heads, n_txt, gw, qscale, kscale, rope, dtype);
+  b.f.rq = const_cast<float*>(rq); b.f.rk = const_cast<float*>(rk);
+  b.dqk = dqk; b.ld_dqk = ld_dqk;
+  b.dqs_txt = b.dqs_img = dqscale;
+  b.dks_txt = b.dks_img = dkscale;
+  return launch_qk_norm_rope_bwd(b, stream);
+}
+
+extern "C" int jagg_test_colsum(const void* X, int x_f32, int rows, int cols, int64_t ld, float* db,
+                                cudaStream_t stream) {
+  JAGG_CHECK_ARG(X && db && rows > 0 && cols > 0 && ld >= cols, "jagg_test_colsum: bad arguments");
+  return launch_colsum(X, x_f32, x_f32 ? JAGG_DTYPE_F32 : JAGG_DTYPE_BF16, rows, cols, ld, db, stream);
+}

@@ -453,3 +453,85 @@ def test_ln_gate_backward_kernels(d, M, rps, ln, gate, dtype):
         assert _rel(dgate - 0.25, torch.zeros(S, d, **f).index_add_(0, seq, dh_ref * yf)) < 1e-5
         sums = torch.zeros(S, d, **f).index_add_(0, seq, dh_ref)
         assert _rel(dbias + 0.5, (gate_v * sums).sum(0)) < 1e-5
+
+
+def _qkn_reference(x, N, n_txt, gw, dh, scale, rope):
+    """RMSNorm per head (eps 1e-6, learned scale) then 2D RoPE: the first dh/4 rotated pairs by
+    the patch row, the rest by the column, pairs (2i, 2i+1), theta_i = 10000^(-2i/(dh/2)),
+    text tokens (the first n_txt of each sequence) not rotated.  x [M, H, dh] f32."""
+    M, H, _ = x.shape
+    y = x * torch.rsqrt((x * x).mean(-1, keepdim=True) + 1e-6) * scale
+    if not rope:
+        return y
+    n = torch.arange(M, device=x.device) % N
+    tok = (n - n_txt).clamp(min=0)
+    npair = dh // 4
+    i = torch.arange(npair, device=x.device, dtype=torch.float32)
+    theta = 10000.0 ** (-2.0 * i / (dh // 2))
+    pos = torch.cat([(tok // gw)[:, None].float().expand(M, npair), (tok % gw)[:, None].float().expand(M, npair)], 1)
+    ang = pos * torch.cat([theta, theta])[None, :]
+    ang = torch.where((n < n_txt)[:, None], torch.zeros_like(ang), ang)
+    c, s = torch.cos(ang)[:, None, :], torch.sin(ang)[:, None, :]
+    y0, y1 = y[..., 0::2], y[..., 1::2]
+    out = torch.empty_like(y)
+    out[..., 0::2] = y0 * c - y1 * s
+    out[..., 1::2] = y0 * s + y1 * c
+    return out
+
+
+@pytest.mark.parametrize("dh,H,N,n_txt,gw,B,dtype,rope", [
+    (128, 4, 1536, 512, 32, 2, torch.bfloat16, True),   # Flux single block: vectorised kernels
+    (128, 3, 1024, 0, 32, 2, torch.bfloat16, True),     # image stream of a double block
+    (128, 2, 512, 512, 32, 3, torch.bfloat16, True),    # text stream: no rotation
+    (128, 2, 300, 44, 16, 2, torch.bfloat16, True),     # ragged sequence, 16 x 16 grid
+    (64, 3, 300, 44, 16, 2, torch.bfloat16, True),      # head dim 64: the per-element kernels
+    (32, 4, 24, 8, 4, 3, torch.float32, True),
+    (128, 2, 256, 0, 16, 1, torch.bfloat16, False)])
+def test_qk_norm_rope_kernels(dh, H, N, n_txt, gw, B, dtype, rope):
+    """Per-head RMSNorm + 2D RoPE forward (normalised, rotated q and k; 1/rms of each) and its
+    backward (gradients of the raw q, k in place; the scale gradients) against PyTorch fp32
+    autograd on the same inputs, in the model's layout (q, k inside a [M, 3d] buffer, the
+    gradient inside a wider one)."""
+    torch.manual_seed(dh + N + n_txt)
+    dev = "cuda"
+    d, M = H * dh, B * N
+    qkv = (torch.randn(M, 3 * d, device=dev) * 2).to(dtype)
+    qs, ks = (1 + 0.1 * torch.randn(dh, device=dev)).to(dtype), (1 + 0.1 * torch.randn(dh, device=dev)).to(dtype)
+    qk = torch.empty(M, 2 * d, device=dev, dtype=dtype)
+    rq, rk = torch.empty(M, H, device=dev), torch.empty(M, H, device=dev)
+    jg.test_qk_norm_rope_fwd(qkv, M, N, H, n_txt, gw, qs, ks, qk, rq, rk, rope=rope)
+    ld = 3 * d + 64
+    g_up = (torch.randn(M, ld, device=dev)).to(dtype)
+    dqk = g_up.clone()
+    dqs, dks = torch.zeros(dh, device=dev), torch.zeros(dh, device=dev)
+    jg.test_qk_norm_rope_bwd(qkv, M, N, H, n_txt, gw, qs, ks, rq, rk, dqk, dqs, dks, rope=rope)
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    xq = qkv[:, :d].float().view(M, H, dh).requires_grad_()
+    xk = qkv[:, d:2 * d].float().view(M, H, dh).requires_grad_()
+    sq, sk = qs.float().requires_grad_(), ks.float().requires_grad_()
+    yq = _qkn_reference(xq, N, n_txt, gw, dh, sq, rope)
+    yk = _qkn_reference(xk, N, n_txt, gw, dh, sk, rope)
+    tol = 1e-2 if dtype == torch.bfloat16 else 1e-5
+    assert _rel(qk[:, :d].float(), yq.reshape(M, d)) < tol
+    assert _rel(qk[:, d:].float(), yk.reshape(M, d)) < tol
+    ref_r = torch.rsqrt((xq.detach() ** 2).mean(-1) + 1e-6)
+    assert _rel(rq, ref_r) < 1e-5
+    (yq.reshape(M, d) * g_up[:, :d].float()).sum().add((yk.reshape(M, d) * g_up[:, d:2 * d].float()).sum()).backward()
+    assert _rel(dqk[:, :d].float(), xq.grad.reshape(M, d)) < 2 * tol
+    assert _rel(dqk[:, d:2 * d].float(), xk.grad.reshape(M, d)) < 2 * tol
+    assert torch.equal(dqk[:, 2 * d:], g_up[:, 2 * d:]), "columns past q, k changed"
+    assert _rel(dqs, sq.grad) < 1e-4 and _rel(dks, sk.grad) < 1e-4
+
+
+@pytest.mark.parametrize("rows,cols,ld,dtype", [(36864, 3072, 3072, torch.bfloat16), (4096, 12288, 21504, torch.bfloat16),
+                                                (333, 2304, 2304, torch.bfloat16), (97, 200, 210, torch.float32)])
+def test_colsum_kernels(rows, cols, ld, dtype):
+    """Bias-gradient column sums (db += sum over rows, into a nonzero db) against PyTorch."""
+    torch.manual_seed(rows + cols)
+    X = torch.randn(rows, ld, device="cuda").to(dtype)
+    db = torch.full((cols,), 0.5, device="cuda")
+    jg.test_colsum(X[:, :cols], db)
+    torch.cuda.synchronize()
+    ref = X[:, :cols].double().sum(0) + 0.5
+    assert _rel(db, ref) < 1e-5
