@@ -196,8 +196,11 @@ constexpr int TC_MAX_EPI_WARPS = 8;
 __host__ __device__ constexpr int tc_threads(int ew) { return 64 + 32 * ew; }
 
 // AUX: the instance can run EPI_MUL_AUX (the input-gradient products, K-major A and
-// MN-major B); the others need no shared memory for a multiplier.
-template <int BN, bool AUX, int EW>
+// MN-major B): 1 = every multiplier chunk of a warp's tile loaded at once (tiles of at most
+// 128 columns), 2 = a two-slot ring per epilogue warp refilled chunk by chunk (256-column
+// tiles: for long K, where the main loop of the next tile covers the epilogue's loads);
+// 0 = no shared memory for a multiplier.
+template <int BN, int AUX, int EW>
 struct TcCfg {
   static constexpr int SPLIT = EW / 4;           // chunk stride of an epilogue warp
   static constexpr int NSTG = EW == 4 ? 2 : 1;   // staging chunks per epilogue warp
@@ -208,7 +211,8 @@ struct TcCfg {
   // chunk of 32 x 32 outputs (4 KB as f32; the bf16 output of EPI_MUL_AUX uses 2 KB), and
   // for EPI_MUL_AUX this warp's multiplier chunks (BN / 64 of 32 x 32 bf16) after it.
   static constexpr int CHUNK_BF16 = 32 * 32 * 2;
-  static constexpr int AUX_WARP_BYTES = NSTG * CHUNK_BF16 + ((BN / 32 + SPLIT - 1) / SPLIT) * CHUNK_BF16;
+  static constexpr int AUX_SLOTS = AUX == 2 ? 2 : (BN / 32 + SPLIT - 1) / SPLIT;
+  static constexpr int AUX_WARP_BYTES = NSTG * CHUNK_BF16 + AUX_SLOTS * CHUNK_BF16;
   static constexpr int EPI_WARP_BYTES =
       AUX && AUX_WARP_BYTES > NSTG * 2 * CHUNK_BF16 ? AUX_WARP_BYTES : NSTG * 2 * CHUNK_BF16;
   static constexpr int EPI_BYTES = EW * EPI_WARP_BYTES;
@@ -223,7 +227,7 @@ struct TcCfg {
   static_assert(SMEM_BYTES <= MAX_SMEM, "shared memory budget");
 };
 
-template <int BN, bool A_MN, bool B_MN, bool AUX, int EW>
+template <int BN, bool A_MN, bool B_MN, int AUX, int EW>
 __global__ void __launch_bounds__(tc_threads(EW), 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmX, TcParams p) {
@@ -237,7 +241,7 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
   uint64_t* empty = full + STAGES;
   uint64_t* tfull = empty + STAGES;
   uint64_t* tempty = tfull + 2;
-  uint64_t* auxbar = tempty + 2;  // one per epilogue warp
+  uint64_t* auxbar = tempty + 2;  // one per epilogue warp (two, one per ring slot, when AUX == 2)
   uint64_t* drainbar = auxbar + TC_MAX_EPI_WARPS;  // the MMA thread's drain after a give-up
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drainbar + 1);
   __shared__ volatile int abort_flag;
@@ -255,7 +259,7 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
       ptx::mbar_init(&tfull[a], 1);
       ptx::mbar_init(&tempty[a], EW);
     }
-    for (int q = 0; q < EW; ++q) ptx::mbar_init(&auxbar[q], 1);
+    for (int q = 0; q < (AUX == 2 ? 2 * EW : EW); ++q) ptx::mbar_init(&auxbar[q], 1);
     ptx::mbar_init(drainbar, 1);
     ptx::fence_mbar_init();
     ptx::prefetch_tmap(&tmA);
@@ -518,6 +522,7 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
     uint8_t* auxs = stg + Cfg::NSTG * Cfg::CHUNK_BF16;  // EPI_MUL_AUX only (bf16 output)
     int acc = 0, sbuf = 0;
     uint32_t acc_phase = 0, aux_phase = 0;
+    uint32_t ring_phase[2] = {0u, 0u};  // AUX == 2: the phase each ring slot waits for next
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
       int tm, tn, ks;
       decode(t, tm, tn, ks);
@@ -527,20 +532,37 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
       const int live_chunks = min(BN / 32, (p.e.N - tn * BN + 31) / 32);
       const int my_chunks = live_chunks > half ? (live_chunks - half + SPLIT - 1) / SPLIT : 0;
       const bool aux_load = mul && rows_live && my_chunks > 0;
+      // AUX == 2: multiplier chunk i of the tile into ring slot i % 2 (this warp's chunks
+      // i < 2 now, chunk i + 2 once chunk i has been used)
+      auto ring_load = [&](int i) {
+        ptx::mbar_arrive_expect_tx(&auxbar[2 * ew + (i & 1)], Cfg::CHUNK_BF16);
+        ptx::tma_load_2d(auxs + (i & 1) * Cfg::CHUNK_BF16, &tmX, &auxbar[2 * ew + (i & 1)],
+                         tn * BN + (half + SPLIT * i) * 32, m0);
+      };
       if (aux_load) {
         // this warp's multiplier chunks of the tile; it finished reading the previous tile's
         __syncwarp();
         if (lane == 0) {
-          ptx::mbar_arrive_expect_tx(&auxbar[ew], my_chunks * Cfg::CHUNK_BF16);
-          for (int i = 0; i < my_chunks; ++i)
-            ptx::tma_load_2d(auxs + i * Cfg::CHUNK_BF16, &tmX, &auxbar[ew], tn * BN + (half + SPLIT * i) * 32,
-                             m0);
+          if constexpr (AUX == 2) {
+            for (int i = 0; i < 2 && i < my_chunks; ++i) ring_load(i);
+          } else {
+            ptx::mbar_arrive_expect_tx(&auxbar[ew], my_chunks * Cfg::CHUNK_BF16);
+            for (int i = 0; i < my_chunks; ++i)
+              ptx::tma_load_2d(auxs + i * Cfg::CHUNK_BF16, &tmX, &auxbar[ew], tn * BN + (half + SPLIT * i) * 32,
+                               m0);
+          }
         }
       }
       bool ok = ptx::mbar_wait(&tfull[acc], acc_phase);
-      if (aux_load) {  // waited for even after a give-up: the multiplier load is in flight
+      if (aux_load && AUX != 2) {  // waited for even after a give-up: the multiplier load is in flight
         ok = ptx::mbar_wait(&auxbar[ew], aux_phase) && ok;
         aux_phase ^= 1u;
+      }
+      if (aux_load && AUX == 2 && !ok) {  // a give-up: wait for the ring loads in flight
+        for (int i = 0; i < 2 && i < my_chunks; ++i) {
+          ptx::mbar_wait(&auxbar[2 * ew + i], ring_phase[i]);
+          ring_phase[i] ^= 1u;
+        }
       }
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) { abort_flag = 1; break; }
@@ -564,13 +586,31 @@ __global__ void __launch_bounds__(tc_threads(EW), 1)
           }
         }
         if (mul) {
-          const uint8_t* ar = auxs + (c / SPLIT) * Cfg::CHUNK_BF16 + lane * 64;
+          const int ci = (c - half) / SPLIT;  // this warp's chunk index within the tile
+          if constexpr (AUX == 2) {
+            // a give-up leaves the slot's load waited for; the chunk is then not stored
+            const bool got = __all_sync(0xffffffffu, ptx::mbar_wait(&auxbar[2 * ew + (ci & 1)], ring_phase[ci & 1]));
+            ring_phase[ci & 1] ^= 1u;
+            if (!got) {
+              abort_flag = 1;
+              if (ci + 1 < my_chunks) {  // the other slot's load is in flight
+                ptx::mbar_wait(&auxbar[2 * ew + ((ci + 1) & 1)], ring_phase[(ci + 1) & 1]);
+                ring_phase[(ci + 1) & 1] ^= 1u;
+              }
+              break;
+            }
+          }
+          const uint8_t* ar = auxs + (AUX == 2 ? (ci & 1) : ci) * Cfg::CHUNK_BF16 + lane * 64;
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
             const uint4 raw = *reinterpret_cast<const uint4*>(ar + ((j ^ ((lane >> 1) & 3)) << 4));
             const bf16* h = reinterpret_cast<const bf16*>(&raw);
 #pragma unroll
             for (int i = 0; i < 8; ++i) v[j * 8 + i] *= __bfloat162float(h[i]);
+          }
+          if constexpr (AUX == 2) {
+            __syncwarp();  // every lane has read the slot: refill it with chunk ci + 2
+            if (lane == 0 && ci + 2 < my_chunks) ring_load(ci + 2);
           }
         }
         // the staging chunk's previous TMA has read it
@@ -918,7 +958,7 @@ int validate(const GemmArgs& g) {
   return JAGG_OK;
 }
 
-template <int BN, bool A_MN, bool B_MN, bool AUX, int EW = 4>
+template <int BN, bool A_MN, bool B_MN, int AUX, int EW = 4>
 int launch_tc(const GemmArgs& g, cudaStream_t stream) {
   using Cfg = TcCfg<BN, AUX, EW>;
   CUtensorMap ta, tb;
@@ -973,35 +1013,38 @@ int launch_tc(const GemmArgs& g, cudaStream_t stream) {
 template <bool A_MN, bool B_MN>
 int dispatch_bn(const GemmArgs& g, cudaStream_t stream) {
   // The multiplier epilogue needs its own shared memory: the input-gradient instance
-  // (K-major A, MN-major B) with BN <= 128.
+  // (K-major A, MN-major B), with every chunk of a warp's tile (BN <= 128) or a two-slot
+  // ring (BN = 256).
   JAGG_CHECK_ARG(g.tile_n == 0 || g.tile_n == 64 || g.tile_n == 128 || g.tile_n == 256, "gemm: tile width %d",
                  g.tile_n);
   if constexpr (!A_MN && B_MN) {
     if (staged_mode(g) == STAGED_MUL_AUX) {
-      JAGG_CHECK_ARG(g.tile_n != 256, "gemm: the multiplier epilogue uses tiles of at most 128 columns");
-      if (g.tile_n == 64 || (g.tile_n == 0 && g.N < 128)) return launch_tc<64, A_MN, B_MN, true>(g, stream);
-      return launch_tc<128, A_MN, B_MN, true>(g, stream);
+      if (g.tile_n == 64 || (g.tile_n == 0 && g.N < 128)) return launch_tc<64, A_MN, B_MN, 1>(g, stream);
+      // 256-column tiles with the multiplier ring when K is long enough for the next tile's
+      // main loop (K / 64 k-blocks) to cover the epilogue's chunk loads
+      if (g.tile_n == 256 || (g.tile_n == 0 && g.N >= 256 && g.K >= 2048)) return launch_tc<256, A_MN, B_MN, 2>(g, stream);
+      return launch_tc<128, A_MN, B_MN, 1>(g, stream);
     }
   }
   if constexpr (!A_MN && !B_MN) {
     // the forward products' arithmetic-heavy epilogues (GELU, gated residual) on 8 warps
     if (staged_mode(g) == STAGED_ROWS) {
       const int nsm = sm_count();
-      if (g.tile_n == 64 || (g.tile_n == 0 && g.N < 128)) return launch_tc<64, false, false, false, 8>(g, stream);
-      if (g.tile_n == 128) return launch_tc<128, false, false, false, 8>(g, stream);
+      if (g.tile_n == 64 || (g.tile_n == 0 && g.N < 128)) return launch_tc<64, false, false, 0, 8>(g, stream);
+      if (g.tile_n == 128) return launch_tc<128, false, false, 0, 8>(g, stream);
       if (g.tile_n == 256 || (g.tile_n == 0 && g.N >= 256 && tile_cost(g, 256, nsm) < tile_cost(g, 128, nsm)))
-        return launch_tc<256, false, false, false, 8>(g, stream);
-      return launch_tc<128, false, false, false, 8>(g, stream);
+        return launch_tc<256, false, false, 0, 8>(g, stream);
+      return launch_tc<128, false, false, 0, 8>(g, stream);
     }
   }
-  if (g.tile_n == 64 || (g.tile_n == 0 && g.N < 128)) return launch_tc<64, A_MN, B_MN, false>(g, stream);
-  if (g.tile_n == 128) return launch_tc<128, A_MN, B_MN, false>(g, stream);
-  if (g.tile_n == 256) return launch_tc<256, A_MN, B_MN, false>(g, stream);
+  if (g.tile_n == 64 || (g.tile_n == 0 && g.N < 128)) return launch_tc<64, A_MN, B_MN, 0>(g, stream);
+  if (g.tile_n == 128) return launch_tc<128, A_MN, B_MN, 0>(g, stream);
+  if (g.tile_n == 256) return launch_tc<256, A_MN, B_MN, 0>(g, stream);
   // Wider tiles halve the B-operand traffic per FLOP (the products are bound by L2
   // bandwidth at 128 x 128), at the price of coarser waves over the SMs.
   const int nsm = sm_count();
-  if (g.N >= 256 && tile_cost(g, 256, nsm) < tile_cost(g, 128, nsm)) return launch_tc<256, A_MN, B_MN, false>(g, stream);
-  return launch_tc<128, A_MN, B_MN, false>(g, stream);
+  if (g.N >= 256 && tile_cost(g, 256, nsm) < tile_cost(g, 128, nsm)) return launch_tc<256, A_MN, B_MN, 0>(g, stream);
+  return launch_tc<128, A_MN, B_MN, 0>(g, stream);
 }
 
 bool tc_eligible(const GemmArgs& g) {

@@ -62,9 +62,10 @@ def test_tcgen05_tile_widths(M, N, K, a_mn, b_mn, tile_n):
     assert _rel(C, ref) < 1e-5
     assert _rel(Cb.float(), ref + bias.float()) < 5e-3
     assert _rel(G, G0 + ref) < 1e-5
-    if not a_mn and b_mn and tile_n != 256:
-        # the multiplier epilogue of the input-gradient products (tiles of at most 128
-        # columns), bf16 output into a wider buffer
+    if not a_mn and b_mn:
+        # the multiplier epilogue of the input-gradient products (every chunk of a warp's
+        # tile at once up to 128 columns, a two-slot ring per warp at 256), bf16 output into
+        # a wider buffer
         X = torch.rand(M, N, device=dev).bfloat16()
         O = torch.full((M, N + 8), 3.0, device=dev, dtype=torch.bfloat16)
         jg.test_gemm(_desc(M, N, K, As, lda, a_mn, Bs, ldb, b_mn, jg.DTYPE_BF16, O, N + 8, jg.DTYPE_BF16, epi=3,
@@ -535,3 +536,29 @@ def test_colsum_kernels(rows, cols, ld, dtype):
     torch.cuda.synchronize()
     ref = X[:, :cols].double().sum(0) + 0.5
     assert _rel(db, ref) < 1e-5
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 600, 2112), (1000, 768, 3072), (128, 1280, 4096)])
+def test_multiplier_epilogue_long_k(M, N, K):
+    """The multiplier epilogue at long K, where the library picks 256-column tiles with the
+    two-slot multiplier ring (the fc2 / lin2 input gradients at the Flux widths), ragged
+    rows and column tiles, against the same product at 128 columns and PyTorch fp32."""
+    torch.manual_seed(M + N + K)
+    dev = "cuda"
+    A = torch.randn(M, K, device=dev).bfloat16()
+    B = (torch.randn(N, K, device=dev) / math.sqrt(K)).bfloat16()
+    Bt = B.t().contiguous()
+    X = torch.rand(M, N, device=dev).bfloat16()
+    ref = (A.float() @ B.float().t()) * X.float()
+    outs = []
+    for tile_n in (0, 128):
+        O = torch.full((M, N + 8), 3.0, device=dev, dtype=torch.bfloat16)
+        jg.test_gemm(_desc(M, N, K, A, K, 0, Bt, N, 1, jg.DTYPE_BF16, O, N + 8, jg.DTYPE_BF16, epi=3, aux=X, ld_aux=N,
+                           tile_n=tile_n))
+        outs.append(O)
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    for O in outs:
+        assert _rel(O[:, :N].float(), ref) < 5e-3
+        assert torch.all(O[:, N:] == 3.0)
+    assert _rel(outs[0][:, :N].float(), outs[1][:, :N].float()) < 5e-3
