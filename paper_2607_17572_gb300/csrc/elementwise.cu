@@ -890,8 +890,9 @@ __global__ void __launch_bounds__(QKN_THREADS) qk_norm_rope_bwd_kernel(QkNormRop
 // in 8-byte vectors and each lane's RMSNorm scales and RoPE frequencies are fixed for the
 // whole kernel.  The angles are the ones rope_angle forms (same expressions), so the forward
 // rotation and its inverse in the backward agree bit for bit.  A warp walks rows, each row's
-// heads two at a time (2 KB of loads in flight per warp in the backward).
-constexpr int QKV_ITEMS = 2;
+// heads two (backward) or four (forward) at a time: 2 KB of loads in flight per warp.
+constexpr int QKV_ITEMS = 2;      // heads per warp iteration of the backward
+constexpr int QKV_ITEMS_FWD = 4;  // and of the forward (fewer live registers)
 
 __device__ __forceinline__ void bf16x4_load(const bf16* p, float (&v)[4]) {
   const uint2 raw = *reinterpret_cast<const uint2*>(p);
@@ -956,16 +957,16 @@ __global__ void __launch_bounds__(QKN_THREADS) qk_norm_rope_fwd_v_kernel(QkNormR
     rope_lane(a, rope_tab, n, lane, cs, sn);
     const bf16* row = static_cast<const bf16*>(a.qkv) + (int64_t)m * a.ld_qkv + 4 * lane;
     bf16* out = static_cast<bf16*>(a.qk_out) + (int64_t)m * 2 * a.d + 4 * lane;
-    for (int h0 = 0; h0 < a.heads; h0 += QKV_ITEMS) {
-      float x[QKV_ITEMS][2][4];
+    for (int h0 = 0; h0 < a.heads; h0 += QKV_ITEMS_FWD) {
+      float x[QKV_ITEMS_FWD][2][4];
 #pragma unroll
-      for (int it = 0; it < QKV_ITEMS; ++it) {
+      for (int it = 0; it < QKV_ITEMS_FWD; ++it) {
         const int hd = h0 + it < a.heads ? h0 + it : h0;
 #pragma unroll
         for (int which = 0; which < 2; ++which) bf16x4_load(row + which * a.d + hd * 128, x[it][which]);
       }
 #pragma unroll
-      for (int it = 0; it < QKV_ITEMS; ++it) {
+      for (int it = 0; it < QKV_ITEMS_FWD; ++it) {
         const int hd = h0 + it;
         if (hd >= a.heads) break;
 #pragma unroll
@@ -1234,7 +1235,7 @@ int launch_qk_norm_rope_fwd(const QkNormRope& a, cudaStream_t s) {
   const int tok = prof_start(s);
   if (qkn_vector(a)) {
     const int64_t vb = ceil_div((int64_t)a.M, (int64_t)QKN_WARPS);
-    const int cap = 4 * sm_count();  // the resident blocks (4 per SM)
+    const int cap = 3 * sm_count();  // the resident blocks (77 registers, 3 per SM)
     qk_norm_rope_fwd_v_kernel<<<(int)(vb < cap ? vb : cap), QKN_THREADS, qkn_table_bytes(a), s>>>(a);
   } else {
     qk_norm_rope_fwd_kernel<<<(int)(blocks < 65536 ? blocks : 65536), QKN_THREADS, 0, s>>>(a);
