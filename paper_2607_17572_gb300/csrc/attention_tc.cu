@@ -1287,6 +1287,361 @@ __global__ void __launch_bounds__(FF_THREADS, 1) fa_fwd_tc_kernel(const __grid_c
   }
 }
 
+// ================================================================== forward, head dim 128
+// One pass over the keys with an online softmax.  Persistent over (pair of 128-query tiles A
+// and B, sequence, head) units; per unit the sequence's 128-key tiles stream through a K ring
+// and a V ring, each K and V tile serving both query tiles.  Tensor memory (512 columns):
+//   S_A [0, 128), S_B [128, 256)   S = Q K^T (f32); P written over it (bf16, two per column)
+//   O_A [256, 384), O_B [384, 512) O += P V (f32), accumulated over the keys
+// Issue order per key tile j: PV_A(j-1), S_A(j), PV_B(j-1), S_B(j), so the softmax of one
+// query tile runs while the products of the other do.  Softmax warps 2-5 own tile A, 6-9 tile
+// B, a thread per query row (no exchange between warps).  Each row keeps a reference maximum m: P = exp(scale (S - m)); when a tile's maximum
+// exceeds m by more than 8 / (scale log2 e) (P would pass 2^8), m moves up and the row's O (once
+// the previous P V product has finished) and running sum l are rescaled, so O is rescaled only
+// while the maximum is still climbing.  P goes to tensor memory in place of the S columns the
+// thread has read and is the A operand of P V.  At the end O / l leaves in bf16 and
+// lse = scale m + ln l.
+constexpr int FF2_THREADS = 320;  // 10 warps
+
+struct Ff2 {
+  static constexpr int D = 128, BQ = 128, BK = 128, NKS = 2, NVS = 3;
+  static constexpr int TILE = 128 * 128 * 2;  // 32 KB: 128 rows x 128 bf16, two 64-column chunks
+  static constexpr int OFF_Q = 0;             // Q_A, Q_B
+  static constexpr int OFF_K = OFF_Q + 2 * TILE;
+  static constexpr int OFF_V = OFF_K + NKS * TILE;
+  static constexpr int OFF_BAR = OFF_V + NVS * TILE;
+  static constexpr int NBAR = 24;
+  static constexpr int SMEM = OFF_BAR + NBAR * 8 + 16 + 1024;  // + alignment of the base to 1024 bytes
+  static_assert(SMEM <= 232448, "shared memory budget");
+  static constexpr uint32_t T_S = 0, T_O = 256;  // S_X at 128 X, O_X at 256 + 128 X
+};
+
+__global__ void __launch_bounds__(FF2_THREADS, 1) fa_fwd_tc128_kernel(const __grid_constant__ FfMaps maps,
+                                                                      FfParams p) {
+  using C = Ff2;
+  constexpr int BQ = C::BQ, BK = C::BK, D = C::D, NKS = C::NKS, NVS = C::NVS;
+  extern __shared__ uint8_t smem_ff2[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_ff2) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = sm + C::OFF_Q;
+  uint8_t* sK = sm + C::OFF_K;
+  uint8_t* sV = sm + C::OFF_V;
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sm + C::OFF_BAR);
+  uint64_t* kfull = bar;                // [NKS] a K tile landed
+  uint64_t* kempty = kfull + NKS;       // [NKS] both S products reading it are done
+  uint64_t* vfull = kempty + NKS;       // [NVS] a V tile landed
+  uint64_t* vempty = vfull + NVS;       // [NVS] both P V products reading it are done
+  uint64_t* qfull = vempty + NVS;       // the unit's Q_A, Q_B landed
+  uint64_t* qfree = qfull + 1;          // the unit's last S products are done
+  uint64_t* bar_s = qfree + 1;          // [2] S_X of a key tile in TMEM
+  uint64_t* pready = bar_s + 2;         // [2] P_X written (and O_X rescaled) by tile X's 4 warps
+  uint64_t* bar_pv = pready + 2;        // [2] the P_X V product of a key tile is done
+  uint64_t* ofree = bar_pv + 2;         // [2] tile X's 4 warps have read O_X
+  uint64_t* bar_drain = ofree + 2;      // the MMA thread's drain after a give-up
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar + C::NBAR);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int N = p.N;
+  const int nk = (N + BK - 1) / BK;
+  const int nq = (N + BQ - 1) / BQ;
+  const int npair = (nq + 1) / 2;
+  const int units = npair * p.B * p.heads;
+  // unit u: query tiles 2 (u % npair) and + 1 of sequence-head u / npair
+  auto unit_of = [&](int u, int& q0, int& b, int& h) {
+    const int bh = u / npair;
+    q0 = (u % npair) * 2 * BQ;
+    b = bh / p.heads;
+    h = bh % p.heads;
+  };
+  auto seg_of = [&](int r) { return r < p.n0 ? 0 : 1; };
+  auto row_in = [&](int r) { return r < p.n0 ? r : r - p.n0; };
+
+  if (threadIdx.x == 0) {
+    *abort_flag = 0;
+    for (int i = 0; i < NKS; ++i) {
+      ptx::mbar_init(&kfull[i], 1);
+      ptx::mbar_init(&kempty[i], 1);
+    }
+    for (int i = 0; i < NVS; ++i) {
+      ptx::mbar_init(&vfull[i], 1);
+      ptx::mbar_init(&vempty[i], 1);
+    }
+    ptx::mbar_init(qfull, 1);
+    ptx::mbar_init(qfree, 1);
+    for (int x = 0; x < 2; ++x) {
+      ptx::mbar_init(&bar_s[x], 1);
+      ptx::mbar_init(&pready[x], 4);
+      ptx::mbar_init(&bar_pv[x], 1);
+      ptx::mbar_init(&ofree[x], 4);
+    }
+    ptx::mbar_init(bar_drain, 1);
+    ptx::fence_mbar_init();
+    for (int sg = 0; sg < 2; ++sg) {
+      ptx::prefetch_tmap(&maps.q[sg]);
+      ptx::prefetch_tmap(&maps.k[sg]);
+      ptx::prefetch_tmap(&maps.v[sg]);
+    }
+  }
+  if (warp == 1) {
+    ptx::tmem_alloc(tmem_slot, 512);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      int gk = 0, gv = 0, i = 0, iq_last = -1;  // K / V tiles issued; the last unit whose Q was issued
+      bool ok = true;
+      for (int u = blockIdx.x; u < units && ok && !*abort_flag; u += gridDim.x, ++i) {
+        int q0, b, h;
+        unit_of(u, q0, b, h);
+        if (!ptx::mbar_wait(qfree, (i & 1) ^ 1)) { ok = false; break; }
+        iq_last = i;
+        ptx::mbar_arrive_expect_tx(qfull, 2 * C::TILE);
+        for (int x = 0; x < 2; ++x) {
+          // query tile B past the last query (odd tile count): a tile of zeros
+          const int qx = q0 + x * BQ < N ? q0 + x * BQ : q0;
+#pragma unroll
+          for (int c = 0; c < D / 64; ++c)
+            ptx::tma_load_3d(sQ + x * C::TILE + c * BQ * 128, &maps.q[seg_of(qx)], qfull,
+                             (int)(p.q_col0 + h * D + c * 64), row_in(qx), b);
+        }
+        for (int j = 0; j < nk && ok; ++j, ++gk, ++gv) {
+          const int k0 = j * BK, sg = seg_of(k0), r = row_in(k0);
+          const int ks = gk % NKS, vs = gv % NVS;
+          if (!ptx::mbar_wait(&kempty[ks], ((gk / NKS) & 1) ^ 1)) { ok = false; break; }
+          ptx::mbar_arrive_expect_tx(&kfull[ks], C::TILE);
+#pragma unroll
+          for (int c = 0; c < D / 64; ++c)
+            ptx::tma_load_3d(sK + ks * C::TILE + c * BK * 128, &maps.k[sg], &kfull[ks],
+                             (int)(p.k_col0 + h * D + c * 64), r, b);
+          if (!ptx::mbar_wait(&vempty[vs], ((gv / NVS) & 1) ^ 1)) { ok = false; ++gk; break; }
+          ptx::mbar_arrive_expect_tx(&vfull[vs], C::TILE);
+#pragma unroll
+          for (int c = 0; c < D / 64; ++c)
+            ptx::tma_load_3d(sV + vs * C::TILE + c * BK * 128, &maps.v[sg], &vfull[vs],
+                             (int)(p.v_col0 + h * D + c * 64), r, b);
+        }
+      }
+      if (!ok) *abort_flag = 1;
+      // after a give-up: wait (bounded) for the copies still landing before exiting
+      if (*abort_flag) {
+        if (iq_last >= 0) ptx::mbar_wait(qfull, iq_last & 1);
+        for (int k = 0; k < NKS && gk - 1 - k >= 0; ++k)
+          ptx::mbar_wait(&kfull[(gk - 1 - k) % NKS], ((gk - 1 - k) / NKS) & 1);
+        for (int k = 0; k < NVS && gv - 1 - k >= 0; ++k)
+          ptx::mbar_wait(&vfull[(gv - 1 - k) % NVS], ((gv - 1 - k) / NVS) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (ptx::elect_one()) {
+      constexpr uint32_t id_s = ptx::idesc_bf16(128, BK, false, false);  // S = Q K^T
+      constexpr uint32_t id_o = ptx::idesc_bf16(128, D, false, true);    // O += P V (A from TMEM)
+      bool ok = true;
+      int gk = 0, gv = 0, i = 0;
+      uint32_t pr_phase[2] = {0u, 0u};  // pready[X] phases consumed
+      auto issue_s = [&](int x, int ks) {  // S_X = Q_X K^T of K stage ks
+        const uint32_t aQ = ptx::smem_u32(sQ + x * C::TILE), aK = ptx::smem_u32(sK + ks * C::TILE);
+#pragma unroll
+        for (int k = 0; k < D / 16; ++k)
+          ptx::umma_bf16(tmem + C::T_S + x * 128, kmajor_desc(aQ, BQ, k), kmajor_desc(aK, BK, k), id_s, k > 0);
+        ptx::umma_commit(&bar_s[x]);
+      };
+      auto issue_pv = [&](int x, int vs, bool first) {  // O_X += P_X V of V stage vs
+        const uint32_t aV = ptx::smem_u32(sV + vs * C::TILE);
+#pragma unroll
+        for (int k = 0; k < BK / 16; ++k)
+          ptx::umma_bf16_ts(tmem + C::T_O + x * 128, tmem + C::T_S + x * 128 + k * 8, mnmajor_desc(aV, BK * 128, k),
+                            id_o, (!first || k > 0) ? 1u : 0u);
+        ptx::umma_commit(&bar_pv[x]);
+      };
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++i) {
+        if (!ptx::mbar_wait(qfull, i & 1)) { ok = false; break; }
+        // key tile 0: S_A, S_B
+        if (!ptx::mbar_wait(&kfull[gk % NKS], (gk / NKS) & 1)) { ok = false; break; }
+        ptx::tc_fence_after();
+        issue_s(0, gk % NKS);
+        issue_s(1, gk % NKS);
+        ptx::umma_commit(&kempty[gk % NKS]);
+        if (nk == 1) ptx::umma_commit(qfree);
+        ++gk;
+        for (int j = 1; j <= nk && ok; ++j) {
+          const int vs = gv % NVS;
+          for (int x = 0; x < 2 && ok; ++x) {
+            // P_X of key tile j - 1, then (j < nk) S_X of key tile j over it
+            if (!ptx::mbar_wait(&pready[x], pr_phase[x])) { ok = false; break; }
+            pr_phase[x] ^= 1u;
+            ptx::tc_fence_after();
+            if (j == 1 && i > 0) {  // O_X of the previous unit has been read
+              if (!ptx::mbar_wait(&ofree[x], (i - 1) & 1)) { ok = false; break; }
+              ptx::tc_fence_after();
+            }
+            if (x == 0 && !ptx::mbar_wait(&vfull[vs], (gv / NVS) & 1)) { ok = false; break; }
+            ptx::tc_fence_after();
+            issue_pv(x, vs, j == 1);
+            if (j < nk) {
+              if (x == 0 && !ptx::mbar_wait(&kfull[gk % NKS], (gk / NKS) & 1)) { ok = false; break; }
+              ptx::tc_fence_after();
+              issue_s(x, gk % NKS);
+            }
+          }
+          if (!ok) break;
+          ptx::umma_commit(&vempty[vs]);
+          ++gv;
+          if (j < nk) {
+            ptx::umma_commit(&kempty[gk % NKS]);
+            if (j == nk - 1) ptx::umma_commit(qfree);
+            ++gk;
+          }
+        }
+      }
+      if (!ok) *abort_flag = 1;
+      if (*abort_flag) {  // MMAs of this thread may still run: drain them before TMEM is freed
+        ptx::umma_commit(bar_drain);
+        ptx::mbar_wait(bar_drain, 0);
+      }
+    }
+  } else {
+    // ---------------------------------------------------------------- softmax, output
+    const int x = (warp - 2) >> 2;       // query tile A (warps 2-5) or B (6-9)
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;   // query row of the tile = TMEM lane
+    const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
+    const uint32_t tS = trow + C::T_S + x * 128, tO = trow + C::T_O + x * 128;
+    const float c2 = p.scale * kLog2eTc;
+    const float kRescale = 8.f / c2;      // P stays below 2^8 between rescales
+    bool ok = true;
+    int i = 0;
+    uint32_t s_phase = 0, pv_phase = 0;  // bar_s[x] / bar_pv[x] phases consumed
+    for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++i) {
+      int q0, b, h;
+      unit_of(u, q0, b, h);
+      float m = -INFINITY, l = 0.f;
+      for (int j = 0; j < nk; ++j) {
+        ok = __all_sync(0xffffffffu, ptx::mbar_wait(&bar_s[x], s_phase));
+        s_phase ^= 1u;
+        if (!ok || *abort_flag) { ok = false; *abort_flag = 1; break; }
+        ptx::tc_fence_after();
+        // The row maximum over columns 0-63 (read again below) and 64-127 (kept in registers):
+        // at most 96 of the row's values are live at once.
+        const int kv = N - j * BK;  // valid keys of the tile
+        float tmax = -INFINITY;
+        uint32_t rh[64];
+        ptx::tmem_ld_32x32b_x32(tS, *reinterpret_cast<uint32_t(*)[32]>(rh));
+        ptx::tmem_ld_32x32b_x32(tS + 32, *reinterpret_cast<uint32_t(*)[32]>(rh + 32));
+        ptx::tmem_ld_wait();
+#pragma unroll
+        for (int c = 0; c < 64; ++c)
+          if (c < kv) tmax = fmaxf(tmax, __uint_as_float(rh[c]));
+        ptx::tmem_ld_32x32b_x32(tS + 64, *reinterpret_cast<uint32_t(*)[32]>(rh));
+        ptx::tmem_ld_32x32b_x32(tS + 96, *reinterpret_cast<uint32_t(*)[32]>(rh + 32));
+        ptx::tmem_ld_wait();
+#pragma unroll
+        for (int c = 0; c < 64; ++c)
+          if (c + 64 < kv) tmax = fmaxf(tmax, __uint_as_float(rh[c]));
+        if (j == 0) {
+          m = tmax;
+        } else if (__any_sync(0xffffffffu, tmax > m + kRescale)) {
+          // the maximum of some row of the warp moved up: the whole warp (the tensor-memory
+          // accesses are warp-wide) rescales O and l to the new references once the previous
+          // P V product has finished; rows whose maximum stayed take the factor 1
+          const float mn = fmaxf(m, tmax);
+          const float f = ptx::ex2_approx((m - mn) * c2);
+          ok = __all_sync(0xffffffffu, ptx::mbar_wait(&bar_pv[x], pv_phase));
+          if (!ok) { *abort_flag = 1; break; }
+          ptx::tc_fence_after();
+#pragma unroll 1
+          for (int c = 0; c < D / 16; ++c) {  // 16 columns at a time: the S row stays in registers
+            uint32_t ro[16];
+            ptx::tmem_ld_32x32b_x16(tO + c * 16, ro);
+            ptx::tmem_ld_wait();
+#pragma unroll
+            for (int e = 0; e < 16; ++e) ro[e] = __float_as_uint(__uint_as_float(ro[e]) * f);
+            ptx::tmem_st_32x32b_x16(tO + c * 16, ro);
+          }
+          l *= f;
+          m = mn;
+        }
+        // rows whose reference stays: P = exp(scale (S - m)), at most 2^8
+        // P of columns 2c, 2c+1 goes to column c, over S values already read
+        const float mc = m * c2;
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {  // columns 0-31, 32-63, read again
+          uint32_t ra[32];
+          ptx::tmem_ld_32x32b_x32(tS + h2 * 32, ra);
+          ptx::tmem_ld_wait();
+#pragma unroll
+          for (int c = 0; c < 32; c += 2) {
+            const int col = h2 * 32 + c;
+            const float p0 = col < kv ? ptx::ex2_approx(fmaf(__uint_as_float(ra[c]), c2, -mc)) : 0.f;
+            const float p1 = col + 1 < kv ? ptx::ex2_approx(fmaf(__uint_as_float(ra[c + 1]), c2, -mc)) : 0.f;
+            l += p0 + p1;
+            ra[c / 2] = pack2_bf16(p0, p1);
+          }
+          ptx::tmem_st_32x32b_x16(tS + h2 * 16, *reinterpret_cast<const uint32_t(*)[16]>(ra));
+        }
+#pragma unroll
+        for (int c = 0; c < 64; c += 2) {  // columns 64-127, from registers
+          const float p0 = c + 64 < kv ? ptx::ex2_approx(fmaf(__uint_as_float(rh[c]), c2, -mc)) : 0.f;
+          const float p1 = c + 65 < kv ? ptx::ex2_approx(fmaf(__uint_as_float(rh[c + 1]), c2, -mc)) : 0.f;
+          l += p0 + p1;
+          rh[c / 2] = pack2_bf16(p0, p1);
+        }
+        ptx::tmem_st_32x32b_x16(tS + 32, *reinterpret_cast<const uint32_t(*)[16]>(rh));
+        ptx::tmem_st_32x32b_x16(tS + 48, *reinterpret_cast<const uint32_t(*)[16]>(rh + 16));
+        ptx::tmem_st_wait();
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(&pready[x]);
+        // the P V product of this tile completes phase pv_phase of bar_pv[x] (the rescale
+        // above waits on the previous tile's)
+        if (j > 0) pv_phase ^= 1u;
+      }
+      if (!ok) break;
+      // the unit's output: O / l once the last P V product is done, and the log-sum-exp
+      ok = __all_sync(0xffffffffu, ptx::mbar_wait(&bar_pv[x], pv_phase));
+      pv_phase ^= 1u;
+      if (!ok || *abort_flag) { ok = false; *abort_flag = 1; break; }
+      ptx::tc_fence_after();
+      const int q = q0 + x * BQ + r;
+      const float inv = 1.f / l;
+#pragma unroll 1
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t ro[32];
+        ptx::tmem_ld_32x32b_x32(tO + c * 32, ro);
+        ptx::tmem_ld_wait();
+        if (q < N) {
+          bf16* o = static_cast<bf16*>(p.o.base(q)) + p.o.off(b, q, N, (int64_t)h * D + c * 32);
+#pragma unroll
+          for (int v = 0; v < 4; ++v) {
+            uint4 w;
+            w.x = pack2_bf16(__uint_as_float(ro[8 * v]) * inv, __uint_as_float(ro[8 * v + 1]) * inv);
+            w.y = pack2_bf16(__uint_as_float(ro[8 * v + 2]) * inv, __uint_as_float(ro[8 * v + 3]) * inv);
+            w.z = pack2_bf16(__uint_as_float(ro[8 * v + 4]) * inv, __uint_as_float(ro[8 * v + 5]) * inv);
+            w.w = pack2_bf16(__uint_as_float(ro[8 * v + 6]) * inv, __uint_as_float(ro[8 * v + 7]) * inv);
+            *reinterpret_cast<uint4*>(o + 8 * v) = w;
+          }
+        }
+      }
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(&ofree[x]);
+      if (q < N) p.lse[((int64_t)b * p.heads + h) * N + q] = p.scale * m + logf(l);
+    }
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, 512);
+  }
+}
+
 // 3D view [sequence][token][column] of a stream buffer (bf16), boxes of 64 columns x `rows`.
 int seg_map(CUtensorMap* m, const void* base, int64_t ld, int ntok, int B, int rows) {
   const uint64_t dims[3] = {(uint64_t)ld, (uint64_t)ntok, (uint64_t)B};
@@ -1445,8 +1800,44 @@ bool attention_fwd_tc_eligible(const AttnArgs& f) {
   return f.q_col0 % 8 == 0 && f.k_col0 % 8 == 0 && f.v_col0 % 8 == 0;
 }
 
+// The head-dim-128 forward (fa_fwd_tc128_kernel).
+int launch_fwd128(const AttnArgs& f, cudaStream_t s) {
+  using C = Ff2;
+  const int n0 = f.q.n0, N = f.N;
+  const int n1 = N - n0;
+  FfMaps maps;
+  for (int sg = 0; sg < 2; ++sg) {
+    const int nt = sg == 0 ? n0 : n1;
+    if (nt <= 0) {  // single stream: the second views are unused copies
+      maps.q[1] = maps.q[0];
+      maps.k[1] = maps.k[0];
+      maps.v[1] = maps.v[0];
+      break;
+    }
+    JAGG_TRY(seg_map(&maps.q[sg], sg ? f.q.p1 : f.q.p0, sg ? f.q.ld1 : f.q.ld0, nt, f.B, C::BQ));
+    JAGG_TRY(seg_map(&maps.k[sg], sg ? f.k.p1 : f.k.p0, sg ? f.k.ld1 : f.k.ld0, nt, f.B, C::BK));
+    JAGG_TRY(seg_map(&maps.v[sg], sg ? f.v.p1 : f.v.p0, sg ? f.v.ld1 : f.v.ld0, nt, f.B, C::BK));
+  }
+  FfParams p;
+  p.B = f.B; p.N = N; p.heads = f.heads; p.n0 = n0 > 0 && n0 < N ? n0 : N;
+  p.scale = f.scale;
+  p.q_col0 = f.q_col0; p.k_col0 = f.k_col0; p.v_col0 = f.v_col0;
+  p.o = f.o;
+  p.lse = f.lse;
+  static bool attr = false;
+  if (!attr) {
+    JAGG_CUDA_TRY(cudaFuncSetAttribute(fa_fwd_tc128_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
+    attr = true;
+  }
+  const int units = ceil_div(ceil_div(N, C::BQ), 2) * f.B * f.heads;
+  const int nsm = sm_count();
+  fa_fwd_tc128_kernel<<<units < nsm ? units : nsm, FF2_THREADS, C::SMEM, s>>>(maps, p);
+  JAGG_LAUNCHED();
+  return JAGG_OK;
+}
+
 int attention_fwd_tc(const AttnArgs& f, cudaStream_t s) {
-  return f.dh == 64 ? launch_fwd<64>(f, s) : launch_fwd<128>(f, s);
+  return f.dh == 64 ? launch_fwd<64>(f, s) : launch_fwd128(f, s);
 }
 
 // Whether the tensor-core backward serves the call: bf16, head dim 64 / 128, the stream

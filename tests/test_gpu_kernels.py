@@ -371,6 +371,43 @@ def test_attention_forward_kernels_on_two_stream_views(dh, N, n0, B, H, impl):
     assert (lse - ref_lse).abs().max().item() < 1e-2
 
 
+@pytest.mark.parametrize("impl", [1, 2])
+@pytest.mark.parametrize("dh", [64, 128])
+def test_attention_forward_online_softmax_with_climbing_maxima(dh, impl):
+    """Scores that climb along the keys at a rate that differs from row to row (a_i b_t along
+    one direction u): in some rows the running maximum moves up by tens of nats over the key
+    tiles, in others it is reached in the first tile, and the rows of one warp disagree on
+    whether to rescale.  Output and log-sum-exp against PyTorch fp32."""
+    B, N, n0, H = 1, 1536, 512, 2
+    d = H * dh
+    g = torch.Generator(device="cpu").manual_seed(dh + 17 * impl)
+    u = torch.randn(dh, generator=g)
+    u /= u.norm()
+    a = torch.randn(N, H, 1, generator=g) * 2.5                        # per-row rate
+    bt = (16.0 * torch.arange(N) / N * math.sqrt(dh)).view(N, 1, 1)  # per-key climb
+    q = torch.randn(N, H, dh, generator=g) + a * u
+    k = torch.randn(N, H, dh, generator=g) + bt * u
+    v = torch.randn(N, H, dh, generator=g)
+    qkv = torch.stack([q, k, v], 1).reshape(B * N, 3 * d).bfloat16().cuda()
+    qf, kf, vf = _attn_ref(qkv, B, N, H, dh)
+    s = (qf @ kf.transpose(-1, -2)) / math.sqrt(dh)
+    climb = s.max(-1).values - s[..., :128].max(-1).values
+    assert climb.max().item() > 20 and (climb == 0).float().mean().item() > 0.2
+    ref_lse = torch.logsumexp(s, -1)
+    ref_o = torch.softmax(s, -1) @ vf
+    x = qkv.view(B, N, -1)
+    o0 = torch.full((B, n0, d), float("nan"), device="cuda", dtype=torch.bfloat16)
+    o1 = torch.full((B, N - n0, d), float("nan"), device="cuda", dtype=torch.bfloat16)
+    lse = torch.full((B, H, N), float("nan"), device="cuda")
+    jg.test_attention_fwd_streams((x[:, :n0].contiguous(), x[:, n0:].contiguous()), (o0, o1), lse, B, N, n0, H,
+                                  dh, impl=impl)
+    torch.cuda.synchronize()
+    assert jg.device_status() == 0
+    o = torch.cat([o0, o1], 1).float().view(B, N, H, dh).transpose(1, 2)
+    assert _rel(o, ref_o) < 1e-2
+    assert (lse - ref_lse).abs().max().item() < 2e-2
+
+
 def test_tcgen05_attention_backward_rejects_unaligned_streams():
     B, N, n0, H, dh = 1, 300, 100, 2, 64
     d = H * dh
