@@ -1298,9 +1298,10 @@ __global__ void __launch_bounds__(FF_THREADS, 1) fa_fwd_tc_kernel(const __grid_c
 // B, a thread per query row (no exchange between warps).  Each row keeps a reference maximum m: P = exp(scale (S - m)); when a tile's maximum
 // exceeds m by more than 8 / (scale log2 e) (P would pass 2^8), m moves up and the row's O (once
 // the previous P V product has finished) and running sum l are rescaled, so O is rescaled only
-// while the maximum is still climbing.  P goes to tensor memory in place of the S columns the
-// thread has read and is the A operand of P V.  At the end O / l leaves in bf16 and
-// lse = scale m + ln l.
+// while the maximum is still climbing.  P goes to tensor memory over S columns 64-127 (read
+// into registers first) and is the A operand of P V, whose key blocks follow that placement.
+// Row maxima take the three-input max, the scale-shift and the row sums the paired f32 forms.
+// At the end O / l leaves in bf16 and lse = scale m + ln l.
 constexpr int FF2_THREADS = 320;  // 10 warps
 
 struct Ff2 {
@@ -1314,7 +1315,45 @@ struct Ff2 {
   static constexpr int SMEM = OFF_BAR + NBAR * 8 + 16 + 1024;  // + alignment of the base to 1024 bytes
   static_assert(SMEM <= 232448, "shared memory budget");
   static constexpr uint32_t T_S = 0, T_O = 256;  // S_X at 128 X, O_X at 256 + 128 X
+  // Column (within S_X) of P of keys 16 kb .. 16 kb + 15, two bf16 per column: key blocks 4-7
+  // at 64-95, 0-3 at 96-127.
+  static __host__ __device__ constexpr uint32_t p_col(int kb) { return 64 + 8 * ((kb + 4) & 7); }
 };
+
+// Keys at or past `kv` (columns col0 + c of the tile) -> -inf.
+template <int n>
+__device__ __forceinline__ void mask_keys(uint32_t (&r)[n], int col0, int kv) {
+#pragma unroll
+  for (int c = 0; c < n; ++c)
+    if (col0 + c >= kv) r[c] = 0xff800000u;
+}
+// Running maxima of n f32 values in four independent chains.
+template <int n>
+__device__ __forceinline__ void row_max4(const uint32_t (&r)[n], float (&mx)[4]) {
+#pragma unroll
+  for (int c = 0; c < n; c += 8) {
+    mx[0] = ptx::max3(mx[0], __uint_as_float(r[c]), __uint_as_float(r[c + 1]));
+    mx[1] = ptx::max3(mx[1], __uint_as_float(r[c + 2]), __uint_as_float(r[c + 3]));
+    mx[2] = ptx::max3(mx[2], __uint_as_float(r[c + 4]), __uint_as_float(r[c + 5]));
+    mx[3] = ptx::max3(mx[3], __uint_as_float(r[c + 6]), __uint_as_float(r[c + 7]));
+  }
+}
+// p = 2^(s c2 - m c2) of n f32 values, packed in place two per word (bf16) into r[0, n/2);
+// the f32 values are added into acc0, acc1.
+template <int n>
+__device__ __forceinline__ void exp_pack(uint32_t (&r)[n], float2 vc2, float2 vmc, float2& acc0, float2& acc1) {
+#pragma unroll
+  for (int c = 0; c < n; c += 4) {
+    const float2 t0 = ptx::fma2(make_float2(__uint_as_float(r[c]), __uint_as_float(r[c + 1])), vc2, vmc);
+    const float2 t1 = ptx::fma2(make_float2(__uint_as_float(r[c + 2]), __uint_as_float(r[c + 3])), vc2, vmc);
+    const float2 p0 = make_float2(ptx::ex2_approx(t0.x), ptx::ex2_approx(t0.y));
+    const float2 p1 = make_float2(ptx::ex2_approx(t1.x), ptx::ex2_approx(t1.y));
+    acc0 = ptx::add2(acc0, p0);
+    acc1 = ptx::add2(acc1, p1);
+    r[c / 2] = pack2_bf16(p0.x, p0.y);
+    r[c / 2 + 1] = pack2_bf16(p1.x, p1.y);
+  }
+}
 
 __global__ void __launch_bounds__(FF2_THREADS, 1) fa_fwd_tc128_kernel(const __grid_constant__ FfMaps maps,
                                                                       FfParams p) {
@@ -1456,8 +1495,8 @@ __global__ void __launch_bounds__(FF2_THREADS, 1) fa_fwd_tc128_kernel(const __gr
         const uint32_t aV = ptx::smem_u32(sV + vs * C::TILE);
 #pragma unroll
         for (int k = 0; k < BK / 16; ++k)
-          ptx::umma_bf16_ts(tmem + C::T_O + x * 128, tmem + C::T_S + x * 128 + k * 8, mnmajor_desc(aV, BK * 128, k),
-                            id_o, (!first || k > 0) ? 1u : 0u);
+          ptx::umma_bf16_ts(tmem + C::T_O + x * 128, tmem + C::T_S + x * 128 + C::p_col(k),
+                            mnmajor_desc(aV, BK * 128, k), id_o, (!first || k > 0) ? 1u : 0u);
         ptx::umma_commit(&bar_pv[x]);
       };
       for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++i) {
@@ -1527,23 +1566,22 @@ __global__ void __launch_bounds__(FF2_THREADS, 1) fa_fwd_tc128_kernel(const __gr
         s_phase ^= 1u;
         if (!ok || *abort_flag) { ok = false; *abort_flag = 1; break; }
         ptx::tc_fence_after();
-        // The row maximum over columns 0-63 (read again below) and 64-127 (kept in registers):
-        // at most 96 of the row's values are live at once.
-        const int kv = N - j * BK;  // valid keys of the tile
-        float tmax = -INFINITY;
+        // The row maximum: keys 0-63 (read again below), then 64-127 (kept in registers).
+        const int kv = N - j * BK;  // valid keys of the tile (at least one)
+        const bool ragged = kv < BK;
         uint32_t rh[64];
+        float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
         ptx::tmem_ld_32x32b_x32(tS, *reinterpret_cast<uint32_t(*)[32]>(rh));
         ptx::tmem_ld_32x32b_x32(tS + 32, *reinterpret_cast<uint32_t(*)[32]>(rh + 32));
         ptx::tmem_ld_wait();
-#pragma unroll
-        for (int c = 0; c < 64; ++c)
-          if (c < kv) tmax = fmaxf(tmax, __uint_as_float(rh[c]));
+        if (ragged) mask_keys(rh, 0, kv);
+        row_max4(rh, mx);
         ptx::tmem_ld_32x32b_x32(tS + 64, *reinterpret_cast<uint32_t(*)[32]>(rh));
         ptx::tmem_ld_32x32b_x32(tS + 96, *reinterpret_cast<uint32_t(*)[32]>(rh + 32));
         ptx::tmem_ld_wait();
-#pragma unroll
-        for (int c = 0; c < 64; ++c)
-          if (c + 64 < kv) tmax = fmaxf(tmax, __uint_as_float(rh[c]));
+        if (ragged) mask_keys(rh, 64, kv);
+        row_max4(rh, mx);
+        const float tmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
         if (j == 0) {
           m = tmax;
         } else if (__any_sync(0xffffffffu, tmax > m + kRescale)) {
@@ -1567,33 +1605,29 @@ __global__ void __launch_bounds__(FF2_THREADS, 1) fa_fwd_tc128_kernel(const __gr
           l *= f;
           m = mn;
         }
-        // rows whose reference stays: P = exp(scale (S - m)), at most 2^8
-        // P of columns 2c, 2c+1 goes to column c, over S values already read
+        // P = exp(scale (S - m)) (at most 2^8) in bf16 at the columns Ff2::p_col gives: keys 64-127 over the
+        // S columns 64-95 (already in registers), keys 0-63 over 96-127, so keys 0-63 can be
+        // read again while keys 64-127 are exponentiated
         const float mc = m * c2;
-#pragma unroll
-        for (int h2 = 0; h2 < 2; ++h2) {  // columns 0-31, 32-63, read again
-          uint32_t ra[32];
-          ptx::tmem_ld_32x32b_x32(tS + h2 * 32, ra);
-          ptx::tmem_ld_wait();
-#pragma unroll
-          for (int c = 0; c < 32; c += 2) {
-            const int col = h2 * 32 + c;
-            const float p0 = col < kv ? ptx::ex2_approx(fmaf(__uint_as_float(ra[c]), c2, -mc)) : 0.f;
-            const float p1 = col + 1 < kv ? ptx::ex2_approx(fmaf(__uint_as_float(ra[c + 1]), c2, -mc)) : 0.f;
-            l += p0 + p1;
-            ra[c / 2] = pack2_bf16(p0, p1);
-          }
-          ptx::tmem_st_32x32b_x16(tS + h2 * 16, *reinterpret_cast<const uint32_t(*)[16]>(ra));
+        const float2 vc2 = make_float2(c2, c2), vmc = make_float2(-mc, -mc);
+        float2 l0 = make_float2(0.f, 0.f), l1 = make_float2(0.f, 0.f);
+        uint32_t ra[32];
+        ptx::tmem_ld_32x32b_x32(tS, ra);
+        exp_pack(rh, vc2, vmc, l0, l1);
+        ptx::tmem_st_32x32b_x16(tS + C::p_col(4), *reinterpret_cast<const uint32_t(*)[16]>(rh));
+        ptx::tmem_st_32x32b_x16(tS + C::p_col(6), *reinterpret_cast<const uint32_t(*)[16]>(rh + 16));
+        uint32_t(&rb)[32] = *reinterpret_cast<uint32_t(*)[32]>(rh + 32);
+        ptx::tmem_ld_32x32b_x32(tS + 32, rb);
+        ptx::tmem_ld_wait();
+        if (ragged) {
+          mask_keys(ra, 0, kv);
+          mask_keys(rb, 32, kv);
         }
-#pragma unroll
-        for (int c = 0; c < 64; c += 2) {  // columns 64-127, from registers
-          const float p0 = c + 64 < kv ? ptx::ex2_approx(fmaf(__uint_as_float(rh[c]), c2, -mc)) : 0.f;
-          const float p1 = c + 65 < kv ? ptx::ex2_approx(fmaf(__uint_as_float(rh[c + 1]), c2, -mc)) : 0.f;
-          l += p0 + p1;
-          rh[c / 2] = pack2_bf16(p0, p1);
-        }
-        ptx::tmem_st_32x32b_x16(tS + 32, *reinterpret_cast<const uint32_t(*)[16]>(rh));
-        ptx::tmem_st_32x32b_x16(tS + 48, *reinterpret_cast<const uint32_t(*)[16]>(rh + 16));
+        exp_pack(ra, vc2, vmc, l0, l1);
+        ptx::tmem_st_32x32b_x16(tS + C::p_col(0), *reinterpret_cast<const uint32_t(*)[16]>(ra));
+        exp_pack(rb, vc2, vmc, l0, l1);
+        ptx::tmem_st_32x32b_x16(tS + C::p_col(2), *reinterpret_cast<const uint32_t(*)[16]>(rb));
+        l += (l0.x + l0.y) + (l1.x + l1.y);
         ptx::tmem_st_wait();
         ptx::tc_fence_before();
         __syncwarp();
