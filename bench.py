@@ -96,7 +96,7 @@ def describe(wl) -> str:
 # bytes, from one ncu capture of the kernel alone (`--kernel gemm`) on the workload's
 # backward products at the step's rows; the roofline's `traffic` is this ratio times the
 # step's algorithmic bytes per launch.  Absent: no capture of the current kernel.
-TRAFFIC_RATIO = {"mmdit_flux1024_bf16": 2.96}
+TRAFFIC_RATIO = {"mmdit_flux1024_bf16": 3.01}
 
 
 def peaks():

@@ -714,6 +714,17 @@ __global__ void copy_rows_kernel(const E* in, int64_t ld_in, int is, int io, int
   }
 }
 
+// Whole rows in 16-byte vectors, a row per block iteration (row pitches, row bytes and both
+// bases 16-byte aligned).
+__global__ void copy_rows_v16_kernel(const uint8_t* in, int64_t ld_in_b, int is, int io, int64_t iss, uint8_t* out,
+                                     int64_t ld_out_b, int os, int oo, int64_t oss, int rows, int nvec) {
+  for (int r = blockIdx.x; r < rows; r += gridDim.x) {
+    const uint4* src = reinterpret_cast<const uint4*>(in + seg_row(r, is, io, iss) * ld_in_b);
+    uint4* dst = reinterpret_cast<uint4*>(out + seg_row(r, os, oo, oss) * ld_out_b);
+    for (int c = threadIdx.x; c < nvec; c += blockDim.x) dst[c] = __ldg(src + c);
+  }
+}
+
 __global__ void attn_rowdot_kernel(const void* dO, const void* O, int64_t ld, float* Dv, int B, int N, int heads,
                                    int dh, int is_f32) {
   // one warp per (row, head)
@@ -1190,9 +1201,17 @@ int launch_gather_rows(const float* in, int64_t ld_in, int seg, int seg_off, int
 int launch_copy_rows(const void* in, int64_t ld_in, int in_seg, int in_seg_off, int64_t in_seg_stride, void* out,
                      int64_t ld_out, int out_seg, int out_seg_off, int64_t out_seg_stride, int rows, int cols,
                      int elem_bytes, cudaStream_t s) {
-  const int g = grid_for((int64_t)rows * cols, 256);
   const int tok = prof_start(s);
-  if (elem_bytes == 4)
+  const int64_t row_b = (int64_t)cols * elem_bytes;
+  const bool v16 = row_b % 16 == 0 && (ld_in * elem_bytes) % 16 == 0 && (ld_out * elem_bytes) % 16 == 0 &&
+                   (reinterpret_cast<uintptr_t>(in) & 15) == 0 && (reinterpret_cast<uintptr_t>(out) & 15) == 0;
+  const int g = grid_for((int64_t)rows * cols, 256);
+  if (v16 && rows > 0) {
+    const int nb = rows < 8 * sm_count() ? rows : 8 * sm_count();
+    copy_rows_v16_kernel<<<nb, 256, 0, s>>>(static_cast<const uint8_t*>(in), ld_in * elem_bytes, in_seg, in_seg_off,
+                                            in_seg_stride, static_cast<uint8_t*>(out), ld_out * elem_bytes, out_seg,
+                                            out_seg_off, out_seg_stride, rows, (int)(row_b / 16));
+  } else if (elem_bytes == 4)
     copy_rows_kernel<float><<<g, 256, 0, s>>>(static_cast<const float*>(in), ld_in, in_seg, in_seg_off, in_seg_stride,
                                              static_cast<float*>(out), ld_out, out_seg, out_seg_off, out_seg_stride,
                                              rows, cols);

@@ -326,38 +326,51 @@ __global__ void aggregate_span_kernel(const float* s, int64_t ld, const double* 
 constexpr int GR_BLOCKS = 1024;
 constexpr int GR_THREADS = 256;
 
+// HAS_B: a second vector b (else <a, b> = |b|^2 = |a|^2 and b is not read); HAS_ACC: the
+// update acc += alpha a.  Each thread loads a run of 8 float4 of each input before using any
+// of them, so 8 (16) loads per thread are in flight; f32 sums over a run fold into f64.
+template <bool HAS_B, bool HAS_ACC>
 __global__ void __launch_bounds__(GR_THREADS) grad_reduce_kernel(const float* a, const float* b, int64_t P,
                                                                  float alpha, float* acc, double* partial) {
-  // Each thread handles runs of 8 float4; f32 sums over a run are folded into f64.
   double sab = 0.0, saa = 0.0, sbb = 0.0;
   const int64_t nvec = P / 4;
   const float4* a4 = reinterpret_cast<const float4*>(a);
-  const float4* b4 = reinterpret_cast<const float4*>(b ? b : a);
+  const float4* b4 = reinterpret_cast<const float4*>(b);
   float4* c4 = reinterpret_cast<float4*>(acc);
   const int64_t stride = (int64_t)GR_BLOCKS * GR_THREADS;
-  int64_t idx = (int64_t)blockIdx.x * GR_THREADS + threadIdx.x;
-  while (idx < nvec) {
-    float fab = 0.f, faa = 0.f, fbb = 0.f;
+  const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int64_t idx = (int64_t)blockIdx.x * GR_THREADS + threadIdx.x; idx < nvec; idx += 8 * stride) {
+    float4 x[8], y[8];
 #pragma unroll
     for (int r = 0; r < 8; ++r) {
       const int64_t q = idx + (int64_t)r * stride;
-      if (q < nvec) {
-        const float4 x = a4[q];
-        const float4 y = b4[q];
-        fab += x.x * y.x + x.y * y.y + x.z * y.z + x.w * y.w;
-        faa += x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w;
-        fbb += y.x * y.x + y.y * y.y + y.z * y.z + y.w * y.w;
-        if (acc) {
+      x[r] = q < nvec ? a4[q] : zero;
+      if constexpr (HAS_B) y[r] = q < nvec ? b4[q] : zero;
+    }
+    float fab = 0.f, faa = 0.f, fbb = 0.f;
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+      faa += x[r].x * x[r].x + x[r].y * x[r].y + x[r].z * x[r].z + x[r].w * x[r].w;
+      if constexpr (HAS_B) {
+        fab += x[r].x * y[r].x + x[r].y * y[r].y + x[r].z * y[r].z + x[r].w * y[r].w;
+        fbb += y[r].x * y[r].x + y[r].y * y[r].y + y[r].z * y[r].z + y[r].w * y[r].w;
+      }
+    }
+    if constexpr (HAS_ACC) {
+#pragma unroll
+      for (int r = 0; r < 8; ++r) {
+        const int64_t q = idx + (int64_t)r * stride;
+        if (q < nvec) {
           float4 c = c4[q];
-          c.x += alpha * x.x; c.y += alpha * x.y; c.z += alpha * x.z; c.w += alpha * x.w;
+          c.x += alpha * x[r].x; c.y += alpha * x[r].y; c.z += alpha * x[r].z; c.w += alpha * x[r].w;
           c4[q] = c;
         }
       }
     }
+    if constexpr (!HAS_B) fab = fbb = faa;
     sab += fab;
     saa += faa;
     sbb += fbb;
-    idx += 8 * stride;
   }
   // scalar tail (P % 4), handled by block 0
   if (blockIdx.x == 0) {
@@ -598,8 +611,15 @@ extern "C" int grad_reduce(const float* a, const float* b, int64_t P, float alph
     }
   }
   const int tok = prof_start(stream);
-  grad_reduce_kernel<<<GR_BLOCKS, GR_THREADS, 0, stream>>>(a, b, P, alpha, acc,
-                                                           out3 ? static_cast<double*>(ws) : nullptr);
+  double* part = out3 ? static_cast<double*>(ws) : nullptr;
+  if (b && acc)
+    grad_reduce_kernel<true, true><<<GR_BLOCKS, GR_THREADS, 0, stream>>>(a, b, P, alpha, acc, part);
+  else if (b)
+    grad_reduce_kernel<true, false><<<GR_BLOCKS, GR_THREADS, 0, stream>>>(a, b, P, alpha, acc, part);
+  else if (acc)
+    grad_reduce_kernel<false, true><<<GR_BLOCKS, GR_THREADS, 0, stream>>>(a, b, P, alpha, acc, part);
+  else
+    grad_reduce_kernel<false, false><<<GR_BLOCKS, GR_THREADS, 0, stream>>>(a, b, P, alpha, acc, part);
   JAGG_LAUNCHED();
   if (out3) {
     grad_reduce_final<<<1, 32, 0, stream>>>(static_cast<const double*>(ws), out3);
