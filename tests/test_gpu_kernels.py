@@ -445,6 +445,9 @@ def test_bounded_wait_gives_up_and_reports_timeout(limit_ns):
     (3072, 333 * 3, 333, True, True, torch.bfloat16),     # sequences that straddle CTA row shares
     (3072, 40, 8, True, True, torch.float32),             # f32 y: the persistent kernel
     (768, 333 * 4, 333, True, True, torch.bfloat16),      # DiT-B width: row-in-registers kernel
+    (768, 256 * 3, 256, True, False, torch.bfloat16),     # DiT-B width, LayerNorm only
+    (768, 77 * 5, 77, False, True, torch.bfloat16),       # DiT-B width, gate only (persistent kernel)
+    (768, 333 * 2, 333, True, True, torch.float32),       # DiT-B width, f32 y
     (1024, 300, 100, True, True, torch.bfloat16),
     (64, 24 * 4, 24, True, True, torch.float32)])
 def test_ln_gate_backward_kernels(d, M, rps, ln, gate, dtype):
