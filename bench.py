@@ -718,7 +718,8 @@ def run_gpu(args, ws, rank):
     ratio = TRAFFIC_RATIO.get(wl.name)
     roofline["traffic"] = ratio * roofline["algorithmic_bytes_per_launch"] if ratio else None
     roofline["frac_of_burst"] = roofline["achieved"] / burst
-    att = family_roofline(fam, "attention_bwd", sustained, psrc, "fa_bwd_tc_kernel (attention backward)")
+    att = family_roofline(fam, "attention_bwd", sustained, psrc,
+                          f"fa_bwd_tc{wl.head_dim}_kernel (attention backward)")
     att["frac_of_burst"] = att["achieved"] / burst
     step_flops = sum(v["flops"] for k, v in fam.items() if k != "gemm_simt")
     families = {k: {"launches_per_step": v["launches"], "ms_per_step": v["ms"],

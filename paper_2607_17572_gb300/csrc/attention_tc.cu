@@ -1,24 +1,10 @@
-// Attention backward on the fifth-generation tensor cores (tcgen05, TMEM accumulators,
-// TMA-fed shared-memory operands), bf16 (appendix, Eqs. bwd_V .. bwd_QK, with the softmax
-// recomputed from the saved log-sum-exp).  Head dim 64: fa_bwd_tc_kernel below; head dim
-// 128: fa_bwd_tc128_kernel further down.
-//
-// Head dim 64.  Persistent: each CTA walks (128-key tile, sequence, head) units; per unit it
-// streams the sequence's 128-query tiles:
-//   S^T = K Q^T, dP^T = V dO^T                      (128 x 128, TMEM)
-//   P^T = exp(scale S^T - lse), dS^T = P^T (dP^T - rowsum(dO O))   (8 warps, -> bf16 smem)
-//   dV += P^T dO, dK += dS^T Q                      (128 x 64, TMEM, whole sequence)
-//   dQ  = dS K  -> 4 warps -> TMA f32 reduce-add into the dQ accumulator.
-// Every product has M = 128.  Each shared tile serves as a K-major and an MN-major
-// operand through two descriptors of the same 128-byte-swizzled layout, so nothing is
-// transposed.  Warp roles: 0 TMA producer, 1 MMA issuer (one elected thread), 2-9 P / dS
-// (two warps per TMEM lane quarter, half the query columns each), 10-13 dQ and the final
-// dK / dV.  One S^T, dP^T buffer (128 + 128 + 64 + 64 + 64 columns); the MMA warp issues S,
-// dP of tile j + 1 before dV, dK, dQ of tile j.
-// Tile-level barrier phases run on across units, and two K, V buffers let the next unit's K,
-// V loads and first products overlap the previous unit's last tiles and its dQ drain.
-// Ragged ends: 3D tensor maps [sequence][token][column] per stream buffer make TMA read
-// zeros past the last token and drop dQ rows past it.
+// Attention on the fifth-generation tensor cores (tcgen05, TMEM accumulators, TMA-fed
+// shared-memory operands), bf16: the backward (appendix, Eqs. bwd_V .. bwd_QK, with the
+// softmax recomputed from the saved log-sum-exp) for head dims 128 and 64
+// (fa_bwd_tc128_kernel, fa_bwd_tc64_kernel), and the forward, one pass with an online
+// softmax at head dim 128 (fa_fwd_tc128_kernel), two passes at 64 (fa_fwd_tc_kernel<64>).
+// Ragged ends and the MMDiT text / image split: 3D tensor maps [sequence][token][column]
+// per stream buffer make TMA read zeros past the last token and drop dQ rows past it.
 #include <cuda.h>
 
 #include "attention.cuh"
@@ -31,42 +17,6 @@ int unit_status_attention_tc(unsigned* v, int clear) { return read_unit_status(v
 namespace {
 
 constexpr float kLog2eTc = 1.4426950408889634f;
-constexpr int FB_THREADS = 448;  // 14 warps
-
-template <int D>
-struct FbCfg {
-  static_assert(D == 64, "head dim 128 has fa_bwd_tc128_kernel");
-  static constexpr int BK = 128;                 // keys per CTA
-  static constexpr int BQ = 128;                 // queries per step
-  static constexpr int NSB = 1;                  // S^T / dP^T TMEM buffers
-  static constexpr int CW = BQ / 2;              // query columns per P / dS warp
-  static constexpr int KV_BYTES = BK * D * 2;
-  static constexpr int QT_BYTES = BQ * D * 2;
-  static constexpr int PS_BYTES = BK * BQ * 2;
-  // short sequences in practice: K, V double-buffered across the CTA's units, two Q / dO
-  // stages
-  static constexpr int KVB = 2;
-  static constexpr int STAGES = 2;
-  static constexpr int DQ_WARP_BYTES = 32 * 32 * 4;  // one 32 x 32 f32 box, used twice per tile
-  static constexpr int OFF_K = 0;                       // KVB buffers
-  static constexpr int OFF_V = OFF_K + KVB * KV_BYTES;    // KVB buffers
-  static constexpr int OFF_Q = OFF_V + KVB * KV_BYTES;
-  static constexpr int OFF_DO = OFF_Q + STAGES * QT_BYTES;
-  static constexpr int OFF_P = OFF_DO + STAGES * QT_BYTES;
-  static constexpr int OFF_DS = OFF_P + PS_BYTES;
-  static constexpr int OFF_DQ = OFF_DS + PS_BYTES;
-  static constexpr int OFF_LSE = OFF_DQ + 4 * DQ_WARP_BYTES;
-  static constexpr int OFF_RD = OFF_LSE + STAGES * BQ * 4;
-  static constexpr int OFF_BAR = OFF_RD + STAGES * BQ * 4;
-  static constexpr int SMEM = OFF_BAR + 256 + 1024;
-  // TMEM columns: S^T [0, 128), dP^T [128, 256), dV, dK, dQ
-  static constexpr int T_DV = 256, T_DK = 320;
-  __host__ __device__ static constexpr int t_s(int) { return 0; }
-  __host__ __device__ static constexpr int t_dp(int) { return 128; }
-  __host__ __device__ static constexpr int t_dq(int) { return 384; }
-  static_assert(SMEM <= 232448, "shared memory budget");
-};
-
 // Tensor maps of one backward call: per stream buffer (0: the first n0 tokens of every
 // sequence, 1: the rest) the query, key, value and output-gradient views, and the dQ
 // accumulator.
@@ -111,398 +61,7 @@ __device__ __forceinline__ void st_row32_packed(uint8_t* tile, int rows, int r, 
   }
 }
 
-// P^T, dS^T of 32 query columns of one key row from S^T, dP^T (f32 bit patterns).
-__device__ __forceinline__ void softmax32(const uint32_t* rs, const uint32_t* rp, const float* lse, const float* rd,
-                                          float scale, uint32_t* hp, uint32_t* hd) {
-#pragma unroll
-  for (int i = 0; i < 32; i += 4) {
-    const float4 l4 = *reinterpret_cast<const float4*>(lse + i);
-    const float4 r4 = *reinterpret_cast<const float4*>(rd + i);
-    const float p0 = ptx::ex2_approx((__uint_as_float(rs[i]) * scale - l4.x) * kLog2eTc);
-    const float p1 = ptx::ex2_approx((__uint_as_float(rs[i + 1]) * scale - l4.y) * kLog2eTc);
-    const float p2 = ptx::ex2_approx((__uint_as_float(rs[i + 2]) * scale - l4.z) * kLog2eTc);
-    const float p3 = ptx::ex2_approx((__uint_as_float(rs[i + 3]) * scale - l4.w) * kLog2eTc);
-    hp[i / 2] = pack2_bf16(p0, p1);
-    hp[i / 2 + 1] = pack2_bf16(p2, p3);
-    hd[i / 2] = pack2_bf16(p0 * (__uint_as_float(rp[i]) - r4.x), p1 * (__uint_as_float(rp[i + 1]) - r4.y));
-    hd[i / 2 + 1] = pack2_bf16(p2 * (__uint_as_float(rp[i + 2]) - r4.z), p3 * (__uint_as_float(rp[i + 3]) - r4.w));
-  }
-}
-
-template <int D>
-__global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_constant__ FbMaps maps, FbParams p) {
-  using C = FbCfg<D>;
-  constexpr int BK = C::BK, BQ = C::BQ, NS = C::STAGES, NSB = C::NSB, CW = C::CW, KVB = C::KVB;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sK = sm + C::OFF_K;
-  uint8_t* sV = sm + C::OFF_V;
-  uint8_t* sQ = sm + C::OFF_Q;
-  uint8_t* sdO = sm + C::OFF_DO;
-  uint8_t* sP = sm + C::OFF_P;
-  uint8_t* sdS = sm + C::OFF_DS;
-  uint8_t* sDQ = sm + C::OFF_DQ;
-  float* sLse = reinterpret_cast<float*>(sm + C::OFF_LSE);
-  float* sRd = reinterpret_cast<float*>(sm + C::OFF_RD);
-  uint64_t* bar = reinterpret_cast<uint64_t*>(sm + C::OFF_BAR);
-  uint64_t* full = bar;                     // [NS] Q, dO, lse, rowsum of a stage landed
-  uint64_t* empty = full + NS;              // [NS] the stage's products are done
-  uint64_t* bar_s = empty + NS;             // [NSB] S^T, dP^T of a tile are in TMEM buffer b
-  uint64_t* bar_dq = bar_s + NSB;           // [NSB] dQ of a tile is in TMEM buffer b
-  uint64_t* bar_dqfree = bar_dq + NSB;      // [NSB] the dQ warps have read it
-  uint64_t* bar_kv = bar_dqfree + NSB;      // [KVB] a unit's K, V landed
-  uint64_t* kv_free = bar_kv + KVB;         // [KVB] a unit's products are done (K, V reusable)
-  uint64_t* bar_p = kv_free + KVB;          // P^T, dS^T written (S^T, dP^T read) by the 8 warps
-  uint64_t* bar_pfree = bar_p + 1;          // the products reading P^T, dS^T are done
-  uint64_t* bar_fin = bar_p + 2;            // a unit's products are done (dK, dV final)
-  uint64_t* bar_kvout = bar_p + 3;          // the dQ warps have read the unit's dK, dV
-  uint64_t* bar_drain = bar_p + 4;          // the MMA thread's drain after a give-up
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_p + 5);
-  __shared__ volatile int abort_flag;
-
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int N = p.N;
-  const int nkt = (N + BK - 1) / BK;
-  const int units = nkt * p.B * p.heads;
-  const int nq = (N + BQ - 1) / BQ;
-  // unit u: key tile u % nkt of sequence-head u / nkt
-  auto unit_of = [&](int u, int& k0, int& b, int& h) {
-    const int bh = u / nkt;
-    k0 = (u % nkt) * BK;
-    b = bh / p.heads;
-    h = bh % p.heads;
-  };
-
-  if (threadIdx.x == 0) {
-    abort_flag = 0;
-    for (int i = 0; i < NS; ++i) {
-      ptx::mbar_init(&full[i], 1 + 32);  // the TMA's expect-tx arrival + one per producer lane's copies
-      ptx::mbar_init(&empty[i], 1);
-    }
-    for (int i = 0; i < NSB; ++i) {
-      ptx::mbar_init(&bar_s[i], 1);
-      ptx::mbar_init(&bar_dq[i], 1);
-      ptx::mbar_init(&bar_dqfree[i], 4);
-    }
-    for (int i = 0; i < KVB; ++i) {
-      ptx::mbar_init(&bar_kv[i], 1);
-      ptx::mbar_init(&kv_free[i], 1);
-    }
-    ptx::mbar_init(bar_p, 8);
-    ptx::mbar_init(bar_pfree, 1);
-    ptx::mbar_init(bar_fin, 1);
-    ptx::mbar_init(bar_kvout, 4);
-    ptx::mbar_init(bar_drain, 1);
-    ptx::fence_mbar_init();
-    for (int sg = 0; sg < 2; ++sg) {
-      ptx::prefetch_tmap(&maps.q[sg]);
-      ptx::prefetch_tmap(&maps.k[sg]);
-      ptx::prefetch_tmap(&maps.v[sg]);
-      ptx::prefetch_tmap(&maps.dO[sg]);
-    }
-    ptx::prefetch_tmap(&maps.dq);
-  }
-  if (warp == 1) {
-    ptx::tmem_alloc(tmem_slot, 512);
-    ptx::tmem_relinquish();
-  }
-  ptx::tc_fence_before();
-  __syncthreads();
-  ptx::tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-
-  // row coordinates inside a stream buffer
-  auto seg_of = [&](int r) { return r < p.n0 ? 0 : 1; };
-  auto row_in = [&](int r) { return r < p.n0 ? r : r - p.n0; };
-
-  if (warp == 0) {
-    // ---------------------------------------------------------------- TMA producer
-    int i = 0;
-    int i_last = -1, g_last = -1;  // the last unit whose K, V and the last tile whose Q, dO were issued
-    for (int u = blockIdx.x; u < units && !abort_flag; u += gridDim.x, ++i) {
-      int k0, b, h;
-      unit_of(u, k0, b, h);
-      const int bh = b * p.heads + h;
-      const int kvb = i % KVB;
-      bool ok = true;
-      if (lane == 0) {
-        if (i >= KVB) ok = ptx::mbar_wait(&kv_free[kvb], ((i / KVB) & 1) ^ 1);
-        if (ok) {
-          const int s = seg_of(k0), r = row_in(k0);
-          ptx::mbar_arrive_expect_tx(&bar_kv[kvb], 2 * C::KV_BYTES);
-#pragma unroll
-          for (int c = 0; c < D / 64; ++c) {
-            ptx::tma_load_3d(sK + kvb * C::KV_BYTES + c * BK * 128, &maps.k[s], &bar_kv[kvb],
-                             (int)(p.k_col0 + h * D + c * 64), r, b);
-            ptx::tma_load_3d(sV + kvb * C::KV_BYTES + c * BK * 128, &maps.v[s], &bar_kv[kvb],
-                             (int)(p.v_col0 + h * D + c * 64), r, b);
-          }
-          i_last = i;
-        }
-      }
-      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-      if (!ok) { abort_flag = 1; break; }
-      for (int j = 0; j < nq; ++j) {
-        const int g = i * nq + j;
-        const int st = g % NS;
-        if (lane == 0) ok = ptx::mbar_wait(&empty[st], ((g / NS) & 1) ^ 1);
-        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-        if (!ok || abort_flag) { abort_flag = 1; break; }
-        const int q0 = j * BQ;
-        // lse and rowsum(dO O) of the tile's queries: asynchronous 4-byte copies (their
-        // addresses need not be 16-byte aligned) whose completion the stage barrier tracks;
-        // +inf / 0 past the last query
-        for (int t = lane; t < BQ; t += 32) {
-          const int q = q0 + t;
-          if (q < N) {
-            ptx::cp_async4(sLse + st * BQ + t, p.lse + (int64_t)bh * N + q);
-            ptx::cp_async4(sRd + st * BQ + t, p.Dv + (int64_t)bh * N + q);
-          } else {
-            sLse[st * BQ + t] = INFINITY;
-            sRd[st * BQ + t] = 0.f;
-          }
-        }
-        ptx::cp_async_arrive_noinc(&full[st]);
-        __syncwarp();
-        if (lane == 0) {
-          const int s = seg_of(q0), r = row_in(q0);
-          ptx::mbar_arrive_expect_tx(&full[st], 2 * C::QT_BYTES);
-#pragma unroll
-          for (int c = 0; c < D / 64; ++c) {
-            ptx::tma_load_3d(sQ + st * C::QT_BYTES + c * BQ * 128, &maps.q[s], &full[st],
-                             (int)(p.q_col0 + h * D + c * 64), r, b);
-            ptx::tma_load_3d(sdO + st * C::QT_BYTES + c * BQ * 128, &maps.dO[s], &full[st], h * D + c * 64, r,
-                             b);
-          }
-        }
-        g_last = g;
-      }
-    }
-    // After a give-up anywhere in the CTA, copies already issued may still be landing in
-    // shared memory: wait (bounded) for the last phase of every buffer before exiting.
-    if (abort_flag && lane == 0) {
-      for (int k = 0; k < KVB && i_last - k >= 0; ++k)
-        ptx::mbar_wait(&bar_kv[(i_last - k) % KVB], ((i_last - k) / KVB) & 1);
-      for (int k = 0; k < NS && g_last - k >= 0; ++k)
-        ptx::mbar_wait(&full[(g_last - k) % NS], ((g_last - k) / NS) & 1);
-    }
-  } else if (warp == 1) {
-    // ---------------------------------------------------------------- MMA issuer
-    if (ptx::elect_one()) {
-      constexpr uint32_t id_s = ptx::idesc_bf16(128, BQ, false, false);
-      constexpr uint32_t id_acc = ptx::idesc_bf16(128, D, false, true);
-      constexpr uint32_t id_dq = ptx::idesc_bf16(128, 64, true, true);
-      const uint32_t aP = ptx::smem_u32(sP), adS = ptx::smem_u32(sdS);
-      bool ok = true;
-      int i = 0;
-      for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++i) {
-        const int kvb = i % KVB;
-        const uint32_t aK = ptx::smem_u32(sK + kvb * C::KV_BYTES), aV = ptx::smem_u32(sV + kvb * C::KV_BYTES);
-        // S^T, dP^T of global tile g into TMEM buffer g % NSB
-        auto issue_s = [&](int g) {
-          const int st = g % NS, bb = g % NSB;
-          const uint32_t aQ = ptx::smem_u32(sQ + st * C::QT_BYTES), adO = ptx::smem_u32(sdO + st * C::QT_BYTES);
-#pragma unroll
-          for (int k = 0; k < D / 16; ++k) {
-            ptx::umma_bf16(tmem + C::t_s(bb), kmajor_desc(aK, BK, k), kmajor_desc(aQ, BQ, k), id_s, k > 0);
-            ptx::umma_bf16(tmem + C::t_dp(bb), kmajor_desc(aV, BK, k), kmajor_desc(adO, BQ, k), id_s, k > 0);
-          }
-          ptx::umma_commit(&bar_s[bb]);
-        };
-        if (!ptx::mbar_wait(&bar_kv[kvb], (i / KVB) & 1)) { ok = false; break; }
-        for (int j = 0; j < NSB && j < nq; ++j) {
-          const int g = i * nq + j;
-          if (!ptx::mbar_wait(&full[g % NS], (g / NS) & 1)) { ok = false; break; }
-          ptx::tc_fence_after();
-          issue_s(g);
-        }
-        for (int j = 0; j < nq && ok; ++j) {
-          const int g = i * nq + j;
-          const int st = g % NS, bb = g % NSB;
-          if (!ptx::mbar_wait(bar_p, g & 1)) { ok = false; break; }
-          ptx::tc_fence_after();
-          // the single S^T / dP^T buffer is consumed: the next tile's products first
-          if (j + 1 < nq) {
-            if (!ptx::mbar_wait(&full[(g + 1) % NS], ((g + 1) / NS) & 1)) { ok = false; break; }
-            ptx::tc_fence_after();
-            issue_s(g + 1);
-          }
-          const uint32_t aQ = ptx::smem_u32(sQ + st * C::QT_BYTES), adO = ptx::smem_u32(sdO + st * C::QT_BYTES);
-          // the first dV, dK products of a unit overwrite the accumulators: the dQ warps have
-          // read the previous unit's
-          if (j == 0 && i > 0) {
-            if (!ptx::mbar_wait(bar_kvout, (i - 1) & 1)) { ok = false; break; }
-            ptx::tc_fence_after();
-          }
-#pragma unroll
-          for (int k = 0; k < BQ / 16; ++k) {
-            const uint32_t acc = (j > 0 || k > 0) ? 1u : 0u;
-            ptx::umma_bf16(tmem + C::T_DV, kmajor_desc(aP, BK, k), mnmajor_desc(adO, BQ * 128, k), id_acc, acc);
-            ptx::umma_bf16(tmem + C::T_DK, kmajor_desc(adS, BK, k), mnmajor_desc(aQ, BQ * 128, k), id_acc, acc);
-          }
-          if (g > 0) {  // the dQ warps have read the previous tile's dQ
-            if (!ptx::mbar_wait(&bar_dqfree[0], (g - 1) & 1)) { ok = false; break; }
-            ptx::tc_fence_after();
-          }
-#pragma unroll
-          for (int k = 0; k < BK / 16; ++k)  // dQ[q][d] = sum_key dS^T[key][q] K[key][d]
-            ptx::umma_bf16(tmem + C::t_dq(bb), mnmajor_desc(adS, BK * 128, k), mnmajor_desc(aK, BK * 128, k),
-                           id_dq, k > 0);
-          ptx::umma_commit(&bar_dq[bb]);
-          ptx::umma_commit(&empty[st]);
-          ptx::umma_commit(bar_pfree);
-        }
-        ptx::umma_commit(&kv_free[kvb]);
-        ptx::umma_commit(bar_fin);
-      }
-      if (!ok) abort_flag = 1;
-      if (abort_flag) {  // MMAs of this thread may still run: drain them before TMEM is freed
-        ptx::umma_commit(bar_drain);
-        ptx::mbar_wait(bar_drain, 0);
-      }
-    }
-  } else if (warp < 10) {
-    // ---------------------------------------------------------------- P / dS, then dK, dV
-    const int quarter = warp & 3, half = (warp - 2) >> 2;
-    const int r = quarter * 32 + lane;  // key row of the tile = TMEM lane
-    const int c0 = half * CW;           // this warp's query columns
-    const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
-    bool ok = true;
-    int i = 0;
-    for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++i) {
-      int k0, b, h;
-      unit_of(u, k0, b, h);
-      for (int j = 0; j < nq; ++j) {
-        const int g = i * nq + j;
-        const int st = g % NS, bb = g % NSB;
-        ok = ptx::mbar_wait(&bar_s[bb], (g / NSB) & 1) && ptx::mbar_wait(&full[st], (g / NS) & 1);
-        ok = __all_sync(0xffffffffu, ok);
-        if (!ok || abort_flag) { ok = false; abort_flag = 1; break; }
-        ptx::tc_fence_after();
-        const float* lse = sLse + st * BQ + c0;
-        const float* rd = sRd + st * BQ + c0;
-        uint32_t hp[CW / 2], hd[CW / 2];
-#pragma unroll
-        for (int c = 0; c < CW / 32; ++c) {
-          uint32_t rs[32], rp[32];
-          ptx::tmem_ld_32x32b_x32(trow + C::t_s(bb) + c0 + c * 32, rs);
-          ptx::tmem_ld_32x32b_x32(trow + C::t_dp(bb) + c0 + c * 32, rp);
-          ptx::tmem_ld_wait();
-          softmax32(rs, rp, lse + c * 32, rd + c * 32, p.scale, hp + c * 16, hd + c * 16);
-        }
-        ptx::tc_fence_before();
-        if (g > 0) ok = ptx::mbar_wait(bar_pfree, (g - 1) & 1);
-        ok = __all_sync(0xffffffffu, ok);
-        if (!ok || abort_flag) { ok = false; abort_flag = 1; break; }
-#pragma unroll
-        for (int c = 0; c < CW / 32; ++c) {
-          st_row32_packed(sP, BK, r, c0 + c * 32, hp + c * 16);
-          st_row32_packed(sdS, BK, r, c0 + c * 32, hd + c * 16);
-        }
-        ptx::fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) ptx::mbar_arrive(bar_p);
-      }
-      if (!ok) break;
-    }
-  } else {
-    // ---------------------------------------------------------------- dQ -> f32 reduce-add
-    const int quarter = warp & 3;
-    const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
-    uint8_t* stg = sDQ + quarter * C::DQ_WARP_BYTES;
-    bool ok = true;
-    int i = 0;
-    for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++i) {
-      int k0, b, h;
-      unit_of(u, k0, b, h);
-      for (int j = 0; j < nq; ++j) {
-        const int g = i * nq + j;
-        const int bb = g % NSB;
-        ok = ptx::mbar_wait(&bar_dq[bb], (g / NSB) & 1);
-        ok = __all_sync(0xffffffffu, ok);
-        if (!ok || abort_flag) { ok = false; abort_flag = 1; break; }
-        ptx::tc_fence_after();
-        uint32_t rq[64];
-        ptx::tmem_ld_32x32b_x32(trow + C::t_dq(bb), *reinterpret_cast<uint32_t(*)[32]>(rq));
-        ptx::tmem_ld_32x32b_x32(trow + C::t_dq(bb) + 32, *reinterpret_cast<uint32_t(*)[32]>(rq + 32));
-        ptx::tmem_ld_wait();
-        ptx::tc_fence_before();
-        __syncwarp();
-        if (lane == 0) ptx::mbar_arrive(&bar_dqfree[bb]);
-        const int q0 = j * BQ;
-        // two 32 x 32 boxes (lane = query, columns = 64 head dims) through one staging box
-#pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-          if (lane == 0) ptx::bulk_wait_read<0>();
-          __syncwarp();
-          uint8_t* srow = stg + lane * 128;
-#pragma unroll
-          for (int v = 0; v < 8; ++v)
-            *reinterpret_cast<float4*>(srow + ((v ^ (lane & 7)) << 4)) =
-                make_float4(__uint_as_float(rq[hh * 32 + 4 * v]) * p.scale,
-                            __uint_as_float(rq[hh * 32 + 4 * v + 1]) * p.scale,
-                            __uint_as_float(rq[hh * 32 + 4 * v + 2]) * p.scale,
-                            __uint_as_float(rq[hh * 32 + 4 * v + 3]) * p.scale);
-          ptx::fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) {
-            const int col = h * D + hh * 32;
-            const int row = q0 + quarter * 32;
-            if (row < N) {
-              ptx::tma_reduce_add_3d(&maps.dq, stg, col, row, b);
-              ptx::bulk_commit();
-            }
-          }
-        }
-      }
-      if (!ok) break;
-      // the unit's dK, dV (key rows of this warp's lane quarter): the P / dS warps move on to
-      // the next unit meanwhile
-      ok = __all_sync(0xffffffffu, ptx::mbar_wait(bar_fin, i & 1));
-      if (!ok || abort_flag) { ok = false; abort_flag = 1; break; }
-      ptx::tc_fence_after();
-      const int key = k0 + quarter * 32 + lane;
-#pragma unroll 1
-      for (int c = 0; c < D / 32; ++c) {
-        uint32_t rv[32], rk[32];
-        ptx::tmem_ld_32x32b_x32(trow + C::T_DV + c * 32, rv);
-        ptx::tmem_ld_32x32b_x32(trow + C::T_DK + c * 32, rk);
-        ptx::tmem_ld_wait();
-        if (key < N) {
-          bf16* dv = static_cast<bf16*>(p.dv.base(key)) + p.dv.off(b, key, N, p.dv_col0 + h * D + c * 32);
-          bf16* dk = static_cast<bf16*>(p.dk.base(key)) + p.dk.off(b, key, N, p.dk_col0 + h * D + c * 32);
-#pragma unroll
-          for (int v = 0; v < 4; ++v) {
-            uint4 a, bb;
-            __nv_bfloat162* ha = reinterpret_cast<__nv_bfloat162*>(&a);
-            __nv_bfloat162* hb = reinterpret_cast<__nv_bfloat162*>(&bb);
-#pragma unroll
-            for (int t = 0; t < 4; ++t) {
-              ha[t] = __floats2bfloat162_rn(__uint_as_float(rv[8 * v + 2 * t]), __uint_as_float(rv[8 * v + 2 * t + 1]));
-              hb[t] = __floats2bfloat162_rn(__uint_as_float(rk[8 * v + 2 * t]) * p.scale,
-                                            __uint_as_float(rk[8 * v + 2 * t + 1]) * p.scale);
-            }
-            *reinterpret_cast<uint4*>(dv + 8 * v) = a;
-            *reinterpret_cast<uint4*>(dk + 8 * v) = bb;
-          }
-        }
-      }
-      ptx::tc_fence_before();
-      __syncwarp();
-      if (lane == 0) ptx::mbar_arrive(bar_kvout);
-    }
-    if (lane == 0) ptx::bulk_wait<0>();
-    __syncwarp();
-  }
-  ptx::tc_fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    ptx::tc_fence_after();
-    ptx::tmem_dealloc(tmem, 512);
-  }
-}
-
-// ================================================================== backward, head dim 128
+// ================================================================== backward, head dims 128 and 64
 // 128-key x 64-query tiles with S^T and dP^T double-buffered in tensor memory.  One CTA per
 // SM, persistent over (128-key tile, sequence, head) units; per unit the sequence's query
 // tiles stream through three Q / dO stages.  Tensor memory (512 columns), buffer b = tile % 2:
@@ -521,12 +80,18 @@ __global__ void __launch_bounds__(FB_THREADS, 1) fa_bwd_tc_kernel(const __grid_c
 // (32 keys x 32 queries per warp), so no warp waits for another and nothing waits for a
 // product to release a shared P / dS tile.  The 4 dQ warps move dQ^T through shared memory
 // into TMA f32 reduce-adds and store each unit's dK, dV at its end.
+// Head dim 64 (fa_bwd_tc64_kernel): the same schedule with dV in [256, 320), dK in [320, 384);
+// dQ^T has 64 rows, so its product takes M = 128 over the stacked A operand [K^T; V^T] (the V
+// tile follows the K tile in shared memory: the second 64-row chunk of A) and lanes 64-127 of
+// the result, V^T dS^T, are not read.  A 64-column product takes as long as a 128-row one on
+// this tensor pipe, so the stacking costs nothing.
 constexpr int FB2_THREADS = 448;  // 14 warps
 
+template <int D_>
 struct Fb2 {
-  static constexpr int D = 128, BK = 128, BQ = 64, NS = 3;
-  static constexpr int KV_BYTES = BK * D * 2;  // 32 KB: two 64-column chunks
-  static constexpr int QT_BYTES = BQ * D * 2;  // 16 KB
+  static constexpr int D = D_, BK = 128, BQ = 64, NS = 3;
+  static constexpr int KV_BYTES = BK * D * 2;  // 32 KB at D = 128 (two 64-column chunks), 16 KB at 64
+  static constexpr int QT_BYTES = BQ * D * 2;  // 16 KB, 8 KB
   static constexpr int DS_BYTES = BK * BQ * 2; // 16 KB
   static constexpr int DQ_WARP_BYTES = 32 * 32 * 4;
   static constexpr int OFF_K = 0;
@@ -543,14 +108,14 @@ struct Fb2 {
   static_assert(SMEM <= 232448, "shared memory budget");
   __host__ __device__ static constexpr uint32_t t_s(int b) { return 128u * b; }
   __host__ __device__ static constexpr uint32_t t_dp(int b) { return 128u * b + 64u; }
-  static constexpr uint32_t T_DV = 256, T_DK = 384;
+  static constexpr uint32_t T_DV = 256, T_DK = 256 + D;
+  static_assert(OFF_V == OFF_K + BK * 128 * (D / 64), "the dQ^T A operand's second chunk");
 };
 
-__global__ void __launch_bounds__(FB2_THREADS, 1) fa_bwd_tc128_kernel(const __grid_constant__ FbMaps maps,
-                                                                      FbParams p) {
-  using C = Fb2;
+template <int D_>
+__device__ __forceinline__ void fa_bwd_v3(const FbMaps& maps, const FbParams& p, uint8_t* smem_fb2) {
+  using C = Fb2<D_>;
   constexpr int BK = C::BK, BQ = C::BQ, D = C::D, NS = C::NS;
-  extern __shared__ uint8_t smem_fb2[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_fb2) + 1023) & ~uintptr_t(1023));
   uint8_t* sK = sm + C::OFF_K;
   uint8_t* sV = sm + C::OFF_V;
@@ -878,7 +443,8 @@ __global__ void __launch_bounds__(FB2_THREADS, 1) fa_bwd_tc128_kernel(const __gr
         if (lane == 0) ptx::mbar_arrive(&dqfree[bb]);
         const int q0 = j * BQ;
         // dQ^T: lane = head-dim index, columns = the tile's 64 queries; two 32 x 32 boxes
-        // (box rows = queries) through one staging box
+        // (box rows = queries) through one staging box (head dim 64: lane quarters 0, 1 only)
+        if (quarter * 32 >= D) continue;
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
           if (lane == 0) ptx::bulk_wait_read<0>();
@@ -942,6 +508,17 @@ __global__ void __launch_bounds__(FB2_THREADS, 1) fa_bwd_tc128_kernel(const __gr
     ptx::tc_fence_after();
     ptx::tmem_dealloc(tmem, 512);
   }
+}
+
+__global__ void __launch_bounds__(FB2_THREADS, 1) fa_bwd_tc128_kernel(const __grid_constant__ FbMaps maps,
+                                                                      FbParams p) {
+  extern __shared__ uint8_t smem_fb2[];
+  fa_bwd_v3<128>(maps, p, smem_fb2);
+}
+__global__ void __launch_bounds__(FB2_THREADS, 1) fa_bwd_tc64_kernel(const __grid_constant__ FbMaps maps,
+                                                                     FbParams p) {
+  extern __shared__ uint8_t smem_fb2[];
+  fa_bwd_v3<64>(maps, p, smem_fb2);
 }
 
 // ================================================================== forward
@@ -1686,56 +1263,11 @@ int seg_map(CUtensorMap* m, const void* base, int64_t ld, int ntok, int B, int r
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
+// The pipelined backward (fa_bwd_tc128_kernel, fa_bwd_tc64_kernel).
 template <int D>
-int launch(const AttnBwdArgs& a, cudaStream_t s) {
-  using C = FbCfg<D>;
-  const AttnArgs& f = a.f;
-  const int n0 = f.q.n0, N = f.N;
-  const int n1 = N - n0;
-  FbMaps maps;
-  for (int sg = 0; sg < 2; ++sg) {
-    const int nt = sg == 0 ? n0 : n1;
-    if (nt <= 0) {  // single stream: the second views are unused copies
-      maps.q[1] = maps.q[0];
-      maps.k[1] = maps.k[0];
-      maps.v[1] = maps.v[0];
-      maps.dO[1] = maps.dO[0];
-      break;
-    }
-    JAGG_TRY(seg_map(&maps.q[sg], sg ? f.q.p1 : f.q.p0, sg ? f.q.ld1 : f.q.ld0, nt, f.B, C::BQ));
-    JAGG_TRY(seg_map(&maps.k[sg], sg ? f.k.p1 : f.k.p0, sg ? f.k.ld1 : f.k.ld0, nt, f.B, C::BK));
-    JAGG_TRY(seg_map(&maps.v[sg], sg ? f.v.p1 : f.v.p0, sg ? f.v.ld1 : f.v.ld0, nt, f.B, C::BK));
-    JAGG_TRY(seg_map(&maps.dO[sg], sg ? a.dO.p1 : a.dO.p0, sg ? a.dO.ld1 : a.dO.ld0, nt, f.B, C::BQ));
-  }
-  {
-    const int64_t cols = (int64_t)f.heads * D;
-    const uint64_t dims[3] = {(uint64_t)cols, (uint64_t)N, (uint64_t)f.B};
-    const uint64_t strides[2] = {(uint64_t)cols * 4, (uint64_t)cols * 4 * N};
-    const uint32_t box[3] = {32, 32, 1};
-    JAGG_TRY(encode_tmap(&maps.dq, true, 3, a.dq_acc, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B));
-  }
-  FbParams p;
-  p.B = f.B; p.N = N; p.heads = f.heads; p.n0 = n0 > 0 && n0 < N ? n0 : N;
-  p.scale = f.scale;
-  p.q_col0 = f.q_col0; p.k_col0 = f.k_col0; p.v_col0 = f.v_col0;
-  p.dk_col0 = a.dk_col0; p.dv_col0 = a.dv_col0;
-  p.lse = f.lse; p.Dv = a.Dv;
-  p.dk = a.dk; p.dv = a.dv;
-  static bool attr = false;
-  if (!attr) {
-    JAGG_CUDA_TRY(cudaFuncSetAttribute(fa_bwd_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
-    attr = true;
-  }
-  const int units = ceil_div(N, C::BK) * f.B * f.heads;
-  const int nsm = sm_count();
-  fa_bwd_tc_kernel<D><<<units < nsm ? units : nsm, FB_THREADS, C::SMEM, s>>>(maps, p);
-  JAGG_LAUNCHED();
-  return JAGG_OK;
-}
-
-// The head-dim-128 backward (fa_bwd_tc128_kernel).
-int launch128(const AttnBwdArgs& a, cudaStream_t s) {
-  using C = Fb2;
+int launch_v3(const AttnBwdArgs& a, cudaStream_t s) {
+  using C = Fb2<D>;
+  auto kernel = D == 128 ? fa_bwd_tc128_kernel : fa_bwd_tc64_kernel;
   const AttnArgs& f = a.f;
   const int n0 = f.q.n0, N = f.N;
   const int n1 = N - n0;
@@ -1770,12 +1302,12 @@ int launch128(const AttnBwdArgs& a, cudaStream_t s) {
   p.dk = a.dk; p.dv = a.dv;
   static bool attr = false;
   if (!attr) {
-    JAGG_CUDA_TRY(cudaFuncSetAttribute(fa_bwd_tc128_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
+    JAGG_CUDA_TRY(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
     attr = true;
   }
   const int units = ceil_div(N, C::BK) * f.B * f.heads;
   const int nsm = sm_count();
-  fa_bwd_tc128_kernel<<<units < nsm ? units : nsm, FB2_THREADS, C::SMEM, s>>>(maps, p);
+  kernel<<<units < nsm ? units : nsm, FB2_THREADS, C::SMEM, s>>>(maps, p);
   JAGG_LAUNCHED();
   return JAGG_OK;
 }
@@ -1894,7 +1426,7 @@ bool attention_bwd_tc_eligible(const AttnBwdArgs& a) {
 }
 
 int attention_bwd_tc(const AttnBwdArgs& a, cudaStream_t s) {
-  return a.f.dh == 64 ? launch<64>(a, s) : launch128(a, s);
+  return a.f.dh == 64 ? launch_v3<64>(a, s) : launch_v3<128>(a, s);
 }
 
 }  // namespace jagg
