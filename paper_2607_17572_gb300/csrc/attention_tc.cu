@@ -37,11 +37,16 @@ struct FbParams {
 // K-major: `rows` rows of 128 B per 64-element K chunk, chunks rows * 128 B apart.
 // MN-major: the K dimension runs down the rows (8-row atoms 1024 B apart), 64-element MN
 // chunks `chunk_bytes` apart.
+// The descriptor of step k is that of the operand's base plus the step's byte offset / 16:
+// the start-address field holds address / 16 in its low 14 bits and every operand lies below
+// 2^18 bytes of shared memory, so the addition never carries out of the field.  With the
+// k-loops unrolled, the base descriptor is formed once per operand and each step costs one
+// add in the single issuing thread.
 __device__ __forceinline__ uint64_t kmajor_desc(uint32_t base, int rows, int k) {
-  return ptx::sdesc_sw128(base + (k >> 2) * (rows * 128) + (k & 3) * 32, 16, 1024);
+  return ptx::sdesc_sw128(base, 16, 1024) + (uint64_t)(((k >> 2) * (rows * 128) + (k & 3) * 32) >> 4);
 }
 __device__ __forceinline__ uint64_t mnmajor_desc(uint32_t base, int chunk_bytes, int k) {
-  return ptx::sdesc_sw128(base + k * 2048, chunk_bytes, 1024);
+  return ptx::sdesc_sw128(base, chunk_bytes, 1024) + (uint64_t)(k * 128);
 }
 
 __device__ __forceinline__ uint32_t pack2_bf16(float lo, float hi) {
