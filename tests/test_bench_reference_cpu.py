@@ -29,8 +29,8 @@ def test_reference_arm_prints_one_contract_line():
 
 def test_oracle_sample_of_an_mmdit_scales_by_the_flop_model():
     """At MMDiT widths the CPU baseline times one endpoint row through one block and scales
-    the time by the FLOP model to one sample's JAGG window; the model's forward matches
-    the survey's per-sequence figures (DiT-B 60.9 GFLOP, Flux-width 4.54 / 15.7 TFLOP)."""
+    the time by the FLOP model to one sample's JAGG window; the model's forward matches the
+    workloads' per-sequence forward FLOPs (DiT-B 60.9 GFLOP, Flux-width 4.54 / 15.7 TFLOP)."""
     sys.path.insert(0, ROOT)
     import bench
     import synth
