@@ -526,7 +526,7 @@ __global__ void __launch_bounds__(FB2_THREADS, 1) fa_bwd_tc64_kernel(const __gri
   fa_bwd_v3<64>(maps, p, smem_fb2);
 }
 
-// ================================================================== forward
+// ================================================================== forward, head dim 64
 // Persistent over (128-query tile, sequence, head) units, two passes over the sequence's
 // 128-key tiles per unit:
 //   pass 1   S = Q K^T (TMEM), the exact row maximum m of the scaled scores;
@@ -541,9 +541,10 @@ constexpr int FF_THREADS = 320;  // 10 warps
 
 template <int D>
 struct FfCfg {
+  static_assert(D == 64, "head dim 128 has fa_fwd_tc128_kernel");
   static constexpr int BQ = 128, BK = 128;
-  static constexpr int NS = D == 64 ? 3 : 2;  // K (pass 1) / K, V (pass 2) stages
-  static constexpr int NP = D == 64 ? 2 : 1;  // P buffers
+  static constexpr int NS = 3;  // K (pass 1) / K, V (pass 2) stages
+  static constexpr int NP = 2;  // P buffers
   static constexpr int Q_BYTES = BQ * D * 2;
   static constexpr int KV_BYTES = BK * D * 2;
   static constexpr int P_BYTES = BQ * BK * 2;
